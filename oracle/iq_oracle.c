@@ -1,0 +1,685 @@
+/*
+ * iq_oracle.c -- TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, CPU definition of what the integer quantized convolution
+ * layer of "Training and Inference for Integer-Based Semantic Segmentation
+ * Network" (Yang, Deng, Yang, Xie, Li; arXiv 2011.14504) computes, forward
+ * and backward.  It exists so that the CUDA library can be checked against
+ * it element by element.  Only the test suite, the smoke check and the CPU
+ * baseline leg of the benchmark may load it; the product path never does.
+ * It shares no code, header or constant table with the CUDA sources.
+ *
+ * Representation: a quantized tensor is (integer codes q, real scale s) and
+ * stands for the real values q*s.  Integer work is exact (int64 / int128);
+ * real-valued scale metadata is IEEE fp64 evaluated in the fixed operation
+ * order written below (build with -ffp-contract=off so no FMA is formed).
+ *
+ * Every function names the passage of the paper it follows:
+ *   Sec. 3.1.1 Eq. (del), Eq. (UQ)    quantization step and uniform quantizer
+ *   Sec. 3.1.1 (constant x2 / x1/2)   for mu, sigma, gamma, beta
+ *   Sec. 3.1.2 Eq. (ScaleFactor),(ScaleQ)   scale quantization
+ *   Sec. 3.1.3 Eq. (SQ),(SR)          stochastic rounding quantizer RQ
+ *   Sec. 3.2.1 Eq. (WQ0),(WQ1)        master / forward weights
+ *   Sec. 3.2.2 Eq. (BN2),(BN4),(BN5) and the quantized-BN equation block
+ *   Sec. 3.2.3 Eq. (AQ1)              activation quantization
+ *   Sec. 3.3.1 Eq. (EQ)               error quantization
+ *   Sec. 3.3.2 Eq. (GQ1),(GQ2)        gradient quantization
+ *   Sec. 3.3.3 Eq. (UQ2)              update quantization
+ * Where the paper is silent the reading taken is stated at the function.
+ */
+#include <stdint.h>
+#include <stddef.h>
+#include <math.h>
+#include <string.h>
+#include <stdlib.h>
+
+typedef __int128 i128;
+typedef unsigned __int128 u128;
+
+/* ------------------------------------------------------------------ */
+/* scalar helpers                                                      */
+/* ------------------------------------------------------------------ */
+
+static int64_t clamp64(int64_t v, int64_t lo, int64_t hi) {
+    return v < lo ? lo : (v > hi ? hi : v);
+}
+
+/* floor(a / b) for b > 0 */
+static i128 floordiv128(i128 a, i128 b) {
+    i128 q = a / b;
+    if ((a % b) != 0 && a < 0) q -= 1;
+    return q;
+}
+
+/* Eq. (UQ) rounds with floor(y + 1/2): round half up, ties toward +inf.
+ * On an fp64 y this is floor(y) + [y - floor(y) >= 1/2]; y - floor(y) is
+ * exact, so no rounding of y + 1/2 can move the result across an integer. */
+static double rhu(double y) {
+    double f = floor(y);
+    return f + ((y - f) >= 0.5 ? 1.0 : 0.0);
+}
+
+/* largest code of a k-bit grid: the clip of Eq. (UQ) at 1 - Delta(k) */
+static int64_t qmax(int k) { return ((int64_t)1 << (k - 1)) - 1; }
+
+/* rhu of an fp64 value, clipped to a k-bit symmetric grid */
+static int64_t code_of(double y, int k) {
+    if (y != y) return 0;                               /* NaN -> 0 */
+    double lim = (double)qmax(k);
+    double r = rhu(y);
+    if (r > lim) r = lim;
+    if (r < -lim) r = -lim;
+    return (int64_t)r;
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 3.1.1: uniform quantizer on real (fp32) inputs                 */
+/* ------------------------------------------------------------------ */
+
+/* UQ(x,k) = Clip(Delta*floor(x/Delta + 1/2), -1+Delta, 1-Delta), Eq. (UQ),
+ * Delta = 2^(1-k), Eq. (del).  Output: codes c with UQ(x,k) = c * 2^(1-k).
+ * x/Delta = x * 2^(k-1) is exact in fp64 for every fp32 x. */
+void or_uq_f32(const float* x, int64_t n, int k, int32_t* code) {
+    for (int64_t i = 0; i < n; i++)
+        code[i] = (int32_t)code_of(ldexp((double)x[i], k - 1), k);
+}
+
+/* 2*UQ(x/2, k): the constant x2 / x1/2 scaling used for mu, sigma, gamma,
+ * beta (Sec. 3.1.1 and the quantized-BN equation block).  Codes c with
+ * value c * 2^(2-k). */
+void or_uq2_f32(const float* x, int64_t n, int k, int32_t* code) {
+    for (int64_t i = 0; i < n; i++)
+        code[i] = (int32_t)code_of(ldexp((double)x[i], k - 2), k);
+}
+
+/* SQ(x,k) = Scale(x) * UQ(x / Scale(x), k), Scale(x) = max|x|
+ * (Eqs. (ScaleFactor),(ScaleQ)); Scale is taken over the whole tensor.
+ * The quotient x/S of two fp32 numbers is formed in fp64; the result of
+ * rhu on it equals rhu of the exact real quotient (see DESIGN notes).
+ * Returns the output scale S * 2^(1-k); S == 0 gives all-zero codes and
+ * scale 2^(1-k). */
+double or_sq_f32(const float* x, int64_t n, int k, int32_t* code) {
+    float S = 0.0f;
+    for (int64_t i = 0; i < n; i++) {
+        float a = fabsf(x[i]);
+        if (a > S) S = a;
+    }
+    if (S == 0.0f) {
+        for (int64_t i = 0; i < n; i++) code[i] = 0;
+        return ldexp(1.0, 1 - k);
+    }
+    for (int64_t i = 0; i < n; i++) {
+        double t = (double)x[i] / (double)S;
+        code[i] = (int32_t)code_of(ldexp(t, k - 1), k);
+    }
+    return ldexp((double)S, 1 - k);
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 3.1.2: scale quantization of an integer-coded tensor            */
+/* ------------------------------------------------------------------ */
+
+/* SQ_k of a tensor given as integer codes q with real scale s.
+ * With M = max|q|:  x / Scale(x) = q / M, so
+ *   code = Clip(floor(q * 2^(k-1) / M + 1/2)) = Clip(floor((2^k q + M) / (2M)))
+ * in exact integer arithmetic, and the output scale is
+ *   Scale(x) * Delta = (s * M) * 2^(1-k).
+ * relu != 0 applies ReLU first (q -> max(q, 0)), i.e. SQ(ReLU(x)).
+ * M == 0 gives all-zero codes and scale s * 2^(1-k). */
+double or_sq_int64(const int64_t* q, int64_t n, double s, int k, int relu,
+                   int32_t* code) {
+    int64_t M = 0;
+    for (int64_t i = 0; i < n; i++) {
+        int64_t v = q[i];
+        if (relu && v < 0) v = 0;
+        int64_t a = v < 0 ? -v : v;
+        if (a > M) M = a;
+    }
+    if (M == 0) {
+        for (int64_t i = 0; i < n; i++) code[i] = 0;
+        return ldexp(s, 1 - k);
+    }
+    for (int64_t i = 0; i < n; i++) {
+        int64_t v = q[i];
+        if (relu && v < 0) v = 0;
+        i128 num = ((i128)v << k) + M;
+        i128 c = floordiv128(num, (i128)2 * M);
+        code[i] = (int32_t)clamp64((int64_t)c, -qmax(k), qmax(k));
+    }
+    return ldexp(s * (double)M, 1 - k);
+}
+
+double or_sq_int32(const int32_t* q, int64_t n, double s, int k, int relu,
+                   int32_t* code) {
+    int64_t* t = (int64_t*)malloc(sizeof(int64_t) * (size_t)(n > 0 ? n : 1));
+    for (int64_t i = 0; i < n; i++) t[i] = q[i];
+    double r = or_sq_int64(t, n, s, k, relu, code);
+    free(t);
+    return r;
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 3.1.3: stochastic rounding with a counter-based generator       */
+/* ------------------------------------------------------------------ */
+
+/* Philox4x64 with 10 rounds (Salmon, Moraes, Dror, Shaw, "Parallel random
+ * numbers: as easy as 1, 2, 3", SC'11).  One round maps (x0,x1,x2,x3) with
+ * key (k0,k1) to (hi(M1*x2)^x1^k0, lo(M1*x2), hi(M0*x0)^x3^k1, lo(M0*x0));
+ * the key is advanced by the Weyl constants between rounds. */
+void or_philox4x64_10(const uint64_t ctr[4], const uint64_t key[2],
+                      uint64_t out[4]) {
+    const uint64_t M0 = 0xD2E7470EE14C6C93ULL, M1 = 0xCA5A826395121157ULL;
+    const uint64_t W0 = 0x9E3779B97F4A7C15ULL, W1 = 0xBB67AE8584CAA73BULL;
+    uint64_t x0 = ctr[0], x1 = ctr[1], x2 = ctr[2], x3 = ctr[3];
+    uint64_t k0 = key[0], k1 = key[1];
+    for (int r = 0; r < 10; r++) {
+        u128 p0 = (u128)M0 * x0;
+        u128 p1 = (u128)M1 * x2;
+        uint64_t y0 = (uint64_t)(p1 >> 64) ^ x1 ^ k0;
+        uint64_t y1 = (uint64_t)p1;
+        uint64_t y2 = (uint64_t)(p0 >> 64) ^ x3 ^ k1;
+        uint64_t y3 = (uint64_t)p0;
+        x0 = y0; x1 = y1; x2 = y2; x3 = y3;
+        k0 += W0; k1 += W1;
+    }
+    out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
+}
+
+/* The 32-bit uniform word used for element i of a stochastically rounded
+ * tensor: Philox4x64-10 with key (seed, layer) and counter (i/8, step, tag, 0);
+ * element i takes 32-bit half (i mod 2) of 64-bit word ((i/2) mod 4). */
+uint32_t or_rq_uniform(uint64_t seed, uint64_t layer, uint64_t step,
+                       uint64_t tag, uint64_t i) {
+    uint64_t ctr[4] = { i >> 3, step, tag, 0 };
+    uint64_t key[2] = { seed, layer };
+    uint64_t o[4];
+    or_philox4x64_10(ctr, key, o);
+    uint64_t w = o[(i >> 1) & 3];
+    return (uint32_t)((i & 1) ? (w >> 32) : (w & 0xffffffffULL));
+}
+
+/* RQ(x,k) = Clip(Delta*Round(x/Delta)), Round stochastic with
+ * P(up) = x - floor(x) (Eqs. (SQ),(SR)), applied to x = G / Scale(G)
+ * as in Eqs. (GQ1),(GQ2).  With M = max|q|, y = q * 2^(k-1) / M:
+ *   f = floor(y), rem = q*2^(k-1) - f*M in [0, M),
+ *   round up iff u * M < rem * 2^32   (u the element's 32-bit uniform),
+ * so P(up) = ceil(rem*2^32/M) / 2^32 = rem/M to within 2^-32.
+ * gq_mode 1 = Eq. (GQ1) (magnitude kept): scale (s*M)*2^(1-k);
+ * gq_mode 2 = Eq. (GQ2) (magnitude dropped): scale 2^(1-k).
+ * M == 0 gives zero codes. */
+double or_rq_int64(const int64_t* q, int64_t n, double s, int k, int gq_mode,
+                   uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
+                   int32_t* code) {
+    int64_t M = 0;
+    for (int64_t i = 0; i < n; i++) {
+        int64_t a = q[i] < 0 ? -q[i] : q[i];
+        if (a > M) M = a;
+    }
+    if (M == 0) {
+        for (int64_t i = 0; i < n; i++) code[i] = 0;
+        return gq_mode == 1 ? ldexp(s, 1 - k) : ldexp(1.0, 1 - k);
+    }
+    for (int64_t i = 0; i < n; i++) {
+        i128 num = (i128)q[i] << (k - 1);
+        i128 f = floordiv128(num, (i128)M);
+        i128 rem = num - f * M;
+        uint32_t u = or_rq_uniform(seed, layer, step, tag, (uint64_t)i);
+        int up = ((u128)u * (u128)M) < ((u128)rem << 32);
+        code[i] = (int32_t)clamp64((int64_t)(f + up), -qmax(k), qmax(k));
+    }
+    return gq_mode == 1 ? ldexp(s * (double)M, 1 - k) : ldexp(1.0, 1 - k);
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 3.2.1: weights                                                 */
+/* ------------------------------------------------------------------ */
+
+/* W_q = UQ(W_m, k_W), Eq. (WQ1), where the master weights W_m sit on the
+ * k_U grid (Eq. (WQ0)) as codes m (value m * 2^(1-k_U)).  Then
+ * W_m / Delta(k_W) = m / 2^(k_U - k_W) and floor(that + 1/2) is an exact
+ * arithmetic shift.  The same map serves the x2-scaled gamma/beta masters
+ * (both grids carry the same factor 2). */
+void or_requant_master(const int32_t* m, int64_t n, int k_u, int k_w,
+                       int32_t* wq) {
+    int sh = k_u - k_w;
+    for (int64_t i = 0; i < n; i++) {
+        i128 v = (i128)m[i] + ((i128)1 << (sh - 1));
+        i128 c = floordiv128(v, (i128)1 << sh);
+        wq[i] = (int32_t)clamp64((int64_t)c, -qmax(k_w), qmax(k_w));
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* Convolution: the MAC of Sec. 3.2.3 on 8-bit W and A (Fig. 4)         */
+/* ------------------------------------------------------------------ */
+
+/* Geometry.  x: NHWC [n][h][w][c]; weights KRSC [k][r][s][c/groups];
+ * output NPQK [n][p][q][k].  Output pixel (p,q) with tap (r,s) reads input
+ * row p*stride_h + r*dil_h - pad_h, column q*stride_w + s*dil_w - pad_w;
+ * outside the image the input is zero.  Group g owns input channels
+ * [g*C/G, (g+1)*C/G) and output channels [g*K/G, (g+1)*K/G). */
+typedef struct {
+    int32_t n, h, w, c, k, r, s;
+    int32_t stride_h, stride_w, pad_h, pad_w, dil_h, dil_w, groups;
+    int32_t p, q;
+} or_conv;
+
+void or_conv_out_size(or_conv* d) {
+    d->p = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    d->q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+}
+
+#define X_AT(n_, h_, w_, c_) x[(((int64_t)(n_) * d->h + (h_)) * d->w + (w_)) * d->c + (c_)]
+#define W_AT(k_, r_, s_, c_) wt[(((int64_t)(k_) * d->r + (r_)) * d->s + (s_)) * cg + (c_)]
+#define Y_AT(n_, p_, q_, k_) ((((int64_t)(n_) * d->p + (p_)) * d->q + (q_)) * d->k + (k_))
+
+/* forward: acc[n,p,q,k] = sum_{r,s,c in group} x[...] * w[k,r,s,c] */
+void or_conv_fwd(const or_conv* d, const int8_t* x, const int8_t* wt,
+                 int32_t* acc) {
+    const int cg = d->c / d->groups, kg = d->k / d->groups;
+    #pragma omp parallel for collapse(2) schedule(static)
+    for (int n = 0; n < d->n; n++)
+        for (int p = 0; p < d->p; p++)
+            for (int q = 0; q < d->q; q++)
+                for (int k = 0; k < d->k; k++) {
+                    int g = k / kg;
+                    int64_t sum = 0;
+                    for (int r = 0; r < d->r; r++) {
+                        int hh = p * d->stride_h + r * d->dil_h - d->pad_h;
+                        if (hh < 0 || hh >= d->h) continue;
+                        for (int s = 0; s < d->s; s++) {
+                            int ww = q * d->stride_w + s * d->dil_w - d->pad_w;
+                            if (ww < 0 || ww >= d->w) continue;
+                            for (int c = 0; c < cg; c++)
+                                sum += (int64_t)X_AT(n, hh, ww, g * cg + c) *
+                                       (int64_t)W_AT(k, r, s, c);
+                        }
+                    }
+                    acc[Y_AT(n, p, q, k)] = (int32_t)sum;
+                }
+}
+
+/* data gradient: the adjoint of the forward map,
+ * dx[n,h,w,c] = sum over (p,q,k,r,s) with h = p*sh + r*dh - ph,
+ * w = q*sw + s*dw - pw of e[n,p,q,k] * w[k,r,s,c].  Scattered image by
+ * image (integer sums, so the order is immaterial). */
+void or_conv_dgrad(const or_conv* d, const int8_t* e, const int8_t* wt,
+                   int32_t* dx) {
+    const int cg = d->c / d->groups, kg = d->k / d->groups;
+    const int64_t img = (int64_t)d->h * d->w * d->c;
+    #pragma omp parallel for schedule(static)
+    for (int n = 0; n < d->n; n++) {
+        int64_t* t = (int64_t*)calloc((size_t)img, sizeof(int64_t));
+        for (int p = 0; p < d->p; p++)
+            for (int q = 0; q < d->q; q++)
+                for (int k = 0; k < d->k; k++) {
+                    int64_t ev = e[Y_AT(n, p, q, k)];
+                    if (ev == 0) continue;
+                    int g = k / kg;
+                    for (int r = 0; r < d->r; r++) {
+                        int hh = p * d->stride_h + r * d->dil_h - d->pad_h;
+                        if (hh < 0 || hh >= d->h) continue;
+                        for (int s = 0; s < d->s; s++) {
+                            int ww = q * d->stride_w + s * d->dil_w - d->pad_w;
+                            if (ww < 0 || ww >= d->w) continue;
+                            for (int c = 0; c < cg; c++)
+                                t[((int64_t)hh * d->w + ww) * d->c + g * cg + c] +=
+                                    ev * (int64_t)W_AT(k, r, s, c);
+                        }
+                    }
+                }
+        for (int64_t i = 0; i < img; i++) dx[n * img + i] = (int32_t)t[i];
+        free(t);
+    }
+}
+
+/* weight gradient: g[k,r,s,c] = sum_{n,p,q} e[n,p,q,k] * x[n, h, w, c_g]
+ * with h, w as in the forward map; int64 accumulation (the sum runs over
+ * N*P*Q products and exceeds 2^31 at segmentation sizes). */
+void or_conv_wgrad(const or_conv* d, const int8_t* e, const int8_t* x,
+                   int64_t* gw) {
+    const int cg = d->c / d->groups, kg = d->k / d->groups;
+    #pragma omp parallel for schedule(static)
+    for (int k = 0; k < d->k; k++) {
+        int g = k / kg;
+        for (int r = 0; r < d->r; r++)
+            for (int s = 0; s < d->s; s++)
+                for (int c = 0; c < cg; c++) {
+                    int64_t sum = 0;
+                    for (int n = 0; n < d->n; n++)
+                        for (int p = 0; p < d->p; p++) {
+                            int hh = p * d->stride_h + r * d->dil_h - d->pad_h;
+                            if (hh < 0 || hh >= d->h) continue;
+                            for (int q = 0; q < d->q; q++) {
+                                int ww = q * d->stride_w + s * d->dil_w - d->pad_w;
+                                if (ww < 0 || ww >= d->w) continue;
+                                sum += (int64_t)e[Y_AT(n, p, q, k)] *
+                                       (int64_t)X_AT(n, hh, ww, g * cg + c);
+                            }
+                        }
+                    gw[(((int64_t)k * d->r + r) * d->s + s) * cg + c] = sum;
+                }
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 3.2.2: quantized L1 batch normalization, forward                */
+/* ------------------------------------------------------------------ */
+
+typedef struct {
+    int32_t k_mu, k_sigma, k_xhat, k_gamma, k_beta, k_a;
+} or_bn_bits;
+
+/* Per-tensor and per-channel values the forward pass produces; the
+ * backward pass consumes c_sigma and s_xhat, the rest is for inspection. */
+typedef struct {
+    double s_xhat;     /* scale of the X codes: M_xhat * 2^(1-k_xhat)      */
+    double s_a;        /* scale of the A codes: M_y * 2^(1-k_a)            */
+    double m_xhat;     /* max |xhat| over the tensor                        */
+    double m_y;        /* max ReLU(y) over the tensor                       */
+    int32_t p_x, p_a;  /* fixed-point shifts of the two per-element maps    */
+} or_bn_out;
+
+static int frexp_exp(double v) { int e; frexp(v, &e); return e; }
+
+/* One L1BN layer in training (batch statistics) or inference (the same
+ * batch statistics; the paper defines no running estimate).  Input: conv
+ * accumulators acc[m][C] with real scale s_acc.  Steps, in the paper's order:
+ *
+ *  Eq. (BN2)  mu_B = (1/m) sum_i x_i,  x_i = acc_i * s_acc
+ *  Eq. (BN5)  sigma_B = (1/m) sum_i |x_i - mu_B|        (no square, no root)
+ *             evaluated exactly as T = sum_i |m*acc_i - S1| (S1 = sum acc),
+ *             sigma_B = T * s_acc / m^2 in fp64.
+ *  QBN block  mu_q = 2*UQ(mu_B/2, k_mu), sigma_q = 2*UQ(sigma_B/2, k_sigma)
+ *  Eq. (BN4)  xhat_i = (x_i - mu_q) / (sigma_q + eps),  eps = 2^(2-k_sigma),
+ *             one step of the sigma_q grid (the paper gives no value).
+ *  QBN block  X = SQ(xhat, k_xhat) with Scale = M_xhat = max|xhat|.
+ *             Per channel xhat is increasing in acc, so M_xhat is reached at
+ *             the channel's largest or smallest accumulator.
+ *  QBN block  gamma_q = 2*UQ(gamma/2, k_gamma), beta_q likewise (codes given)
+ *             y_i = gamma_q * xhat_q,i + beta_q
+ *  Eq. (AQ1)  A = SQ(ReLU(y), k_a) with Scale = M_y = max ReLU(y).
+ *
+ * Element-wise the two quantizers are evaluated in fixed point, as an
+ * integer-only device would: per channel the code of X is
+ * rhu(a_c*acc + b_c) for real a_c, b_c, computed as
+ *   X = floor((F_c*acc + B_c) / 2^P),  F_c = rhu(a_c 2^P),
+ *   B_c = rhu(b_c 2^P) + 2^(P-1),
+ * with one shift P per tensor chosen as large as int64 allows; A from X
+ * likewise.  All fp64 steps are written out in evaluation order. */
+int or_bn_fwd(int64_t m, int32_t C, const int32_t* acc, double s_acc,
+              const int32_t* gam, const int32_t* bet, const or_bn_bits* b,
+              int16_t* X, int8_t* A, int32_t* c_mu, int32_t* c_sigma,
+              int64_t* F, int64_t* Bc, int64_t* G, int64_t* H,
+              or_bn_out* out) {
+    if (m <= 0 || C <= 0) return -1;
+    int64_t* S1 = (int64_t*)calloc((size_t)C, sizeof(int64_t));
+    int64_t* hi = (int64_t*)malloc(sizeof(int64_t) * (size_t)C);
+    int64_t* lo = (int64_t*)malloc(sizeof(int64_t) * (size_t)C);
+    u128* T = (u128*)calloc((size_t)C, sizeof(u128));
+    for (int c = 0; c < C; c++) { hi[c] = INT64_MIN; lo[c] = INT64_MAX; }
+    /* Eq. (BN2): channel sums and extremes */
+    for (int64_t i = 0; i < m; i++)
+        for (int c = 0; c < C; c++) {
+            int64_t v = acc[i * C + c];
+            S1[c] += v;
+            if (v > hi[c]) hi[c] = v;
+            if (v < lo[c]) lo[c] = v;
+        }
+    /* Eq. (BN5): T = sum |m*acc - S1| exactly */
+    for (int64_t i = 0; i < m; i++)
+        for (int c = 0; c < C; c++) {
+            i128 dv = (i128)m * acc[i * C + c] - S1[c];
+            T[c] += (u128)(dv < 0 ? -dv : dv);
+        }
+    const double mu_step = ldexp(1.0, 2 - b->k_mu);       /* grid of mu_q */
+    const double sg_step = ldexp(1.0, 2 - b->k_sigma);    /* grid of sigma_q = eps */
+    double* den = (double*)malloc(sizeof(double) * (size_t)C);
+    double* muq = (double*)malloc(sizeof(double) * (size_t)C);
+    const double md = (double)m;
+    for (int c = 0; c < C; c++) {
+        double mu_b = ((double)S1[c] * s_acc) / md;
+        double sg_b = ((double)T[c] * s_acc) / (md * md);
+        int64_t cm = code_of(ldexp(mu_b, b->k_mu - 2), b->k_mu);
+        int64_t cs = code_of(ldexp(sg_b, b->k_sigma - 2), b->k_sigma);
+        c_mu[c] = (int32_t)cm;
+        c_sigma[c] = (int32_t)cs;
+        muq[c] = (double)cm * mu_step;
+        den[c] = (double)(cs + 1) * sg_step;              /* sigma_q + eps */
+    }
+    /* M_xhat from the channel extremes */
+    double mx = 0.0, vmax = 0.0;
+    for (int c = 0; c < C; c++) {
+        double xh = ((double)hi[c] * s_acc - muq[c]) / den[c];
+        double xl = ((double)lo[c] * s_acc - muq[c]) / den[c];
+        if (fabs(xh) > mx) mx = fabs(xh);
+        if (fabs(xl) > mx) mx = fabs(xl);
+        double av = fabs((double)hi[c]) > fabs((double)lo[c]) ? fabs((double)hi[c]) : fabs((double)lo[c]);
+        if (av > vmax) vmax = av;
+    }
+    out->m_xhat = mx;
+    out->s_xhat = mx > 0.0 ? ldexp(mx, 1 - b->k_xhat) : ldexp(1.0, 1 - b->k_xhat);
+    const int64_t xq = qmax(b->k_xhat);
+    /* fixed-point map acc -> X */
+    int px = 0;
+    if (mx > 0.0) {
+        const double qx = ldexp(1.0, b->k_xhat - 1) / mx;
+        double lmax = 0.0;
+        for (int c = 0; c < C; c++) {
+            double a = (s_acc / den[c]) * qx;
+            double bb = (-muq[c] / den[c]) * qx;
+            double l = fabs(a) * vmax + fabs(bb);
+            if (l > lmax) lmax = l;
+        }
+        px = 62 - frexp_exp(lmax + 1.0);
+        if (px > 62) px = 62;
+        if (px < 1) { px = 1; }
+        for (int c = 0; c < C; c++) {
+            double a = (s_acc / den[c]) * qx;
+            double bb = (-muq[c] / den[c]) * qx;
+            F[c] = (int64_t)rhu(ldexp(a, px));
+            Bc[c] = (int64_t)rhu(ldexp(bb, px)) + ((int64_t)1 << (px - 1));
+        }
+    } else {
+        px = 1;
+        for (int c = 0; c < C; c++) { F[c] = 0; Bc[c] = 0; }
+    }
+    out->p_x = px;
+    /* X at the channel extremes (X is nondecreasing in acc: F_c >= 0) */
+    const double gstep = ldexp(1.0, 2 - b->k_gamma), bstep = ldexp(1.0, 2 - b->k_beta);
+    double my = 0.0;
+    for (int c = 0; c < C; c++) {
+        int64_t xs[2] = { hi[c], lo[c] };
+        for (int j = 0; j < 2; j++) {
+            i128 t = (i128)F[c] * xs[j] + Bc[c];
+            int64_t xc = clamp64((int64_t)(t >> px), -xq, xq);
+            double t1 = ((double)gam[c] * gstep) * out->s_xhat;
+            double y = t1 * (double)xc + (double)bet[c] * bstep;
+            if (y > my) my = y;
+        }
+    }
+    out->m_y = my;
+    out->s_a = my > 0.0 ? ldexp(my, 1 - b->k_a) : ldexp(1.0, 1 - b->k_a);
+    const int64_t aq = qmax(b->k_a);
+    int pa = 1;
+    if (my > 0.0) {
+        const double qa = ldexp(1.0, b->k_a - 1) / my;
+        double lmax = 0.0;
+        for (int c = 0; c < C; c++) {
+            double t1 = ((double)gam[c] * gstep) * out->s_xhat;
+            double l = fabs(t1 * qa) * (double)xq + fabs(((double)bet[c] * bstep) * qa);
+            if (l > lmax) lmax = l;
+        }
+        pa = 62 - frexp_exp(lmax + 1.0);
+        if (pa > 62) pa = 62;
+        if (pa < 1) pa = 1;
+        for (int c = 0; c < C; c++) {
+            double t1 = ((double)gam[c] * gstep) * out->s_xhat;
+            G[c] = (int64_t)rhu(ldexp(t1 * qa, pa));
+            H[c] = (int64_t)rhu(ldexp(((double)bet[c] * bstep) * qa, pa)) + ((int64_t)1 << (pa - 1));
+        }
+    } else {
+        for (int c = 0; c < C; c++) { G[c] = 0; H[c] = 0; }
+    }
+    out->p_a = pa;
+    /* element-wise: X = Q_xhat(xhat), A = Q_A(ReLU(gamma_q xhat_q + beta_q)) */
+    for (int64_t i = 0; i < m; i++)
+        for (int c = 0; c < C; c++) {
+            i128 t = (i128)F[c] * acc[i * C + c] + Bc[c];
+            int64_t xc = clamp64((int64_t)(t >> px), -xq, xq);
+            if (X) X[i * C + c] = (int16_t)xc;
+            i128 u = (i128)G[c] * xc + H[c];
+            A[i * C + c] = (int8_t)clamp64((int64_t)(u >> pa), 0, aq);
+        }
+    free(S1); free(hi); free(lo); free(T); free(den); free(muq);
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 3.3: backward through ReLU and quantized L1BN                   */
+/* ------------------------------------------------------------------ */
+
+/* Input: the error of this layer's activation e_A (codes, scale s_e; it is
+ * E_1 of Eq. (EQ) coming from the next layer), the forward outputs A and X,
+ * the gamma codes and the sigma_q codes.  Steps:
+ *   ReLU:   e_y,i = e_A,i if A_i > 0 else 0 (the mask of the stored A).
+ *   d beta_c = s_e * sum e_y;  d gamma_c = s_e * s_X * sum e_y * X
+ *            (returned as the integer sums; their scales are s_e, s_e*s_X).
+ *   E_2 = Q_E(gamma_q * e_y, k_E2), Eq. (EQ): SQ of z_i = e_y,i * g_c.
+ *   L1BN backward (derived from Eqs. (BN4),(BN5); the paper prints none):
+ *     d x_i = (1/(sigma_q+eps)) [ g_i - mean(g) - mean(g xhat) (sgn_i - mean(sgn)) ]
+ *     with g = E_2 (real), xhat = X * s_X, sgn_i = sign(X_i); means over the
+ *     channel's m elements, straight-through for the mu/sigma quantizers.
+ *   E_conv = Q_E(d x, k_E) (SQ8), the error the conv's dgrad/wgrad consume.
+ * Per element the last step is one fixed-point affine map of (E_2, sgn). */
+int or_bn_bwd(int64_t m, int32_t C, const int8_t* eA, double s_e,
+              const int8_t* A, const int16_t* X, double s_x,
+              const int32_t* gam, const int32_t* c_sigma, int k_sigma,
+              int k_gamma, int k_e2, int k_e, int8_t* E, double* s_out,
+              int64_t* dgam, int64_t* dbet) {
+    if (m <= 0 || C <= 0) return -1;
+    /* ReLU mask and gamma/beta gradient sums */
+    int64_t M2 = 0;
+    for (int c = 0; c < C; c++) { dgam[c] = 0; dbet[c] = 0; }
+    for (int64_t i = 0; i < m; i++)
+        for (int c = 0; c < C; c++) {
+            int64_t ey = A[i * C + c] > 0 ? eA[i * C + c] : 0;
+            dbet[c] += ey;
+            dgam[c] += ey * (int64_t)X[i * C + c];
+            int64_t z = ey * (int64_t)gam[c];
+            if (z < 0) z = -z;
+            if (z > M2) M2 = z;
+        }
+    /* E_2 = SQ_{k_e2}(gamma_q e_y) */
+    const double s_z = s_e * ldexp(1.0, 2 - k_gamma);
+    const double s_e2 = M2 > 0 ? ldexp(s_z * (double)M2, 1 - k_e2) : ldexp(s_z, 1 - k_e2);
+    int32_t* E2 = (int32_t*)malloc(sizeof(int32_t) * (size_t)(m * C));
+    for (int64_t i = 0; i < m; i++)
+        for (int c = 0; c < C; c++) {
+            int64_t ey = A[i * C + c] > 0 ? eA[i * C + c] : 0;
+            int64_t z = ey * (int64_t)gam[c];
+            if (M2 == 0) { E2[i * C + c] = 0; continue; }
+            i128 q = floordiv128(((i128)z << k_e2) + M2, (i128)2 * M2);
+            E2[i * C + c] = (int32_t)clamp64((int64_t)q, -qmax(k_e2), qmax(k_e2));
+        }
+    /* channel means of E_2, E_2*X and sign(X) as exact integer sums */
+    int64_t* SE = (int64_t*)calloc((size_t)C, sizeof(int64_t));
+    int64_t* SEX = (int64_t*)calloc((size_t)C, sizeof(int64_t));
+    int64_t* SS = (int64_t*)calloc((size_t)C, sizeof(int64_t));
+    for (int64_t i = 0; i < m; i++)
+        for (int c = 0; c < C; c++) {
+            int64_t e2 = E2[i * C + c];
+            int64_t xv = X[i * C + c];
+            SE[c] += e2;
+            SEX[c] += e2 * xv;
+            SS[c] += (xv > 0) - (xv < 0);
+        }
+    /* per channel: d x_i = w_c * (E2_i + kap_c * sgn_i + lam_c) */
+    double* w = (double*)malloc(sizeof(double) * (size_t)C);
+    double* kap = (double*)malloc(sizeof(double) * (size_t)C);
+    double* lam = (double*)malloc(sizeof(double) * (size_t)C);
+    const double md = (double)m;
+    const double sg_step = ldexp(1.0, 2 - k_sigma);
+    for (int c = 0; c < C; c++) {
+        double gx = ((double)SEX[c] * s_x) / md;           /* mean(g xhat) / s_e2 */
+        kap[c] = -gx;
+        lam[c] = gx * ((double)SS[c] / md) - (double)SE[c] / md;
+        w[c] = s_e2 / ((double)(c_sigma[c] + 1) * sg_step);
+    }
+    /* Scale of d x: the largest |d x_i| over the tensor */
+    double M = 0.0;
+    for (int64_t i = 0; i < m; i++)
+        for (int c = 0; c < C; c++) {
+            int64_t xv = X[i * C + c];
+            double sg = (double)((xv > 0) - (xv < 0));
+            double dx = w[c] * (((double)E2[i * C + c] + kap[c] * sg) + lam[c]);
+            if (fabs(dx) > M) M = fabs(dx);
+        }
+    const int64_t eq = qmax(k_e);
+    if (M == 0.0) {
+        for (int64_t i = 0; i < m * C; i++) E[i] = 0;
+        *s_out = ldexp(1.0, 1 - k_e);
+    } else {
+        const double qe = ldexp(1.0, k_e - 1) / M;
+        const double emax = (double)qmax(k_e2);
+        double lmax = 0.0;
+        for (int c = 0; c < C; c++) {
+            double om = w[c] * qe;
+            double l = fabs(om) * emax + fabs(om * kap[c]) + fabs(om * lam[c]);
+            if (l > lmax) lmax = l;
+        }
+        int pe = 62 - frexp_exp(lmax + 1.0);
+        if (pe > 62) pe = 62;
+        if (pe < 1) pe = 1;
+        for (int c = 0; c < C; c++) {
+            double om = w[c] * qe;
+            int64_t fw = (int64_t)rhu(ldexp(om, pe));
+            int64_t fk = (int64_t)rhu(ldexp(om * kap[c], pe));
+            int64_t fl = (int64_t)rhu(ldexp(om * lam[c], pe)) + ((int64_t)1 << (pe - 1));
+            for (int64_t i = 0; i < m; i++) {
+                int64_t xv = X[i * C + c];
+                int64_t sg = (xv > 0) - (xv < 0);
+                i128 t = (i128)fw * E2[i * C + c] + (i128)fk * sg + fl;
+                E[i * C + c] = (int8_t)clamp64((int64_t)(t >> pe), -eq, eq);
+            }
+        }
+        *s_out = ldexp(M, 1 - k_e);
+    }
+    free(E2); free(SE); free(SEX); free(SS); free(w); free(kap); free(lam);
+    return 0;
+}
+
+/* ReLU backward for layers without BN: e_acc = e_A where A > 0 (same
+ * codes, same scale). */
+void or_relu_bwd(int64_t n, const int8_t* eA, const int8_t* A, int8_t* e) {
+    for (int64_t i = 0; i < n; i++) e[i] = A[i] > 0 ? eA[i] : 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 3.3.3: update                                                  */
+/* ------------------------------------------------------------------ */
+
+/* Delta W = Q_U(G_q, k_U) = UQ(G_q * lr, k_U), Eq. (UQ2), with G_q given as
+ * codes c and scale s_g, lr = 2^(-lr_log2) (a power of two, halved
+ * discretely as the paper's schedule does).  The master codes m live on the
+ * k_U grid (value m * 2^(1-k_U), or m * 2^(2-k_U) for the x2-scaled
+ * gamma/beta masters, x2 != 0).  Plain SGD: m <- Clip(m - dW).
+ * Then the forward copy is regenerated: w_q = UQ(W_m, k_W), Eq. (WQ1). */
+void or_update(int64_t n, int32_t* master, int32_t* wq, const int32_t* gc,
+               double s_g, int lr_log2, int k_u, int k_w, int x2) {
+    const int sh = (x2 ? k_u - 2 : k_u - 1) - lr_log2;
+    for (int64_t i = 0; i < n; i++) {
+        double t = (double)gc[i] * s_g;
+        int64_t du = code_of(ldexp(t, sh), k_u);
+        int64_t nm = clamp64((int64_t)master[i] - du, -qmax(k_u), qmax(k_u));
+        master[i] = (int32_t)nm;
+    }
+    or_requant_master(master, n, k_u, k_w, wq);
+}
+
+/* Correctly rounded conversion of a 128-bit unsigned integer to fp64 (the
+ * conversion the sigma_B step applies to T); exposed for its test. */
+double or_u128_to_double(uint64_t hi, uint64_t lo) {
+    u128 v = ((u128)hi << 64) | lo;
+    return (double)v;
+}
