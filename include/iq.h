@@ -1,0 +1,239 @@
+/*
+ * iq.h -- C ABI of the integer quantized convolution layer for GB300 (sm_103a).
+ *
+ * Method: "Training and Inference for Integer-Based Semantic Segmentation
+ * Network" (Yang, Deng, Yang, Xie, Li; arXiv 2011.14504), Sec. 3.
+ *
+ * Conventions shared by every entry point
+ *  - A quantized tensor is integer codes plus one real scale: value = code * scale.
+ *    Scales are IEEE fp64 values that live in DEVICE memory (a `double*`), so a
+ *    chain of calls never synchronizes with the host.  An input scale is read by
+ *    the kernels; an output scale is written by them.
+ *  - Every tensor pointer is a device pointer to caller-owned memory.  The
+ *    library allocates nothing and keeps no state between calls: scratch space is
+ *    the `ws` argument, whose minimum size the matching *_workspace_size call
+ *    returns (a NULL `ws` with ws_bytes == 0 is accepted when that size is 0).
+ *  - Layouts: activations and errors NHWC (channels innermost), filters KRSC
+ *    (K output channels, R x S taps, C/groups channels innermost), per-channel
+ *    vectors length C.  All integer codes are two's complement.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream).  Argument errors are reported before anything is enqueued;
+ *    kernel-side failures surface as IQ_ERR_CUDA from the launch check.
+ *  - Determinism: identical inputs, seed and step give identical bits on every
+ *    run; all reductions are integer (order-independent) and the fp64 scale
+ *    steps follow a fixed operation order.
+ *  - Bit widths follow the paper's defaults (Sec. 5): k_W = k_A = k_E1 = k_G = 8,
+ *    k_U = 24, k_mu = k_sigma = k_xhat = 16, k_gamma = k_beta = 8, k_E2 in {8,16}.
+ */
+#ifndef IQ_H
+#define IQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* iq_stream; /* cudaStream_t */
+
+typedef enum {
+    IQ_OK = 0,
+    IQ_ERR_INVALID_ARG = 1,   /* NULL pointer, bad size, bad bit width, bad layout */
+    IQ_ERR_UNSUPPORTED = 2,   /* valid request this build does not implement */
+    IQ_ERR_WORKSPACE = 3,     /* ws smaller than the *_workspace_size result */
+    IQ_ERR_OVERFLOW_RISK = 4, /* int32 accumulation could overflow at this shape */
+    IQ_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up */
+    IQ_ERR_CUDA = 6           /* a CUDA launch or runtime call failed */
+} iq_status;
+
+/* element types */
+enum { IQ_I8 = 1, IQ_I16 = 2, IQ_I32 = 3, IQ_I64 = 4, IQ_F32 = 5, IQ_U8 = 6 };
+
+/* quantizer modes */
+enum {
+    IQ_MODE_UQ = 0,      /* Eq. (UQ): codes of UQ(x,k), scale 2^(1-k)                   */
+    IQ_MODE_UQ2 = 1,     /* 2*UQ(x/2,k) (Sec. 3.1.1 x2 scaling): scale 2^(2-k)           */
+    IQ_MODE_SQ = 2,      /* Eq. (ScaleQ): Scale(x) = max|x| over the tensor             */
+    IQ_MODE_SQ_RELU = 3, /* SQ(ReLU(x)): Eq. (AQ1) after the activation                 */
+    IQ_MODE_RQ_GQ1 = 4,  /* Eq. (GQ1): Scale(G) * RQ(G/Scale(G), k), stochastic (SR)    */
+    IQ_MODE_RQ_GQ2 = 5   /* Eq. (GQ2): RQ(G/Scale(G), k), magnitude dropped             */
+};
+
+/* Convolution geometry.  Input NHWC [n][h][w][c]; filters KRSC [k][r][s][c/groups];
+ * output [n][p][q][k] with p = (h + 2 pad_h - dil_h (r-1) - 1) / stride_h + 1 (q alike).
+ * Output pixel (p,q), tap (r,s) reads input row p*stride_h + r*dil_h - pad_h and
+ * column q*stride_w + s*dil_w - pad_w; outside the image the input is zero.
+ * Group g maps input channels [g c/G, (g+1) c/G) to outputs [g k/G, (g+1) k/G). */
+typedef struct {
+    int32_t n, h, w, c;
+    int32_t k, r, s;
+    int32_t stride_h, stride_w, pad_h, pad_w, dil_h, dil_w, groups;
+} iq_conv_desc;
+
+/* Bit widths of the quantized L1BN objects (Sec. 3.2.2 equation block, Eq. (AQ1)). */
+typedef struct {
+    int32_t k_mu, k_sigma, k_xhat, k_gamma, k_beta, k_a;
+} iq_bn_bits;
+
+/* Per-tensor fp64 values of an L1BN forward pass, written to `bn_scales`
+ * (device, IQ_BN_SCALES doubles) and read back by the backward pass. */
+enum {
+    IQ_BN_S_XHAT = 0, /* scale of the X (= Q_xhat(xhat)) codes: M_xhat * 2^(1-k_xhat) */
+    IQ_BN_M_XHAT = 1, /* max |xhat| over the tensor                                      */
+    IQ_BN_M_Y = 2,    /* max ReLU(gamma_q xhat_q + beta_q) over the tensor               */
+    IQ_BN_S_ACC = 3,  /* scale of the conv accumulators the pass consumed               */
+    IQ_BN_S_A = 4,    /* scale of the A codes (also written to s_a)                     */
+    IQ_BN_SCALES = 8
+};
+
+const char* iq_status_str(iq_status s);
+int iq_version(void);
+
+/* Output size of a convolution (host-side, no device work). */
+iq_status iq_conv_out_size(const iq_conv_desc* d, int32_t* p, int32_t* q);
+
+/* Workspace sizes in bytes (host-side, no device work). */
+iq_status iq_quantize_workspace_size(int64_t n, size_t* bytes);
+iq_status iq_conv_fwd_workspace_size(const iq_conv_desc* d, int with_bn, size_t* bytes);
+iq_status iq_conv_dgrad_workspace_size(const iq_conv_desc* d, size_t* bytes);
+iq_status iq_conv_wgrad_workspace_size(const iq_conv_desc* d, size_t* bytes);
+iq_status iq_bn_int_workspace_size(int64_t m, int32_t c, size_t* bytes);
+
+/* iq_quantize -- real (fp32) tensor to k-bit codes, Sec. 3.1 (Eqs. (del),(UQ),
+ * (ScaleFactor),(ScaleQ)).
+ *   x        fp32[n], finite values (non-finite inputs give unspecified codes)
+ *   k        2..16 for SQ, 2..24 for UQ/UQ2
+ *   mode     IQ_MODE_UQ, IQ_MODE_UQ2, IQ_MODE_SQ or IQ_MODE_SQ_RELU
+ *   out_dtype IQ_I8 (k <= 8), IQ_I16 (k <= 16) or IQ_I32
+ *   codes    out, n elements of out_dtype
+ *   scale    out, one device double: the scale of the codes
+ * UQ codes: clip(floor(x 2^(k-1) + 1/2)).  SQ: S = max|x|, codes
+ * clip(floor(x 2^(k-1)/S + 1/2)) (exact rational value of x/S), scale S 2^(1-k). */
+iq_status iq_quantize(const float* x, int64_t n, int k, int mode, int out_dtype, void* codes,
+                      double* scale, void* ws, size_t ws_bytes, iq_stream stream);
+
+/* iq_quantize_image_u8 -- the network input: real pixel p/255 quantized with
+ * Q_A = SQ(., 8) (Eq. (AQ1); Sec. 5 feeds images to the first conv).  With
+ * P = max pixel, code = floor((256 p + P) / (2P)), clipped to 127; scale
+ * (P/255) 2^-7.  Input uint8 NHWC (nchw = 0) or NCHW (nchw = 1) with c channels;
+ * output int8 NHWC with c_out >= c channels, channels c..c_out-1 zero (padding
+ * for aligned loads in the first convolution). */
+iq_status iq_quantize_image_u8(const uint8_t* img, int32_t n, int32_t h, int32_t w, int32_t c,
+                               int nchw, int32_t c_out, int8_t* codes, double* scale, void* ws,
+                               size_t ws_bytes, iq_stream stream);
+
+/* iq_requantize -- integer-coded tensor (codes q, device scale s_in) to k-bit codes.
+ *   mode IQ_MODE_SQ / IQ_MODE_SQ_RELU: Eq. (ScaleQ) with M = max|q|:
+ *        code = clip(floor((2^k q + M) / (2M))), s_out = (s_in M) 2^(1-k).
+ *   mode IQ_MODE_RQ_GQ1 / IQ_MODE_RQ_GQ2: Eqs. (SQ),(SR),(GQ1),(GQ2): y = q 2^(k-1)/M
+ *        rounded up with probability y - floor(y) using Philox4x64-10 with key
+ *        (seed, layer) and counter (i/8, step, tag, 0) (32-bit half i%2 of word
+ *        (i/2)%4 for element i); s_out = (s_in M) 2^(1-k) (GQ1) or 2^(1-k) (GQ2).
+ *   in_dtype IQ_I32 or IQ_I64 (|q| < 2^40); k 2..16; out_dtype IQ_I8/IQ_I16/IQ_I32.
+ *   M == 0 gives zero codes. */
+iq_status iq_requantize(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
+                        int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
+                        void* codes, int out_dtype, double* s_out, void* ws, size_t ws_bytes,
+                        iq_stream stream);
+
+/* iq_weight_requant -- forward weights from master weights, Eqs. (WQ0),(WQ1):
+ * master codes m on the k_u grid (value m 2^(1-k_u)), wq = clip(floor((m + 2^(k_u-k_w-1))
+ * / 2^(k_u-k_w))) = UQ(W_m, k_w).  Scale of wq is 2^(1-k_w) (x2 grids: 2^(2-k_w)). */
+iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_u, int k_w,
+                            iq_stream stream);
+
+/* iq_conv_fwd -- the quantized conv layer forward (Sec. 3.2, Fig. 4):
+ * acc = conv(x, w) in exact int32 (8-bit x and W, Sec. 3.2.3), then either
+ *   bn == NULL:  A = Q_A(act(acc s_acc)) = SQ(., 8), Eq. (AQ1), act = ReLU if relu else identity;
+ *   bn != NULL:  quantized L1BN (Eqs. (BN2),(BN4),(BN5) and the QBN block; the same
+ *                computation as iq_bn_int_fwd) + ReLU + Q_A.
+ *   x      int8 NHWC [n][h][w][c];  s_x: device double (scale of x)
+ *   w      int8 KRSC, codes of W_q = UQ(W_m, 8) (scale 2^-7; s_acc = s_x 2^-7)
+ *   gamma, beta  device int32[k]: codes of gamma_q = 2 UQ(gamma/2, k_gamma) etc. (bn only)
+ *   bits   bit widths (bn only; NULL = paper defaults)
+ *   a      out int8 NHWC [n][p][q][k];  s_a: out device double
+ *   xhat   out int16 [n][p][q][k], the X codes kept for backward (bn only, may be NULL)
+ *   bn_codes  out device int32[2k]: mu_q codes then sigma_q codes (bn only, may be NULL)
+ *   bn_scales out device double[IQ_BN_SCALES] (bn only, may be NULL)
+ *   acc_out   optional out int32 [n][p][q][k]: the raw accumulators
+ * Returns IQ_ERR_OVERFLOW_RISK when (c/groups) r s 127^2 >= 2^31. */
+iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
+                      const int8_t* w, const int32_t* gamma, const int32_t* beta,
+                      const iq_bn_bits* bits, int use_bn, int relu, int8_t* a, double* s_a,
+                      int16_t* xhat, int32_t* bn_codes, double* bn_scales, int32_t* acc_out,
+                      void* ws, size_t ws_bytes, iq_stream stream);
+
+/* iq_conv_dgrad -- error of the layer input (Sec. 3.3.1, Eq. (EQ)):
+ * dx = conv_transpose(e, w) in exact int32, then E_1 = SQ(dx, 8).
+ *   e    int8 [n][p][q][k] error codes at the conv output; s_e device double
+ *   w    int8 KRSC forward weights (scale 2^-7)
+ *   dx   out int8 NHWC [n][h][w][c]; s_dx out device double = (s_e 2^-7 M) 2^-7
+ *   acc_out optional out int32 [n][h][w][c] */
+iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
+                        const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out, void* ws,
+                        size_t ws_bytes, iq_stream stream);
+
+/* iq_conv_wgrad -- weight gradient and its quantization (Sec. 3.3.2):
+ * G[k][r][s][c] = sum_{n,p,q} e[n,p,q,k] x[n, h(p,r), w(q,s), c] in exact int64, then
+ * G_q = Eq. (GQ1) (gq_mode 1, networks with BN) or Eq. (GQ2) (gq_mode 2, without).
+ *   e, s_e  error codes at the conv output and their scale
+ *   x, s_x  the forward input codes and their scale (s_G = s_e s_x)
+ *   seed, layer, step  Philox key/counter words of the stochastic rounding (tag 0)
+ *   g       out int8 KRSC gradient codes;  s_g out device double
+ *   g_acc_out optional out int64 KRSC: the exact sums */
+iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
+                        const int8_t* x, const double* s_x, int gq_mode, uint64_t seed,
+                        uint64_t layer, uint64_t step, int8_t* g, double* s_g,
+                        int64_t* g_acc_out, void* ws, size_t ws_bytes, iq_stream stream);
+
+/* iq_bn_int_fwd -- quantized L1BN + ReLU + Q_A on int32 accumulators acc[m][c] with
+ * scale s_acc (Sec. 3.2.2, Eqs. (BN2),(BN4),(BN5), QBN block, Eq. (AQ1)):
+ *   mu_B = mean x, sigma_B = mean |x - mu_B| (exact integer sums), mu_q = 2 UQ(mu_B/2, k_mu),
+ *   sigma_q = 2 UQ(sigma_B/2, k_sigma), xhat = (x - mu_q)/(sigma_q + eps) with eps one
+ *   sigma_q grid step, X = SQ(xhat, k_xhat), y = gamma_q xhat_q + beta_q, A = SQ(ReLU(y), k_a).
+ *   The element-wise maps acc -> X -> A are per-channel fixed-point affine maps
+ *   floor((F acc + B) / 2^P) whose constants come from fixed-order fp64 steps.
+ *   Batch statistics are used in training and inference alike (the paper defines
+ *   no running estimate).
+ *   xhat out int16 [m][c] (may be NULL for inference); a out int8 [m][c]; s_a out double
+ *   bn_codes out int32[2c]; bn_scales out double[IQ_BN_SCALES]
+ *   bn_fixed optional out int64[4c + 2]: F[c], B[c], G[c], H[c], P_x, P_a */
+iq_status iq_bn_int_fwd(const int32_t* acc, int64_t m, int32_t c, const double* s_acc,
+                        const int32_t* gamma, const int32_t* beta, const iq_bn_bits* bits,
+                        int16_t* xhat, int8_t* a, double* s_a, int32_t* bn_codes,
+                        double* bn_scales, int64_t* bn_fixed, void* ws, size_t ws_bytes,
+                        iq_stream stream);
+
+/* iq_bn_int_bwd -- backward through Q_A/ReLU and the quantized L1BN (Sec. 3.3.1):
+ *   e_y = e_a where a > 0 (ReLU mask of the stored activation codes);
+ *   dbeta[c] = sum e_y (scale s_e), dgamma[c] = sum e_y X (scale s_e s_xhat), int64 out;
+ *   E_2 = SQ(gamma_q e_y, k_e2), Eq. (EQ);
+ *   dx_i = (1/(sigma_q+eps)) [g_i - mean g - mean(g xhat) (sign X_i - mean sign X)],
+ *   the derivative of Eqs. (BN4),(BN5) (straight-through for the mu/sigma quantizers);
+ *   e = SQ(dx, 8), the conv-output error fed to iq_conv_dgrad / iq_conv_wgrad.
+ *   e_a, s_e   int8 [m][c] error codes of this layer's activation and their scale
+ *   a, xhat    the forward outputs;  gamma int32[c];  bn_codes, bn_scales from the forward
+ *   e          out int8 [m][c];  s_e_out out device double */
+iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const int8_t* a,
+                        const int16_t* xhat, int64_t m, int32_t c, const int32_t* gamma,
+                        const int32_t* bn_codes, const double* bn_scales,
+                        const iq_bn_bits* bits, int k_e2, int8_t* e, double* s_e_out,
+                        int64_t* dgamma, int64_t* dbeta, void* ws, size_t ws_bytes,
+                        iq_stream stream);
+
+/* iq_relu_bwd -- layers without BN: e = e_a where a > 0, else 0 (same scale). */
+iq_status iq_relu_bwd(const int8_t* e_a, const int8_t* a, int64_t n, int8_t* e,
+                      iq_stream stream);
+
+/* iq_update -- Eq. (UQ2): Delta W = UQ(G_q lr, k_u) with lr = 2^-lr_log2, plain SGD
+ * master <- clip(master - Delta W) on the k_u grid, then wq = UQ(W_m, k_w) (Eq. (WQ1)).
+ *   master int32[n] in/out (codes on the k_u grid; x2 != 0: the x2-scaled gamma/beta grid)
+ *   wq     out int8[n];  g int8[n] gradient codes with device scale s_g */
+iq_status iq_update(int32_t* master, int8_t* wq, const int8_t* g, const double* s_g,
+                    int64_t n, int lr_log2, int k_u, int k_w, int x2, iq_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* IQ_H */

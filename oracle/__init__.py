@@ -95,6 +95,8 @@ def _declare(L):
     L.or_bn_bwd.restype = _I32
     L.or_relu_bwd.argtypes = [_I64, _P, _P, _P]
     L.or_update.argtypes = [_I64, _P, _P, _P, _D, _I32, _I32, _I32, _I32]
+    L.or_quantize_image_u8.argtypes = [_P, _I64, _I32, _I32, _P]
+    L.or_quantize_image_u8.restype = _D
     L.or_u128_to_double.argtypes = [_U64, _U64]
     L.or_u128_to_double.restype = _D
 
@@ -170,6 +172,15 @@ def requant_master(m, k_u: int = 24, k_w: int = 8) -> np.ndarray:
     out = np.empty(m.shape, np.int32)
     lib().or_requant_master(_ptr(m), m.size, k_u, k_w, _ptr(out))
     return out
+
+
+def quantize_image_u8(img, c_out: int):
+    """Network input: pixel/255 -> SQ8 codes, NHWC uint8 -> NHWC int8 with c_out channels."""
+    img = _c(img, np.uint8)
+    n, h, w, c = img.shape
+    out = np.empty((n, h, w, c_out), np.int8)
+    s = lib().or_quantize_image_u8(_ptr(img), n * h * w, c, c_out, _ptr(out))
+    return out, s
 
 
 def u128_to_double(v: int) -> float:

@@ -683,3 +683,24 @@ double or_u128_to_double(uint64_t hi, uint64_t lo) {
     u128 v = ((u128)hi << 64) | lo;
     return (double)v;
 }
+
+/* Network input (Sec. 5 feeds images to the first conv; Eq. (AQ1)): the real
+ * pixel value p/255 quantized with SQ(., 8).  Scale = P/255 with P the largest
+ * pixel, so x/Scale = p/P and code = floor((256 p + P) / (2P)), clipped at 127;
+ * output scale (P/255) * 2^-7.  Input uint8 NHWC with c channels, output int8
+ * NHWC with c_out >= c channels (the extra channels zero). */
+double or_quantize_image_u8(const uint8_t* img, int64_t npix, int c, int c_out,
+                            int8_t* out) {
+    int64_t P = 0;
+    for (int64_t i = 0; i < npix * c; i++) if (img[i] > P) P = img[i];
+    for (int64_t p = 0; p < npix; p++)
+        for (int j = 0; j < c_out; j++) {
+            int64_t v = 0;
+            if (j < c && P > 0) {
+                v = (256 * (int64_t)img[p * c + j] + P) / (2 * P);
+                if (v > 127) v = 127;
+            }
+            out[p * c_out + j] = (int8_t)v;
+        }
+    return P > 0 ? ldexp((double)P / 255.0, -7) : ldexp(1.0, -7);
+}

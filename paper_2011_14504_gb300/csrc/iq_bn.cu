@@ -1,0 +1,795 @@
+// iq_bn.cu -- quantized L1 batch normalization (Sec. 3.2.2) with ReLU and Q_A
+// (Eq. (AQ1)), forward and backward (Sec. 3.3.1).
+//
+// Data: acc / errors are [m][C] row-major (NHWC flattened), C % 4 == 0.
+// Every per-channel pass uses one launch shape: T threads in total with
+// T % (C/4) == 0, so thread t always owns the same 4 channels (t % (C/4)) and
+// keeps their partial sums in registers; blocks combine in shared memory and
+// add into global integer accumulators (order-independent, hence deterministic).
+// Loads are 16 bytes (4 int32 accumulators, or 4 int8 / int16 codes).
+#include "iq_internal.cuh"
+
+#include <climits>
+
+namespace iq {
+
+namespace {
+
+struct ChanGrid {
+    int blocks;
+    int64_t threads;
+};
+
+int64_t gcd64(int64_t a, int64_t b) {
+    while (b) { int64_t t = a % b; a = b; b = t; }
+    return a;
+}
+
+ChanGrid chan_grid(int64_t m, int32_t C4, int max_blocks = 152 * 8) {
+    int64_t unit = C4 / gcd64(kThreads, C4);  // blocks so that unit*256 % C4 == 0
+    int64_t want = (m * C4 + kThreads - 1) / kThreads;
+    if (want > max_blocks) want = max_blocks;
+    if (want < 1) want = 1;
+    want = (want + unit - 1) / unit * unit;
+    ChanGrid g;
+    g.blocks = (int)want;
+    g.threads = want * kThreads;
+    return g;
+}
+
+__device__ __forceinline__ void unpack4_i8(int v, int out[4]) {
+#pragma unroll
+    for (int j = 0; j < 4; j++) out[j] = (int)(int8_t)(v >> (8 * j));
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ workspace
+
+size_t bn_fwd_ws_bytes(int32_t C) {
+    WsCursor c(nullptr, 0);
+    bn_stats_carve(c, C);
+    return c.off + 256;
+}
+
+BnStats bn_stats_carve(WsCursor& cur, int32_t C) {
+    BnStats s;
+    s.s1 = cur.take<unsigned long long>(C);
+    s.hi = cur.take<int>(C);
+    s.lo = cur.take<int>(C);
+    s.dev = cur.take<unsigned long long>(C);
+    s.ngt = cur.take<unsigned long long>(C);
+    s.F = cur.take<long long>(C);
+    s.B = cur.take<long long>(C);
+    s.G = cur.take<long long>(C);
+    s.H = cur.take<long long>(C);
+    s.codes = cur.take<int>(2 * (size_t)C);
+    s.px = cur.take<int>(4);
+    s.scal = cur.take<double>(IQ_BN_SCALES);
+    return s;
+}
+
+__global__ void k_bn_init(BnStats s, int32_t C) {
+    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < C; c += gridDim.x * blockDim.x) {
+        s.s1[c] = 0; s.dev[c] = 0; s.ngt[c] = 0;
+        s.hi[c] = INT_MIN; s.lo[c] = INT_MAX;
+    }
+}
+
+iq_status bn_stats_init(const BnStats& s, int32_t C, cudaStream_t st) {
+    k_bn_init<<<(C + 255) / 256, 256, 0, st>>>(s, C);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+// ------------------------------------------------------------------ Eq. (BN2): sums, extremes
+
+__global__ void __launch_bounds__(kThreads) k_bn_stats(const int32_t* __restrict__ acc,
+                                                       int64_t m, int32_t C, BnStats s) {
+    __shared__ unsigned long long sh_s1[1024];
+    __shared__ int sh_hi[1024], sh_lo[1024];
+    const int C4 = C >> 2;
+    const bool use_sh = C <= 1024;
+    if (use_sh)
+        for (int c = threadIdx.x; c < C; c += blockDim.x) { sh_s1[c] = 0; sh_hi[c] = INT_MIN; sh_lo[c] = INT_MAX; }
+    __syncthreads();
+    const int64_t T = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % C4);
+    const int64_t rstride = T / C4;
+    long long s1[4] = {0, 0, 0, 0};
+    int hi[4] = {INT_MIN, INT_MIN, INT_MIN, INT_MIN}, lo[4] = {INT_MAX, INT_MAX, INT_MAX, INT_MAX};
+    const int4* a4 = reinterpret_cast<const int4*>(acc);
+    for (int64_t r = t / C4; r < m; r += rstride) {
+        int4 v = a4[r * C4 + g];
+        int vs[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) { s1[j] += vs[j]; hi[j] = max(hi[j], vs[j]); lo[j] = min(lo[j], vs[j]); }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        int c = 4 * g + j;
+        if (use_sh) {
+            atomicAdd(&sh_s1[c], (unsigned long long)s1[j]);
+            atomicMax(&sh_hi[c], hi[j]);
+            atomicMin(&sh_lo[c], lo[j]);
+        } else {
+            atomicAdd(&s.s1[c], (unsigned long long)s1[j]);
+            atomicMax(&s.hi[c], hi[j]);
+            atomicMin(&s.lo[c], lo[j]);
+        }
+    }
+    if (use_sh) {
+        __syncthreads();
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            atomicAdd(&s.s1[c], sh_s1[c]);
+            atomicMax(&s.hi[c], sh_hi[c]);
+            atomicMin(&s.lo[c], sh_lo[c]);
+        }
+    }
+}
+
+iq_status bn_stats_pass(const int32_t* acc, int64_t m, int32_t C, const BnStats& s,
+                        cudaStream_t st) {
+    ChanGrid g = chan_grid(m, C / 4);
+    k_bn_stats<<<g.blocks, kThreads, 0, st>>>(acc, m, C, s);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+// ------------------------------------------------------------------ Eq. (BN5): deviation sums
+// sum_i |m acc_i - S1| = m * sum_i |acc_i - f| + rho * (m - 2 #(acc_i > f)),
+// f = floor(S1/m), rho = S1 - f m; this pass sums |acc - f| and counts acc > f.
+
+__device__ __forceinline__ int64_t floordiv_i64(int64_t a, int64_t b) {
+    int64_t q = a / b;
+    if ((a % b) != 0 && a < 0) q -= 1;
+    return q;
+}
+
+__global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__ acc, int64_t m,
+                                                     int32_t C, BnStats s) {
+    __shared__ unsigned long long sh_d[1024], sh_n[1024];
+    const int C4 = C >> 2;
+    const bool use_sh = C <= 1024;
+    if (use_sh)
+        for (int c = threadIdx.x; c < C; c += blockDim.x) { sh_d[c] = 0; sh_n[c] = 0; }
+    __syncthreads();
+    const int64_t T = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % C4);
+    const int64_t rstride = T / C4;
+    int64_t f[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) f[j] = floordiv_i64((int64_t)s.s1[4 * g + j], m);
+    unsigned long long d[4] = {0, 0, 0, 0}, n[4] = {0, 0, 0, 0};
+    const int4* a4 = reinterpret_cast<const int4*>(acc);
+    for (int64_t r = t / C4; r < m; r += rstride) {
+        int4 v = a4[r * C4 + g];
+        int vs[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            int64_t dv = (int64_t)vs[j] - f[j];
+            d[j] += (unsigned long long)(dv < 0 ? -dv : dv);
+            n[j] += dv > 0;
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        int c = 4 * g + j;
+        if (use_sh) { atomicAdd(&sh_d[c], d[j]); atomicAdd(&sh_n[c], n[j]); }
+        else { atomicAdd(&s.dev[c], d[j]); atomicAdd(&s.ngt[c], n[j]); }
+    }
+    if (use_sh) {
+        __syncthreads();
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            atomicAdd(&s.dev[c], sh_d[c]);
+            atomicAdd(&s.ngt[c], sh_n[c]);
+        }
+    }
+}
+
+// ------------------------------------------------------------------ finalize (one block)
+
+__device__ double block_max_d(double v, double* sh) {
+    // v >= 0 on every thread
+    for (int o = 16; o > 0; o >>= 1) v = fmax(v, __shfl_xor_sync(0xffffffffu, v, o));
+    int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    __syncthreads();
+    if (l == 0) sh[w] = v;
+    __syncthreads();
+    double r = 0.0;
+    int nw = (blockDim.x + 31) >> 5;
+    for (int i = 0; i < nw; i++) r = fmax(r, sh[i]);
+    __syncthreads();
+    return r;
+}
+
+__device__ __forceinline__ int frexp_exp(double v) {
+    int e;
+    frexp(v, &e);
+    return e;
+}
+
+// The fp64 steps below follow the oracle's operation order one for one:
+// mu_B = (S1 s_acc)/m, sigma_B = (T s_acc)/(m m), codes by rhu of v 2^(k-2),
+// xhat(v) = (v s_acc - mu_q)/den, a_c = (s_acc/den) qx, b_c = (-mu_q/den) qx, ...
+__global__ void __launch_bounds__(1024) k_bn_finalize(
+    BnStats s, int64_t m, int32_t C, const double* __restrict__ s_acc_p,
+    const int32_t* __restrict__ gam, const int32_t* __restrict__ bet, iq_bn_bits b,
+    int32_t* __restrict__ codes /* [2C] c_mu, c_sigma */) {
+    __shared__ double red[32];
+    const double s_acc = *s_acc_p;
+    const double md = (double)m;
+    const double mu_step = ldexp(1.0, 2 - b.k_mu), sg_step = ldexp(1.0, 2 - b.k_sigma);
+    double mx = 0.0, vmax = 0.0;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        int64_t S1 = (int64_t)s.s1[c];
+        int64_t f = floordiv_i64(S1, m);
+        int64_t rho = S1 - f * m;
+        i128 T = (i128)m * (i128)(int64_t)s.dev[c] + (i128)rho * (i128)(m - 2 * (int64_t)s.ngt[c]);
+        double mu_b = __ddiv_rn(__dmul_rn((double)S1, s_acc), md);
+        double sg_b = __ddiv_rn(__dmul_rn(u128_to_double((u128)T), s_acc), __dmul_rn(md, md));
+        int64_t cm = code_of(ldexp(mu_b, b.k_mu - 2), b.k_mu);
+        int64_t cs = code_of(ldexp(sg_b, b.k_sigma - 2), b.k_sigma);
+        codes[c] = (int32_t)cm;
+        codes[C + c] = (int32_t)cs;
+        double muq = __dmul_rn((double)cm, mu_step);
+        double den = __dmul_rn((double)(cs + 1), sg_step);
+        double xh = __ddiv_rn(__dsub_rn(__dmul_rn((double)s.hi[c], s_acc), muq), den);
+        double xl = __ddiv_rn(__dsub_rn(__dmul_rn((double)s.lo[c], s_acc), muq), den);
+        mx = fmax(mx, fmax(fabs(xh), fabs(xl)));
+        vmax = fmax(vmax, fmax(fabs((double)s.hi[c]), fabs((double)s.lo[c])));
+    }
+    __syncthreads();
+    mx = block_max_d(mx, red);
+    vmax = block_max_d(vmax, red);
+    const double s_xhat = mx > 0.0 ? ldexp(mx, 1 - b.k_xhat) : ldexp(1.0, 1 - b.k_xhat);
+    const int64_t xq = qmax(b.k_xhat);
+    int px = 1;
+    if (mx > 0.0) {
+        const double qx = __ddiv_rn(ldexp(1.0, b.k_xhat - 1), mx);
+        double lmax = 0.0;
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            double muq = __dmul_rn((double)codes[c], mu_step);
+            double den = __dmul_rn((double)(codes[C + c] + 1), sg_step);
+            double a = __dmul_rn(__ddiv_rn(s_acc, den), qx);
+            double bb = __dmul_rn(__ddiv_rn(-muq, den), qx);
+            lmax = fmax(lmax, __dadd_rn(__dmul_rn(fabs(a), vmax), fabs(bb)));
+        }
+        lmax = block_max_d(lmax, red);
+        px = 62 - frexp_exp(__dadd_rn(lmax, 1.0));
+        px = px > 62 ? 62 : (px < 1 ? 1 : px);
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            double muq = __dmul_rn((double)codes[c], mu_step);
+            double den = __dmul_rn((double)(codes[C + c] + 1), sg_step);
+            double a = __dmul_rn(__ddiv_rn(s_acc, den), qx);
+            double bb = __dmul_rn(__ddiv_rn(-muq, den), qx);
+            s.F[c] = (long long)rhu(ldexp(a, px));
+            s.B[c] = (long long)rhu(ldexp(bb, px)) + (1LL << (px - 1));
+        }
+    } else {
+        for (int c = threadIdx.x; c < C; c += blockDim.x) { s.F[c] = 0; s.B[c] = 0; }
+    }
+    __syncthreads();
+    const double gstep = ldexp(1.0, 2 - b.k_gamma), bstep = ldexp(1.0, 2 - b.k_beta);
+    double my = 0.0;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        int64_t xs[2] = {s.hi[c], s.lo[c]};
+        double t1 = __dmul_rn(__dmul_rn((double)gam[c], gstep), s_xhat);
+        for (int j = 0; j < 2; j++) {
+            long long t = (long long)s.F[c] * xs[j] + s.B[c];
+            int64_t xc = clamp64(t >> px, -xq, xq);
+            double y = __dadd_rn(__dmul_rn(t1, (double)xc), __dmul_rn((double)bet[c], bstep));
+            my = fmax(my, y);
+        }
+    }
+    my = block_max_d(my, red);
+    const double s_a = my > 0.0 ? ldexp(my, 1 - b.k_a) : ldexp(1.0, 1 - b.k_a);
+    int pa = 1;
+    if (my > 0.0) {
+        const double qa = __ddiv_rn(ldexp(1.0, b.k_a - 1), my);
+        double lmax = 0.0;
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            double t1 = __dmul_rn(__dmul_rn((double)gam[c], gstep), s_xhat);
+            double bq = __dmul_rn((double)bet[c], bstep);
+            lmax = fmax(lmax, __dadd_rn(__dmul_rn(fabs(__dmul_rn(t1, qa)), (double)xq),
+                                        fabs(__dmul_rn(bq, qa))));
+        }
+        lmax = block_max_d(lmax, red);
+        pa = 62 - frexp_exp(__dadd_rn(lmax, 1.0));
+        pa = pa > 62 ? 62 : (pa < 1 ? 1 : pa);
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            double t1 = __dmul_rn(__dmul_rn((double)gam[c], gstep), s_xhat);
+            double bq = __dmul_rn((double)bet[c], bstep);
+            s.G[c] = (long long)rhu(ldexp(__dmul_rn(t1, qa), pa));
+            s.H[c] = (long long)rhu(ldexp(__dmul_rn(bq, qa), pa)) + (1LL << (pa - 1));
+        }
+    } else {
+        for (int c = threadIdx.x; c < C; c += blockDim.x) { s.G[c] = 0; s.H[c] = 0; }
+    }
+    if (threadIdx.x == 0) {
+        s.px[0] = px;
+        s.px[1] = pa;
+        s.scal[IQ_BN_S_XHAT] = s_xhat;
+        s.scal[IQ_BN_M_XHAT] = mx;
+        s.scal[IQ_BN_M_Y] = my;
+        s.scal[IQ_BN_S_ACC] = s_acc;
+        s.scal[IQ_BN_S_A] = s_a;
+        for (int i = IQ_BN_S_A + 1; i < IQ_BN_SCALES; i++) s.scal[i] = 0.0;
+    }
+}
+
+// ------------------------------------------------------------------ fused requant pass
+// X = clip(floor((F acc + B) / 2^Px)), A = clip(floor((G X + H) / 2^Pa), 0, 2^(k_a-1)-1)
+
+__global__ void __launch_bounds__(kThreads) k_bn_requant(const int32_t* __restrict__ acc,
+                                                         int64_t m, int32_t C, BnStats s,
+                                                         int kx, int ka,
+                                                         int16_t* __restrict__ X,
+                                                         int8_t* __restrict__ A) {
+    const int C4 = C >> 2;
+    const int64_t T = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % C4);
+    const int64_t rstride = T / C4;
+    const int px = s.px[0], pa = s.px[1];
+    const int64_t xq = qmax(kx), aq = qmax(ka);
+    long long F[4], B[4], G[4], H[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        F[j] = s.F[4 * g + j]; B[j] = s.B[4 * g + j];
+        G[j] = s.G[4 * g + j]; H[j] = s.H[4 * g + j];
+    }
+    const int4* a4 = reinterpret_cast<const int4*>(acc);
+    for (int64_t r = t / C4; r < m; r += rstride) {
+        int64_t v = r * C4 + g;
+        int4 in = a4[v];
+        int vs[4] = {in.x, in.y, in.z, in.w};
+        int xo[4];
+        uint32_t ao = 0;
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            long long tx = F[j] * (long long)vs[j] + B[j];
+            int64_t xc = clamp64(tx >> px, -xq, xq);
+            xo[j] = (int)xc;
+            long long ta = G[j] * xc + H[j];
+            int64_t ac = clamp64(ta >> pa, 0, aq);
+            ao |= ((uint32_t)ac & 0xffu) << (8 * j);
+        }
+        if (X) {
+            uint2 xv;
+            xv.x = ((uint32_t)(uint16_t)xo[0]) | ((uint32_t)(uint16_t)xo[1] << 16);
+            xv.y = ((uint32_t)(uint16_t)xo[2]) | ((uint32_t)(uint16_t)xo[3] << 16);
+            reinterpret_cast<uint2*>(X)[v] = xv;
+        }
+        reinterpret_cast<uint32_t*>(A)[v] = ao;
+    }
+}
+
+__global__ void k_bn_export(BnStats s, int32_t C, const int32_t* __restrict__ codes_ws,
+                            double* __restrict__ s_a, int32_t* __restrict__ bn_codes,
+                            double* __restrict__ bn_scales, int64_t* __restrict__ bn_fixed) {
+    int t = blockIdx.x * blockDim.x + threadIdx.x;
+    if (t == 0) {
+        if (s_a) *s_a = s.scal[IQ_BN_S_A];
+        if (bn_scales)
+            for (int i = 0; i < IQ_BN_SCALES; i++) bn_scales[i] = s.scal[i];
+        if (bn_fixed) { bn_fixed[4 * C] = s.px[0]; bn_fixed[4 * C + 1] = s.px[1]; }
+    }
+    for (int c = t; c < C; c += gridDim.x * blockDim.x) {
+        if (bn_codes) { bn_codes[c] = codes_ws[c]; bn_codes[C + c] = codes_ws[C + c]; }
+        if (bn_fixed) {
+            bn_fixed[c] = s.F[c]; bn_fixed[C + c] = s.B[c];
+            bn_fixed[2 * C + c] = s.G[c]; bn_fixed[3 * C + c] = s.H[c];
+        }
+    }
+}
+
+iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const double* s_acc,
+                             const int32_t* gamma, const int32_t* beta, const iq_bn_bits& b,
+                             const BnStats& s, int16_t* xhat, int8_t* a, double* s_a,
+                             int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
+                             cudaStream_t st) {
+    ChanGrid g = chan_grid(m, C / 4);
+    k_bn_dev<<<g.blocks, kThreads, 0, st>>>(acc, m, C, s);
+    IQ_LAUNCH_CHECK();
+    k_bn_finalize<<<1, 1024, 0, st>>>(s, m, C, s_acc, gamma, beta, b, s.codes);
+    IQ_LAUNCH_CHECK();
+    ChanGrid g2 = chan_grid(m, C / 4, 152 * 16);
+    k_bn_requant<<<g2.blocks, kThreads, 0, st>>>(acc, m, C, s, b.k_xhat, b.k_a, xhat, a);
+    IQ_LAUNCH_CHECK();
+    k_bn_export<<<(C + 255) / 256, 256, 0, st>>>(s, C, s.codes, s_a, bn_codes, bn_scales,
+                                                 bn_fixed);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+// ==================================================================== backward
+// pass 1: e_y = e_a [a > 0]; per channel sum e_y, sum e_y X; max |e_y gamma|
+// fin 1 : E_2 = SQ_{k_e2}(e_y gamma) constants
+// pass 2: per channel sum E_2, sum E_2 X, sum sign X; E_2 extremes per sign class
+// fin 2 : d x_i = w_c (E_2 + kap_c sgn + lam_c); M = max |d x|; fixed-point SQ8 map
+// pass 3: e = clip(floor((fw E_2 + fk sgn + fl) / 2^P))
+
+struct BnBwd {
+    unsigned long long* sb;   // sum e_y
+    unsigned long long* sg;   // sum e_y X
+    unsigned long long* se;   // sum E_2
+    unsigned long long* sex;  // sum E_2 X
+    unsigned long long* ss;   // sum sign X
+    int* emin;                // [3C] per sign class (-1, 0, +1)
+    int* emax;                // [3C]
+    long long* fw;
+    long long* fk;
+    long long* fl;
+    unsigned* zmax;           // [1]
+    int* pe;                  // [1]
+    RqDiv* e2div;             // [1]
+    double* scal;             // [2]: s_e2, s_out
+};
+
+static BnBwd bnb_carve(WsCursor& cur, int32_t C) {
+    BnBwd w;
+    w.sb = cur.take<unsigned long long>(C);
+    w.sg = cur.take<unsigned long long>(C);
+    w.se = cur.take<unsigned long long>(C);
+    w.sex = cur.take<unsigned long long>(C);
+    w.ss = cur.take<unsigned long long>(C);
+    w.emin = cur.take<int>(3 * (size_t)C);
+    w.emax = cur.take<int>(3 * (size_t)C);
+    w.fw = cur.take<long long>(C);
+    w.fk = cur.take<long long>(C);
+    w.fl = cur.take<long long>(C);
+    w.zmax = cur.take<unsigned>(1);
+    w.pe = cur.take<int>(1);
+    w.e2div = cur.take<RqDiv>(1);
+    w.scal = cur.take<double>(2);
+    return w;
+}
+
+__global__ void k_bnb_init(BnBwd w, int32_t C) {
+    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < C; c += gridDim.x * blockDim.x) {
+        w.sb[c] = 0; w.sg[c] = 0; w.se[c] = 0; w.sex[c] = 0; w.ss[c] = 0;
+        for (int j = 0; j < 3; j++) { w.emin[3 * c + j] = INT_MAX; w.emax[3 * c + j] = INT_MIN; }
+        if (c == 0) *w.zmax = 0;
+    }
+}
+
+__device__ __forceinline__ void load4_e_a_x(int64_t v, const int8_t* ea, const int8_t* a,
+                                            const int16_t* X, int e[4], int am[4], int x[4]) {
+    unpack4_i8(reinterpret_cast<const int*>(ea)[v], e);
+    unpack4_i8(reinterpret_cast<const int*>(a)[v], am);
+    uint2 xv = reinterpret_cast<const uint2*>(X)[v];
+    x[0] = (int)(int16_t)(xv.x & 0xffffu); x[1] = (int)(int16_t)(xv.x >> 16);
+    x[2] = (int)(int16_t)(xv.y & 0xffffu); x[3] = (int)(int16_t)(xv.y >> 16);
+}
+
+__global__ void __launch_bounds__(kThreads) k_bnb_pass1(const int8_t* __restrict__ ea,
+                                                        const int8_t* __restrict__ a,
+                                                        const int16_t* __restrict__ X,
+                                                        const int32_t* __restrict__ gam,
+                                                        int64_t m, int32_t C, BnBwd w) {
+    __shared__ unsigned long long sh_b[1024], sh_g[1024];
+    const int C4 = C >> 2;
+    const bool use_sh = C <= 1024;
+    if (use_sh)
+        for (int c = threadIdx.x; c < C; c += blockDim.x) { sh_b[c] = 0; sh_g[c] = 0; }
+    __syncthreads();
+    const int64_t T = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % C4);
+    const int64_t rstride = T / C4;
+    int gm[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) gm[j] = gam[4 * g + j];
+    long long sb[4] = {0, 0, 0, 0}, sg[4] = {0, 0, 0, 0};
+    uint32_t zm = 0;
+    for (int64_t r = t / C4; r < m; r += rstride) {
+        int e[4], am[4], x[4];
+        load4_e_a_x(r * C4 + g, ea, a, X, e, am, x);
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            int ey = am[j] > 0 ? e[j] : 0;
+            sb[j] += ey;
+            sg[j] += (long long)ey * x[j];
+            int z = ey * gm[j];
+            zm = max(zm, (uint32_t)(z < 0 ? -z : z));
+        }
+    }
+    zm = warp_max_u32(zm);
+    if ((threadIdx.x & 31) == 0 && zm) atomicMax(w.zmax, zm);
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        int c = 4 * g + j;
+        if (use_sh) { atomicAdd(&sh_b[c], (unsigned long long)sb[j]); atomicAdd(&sh_g[c], (unsigned long long)sg[j]); }
+        else { atomicAdd(&w.sb[c], (unsigned long long)sb[j]); atomicAdd(&w.sg[c], (unsigned long long)sg[j]); }
+    }
+    if (use_sh) {
+        __syncthreads();
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            atomicAdd(&w.sb[c], sh_b[c]);
+            atomicAdd(&w.sg[c], sh_g[c]);
+        }
+    }
+}
+
+// E_2 = SQ_{k}(z) with M2 = max|z|: floor((2^k (z + M2) + M2) / (2 M2)) - 2^(k-1)
+__global__ void k_bnb_fin1(BnBwd w, const double* __restrict__ s_e, int k_gamma, int k_e2) {
+    uint32_t M2 = *w.zmax;
+    double s_z = __dmul_rn(*s_e, ldexp(1.0, 2 - k_gamma));
+    w.scal[0] = M2 ? ldexp(__dmul_rn(s_z, (double)M2), 1 - k_e2) : ldexp(s_z, 1 - k_e2);
+    RqDiv d;
+    d.M = M2;
+    d.div = make_udiv(M2 ? 2ull * M2 : 1ull);
+    *w.e2div = d;
+}
+
+__device__ __forceinline__ int e2_code(int z, const RqDiv& d, int k) {
+    if (!d.M) return 0;
+    uint64_t num = ((uint64_t)((int64_t)z + (int64_t)d.M) << k) + d.M;
+    int64_t c = (int64_t)udiv(num, d.div) - (int64_t(1) << (k - 1));
+    return (int)clamp64(c, -qmax(k), qmax(k));
+}
+
+__global__ void __launch_bounds__(kThreads) k_bnb_pass2(const int8_t* __restrict__ ea,
+                                                        const int8_t* __restrict__ a,
+                                                        const int16_t* __restrict__ X,
+                                                        const int32_t* __restrict__ gam,
+                                                        int64_t m, int32_t C, int k_e2, BnBwd w) {
+    __shared__ unsigned long long sh_e[512], sh_x[512], sh_s[512];
+    __shared__ int sh_mn[3 * 512], sh_mx[3 * 512];
+    const int C4 = C >> 2;
+    const bool use_sh = C <= 512;
+    if (use_sh)
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            sh_e[c] = 0; sh_x[c] = 0; sh_s[c] = 0;
+            for (int j = 0; j < 3; j++) { sh_mn[3 * c + j] = INT_MAX; sh_mx[3 * c + j] = INT_MIN; }
+        }
+    __syncthreads();
+    const RqDiv d = *w.e2div;
+    const int64_t T = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % C4);
+    const int64_t rstride = T / C4;
+    int gm[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) gm[j] = gam[4 * g + j];
+    long long se[4] = {0, 0, 0, 0}, sx[4] = {0, 0, 0, 0}, ss[4] = {0, 0, 0, 0};
+    int mn[4][3], mx[4][3];
+#pragma unroll
+    for (int j = 0; j < 4; j++)
+#pragma unroll
+        for (int q = 0; q < 3; q++) { mn[j][q] = INT_MAX; mx[j][q] = INT_MIN; }
+    for (int64_t r = t / C4; r < m; r += rstride) {
+        int e[4], am[4], x[4];
+        load4_e_a_x(r * C4 + g, ea, a, X, e, am, x);
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            int ey = am[j] > 0 ? e[j] : 0;
+            int e2 = e2_code(ey * gm[j], d, k_e2);
+            int sgn = (x[j] > 0) - (x[j] < 0);
+            se[j] += e2;
+            sx[j] += (long long)e2 * x[j];
+            ss[j] += sgn;
+            int q = sgn + 1;
+#pragma unroll
+            for (int qq = 0; qq < 3; qq++)
+                if (qq == q) { mn[j][qq] = min(mn[j][qq], e2); mx[j][qq] = max(mx[j][qq], e2); }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        int c = 4 * g + j;
+        if (use_sh) {
+            atomicAdd(&sh_e[c], (unsigned long long)se[j]);
+            atomicAdd(&sh_x[c], (unsigned long long)sx[j]);
+            atomicAdd(&sh_s[c], (unsigned long long)ss[j]);
+            for (int q = 0; q < 3; q++) { atomicMin(&sh_mn[3 * c + q], mn[j][q]); atomicMax(&sh_mx[3 * c + q], mx[j][q]); }
+        } else {
+            atomicAdd(&w.se[c], (unsigned long long)se[j]);
+            atomicAdd(&w.sex[c], (unsigned long long)sx[j]);
+            atomicAdd(&w.ss[c], (unsigned long long)ss[j]);
+            for (int q = 0; q < 3; q++) { atomicMin(&w.emin[3 * c + q], mn[j][q]); atomicMax(&w.emax[3 * c + q], mx[j][q]); }
+        }
+    }
+    if (use_sh) {
+        __syncthreads();
+        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+            atomicAdd(&w.se[c], sh_e[c]);
+            atomicAdd(&w.sex[c], sh_x[c]);
+            atomicAdd(&w.ss[c], sh_s[c]);
+            for (int q = 0; q < 3; q++) { atomicMin(&w.emin[3 * c + q], sh_mn[3 * c + q]); atomicMax(&w.emax[3 * c + q], sh_mx[3 * c + q]); }
+        }
+    }
+}
+
+// Per channel (oracle order): gx = (SEX s_x)/m; kap = -gx; lam = gx (SS/m) - SE/m;
+// w = s_e2 / ((c_sigma + 1) sg_step); d x = w ((E_2 + kap sgn) + lam).
+__global__ void __launch_bounds__(1024) k_bnb_fin2(BnBwd w, int64_t m, int32_t C,
+                                                   const int32_t* __restrict__ csig,
+                                                   const double* __restrict__ bn_scales,
+                                                   int k_sigma, int k_e2, int k_e,
+                                                   double* __restrict__ s_out) {
+    __shared__ double red[32];
+    const double md = (double)m;
+    const double s_x = bn_scales[IQ_BN_S_XHAT];
+    const double s_e2 = w.scal[0];
+    const double sg_step = ldexp(1.0, 2 - k_sigma);
+    double M = 0.0;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        double gx = __ddiv_rn(__dmul_rn((double)(long long)w.sex[c], s_x), md);
+        double kap = -gx;
+        double lam = __dsub_rn(__dmul_rn(gx, __ddiv_rn((double)(long long)w.ss[c], md)),
+                               __ddiv_rn((double)(long long)w.se[c], md));
+        double wc = __ddiv_rn(s_e2, __dmul_rn((double)(csig[c] + 1), sg_step));
+        for (int q = 0; q < 3; q++) {
+            int lo = w.emin[3 * c + q], hi = w.emax[3 * c + q];
+            if (lo > hi) continue;  // empty sign class
+            double sg = (double)(q - 1);
+            double ks = __dmul_rn(kap, sg);
+            double d0 = __dmul_rn(wc, __dadd_rn(__dadd_rn((double)lo, ks), lam));
+            double d1 = __dmul_rn(wc, __dadd_rn(__dadd_rn((double)hi, ks), lam));
+            M = fmax(M, fmax(fabs(d0), fabs(d1)));
+        }
+    }
+    M = block_max_d(M, red);
+    if (M == 0.0) {
+        for (int c = threadIdx.x; c < C; c += blockDim.x) { w.fw[c] = 0; w.fk[c] = 0; w.fl[c] = 0; }
+        if (threadIdx.x == 0) { *w.pe = 1; w.scal[1] = ldexp(1.0, 1 - k_e); *s_out = w.scal[1]; }
+        return;
+    }
+    const double qe = __ddiv_rn(ldexp(1.0, k_e - 1), M);
+    const double emax = (double)qmax(k_e2);
+    double lmax = 0.0;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        double gx = __ddiv_rn(__dmul_rn((double)(long long)w.sex[c], s_x), md);
+        double kap = -gx;
+        double lam = __dsub_rn(__dmul_rn(gx, __ddiv_rn((double)(long long)w.ss[c], md)),
+                               __ddiv_rn((double)(long long)w.se[c], md));
+        double wc = __ddiv_rn(s_e2, __dmul_rn((double)(csig[c] + 1), sg_step));
+        double om = __dmul_rn(wc, qe);
+        double l = __dadd_rn(__dadd_rn(__dmul_rn(fabs(om), emax), fabs(__dmul_rn(om, kap))),
+                             fabs(__dmul_rn(om, lam)));
+        lmax = fmax(lmax, l);
+    }
+    lmax = block_max_d(lmax, red);
+    int pe = 62 - frexp_exp(__dadd_rn(lmax, 1.0));
+    pe = pe > 62 ? 62 : (pe < 1 ? 1 : pe);
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        double gx = __ddiv_rn(__dmul_rn((double)(long long)w.sex[c], s_x), md);
+        double kap = -gx;
+        double lam = __dsub_rn(__dmul_rn(gx, __ddiv_rn((double)(long long)w.ss[c], md)),
+                               __ddiv_rn((double)(long long)w.se[c], md));
+        double wc = __ddiv_rn(s_e2, __dmul_rn((double)(csig[c] + 1), sg_step));
+        double om = __dmul_rn(wc, qe);
+        w.fw[c] = (long long)rhu(ldexp(om, pe));
+        w.fk[c] = (long long)rhu(ldexp(__dmul_rn(om, kap), pe));
+        w.fl[c] = (long long)rhu(ldexp(__dmul_rn(om, lam), pe)) + (1LL << (pe - 1));
+    }
+    if (threadIdx.x == 0) { *w.pe = pe; w.scal[1] = ldexp(M, 1 - k_e); *s_out = w.scal[1]; }
+}
+
+__global__ void __launch_bounds__(kThreads) k_bnb_pass3(const int8_t* __restrict__ ea,
+                                                        const int8_t* __restrict__ a,
+                                                        const int16_t* __restrict__ X,
+                                                        const int32_t* __restrict__ gam,
+                                                        int64_t m, int32_t C, int k_e2, int k_e,
+                                                        BnBwd w, int8_t* __restrict__ out) {
+    const RqDiv d = *w.e2div;
+    const int pe = *w.pe;
+    const int64_t eq = qmax(k_e);
+    const int C4 = C >> 2;
+    const int64_t T = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % C4);
+    const int64_t rstride = T / C4;
+    int gm[4];
+    long long fw[4], fk[4], fl[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        gm[j] = gam[4 * g + j];
+        fw[j] = w.fw[4 * g + j]; fk[j] = w.fk[4 * g + j]; fl[j] = w.fl[4 * g + j];
+    }
+    for (int64_t r = t / C4; r < m; r += rstride) {
+        int64_t v = r * C4 + g;
+        int e[4], am[4], x[4];
+        load4_e_a_x(v, ea, a, X, e, am, x);
+        uint32_t o = 0;
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            int ey = am[j] > 0 ? e[j] : 0;
+            int e2 = e2_code(ey * gm[j], d, k_e2);
+            int sgn = (x[j] > 0) - (x[j] < 0);
+            long long tt = fw[j] * (long long)e2 + fk[j] * (long long)sgn + fl[j];
+            int64_t c = clamp64(tt >> pe, -eq, eq);
+            o |= ((uint32_t)c & 0xffu) << (8 * j);
+        }
+        reinterpret_cast<uint32_t*>(out)[v] = o;
+    }
+}
+
+size_t bn_bwd_ws_bytes(int32_t C) {
+    WsCursor c(nullptr, 0);
+    bnb_carve(c, C);
+    return c.off + 256;
+}
+
+}  // namespace iq
+
+using namespace iq;
+
+// ==================================================================== C ABI
+
+extern "C" iq_status iq_bn_int_workspace_size(int64_t m, int32_t c, size_t* bytes) {
+    if (!bytes || m < 0 || c <= 0) return IQ_ERR_INVALID_ARG;
+    size_t f = bn_fwd_ws_bytes(c), b = bn_bwd_ws_bytes(c);
+    *bytes = f > b ? f : b;
+    return IQ_OK;
+}
+
+static bool bn_shape_ok(int64_t m, int32_t c) {
+    return m > 0 && c > 0 && (c % 4) == 0 && c <= 65536 && m < (int64_t(1) << 40);
+}
+
+extern "C" iq_status iq_bn_int_fwd(const int32_t* acc, int64_t m, int32_t c, const double* s_acc,
+                                   const int32_t* gamma, const int32_t* beta,
+                                   const iq_bn_bits* bits, int16_t* xhat, int8_t* a, double* s_a,
+                                   int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
+                                   void* ws, size_t ws_bytes, iq_stream stream) {
+    if (!acc || !s_acc || !gamma || !beta || !a || !s_a) return IQ_ERR_INVALID_ARG;
+    if (!bn_shape_ok(m, c)) return (m > 0 && c > 0) ? IQ_ERR_UNSUPPORTED : IQ_ERR_INVALID_ARG;
+    iq_bn_bits b = bn_bits_or_default(bits);
+    if (!bn_bits_valid(b)) return IQ_ERR_INVALID_ARG;
+    if (((uintptr_t)acc | (uintptr_t)a | (uintptr_t)xhat) & 15) return IQ_ERR_INVALID_ARG;
+    size_t need = bn_fwd_ws_bytes(c);
+    if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    WsCursor cur(ws, ws_bytes);
+    BnStats s = bn_stats_carve(cur, c);
+    iq_status r = bn_stats_init(s, c, st);
+    if (r != IQ_OK) return r;
+    r = bn_stats_pass(acc, m, c, s, st);
+    if (r != IQ_OK) return r;
+    return bn_fwd_after_stats(acc, m, c, s_acc, gamma, beta, b, s, xhat, a, s_a, bn_codes,
+                              bn_scales, bn_fixed, st);
+}
+
+extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const int8_t* a,
+                                   const int16_t* xhat, int64_t m, int32_t c,
+                                   const int32_t* gamma, const int32_t* bn_codes,
+                                   const double* bn_scales, const iq_bn_bits* bits, int k_e2,
+                                   int8_t* e, double* s_e_out, int64_t* dgamma, int64_t* dbeta,
+                                   void* ws, size_t ws_bytes, iq_stream stream) {
+    if (!e_a || !s_e || !a || !xhat || !gamma || !bn_codes || !bn_scales || !e || !s_e_out)
+        return IQ_ERR_INVALID_ARG;
+    if (!bn_shape_ok(m, c)) return (m > 0 && c > 0) ? IQ_ERR_UNSUPPORTED : IQ_ERR_INVALID_ARG;
+    iq_bn_bits b = bn_bits_or_default(bits);
+    if (!bn_bits_valid(b) || k_e2 < 2 || k_e2 > 16) return IQ_ERR_INVALID_ARG;
+    if (((uintptr_t)e_a | (uintptr_t)a | (uintptr_t)xhat | (uintptr_t)e) & 15)
+        return IQ_ERR_INVALID_ARG;
+    size_t need = bn_bwd_ws_bytes(c);
+    if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    WsCursor cur(ws, ws_bytes);
+    BnBwd w = bnb_carve(cur, c);
+    k_bnb_init<<<(c + 255) / 256, 256, 0, st>>>(w, c);
+    IQ_LAUNCH_CHECK();
+    ChanGrid g = chan_grid(m, c / 4);
+    k_bnb_pass1<<<g.blocks, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, w);
+    IQ_LAUNCH_CHECK();
+    k_bnb_fin1<<<1, 1, 0, st>>>(w, s_e, b.k_gamma, k_e2);
+    IQ_LAUNCH_CHECK();
+    k_bnb_pass2<<<g.blocks, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, k_e2, w);
+    IQ_LAUNCH_CHECK();
+    k_bnb_fin2<<<1, 1024, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma, k_e2, 8, s_e_out);
+    IQ_LAUNCH_CHECK();
+    ChanGrid g3 = chan_grid(m, c / 4, 152 * 16);
+    k_bnb_pass3<<<g3.blocks, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, k_e2, 8, w, e);
+    IQ_LAUNCH_CHECK();
+    if (dgamma)
+        IQ_CUDA_CHECK(cudaMemcpyAsync(dgamma, w.sg, sizeof(int64_t) * c, cudaMemcpyDeviceToDevice, st));
+    if (dbeta)
+        IQ_CUDA_CHECK(cudaMemcpyAsync(dbeta, w.sb, sizeof(int64_t) * c, cudaMemcpyDeviceToDevice, st));
+    return IQ_OK;
+}

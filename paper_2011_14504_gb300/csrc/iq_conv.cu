@@ -1,0 +1,544 @@
+// iq_conv.cu -- the 8-bit convolution (the MAC of Sec. 3.2.3 on 8-bit W and A) as
+// implicit GEMMs, forward, data gradient and weight gradient, plus the C ABI of the
+// conv layer (Sec. 3.2 forward with Q_A or quantized L1BN, Sec. 3.3 backward).
+//
+// This file holds the portable CUDA-core path: 64x64 output tiles, 32-byte K
+// slices staged in shared memory packed 4 codes per word, dp4a MACs with int32
+// accumulation.  The tensor-core path (iq_conv_tc.cu) takes the shapes it supports.
+#include "iq_internal.cuh"
+#include "iq_conv_tc.cuh"
+
+#include <climits>
+
+namespace iq {
+
+enum ConvOp { OP_FWD = 0, OP_DGRAD = 1, OP_WGRAD = 2 };
+
+struct ConvP {
+    int N, H, W, C, K, R, S, sh, sw, ph, pw, dh, dw, G, P, Q;
+    int Cg, Kg;
+    int64_t M;       // GEMM rows: fwd N*P*Q, dgrad N*H*W, wgrad Kg
+    int ncols;       // GEMM cols per group: fwd Kg, dgrad Cg, wgrad R*S*Cg
+    int kin;         // fwd: Cg rounded up to 32; dgrad: Kg rounded up to 32
+    int64_t npq;     // wgrad: N*P*Q
+    int64_t chunk;   // wgrad: reduction length per split (multiple of 32)
+    int nsplit;      // wgrad: splits per group
+};
+
+constexpr int BM = 64, BN = 64, BK = 32;
+
+__device__ __forceinline__ void load8_bytes(const int8_t* p, int nvalid, uint32_t& lo,
+                                            uint32_t& hi) {
+    uint32_t b[8];
+#pragma unroll
+    for (int j = 0; j < 8; j++) b[j] = j < nvalid ? (uint32_t)(uint8_t)p[j] : 0u;
+    lo = b[0] | (b[1] << 8) | (b[2] << 16) | (b[3] << 24);
+    hi = b[4] | (b[5] << 8) | (b[6] << 16) | (b[7] << 24);
+}
+
+template <int OP>
+__global__ void __launch_bounds__(256) k_conv_simt(ConvP cp, const int8_t* __restrict__ A_src,
+                                                   const int8_t* __restrict__ B_src,
+                                                   int32_t* __restrict__ out32,
+                                                   long long* __restrict__ out64,
+                                                   unsigned long long* __restrict__ s1,
+                                                   int* __restrict__ hi_c, int* __restrict__ lo_c,
+                                                   unsigned long long* __restrict__ amax) {
+    __shared__ __align__(16) uint32_t As[BK / 4][BM];
+    __shared__ __align__(16) uint32_t Bs[BK / 4][BN];
+    __shared__ int s_n[BK], s_p[BK], s_q[BK];
+    __shared__ unsigned long long st_s1[BN];
+    __shared__ int st_hi[BN], st_lo[BN];
+
+    const int t = threadIdx.x;
+    const int ty = t >> 4, tx = t & 15;
+    const int lrow = t >> 2, lk = (t & 3) * 8;
+    int g, split = 0;
+    if (OP == OP_WGRAD) { g = blockIdx.z / cp.nsplit; split = blockIdx.z % cp.nsplit; }
+    else g = blockIdx.z;
+    const int64_t m0 = (int64_t)blockIdx.x * BM;
+    const int n0 = blockIdx.y * BN;
+
+    // per-thread decode of its load rows
+    const int64_t am = m0 + lrow;           // A row
+    const int bcol = n0 + lrow;             // B row (GEMM column)
+    int a_n = 0, a_p = 0, a_q = 0;
+    bool a_ok = am < cp.M;
+    if (OP == OP_FWD && a_ok) {
+        int64_t pq = (int64_t)cp.P * cp.Q;
+        a_n = (int)(am / pq);
+        int64_t rem = am - (int64_t)a_n * pq;
+        a_p = (int)(rem / cp.Q);
+        a_q = (int)(rem - (int64_t)a_p * cp.Q);
+    } else if (OP == OP_DGRAD && a_ok) {
+        int64_t hw = (int64_t)cp.H * cp.W;
+        a_n = (int)(am / hw);
+        int64_t rem = am - (int64_t)a_n * hw;
+        a_p = (int)(rem / cp.W);   // input row h
+        a_q = (int)(rem - (int64_t)a_p * cp.W);  // input col w
+    }
+    const bool b_ok = bcol < cp.ncols;
+    int b_r = 0, b_s = 0, b_c = 0;
+    if (OP == OP_WGRAD && b_ok) {
+        b_c = bcol % cp.Cg;
+        int rs = bcol / cp.Cg;
+        b_r = rs / cp.S;
+        b_s = rs % cp.S;
+    }
+
+    int acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; i++)
+#pragma unroll
+        for (int j = 0; j < 4; j++) acc[i][j] = 0;
+
+    // K iteration space
+    int64_t ktiles;
+    int64_t kbase0 = 0;
+    if (OP == OP_FWD) ktiles = (int64_t)cp.R * cp.S * (cp.kin / BK);
+    else if (OP == OP_DGRAD) ktiles = (int64_t)cp.R * cp.S * (cp.kin / BK);
+    else {
+        kbase0 = (int64_t)split * cp.chunk;
+        int64_t kend = kbase0 + cp.chunk;
+        if (kend > cp.npq) kend = cp.npq;
+        ktiles = kend > kbase0 ? (kend - kbase0 + BK - 1) / BK : 0;
+    }
+    const bool vec8 = (OP == OP_FWD) ? ((cp.Cg % 8) == 0 && (cp.C % 8) == 0)
+                                     : (OP == OP_DGRAD) ? ((cp.Kg % 8) == 0 && (cp.K % 8) == 0)
+                                                        : false;
+
+    for (int64_t kt = 0; kt < ktiles; kt++) {
+        uint32_t alo = 0, ahi = 0, blo = 0, bhi = 0;
+        if (OP == OP_FWD || OP == OP_DGRAD) {
+            int per = cp.kin / BK;
+            int tap = (int)(kt / per);
+            int c0 = (int)(kt - (int64_t)tap * per) * BK + lk;
+            int r = tap / cp.S, s = tap % cp.S;
+            int limit = (OP == OP_FWD) ? cp.Cg : cp.Kg;
+            int nvalid = limit - c0;
+            nvalid = nvalid < 0 ? 0 : (nvalid > 8 ? 8 : nvalid);
+            if (OP == OP_FWD) {
+                int hh = a_p * cp.sh + r * cp.dh - cp.ph;
+                int ww = a_q * cp.sw + s * cp.dw - cp.pw;
+                if (a_ok && nvalid > 0 && hh >= 0 && hh < cp.H && ww >= 0 && ww < cp.W) {
+                    const int8_t* p = A_src + (((int64_t)a_n * cp.H + hh) * cp.W + ww) * cp.C +
+                                      (int64_t)g * cp.Cg + c0;
+                    if (vec8) { int2 v = *reinterpret_cast<const int2*>(p); alo = v.x; ahi = v.y; }
+                    else load8_bytes(p, nvalid, alo, ahi);
+                }
+                if (b_ok && nvalid > 0) {
+                    int kg = g * cp.Kg + bcol;
+                    const int8_t* p = B_src + (((int64_t)kg * cp.R + r) * cp.S + s) * cp.Cg + c0;
+                    if (vec8) { int2 v = *reinterpret_cast<const int2*>(p); blo = v.x; bhi = v.y; }
+                    else load8_bytes(p, nvalid, blo, bhi);
+                }
+            } else {
+                int ph_ = a_p + cp.ph - r * cp.dh;
+                int pw_ = a_q + cp.pw - s * cp.dw;
+                bool ok = a_ok && nvalid > 0 && ph_ >= 0 && pw_ >= 0 && (ph_ % cp.sh) == 0 &&
+                          (pw_ % cp.sw) == 0;
+                if (ok) {
+                    int p = ph_ / cp.sh, q = pw_ / cp.sw;
+                    if (p < cp.P && q < cp.Q) {
+                        const int8_t* src = A_src + (((int64_t)a_n * cp.P + p) * cp.Q + q) * cp.K +
+                                            (int64_t)g * cp.Kg + c0;
+                        if (vec8) { int2 v = *reinterpret_cast<const int2*>(src); alo = v.x; ahi = v.y; }
+                        else load8_bytes(src, nvalid, alo, ahi);
+                    }
+                }
+                if (b_ok && nvalid > 0) {
+                    // transposed weights [G][Cg][R][S][Kg]
+                    const int8_t* src = B_src + ((((int64_t)g * cp.Cg + bcol) * cp.R + r) * cp.S + s) *
+                                                    cp.Kg + c0;
+                    if (vec8) { int2 v = *reinterpret_cast<const int2*>(src); blo = v.x; bhi = v.y; }
+                    else load8_bytes(src, nvalid, blo, bhi);
+                }
+            }
+        } else {
+            // wgrad: decode the 32 reduction pixels of this tile once
+            int64_t kb = kbase0 + kt * BK;
+            if (t < BK) {
+                int64_t j = kb + t;
+                int64_t kend = kbase0 + cp.chunk;
+                if (j < cp.npq && j < kend) {
+                    int64_t pq = (int64_t)cp.P * cp.Q;
+                    int nn = (int)(j / pq);
+                    int64_t rem = j - (int64_t)nn * pq;
+                    s_n[t] = nn;
+                    s_p[t] = (int)(rem / cp.Q);
+                    s_q[t] = (int)(rem - (int64_t)s_p[t] * cp.Q);
+                } else {
+                    s_n[t] = -1;
+                }
+            }
+            __syncthreads();
+            uint32_t ab[8], bb[8];
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                int jj = lk + j;
+                int nn = s_n[jj];
+                ab[j] = 0; bb[j] = 0;
+                if (nn >= 0) {
+                    int64_t pix = ((int64_t)nn * cp.P + s_p[jj]) * cp.Q + s_q[jj];
+                    if (a_ok) ab[j] = (uint8_t)A_src[pix * cp.K + (int64_t)g * cp.Kg + am];
+                    if (b_ok) {
+                        int hh = s_p[jj] * cp.sh + b_r * cp.dh - cp.ph;
+                        int ww = s_q[jj] * cp.sw + b_s * cp.dw - cp.pw;
+                        if (hh >= 0 && hh < cp.H && ww >= 0 && ww < cp.W)
+                            bb[j] = (uint8_t)B_src[(((int64_t)nn * cp.H + hh) * cp.W + ww) * cp.C +
+                                                   (int64_t)g * cp.Cg + b_c];
+                    }
+                }
+            }
+            alo = ab[0] | (ab[1] << 8) | (ab[2] << 16) | (ab[3] << 24);
+            ahi = ab[4] | (ab[5] << 8) | (ab[6] << 16) | (ab[7] << 24);
+            blo = bb[0] | (bb[1] << 8) | (bb[2] << 16) | (bb[3] << 24);
+            bhi = bb[4] | (bb[5] << 8) | (bb[6] << 16) | (bb[7] << 24);
+        }
+        As[lk / 4][lrow] = alo;
+        As[lk / 4 + 1][lrow] = ahi;
+        Bs[lk / 4][lrow] = blo;
+        Bs[lk / 4 + 1][lrow] = bhi;
+        __syncthreads();
+#pragma unroll
+        for (int kw = 0; kw < BK / 4; kw++) {
+            uint4 av = *reinterpret_cast<const uint4*>(&As[kw][ty * 4]);
+            uint4 bv = *reinterpret_cast<const uint4*>(&Bs[kw][tx * 4]);
+            int a4[4] = {(int)av.x, (int)av.y, (int)av.z, (int)av.w};
+            int b4[4] = {(int)bv.x, (int)bv.y, (int)bv.z, (int)bv.w};
+#pragma unroll
+            for (int i = 0; i < 4; i++)
+#pragma unroll
+                for (int j = 0; j < 4; j++) acc[i][j] = __dp4a(a4[i], b4[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+
+    // ---------------- epilogue
+    if (OP == OP_FWD) {
+        if (t < BN) { st_s1[t] = 0; st_hi[t] = INT_MIN; st_lo[t] = INT_MAX; }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            int col = n0 + tx * 4 + j;
+            if (col >= cp.ncols) continue;
+            long long sum = 0;
+            int h = INT_MIN, l = INT_MAX;
+            bool any = false;
+#pragma unroll
+            for (int i = 0; i < 4; i++) {
+                int64_t m = m0 + ty * 4 + i;
+                if (m >= cp.M) continue;
+                int v = acc[i][j];
+                out32[m * cp.K + (int64_t)g * cp.Kg + col] = v;
+                sum += v; h = max(h, v); l = min(l, v); any = true;
+            }
+            if (any) {
+                atomicAdd(&st_s1[tx * 4 + j], (unsigned long long)sum);
+                atomicMax(&st_hi[tx * 4 + j], h);
+                atomicMin(&st_lo[tx * 4 + j], l);
+            }
+        }
+        __syncthreads();
+        if (t < BN && n0 + t < cp.ncols && s1) {
+            int c = g * cp.Kg + n0 + t;
+            atomicAdd(&s1[c], st_s1[t]);
+            atomicMax(&hi_c[c], st_hi[t]);
+            atomicMin(&lo_c[c], st_lo[t]);
+        }
+    } else if (OP == OP_DGRAD) {
+        uint32_t mx = 0;
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+            int64_t m = m0 + ty * 4 + i;
+            if (m >= cp.M) continue;
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                int col = n0 + tx * 4 + j;
+                if (col >= cp.ncols) continue;
+                int v = acc[i][j];
+                out32[m * cp.C + (int64_t)g * cp.Cg + col] = v;
+                mx = max(mx, (uint32_t)(v < 0 ? -v : v));
+            }
+        }
+        mx = warp_max_u32(mx);
+        if ((t & 31) == 0 && mx) atomicMax(amax, (unsigned long long)mx);
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+            int64_t k = m0 + ty * 4 + i;
+            if (k >= cp.M) continue;
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                int col = n0 + tx * 4 + j;
+                if (col >= cp.ncols || acc[i][j] == 0) continue;
+                atomicAdd(reinterpret_cast<unsigned long long*>(
+                              &out64[((int64_t)g * cp.Kg + k) * cp.ncols + col]),
+                          (unsigned long long)(long long)acc[i][j]);
+            }
+        }
+    }
+}
+
+// dgrad weights: w[K][R][S][Cg] -> wT[G][Cg][R][S][Kg]
+__global__ void k_transpose_w(const int8_t* __restrict__ w, int8_t* __restrict__ wt, int K,
+                              int R, int S, int Cg, int G) {
+    int Kg = K / G;
+    int64_t total = (int64_t)K * R * S * Cg;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        int c = (int)(i % Cg);
+        int64_t t = i / Cg;
+        int s = (int)(t % S); t /= S;
+        int r = (int)(t % R);
+        int k = (int)(t / R);
+        int g = k / Kg, kl = k % Kg;
+        wt[((((int64_t)g * Cg + c) * R + r) * S + s) * Kg + kl] = w[i];
+    }
+}
+
+// ------------------------------------------------------------------ small scale kernels
+
+__global__ void k_scale_mul_pow2(const double* __restrict__ a, int e, double* __restrict__ out) {
+    *out = ldexp(*a, e);
+}
+__global__ void k_scale_mul(const double* __restrict__ a, const double* __restrict__ b,
+                            double* __restrict__ out) {
+    *out = __dmul_rn(*a, *b);
+}
+// M for SQ of the conv output from the per-channel extremes
+__global__ void k_max_from_stats(const int* __restrict__ hi, const int* __restrict__ lo, int C,
+                                 int relu, unsigned long long* __restrict__ cell) {
+    uint64_t m = 0;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        int64_t h = hi[c], l = lo[c];
+        uint64_t v = relu ? (uint64_t)(h > 0 ? h : 0)
+                          : (uint64_t)max(h < 0 ? -h : h, l < 0 ? -l : l);
+        m = v > m ? v : m;
+    }
+    m = warp_max_u64(m);
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(cell, (unsigned long long)m);
+}
+
+// ------------------------------------------------------------------ geometry helpers
+
+static bool desc_ok(const iq_conv_desc* d) {
+    if (!d) return false;
+    if (d->n <= 0 || d->h <= 0 || d->w <= 0 || d->c <= 0 || d->k <= 0 || d->r <= 0 || d->s <= 0)
+        return false;
+    if (d->stride_h <= 0 || d->stride_w <= 0 || d->pad_h < 0 || d->pad_w < 0 || d->dil_h <= 0 ||
+        d->dil_w <= 0 || d->groups <= 0)
+        return false;
+    if (d->c % d->groups || d->k % d->groups) return false;
+    int p = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1);
+    int q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1);
+    return p >= 0 && q >= 0;
+}
+
+static ConvP make_params(const iq_conv_desc* d) {
+    ConvP c;
+    c.N = d->n; c.H = d->h; c.W = d->w; c.C = d->c; c.K = d->k; c.R = d->r; c.S = d->s;
+    c.sh = d->stride_h; c.sw = d->stride_w; c.ph = d->pad_h; c.pw = d->pad_w;
+    c.dh = d->dil_h; c.dw = d->dil_w; c.G = d->groups;
+    c.P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    c.Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    c.Cg = d->c / d->groups;
+    c.Kg = d->k / d->groups;
+    c.M = 0; c.ncols = 0; c.kin = 0; c.npq = (int64_t)c.N * c.P * c.Q; c.chunk = 0; c.nsplit = 1;
+    return c;
+}
+
+static int64_t roundup(int64_t a, int64_t b) { return (a + b - 1) / b * b; }
+
+struct FwdWs {
+    int32_t* acc;
+    BnStats st;
+    void* rq;
+    double* s_acc;
+};
+
+static size_t fwd_ws_layout(const iq_conv_desc* d, int with_acc, void* base, size_t cap,
+                            FwdWs* out) {
+    ConvP cp = make_params(d);
+    WsCursor cur(base, cap);
+    FwdWs w;
+    w.acc = with_acc ? cur.take<int32_t>((size_t)cp.npq * cp.K) : nullptr;
+    w.st = bn_stats_carve(cur, cp.K);
+    w.rq = cur.take<char>(requant_ws_bytes());
+    w.s_acc = cur.take<double>(1);
+    if (out) *out = w;
+    return cur.off + 256;
+}
+
+}  // namespace iq
+
+using namespace iq;
+
+// ==================================================================== C ABI
+
+extern "C" iq_status iq_conv_out_size(const iq_conv_desc* d, int32_t* p, int32_t* q) {
+    if (!desc_ok(d) || !p || !q) return IQ_ERR_INVALID_ARG;
+    ConvP c = make_params(d);
+    *p = c.P;
+    *q = c.Q;
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_conv_fwd_workspace_size(const iq_conv_desc* d, int with_bn, size_t* bytes) {
+    (void)with_bn;
+    if (!desc_ok(d) || !bytes) return IQ_ERR_INVALID_ARG;
+    *bytes = fwd_ws_layout(d, 1, nullptr, 0, nullptr);
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_conv_dgrad_workspace_size(const iq_conv_desc* d, size_t* bytes) {
+    if (!desc_ok(d) || !bytes) return IQ_ERR_INVALID_ARG;
+    WsCursor cur(nullptr, 0);
+    cur.take<int8_t>((size_t)d->k * d->r * d->s * (d->c / d->groups));
+    cur.take<int32_t>((size_t)d->n * d->h * d->w * d->c);
+    cur.take<char>(requant_ws_bytes());
+    cur.take<double>(1);
+    *bytes = cur.off + 256;
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_conv_wgrad_workspace_size(const iq_conv_desc* d, size_t* bytes) {
+    if (!desc_ok(d) || !bytes) return IQ_ERR_INVALID_ARG;
+    WsCursor cur(nullptr, 0);
+    cur.take<int64_t>((size_t)d->k * d->r * d->s * (d->c / d->groups));
+    cur.take<char>(requant_ws_bytes());
+    cur.take<double>(1);
+    *bytes = cur.off + 256;
+    return IQ_OK;
+}
+
+static bool crs_overflow(const iq_conv_desc* d) {
+    int64_t crs = (int64_t)(d->c / d->groups) * d->r * d->s;
+    return crs * 127 * 127 >= (int64_t(1) << 31);
+}
+
+extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
+                                 const int8_t* w, const int32_t* gamma, const int32_t* beta,
+                                 const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
+                                 double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
+                                 int32_t* acc_out, void* ws, size_t ws_bytes, iq_stream stream) {
+    if (!desc_ok(d) || !x || !s_x || !w || !a || !s_a) return IQ_ERR_INVALID_ARG;
+    if (crs_overflow(d)) return IQ_ERR_OVERFLOW_RISK;
+    iq_bn_bits b = bn_bits_or_default(bits);
+    if (use_bn) {
+        if (!gamma || !beta || !bn_bits_valid(b)) return IQ_ERR_INVALID_ARG;
+        if (d->k % 4) return IQ_ERR_UNSUPPORTED;
+        if (((uintptr_t)a | (uintptr_t)xhat | (uintptr_t)acc_out) & 15) return IQ_ERR_INVALID_ARG;
+    }
+    cudaStream_t st = (cudaStream_t)stream;
+    FwdWs L;
+    size_t need = fwd_ws_layout(d, acc_out == nullptr, nullptr, 0, nullptr);
+    if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    fwd_ws_layout(d, acc_out == nullptr, ws, ws_bytes, &L);
+    int32_t* acc = acc_out ? acc_out : L.acc;
+    ConvP cp = make_params(d);
+    cp.M = cp.npq;
+    cp.ncols = cp.Kg;
+    cp.kin = (int)roundup(cp.Cg, BK);
+
+    iq_status r = bn_stats_init(L.st, cp.K, st);
+    if (r != IQ_OK) return r;
+    k_scale_mul_pow2<<<1, 1, 0, st>>>(s_x, -7, L.s_acc);  // s_acc = s_x * 2^-7 (W_q step)
+    IQ_LAUNCH_CHECK();
+    bool done = false;
+    r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, st, &done);
+    if (r != IQ_OK) return r;
+    if (!done) {
+        dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
+        k_conv_simt<OP_FWD><<<grid, 256, 0, st>>>(cp, x, w, acc, nullptr, L.st.s1, L.st.hi,
+                                                  L.st.lo, nullptr);
+        IQ_LAUNCH_CHECK();
+    }
+    if (use_bn)
+        return bn_fwd_after_stats(acc, cp.M, cp.K, L.s_acc, gamma, beta, b, L.st, xhat, a, s_a,
+                                  bn_codes, bn_scales, nullptr, st);
+    // Q_A = SQ(act(acc), 8) with M from the per-channel extremes
+    unsigned long long* cell = (unsigned long long*)L.rq;
+    IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
+    k_max_from_stats<<<1, 1024, 0, st>>>(L.st.hi, L.st.lo, cp.K, relu, cell);
+    IQ_LAUNCH_CHECK();
+    return requant_apply(acc, IQ_I32, cp.npq * cp.K, L.s_acc, 8,
+                         relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ, 0, 0, 0, 0, a, IQ_I8, s_a, L.rq, st);
+}
+
+extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
+                                   const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
+                                   void* ws, size_t ws_bytes, iq_stream stream) {
+    if (!desc_ok(d) || !e || !s_e || !w || !dx || !s_dx) return IQ_ERR_INVALID_ARG;
+    int64_t krs = (int64_t)(d->k / d->groups) * d->r * d->s;
+    if (krs * 127 * 127 >= (int64_t(1) << 31)) return IQ_ERR_OVERFLOW_RISK;
+    size_t need = 0;
+    iq_conv_dgrad_workspace_size(d, &need);
+    if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    ConvP cp = make_params(d);
+    WsCursor cur(ws, ws_bytes);
+    int8_t* wt = cur.take<int8_t>((size_t)d->k * d->r * d->s * cp.Cg);
+    int32_t* accw = cur.take<int32_t>((size_t)d->n * d->h * d->w * d->c);
+    void* rq = cur.take<char>(requant_ws_bytes());
+    double* s_in = cur.take<double>(1);
+    int32_t* acc = acc_out ? acc_out : accw;
+    int64_t wn = (int64_t)d->k * d->r * d->s * cp.Cg;
+    k_transpose_w<<<grid_for(wn), kThreads, 0, st>>>(w, wt, d->k, d->r, d->s, cp.Cg, d->groups);
+    IQ_LAUNCH_CHECK();
+    unsigned long long* cell = (unsigned long long*)rq;
+    IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
+    cp.M = (int64_t)d->n * d->h * d->w;
+    cp.ncols = cp.Cg;
+    cp.kin = (int)roundup(cp.Kg, BK);
+    dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
+    k_conv_simt<OP_DGRAD><<<grid, 256, 0, st>>>(cp, e, wt, acc, nullptr, nullptr, nullptr,
+                                                nullptr, cell);
+    IQ_LAUNCH_CHECK();
+    k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, -7, s_in);
+    IQ_LAUNCH_CHECK();
+    return requant_apply(acc, IQ_I32, cp.M * d->c, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
+                         s_dx, rq, st);
+}
+
+extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
+                                   const int8_t* x, const double* s_x, int gq_mode, uint64_t seed,
+                                   uint64_t layer, uint64_t step, int8_t* g, double* s_g,
+                                   int64_t* g_acc_out, void* ws, size_t ws_bytes,
+                                   iq_stream stream) {
+    if (!desc_ok(d) || !e || !s_e || !x || !s_x || !g || !s_g) return IQ_ERR_INVALID_ARG;
+    if (gq_mode != 1 && gq_mode != 2) return IQ_ERR_INVALID_ARG;
+    size_t need = 0;
+    iq_conv_wgrad_workspace_size(d, &need);
+    if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    ConvP cp = make_params(d);
+    // |G| < npq 127^2 must stay below 2^40 for the requantizer
+    if ((double)cp.npq * 16129.0 >= 1099511627776.0) return IQ_ERR_OVERFLOW_RISK;
+    cudaStream_t st = (cudaStream_t)stream;
+    WsCursor cur(ws, ws_bytes);
+    int64_t gn = (int64_t)d->k * d->r * d->s * cp.Cg;
+    int64_t* gw = cur.take<int64_t>((size_t)gn);
+    void* rq = cur.take<char>(requant_ws_bytes());
+    double* s_in = cur.take<double>(1);
+    int64_t* G = g_acc_out ? g_acc_out : gw;
+    IQ_CUDA_CHECK(cudaMemsetAsync(G, 0, sizeof(int64_t) * gn, st));
+    cp.M = cp.Kg;
+    cp.ncols = d->r * d->s * cp.Cg;
+    int64_t tiles = ((cp.M + BM - 1) / BM) * ((cp.ncols + BN - 1) / BN) * cp.G;
+    int64_t want_split = (152 * 8 + tiles - 1) / tiles;
+    int64_t max_split = (cp.npq + 1023) / 1024;   // chunk >= 1024 reduction pixels
+    if (want_split > max_split) want_split = max_split;
+    if (want_split < 1) want_split = 1;
+    cp.chunk = roundup((cp.npq + want_split - 1) / want_split, BK);
+    if (cp.chunk > 65536) cp.chunk = 65536;      // int32 partial sums: 65536 * 127^2 < 2^31
+    cp.nsplit = (int)((cp.npq + cp.chunk - 1) / cp.chunk);
+    dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN),
+              (unsigned)(cp.G * cp.nsplit));
+    k_conv_simt<OP_WGRAD><<<grid, 256, 0, st>>>(cp, e, x, nullptr, (long long*)G, nullptr, nullptr,
+                                                nullptr, nullptr);
+    IQ_LAUNCH_CHECK();
+    k_scale_mul<<<1, 1, 0, st>>>(s_e, s_x, s_in);
+    IQ_LAUNCH_CHECK();
+    return requant_int(G, IQ_I64, gn, s_in, 8, gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2,
+                       seed, layer, step, 0, g, IQ_I8, s_g, rq, st);
+}

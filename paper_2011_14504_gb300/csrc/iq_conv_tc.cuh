@@ -1,0 +1,14 @@
+// iq_conv_tc.cuh -- tensor-core (tcgen05) convolution path.
+#pragma once
+
+#include "iq_internal.cuh"
+
+namespace iq {
+
+// Forward convolution on the 5th-generation tensor cores when the shape is
+// supported; sets *done = false (and enqueues nothing) otherwise.  Writes the int32
+// accumulators and the per-channel sum / max / min like the CUDA-core path.
+iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, int32_t* acc,
+                      unsigned long long* s1, int* hi, int* lo, cudaStream_t st, bool* done);
+
+}  // namespace iq

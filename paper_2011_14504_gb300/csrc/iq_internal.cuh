@@ -1,0 +1,65 @@
+// iq_internal.cuh -- launchers shared between the translation units of the library.
+#pragma once
+
+#include "iq_common.cuh"
+
+namespace iq {
+
+// Scratch needed by requant_int (bytes).
+size_t requant_ws_bytes();
+
+// SQ / RQ of an integer-coded tensor (see iq_requantize in iq.h).  `relu` applies
+// to the SQ modes only.  `out` has out_dtype elements.
+iq_status requant_int(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
+                      int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
+                      void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st);
+
+// The same with max |q| already in the first 8 bytes of ws (an unsigned long long).
+iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
+                        int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
+                        void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st);
+
+// Per-channel statistics buffers of a BN layer, in the workspace.
+struct BnStats {
+    unsigned long long* s1;   // sum acc (two's complement int64)
+    int* hi;                  // max acc
+    int* lo;                  // min acc
+    unsigned long long* dev;  // sum |acc - floor(S1/m)|
+    unsigned long long* ngt;  // #(acc > floor(S1/m))
+    long long* F;             // fixed-point maps acc -> X and X -> A
+    long long* B;
+    long long* G;
+    long long* H;
+    int* codes;               // [2C]: mu_q codes, sigma_q codes
+    int* px;                  // shifts [2]
+    double* scal;             // IQ_BN_SCALES doubles (workspace copy)
+};
+
+size_t bn_fwd_ws_bytes(int32_t C);
+BnStats bn_stats_carve(WsCursor& cur, int32_t C);
+// zero sums, hi = INT_MIN, lo = INT_MAX
+iq_status bn_stats_init(const BnStats& s, int32_t C, cudaStream_t st);
+// channel sums / extremes of acc[m][C] (when the producer did not fuse them)
+iq_status bn_stats_pass(const int32_t* acc, int64_t m, int32_t C, const BnStats& s,
+                        cudaStream_t st);
+// everything after the statistics: deviation pass, finalize, requant pass
+iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const double* s_acc,
+                             const int32_t* gamma, const int32_t* beta, const iq_bn_bits& b,
+                             const BnStats& s, int16_t* xhat, int8_t* a, double* s_a,
+                             int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
+                             cudaStream_t st);
+
+inline iq_bn_bits bn_bits_or_default(const iq_bn_bits* b) {
+    if (b) return *b;
+    iq_bn_bits d;
+    d.k_mu = 16; d.k_sigma = 16; d.k_xhat = 16; d.k_gamma = 8; d.k_beta = 8; d.k_a = 8;
+    return d;
+}
+
+inline bool bn_bits_valid(const iq_bn_bits& b) {
+    return b.k_mu >= 2 && b.k_mu <= 24 && b.k_sigma >= 2 && b.k_sigma <= 24 &&
+           b.k_xhat >= 2 && b.k_xhat <= 16 && b.k_gamma >= 2 && b.k_gamma <= 16 &&
+           b.k_beta >= 2 && b.k_beta <= 16 && b.k_a >= 2 && b.k_a <= 8;
+}
+
+}  // namespace iq

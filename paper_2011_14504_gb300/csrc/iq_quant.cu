@@ -1,0 +1,457 @@
+// iq_quant.cu -- the quantizers of Sec. 3.1 and the update of Sec. 3.3.3.
+//
+// Bandwidth-bound element-wise kernels: 16-byte loads where the layout allows,
+// grid-stride loops over a grid of a few blocks per SM, warp-shuffle + one
+// atomic per warp for the tensor-wide max |x| that Scale(x) needs.
+#include "iq_internal.cuh"
+
+#include <climits>
+
+namespace iq {
+
+// ------------------------------------------------------------------ absmax
+
+// max |x| of fp32 data as the bit pattern of |x| (non-negative floats order as
+// their unsigned bit patterns).
+__global__ void k_absmax_f32(const float* __restrict__ x, int64_t n, int relu,
+                             unsigned* __restrict__ cell) {
+    uint32_t m = 0;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    int64_t n4 = (((uintptr_t)x & 15) == 0) ? n / 4 : 0;
+    const float4* x4 = reinterpret_cast<const float4*>(x);
+    for (int64_t v = i; v < n4; v += stride) {
+        float4 f = x4[v];
+        float a[4] = {f.x, f.y, f.z, f.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            float t = relu ? fmaxf(a[j], 0.0f) : fabsf(a[j]);
+            m = max(m, __float_as_uint(t));
+        }
+    }
+    for (int64_t v = n4 * 4 + i; v < n; v += stride) {
+        float t = relu ? fmaxf(x[v], 0.0f) : fabsf(x[v]);
+        m = max(m, __float_as_uint(t));
+    }
+    m = warp_max_u32(m);
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(cell, m);
+}
+
+template <typename T>
+__global__ void k_absmax_int(const T* __restrict__ q, int64_t n, int relu,
+                             unsigned long long* __restrict__ cell) {
+    uint64_t m = 0;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        int64_t v = (int64_t)q[i];
+        if (relu && v < 0) v = 0;
+        uint64_t a = (uint64_t)(v < 0 ? -v : v);
+        m = a > m ? a : m;
+    }
+    m = warp_max_u64(m);
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(cell, (unsigned long long)m);
+}
+
+// ------------------------------------------------------------------ stores
+
+__device__ __forceinline__ void store_code(void* out, int dtype, int64_t i, int64_t c) {
+    if (dtype == IQ_I8) ((int8_t*)out)[i] = (int8_t)c;
+    else if (dtype == IQ_I16) ((int16_t*)out)[i] = (int16_t)c;
+    else ((int32_t*)out)[i] = (int32_t)c;
+}
+
+// ------------------------------------------------------------------ UQ / UQ2 / SQ on fp32
+
+// Eq. (UQ): code = clip(floor(x 2^sh + 1/2)), sh = k-1 (UQ) or k-2 (2*UQ(x/2)).
+__global__ void k_uq_f32(const float* __restrict__ x, int64_t n, int k, int sh,
+                         void* __restrict__ out, int dtype) {
+    const double p2 = ldexp(1.0, sh);
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
+        store_code(out, dtype, i, code_of(__dmul_rn((double)x[i], p2), k));
+}
+
+// Eq. (ScaleQ) on fp32: S = max|x| (cell, as bits); code = clip(rhu(x/S 2^(k-1)))
+// with x/S formed in fp64 (its rhu equals that of the exact quotient).
+__global__ void k_sq_f32(const float* __restrict__ x, int64_t n, int k, int relu,
+                         const unsigned* __restrict__ cell, void* __restrict__ out, int dtype) {
+    const float S = __uint_as_float(*cell);
+    const double Sd = (double)S, p2 = ldexp(1.0, k - 1);
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        float v = relu ? fmaxf(x[i], 0.0f) : x[i];
+        int64_t c = 0;
+        if (S != 0.0f) c = code_of(__dmul_rn(__ddiv_rn((double)v, Sd), p2), k);
+        store_code(out, dtype, i, c);
+    }
+}
+
+__global__ void k_set_double(double* p, double v) { *p = v; }
+
+__global__ void k_sq_f32_scale(const unsigned* __restrict__ cell, int k, double* s_out) {
+    float S = __uint_as_float(*cell);
+    *s_out = S != 0.0f ? ldexp((double)S, 1 - k) : ldexp(1.0, 1 - k);
+}
+
+// ------------------------------------------------------------------ SQ / RQ on integer codes
+
+struct RqParams {
+    uint64_t M;
+    UDiv div;      // by 2M (SQ) or by M (RQ)
+    double s_out;
+};
+
+size_t requant_ws_bytes() { return 512; }
+
+__global__ void k_rq_finalize(const unsigned long long* __restrict__ cell,
+                              const double* __restrict__ s_in, int k, int mode,
+                              RqParams* __restrict__ prm, double* __restrict__ s_out) {
+    uint64_t M = *cell;
+    double s = s_in ? *s_in : 1.0;
+    RqParams p;
+    p.M = M;
+    bool rq = mode == IQ_MODE_RQ_GQ1 || mode == IQ_MODE_RQ_GQ2;
+    p.div = make_udiv(M == 0 ? 1 : (rq ? M : 2 * M));
+    double Md = (double)M;
+    if (mode == IQ_MODE_RQ_GQ2) p.s_out = ldexp(1.0, 1 - k);
+    else p.s_out = M ? ldexp(__dmul_rn(s, Md), 1 - k) : ldexp(s, 1 - k);
+    *prm = p;
+    if (s_out) *s_out = p.s_out;
+}
+
+// SQ: code = floor((2^k (q + M) + M) / (2M)) - 2^(k-1), the non-negative shift of
+// floor((2^k q + M) / (2M)); the numerator is < 2^(k+1) M + M < 2^57.
+template <typename T>
+__global__ void k_sq_int(const T* __restrict__ q, int64_t n, int k, int relu,
+                         const RqParams* __restrict__ prm, void* __restrict__ out, int dtype) {
+    const RqParams p = *prm;
+    const int64_t lim = qmax(k);
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        int64_t v = (int64_t)q[i];
+        if (relu && v < 0) v = 0;
+        int64_t c = 0;
+        if (p.M) {
+            uint64_t num = ((uint64_t)(v + (int64_t)p.M) << k) + p.M;
+            c = (int64_t)udiv(num, p.div) - (int64_t(1) << (k - 1));
+            c = clamp64(c, -lim, lim);
+        }
+        store_code(out, dtype, i, c);
+    }
+}
+
+// RQ (Eqs. (SQ),(SR)): with num = (q + M) 2^(k-1) >= 0, f = floor(num/M) - 2^(k-1),
+// rem = num mod M; round up iff u M < rem 2^32 for the element's Philox word u.
+// One Philox block serves 8 consecutive elements.
+template <typename T>
+__global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
+                         const RqParams* __restrict__ prm, uint64_t seed, uint64_t layer,
+                         uint64_t step, uint64_t tag, void* __restrict__ out, int dtype) {
+    const RqParams p = *prm;
+    const int64_t lim = qmax(k);
+    const int64_t nb = (n + 7) / 8;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nb; b += stride) {
+        uint64_t w[4];
+        philox4x64_10((uint64_t)b, step, tag, 0, seed, layer, w);
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            int64_t i = b * 8 + j;
+            if (i >= n) break;
+            int64_t c = 0;
+            if (p.M) {
+                uint64_t num = (uint64_t)((int64_t)q[i] + (int64_t)p.M) << (k - 1);
+                uint64_t fq = udiv(num, p.div);
+                uint64_t rem = num - fq * p.M;
+                uint64_t word = w[j >> 1];
+                uint32_t u = (j & 1) ? (uint32_t)(word >> 32) : (uint32_t)word;
+                bool up = ((u128)u * p.M) < ((u128)rem << 32);
+                c = (int64_t)fq - (int64_t(1) << (k - 1)) + (up ? 1 : 0);
+                c = clamp64(c, -lim, lim);
+            }
+            store_code(out, dtype, i, c);
+        }
+    }
+}
+
+iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
+                        int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
+                        void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st) {
+    unsigned long long* cell = (unsigned long long*)ws;
+    RqParams* prm = (RqParams*)((char*)ws + 256);
+    bool relu = mode == IQ_MODE_SQ_RELU;
+    int g = grid_for(n);
+    k_rq_finalize<<<1, 1, 0, st>>>(cell, s_in, k, mode, prm, s_out);
+    IQ_LAUNCH_CHECK();
+    if (n == 0) return IQ_OK;
+    if (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) {
+        if (in_dtype == IQ_I32)
+            k_sq_int<int32_t><<<g, kThreads, 0, st>>>((const int32_t*)q, n, k, relu, prm, out,
+                                                      out_dtype);
+        else
+            k_sq_int<int64_t><<<g, kThreads, 0, st>>>((const int64_t*)q, n, k, relu, prm, out,
+                                                      out_dtype);
+    } else {
+        int gb = grid_for((n + 7) / 8);
+        if (in_dtype == IQ_I32)
+            k_rq_int<int32_t><<<gb, kThreads, 0, st>>>((const int32_t*)q, n, k, prm, seed, layer,
+                                                       step, tag, out, out_dtype);
+        else
+            k_rq_int<int64_t><<<gb, kThreads, 0, st>>>((const int64_t*)q, n, k, prm, seed, layer,
+                                                       step, tag, out, out_dtype);
+    }
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+iq_status requant_int(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
+                      int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
+                      void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st) {
+    unsigned long long* cell = (unsigned long long*)ws;
+    bool relu = mode == IQ_MODE_SQ_RELU;
+    IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
+    if (n > 0) {
+        int g = grid_for(n);
+        if (in_dtype == IQ_I32)
+            k_absmax_int<int32_t><<<g, kThreads, 0, st>>>((const int32_t*)q, n, relu, cell);
+        else
+            k_absmax_int<int64_t><<<g, kThreads, 0, st>>>((const int64_t*)q, n, relu, cell);
+        IQ_LAUNCH_CHECK();
+    }
+    return requant_apply(q, in_dtype, n, s_in, k, mode, seed, layer, step, tag, out, out_dtype,
+                         s_out, ws, st);
+}
+
+// ------------------------------------------------------------------ image input
+
+// pixel/255 -> SQ8: code = floor((256 p + P) / (2P)) for P = max pixel.
+__global__ void k_absmax_u8(const uint8_t* __restrict__ x, int64_t n, unsigned* cell) {
+    uint32_t m = 0;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
+        m = max(m, (uint32_t)x[i]);
+    m = warp_max_u32(m);
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(cell, m);
+}
+
+__global__ void k_image_sq8(const uint8_t* __restrict__ img, int32_t N, int32_t H, int32_t W,
+                            int32_t Cin, int nchw, int32_t Cout, const unsigned* __restrict__ cell,
+                            int8_t* __restrict__ out) {
+    const uint32_t P = *cell;
+    const int64_t total = (int64_t)N * H * W * Cout;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+        int32_t c = (int32_t)(i % Cout);
+        int64_t pix = i / Cout;
+        int8_t code = 0;
+        if (c < Cin && P) {
+            int64_t w = pix % W, h = (pix / W) % H, nn = pix / ((int64_t)W * H);
+            int64_t src = nchw ? ((nn * Cin + c) * H + h) * W + w : pix * Cin + c;
+            uint32_t p = img[src];
+            uint32_t v = (256u * p + P) / (2u * P);
+            code = (int8_t)(v > 127u ? 127u : v);
+        }
+        out[i] = code;
+    }
+}
+
+__global__ void k_image_scale(const unsigned* __restrict__ cell, double* s) {
+    uint32_t P = *cell;
+    *s = P ? ldexp(__ddiv_rn((double)P, 255.0), -7) : ldexp(1.0, -7);
+}
+
+// ------------------------------------------------------------------ weights and update
+
+// Eq. (WQ1): wq = clip(floor((m + 2^(sh-1)) / 2^sh)), sh = k_u - k_w.
+__global__ void k_weight_requant(const int32_t* __restrict__ m, int8_t* __restrict__ wq,
+                                 int64_t n, int sh, int k_w) {
+    const int64_t lim = qmax(k_w);
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        int64_t v = ((int64_t)m[i] + (int64_t(1) << (sh - 1))) >> sh;
+        wq[i] = (int8_t)clamp64(v, -lim, lim);
+    }
+}
+
+// Eq. (UQ2): dW = UQ(G_q lr, k_u) = clip(rhu(c s_g 2^(k_u-1-lr_log2))) (x2 grid: k_u-2),
+// m <- clip(m - dW), then wq = UQ(W_m, k_w).
+__global__ void k_update(int32_t* __restrict__ master, int8_t* __restrict__ wq,
+                         const int8_t* __restrict__ g, const double* __restrict__ s_g,
+                         int64_t n, int sh, int k_u, int k_w) {
+    const double s = *s_g;
+    const double p2 = ldexp(1.0, sh);
+    const int64_t lu = qmax(k_u), lw = qmax(k_w);
+    const int dsh = k_u - k_w;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        double t = __dmul_rn(__dmul_rn((double)g[i], s), p2);
+        int64_t du = code_of(t, k_u);
+        int64_t nm = clamp64((int64_t)master[i] - du, -lu, lu);
+        master[i] = (int32_t)nm;
+        int64_t v = (nm + (int64_t(1) << (dsh - 1))) >> dsh;
+        wq[i] = (int8_t)clamp64(v, -lw, lw);
+    }
+}
+
+__global__ void k_relu_bwd(const int8_t* __restrict__ ea, const int8_t* __restrict__ a,
+                           int64_t n, int8_t* __restrict__ e) {
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    bool vec = (((uintptr_t)ea | (uintptr_t)a | (uintptr_t)e) & 15) == 0;
+    int64_t n16 = vec ? n / 16 : 0;
+    for (int64_t v = i0; v < n16; v += stride) {
+        int4 x = reinterpret_cast<const int4*>(ea)[v];
+        int4 m = reinterpret_cast<const int4*>(a)[v];
+        int xs[4] = {x.x, x.y, x.z, x.w}, ms[4] = {m.x, m.y, m.z, m.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            uint32_t r = 0;
+#pragma unroll
+            for (int b = 0; b < 4; b++) {
+                int8_t mv = (int8_t)(ms[j] >> (8 * b));
+                uint32_t xv = ((uint32_t)xs[j] >> (8 * b)) & 0xffu;
+                r |= (mv > 0 ? xv : 0u) << (8 * b);
+            }
+            xs[j] = (int)r;
+        }
+        reinterpret_cast<int4*>(e)[v] = make_int4(xs[0], xs[1], xs[2], xs[3]);
+    }
+    for (int64_t i = n16 * 16 + i0; i < n; i += stride) e[i] = a[i] > 0 ? ea[i] : 0;
+}
+
+}  // namespace iq
+
+using namespace iq;
+
+// ==================================================================== C ABI
+
+extern "C" const char* iq_status_str(iq_status s) {
+    switch (s) {
+        case IQ_OK: return "ok";
+        case IQ_ERR_INVALID_ARG: return "invalid argument";
+        case IQ_ERR_UNSUPPORTED: return "unsupported";
+        case IQ_ERR_WORKSPACE: return "workspace too small";
+        case IQ_ERR_OVERFLOW_RISK: return "int32 accumulation could overflow";
+        case IQ_ERR_TIMEOUT: return "device wait timed out";
+        case IQ_ERR_CUDA: return "CUDA error";
+    }
+    return "unknown status";
+}
+
+extern "C" int iq_version(void) { return 1; }
+
+extern "C" iq_status iq_quantize_workspace_size(int64_t n, size_t* bytes) {
+    if (!bytes || n < 0) return IQ_ERR_INVALID_ARG;
+    *bytes = requant_ws_bytes();
+    return IQ_OK;
+}
+
+static bool dtype_holds(int dtype, int k) {
+    return (dtype == IQ_I8 && k <= 8) || (dtype == IQ_I16 && k <= 16) ||
+           (dtype == IQ_I32 && k <= 24);
+}
+
+extern "C" iq_status iq_quantize(const float* x, int64_t n, int k, int mode, int out_dtype,
+                                 void* codes, double* scale, void* ws, size_t ws_bytes,
+                                 iq_stream stream) {
+    cudaStream_t st = (cudaStream_t)stream;
+    if (n < 0 || (n > 0 && (!x || !codes)) || k < 2) return IQ_ERR_INVALID_ARG;
+    if (!dtype_holds(out_dtype, k)) return IQ_ERR_INVALID_ARG;
+    if (mode == IQ_MODE_UQ || mode == IQ_MODE_UQ2) {
+        if (k > 24) return IQ_ERR_INVALID_ARG;
+        if (n > 0) {
+            k_uq_f32<<<grid_for(n), kThreads, 0, st>>>(x, n, k, mode == IQ_MODE_UQ ? k - 1 : k - 2,
+                                                        codes, out_dtype);
+            IQ_LAUNCH_CHECK();
+        }
+        if (scale) {
+            k_set_double<<<1, 1, 0, st>>>(scale, ldexp(1.0, mode == IQ_MODE_UQ ? 1 - k : 2 - k));
+            IQ_LAUNCH_CHECK();
+        }
+        return IQ_OK;
+    }
+    if (mode != IQ_MODE_SQ && mode != IQ_MODE_SQ_RELU) return IQ_ERR_INVALID_ARG;
+    if (k > 16 || !scale) return IQ_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < requant_ws_bytes()) return IQ_ERR_WORKSPACE;
+    unsigned* cell = (unsigned*)ws;
+    int relu = mode == IQ_MODE_SQ_RELU;
+    IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned), st));
+    if (n > 0) {
+        k_absmax_f32<<<grid_for(n / 4 + 1), kThreads, 0, st>>>(x, n, relu, cell);
+        IQ_LAUNCH_CHECK();
+        k_sq_f32<<<grid_for(n), kThreads, 0, st>>>(x, n, k, relu, cell, codes, out_dtype);
+        IQ_LAUNCH_CHECK();
+    }
+    k_sq_f32_scale<<<1, 1, 0, st>>>(cell, k, scale);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_quantize_image_u8(const uint8_t* img, int32_t n, int32_t h, int32_t w,
+                                          int32_t c, int nchw, int32_t c_out, int8_t* codes,
+                                          double* scale, void* ws, size_t ws_bytes,
+                                          iq_stream stream) {
+    cudaStream_t st = (cudaStream_t)stream;
+    if (!img || !codes || !scale || n <= 0 || h <= 0 || w <= 0 || c <= 0 || c_out < c)
+        return IQ_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < requant_ws_bytes()) return IQ_ERR_WORKSPACE;
+    unsigned* cell = (unsigned*)ws;
+    int64_t nin = (int64_t)n * h * w * c;
+    IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned), st));
+    k_absmax_u8<<<grid_for(nin), kThreads, 0, st>>>(img, nin, cell);
+    IQ_LAUNCH_CHECK();
+    k_image_sq8<<<grid_for((int64_t)n * h * w * c_out), kThreads, 0, st>>>(img, n, h, w, c, nchw,
+                                                                           c_out, cell, codes);
+    IQ_LAUNCH_CHECK();
+    k_image_scale<<<1, 1, 0, st>>>(cell, scale);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_requantize(const void* q, int in_dtype, int64_t n, const double* s_in,
+                                   int k, int mode, uint64_t seed, uint64_t layer, uint64_t step,
+                                   uint64_t tag, void* codes, int out_dtype, double* s_out,
+                                   void* ws, size_t ws_bytes, iq_stream stream) {
+    if (n < 0 || (n > 0 && (!q || !codes)) || !s_out) return IQ_ERR_INVALID_ARG;
+    if (in_dtype != IQ_I32 && in_dtype != IQ_I64) return IQ_ERR_INVALID_ARG;
+    if (k < 2 || k > 16 || !dtype_holds(out_dtype, k)) return IQ_ERR_INVALID_ARG;
+    if (mode < IQ_MODE_SQ || mode > IQ_MODE_RQ_GQ2) return IQ_ERR_INVALID_ARG;
+    if (mode != IQ_MODE_RQ_GQ2 && !s_in) return IQ_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < requant_ws_bytes()) return IQ_ERR_WORKSPACE;
+    return requant_int(q, in_dtype, n, s_in, k, mode, seed, layer, step, tag, codes, out_dtype,
+                       s_out, ws, (cudaStream_t)stream);
+}
+
+extern "C" iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_u,
+                                       int k_w, iq_stream stream) {
+    if (!master || !wq || n < 0 || k_w < 2 || k_w > 8 || k_u <= k_w || k_u > 31)
+        return IQ_ERR_INVALID_ARG;
+    if (n == 0) return IQ_OK;
+    k_weight_requant<<<grid_for(n), kThreads, 0, (cudaStream_t)stream>>>(master, wq, n, k_u - k_w,
+                                                                          k_w);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_update(int32_t* master, int8_t* wq, const int8_t* g, const double* s_g,
+                               int64_t n, int lr_log2, int k_u, int k_w, int x2,
+                               iq_stream stream) {
+    if (!master || !wq || !g || !s_g || n < 0 || k_w < 2 || k_w > 8 || k_u <= k_w || k_u > 31)
+        return IQ_ERR_INVALID_ARG;
+    if (lr_log2 < 0 || lr_log2 > 60) return IQ_ERR_INVALID_ARG;
+    if (n == 0) return IQ_OK;
+    int sh = (x2 ? k_u - 2 : k_u - 1) - lr_log2;
+    k_update<<<grid_for(n), kThreads, 0, (cudaStream_t)stream>>>(master, wq, g, s_g, n, sh, k_u,
+                                                                  k_w);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_relu_bwd(const int8_t* e_a, const int8_t* a, int64_t n, int8_t* e,
+                                 iq_stream stream) {
+    if (!e_a || !a || !e || n < 0) return IQ_ERR_INVALID_ARG;
+    if (n == 0) return IQ_OK;
+    k_relu_bwd<<<grid_for(n / 16 + 1), kThreads, 0, (cudaStream_t)stream>>>(e_a, a, n, e);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}

@@ -1,0 +1,269 @@
+"""Thin Python binding of the iq C ABI (``include/iq.h``).
+
+Argument marshalling only: every step of the computation runs in the CUDA
+kernels of ``libiq.so``.  Tensors are torch CUDA tensors used as plain device
+memory; the stream defaults to torch's current stream.  There is no fallback:
+if the library cannot be loaded the import-time ``load()`` raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import torch
+
+from . import build as _build
+
+IQ_OK, IQ_ERR_INVALID_ARG, IQ_ERR_UNSUPPORTED, IQ_ERR_WORKSPACE = 0, 1, 2, 3
+IQ_ERR_OVERFLOW_RISK, IQ_ERR_TIMEOUT, IQ_ERR_CUDA = 4, 5, 6
+IQ_I8, IQ_I16, IQ_I32, IQ_I64, IQ_F32, IQ_U8 = 1, 2, 3, 4, 5, 6
+IQ_MODE_UQ, IQ_MODE_UQ2, IQ_MODE_SQ, IQ_MODE_SQ_RELU, IQ_MODE_RQ_GQ1, IQ_MODE_RQ_GQ2 = range(6)
+IQ_BN_S_XHAT, IQ_BN_M_XHAT, IQ_BN_M_Y, IQ_BN_S_ACC, IQ_BN_S_A, IQ_BN_SCALES = 0, 1, 2, 3, 4, 8
+
+EXPORTS = [
+    "iq_status_str", "iq_version", "iq_conv_out_size", "iq_quantize_workspace_size",
+    "iq_conv_fwd_workspace_size", "iq_conv_dgrad_workspace_size", "iq_conv_wgrad_workspace_size",
+    "iq_bn_int_workspace_size", "iq_quantize", "iq_quantize_image_u8", "iq_requantize",
+    "iq_weight_requant", "iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad", "iq_bn_int_fwd",
+    "iq_bn_int_bwd", "iq_relu_bwd", "iq_update",
+]
+
+
+class IqError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn}: {status_str(code)} ({code})")
+        self.code = code
+
+
+class ConvDesc(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in
+                ("n", "h", "w", "c", "k", "r", "s", "stride_h", "stride_w", "pad_h", "pad_w",
+                 "dil_h", "dil_w", "groups")]
+
+
+class BnBits(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in ("k_mu", "k_sigma", "k_xhat", "k_gamma", "k_beta", "k_a")]
+
+
+_P = C.c_void_p
+_I = C.c_int
+_I32 = C.c_int32
+_I64 = C.c_int64
+_U64 = C.c_uint64
+_SZ = C.c_size_t
+_L = None
+
+
+def load(path: str | None = None):
+    """Load libiq.so (building it in-tree if needed).  Raises if unavailable."""
+    global _L
+    if _L is not None:
+        return _L
+    if path is None:
+        path = _build.LIB if os.path.exists(_build.LIB) else _build.build()
+    L = C.CDLL(path)
+    L.iq_status_str.restype = C.c_char_p
+    L.iq_status_str.argtypes = [_I]
+    L.iq_version.restype = _I
+    L.iq_conv_out_size.argtypes = [C.POINTER(ConvDesc), C.POINTER(_I32), C.POINTER(_I32)]
+    L.iq_quantize_workspace_size.argtypes = [_I64, C.POINTER(_SZ)]
+    L.iq_conv_fwd_workspace_size.argtypes = [C.POINTER(ConvDesc), _I, C.POINTER(_SZ)]
+    L.iq_conv_dgrad_workspace_size.argtypes = [C.POINTER(ConvDesc), C.POINTER(_SZ)]
+    L.iq_conv_wgrad_workspace_size.argtypes = [C.POINTER(ConvDesc), C.POINTER(_SZ)]
+    L.iq_bn_int_workspace_size.argtypes = [_I64, _I32, C.POINTER(_SZ)]
+    L.iq_quantize.argtypes = [_P, _I64, _I, _I, _I, _P, _P, _P, _SZ, _P]
+    L.iq_quantize_image_u8.argtypes = [_P, _I32, _I32, _I32, _I32, _I, _I32, _P, _P, _P, _SZ, _P]
+    L.iq_requantize.argtypes = [_P, _I, _I64, _P, _I, _I, _U64, _U64, _U64, _U64, _P, _I, _P, _P,
+                                _SZ, _P]
+    L.iq_weight_requant.argtypes = [_P, _P, _I64, _I, _I, _P]
+    L.iq_conv_fwd.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, C.POINTER(BnBits), _I, _I,
+                              _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
+    L.iq_conv_dgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
+    L.iq_conv_wgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _I, _U64, _U64, _U64, _P, _P,
+                                _P, _P, _SZ, _P]
+    L.iq_bn_int_fwd.argtypes = [_P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _P, _P, _P, _P, _P,
+                                _P, _P, _SZ, _P]
+    L.iq_bn_int_bwd.argtypes = [_P, _P, _P, _P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _I, _P,
+                                _P, _P, _P, _P, _SZ, _P]
+    L.iq_relu_bwd.argtypes = [_P, _P, _I64, _P, _P]
+    L.iq_update.argtypes = [_P, _P, _P, _P, _I64, _I, _I, _I, _I, _P]
+    for f in EXPORTS:
+        if f not in ("iq_status_str", "iq_version"):
+            getattr(L, f).restype = _I
+    _L = L
+    return L
+
+
+def status_str(code: int) -> str:
+    return load().iq_status_str(code).decode()
+
+
+def _p(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(fn: str, rc: int):
+    if rc != IQ_OK:
+        raise IqError(fn, rc)
+
+
+def _ws(nbytes: int, device) -> torch.Tensor:
+    return torch.empty(max(int(nbytes), 1), dtype=torch.uint8, device=device)
+
+
+def conv_desc(n, h, w, c, k, r, s, stride=1, pad=0, dil=1, groups=1) -> ConvDesc:
+    return ConvDesc(n, h, w, c, k, r, s, stride, stride, pad, pad, dil, dil, groups)
+
+
+def bn_bits(k_mu=16, k_sigma=16, k_xhat=16, k_gamma=8, k_beta=8, k_a=8) -> BnBits:
+    return BnBits(k_mu, k_sigma, k_xhat, k_gamma, k_beta, k_a)
+
+
+# ---------------------------------------------------------------- queries
+
+def iq_conv_out_size(d: ConvDesc):
+    p, q = _I32(), _I32()
+    _check("iq_conv_out_size", load().iq_conv_out_size(C.byref(d), C.byref(p), C.byref(q)))
+    return p.value, q.value
+
+
+def _size(fn, *args) -> int:
+    b = _SZ()
+    _check(fn, getattr(load(), fn)(*args, C.byref(b)))
+    return b.value
+
+
+def iq_quantize_workspace_size(n: int) -> int:
+    return _size("iq_quantize_workspace_size", n)
+
+
+def iq_conv_fwd_workspace_size(d: ConvDesc, with_bn: bool = False) -> int:
+    return _size("iq_conv_fwd_workspace_size", C.byref(d), int(with_bn))
+
+
+def iq_conv_dgrad_workspace_size(d: ConvDesc) -> int:
+    return _size("iq_conv_dgrad_workspace_size", C.byref(d))
+
+
+def iq_conv_wgrad_workspace_size(d: ConvDesc) -> int:
+    return _size("iq_conv_wgrad_workspace_size", C.byref(d))
+
+
+def iq_bn_int_workspace_size(m: int, c: int) -> int:
+    return _size("iq_bn_int_workspace_size", m, c)
+
+
+# ---------------------------------------------------------------- operations
+
+def iq_quantize(x, k, mode, codes, scale, ws=None, stream=None):
+    out_dtype = {torch.int8: IQ_I8, torch.int16: IQ_I16, torch.int32: IQ_I32}[codes.dtype]
+    if ws is None:
+        ws = _ws(iq_quantize_workspace_size(x.numel()), x.device)
+    _check("iq_quantize", load().iq_quantize(_p(x), x.numel(), k, mode, out_dtype, _p(codes),
+                                             _p(scale), _p(ws), ws.numel(), _stream(stream)))
+
+
+def iq_quantize_image_u8(img, nchw, c_out, codes, scale, ws=None, stream=None):
+    if nchw:
+        n, c, h, w = img.shape
+    else:
+        n, h, w, c = img.shape
+    if ws is None:
+        ws = _ws(iq_quantize_workspace_size(img.numel()), img.device)
+    _check("iq_quantize_image_u8",
+           load().iq_quantize_image_u8(_p(img), n, h, w, c, int(nchw), c_out, _p(codes),
+                                       _p(scale), _p(ws), ws.numel(), _stream(stream)))
+
+
+def iq_requantize(q, s_in, k, mode, codes, s_out, seed=0, layer=0, step=0, tag=0, ws=None,
+                  stream=None):
+    in_dtype = {torch.int32: IQ_I32, torch.int64: IQ_I64}[q.dtype]
+    out_dtype = {torch.int8: IQ_I8, torch.int16: IQ_I16, torch.int32: IQ_I32}[codes.dtype]
+    if ws is None:
+        ws = _ws(iq_quantize_workspace_size(q.numel()), q.device)
+    _check("iq_requantize",
+           load().iq_requantize(_p(q), in_dtype, q.numel(), _p(s_in), k, mode, seed, layer, step,
+                                tag, _p(codes), out_dtype, _p(s_out), _p(ws), ws.numel(),
+                                _stream(stream)))
+
+
+def iq_weight_requant(master, wq, k_u=24, k_w=8, stream=None):
+    _check("iq_weight_requant", load().iq_weight_requant(_p(master), _p(wq), master.numel(), k_u,
+                                                         k_w, _stream(stream)))
+
+
+def iq_conv_fwd(d: ConvDesc, x, s_x, w, a, s_a, gamma=None, beta=None, bits=None, use_bn=False,
+                relu=True, xhat=None, bn_codes=None, bn_scales=None, acc_out=None, ws=None,
+                stream=None):
+    if ws is None:
+        ws = _ws(iq_conv_fwd_workspace_size(d, use_bn), x.device)
+    _check("iq_conv_fwd",
+           load().iq_conv_fwd(C.byref(d), _p(x), _p(s_x), _p(w), _p(gamma), _p(beta),
+                              C.byref(bits) if bits is not None else None, int(use_bn),
+                              int(relu), _p(a), _p(s_a), _p(xhat), _p(bn_codes), _p(bn_scales),
+                              _p(acc_out), _p(ws), ws.numel(), _stream(stream)))
+
+
+def iq_conv_dgrad(d: ConvDesc, e, s_e, w, dx, s_dx, acc_out=None, ws=None, stream=None):
+    if ws is None:
+        ws = _ws(iq_conv_dgrad_workspace_size(d), e.device)
+    _check("iq_conv_dgrad",
+           load().iq_conv_dgrad(C.byref(d), _p(e), _p(s_e), _p(w), _p(dx), _p(s_dx), _p(acc_out),
+                                _p(ws), ws.numel(), _stream(stream)))
+
+
+def iq_conv_wgrad(d: ConvDesc, e, s_e, x, s_x, g, s_g, gq_mode=1, seed=0, layer=0, step=0,
+                  g_acc_out=None, ws=None, stream=None):
+    if ws is None:
+        ws = _ws(iq_conv_wgrad_workspace_size(d), e.device)
+    _check("iq_conv_wgrad",
+           load().iq_conv_wgrad(C.byref(d), _p(e), _p(s_e), _p(x), _p(s_x), gq_mode, seed, layer,
+                                step, _p(g), _p(s_g), _p(g_acc_out), _p(ws), ws.numel(),
+                                _stream(stream)))
+
+
+def iq_bn_int_fwd(acc, s_acc, gamma, beta, a, s_a, xhat=None, bn_codes=None, bn_scales=None,
+                  bn_fixed=None, bits=None, ws=None, stream=None):
+    c = acc.shape[-1]
+    m = acc.numel() // c
+    if ws is None:
+        ws = _ws(iq_bn_int_workspace_size(m, c), acc.device)
+    _check("iq_bn_int_fwd",
+           load().iq_bn_int_fwd(_p(acc), m, c, _p(s_acc), _p(gamma), _p(beta),
+                                C.byref(bits) if bits is not None else None, _p(xhat), _p(a),
+                                _p(s_a), _p(bn_codes), _p(bn_scales), _p(bn_fixed), _p(ws),
+                                ws.numel(), _stream(stream)))
+
+
+def iq_bn_int_bwd(e_a, s_e, a, xhat, gamma, bn_codes, bn_scales, e, s_e_out, dgamma=None,
+                  dbeta=None, k_e2=16, bits=None, ws=None, stream=None):
+    c = e_a.shape[-1]
+    m = e_a.numel() // c
+    if ws is None:
+        ws = _ws(iq_bn_int_workspace_size(m, c), e_a.device)
+    _check("iq_bn_int_bwd",
+           load().iq_bn_int_bwd(_p(e_a), _p(s_e), _p(a), _p(xhat), m, c, _p(gamma), _p(bn_codes),
+                                _p(bn_scales), C.byref(bits) if bits is not None else None, k_e2,
+                                _p(e), _p(s_e_out), _p(dgamma), _p(dbeta), _p(ws), ws.numel(),
+                                _stream(stream)))
+
+
+def iq_relu_bwd(e_a, a, e, stream=None):
+    _check("iq_relu_bwd", load().iq_relu_bwd(_p(e_a), _p(a), e_a.numel(), _p(e), _stream(stream)))
+
+
+def iq_update(master, wq, g, s_g, lr_log2, k_u=24, k_w=8, x2=False, stream=None):
+    _check("iq_update", load().iq_update(_p(master), _p(wq), _p(g), _p(s_g), master.numel(),
+                                         lr_log2, k_u, k_w, int(x2), _stream(stream)))

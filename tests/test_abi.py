@@ -1,0 +1,86 @@
+"""CPU-side checks of the C ABI: the library builds and loads, exports every entry point
+that include/iq.h declares, and rejects bad arguments before launching anything."""
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2011_14504_gb300 import build as B
+from paper_2011_14504_gb300 import iq
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_entry_points():
+    src = open(os.path.join(ROOT, "include", "iq.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:iq_status|const char\*|int)\s+(iq_\w+)\s*\(", src,
+                                 re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return iq.load()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    decl = declared_entry_points()
+    assert len(decl) >= 19
+    out = subprocess.run(["nm", "-D", "--defined-only", B.LIB], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\bT (iq_\w+)", out))
+    missing = [d for d in decl if d not in exported]
+    assert not missing, missing
+    assert sorted(decl) == sorted(iq.EXPORTS)
+
+
+def test_status_strings_and_version(lib):
+    assert iq.status_str(0) == "ok"
+    assert "workspace" in iq.status_str(3)
+    assert lib.iq_version() >= 1
+
+
+def test_conv_out_size_and_workspace_queries(lib):
+    d = iq.conv_desc(1, 32, 32, 64, 64, 3, 3, 1, 1)
+    assert iq.iq_conv_out_size(d) == (32, 32)
+    d2 = iq.conv_desc(2, 65, 65, 256, 256, 3, 3, 1, 24, 24)    # ASPP rate 24 on 65x65
+    assert iq.iq_conv_out_size(d2) == (65, 65)
+    d3 = iq.conv_desc(16, 513, 513, 4, 64, 7, 7, 2, 3)          # stem
+    assert iq.iq_conv_out_size(d3) == (257, 257)
+    assert iq.iq_conv_fwd_workspace_size(d) >= 32 * 32 * 64 * 4
+    assert iq.iq_conv_dgrad_workspace_size(d) >= 32 * 32 * 64 * 4
+    assert iq.iq_conv_wgrad_workspace_size(d) >= 64 * 9 * 64 * 8
+    assert iq.iq_bn_int_workspace_size(1024, 64) > 0
+
+
+def test_invalid_arguments_rejected_before_launch(lib):
+    bad = iq.conv_desc(1, 8, 8, 6, 4, 3, 3, 1, 1, 1, 4)        # C not divisible by groups
+    with pytest.raises(iq.IqError) as e:
+        iq.iq_conv_out_size(bad)
+    assert e.value.code == iq.IQ_ERR_INVALID_ARG
+    d = iq.conv_desc(1, 8, 8, 8, 8, 3, 3, 1, 1)
+    rc = lib.iq_conv_fwd(C.byref(d), None, None, None, None, None, None, 0, 1, None, None, None,
+                         None, None, None, None, 0, None)
+    assert rc == iq.IQ_ERR_INVALID_ARG
+    # a shape beyond the int32 accumulation bound: 1024*12*12*127^2 >= 2^31
+    big = iq.conv_desc(1, 12, 12, 1024, 8, 12, 12)
+    rc = lib.iq_conv_fwd(C.byref(big), 1, 1, 1, None, None, None, 0, 1, 1, 1, None, None, None,
+                         None, None, 0, None)
+    assert rc == iq.IQ_ERR_OVERFLOW_RISK
+    # workspace too small
+    rc = lib.iq_conv_fwd(C.byref(d), 1, 1, 1, None, None, None, 0, 1, 1, 1, None, None, None,
+                         None, None, 16, None)
+    assert rc == iq.IQ_ERR_WORKSPACE
+    # bad bit width / dtype combination
+    rc = lib.iq_quantize(1, 10, 16, iq.IQ_MODE_UQ, iq.IQ_I8, 1, 1, 1, 4096, None)
+    assert rc == iq.IQ_ERR_INVALID_ARG
+    rc = lib.iq_requantize(1, iq.IQ_I32, 10, 1, 8, 99, 0, 0, 0, 0, 1, iq.IQ_I8, 1, 1, 4096, None)
+    assert rc == iq.IQ_ERR_INVALID_ARG
+    # BN needs C % 4 == 0
+    rc = lib.iq_bn_int_fwd(16, 10, 6, 1, 1, 1, None, None, 16, 1, None, None, None, 16, 1 << 20,
+                           None)
+    assert rc == iq.IQ_ERR_UNSUPPORTED
+    rc = lib.iq_update(1, 1, 1, 1, 10, -1, 24, 8, 0, None)
+    assert rc == iq.IQ_ERR_INVALID_ARG

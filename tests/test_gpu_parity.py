@@ -1,0 +1,300 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle, element by element.
+
+Integer outputs must be bit-exact; fp64 scale outputs must be equal (0 ULP): both
+sides evaluate the same fixed-order fp64 steps.  Inputs come from the seeded
+generators only.  Sizes span several tiles and a ragged tail.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2011_14504_gb300 import iq
+from paper_2011_14504_gb300 import synthetic as S
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+
+def dev(a, dtype=None):
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    if dtype is not None:
+        t = t.to(dtype)
+    return t.to(DEV)
+
+
+def dscal(v=0.0):
+    return torch.tensor([v], dtype=torch.float64, device=DEV)
+
+
+def host(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+# ----------------------------------------------------------------- quantizers
+
+@pytest.mark.parametrize("k", [8, 16, 24])
+@pytest.mark.parametrize("mode", [iq.IQ_MODE_UQ, iq.IQ_MODE_UQ2])
+def test_uq_bitpattern_sweep(k, mode):
+    # a strided sweep over all 2^32 fp32 bit patterns (finite ones), plus near-ties
+    bits = np.arange(0, 2 ** 32, 9973, dtype=np.uint64).astype(np.uint32)
+    x = bits.view(np.float32)
+    x = x[np.isfinite(x)]
+    d = 2.0 ** (1 - k)
+    j = np.arange(-(2 ** min(k - 1, 12)), 2 ** min(k - 1, 12))
+    t = ((j + 0.5) * d * (2 if mode == iq.IQ_MODE_UQ2 else 1)).astype(np.float32)
+    x = np.concatenate([x, t, np.nextafter(t, np.float32(1e30)), np.nextafter(t, np.float32(-1e30))])
+    out = torch.empty(x.size, dtype=torch.int32, device=DEV)
+    s = dscal()
+    iq.iq_quantize(dev(x), k, mode, out, s)
+    want = O.uq(x, k) if mode == iq.IQ_MODE_UQ else O.uq2(x, k)
+    assert np.array_equal(host(out), want)
+    assert host(s)[0] == 2.0 ** ((1 if mode == iq.IQ_MODE_UQ else 2) - k)
+
+
+@pytest.mark.parametrize("k,dtype", [(8, torch.int8), (16, torch.int16)])
+def test_sq_float(k, dtype):
+    g = S.rng(1)
+    x = np.concatenate([S.float_uniform(g, 100003, -3, 3), np.float32([3.5, -0.0])])
+    out = torch.empty(x.size, dtype=dtype, device=DEV)
+    s = dscal()
+    iq.iq_quantize(dev(x), k, iq.IQ_MODE_SQ, out, s)
+    want, ws = O.sq_float(x, k)
+    assert np.array_equal(host(out).astype(np.int32), want)
+    assert host(s)[0] == ws
+
+
+def test_sq_float_all_zero_and_empty():
+    x = np.zeros(1000, np.float32)
+    out = torch.empty(1000, dtype=torch.int8, device=DEV)
+    s = dscal()
+    iq.iq_quantize(dev(x), 8, iq.IQ_MODE_SQ, out, s)
+    assert (host(out) == 0).all() and host(s)[0] == 2.0 ** -7
+    e = torch.empty(0, dtype=torch.float32, device=DEV)
+    iq.iq_quantize(e, 8, iq.IQ_MODE_SQ, torch.empty(0, dtype=torch.int8, device=DEV), s)
+    assert host(s)[0] == 2.0 ** -7
+
+
+def test_image_input():
+    g = S.rng(2)
+    img = S.images_u8(g, 2, 37, 41)
+    codes = torch.empty((2, 37, 41, 4), dtype=torch.int8, device=DEV)
+    s = dscal()
+    iq.iq_quantize_image_u8(dev(img), False, 4, codes, s)
+    want, ws = O.quantize_image_u8(img, 4)
+    assert np.array_equal(host(codes), want) and host(s)[0] == ws
+    # NCHW input gives the same codes
+    codes2 = torch.empty_like(codes)
+    iq.iq_quantize_image_u8(dev(np.ascontiguousarray(img.transpose(0, 3, 1, 2))), True, 4, codes2, s)
+    assert np.array_equal(host(codes2), want)
+
+
+@pytest.mark.parametrize("relu", [False, True])
+def test_requantize_sq_int32(relu):
+    g = S.rng(3)
+    q = g.integers(-404644352, 404644353, size=77777).astype(np.int32)
+    out = torch.empty(q.size, dtype=torch.int8, device=DEV)
+    so = dscal()
+    iq.iq_requantize(dev(q), dscal(2.0 ** -20), 8, iq.IQ_MODE_SQ_RELU if relu else iq.IQ_MODE_SQ,
+                     out, so)
+    want, ws = O.sq_int(q, 2.0 ** -20, 8, relu)
+    assert np.array_equal(host(out).astype(np.int32), want)
+    assert host(so)[0] == ws
+
+
+@pytest.mark.parametrize("mode,gq", [(iq.IQ_MODE_RQ_GQ1, 1), (iq.IQ_MODE_RQ_GQ2, 2)])
+def test_requantize_rq_int64(mode, gq):
+    g = S.rng(4)
+    q = (g.standard_normal(50001) * 3e9).astype(np.int64)
+    for step in (0, 7):
+        out = torch.empty(q.size, dtype=torch.int8, device=DEV)
+        so = dscal()
+        iq.iq_requantize(dev(q), dscal(1.5e-9), 8, mode, out, so, seed=1234, layer=5, step=step,
+                         tag=2)
+        want, ws = O.rq_int(q, 1.5e-9, 8, gq, 1234, 5, step, 2)
+        assert np.array_equal(host(out).astype(np.int32), want)
+        assert host(so)[0] == ws
+
+
+def test_weight_requant_and_update():
+    g = S.rng(5)
+    m = S.master_weights(g, 100001, 576)
+    wq = torch.empty(m.size, dtype=torch.int8, device=DEV)
+    md = dev(m)
+    iq.iq_weight_requant(md, wq)
+    assert np.array_equal(host(wq).astype(np.int32), O.requant_master(m))
+    gc = S.int8_uniform(g, m.size)
+    for s_g, e, x2 in ((2.0 ** -7, 10, False), (3.3e-5, 4, False), (1.7e-3, 6, True)):
+        md = dev(m)
+        iq.iq_update(md, wq, dev(gc), dscal(s_g), e, x2=x2)
+        wm, wwq = O.update(m, gc.astype(np.int32), s_g, e, x2=x2)
+        assert np.array_equal(host(md), wm)
+        assert np.array_equal(host(wq).astype(np.int32), wwq)
+
+
+def test_relu_bwd():
+    g = S.rng(6)
+    ea = S.int8_uniform(g, 100003)
+    a = S.int8_uniform(g, 100003, -3, 127)
+    e = torch.empty(ea.size, dtype=torch.int8, device=DEV)
+    iq.iq_relu_bwd(dev(ea), dev(a), e)
+    assert np.array_equal(host(e), O.relu_bwd(ea, a))
+
+
+# ----------------------------------------------------------------- convolution
+
+CONV_CASES = [
+    # n, h, w, c, k, r, s, stride, pad, dil, groups
+    (1, 32, 32, 64, 64, 3, 3, 1, 1, 1, 1),      # the single-layer workload
+    (2, 13, 11, 16, 24, 3, 3, 1, 1, 1, 1),      # ragged M and N tiles
+    (1, 17, 19, 32, 40, 3, 3, 2, 1, 1, 1),      # stride 2
+    (2, 15, 15, 16, 16, 3, 3, 1, 4, 4, 1),      # atrous
+    (1, 9, 9, 24, 12, 1, 1, 1, 0, 1, 1),        # 1x1
+    (1, 10, 12, 12, 8, 3, 3, 1, 1, 1, 4),       # grouped, C/G = 3 (byte path)
+    (2, 20, 20, 4, 16, 7, 7, 2, 3, 1, 1),       # stem-like, C padded to 4
+    (1, 7, 7, 256, 32, 7, 7, 1, 3, 1, 1),       # fc6-like, CRS = 12544
+    (1, 65, 3, 8, 8, 3, 3, 1, 12, 12, 1),       # ASPP-like rate beyond the map
+]
+
+
+def _conv_case(ci, seed):
+    n, h, w, c, k, r, s, st, pd, dl, gr = CONV_CASES[ci]
+    cv = O.Conv(n, h, w, c, k, r, s, st, pd, dl, gr)
+    d = iq.conv_desc(n, h, w, c, k, r, s, st, pd, dl, gr)
+    g = S.rng(seed)
+    p, q = cv.pq
+    x = S.int8_uniform(g, (n, h, w, c))
+    wm = S.master_weights(g, (k, r, s, c // gr), c // gr * r * s)
+    wq = O.requant_master(wm).astype(np.int8)
+    e = S.int8_uniform(g, (n, p, q, k))
+    return cv, d, x, wq, e
+
+
+@pytest.mark.parametrize("ci", range(len(CONV_CASES)))
+@pytest.mark.parametrize("relu", [True, False])
+def test_conv_fwd_no_bn(ci, relu):
+    cv, d, x, w, _ = _conv_case(ci, 10 + ci)
+    p, q = cv.pq
+    a = torch.empty((cv.n, p, q, cv.k), dtype=torch.int8, device=DEV)
+    acc = torch.empty((cv.n, p, q, cv.k), dtype=torch.int32, device=DEV)
+    s_a = dscal()
+    s_x = 2.0 ** -7 * 0.37
+    iq.iq_conv_fwd(d, dev(x), dscal(s_x), dev(w), a, s_a, relu=relu, acc_out=acc)
+    want_acc = O.conv_fwd(cv, x, w)
+    assert np.array_equal(host(acc), want_acc)
+    want_a, want_s = O.sq_int(want_acc, s_x * 2.0 ** -7, 8, relu)
+    assert np.array_equal(host(a).astype(np.int32), want_a)
+    assert host(s_a)[0] == want_s
+
+
+@pytest.mark.parametrize("ci", range(len(CONV_CASES)))
+def test_conv_dgrad(ci):
+    cv, d, x, w, e = _conv_case(ci, 30 + ci)
+    dx = torch.empty((cv.n, cv.h, cv.w, cv.c), dtype=torch.int8, device=DEV)
+    acc = torch.empty((cv.n, cv.h, cv.w, cv.c), dtype=torch.int32, device=DEV)
+    s_dx = dscal()
+    s_e = 3.1e-6
+    iq.iq_conv_dgrad(d, dev(e), dscal(s_e), dev(w), dx, s_dx, acc_out=acc)
+    want_acc = O.conv_dgrad(cv, e, w)
+    assert np.array_equal(host(acc), want_acc)
+    want, ws = O.sq_int(want_acc, s_e * 2.0 ** -7, 8)
+    assert np.array_equal(host(dx).astype(np.int32), want)
+    assert host(s_dx)[0] == ws
+
+
+@pytest.mark.parametrize("ci", range(len(CONV_CASES)))
+@pytest.mark.parametrize("gq", [1, 2])
+def test_conv_wgrad(ci, gq):
+    cv, d, x, w, e = _conv_case(ci, 50 + ci)
+    gco = torch.empty(w.shape, dtype=torch.int8, device=DEV)
+    gacc = torch.empty(w.shape, dtype=torch.int64, device=DEV)
+    s_g = dscal()
+    s_e, s_x = 3.1e-6, 0.02
+    iq.iq_conv_wgrad(d, dev(e), dscal(s_e), dev(x), dscal(s_x), gco, s_g, gq_mode=gq, seed=99,
+                     layer=ci, step=3, g_acc_out=gacc)
+    want_acc = O.conv_wgrad(cv, e, x)
+    assert np.array_equal(host(gacc), want_acc)
+    want, ws = O.rq_int(want_acc, s_e * s_x, 8, gq, 99, ci, 3, 0)
+    assert np.array_equal(host(gco).astype(np.int32), want)
+    assert host(s_g)[0] == ws
+
+
+# ----------------------------------------------------------------- L1BN
+
+def _bn_ref(acc, s_acc, gam, bet, k_e2=16):
+    return O.bn_fwd(acc, s_acc, gam, bet)
+
+
+@pytest.mark.parametrize("m,C,spread,offset", [(1024, 64, 3000, 500), (777, 32, 20, 40000),
+                                               (300, 1032, 1e6, 1e6), (64, 2048, 5e5, 0)])
+def test_bn_int_fwd(m, C, spread, offset):
+    g = S.rng(int(m + C))
+    acc = (g.standard_normal((m, C)) * spread + g.integers(-offset, offset + 1, C)).astype(np.int32)
+    gam, bet = S.bn_gamma_beta_codes(g, C)
+    s_acc = 2.0 ** -14 * 1.7
+    X = torch.empty((m, C), dtype=torch.int16, device=DEV)
+    A = torch.empty((m, C), dtype=torch.int8, device=DEV)
+    codes = torch.empty(2 * C, dtype=torch.int32, device=DEV)
+    scal = torch.empty(iq.IQ_BN_SCALES, dtype=torch.float64, device=DEV)
+    fixed = torch.empty(4 * C + 2, dtype=torch.int64, device=DEV)
+    s_a = dscal()
+    iq.iq_bn_int_fwd(dev(acc), dscal(s_acc), dev(gam), dev(bet), A, s_a, xhat=X, bn_codes=codes,
+                     bn_scales=scal, bn_fixed=fixed)
+    r = O.bn_fwd(acc, s_acc, gam, bet)
+    fx = host(fixed)
+    assert np.array_equal(host(codes), np.concatenate([r.c_mu, r.c_sigma]))
+    assert np.array_equal(fx[:C], r.F) and np.array_equal(fx[C:2 * C], r.B)
+    assert np.array_equal(fx[2 * C:3 * C], r.G) and np.array_equal(fx[3 * C:4 * C], r.H)
+    assert fx[4 * C] == r.p_x and fx[4 * C + 1] == r.p_a
+    sc = host(scal)
+    assert sc[iq.IQ_BN_S_XHAT] == r.s_xhat and sc[iq.IQ_BN_M_XHAT] == r.m_xhat
+    assert sc[iq.IQ_BN_M_Y] == r.m_y and sc[iq.IQ_BN_S_A] == r.s_a and host(s_a)[0] == r.s_a
+    assert np.array_equal(host(X), r.X)
+    assert np.array_equal(host(A), r.A)
+
+
+def test_conv_fwd_bn_single_layer_workload():
+    # N=1, C=K=64, 32x32, 3x3 s1 p1, L1BN + ReLU + Q_A (the single-layer case)
+    cv, d, x, w, _ = _conv_case(0, 70)
+    g = S.rng(71)
+    gam, bet = S.bn_gamma_beta_codes(g, 64)
+    s_x = 2.0 ** -7
+    A = torch.empty((1, 32, 32, 64), dtype=torch.int8, device=DEV)
+    X = torch.empty((1, 32, 32, 64), dtype=torch.int16, device=DEV)
+    codes = torch.empty(128, dtype=torch.int32, device=DEV)
+    scal = torch.empty(iq.IQ_BN_SCALES, dtype=torch.float64, device=DEV)
+    s_a = dscal()
+    iq.iq_conv_fwd(d, dev(x), dscal(s_x), dev(w), A, s_a, gamma=dev(gam), beta=dev(bet),
+                   bits=iq.bn_bits(), use_bn=True, xhat=X, bn_codes=codes, bn_scales=scal)
+    acc = O.conv_fwd(cv, x, w)
+    r = O.bn_fwd(acc.reshape(-1, 64), s_x * 2.0 ** -7, gam, bet)
+    assert np.array_equal(host(X).reshape(-1, 64), r.X)
+    assert np.array_equal(host(A).reshape(-1, 64), r.A)
+    assert host(s_a)[0] == r.s_a
+
+
+@pytest.mark.parametrize("k_e2", [16, 8])
+@pytest.mark.parametrize("m,C", [(1024, 64), (333, 1028), (200, 2048)])
+def test_bn_int_bwd(m, C, k_e2):
+    g = S.rng(m * 7 + C + k_e2)
+    acc = (g.standard_normal((m, C)) * 4000 + g.integers(-300, 301, C)).astype(np.int32)
+    gam, bet = S.bn_gamma_beta_codes(g, C)
+    s_acc = 2.0 ** -14
+    r = O.bn_fwd(acc, s_acc, gam, bet)
+    ea = S.int8_uniform(g, (m, C))
+    s_e = 2.0 ** -21 * 1.3
+    E, s_E, dg, db = O.bn_bwd(ea, s_e, r.A, r.X, r.s_xhat, gam, r.c_sigma, k_e2=k_e2)
+    codes = dev(np.concatenate([r.c_mu, r.c_sigma]))
+    scal = np.zeros(iq.IQ_BN_SCALES)
+    scal[iq.IQ_BN_S_XHAT] = r.s_xhat
+    e_out = torch.empty((m, C), dtype=torch.int8, device=DEV)
+    s_out = dscal()
+    dgam = torch.empty(C, dtype=torch.int64, device=DEV)
+    dbet = torch.empty(C, dtype=torch.int64, device=DEV)
+    iq.iq_bn_int_bwd(dev(ea), dscal(s_e), dev(r.A), dev(r.X), dev(gam), codes, dev(scal), e_out,
+                     s_out, dgamma=dgam, dbeta=dbet, k_e2=k_e2)
+    assert np.array_equal(host(dgam), dg) and np.array_equal(host(dbet), db)
+    assert np.array_equal(host(e_out), E)
+    assert host(s_out)[0] == s_E

@@ -511,3 +511,16 @@ def test_relu_bwd_mask():
     eA = np.array([5, -3, 7, 0, -9], np.int8)
     A = np.array([1, 0, 127, 3, 0], np.int8)
     assert O.relu_bwd(eA, A).tolist() == [5, 0, 7, 0, 0]
+
+
+def test_image_input_quantization_exact():
+    g = S.rng(60)
+    img = S.images_u8(g, 2, 5, 7)
+    img[0, 0, 0, 0] = 200
+    img = np.minimum(img, 200).astype(np.uint8)
+    codes, s = O.quantize_image_u8(img, 4)
+    P = int(img.max())
+    want = [clip(rhu_exact(Fr(int(p), 255) / Fr(P, 255) * 128), 8) for p in img.reshape(-1)]
+    assert codes[..., :3].reshape(-1).tolist() == want
+    assert (codes[..., 3] == 0).all()
+    assert s == P / 255 * 2 ** -7
