@@ -355,6 +355,7 @@ struct FwdWs {
     BnStats st;
     void* rq;
     double* s_acc;
+    void* tc;
 };
 
 static size_t fwd_ws_layout(const iq_conv_desc* d, int with_acc, void* base, size_t cap,
@@ -366,6 +367,7 @@ static size_t fwd_ws_layout(const iq_conv_desc* d, int with_acc, void* base, siz
     w.st = bn_stats_carve(cur, cp.K);
     w.rq = cur.take<char>(requant_ws_bytes());
     w.s_acc = cur.take<double>(1);
+    w.tc = cur.take<char>(conv_fwd_tc_ws_bytes(d));
     if (out) *out = w;
     return cur.off + 256;
 }
@@ -446,7 +448,7 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     k_scale_mul_pow2<<<1, 1, 0, st>>>(s_x, -7, L.s_acc);  // s_acc = s_x * 2^-7 (W_q step)
     IQ_LAUNCH_CHECK();
     bool done = false;
-    r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, st, &done);
+    r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done);
     if (r != IQ_OK) return r;
     if (!done) {
         dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);

@@ -8,7 +8,11 @@ namespace iq {
 // Forward convolution on the 5th-generation tensor cores when the shape is
 // supported; sets *done = false (and enqueues nothing) otherwise.  Writes the int32
 // accumulators and the per-channel sum / max / min like the CUDA-core path.
+// `ws` must hold conv_fwd_tc_ws_bytes(d) bytes (the fp16 copy of the weights).
+size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d);
+bool conv_fwd_tc_supported(const iq_conv_desc* d);
 iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, int32_t* acc,
-                      unsigned long long* s1, int* hi, int* lo, cudaStream_t st, bool* done);
+                      unsigned long long* s1, int* hi, int* lo, void* ws, cudaStream_t st,
+                      bool* done);
 
 }  // namespace iq

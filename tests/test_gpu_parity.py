@@ -298,3 +298,50 @@ def test_bn_int_bwd(m, C, k_e2):
     assert np.array_equal(host(dgam), dg) and np.array_equal(host(dbet), db)
     assert np.array_equal(host(e_out), E)
     assert host(s_out)[0] == s_E
+
+
+# ----------------------------------------------------------------- tensor-core path specifics
+
+TC_CASES = [
+    # n, h, w, c, k, r, s, stride, pad, dil: shapes the tcgen05 kernel takes
+    (2, 16, 16, 512, 256, 3, 3, 1, 1, 1),   # 5 fp32 chunks, 2 N tiles, 4 M tiles
+    (1, 29, 31, 128, 136, 3, 3, 1, 2, 2),   # ragged M and N, dilation 2
+    (3, 9, 10, 64, 72, 1, 1, 1, 0, 1),      # 1x1, ragged
+    (1, 33, 33, 256, 64, 3, 3, 2, 1, 1),    # stride 2
+]
+
+
+@pytest.mark.parametrize("ci", range(len(TC_CASES)))
+def test_conv_fwd_tc_shapes(ci):
+    n, h, w, c, k, r, s, st, pd, dl = TC_CASES[ci]
+    cv = O.Conv(n, h, w, c, k, r, s, st, pd, dl)
+    d = iq.conv_desc(n, h, w, c, k, r, s, st, pd, dl)
+    g = S.rng(90 + ci)
+    x = S.int8_uniform(g, (n, h, w, c))
+    wq = O.requant_master(S.master_weights(g, (k, r, s, c), c * r * s)).astype(np.int8)
+    p, q = cv.pq
+    a = torch.empty((n, p, q, k), dtype=torch.int8, device=DEV)
+    acc = torch.empty((n, p, q, k), dtype=torch.int32, device=DEV)
+    s_a = dscal()
+    iq.iq_conv_fwd(d, dev(x), dscal(0.01), dev(wq), a, s_a, relu=True, acc_out=acc)
+    want = O.conv_fwd(cv, x, wq)
+    assert np.array_equal(host(acc), want)
+    wa, ws_ = O.sq_int(want, 0.01 * 2.0 ** -7, 8, True)
+    assert np.array_equal(host(a).astype(np.int32), wa) and host(s_a)[0] == ws_
+
+
+@pytest.mark.parametrize("sign", [1, -1])
+def test_conv_fwd_adversarial_full_scale(sign):
+    # all codes at +-127: every fp32 chunk holds 1024 * 127^2 = 16,516,096 < 2^24 and
+    # the int32 total is 4608 * 127^2 for interior pixels
+    n, h, w, c, k = 1, 6, 6, 512, 128
+    cv = O.Conv(n, h, w, c, k, 3, 3, 1, 1)
+    d = iq.conv_desc(n, h, w, c, k, 3, 3, 1, 1)
+    x = np.full((n, h, w, c), 127, np.int8)
+    wq = np.full((k, 3, 3, c), 127 * sign, np.int8)
+    a = torch.empty((n, h, w, k), dtype=torch.int8, device=DEV)
+    acc = torch.empty((n, h, w, k), dtype=torch.int32, device=DEV)
+    iq.iq_conv_fwd(d, dev(x), dscal(1.0), dev(wq), a, dscal(), relu=False, acc_out=acc)
+    got = host(acc)
+    assert np.array_equal(got, O.conv_fwd(cv, x, wq))
+    assert got[0, 2, 2, 0] == sign * 4608 * 16129
