@@ -90,6 +90,10 @@ enum {
 const char* iq_status_str(iq_status s);
 int iq_version(void);
 
+/* Number of kernels the library has enqueued in this process (host-side counter; the
+ * paper has no counterpart -- it lets a caller count device launches in a region). */
+unsigned long long iq_launch_count(void);
+
 /* Output size of a convolution (host-side, no device work). */
 iq_status iq_conv_out_size(const iq_conv_desc* d, int32_t* p, int32_t* q);
 
@@ -169,7 +173,8 @@ iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
  *   e    int8 [n][p][q][k] error codes at the conv output; s_e device double
  *   w    int8 KRSC forward weights (scale 2^-7)
  *   dx   out int8 NHWC [n][h][w][c]; s_dx out device double = (s_e 2^-7 M) 2^-7
- *   acc_out optional out int32 [n][h][w][c] */
+ *   acc_out optional out int32 [n][h][w][c]; must be NULL when (k/groups) r s 127^2 >= 2^31,
+ *           where the sums are accumulated in int64 (IQ_ERR_UNSUPPORTED otherwise) */
 iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
                         const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out, void* ws,
                         size_t ws_bytes, iq_stream stream);
@@ -232,6 +237,61 @@ iq_status iq_relu_bwd(const int8_t* e_a, const int8_t* a, int64_t n, int8_t* e,
  *   wq     out int8[n];  g int8[n] gradient codes with device scale s_g */
 iq_status iq_update(int32_t* master, int8_t* wq, const int8_t* g, const double* s_g,
                     int64_t n, int lr_log2, int k_u, int k_w, int x2, iq_stream stream);
+
+/* ---------------------------------------------------------------- network glue
+ * (Sec. 2.1 and Sec. 5: the FCN-VGG16 encoder pools, its trainable bilinear-initialised
+ * transposed-convolution decoder, and its MSE loss on quantized logits.) */
+
+/* iq_maxpool_fwd -- k x k max pooling, stride s, padding p (padding never wins), on int8
+ * codes (positive scale: the scale passes through unchanged).  arg (uint8, output shape)
+ * records the tap index r*k + t of the first maximum in scan order for the backward. */
+iq_status iq_maxpool_fwd(const int8_t* x, int32_t n, int32_t h, int32_t w, int32_t c, int32_t k,
+                         int32_t s, int32_t p, int8_t* y, uint8_t* arg, iq_stream stream);
+
+/* iq_maxpool_bwd -- routes each output error to its window's first maximum.  Without
+ * overlap (k <= s) the codes pass through and s_ex = s_e; with overlap the int32 sums are
+ * requantized with Q_E = SQ(., 8).  n, h, w, c are the INPUT dimensions. */
+iq_status iq_maxpool_bwd(const int8_t* e, const double* s_e, const uint8_t* arg, int32_t n,
+                         int32_t h, int32_t w, int32_t c, int32_t k, int32_t s, int32_t p,
+                         int8_t* ex, double* s_ex, void* ws, size_t ws_bytes, iq_stream stream);
+
+/* Workspace of the three upsampling calls below. */
+iq_status iq_upsample_workspace_size(int32_t n, int32_t h, int32_t w, int32_t c, int32_t R,
+                                     size_t* bytes);
+
+/* iq_upsample_fwd -- per-channel (depthwise) transposed convolution, the FCN decoder:
+ * out[n,H,W,c] = sum_{i,j} x[n,i,j,c] w[c][H+pad-i*stride][W+pad-j*stride] over taps inside
+ * the R x R kernel, H = (h-1) stride - 2 pad + R; exact int32, then Q_A = SQ(., 8) (the
+ * quantized logits).  x int8 [n][h][w][c] with device scale s_x; w int8 [c][R][R] (scale
+ * 2^-7); out int8 [n][H][W][c]; s_out device double; acc_out optional int32. */
+iq_status iq_upsample_fwd(const int8_t* x, const double* s_x, const int8_t* w, int32_t n,
+                          int32_t h, int32_t wd, int32_t c, int32_t R, int32_t stride,
+                          int32_t pad, int8_t* out, double* s_out, int32_t* acc_out, void* ws,
+                          size_t ws_bytes, iq_stream stream);
+
+/* iq_upsample_bwd -- its data gradient (Eq. (EQ)): ex[n,i,j,c] = sum_{r,t} E[n, i stride + r - pad,
+ * j stride + t - pad, c] w[c][r][t] exact int32, then SQ(., 8).  Dimensions as in the forward. */
+iq_status iq_upsample_bwd(const int8_t* E, const double* s_e, const int8_t* w, int32_t n,
+                          int32_t h, int32_t wd, int32_t c, int32_t R, int32_t stride,
+                          int32_t pad, int8_t* ex, double* s_ex, int32_t* acc_out, void* ws,
+                          size_t ws_bytes, iq_stream stream);
+
+/* iq_upsample_wgrad -- its weight gradient g[c][r][t] = sum_{n,i,j} x[n,i,j,c] E[...] exact
+ * int64, then Eq. (GQ1) / (GQ2) as in iq_conv_wgrad. */
+iq_status iq_upsample_wgrad(const int8_t* x, const double* s_x, const int8_t* E, const double* s_e,
+                            int32_t n, int32_t h, int32_t wd, int32_t c, int32_t R, int32_t stride,
+                            int32_t pad, int gq_mode, uint64_t seed, uint64_t layer,
+                            uint64_t step, int8_t* g, double* s_g, int64_t* g_acc_out, void* ws,
+                            size_t ws_bytes, iq_stream stream);
+
+/* iq_mse_grad -- gradient of the MSE loss on quantized logits (Sec. 5, FCN), up to its
+ * constant factor: E = z s_z - onehot(label) per pixel and class, then Q_E = SQ(E, 8).
+ * z int8 [npix][c] with device scale s_z; labels uint8 [npix] (values >= c: no target);
+ * E out int8 [npix][c]; s_e out device double.  ws >= 1024 bytes.  The element map is the
+ * fixed-point floor((F z + B_t) / 2^P) of rhu(E 2^7 / max|E|). */
+iq_status iq_mse_grad(const int8_t* z, const double* s_z, const uint8_t* labels, int64_t npix,
+                      int32_t c, int8_t* E, double* s_e, void* ws, size_t ws_bytes,
+                      iq_stream stream);
 
 #ifdef __cplusplus
 }

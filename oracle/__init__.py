@@ -97,6 +97,11 @@ def _declare(L):
     L.or_update.argtypes = [_I64, _P, _P, _P, _D, _I32, _I32, _I32, _I32]
     L.or_quantize_image_u8.argtypes = [_P, _I64, _I32, _I32, _P]
     L.or_quantize_image_u8.restype = _D
+    L.or_maxpool_fwd.argtypes = [_P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P,
+                                 C.POINTER(C.c_int), C.POINTER(C.c_int)]
+    L.or_maxpool_bwd.argtypes = [_P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P]
+    L.or_mse_grad.argtypes = [_P, _I64, _I32, _D, _P, _I32, _P]
+    L.or_mse_grad.restype = _D
     L.or_u128_to_double.argtypes = [_U64, _U64]
     L.or_u128_to_double.restype = _D
 
@@ -228,12 +233,12 @@ def conv_fwd(cv: Conv, x, w) -> np.ndarray:
 
 
 def conv_dgrad(cv: Conv, e, w) -> np.ndarray:
-    """Adjoint of conv_fwd in x: int8 e (NPQK), int8 w -> int32 NHWC."""
+    """Adjoint of conv_fwd in x: int8 e (NPQK), int8 w -> int64 NHWC (exact sums)."""
     d = cv.desc()
     e = _c(e, np.int8)
     w = _c(w, np.int8)
     assert e.size == cv.n * d.p * d.q * cv.k
-    out = np.empty((cv.n, cv.h, cv.w, cv.c), np.int32)
+    out = np.empty((cv.n, cv.h, cv.w, cv.c), np.int64)
     lib().or_conv_dgrad(C.byref(d), _ptr(e), _ptr(w), _ptr(out))
     return out
 
@@ -330,3 +335,37 @@ def update(master, gcodes, s_g: float, lr_log2: int, k_u=24, k_w=8, x2=False):
     wq = np.empty(m.shape, np.int32)
     lib().or_update(m.size, _ptr(m), _ptr(wq), _ptr(g), float(s_g), lr_log2, k_u, k_w, int(x2))
     return m, wq
+
+
+# ---------------------------------------------------------------- network glue
+
+def maxpool_fwd(x, k: int, s: int, p: int = 0):
+    """Max pooling of codes; returns (y, argmax tap index)."""
+    x = _c(x, np.int8)
+    n, h, w, c = x.shape
+    P = (h + 2 * p - k) // s + 1
+    Q = (w + 2 * p - k) // s + 1
+    y = np.empty((n, P, Q, c), np.int8)
+    a = np.empty((n, P, Q, c), np.uint8)
+    ph, pw = C.c_int(), C.c_int()
+    lib().or_maxpool_fwd(_ptr(x), n, h, w, c, k, s, p, _ptr(y), _ptr(a), C.byref(ph), C.byref(pw))
+    return y, a
+
+
+def maxpool_bwd(e, arg, in_shape, k: int, s: int, p: int = 0) -> np.ndarray:
+    e = _c(e, np.int8)
+    arg = _c(arg, np.uint8)
+    n, h, w, c = in_shape
+    ex = np.empty((n, h, w, c), np.int32)
+    lib().or_maxpool_bwd(_ptr(e), _ptr(arg), n, h, w, c, k, s, p, _ptr(ex))
+    return ex
+
+
+def mse_grad(z, s_z: float, labels, k: int = 8):
+    """Q_E of the MSE-loss gradient z s_z - onehot(label) on quantized logits."""
+    z = _c(z, np.int8)
+    lab = _c(labels, np.uint8)
+    c = z.shape[-1]
+    E = np.empty(z.shape, np.int8)
+    s = lib().or_mse_grad(_ptr(z), z.size // c, c, float(s_z), _ptr(lab), k, _ptr(E))
+    return E, s

@@ -302,9 +302,10 @@ void or_conv_fwd(const or_conv* d, const int8_t* x, const int8_t* wt,
 /* data gradient: the adjoint of the forward map,
  * dx[n,h,w,c] = sum over (p,q,k,r,s) with h = p*sh + r*dh - ph,
  * w = q*sw + s*dw - pw of e[n,p,q,k] * w[k,r,s,c].  Scattered image by
- * image (integer sums, so the order is immaterial). */
+ * image (integer sums, so the order is immaterial); int64 result, since the
+ * reduction over k, r, s can exceed 2^31 (fc6: 4096 * 49 products). */
 void or_conv_dgrad(const or_conv* d, const int8_t* e, const int8_t* wt,
-                   int32_t* dx) {
+                   int64_t* dx) {
     const int cg = d->c / d->groups, kg = d->k / d->groups;
     const int64_t img = (int64_t)d->h * d->w * d->c;
     #pragma omp parallel for schedule(static)
@@ -328,7 +329,7 @@ void or_conv_dgrad(const or_conv* d, const int8_t* e, const int8_t* wt,
                         }
                     }
                 }
-        for (int64_t i = 0; i < img; i++) dx[n * img + i] = (int32_t)t[i];
+        for (int64_t i = 0; i < img; i++) dx[n * img + i] = t[i];
         free(t);
     }
 }
@@ -703,4 +704,89 @@ double or_quantize_image_u8(const uint8_t* img, int64_t npix, int c, int c_out,
             out[p * c_out + j] = (int8_t)v;
         }
     return P > 0 ? ldexp((double)P / 255.0, -7) : ldexp(1.0, -7);
+}
+
+/* ------------------------------------------------------------------ */
+/* Network glue of the FCN-VGG16 path (Sec. 2.1, Sec. 5)                */
+/* ------------------------------------------------------------------ */
+
+/* Max pooling on codes (the scale is positive, so the max of the codes is the
+ * code of the max).  Window k x k, stride s, zero-size padding p counted as
+ * -infinity.  The position of the first maximum in (r, s) scan order is kept
+ * for the backward pass (tap index r*k + s; 255 when the window is empty). */
+void or_maxpool_fwd(const int8_t* x, int n, int h, int w, int c, int k, int s, int p,
+                    int8_t* y, uint8_t* arg, int* ph, int* pw) {
+    int P = (h + 2 * p - k) / s + 1, Q = (w + 2 * p - k) / s + 1;
+    *ph = P; *pw = Q;
+    for (int b = 0; b < n; b++)
+        for (int i = 0; i < P; i++)
+            for (int j = 0; j < Q; j++)
+                for (int ch = 0; ch < c; ch++) {
+                    int best = -1000, bi = 255;
+                    for (int r = 0; r < k; r++)
+                        for (int t = 0; t < k; t++) {
+                            int hh = i * s + r - p, ww = j * s + t - p;
+                            if (hh < 0 || hh >= h || ww < 0 || ww >= w) continue;
+                            int v = x[(((int64_t)b * h + hh) * w + ww) * c + ch];
+                            if (v > best) { best = v; bi = r * k + t; }
+                        }
+                    int64_t o = (((int64_t)b * P + i) * Q + j) * c + ch;
+                    y[o] = (int8_t)(bi == 255 ? 0 : best);
+                    arg[o] = (uint8_t)bi;
+                }
+}
+
+/* Backward of max pooling: each output error goes to its window's first
+ * maximum; overlapping windows add.  Returns the int32 sums. */
+void or_maxpool_bwd(const int8_t* e, const uint8_t* arg, int n, int h, int w, int c, int k,
+                    int s, int p, int32_t* ex) {
+    int P = (h + 2 * p - k) / s + 1, Q = (w + 2 * p - k) / s + 1;
+    memset(ex, 0, sizeof(int32_t) * (size_t)n * h * w * c);
+    for (int b = 0; b < n; b++)
+        for (int i = 0; i < P; i++)
+            for (int j = 0; j < Q; j++)
+                for (int ch = 0; ch < c; ch++) {
+                    int64_t o = (((int64_t)b * P + i) * Q + j) * c + ch;
+                    if (arg[o] == 255) continue;
+                    int r = arg[o] / k, t = arg[o] % k;
+                    int hh = i * s + r - p, ww = j * s + t - p;
+                    ex[(((int64_t)b * h + hh) * w + ww) * c + ch] += e[o];
+                }
+}
+
+/* Gradient of the MSE loss on quantized logits (Sec. 5, FCN: MSE loss), up to
+ * its constant factor: E = z s_z - onehot(label) per element, then Q_E = SQ(E, k)
+ * (Eq. (EQ)).  With M = max |E| (fp64, over all elements), the code is
+ * Clip(rhu(E 2^(k-1) / M)) evaluated, like the BN maps, as the fixed-point map
+ * floor((F z + B_t) / 2^P) with F = rhu(s_z q 2^P), B_t = rhu(-t q 2^P) + 2^(P-1),
+ * q = 2^(k-1)/M, t in {0,1}.  Labels >= c (e.g. 255) have no target. */
+double or_mse_grad(const int8_t* z, int64_t npix, int c, double s_z, const uint8_t* lab, int k,
+                   int8_t* E) {
+    double M = 0.0;
+    for (int64_t i = 0; i < npix; i++)
+        for (int ch = 0; ch < c; ch++) {
+            double t = lab[i] == ch ? 1.0 : 0.0;
+            double v = (double)z[i * c + ch] * s_z - t;
+            if (fabs(v) > M) M = fabs(v);
+        }
+    const int64_t lim = qmax(k);
+    if (M == 0.0) {
+        memset(E, 0, (size_t)(npix * c));
+        return ldexp(1.0, 1 - k);
+    }
+    const double q = ldexp(1.0, k - 1) / M;
+    double lmax = fabs(s_z * q) * 127.0 + fabs(q);
+    int P = 62 - frexp_exp(lmax + 1.0);
+    if (P > 62) P = 62;
+    if (P < 1) P = 1;
+    int64_t F = (int64_t)rhu(ldexp(s_z * q, P));
+    int64_t B0 = ((int64_t)1 << (P - 1));
+    int64_t B1 = (int64_t)rhu(ldexp(-q, P)) + ((int64_t)1 << (P - 1));
+    for (int64_t i = 0; i < npix; i++)
+        for (int ch = 0; ch < c; ch++) {
+            int64_t b = lab[i] == ch ? B1 : B0;
+            i128 t = (i128)F * z[i * c + ch] + b;
+            E[i * c + ch] = (int8_t)clamp64((int64_t)(t >> P), -lim, lim);
+        }
+    return ldexp(M, 1 - k);
 }

@@ -154,4 +154,13 @@ struct WsCursor {
         if (e_ != cudaSuccess) return IQ_ERR_CUDA;           \
     } while (0)
 
-#define IQ_LAUNCH_CHECK() IQ_CUDA_CHECK(cudaGetLastError())
+namespace iq {
+// number of kernels this library has enqueued (host-side count, for diagnostics)
+void count_launch();
+}  // namespace iq
+
+#define IQ_LAUNCH_CHECK()                 \
+    do {                                  \
+        iq::count_launch();               \
+        IQ_CUDA_CHECK(cudaGetLastError()); \
+    } while (0)

@@ -36,7 +36,7 @@ __device__ __forceinline__ void load8_bytes(const int8_t* p, int nvalid, uint32_
     hi = b[4] | (b[5] << 8) | (b[6] << 16) | (b[7] << 24);
 }
 
-template <int OP>
+template <int OP, bool WIDE>
 __global__ void __launch_bounds__(256) k_conv_simt(ConvP cp, const int8_t* __restrict__ A_src,
                                                    const int8_t* __restrict__ B_src,
                                                    int32_t* __restrict__ out32,
@@ -87,10 +87,17 @@ __global__ void __launch_bounds__(256) k_conv_simt(ConvP cp, const int8_t* __res
     }
 
     int acc[4][4];
+    long long wacc[WIDE ? 4 : 1][WIDE ? 4 : 1];
 #pragma unroll
     for (int i = 0; i < 4; i++)
 #pragma unroll
         for (int j = 0; j < 4; j++) acc[i][j] = 0;
+    if (WIDE) {
+#pragma unroll
+        for (int i = 0; i < (WIDE ? 4 : 1); i++)
+#pragma unroll
+            for (int j = 0; j < (WIDE ? 4 : 1); j++) wacc[i][j] = 0;
+    }
 
     // K iteration space
     int64_t ktiles;
@@ -212,6 +219,16 @@ __global__ void __launch_bounds__(256) k_conv_simt(ConvP cp, const int8_t* __res
                 for (int j = 0; j < 4; j++) acc[i][j] = __dp4a(a4[i], b4[j], acc[i][j]);
         }
         __syncthreads();
+        if (WIDE) {
+            // fold the 32-product tile sums into int64 (the reduction exceeds int32 range)
+#pragma unroll
+            for (int i = 0; i < 4; i++)
+#pragma unroll
+                for (int j = 0; j < 4; j++) {
+                    wacc[i & (WIDE ? 3 : 0)][j & (WIDE ? 3 : 0)] += acc[i][j];
+                    acc[i][j] = 0;
+                }
+        }
     }
 
     // ---------------- epilogue
@@ -247,7 +264,7 @@ __global__ void __launch_bounds__(256) k_conv_simt(ConvP cp, const int8_t* __res
             atomicMin(&lo_c[c], st_lo[t]);
         }
     } else if (OP == OP_DGRAD) {
-        uint32_t mx = 0;
+        uint64_t mx = 0;
 #pragma unroll
         for (int i = 0; i < 4; i++) {
             int64_t m = m0 + ty * 4 + i;
@@ -256,12 +273,14 @@ __global__ void __launch_bounds__(256) k_conv_simt(ConvP cp, const int8_t* __res
             for (int j = 0; j < 4; j++) {
                 int col = n0 + tx * 4 + j;
                 if (col >= cp.ncols) continue;
-                int v = acc[i][j];
-                out32[m * cp.C + (int64_t)g * cp.Cg + col] = v;
-                mx = max(mx, (uint32_t)(v < 0 ? -v : v));
+                long long v = WIDE ? wacc[i & (WIDE ? 3 : 0)][j & (WIDE ? 3 : 0)] : acc[i][j];
+                if (WIDE) out64[m * cp.C + (int64_t)g * cp.Cg + col] = v;
+                else out32[m * cp.C + (int64_t)g * cp.Cg + col] = (int)v;
+                uint64_t a = (uint64_t)(v < 0 ? -v : v);
+                mx = a > mx ? a : mx;
             }
         }
-        mx = warp_max_u32(mx);
+        mx = warp_max_u64(mx);
         if ((t & 31) == 0 && mx) atomicMax(amax, (unsigned long long)mx);
     } else {
 #pragma unroll
@@ -393,11 +412,16 @@ extern "C" iq_status iq_conv_fwd_workspace_size(const iq_conv_desc* d, int with_
     return IQ_OK;
 }
 
+static bool dgrad_wide(const iq_conv_desc* d) {
+    int64_t krs = (int64_t)(d->k / d->groups) * d->r * d->s;
+    return krs * 127 * 127 >= (int64_t(1) << 31);
+}
+
 extern "C" iq_status iq_conv_dgrad_workspace_size(const iq_conv_desc* d, size_t* bytes) {
     if (!desc_ok(d) || !bytes) return IQ_ERR_INVALID_ARG;
     WsCursor cur(nullptr, 0);
     cur.take<int8_t>((size_t)d->k * d->r * d->s * (d->c / d->groups));
-    cur.take<int32_t>((size_t)d->n * d->h * d->w * d->c);
+    cur.take<int64_t>((size_t)d->n * d->h * d->w * d->c);   // int32, or int64 when wide
     cur.take<char>(requant_ws_bytes());
     cur.take<double>(1);
     *bytes = cur.off + 256;
@@ -452,7 +476,7 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     if (r != IQ_OK) return r;
     if (!done) {
         dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
-        k_conv_simt<OP_FWD><<<grid, 256, 0, st>>>(cp, x, w, acc, nullptr, L.st.s1, L.st.hi,
+        k_conv_simt<OP_FWD, false><<<grid, 256, 0, st>>>(cp, x, w, acc, nullptr, L.st.s1, L.st.hi,
                                                   L.st.lo, nullptr);
         IQ_LAUNCH_CHECK();
     }
@@ -472,8 +496,10 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
                                    const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
                                    void* ws, size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d) || !e || !s_e || !w || !dx || !s_dx) return IQ_ERR_INVALID_ARG;
-    int64_t krs = (int64_t)(d->k / d->groups) * d->r * d->s;
-    if (krs * 127 * 127 >= (int64_t(1) << 31)) return IQ_ERR_OVERFLOW_RISK;
+    const bool wide = dgrad_wide(d);
+    if (wide && acc_out) return IQ_ERR_UNSUPPORTED;   // the sums need 64 bits: no int32 copy
+    if ((int64_t)(d->k / d->groups) * d->r * d->s >= (int64_t(1) << 31) / 4)
+        return IQ_ERR_OVERFLOW_RISK;
     size_t need = 0;
     iq_conv_dgrad_workspace_size(d, &need);
     if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
@@ -481,10 +507,9 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     ConvP cp = make_params(d);
     WsCursor cur(ws, ws_bytes);
     int8_t* wt = cur.take<int8_t>((size_t)d->k * d->r * d->s * cp.Cg);
-    int32_t* accw = cur.take<int32_t>((size_t)d->n * d->h * d->w * d->c);
+    int64_t* accw = cur.take<int64_t>((size_t)d->n * d->h * d->w * d->c);
     void* rq = cur.take<char>(requant_ws_bytes());
     double* s_in = cur.take<double>(1);
-    int32_t* acc = acc_out ? acc_out : accw;
     int64_t wn = (int64_t)d->k * d->r * d->s * cp.Cg;
     k_transpose_w<<<grid_for(wn), kThreads, 0, st>>>(w, wt, d->k, d->r, d->s, cp.Cg, d->groups);
     IQ_LAUNCH_CHECK();
@@ -494,10 +519,18 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     cp.ncols = cp.Cg;
     cp.kin = (int)roundup(cp.Kg, BK);
     dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
-    k_conv_simt<OP_DGRAD><<<grid, 256, 0, st>>>(cp, e, wt, acc, nullptr, nullptr, nullptr,
-                                                nullptr, cell);
-    IQ_LAUNCH_CHECK();
     k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, -7, s_in);
+    IQ_LAUNCH_CHECK();
+    if (wide) {
+        k_conv_simt<OP_DGRAD, true><<<grid, 256, 0, st>>>(cp, e, wt, nullptr, (long long*)accw,
+                                                          nullptr, nullptr, nullptr, cell);
+        IQ_LAUNCH_CHECK();
+        return requant_apply(accw, IQ_I64, cp.M * d->c, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx,
+                             IQ_I8, s_dx, rq, st);
+    }
+    int32_t* acc = acc_out ? acc_out : reinterpret_cast<int32_t*>(accw);
+    k_conv_simt<OP_DGRAD, false><<<grid, 256, 0, st>>>(cp, e, wt, acc, nullptr, nullptr, nullptr,
+                                                       nullptr, cell);
     IQ_LAUNCH_CHECK();
     return requant_apply(acc, IQ_I32, cp.M * d->c, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
                          s_dx, rq, st);
@@ -536,7 +569,7 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
     cp.nsplit = (int)((cp.npq + cp.chunk - 1) / cp.chunk);
     dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN),
               (unsigned)(cp.G * cp.nsplit));
-    k_conv_simt<OP_WGRAD><<<grid, 256, 0, st>>>(cp, e, x, nullptr, (long long*)G, nullptr, nullptr,
+    k_conv_simt<OP_WGRAD, false><<<grid, 256, 0, st>>>(cp, e, x, nullptr, (long long*)G, nullptr, nullptr,
                                                 nullptr, nullptr);
     IQ_LAUNCH_CHECK();
     k_scale_mul<<<1, 1, 0, st>>>(s_e, s_x, s_in);

@@ -5,9 +5,13 @@
 // atomic per warp for the tensor-wide max |x| that Scale(x) needs.
 #include "iq_internal.cuh"
 
+#include <atomic>
 #include <climits>
 
 namespace iq {
+
+static std::atomic<unsigned long long> g_launches{0};
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 // ------------------------------------------------------------------ absmax
 
@@ -339,6 +343,8 @@ extern "C" const char* iq_status_str(iq_status s) {
 }
 
 extern "C" int iq_version(void) { return 1; }
+
+extern "C" unsigned long long iq_launch_count(void) { return g_launches.load(); }
 
 extern "C" iq_status iq_quantize_workspace_size(int64_t n, size_t* bytes) {
     if (!bytes || n < 0) return IQ_ERR_INVALID_ARG;

@@ -1,0 +1,237 @@
+"""FCN-VGG16 on the iq C ABI: the quantized training step and inference pass.
+
+Network (Sec. 2.1 / Sec. 5): the 13 VGG16 3x3 convolutions with 5 max pools, fc6 as a
+7x7 convolution (padding 3) and fc7 as a 1x1 convolution (4096 channels), a 1x1
+score layer over the classes, and a 32x per-class transposed-convolution decoder
+(kernel 64, stride 32, padding 16, bilinear-initialised, trainable).  No BN (Sec. 5:
+FCN uses GQ2 and the MSE loss).
+
+Dataflow per layer (Sec. 3.2-3.3): W_q = UQ(W_m, 8) from 24-bit master weights,
+int32 convolution, A = Q_A(ReLU(acc)) = SQ(., 8); backward e = e_A [A > 0],
+E_1 = SQ(dgrad, 8), G_q = RQ(G/Scale(G), 8) (Eq. (GQ2)), W_m -= UQ(G_q lr, 24).
+
+Every step runs in the library's kernels; this module only allocates device memory
+(torch tensors) and sequences the C ABI calls on one stream.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+import torch
+
+from . import iq
+from . import synthetic as S
+
+UP_R, UP_STRIDE, UP_PAD = 64, 32, 16
+
+
+@dataclass
+class Conv:
+    name: str
+    desc: iq.ConvDesc
+    cin: int
+    cout: int
+    r: int
+    pad: int
+    relu: bool
+    layer_id: int
+    master: torch.Tensor = None
+    wq: torch.Tensor = None
+    g: torch.Tensor = None
+    s_g: torch.Tensor = None
+    x: torch.Tensor = None        # input codes (NHWC)
+    s_x: torch.Tensor = None
+    a: torch.Tensor = None        # output codes
+    s_a: torch.Tensor = None
+    ea: torch.Tensor = None       # error of the output (E_1)
+    s_ea: torch.Tensor = None
+    e: torch.Tensor = None        # error after the ReLU mask
+    ex: torch.Tensor = None       # error of the input (dgrad output)
+    s_ex: torch.Tensor = None
+    macs: int = 0
+
+
+@dataclass
+class Pool:
+    x: torch.Tensor
+    y: torch.Tensor
+    arg: torch.Tensor
+    ey: torch.Tensor = None       # error of the pooled output
+    s_ey: torch.Tensor = None
+    ex: torch.Tensor = None       # error of the pool input
+    s_ex: torch.Tensor = None
+
+
+class FcnVgg16:
+    """Preallocated FCN-VGG16 for a fixed batch shape.
+
+    width scales every channel count (1.0 = the paper's network); tests use small widths."""
+
+    def __init__(self, n: int, h: int, w: int, classes: int = 150, width: float = 1.0,
+                 seed: int = 0, lr_log2: int = 10, device: str = "cuda", train: bool = True):
+        assert h % 32 == 0 and w % 32 == 0, "the 32x decoder needs sizes divisible by 32"
+        self.n, self.h, self.w, self.classes = n, h, w, classes
+        self.dev = torch.device(device)
+        self.lr_log2 = lr_log2
+        self.train = train
+        self.step_count = 0
+        self.seed = seed
+        dev = self.dev
+
+        def scal():
+            return torch.zeros(1, dtype=torch.float64, device=dev)
+
+        self.img_codes = torch.empty((n, h, w, 4), dtype=torch.int8, device=dev)
+        self.s_img = scal()
+        self.layers: list = []   # Conv and Pool in forward order
+        self.convs: list = []
+        weights, up_filters = S.fcn_vgg16_weights(seed, classes, width)
+        cur, s_cur, hh, ww = self.img_codes, self.s_img, h, w
+        lid = 0
+        for name, cin, cout, r, pad, relu in S.fcn_vgg16_channels(classes, width):
+            if name == "pool":
+                y = torch.empty((n, hh // 2, ww // 2, cin), dtype=torch.int8, device=dev)
+                arg = torch.empty_like(y, dtype=torch.uint8)
+                self.layers.append(Pool(cur, y, arg))
+                cur, hh, ww = y, hh // 2, ww // 2
+                continue
+            cur, s_cur = self._add_conv(name, cur, s_cur, cin, cout, r, pad, relu, lid, hh, ww,
+                                        weights[lid])
+            lid += 1
+        self.score, self.s_score, self.score_hw = cur, s_cur, (hh, ww)
+        # decoder: per-class transposed convolution, W_m = UQ(W, 24) (Eq. (WQ0))
+        self.up_layer_id = lid
+        self.up_master = self._master(up_filters)
+        self.up_wq = torch.empty((classes, UP_R, UP_R), dtype=torch.int8, device=dev)
+        iq.iq_weight_requant(self.up_master, self.up_wq)
+        self.z = torch.empty((n, h, w, classes), dtype=torch.int8, device=dev)
+        self.s_z = scal()
+        if train:
+            self.Ez = torch.empty_like(self.z)
+            self.s_Ez = scal()
+            self.up_g = torch.empty_like(self.up_wq)
+            self.up_s_g = scal()
+            self.e_score = torch.empty_like(self.score)
+            self.s_e_score = scal()
+        self.up_macs = n * h * w * classes * 4   # <= 2 x 2 taps per output pixel
+        self._alloc_backward()
+        self.ws = torch.empty(self._ws_bytes(), dtype=torch.uint8, device=dev)
+
+    def _master(self, w_fp32: np.ndarray) -> torch.Tensor:
+        """Master weights W_m = UQ(W, 24) (Eq. (WQ0)) computed on the device."""
+        w = torch.from_numpy(np.ascontiguousarray(w_fp32)).to(self.dev)
+        m = torch.empty(w.shape, dtype=torch.int32, device=self.dev)
+        iq.iq_quantize(w, 24, iq.IQ_MODE_UQ, m, torch.zeros(1, dtype=torch.float64,
+                                                            device=self.dev))
+        return m
+
+    # ------------------------------------------------------------------ construction
+
+    def _add_conv(self, name, x, s_x, cin, cout, r, pad, relu, lid, hh, ww, w_fp32):
+        n, dev = self.n, self.dev
+        d = iq.conv_desc(n, hh, ww, cin, cout, r, r, 1, pad)
+        L = Conv(name, d, cin, cout, r, pad, relu, lid)
+        L.master = self._master(w_fp32)
+        L.wq = torch.empty((cout, r, r, cin), dtype=torch.int8, device=dev)
+        iq.iq_weight_requant(L.master, L.wq)
+        L.x, L.s_x = x, s_x
+        L.a = torch.empty((n, hh, ww, cout), dtype=torch.int8, device=dev)
+        L.s_a = torch.zeros(1, dtype=torch.float64, device=dev)
+        L.macs = n * hh * ww * cout * r * r * (3 if cin == 4 else cin)
+        self.layers.append(L)
+        self.convs.append(L)
+        return L.a, L.s_a
+
+    def _alloc_backward(self):
+        if not self.train:
+            return
+        dev = self.dev
+        for L in self.convs:
+            L.ea = torch.empty_like(L.a)
+            L.s_ea = torch.zeros(1, dtype=torch.float64, device=dev)
+            L.e = torch.empty_like(L.a)
+            L.g = torch.empty_like(L.wq)
+            L.s_g = torch.zeros(1, dtype=torch.float64, device=dev)
+            if L.layer_id > 0:
+                L.ex = torch.empty_like(L.x)
+                L.s_ex = torch.zeros(1, dtype=torch.float64, device=dev)
+        for P in self.layers:
+            if isinstance(P, Pool):
+                P.ex = torch.empty_like(P.x)
+                P.s_ex = torch.zeros(1, dtype=torch.float64, device=dev)
+
+    def _ws_bytes(self) -> int:
+        b = iq.iq_quantize_workspace_size(self.img_codes.numel())
+        for L in self.convs:
+            b = max(b, iq.iq_conv_fwd_workspace_size(L.desc, False))
+            if self.train:
+                b = max(b, iq.iq_conv_dgrad_workspace_size(L.desc),
+                        iq.iq_conv_wgrad_workspace_size(L.desc))
+        hs, ws_ = self.score_hw
+        b = max(b, iq.iq_upsample_workspace_size(self.n, hs, ws_, self.classes, UP_R))
+        return b + 4096
+
+    # ------------------------------------------------------------------ passes
+
+    @property
+    def macs_forward(self) -> int:
+        return sum(L.macs for L in self.convs) + self.up_macs
+
+    @property
+    def macs_step(self) -> int:
+        # forward, data gradient (not for the first layer) and weight gradient of every conv
+        f = sum(L.macs for L in self.convs)
+        dg = sum(L.macs for L in self.convs if L.layer_id > 0)
+        return f + dg + f + 3 * self.up_macs
+
+    def forward(self, img_u8: torch.Tensor, stream=None):
+        ws = self.ws
+        iq.iq_quantize_image_u8(img_u8, False, 4, self.img_codes, self.s_img, ws=ws, stream=stream)
+        for item in self.layers:
+            if isinstance(item, Pool):
+                iq.iq_maxpool_fwd(item.x, 2, 2, 0, item.y, item.arg, stream=stream)
+                continue
+            L = item
+            iq.iq_conv_fwd(L.desc, L.x, L.s_x, L.wq, L.a, L.s_a, relu=L.relu, ws=ws,
+                           stream=stream)
+        iq.iq_upsample_fwd(self.score, self.s_score, self.up_wq, UP_R, UP_STRIDE, UP_PAD, self.z,
+                           self.s_z, ws=ws, stream=stream)
+
+    def backward_update(self, labels: torch.Tensor, stream=None):
+        assert self.train
+        ws, step, seed, lr = self.ws, self.step_count, self.seed, self.lr_log2
+        iq.iq_mse_grad(self.z, self.s_z, labels, self.Ez, self.s_Ez, ws=ws, stream=stream)
+        hs, wsz = self.score_hw
+        iq.iq_upsample_wgrad(self.score, self.s_score, self.Ez, self.s_Ez, UP_R, UP_STRIDE, UP_PAD,
+                             self.up_g, self.up_s_g, gq_mode=2, seed=seed,
+                             layer=self.up_layer_id, step=step, ws=ws, stream=stream)
+        iq.iq_upsample_bwd(self.Ez, self.s_Ez, self.up_wq, self.score.shape, UP_R, UP_STRIDE,
+                           UP_PAD, self.e_score, self.s_e_score, ws=ws, stream=stream)
+        iq.iq_update(self.up_master, self.up_wq, self.up_g, self.up_s_g, lr, stream=stream)
+        # error arriving at the output of the current item, walking backwards
+        err, s_err = self.e_score, self.s_e_score
+        for item in reversed(self.layers):
+            if isinstance(item, Pool):
+                iq.iq_maxpool_bwd(err, s_err, item.arg, item.x.shape, 2, 2, 0, item.ex, item.s_ex,
+                                  ws=ws, stream=stream)
+                err, s_err = item.ex, item.s_ex
+                continue
+            L = item
+            if L.relu:
+                iq.iq_relu_bwd(err, L.a, L.e, stream=stream)
+                e = L.e
+            else:
+                e = err
+            if L.layer_id > 0:
+                iq.iq_conv_dgrad(L.desc, e, s_err, L.wq, L.ex, L.s_ex, ws=ws, stream=stream)
+            iq.iq_conv_wgrad(L.desc, e, s_err, L.x, L.s_x, L.g, L.s_g, gq_mode=2, seed=seed,
+                             layer=L.layer_id, step=step, ws=ws, stream=stream)
+            iq.iq_update(L.master, L.wq, L.g, L.s_g, lr, stream=stream)
+            if L.layer_id > 0:
+                err, s_err = L.ex, L.s_ex
+        self.step_count += 1
+
+    def train_step(self, img_u8, labels, stream=None):
+        self.forward(img_u8, stream)
+        self.backward_update(labels, stream)

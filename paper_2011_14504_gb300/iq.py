@@ -21,11 +21,13 @@ IQ_MODE_UQ, IQ_MODE_UQ2, IQ_MODE_SQ, IQ_MODE_SQ_RELU, IQ_MODE_RQ_GQ1, IQ_MODE_RQ
 IQ_BN_S_XHAT, IQ_BN_M_XHAT, IQ_BN_M_Y, IQ_BN_S_ACC, IQ_BN_S_A, IQ_BN_SCALES = 0, 1, 2, 3, 4, 8
 
 EXPORTS = [
-    "iq_status_str", "iq_version", "iq_conv_out_size", "iq_quantize_workspace_size",
+    "iq_status_str", "iq_version", "iq_launch_count", "iq_conv_out_size", "iq_quantize_workspace_size",
     "iq_conv_fwd_workspace_size", "iq_conv_dgrad_workspace_size", "iq_conv_wgrad_workspace_size",
     "iq_bn_int_workspace_size", "iq_quantize", "iq_quantize_image_u8", "iq_requantize",
     "iq_weight_requant", "iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad", "iq_bn_int_fwd",
-    "iq_bn_int_bwd", "iq_relu_bwd", "iq_update",
+    "iq_bn_int_bwd", "iq_relu_bwd", "iq_update", "iq_maxpool_fwd", "iq_maxpool_bwd",
+    "iq_upsample_workspace_size", "iq_upsample_fwd", "iq_upsample_bwd", "iq_upsample_wgrad",
+    "iq_mse_grad",
 ]
 
 
@@ -65,6 +67,8 @@ def load(path: str | None = None):
     L.iq_status_str.restype = C.c_char_p
     L.iq_status_str.argtypes = [_I]
     L.iq_version.restype = _I
+    L.iq_launch_count.restype = C.c_ulonglong
+    L.iq_launch_count.argtypes = []
     L.iq_conv_out_size.argtypes = [C.POINTER(ConvDesc), C.POINTER(_I32), C.POINTER(_I32)]
     L.iq_quantize_workspace_size.argtypes = [_I64, C.POINTER(_SZ)]
     L.iq_conv_fwd_workspace_size.argtypes = [C.POINTER(ConvDesc), _I, C.POINTER(_SZ)]
@@ -87,11 +91,26 @@ def load(path: str | None = None):
                                 _P, _P, _P, _P, _SZ, _P]
     L.iq_relu_bwd.argtypes = [_P, _P, _I64, _P, _P]
     L.iq_update.argtypes = [_P, _P, _P, _P, _I64, _I, _I, _I, _I, _P]
+    L.iq_maxpool_fwd.argtypes = [_P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P]
+    L.iq_maxpool_bwd.argtypes = [_P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P,
+                                 _SZ, _P]
+    L.iq_upsample_workspace_size.argtypes = [_I32, _I32, _I32, _I32, _I32, C.POINTER(_SZ)]
+    L.iq_upsample_fwd.argtypes = [_P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P,
+                                  _P, _SZ, _P]
+    L.iq_upsample_bwd.argtypes = [_P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P,
+                                  _P, _SZ, _P]
+    L.iq_upsample_wgrad.argtypes = [_P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _I,
+                                    _U64, _U64, _U64, _P, _P, _P, _P, _SZ, _P]
+    L.iq_mse_grad.argtypes = [_P, _P, _P, _I64, _I32, _P, _P, _P, _SZ, _P]
     for f in EXPORTS:
-        if f not in ("iq_status_str", "iq_version"):
+        if f not in ("iq_status_str", "iq_version", "iq_launch_count"):
             getattr(L, f).restype = _I
     _L = L
     return L
+
+
+def launch_count() -> int:
+    return int(load().iq_launch_count())
 
 
 def status_str(code: int) -> str:
@@ -267,3 +286,62 @@ def iq_relu_bwd(e_a, a, e, stream=None):
 def iq_update(master, wq, g, s_g, lr_log2, k_u=24, k_w=8, x2=False, stream=None):
     _check("iq_update", load().iq_update(_p(master), _p(wq), _p(g), _p(s_g), master.numel(),
                                          lr_log2, k_u, k_w, int(x2), _stream(stream)))
+
+
+# ---------------------------------------------------------------- network glue
+
+def iq_maxpool_fwd(x, k, s, p, y, arg, stream=None):
+    n, h, w, c = x.shape
+    _check("iq_maxpool_fwd", load().iq_maxpool_fwd(_p(x), n, h, w, c, k, s, p, _p(y), _p(arg),
+                                                   _stream(stream)))
+
+
+def iq_maxpool_bwd(e, s_e, arg, in_shape, k, s, p, ex, s_ex, ws=None, stream=None):
+    n, h, w, c = in_shape
+    if ws is None:
+        ws = _ws(n * h * w * c * 4 + 4096, e.device)
+    _check("iq_maxpool_bwd", load().iq_maxpool_bwd(_p(e), _p(s_e), _p(arg), n, h, w, c, k, s, p,
+                                                   _p(ex), _p(s_ex), _p(ws), ws.numel(),
+                                                   _stream(stream)))
+
+
+def iq_upsample_workspace_size(n, h, w, c, R) -> int:
+    return _size("iq_upsample_workspace_size", n, h, w, c, R)
+
+
+def iq_upsample_fwd(x, s_x, w, R, stride, pad, out, s_out, acc_out=None, ws=None, stream=None):
+    n, h, wd, c = x.shape
+    if ws is None:
+        ws = _ws(iq_upsample_workspace_size(n, h, wd, c, R), x.device)
+    _check("iq_upsample_fwd", load().iq_upsample_fwd(_p(x), _p(s_x), _p(w), n, h, wd, c, R, stride,
+                                                     pad, _p(out), _p(s_out), _p(acc_out), _p(ws),
+                                                     ws.numel(), _stream(stream)))
+
+
+def iq_upsample_bwd(E, s_e, w, x_shape, R, stride, pad, ex, s_ex, acc_out=None, ws=None,
+                    stream=None):
+    n, h, wd, c = x_shape
+    if ws is None:
+        ws = _ws(iq_upsample_workspace_size(n, h, wd, c, R), E.device)
+    _check("iq_upsample_bwd", load().iq_upsample_bwd(_p(E), _p(s_e), _p(w), n, h, wd, c, R, stride,
+                                                     pad, _p(ex), _p(s_ex), _p(acc_out), _p(ws),
+                                                     ws.numel(), _stream(stream)))
+
+
+def iq_upsample_wgrad(x, s_x, E, s_e, R, stride, pad, g, s_g, gq_mode=2, seed=0, layer=0, step=0,
+                      g_acc_out=None, ws=None, stream=None):
+    n, h, wd, c = x.shape
+    if ws is None:
+        ws = _ws(iq_upsample_workspace_size(n, h, wd, c, R), x.device)
+    _check("iq_upsample_wgrad",
+           load().iq_upsample_wgrad(_p(x), _p(s_x), _p(E), _p(s_e), n, h, wd, c, R, stride, pad,
+                                    gq_mode, seed, layer, step, _p(g), _p(s_g), _p(g_acc_out),
+                                    _p(ws), ws.numel(), _stream(stream)))
+
+
+def iq_mse_grad(z, s_z, labels, E, s_e, ws=None, stream=None):
+    c = z.shape[-1]
+    if ws is None:
+        ws = _ws(4096, z.device)
+    _check("iq_mse_grad", load().iq_mse_grad(_p(z), _p(s_z), _p(labels), z.numel() // c, c, _p(E),
+                                             _p(s_e), _p(ws), ws.numel(), _stream(stream)))

@@ -11,7 +11,6 @@ from __future__ import annotations
 
 import numpy as np
 
-K_U = 24  # bit width of the master-weight grid (Sec. 5, k_U = 24)
 
 
 def rng(seed: int) -> np.random.Generator:
@@ -23,13 +22,58 @@ def int8_uniform(g: np.random.Generator, shape, lo: int = -127, hi: int = 127) -
     return g.integers(lo, hi + 1, size=shape, dtype=np.int64).astype(np.int8)
 
 
-def master_weights(g: np.random.Generator, shape, fan_in: int) -> np.ndarray:
-    """He (MSRA) initialisation, std sqrt(2/fan_in), drawn directly as integer codes
-    on the 2^-23 master grid: a rounded Gaussian clipped to +-(2^23 - 1)."""
+def he_weights(g: np.random.Generator, shape, fan_in: int) -> np.ndarray:
+    """He (MSRA) initialisation, N(0, sqrt(2/fan_in)), as fp32 real weights (the
+    method's W_m = UQ(W, k_U), Eq. (WQ0), is applied by whoever consumes them)."""
     std = np.sqrt(2.0 / fan_in)
-    lim = 2 ** (K_U - 1) - 1
-    v = np.rint(g.standard_normal(size=shape) * std * 2 ** (K_U - 1))
-    return np.clip(v, -lim, lim).astype(np.int32)
+    return (g.standard_normal(size=shape) * std).astype(np.float32)
+
+
+def bilinear_filters(classes: int, R: int) -> np.ndarray:
+    """Bilinear upsampling filters, one R x R filter per class, fp32 [classes][R][R]
+    (the FCN decoder initialisation)."""
+    f = (R + 1) // 2
+    center = f - 1 if R % 2 == 1 else f - 0.5
+    k1 = 1 - np.abs(np.arange(R) - center) / f
+    return np.broadcast_to(np.outer(k1, k1).astype(np.float32), (classes, R, R)).copy()
+
+
+VGG16 = [64, 64, "P", 128, 128, "P", 256, 256, 256, "P", 512, 512, 512, "P", 512, 512, 512, "P"]
+
+
+def fcn_vgg16_channels(classes: int = 150, width: float = 1.0):
+    """(name, cin, cout, r, pad, relu) of the FCN-VGG16 convolutions in forward order; the
+    3 RGB input channels are padded to 4.  width scales every hidden channel count."""
+    def ch(c):
+        return max(8, int(round(c * width)) // 8 * 8)
+    out, cin, i = [], 4, 0
+    for item in VGG16:
+        if item == "P":
+            out.append(("pool", cin, cin, 2, 0, False))
+            continue
+        i += 1
+        out.append((f"conv{i}", cin, ch(item), 3, 1, True))
+        cin = ch(item)
+    out.append(("fc6", cin, ch(4096), 7, 3, True))
+    out.append(("fc7", ch(4096), ch(4096), 1, 0, True))
+    out.append(("score", ch(4096), classes, 1, 0, False))
+    return out
+
+
+def fcn_vgg16_weights(seed: int, classes: int = 150, width: float = 1.0):
+    """fp32 initial weights of FCN-VGG16: He-initialised KRSC filters for every conv
+    (channel 3 of the first layer, the RGB padding, is zero) and the bilinear decoder."""
+    g = rng(seed)
+    ws = []
+    for name, cin, cout, r, pad, relu in fcn_vgg16_channels(classes, width):
+        if name == "pool":
+            continue
+        fan_in = (3 if cin == 4 else cin) * r * r
+        w = he_weights(g, (cout, r, r, cin), fan_in)
+        if cin == 4:
+            w[..., 3] = 0.0
+        ws.append(w)
+    return ws, bilinear_filters(classes, 64)
 
 
 def bn_gamma_beta_codes(g: np.random.Generator, channels: int):

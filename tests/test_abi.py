@@ -15,7 +15,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 def declared_entry_points():
     src = open(os.path.join(ROOT, "include", "iq.h")).read()
-    return sorted(set(re.findall(r"^\s*(?:iq_status|const char\*|int)\s+(iq_\w+)\s*\(", src,
+    return sorted(set(re.findall(r"^\s*(?:iq_status|const char\*|int|unsigned long long)\s+(iq_\w+)\s*\(", src,
                                  re.M)))
 
 

@@ -1,0 +1,57 @@
+"""FCN-VGG16 training steps on the GPU against the oracle network, free-running.
+
+A reduced-width network (same layer structure, channels x 1/8) on 64 x 64 images keeps
+the oracle in seconds; both sides start from the same fp32 initial weights and consume
+identical input bytes, so every intermediate must agree bit for bit, step after step.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from oracle.fcn import OracleFcn
+from paper_2011_14504_gb300 import synthetic as S
+from paper_2011_14504_gb300.fcn import FcnVgg16, Pool
+
+pytestmark = pytest.mark.gpu
+
+
+def host(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+@pytest.mark.parametrize("classes,width,n", [(21, 0.125, 2), (150, 0.0625, 1)])
+def test_fcn_train_steps_match_oracle(classes, width, n):
+    h = w = 64
+    seed = 3
+    g = S.rng(100 + classes)
+    net = FcnVgg16(n, h, w, classes=classes, width=width, seed=seed, lr_log2=6)
+    chans = S.fcn_vgg16_channels(classes, width)
+    wts, up = S.fcn_vgg16_weights(seed, classes, width)
+    ora = OracleFcn(chans, wts, up, classes, seed=seed, lr_log2=6)
+    for step in range(2):
+        img = S.images_u8(g, n, h, w)
+        lab = S.labels_voronoi(g, n, h, w, classes, sites=6)
+        net.train_step(torch.from_numpy(img).cuda(), torch.from_numpy(lab).cuda())
+        tr = ora.forward(img)
+        convs = [it for it in tr["layers"] if it[0] == "conv"]
+        for L, it in zip(net.convs, convs):
+            _, li, cv, x, s_x, wq, acc, a, s_a, relu = it
+            assert np.array_equal(host(L.a), a), (step, L.name)
+            assert host(L.s_a)[0] == s_a, (step, L.name)
+        cvu, score, s_score, up_wq, zacc, z, s_z = tr["up"]
+        assert np.array_equal(host(net.z), z) and host(net.s_z)[0] == s_z
+        out = ora.backward_update(tr, lab)
+        E, s_E = out["E"]
+        assert np.array_equal(host(net.Ez), E) and host(net.s_Ez)[0] == s_E
+        assert np.array_equal(host(net.e_score), out["e_score"][0])
+        assert np.array_equal(host(net.up_g), out["up_g"][1])
+        for L in net.convs:
+            G, gq, s_g = out["grads"][L.layer_id]
+            assert np.array_equal(host(L.g), gq.astype(np.int8)), (step, L.name)
+            assert host(L.s_g)[0] == s_g
+            if L.layer_id > 0:
+                assert np.array_equal(host(L.ex), out["ex"][L.layer_id][0]), (step, L.name)
+            assert np.array_equal(host(L.master), ora.masters[L.layer_id]), (step, L.name)
+        assert np.array_equal(host(net.up_master), ora.up_master)

@@ -120,7 +120,7 @@ def test_requantize_rq_int64(mode, gq):
 
 def test_weight_requant_and_update():
     g = S.rng(5)
-    m = S.master_weights(g, 100001, 576)
+    m = O.uq(S.he_weights(g, 100001, 576), 24)
     wq = torch.empty(m.size, dtype=torch.int8, device=DEV)
     md = dev(m)
     iq.iq_weight_requant(md, wq)
@@ -166,7 +166,7 @@ def _conv_case(ci, seed):
     g = S.rng(seed)
     p, q = cv.pq
     x = S.int8_uniform(g, (n, h, w, c))
-    wm = S.master_weights(g, (k, r, s, c // gr), c // gr * r * s)
+    wm = O.uq(S.he_weights(g, (k, r, s, c // gr), c // gr * r * s), 24)
     wq = O.requant_master(wm).astype(np.int8)
     e = S.int8_uniform(g, (n, p, q, k))
     return cv, d, x, wq, e
@@ -318,7 +318,7 @@ def test_conv_fwd_tc_shapes(ci):
     d = iq.conv_desc(n, h, w, c, k, r, s, st, pd, dl)
     g = S.rng(90 + ci)
     x = S.int8_uniform(g, (n, h, w, c))
-    wq = O.requant_master(S.master_weights(g, (k, r, s, c), c * r * s)).astype(np.int8)
+    wq = O.requant_master(O.uq(S.he_weights(g, (k, r, s, c), c * r * s), 24)).astype(np.int8)
     p, q = cv.pq
     a = torch.empty((n, p, q, k), dtype=torch.int8, device=DEV)
     acc = torch.empty((n, p, q, k), dtype=torch.int32, device=DEV)
@@ -345,3 +345,93 @@ def test_conv_fwd_adversarial_full_scale(sign):
     got = host(acc)
     assert np.array_equal(got, O.conv_fwd(cv, x, wq))
     assert got[0, 2, 2, 0] == sign * 4608 * 16129
+
+
+# ----------------------------------------------------------------- network glue
+
+@pytest.mark.parametrize("k,s,p", [(2, 2, 0), (3, 2, 1)])
+def test_maxpool(k, s, p):
+    g = S.rng(k * 10 + s)
+    x = S.int8_uniform(g, (2, 37, 30, 24), -9, 9)
+    y_o, a_o = O.maxpool_fwd(x, k, s, p)
+    y = torch.empty(y_o.shape, dtype=torch.int8, device=DEV)
+    a = torch.empty(y_o.shape, dtype=torch.uint8, device=DEV)
+    iq.iq_maxpool_fwd(dev(x), k, s, p, y, a)
+    assert np.array_equal(host(y), y_o) and np.array_equal(host(a), a_o)
+    e = S.int8_uniform(g, y_o.shape)
+    ex = torch.empty(x.shape, dtype=torch.int8, device=DEV)
+    s_ex = dscal()
+    iq.iq_maxpool_bwd(dev(e), dscal(0.5), a, x.shape, k, s, p, ex, s_ex)
+    sums = O.maxpool_bwd(e, a_o, x.shape, k, s, p)
+    if k <= s:
+        assert np.array_equal(host(ex).astype(np.int32), sums) and host(s_ex)[0] == 0.5
+    else:
+        want, ws_ = O.sq_int(sums, 0.5, 8)
+        assert np.array_equal(host(ex).astype(np.int32), want) and host(s_ex)[0] == ws_
+
+
+@pytest.mark.parametrize("n,h,c,R,st,pd", [(1, 2, 150, 64, 32, 16), (2, 3, 21, 16, 8, 4)])
+def test_upsample_fwd_bwd_wgrad(n, h, c, R, st, pd):
+    g = S.rng(c + R)
+    H = (h - 1) * st - 2 * pd + R
+    cv = O.Conv(n, H, H, c, c, R, R, st, pd, 1, c)      # the strided conv it is the adjoint of
+    assert cv.pq == (h, h)
+    x = S.int8_uniform(g, (n, h, h, c))
+    w = S.int8_uniform(g, (c, R, R, 1))
+    out = torch.empty((n, H, H, c), dtype=torch.int8, device=DEV)
+    acc = torch.empty((n, H, H, c), dtype=torch.int32, device=DEV)
+    s_out = dscal()
+    iq.iq_upsample_fwd(dev(x), dscal(0.03), dev(w), R, st, pd, out, s_out, acc_out=acc)
+    want_acc = O.conv_dgrad(cv, x, w)
+    assert np.array_equal(host(acc), want_acc)
+    want, ws_ = O.sq_int(want_acc, 0.03 * 2.0 ** -7, 8)
+    assert np.array_equal(host(out).astype(np.int32), want) and host(s_out)[0] == ws_
+    E = S.int8_uniform(g, (n, H, H, c))
+    ex = torch.empty((n, h, h, c), dtype=torch.int8, device=DEV)
+    eacc = torch.empty((n, h, h, c), dtype=torch.int32, device=DEV)
+    s_ex = dscal()
+    iq.iq_upsample_bwd(dev(E), dscal(1e-3), dev(w), (n, h, h, c), R, st, pd, ex, s_ex, acc_out=eacc)
+    want_e = O.conv_fwd(cv, E, w)
+    assert np.array_equal(host(eacc), want_e)
+    want, ws_ = O.sq_int(want_e, 1e-3 * 2.0 ** -7, 8)
+    assert np.array_equal(host(ex).astype(np.int32), want) and host(s_ex)[0] == ws_
+    gq = torch.empty((c, R, R), dtype=torch.int8, device=DEV)
+    gacc = torch.empty((c, R, R), dtype=torch.int64, device=DEV)
+    s_g = dscal()
+    iq.iq_upsample_wgrad(dev(x), dscal(0.03), dev(E), dscal(1e-3), R, st, pd, gq, s_g, gq_mode=2,
+                         seed=5, layer=19, step=2, g_acc_out=gacc)
+    want_g = O.conv_wgrad(cv, x, E).reshape(c, R, R)
+    assert np.array_equal(host(gacc), want_g)
+    want, ws_ = O.rq_int(want_g, 0.03 * 1e-3, 8, 2, 5, 19, 2, 0)
+    assert np.array_equal(host(gq).astype(np.int32), want) and host(s_g)[0] == ws_
+
+
+def test_mse_grad():
+    g = S.rng(77)
+    z = S.int8_uniform(g, (2, 33, 17, 150))
+    lab = S.labels_voronoi(g, 2, 33, 17, 150, sites=8)
+    E = torch.empty(z.shape, dtype=torch.int8, device=DEV)
+    s_e = dscal()
+    iq.iq_mse_grad(dev(z), dscal(0.0123), dev(lab), E, s_e)
+    want, ws_ = O.mse_grad(z, 0.0123, lab)
+    assert np.array_equal(host(E), want) and host(s_e)[0] == ws_
+
+
+def test_conv_dgrad_int64_reduction():
+    # (k/groups) r s = 20000 * 49 products: sums beyond int32 range, accumulated in int64
+    n, h, w, c, k = 1, 3, 3, 8, 20000
+    cv = O.Conv(n, h, w, c, k, 7, 7, 1, 3)
+    d = iq.conv_desc(n, h, w, c, k, 7, 7, 1, 3)
+    e = np.full((n, h, w, k), 127, np.int8)
+    wq = np.full((k, 7, 7, c), 127, np.int8)
+    wq[:, :, :, 1] = -127
+    dx = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
+    s_dx = dscal()
+    iq.iq_conv_dgrad(d, dev(e), dscal(1e-4), dev(wq), dx, s_dx)
+    want_acc = O.conv_dgrad(cv, e, wq)
+    assert np.abs(want_acc).max() > 2 ** 31
+    want, ws_ = O.sq_int(want_acc, 1e-4 * 2.0 ** -7, 8)
+    assert np.array_equal(host(dx).astype(np.int32), want) and host(s_dx)[0] == ws_
+    with pytest.raises(iq.IqError):
+        iq.iq_conv_dgrad(d, dev(e), dscal(1e-4), dev(wq), dx, s_dx,
+                         acc_out=torch.empty((n, h, w, c), dtype=torch.int32, device=DEV))

@@ -209,7 +209,7 @@ def test_rq_probability_matches_fraction():
 
 def test_master_to_forward_weights():
     g = S.rng(21)
-    m = S.master_weights(g, 5000, 9)
+    m = O.uq(S.he_weights(g, 5000, 9), 24)
     m[:4] = [2 ** 15, -(2 ** 15), 2 ** 23 - 1, -(2 ** 23 - 1)]
     got = O.requant_master(m)
     want = [clip(rhu_exact(Fr(int(v), 2 ** 16)), 8) for v in m]
@@ -219,7 +219,7 @@ def test_master_to_forward_weights():
 
 def test_update_gq2_shift_identity_and_clip():
     g = S.rng(22)
-    m = S.master_weights(g, 4000, 64)
+    m = O.uq(S.he_weights(g, 4000, 64), 24)
     gc = S.int8_uniform(g, 4000).astype(np.int32)
     for e in (6, 10, 16):
         m2, wq = O.update(m, gc, 2.0 ** -7, e)
@@ -524,3 +524,54 @@ def test_image_input_quantization_exact():
     assert codes[..., :3].reshape(-1).tolist() == want
     assert (codes[..., 3] == 0).all()
     assert s == P / 255 * 2 ** -7
+
+
+# ----------------------------------------------------------------- network glue
+
+def test_maxpool_matches_torch_and_routes_first_max():
+    g = S.rng(70)
+    x = S.int8_uniform(g, (2, 9, 8, 5), -5, 5)   # many ties
+    for k, s, p in ((2, 2, 0), (3, 2, 1)):
+        y, a = O.maxpool_fwd(x, k, s, p)
+        t = torch.from_numpy(x.astype(np.float64)).permute(0, 3, 1, 2)
+        want = torch.nn.functional.max_pool2d(t, k, s, p).permute(0, 2, 3, 1).numpy()
+        assert np.array_equal(y, want.astype(np.int8))
+        e = S.int8_uniform(g, y.shape)
+        ex = O.maxpool_bwd(e, a, x.shape, k, s, p)
+        # the routed error sums to the output error (every window has a maximum)
+        assert ex.sum(dtype=np.int64) == e.sum(dtype=np.int64)
+        # first maximum in scan order (ties): check a few windows by hand
+        for (b, i, j, c) in [(0, 0, 0, 0), (1, 1, 2, 3), (0, 3, 3, 4)]:
+            win = [(r, q) for r in range(k) for q in range(k)
+                   if 0 <= i * s + r - p < 9 and 0 <= j * s + q - p < 8]
+            vals = [x[b, i * s + r - p, j * s + q - p, c] for r, q in win]
+            r, q = win[int(np.argmax(vals))]
+            assert a[b, i, j, c] == r * k + q
+
+
+def test_mse_grad_exact_rationals():
+    g = S.rng(71)
+    z = S.int8_uniform(g, (2, 7, 5, 6))
+    lab = g.integers(0, 6, size=(2, 7, 5)).astype(np.uint8)
+    lab[0, 0, 0] = 255     # no target at this pixel
+    s_z = 3.0 * 2.0 ** -9
+    E, s = O.mse_grad(z, s_z, lab)
+    sz = Fr(s_z)
+    vals = [[(int(z[idx + (c,)]) * sz - (1 if lab[idx] == c else 0)) for c in range(6)]
+            for idx in np.ndindex(2, 7, 5)]
+    M = max(abs(v) for row in vals for v in row)
+    want = np.array([[clip(rhu_exact(v / M * 128), 8) for v in row] for row in vals])
+    d = np.abs(want - E.reshape(-1, 6))
+    assert d.max() <= 1 and (d > 0).mean() < 1e-3
+    assert s == float(M) * 2 ** -7
+
+
+def test_dgrad_exceeds_int32_and_is_exact():
+    # 3x3 image, 7x7 kernel, pad 3: every one of the 9 output pixels reaches every
+    # input pixel, so dx = 9 * k * 127^2 in closed form (beyond 2^31 for k = 20000)
+    cv = O.Conv(1, 3, 3, 2, 20000, 7, 7, 1, 3)
+    e = np.full((1, 3, 3, 20000), 127, np.int8)
+    w = np.full((20000, 7, 7, 2), 127, np.int8)
+    w[..., 1] = -127
+    dx = O.conv_dgrad(cv, e, w)
+    assert (dx[..., 0] == 9 * 20000 * 16129).all() and (dx[..., 1] == -9 * 20000 * 16129).all()
