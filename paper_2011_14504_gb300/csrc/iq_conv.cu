@@ -424,6 +424,8 @@ extern "C" iq_status iq_conv_dgrad_workspace_size(const iq_conv_desc* d, size_t*
     cur.take<int64_t>((size_t)d->n * d->h * d->w * d->c);   // int32, or int64 when wide
     cur.take<char>(requant_ws_bytes());
     cur.take<double>(1);
+    bn_stats_carve(cur, d->c);
+    cur.take<char>(conv_dgrad_tc_ws_bytes(d));
     *bytes = cur.off + 256;
     return IQ_OK;
 }
@@ -434,6 +436,7 @@ extern "C" iq_status iq_conv_wgrad_workspace_size(const iq_conv_desc* d, size_t*
     cur.take<int64_t>((size_t)d->k * d->r * d->s * (d->c / d->groups));
     cur.take<char>(requant_ws_bytes());
     cur.take<double>(1);
+    cur.take<char>(conv_wgrad_tc_ws_bytes(d));
     *bytes = cur.off + 256;
     return IQ_OK;
 }
@@ -510,30 +513,59 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     int64_t* accw = cur.take<int64_t>((size_t)d->n * d->h * d->w * d->c);
     void* rq = cur.take<char>(requant_ws_bytes());
     double* s_in = cur.take<double>(1);
+    BnStats stats = bn_stats_carve(cur, d->c);
+    void* tcws = cur.take<char>(conv_dgrad_tc_ws_bytes(d));
+    const int64_t total = (int64_t)d->n * d->h * d->w * d->c;
+    unsigned long long* cell = (unsigned long long*)rq;
+    k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, -7, s_in);
+    IQ_LAUNCH_CHECK();
+    int32_t* acc = acc_out ? acc_out : reinterpret_cast<int32_t*>(accw);
+    // tensor-core path: stride 1, as a forward pass over the errors
+    if (conv_dgrad_tc_supported(d)) {
+        bool done = false;
+        iq_status r;
+        if (wide) {
+            IQ_CUDA_CHECK(cudaMemsetAsync(accw, 0, sizeof(int64_t) * total, st));
+            r = conv_dgrad_tc(d, e, w, nullptr, (long long*)accw, nullptr, nullptr, nullptr, tcws,
+                              st, &done);
+            if (r != IQ_OK) return r;
+            if (done)
+                return requant_int(accw, IQ_I64, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
+                                   s_dx, rq, st);
+        } else {
+            r = bn_stats_init(stats, d->c, st);
+            if (r != IQ_OK) return r;
+            r = conv_dgrad_tc(d, e, w, acc, nullptr, stats.s1, stats.hi, stats.lo, tcws, st, &done);
+            if (r != IQ_OK) return r;
+            if (done) {
+                IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
+                k_max_from_stats<<<1, 1024, 0, st>>>(stats.hi, stats.lo, d->c, 0, cell);
+                IQ_LAUNCH_CHECK();
+                return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx,
+                                     IQ_I8, s_dx, rq, st);
+            }
+        }
+    }
     int64_t wn = (int64_t)d->k * d->r * d->s * cp.Cg;
     k_transpose_w<<<grid_for(wn), kThreads, 0, st>>>(w, wt, d->k, d->r, d->s, cp.Cg, d->groups);
     IQ_LAUNCH_CHECK();
-    unsigned long long* cell = (unsigned long long*)rq;
     IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
     cp.M = (int64_t)d->n * d->h * d->w;
     cp.ncols = cp.Cg;
     cp.kin = (int)roundup(cp.Kg, BK);
     dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
-    k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, -7, s_in);
-    IQ_LAUNCH_CHECK();
     if (wide) {
         k_conv_simt<OP_DGRAD, true><<<grid, 256, 0, st>>>(cp, e, wt, nullptr, (long long*)accw,
                                                           nullptr, nullptr, nullptr, cell);
         IQ_LAUNCH_CHECK();
-        return requant_apply(accw, IQ_I64, cp.M * d->c, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx,
-                             IQ_I8, s_dx, rq, st);
+        return requant_apply(accw, IQ_I64, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
+                             s_dx, rq, st);
     }
-    int32_t* acc = acc_out ? acc_out : reinterpret_cast<int32_t*>(accw);
     k_conv_simt<OP_DGRAD, false><<<grid, 256, 0, st>>>(cp, e, wt, acc, nullptr, nullptr, nullptr,
                                                        nullptr, cell);
     IQ_LAUNCH_CHECK();
-    return requant_apply(acc, IQ_I32, cp.M * d->c, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
-                         s_dx, rq, st);
+    return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8, s_dx, rq,
+                         st);
 }
 
 extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
@@ -555,8 +587,20 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
     int64_t* gw = cur.take<int64_t>((size_t)gn);
     void* rq = cur.take<char>(requant_ws_bytes());
     double* s_in = cur.take<double>(1);
+    void* tcws = cur.take<char>(conv_wgrad_tc_ws_bytes(d));
     int64_t* G = g_acc_out ? g_acc_out : gw;
     IQ_CUDA_CHECK(cudaMemsetAsync(G, 0, sizeof(int64_t) * gn, st));
+    k_scale_mul<<<1, 1, 0, st>>>(s_e, s_x, s_in);
+    IQ_LAUNCH_CHECK();
+    {
+        bool done = false;
+        iq_status r = conv_wgrad_tc(d, e, x, (long long*)G, tcws, st, &done);
+        if (r != IQ_OK) return r;
+        if (done)
+            return requant_int(G, IQ_I64, gn, s_in, 8,
+                               gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2, seed, layer, step,
+                               0, g, IQ_I8, s_g, rq, st);
+    }
     cp.M = cp.Kg;
     cp.ncols = d->r * d->s * cp.Cg;
     int64_t tiles = ((cp.M + BM - 1) / BM) * ((cp.ncols + BN - 1) / BN) * cp.G;
@@ -569,10 +613,8 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
     cp.nsplit = (int)((cp.npq + cp.chunk - 1) / cp.chunk);
     dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN),
               (unsigned)(cp.G * cp.nsplit));
-    k_conv_simt<OP_WGRAD, false><<<grid, 256, 0, st>>>(cp, e, x, nullptr, (long long*)G, nullptr, nullptr,
-                                                nullptr, nullptr);
-    IQ_LAUNCH_CHECK();
-    k_scale_mul<<<1, 1, 0, st>>>(s_e, s_x, s_in);
+    k_conv_simt<OP_WGRAD, false><<<grid, 256, 0, st>>>(cp, e, x, nullptr, (long long*)G, nullptr,
+                                                       nullptr, nullptr, nullptr);
     IQ_LAUNCH_CHECK();
     return requant_int(G, IQ_I64, gn, s_in, 8, gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2,
                        seed, layer, step, 0, g, IQ_I8, s_g, rq, st);

@@ -1,65 +1,78 @@
-// iq_conv_tc.cu -- the 8-bit convolution on the 5th-generation tensor cores (tcgen05).
+// iq_conv_tc.cu -- the 8-bit convolutions on the 5th-generation tensor cores (tcgen05).
 //
 // sm_103a has no integer UMMA (`tcgen05.mma .kind::i8` is rejected for this target), so
-// the codes travel as fp16 "carriers": every int8 code is exactly representable in fp16,
-// every product |a b| <= 127^2 is exact, and fp32 accumulation of at most 1024 such
-// products stays below 2^24 and is therefore exact.  The K loop is cut into chunks of
-// 1024 (16 k-blocks of 64); each chunk accumulates in its own fp32 TMEM buffer and the
-// epilogue folds it into int32 registers, so the result is the exact int32 convolution.
+// the codes travel as fp16 "carriers": every int8 code is exact in fp16, every product
+// |a b| <= 127^2 is exact, and fp32 accumulation of at most 1024 such products stays
+// below 2^24 and is therefore exact.  The K loop is cut into chunks of 16 k-blocks
+// (1024 products); the epilogue folds every fp32 chunk into an int32 running sum kept in
+// TMEM, so the result is the exact integer convolution.
 //
-// Implicit GEMM: D[M x N] = A[M x K] B[N x K]^T with M = N*P*Q output pixels,
-// N = output channels, K = R*S*C taps x channels.  One CTA computes a 128 x 128 tile.
-//   warps 0-3  producers: thread t gathers A row t (one output pixel) for each k-block
-//              (64 int8 codes, 16-byte loads, zero outside the image), widens them to fp16
-//              and stores them in the 128-byte-swizzled K-major UMMA layout; thread 0 also
-//              issues the TMA load of the weight tile (pre-widened to fp16 once per call).
-//   warp 8     allocates TMEM; lane 0 issues tcgen05.mma (M=128, N=128, K=16) and commits.
-//   warps 4-7  epilogue: TMEM -> registers (fp32 -> int32 fold per chunk), then the tile
-//              goes through shared memory for per-channel sum/max/min and coalesced stores.
-// All mbarrier waits are bounded (about one second); on expiry the CTA records an error
-// word, drains what it issued and returns.
+// One kernel, two operand layouts:
+//   FWD   (forward, and the stride-1 data gradient as a forward pass over the errors with
+//          flipped, transposed weights): D[M x N] = A[M x K] B[N x K]^T, M = output pixels,
+//          N = output channels, K = taps x channels.  A is gathered per output pixel
+//          (K-major), B (fp16 weights, widened once per call) arrives by TMA.
+//   WGRAD (weight gradient): D[Kout x RSC] = sum over pixels of E^T X, both operands
+//          MN-major (channels contiguous), gathered per pixel.
+// Tile 128 x 256 x 64, 4 shared-memory stages.  Warps 0-3 gather / widen / store the
+// operands, warp 8 allocates TMEM and issues tcgen05.mma (M=128, N=256, K=16), warps 4-7
+// fold the chunks and run the epilogue: either int32 stores plus per-channel sum / max /
+// min, or int64 atomic adds (weight gradients and split reductions).
+// Every mbarrier wait is bounded (about one second); on expiry the CTA records an error
+// word, drains what it issued and returns, and later CTAs of the launch exit at once.
 #include "iq_conv_tc.cuh"
 #include "iq_tc_ptx.cuh"
 
 #include <climits>
+#include <cstring>
 #include <cudaTypedefs.h>
 
 namespace iq {
 
 namespace {
 
-constexpr int TC_BM = 128;
-constexpr int TC_BN = 128;
-constexpr int TC_BK = 64;                  // fp16 elements per k-block = 128 bytes
-constexpr int TC_STAGES = 4;
-constexpr int TC_CHUNK_KB = 16;            // 16 k-blocks = 1024 products per fp32 chunk
-constexpr int TC_A_BYTES = TC_BM * 128;    // 16 KB
-constexpr int TC_B_BYTES = TC_BN * 128;    // 16 KB
-constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
-constexpr int TC_THREADS = 288;
-constexpr int TC_TMEM_COLS = 2 * TC_BN;    // two fp32 chunk buffers
-constexpr int TC_SMEM = TC_STAGES * TC_STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
-static_assert(TC_BM * (TC_BN + 1) * 4 <= TC_STAGES * TC_STAGE_BYTES, "epilogue tile fits");
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = 64;                    // fp16 elements per k-block = 128 bytes
+constexpr int STAGES = 4;
+constexpr int CHUNK_KB = 16;              // 1024 products per fp32 chunk
+constexpr int A_BYTES = BM * 128;         // 16 KB
+constexpr int B_BYTES = BN * 128;         // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int THREADS = 288;
+constexpr int TMEM_COLS = 512;            // [0,256) fp32 chunk, [256,512) int32 running sum
+constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+constexpr int TILE_LD = BN + 1;           // epilogue tile row pitch (int32)
+static_assert(BM * TILE_LD * 4 <= STAGES * STAGE_BYTES, "epilogue tile fits");
 
-struct TcConv {
+enum { MODE_FWD = 0, MODE_WGRAD = 1 };
+enum { OUT_STATS = 0, OUT_ATOMIC64 = 1 };
+
+struct TcP {
+    int mode, out;
+    // geometry of the convolution whose operands are gathered
     int N, H, W, C, K, R, S, sh, sw, ph, pw, dh, dw, P, Q;
-    int64_t M;
-    int kdim;     // R*S*C
-    int kpad;     // kdim rounded up to 64
-    int nkb;      // kpad / 64
-    int tap_mode; // C % 64 == 0: every k-block lies inside one tap
+    int cstride;     // FWD: channel stride of x (>= C) and channel offset of the slice
+    int cofs;
+    int64_t M;       // GEMM rows
+    int ncols;       // GEMM columns
+    int kdim, kpad;  // FWD: R*S*C and rounded to 64
+    int tap_mode;    // FWD: C % 64 == 0
+    int nkb_total;   // k-blocks of the whole reduction
+    int kb_per_split;
+    int64_t npq;     // WGRAD: reduction length N*P*Q
 };
 
 struct Bars {
-    uint64_t full_a[TC_STAGES];
-    uint64_t full_b[TC_STAGES];
-    uint64_t empty[TC_STAGES];
-    uint64_t accf[2];
-    uint64_t acce[2];
+    uint64_t full_a[STAGES];
+    uint64_t full_b[STAGES];
+    uint64_t empty[STAGES];
+    uint64_t accf;
+    uint64_t acce;
     uint64_t done;
     uint32_t tmem_base;
     int abort;
-    int never;   // stays 0: the abort word of the drain waits, which must not short-cut
+    int never;
 };
 
 __device__ __forceinline__ void record_abort(Bars* b, int* err, int code) {
@@ -67,29 +80,29 @@ __device__ __forceinline__ void record_abort(Bars* b, int* err, int code) {
     if (err) atomicExch(err, code);
 }
 
-// 64 consecutive K-elements (k-block kb) of A row (n, pp, qq), as 16 words of int8.
-__device__ __forceinline__ void gather_a(const TcConv& p, const int8_t* __restrict__ x, bool valid,
-                                         int n, int pp, int qq, int kb, uint32_t (&w)[16]) {
+// ---------------------------------------------------------------- FWD gather (K-major A)
+
+__device__ __forceinline__ void gather_fwd(const TcP& p, const int8_t* __restrict__ x, bool valid,
+                                           int n, int pp, int qq, int kb, uint32_t (&w)[16]) {
 #pragma unroll
     for (int i = 0; i < 16; i++) w[i] = 0;
-    if (!valid) return;
-    const int kpos = kb * TC_BK;
+    if (!valid || kb >= p.nkb_total) return;
+    const int kpos = kb * BK;
     if (p.tap_mode) {
         const int tap = kpos / p.C;
         const int c0 = kpos - tap * p.C;
-        const int r = tap / p.S, s = tap - (tap / p.S) * p.S;
+        const int r = tap / p.S, s = tap - r * p.S;
         const int hh = pp * p.sh + r * p.dh - p.ph;
         const int ww = qq * p.sw + s * p.dw - p.pw;
         if (hh < 0 || hh >= p.H || ww < 0 || ww >= p.W) return;
         const uint4* src = reinterpret_cast<const uint4*>(
-            x + (((int64_t)n * p.H + hh) * p.W + ww) * p.C + c0);
+            x + (((int64_t)n * p.H + hh) * p.W + ww) * p.cstride + p.cofs + c0);
 #pragma unroll
         for (int i = 0; i < 4; i++) {
             uint4 v = __ldg(src + i);
             w[4 * i + 0] = v.x; w[4 * i + 1] = v.y; w[4 * i + 2] = v.z; w[4 * i + 3] = v.w;
         }
     } else {
-        // C % 4 == 0: each 4-code word holds 4 channels of one tap
         int tap = kpos / p.C;
         int c = kpos - tap * p.C;
 #pragma unroll
@@ -100,7 +113,7 @@ __device__ __forceinline__ void gather_a(const TcConv& p, const int8_t* __restri
                 const int ww = qq * p.sw + s * p.dw - p.pw;
                 if (hh >= 0 && hh < p.H && ww >= 0 && ww < p.W)
                     w[i] = __ldg(reinterpret_cast<const uint32_t*>(
-                        x + (((int64_t)n * p.H + hh) * p.W + ww) * p.C + c));
+                        x + (((int64_t)n * p.H + hh) * p.W + ww) * p.cstride + p.cofs + c));
             }
             c += 4;
             if (c == p.C) { c = 0; tap++; }
@@ -108,43 +121,150 @@ __device__ __forceinline__ void gather_a(const TcConv& p, const int8_t* __restri
     }
 }
 
-__global__ void __launch_bounds__(TC_THREADS, 1)
-    k_conv_fwd_tc(const __grid_constant__ CUtensorMap wmap, TcConv p,
-                  const int8_t* __restrict__ x, int32_t* __restrict__ acc,
-                  unsigned long long* __restrict__ s1, int* __restrict__ hi_c,
-                  int* __restrict__ lo_c, int* __restrict__ err) {
+// K-major 128-byte-swizzled row store of 64 fp16 (from 64 int8 codes)
+__device__ __forceinline__ void store_kmajor_row(uint8_t* tile, int row, const uint32_t (&w)[16]) {
+    uint8_t* dst = tile + row * 128;
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+        uint32_t o0, o1, o2, o3;
+        tc::i8x4_to_f16x4(w[2 * j], o0, o1);
+        tc::i8x4_to_f16x4(w[2 * j + 1], o2, o3);
+        *reinterpret_cast<uint4*>(dst + ((j ^ (row & 7)) << 4)) = make_uint4(o0, o1, o2, o3);
+    }
+}
+
+// ---------------------------------------------------------------- WGRAD gather (MN-major)
+// Thread t of the producers owns reduction row j = t/2 of the k-block and half h = t%2:
+// A chunks (16 channels each) 4h..4h+3 of E[npq][m0 + 0..127] and B blocks 2h, 2h+1
+// (64 consecutive RSC columns each, inside one tap since C % 64 == 0).
+
+struct WgRow {
+    bool valid;
+    int n, pp, qq;
+};
+
+__device__ __forceinline__ WgRow wg_row(const TcP& p, int64_t j) {
+    WgRow r;
+    r.valid = j < p.npq;
+    r.n = r.pp = r.qq = 0;
+    if (r.valid) {
+        const int64_t pq = (int64_t)p.P * p.Q;
+        r.n = (int)(j / pq);
+        const int64_t rem = j - (int64_t)r.n * pq;
+        r.pp = (int)(rem / p.Q);
+        r.qq = (int)(rem - (int64_t)r.pp * p.Q);
+    }
+    return r;
+}
+
+__device__ __forceinline__ void gather_wgrad(const TcP& p, const int8_t* __restrict__ e,
+                                             const int8_t* __restrict__ x, int64_t m0, int n0,
+                                             const WgRow& rw, int h, uint4 (&a)[4], uint4 (&b)[8]) {
+#pragma unroll
+    for (int i = 0; i < 4; i++) a[i] = make_uint4(0, 0, 0, 0);
+#pragma unroll
+    for (int i = 0; i < 8; i++) b[i] = make_uint4(0, 0, 0, 0);
+    if (!rw.valid) return;
+    const int64_t pix = ((int64_t)rw.n * p.P + rw.pp) * p.Q + rw.qq;
+    // A: E[pix][m0 + 64h .. m0 + 64h + 63]; K_out % 16 == 0 so a chunk is all in or all out
+    const int8_t* erow = e + pix * p.K;
+#pragma unroll
+    for (int i = 0; i < 4; i++) {
+        const int64_t m = m0 + 64 * h + 16 * i;
+        if (m < p.M) a[i] = __ldg(reinterpret_cast<const uint4*>(erow + m));
+    }
+#pragma unroll
+    for (int bb = 0; bb < 2; bb++) {
+        const int col = n0 + 64 * (2 * h + bb);
+        if (col >= p.ncols) continue;
+        const int tap = col / p.C;
+        const int c0 = col - tap * p.C;
+        const int r = tap / p.S, s = tap - r * p.S;
+        const int hh = rw.pp * p.sh + r * p.dh - p.ph;
+        const int ww = rw.qq * p.sw + s * p.dw - p.pw;
+        if (hh < 0 || hh >= p.H || ww < 0 || ww >= p.W) continue;
+        const uint4* src = reinterpret_cast<const uint4*>(
+            x + (((int64_t)rw.n * p.H + hh) * p.W + ww) * p.C + c0);
+#pragma unroll
+        for (int i = 0; i < 4; i++) b[4 * bb + i] = __ldg(src + i);
+    }
+}
+
+// MN-major 128-byte-swizzled layout: atoms of 8 K-rows x 64 MN-elements (1024 bytes);
+// K-groups of 8 rows at stride 1024 (SBO), 64-wide MN blocks at stride 8192 (LBO).
+__device__ __forceinline__ void store_mnmajor_chunk(uint8_t* tile, int j, int mchunk,
+                                                    uint32_t w0, uint32_t w1, uint32_t w2,
+                                                    uint32_t w3) {
+    // mchunk indexes 16-element groups along MN; 16 int8 -> 2 x 16-byte fp16 chunks
+    const int mb = mchunk >> 2;                 // 64-element block
+    const int c8 = (mchunk & 3) * 2;            // first 8-element chunk within the 128-byte row
+    uint8_t* atom = tile + mb * 8192 + (j >> 3) * 1024 + (j & 7) * 128;
+    uint32_t o0, o1, o2, o3, o4, o5, o6, o7;
+    tc::i8x4_to_f16x4(w0, o0, o1);
+    tc::i8x4_to_f16x4(w1, o2, o3);
+    tc::i8x4_to_f16x4(w2, o4, o5);
+    tc::i8x4_to_f16x4(w3, o6, o7);
+    *reinterpret_cast<uint4*>(atom + ((c8 ^ (j & 7)) << 4)) = make_uint4(o0, o1, o2, o3);
+    *reinterpret_cast<uint4*>(atom + (((c8 + 1) ^ (j & 7)) << 4)) = make_uint4(o4, o5, o6, o7);
+}
+
+__device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFF);
+    d |= (uint64_t)(8192 >> 4) << 16;   // LBO: stride between 64-element MN blocks
+    d |= (uint64_t)(1024 >> 4) << 32;   // SBO: stride between 8-row K groups
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool mn_major) {
+    return (1u << 4) | ((mn_major ? 1u : 0u) << 15) | ((mn_major ? 1u : 0u) << 16) |
+           ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// ---------------------------------------------------------------- the kernel
+
+__global__ void __launch_bounds__(THREADS, 1)
+    k_conv_tc(const __grid_constant__ CUtensorMap wmap, TcP p, const int8_t* __restrict__ xa,
+              const int8_t* __restrict__ xb, int32_t* __restrict__ out32,
+              long long* __restrict__ out64, unsigned long long* __restrict__ s1,
+              int* __restrict__ hi_c, int* __restrict__ lo_c, int* __restrict__ err) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    Bars* bars = reinterpret_cast<Bars*>(smem + TC_STAGES * TC_STAGE_BYTES);
+    Bars* bars = reinterpret_cast<Bars*>(smem + STAGES * STAGE_BYTES);
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
-    // a CTA that timed out earlier in this launch makes the rest leave at once
-    if (*reinterpret_cast<volatile int*>(err) != 0) return;
-    const int64_t m0 = (int64_t)blockIdx.x * TC_BM;
-    const int n0 = blockIdx.y * TC_BN;
-    const int nkb = p.nkb;
-    const int nchunks = (nkb + TC_CHUNK_KB - 1) / TC_CHUNK_KB;
+    // a CTA that timed out earlier in this launch makes the rest leave at once; one
+    // thread reads the word so that the whole CTA takes the same branch
+    if (__syncthreads_or(tid == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    const int64_t m0 = (int64_t)blockIdx.x * BM;
+    const int n0 = blockIdx.y * BN;
+    const int kb0 = blockIdx.z * p.kb_per_split;
+    int nkb = p.nkb_total - kb0;
+    if (nkb > p.kb_per_split) nkb = p.kb_per_split;
+    if (nkb <= 0) return;
+    const int nchunks = (nkb + CHUNK_KB - 1) / CHUNK_KB;
+    const bool wg = p.mode == MODE_WGRAD;
 
     if (tid == 0) {
-        for (int s = 0; s < TC_STAGES; s++) {
+        for (int s = 0; s < STAGES; s++) {
             tc::mbar_init(&bars->full_a[s], 128);
             tc::mbar_init(&bars->full_b[s], 1);
             tc::mbar_init(&bars->empty[s], 1);
         }
-        for (int b = 0; b < 2; b++) {
-            tc::mbar_init(&bars->accf[b], 1);
-            tc::mbar_init(&bars->acce[b], 128);
-        }
+        tc::mbar_init(&bars->accf, 1);
+        tc::mbar_init(&bars->acce, 128);
         tc::mbar_init(&bars->done, 1);
         bars->abort = 0;
         bars->never = 0;
         tc::mbar_fence_init();
-        tc::tma_prefetch_desc(&wmap);
+        if (!wg) tc::tma_prefetch_desc(&wmap);
     }
     if (warp == 8) {
-        tc::tmem_alloc(&bars->tmem_base, TC_TMEM_COLS);
+        tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
         tc::tmem_relinquish();
     }
     tc::tc_fence_before();
@@ -154,141 +274,193 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     volatile int* abort_flag = &bars->abort;
 
     if (warp < 4) {
-        // ------------------------------------------------ producers
-        const int row = tid;
-        const int64_t m = m0 + row;
-        const bool valid = m < p.M;
-        int n = 0, pp = 0, qq = 0;
-        if (valid) {
-            const int64_t pq = (int64_t)p.P * p.Q;
-            n = (int)(m / pq);
-            const int64_t rem = m - (int64_t)n * pq;
-            pp = (int)(rem / p.Q);
-            qq = (int)(rem - (int64_t)pp * p.Q);
-        }
-        uint32_t cur[16], nxt[16];
-        gather_a(p, x, valid, n, pp, qq, 0, cur);
+        // ================================================ producers
         int issued_b = 0;
-        for (int kb = 0; kb < nkb; kb++) {
-            const int s = kb % TC_STAGES;
-            const uint32_t it = (uint32_t)(kb / TC_STAGES);
-            if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
-                record_abort(bars, err, 1);
-                break;
+        if (!wg) {
+            const int row = tid;
+            const int64_t m = m0 + row;
+            const bool valid = m < p.M;
+            int n = 0, pp = 0, qq = 0;
+            if (valid) {
+                const int64_t pq = (int64_t)p.P * p.Q;
+                n = (int)(m / pq);
+                const int64_t rem = m - (int64_t)n * pq;
+                pp = (int)(rem / p.Q);
+                qq = (int)(rem - (int64_t)pp * p.Q);
             }
-            uint8_t* a_tile = smem + s * TC_STAGE_BYTES;
-            uint8_t* b_tile = a_tile + TC_A_BYTES;
-            if (tid == 0) {
-                tc::mbar_expect_tx(&bars->full_b[s], TC_B_BYTES);
-                tc::tma_load_2d(b_tile, &wmap, &bars->full_b[s], kb * TC_BK, n0);
-                tc::mbar_arrive(&bars->full_b[s]);
-                issued_b = kb + 1;
-            }
-            if (kb + 1 < nkb) gather_a(p, x, valid, n, pp, qq, kb + 1, nxt);
-            uint8_t* dst_row = a_tile + row * 128;
+            uint32_t c0[16], c1[16], c2[16];
+            gather_fwd(p, xa, valid, n, pp, qq, kb0, c0);
+            gather_fwd(p, xa, valid, n, pp, qq, kb0 + 1, c1);
+            for (int kb = 0; kb < nkb; kb++) {
+                const int s = kb % STAGES;
+                const uint32_t it = (uint32_t)(kb / STAGES);
+                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                    record_abort(bars, err, 1);
+                    break;
+                }
+                uint8_t* a_tile = smem + s * STAGE_BYTES;
+                if (tid == 0) {
+                    tc::mbar_expect_tx(&bars->full_b[s], B_BYTES);
+                    tc::tma_load_2d(a_tile + A_BYTES, &wmap, &bars->full_b[s], (kb0 + kb) * BK, n0);
+                    tc::mbar_arrive(&bars->full_b[s]);
+                    issued_b = kb + 1;
+                }
+                if (kb + 2 < nkb) gather_fwd(p, xa, valid, n, pp, qq, kb0 + kb + 2, c2);
+                store_kmajor_row(a_tile, row, c0);
+                tc::fence_proxy_async_smem();
+                tc::mbar_arrive(&bars->full_a[s]);
 #pragma unroll
-            for (int j = 0; j < 8; j++) {
-                uint32_t o0, o1, o2, o3;
-                tc::i8x4_to_f16x4(cur[2 * j], o0, o1);
-                tc::i8x4_to_f16x4(cur[2 * j + 1], o2, o3);
-                *reinterpret_cast<uint4*>(dst_row + ((j ^ (row & 7)) << 4)) =
-                    make_uint4(o0, o1, o2, o3);
+                for (int i = 0; i < 16; i++) { c0[i] = c1[i]; c1[i] = c2[i]; }
             }
-            tc::fence_proxy_async_smem();
-            tc::mbar_arrive(&bars->full_a[s]);
+        } else {
+            const int j = tid >> 1, h = tid & 1;
+            uint4 a0[4], b0[8], a1[4], b1[8];
+            WgRow r0 = wg_row(p, (int64_t)kb0 * BK + j);
+            gather_wgrad(p, xa, xb, m0, n0, r0, h, a0, b0);
+            for (int kb = 0; kb < nkb; kb++) {
+                const int s = kb % STAGES;
+                const uint32_t it = (uint32_t)(kb / STAGES);
+                if (kb + 1 < nkb) {
+                    WgRow r1 = wg_row(p, (int64_t)(kb0 + kb + 1) * BK + j);
+                    gather_wgrad(p, xa, xb, m0, n0, r1, h, a1, b1);
+                }
+                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                    record_abort(bars, err, 1);
+                    break;
+                }
+                uint8_t* a_tile = smem + s * STAGE_BYTES;
+                uint8_t* b_tile = a_tile + A_BYTES;
 #pragma unroll
-            for (int i = 0; i < 16; i++) cur[i] = nxt[i];
+                for (int i = 0; i < 4; i++)
+                    store_mnmajor_chunk(a_tile, j, 4 * h + i, a0[i].x, a0[i].y, a0[i].z, a0[i].w);
+#pragma unroll
+                for (int i = 0; i < 8; i++)
+                    store_mnmajor_chunk(b_tile, j, 8 * h + i, b0[i].x, b0[i].y, b0[i].z, b0[i].w);
+                tc::fence_proxy_async_smem();
+                tc::mbar_arrive(&bars->full_a[s]);
+                if (tid == 0) tc::mbar_arrive(&bars->full_b[s]);
+#pragma unroll
+                for (int i = 0; i < 4; i++) a0[i] = a1[i];
+#pragma unroll
+                for (int i = 0; i < 8; i++) b0[i] = b1[i];
+            }
         }
-        if (tid == 0 && *abort_flag) {
-            // let the weight tiles already requested land before the CTA leaves
-            for (int kb = (issued_b > TC_STAGES ? issued_b - TC_STAGES : 0); kb < issued_b; kb++)
-                tc::mbar_wait(&bars->full_b[kb % TC_STAGES], (uint32_t)(kb / TC_STAGES) & 1,
+        if (!wg && tid == 0 && *abort_flag) {
+            for (int kb = (issued_b > STAGES ? issued_b - STAGES : 0); kb < issued_b; kb++)
+                tc::mbar_wait(&bars->full_b[kb % STAGES], (uint32_t)(kb / STAGES) & 1,
                               &bars->never);
         }
     } else if (warp == 8) {
-        // ------------------------------------------------ MMA issuer
+        // ================================================ MMA issuer
         if (lane == 0) {
-            const uint32_t idesc = tc::idesc_f16_f32(TC_BM, TC_BN);
+            const uint32_t idesc = idesc_f16(BM, BN, wg);
             bool ok = true;
             for (int kb = 0; kb < nkb && ok; kb++) {
-                const int s = kb % TC_STAGES;
-                const uint32_t it = (uint32_t)(kb / TC_STAGES);
-                const int chunk = kb / TC_CHUNK_KB;
-                const int buf = chunk & 1;
-                const bool first = (kb % TC_CHUNK_KB) == 0;
-                const bool last = ((kb % TC_CHUNK_KB) == TC_CHUNK_KB - 1) || kb == nkb - 1;
-                if (first && !tc::mbar_wait(&bars->acce[buf], (uint32_t)((chunk >> 1) & 1) ^ 1,
-                                            abort_flag)) { ok = false; break; }
+                const int s = kb % STAGES;
+                const uint32_t it = (uint32_t)(kb / STAGES);
+                const int chunk = kb / CHUNK_KB;
+                const bool first = (kb % CHUNK_KB) == 0;
+                const bool last = ((kb % CHUNK_KB) == CHUNK_KB - 1) || kb == nkb - 1;
+                // the fp32 buffer is free once the epilogue folded the previous chunk
+                if (first && chunk > 0 &&
+                    !tc::mbar_wait(&bars->acce, (uint32_t)(chunk - 1) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
                 if (!tc::mbar_wait(&bars->full_b[s], it & 1, abort_flag) ||
-                    !tc::mbar_wait(&bars->full_a[s], it & 1, abort_flag)) { ok = false; break; }
+                    !tc::mbar_wait(&bars->full_a[s], it & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
                 tc::tc_fence_after();
-                const uint32_t a_addr = tc::smem_u32(smem + s * TC_STAGE_BYTES);
-                const uint32_t b_addr = a_addr + TC_A_BYTES;
+                const uint32_t a_addr = tc::smem_u32(smem + s * STAGE_BYTES);
+                const uint32_t b_addr = a_addr + A_BYTES;
 #pragma unroll
-                for (int j = 0; j < TC_BK / 16; j++) {
-                    tc::umma_f16(tmem + buf * TC_BN, tc::sdesc_kmajor_sw128(a_addr + 32 * j),
-                                 tc::sdesc_kmajor_sw128(b_addr + 32 * j), idesc,
-                                 (first && j == 0) ? 0u : 1u);
+                for (int k = 0; k < BK / 16; k++) {
+                    uint64_t ad, bd;
+                    if (wg) {
+                        ad = sdesc_mnmajor_sw128(a_addr + 2 * 1024 * k);
+                        bd = sdesc_mnmajor_sw128(b_addr + 2 * 1024 * k);
+                    } else {
+                        ad = tc::sdesc_kmajor_sw128(a_addr + 32 * k);
+                        bd = tc::sdesc_kmajor_sw128(b_addr + 32 * k);
+                    }
+                    tc::umma_f16(tmem, ad, bd, idesc, (first && k == 0) ? 0u : 1u);
                 }
                 tc::umma_commit(&bars->empty[s]);
-                if (last) tc::umma_commit(&bars->accf[buf]);
+                if (last) tc::umma_commit(&bars->accf);
             }
             if (!ok) record_abort(bars, err, 2);
-            // every MMA issued must finish before TMEM is released
             tc::umma_commit(&bars->done);
             tc::mbar_wait(&bars->done, 0, &bars->never);
         }
         __syncwarp();
     } else {
-        // ------------------------------------------------ epilogue (warps 4..7)
+        // ================================================ epilogue (warps 4..7)
         const int row = tid - 128;
         const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-        int accv[TC_BN];
-#pragma unroll
-        for (int j = 0; j < TC_BN; j++) accv[j] = 0;
+        const uint32_t tD = tmem + lane_base;            // fp32 chunk, columns [0, 256)
+        const uint32_t tR = tmem + lane_base + BN;       // int32 running sum, [256, 512)
+        int* tile = reinterpret_cast<int*>(smem);
         bool ok = true;
         for (int c = 0; c < nchunks; c++) {
-            const int buf = c & 1;
-            if (!tc::mbar_wait(&bars->accf[buf], (uint32_t)(c >> 1) & 1, abort_flag)) {
+            if (!tc::mbar_wait(&bars->accf, (uint32_t)c & 1, abort_flag)) {
                 ok = false;
                 record_abort(bars, err, 3);
                 break;
             }
             tc::tc_fence_after();
-#pragma unroll
-            for (int cb = 0; cb < TC_BN / 32; cb++) {
-                uint32_t r[32];
-                tc::tmem_ld_32x32b_x32(tmem + lane_base + buf * TC_BN + cb * 32, r);
+            // after the last chunk every MMA has completed (and with it every operand
+            // write and read), so the stage buffers are free for the epilogue tile
+            const bool lastc = c == nchunks - 1;
+#pragma unroll 1
+            for (int cb = 0; cb < BN / 32; cb++) {
+                uint32_t d[32], r[32];
+                tc::tmem_ld_32x32b_x32(tD + cb * 32, d);
+                if (c > 0) tc::tmem_ld_32x32b_x32(tR + cb * 32, r);
                 tc::tmem_ld_wait();
 #pragma unroll
-                for (int i = 0; i < 32; i++) accv[cb * 32 + i] += __float2int_rn(__uint_as_float(r[i]));
-            }
-            tc::tc_fence_before();
-            tc::mbar_arrive(&bars->acce[buf]);
-        }
-        // tile -> shared memory (stage buffers are free: every MMA has completed)
-        int* tile = reinterpret_cast<int*>(smem);
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (ok && !*abort_flag) {
-#pragma unroll
-            for (int j = 0; j < TC_BN; j++) tile[row * (TC_BN + 1) + j] = accv[j];
-        }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (ok && !*abort_flag) {
-            const int rows = (int)((p.M - m0) < TC_BM ? (p.M - m0) : TC_BM);
-            const int col = row;  // one output channel per thread
-            if (n0 + col < p.K) {
-                long long sum = 0;
-                int h = INT_MIN, l = INT_MAX;
-                for (int i = 0; i < rows; i++) {
-                    int v = tile[i * (TC_BN + 1) + col];
-                    sum += v; h = max(h, v); l = min(l, v);
+                for (int i = 0; i < 32; i++) {
+                    int v = __float2int_rn(__uint_as_float(d[i]));
+                    r[i] = (uint32_t)((c > 0 ? (int)r[i] : 0) + v);
                 }
-                atomicAdd(&s1[n0 + col], (unsigned long long)sum);
-                atomicMax(&hi_c[n0 + col], h);
-                atomicMin(&lo_c[n0 + col], l);
-                for (int i = 0; i < rows; i++)
-                    acc[(m0 + i) * p.K + n0 + col] = tile[i * (TC_BN + 1) + col];
+                if (!lastc) {
+                    tc::tmem_st_32x32b_x32(tR + cb * 32, r);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; i++) tile[row * TILE_LD + cb * 32 + i] = (int)r[i];
+                }
+            }
+            if (!lastc) tc::tmem_st_wait();
+            tc::tc_fence_before();
+            tc::mbar_arrive(&bars->acce);
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (ok && !*abort_flag) {
+            const int rows = (int)((p.M - m0) < BM ? (p.M - m0) : BM);
+            for (int col = row; col < BN; col += 128) {
+                const int gcol = n0 + col;
+                if (gcol >= p.ncols) continue;
+                if (p.out == OUT_STATS) {
+                    long long sum = 0;
+                    int h = INT_MIN, l = INT_MAX;
+                    for (int i = 0; i < rows; i++) {
+                        int v = tile[i * TILE_LD + col];
+                        sum += v; h = max(h, v); l = min(l, v);
+                        out32[(m0 + i) * p.ncols + gcol] = v;
+                    }
+                    atomicAdd(&s1[gcol], (unsigned long long)sum);
+                    atomicMax(&hi_c[gcol], h);
+                    atomicMin(&lo_c[gcol], l);
+                } else {
+                    for (int i = 0; i < rows; i++) {
+                        int v = tile[i * TILE_LD + col];
+                        if (v)
+                            atomicAdd(reinterpret_cast<unsigned long long*>(
+                                          &out64[(m0 + i) * p.ncols + gcol]),
+                                      (unsigned long long)(long long)v);
+                    }
+                }
             }
         }
     }
@@ -296,7 +468,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     __syncthreads();
     if (warp == 8) {
         tc::tc_fence_after();
-        tc::tmem_dealloc(tmem, TC_TMEM_COLS);
+        tc::tmem_dealloc(tmem, TMEM_COLS);
     }
 }
 
@@ -308,6 +480,25 @@ __global__ void k_widen_weights(const int8_t* __restrict__ w, __half* __restrict
          i += (int64_t)gridDim.x * blockDim.x) {
         int k = (int)(i / kpad), j = (int)(i - (int64_t)k * kpad);
         wf[i] = __int2half_rn(j < kdim ? (int)w[(int64_t)k * kdim + j] : 0);
+    }
+}
+
+// data-gradient weights: w[K][R][S][C] -> [C][R][S][kc] flipped in r and s, fp16, for the
+// K-channel slice [kofs, kofs + kc); rows of kpad >= R*S*kc
+__global__ void k_widen_weights_dgrad(const int8_t* __restrict__ w, __half* __restrict__ wf, int K,
+                                      int R, int S, int C, int kofs, int kc, int kpad) {
+    int64_t total = (int64_t)C * kpad;
+    const int kdim = R * S * kc;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        int c = (int)(i / kpad), j = (int)(i - (int64_t)c * kpad);
+        int v = 0;
+        if (j < kdim) {
+            int k = j % kc, rs = j / kc;
+            int r = rs / S, s = rs % S;
+            v = w[(((int64_t)(kofs + k) * R + (R - 1 - r)) * S + (S - 1 - s)) * C + c];
+        }
+        wf[i] = __int2half_rn(v);
     }
 }
 
@@ -329,42 +520,77 @@ bool tc_env_disabled() {
     return e && e[0] == '1';
 }
 
+iq_status encode_weights(const __half* wf, int rows, int kpad, CUtensorMap* map) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
+    if (!enc) return IQ_ERR_UNSUPPORTED;
+    cuuint64_t gdim[2] = {(cuuint64_t)kpad, (cuuint64_t)rows};
+    cuuint64_t gstride[1] = {(cuuint64_t)kpad * 2};
+    cuuint32_t box[2] = {64, BN};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, (void*)wf, gdim, gstride, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
+}
+
+iq_status launch(const CUtensorMap& map, const TcP& p, int nsplit, const int8_t* xa,
+                 const int8_t* xb, int32_t* out32, long long* out64, unsigned long long* s1,
+                 int* hi, int* lo, int* err, cudaStream_t st) {
+    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       SMEM));
+    dim3 grid((unsigned)((p.M + BM - 1) / BM), (unsigned)((p.ncols + BN - 1) / BN),
+              (unsigned)nsplit);
+    k_conv_tc<<<grid, THREADS, SMEM, st>>>(map, p, xa, xb, out32, out64, s1, hi, lo, err);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+void fill_geom(TcP& p, const iq_conv_desc* d) {
+    p.N = d->n; p.H = d->h; p.W = d->w; p.C = d->c; p.K = d->k; p.R = d->r; p.S = d->s;
+    p.sh = d->stride_h; p.sw = d->stride_w; p.ph = d->pad_h; p.pw = d->pad_w;
+    p.dh = d->dil_h; p.dw = d->dil_w;
+    p.P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    p.Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    p.cstride = d->c;
+    p.cofs = 0;
+}
+
+// k-blocks per split so that each split's int32 running sum cannot overflow
+constexpr int MAX_KB_INT32 = 133120 / 64;   // 2080 k-blocks: 133120 * 127^2 < 2^31
+
 }  // namespace
+
+// ================================================================ forward
 
 size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d) {
     int64_t kdim = (int64_t)d->r * d->s * (d->c / d->groups);
     int64_t kpad = (kdim + 63) / 64 * 64;
-    return (size_t)(d->k * kpad * 2) + 256 + 256;
+    return (size_t)(d->k * kpad * 2) + 512;
 }
 
 bool conv_fwd_tc_supported(const iq_conv_desc* d) {
     if (tc_env_disabled()) return false;
-    if (d->groups != 1) return false;
-    if (d->c % 4) return false;
-    if (d->k % 8) return false;   // TMA row stride of the fp16 weights is 16-byte aligned anyway
-    return true;
+    return d->groups == 1 && d->c % 4 == 0 && d->k % 8 == 0;
 }
 
 iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, int32_t* acc,
                       unsigned long long* s1, int* hi, int* lo, void* ws, cudaStream_t st,
                       bool* done) {
     *done = false;
-    if (!conv_fwd_tc_supported(d)) return IQ_OK;
-    if (((uintptr_t)x & 15) != 0) return IQ_OK;
-    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
-    if (!enc) return IQ_OK;
-    TcConv p;
-    p.N = d->n; p.H = d->h; p.W = d->w; p.C = d->c; p.K = d->k; p.R = d->r; p.S = d->s;
-    p.sh = d->stride_h; p.sw = d->stride_w; p.ph = d->pad_h; p.pw = d->pad_w;
-    p.dh = d->dil_h; p.dw = d->dil_w;
-    p.P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
-    p.Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    if (!conv_fwd_tc_supported(d) || ((uintptr_t)x & 15) != 0 || !get_encode()) return IQ_OK;
+    TcP p;
+    fill_geom(p, d);
+    p.mode = MODE_FWD;
+    p.out = OUT_STATS;
     p.M = (int64_t)p.N * p.P * p.Q;
+    p.ncols = p.K;
     p.kdim = d->r * d->s * d->c;
     p.kpad = (p.kdim + 63) / 64 * 64;
-    p.nkb = p.kpad / 64;
     p.tap_mode = (d->c % 64) == 0;
-
+    p.nkb_total = p.kpad / 64;
+    p.kb_per_split = p.nkb_total;
+    p.npq = 0;
+    if (p.nkb_total > MAX_KB_INT32) return IQ_OK;   // cannot happen under the CRS bound
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     __half* wf = reinterpret_cast<__half*>(wsb);
     int* err = reinterpret_cast<int*>(wsb + (size_t)p.K * p.kpad * 2);
@@ -372,24 +598,133 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
                                                                          p.kpad);
     IQ_LAUNCH_CHECK();
     IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
-
     CUtensorMap map;
-    cuuint64_t gdim[2] = {(cuuint64_t)p.kpad, (cuuint64_t)p.K};
-    cuuint64_t gstride[1] = {(cuuint64_t)p.kpad * 2};
-    cuuint32_t box[2] = {64, TC_BN};
-    cuuint32_t estr[2] = {1, 1};
-    CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, wf, gdim, gstride, box, estr,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return IQ_ERR_CUDA;
+    iq_status r = encode_weights(wf, p.K, p.kpad, &map);
+    if (r != IQ_OK) return r;
+    r = launch(map, p, 1, x, nullptr, acc, nullptr, s1, hi, lo, err, st);
+    if (r == IQ_OK) *done = true;
+    return r;
+}
 
-    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       TC_SMEM));
-    dim3 grid((unsigned)((p.M + TC_BM - 1) / TC_BM), (unsigned)((p.K + TC_BN - 1) / TC_BN), 1);
-    k_conv_fwd_tc<<<grid, TC_THREADS, TC_SMEM, st>>>(map, p, x, acc, s1, hi, lo, err);
-    IQ_LAUNCH_CHECK();
+// ================================================================ data gradient (stride 1)
+// dx = conv(e, w') with w'[c][r][s][k] = w[k][R-1-r][S-1-s][c], pad' = dil (R-1) - pad.
+// When (K R S) 127^2 could overflow int32 the reduction is split over channel slices of e
+// whose int32 partial results are added in int64.
+
+int conv_dgrad_tc_slices(const iq_conv_desc* d) {
+    int nsl = 1;
+    while (nsl <= d->k &&
+           ((int64_t)(d->k / nsl) * d->r * d->s * 16129 >= (int64_t(1) << 31) || (d->k % nsl) ||
+            ((d->k / nsl) % 4)))
+        nsl++;
+    return nsl <= d->k ? nsl : 0;
+}
+
+size_t conv_dgrad_tc_ws_bytes(const iq_conv_desc* d) {
+    int nsl = conv_dgrad_tc_slices(d);
+    if (nsl < 1) nsl = 1;
+    int64_t kpad = ((int64_t)d->r * d->s * (d->k / nsl) + 63) / 64 * 64;
+    return (size_t)(d->c * kpad * 2) + 512;
+}
+
+bool conv_dgrad_tc_supported(const iq_conv_desc* d) {
+    if (tc_env_disabled()) return false;
+    if (d->groups != 1 || d->stride_h != 1 || d->stride_w != 1) return false;
+    if (d->k % 4 || d->c % 8) return false;
+    if (d->dil_h * (d->r - 1) < d->pad_h || d->dil_w * (d->s - 1) < d->pad_w) return false;
+    return conv_dgrad_tc_slices(d) >= 1;
+}
+
+iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w, int32_t* out32,
+                        long long* out64, unsigned long long* s1, int* hi, int* lo, void* ws,
+                        cudaStream_t st, bool* done) {
+    *done = false;
+    if (!conv_dgrad_tc_supported(d) || ((uintptr_t)e & 15) != 0 || !get_encode()) return IQ_OK;
+    const int nsl = conv_dgrad_tc_slices(d);
+    if (nsl > 1 && !out64) return IQ_OK;
+    if (nsl == 1 && !out32) return IQ_OK;
+    iq_conv_desc g = *d;   // the forward problem over the errors
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    g.h = P; g.w = Q; g.c = d->k; g.k = d->c;
+    g.pad_h = d->dil_h * (d->r - 1) - d->pad_h;
+    g.pad_w = d->dil_w * (d->s - 1) - d->pad_w;
+    const int kc = d->k / nsl;
+    TcP p;
+    fill_geom(p, &g);
+    p.C = kc;                 // channels per slice
+    p.cstride = d->k;
+    p.mode = MODE_FWD;
+    p.out = nsl == 1 ? OUT_STATS : OUT_ATOMIC64;
+    p.M = (int64_t)d->n * d->h * d->w;
+    p.ncols = d->c;
+    p.kdim = d->r * d->s * kc;
+    p.kpad = (p.kdim + 63) / 64 * 64;
+    p.tap_mode = (kc % 64) == 0;
+    p.nkb_total = p.kpad / 64;
+    p.kb_per_split = p.nkb_total;
+    p.npq = 0;
+    if (p.P != d->h || p.Q != d->w) return IQ_OK;
+    char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
+    __half* wf = reinterpret_cast<__half*>(wsb);
+    int* err = reinterpret_cast<int*>(wsb + (size_t)d->c * p.kpad * 2);
+    IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
+    for (int sl = 0; sl < nsl; sl++) {
+        k_widen_weights_dgrad<<<grid_for((int64_t)d->c * p.kpad), kThreads, 0, st>>>(
+            w, wf, d->k, d->r, d->s, d->c, sl * kc, kc, p.kpad);
+        IQ_LAUNCH_CHECK();
+        CUtensorMap map;
+        iq_status r = encode_weights(wf, d->c, p.kpad, &map);
+        if (r != IQ_OK) return r;
+        p.cofs = sl * kc;
+        r = launch(map, p, 1, e, nullptr, out32, out64, s1, hi, lo, err, st);
+        if (r != IQ_OK) return r;
+    }
     *done = true;
     return IQ_OK;
+}
+
+// ================================================================ weight gradient
+
+size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc*) { return 512; }
+
+bool conv_wgrad_tc_supported(const iq_conv_desc* d) {
+    if (tc_env_disabled()) return false;
+    return d->groups == 1 && d->c % 64 == 0 && d->k % 16 == 0;
+}
+
+// G (int64 KRSC, zeroed by the caller) += E^T im2col(x)
+iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
+                        void* ws, cudaStream_t st, bool* done) {
+    *done = false;
+    if (!conv_wgrad_tc_supported(d) || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
+    TcP p;
+    fill_geom(p, d);
+    p.mode = MODE_WGRAD;
+    p.out = OUT_ATOMIC64;
+    p.M = p.K;
+    p.ncols = p.R * p.S * p.C;
+    p.npq = (int64_t)p.N * p.P * p.Q;
+    p.kdim = 0; p.kpad = 0; p.tap_mode = 1;
+    const int64_t nkb = (p.npq + BK - 1) / BK;
+    if (nkb > INT_MAX) return IQ_OK;
+    p.nkb_total = (int)nkb;
+    const int64_t tiles = ((p.M + BM - 1) / BM) * ((p.ncols + BN - 1) / BN);
+    // enough splits to fill the GPU twice over, each split within the int32 bound
+    int64_t want = (2 * 152 + tiles - 1) / tiles;
+    int64_t kbs = (nkb + want - 1) / want;
+    if (kbs < 32) kbs = 32;
+    if (kbs > MAX_KB_INT32) kbs = MAX_KB_INT32;
+    p.kb_per_split = (int)kbs;
+    const int nsplit = (int)((nkb + kbs - 1) / kbs);
+    char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
+    int* err = reinterpret_cast<int*>(wsb);
+    IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
+    CUtensorMap dummy;
+    memset(&dummy, 0, sizeof(dummy));
+    iq_status r = launch(dummy, p, nsplit, e, x, nullptr, G, nullptr, nullptr, nullptr, err, st);
+    if (r == IQ_OK) *done = true;
+    return r;
 }
 
 }  // namespace iq

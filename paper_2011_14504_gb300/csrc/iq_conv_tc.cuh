@@ -15,4 +15,20 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
                       unsigned long long* s1, int* hi, int* lo, void* ws, cudaStream_t st,
                       bool* done);
 
+// Stride-1 data gradient as a forward pass over the errors with flipped, transposed
+// weights.  Writes int32 sums to out32 plus per-channel sum/max/min when the reduction
+// (k r s) fits int32, else adds int64 sums into out64 (zeroed by the caller).
+size_t conv_dgrad_tc_ws_bytes(const iq_conv_desc* d);
+bool conv_dgrad_tc_supported(const iq_conv_desc* d);
+int conv_dgrad_tc_slices(const iq_conv_desc* d);
+iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w, int32_t* out32,
+                        long long* out64, unsigned long long* s1, int* hi, int* lo, void* ws,
+                        cudaStream_t st, bool* done);
+
+// Weight gradient: adds the exact int64 sums into G (KRSC, zeroed by the caller).
+size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d);
+bool conv_wgrad_tc_supported(const iq_conv_desc* d);
+iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
+                        void* ws, cudaStream_t st, bool* done);
+
 }  // namespace iq

@@ -305,9 +305,10 @@ def test_bn_int_bwd(m, C, k_e2):
 TC_CASES = [
     # n, h, w, c, k, r, s, stride, pad, dil: shapes the tcgen05 kernel takes
     (2, 16, 16, 512, 256, 3, 3, 1, 1, 1),   # 5 fp32 chunks, 2 N tiles, 4 M tiles
-    (1, 29, 31, 128, 136, 3, 3, 1, 2, 2),   # ragged M and N, dilation 2
-    (3, 9, 10, 64, 72, 1, 1, 1, 0, 1),      # 1x1, ragged
-    (1, 33, 33, 256, 64, 3, 3, 2, 1, 1),    # stride 2
+    (1, 29, 31, 128, 144, 3, 3, 1, 2, 2),   # ragged M and N, dilation 2
+    (3, 9, 10, 64, 80, 1, 1, 1, 0, 1),      # 1x1, ragged
+    (1, 33, 33, 256, 64, 3, 3, 2, 1, 1),    # stride 2 (data gradient on CUDA cores)
+    (4, 40, 40, 64, 64, 3, 3, 1, 1, 1),     # weight gradient split over 100 k-blocks
 ]
 
 
@@ -328,6 +329,25 @@ def test_conv_fwd_tc_shapes(ci):
     assert np.array_equal(host(acc), want)
     wa, ws_ = O.sq_int(want, 0.01 * 2.0 ** -7, 8, True)
     assert np.array_equal(host(a).astype(np.int32), wa) and host(s_a)[0] == ws_
+    # data and weight gradients of the same shape
+    e = S.int8_uniform(g, (n, p, q, k))
+    dx = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
+    dacc = torch.empty((n, h, w, c), dtype=torch.int32, device=DEV)
+    s_dx = dscal()
+    iq.iq_conv_dgrad(d, dev(e), dscal(2e-5), dev(wq), dx, s_dx, acc_out=dacc)
+    want_d = O.conv_dgrad(cv, e, wq)
+    assert np.array_equal(host(dacc), want_d)
+    wd, wds = O.sq_int(want_d, 2e-5 * 2.0 ** -7, 8)
+    assert np.array_equal(host(dx).astype(np.int32), wd) and host(s_dx)[0] == wds
+    gq = torch.empty(wq.shape, dtype=torch.int8, device=DEV)
+    gacc = torch.empty(wq.shape, dtype=torch.int64, device=DEV)
+    s_g = dscal()
+    iq.iq_conv_wgrad(d, dev(e), dscal(2e-5), dev(x), dscal(0.01), gq, s_g, gq_mode=1, seed=4,
+                     layer=ci, step=1, g_acc_out=gacc)
+    want_g = O.conv_wgrad(cv, e, x)
+    assert np.array_equal(host(gacc), want_g)
+    wg, wgs = O.rq_int(want_g, 2e-5 * 0.01, 8, 1, 4, ci, 1, 0)
+    assert np.array_equal(host(gq).astype(np.int32), wg) and host(s_g)[0] == wgs
 
 
 @pytest.mark.parametrize("sign", [1, -1])
