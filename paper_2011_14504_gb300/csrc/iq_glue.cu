@@ -81,6 +81,38 @@ __global__ void k_maxpool_bwd(const int8_t* __restrict__ e, const uint8_t* __res
     }
 }
 
+// windows that do not overlap (k == s, no padding): each window scatters its error to
+// its first maximum; every input receives at most one error.  4 channels per thread.
+__global__ void k_maxpool_bwd_tiled(const int8_t* __restrict__ e, const uint8_t* __restrict__ arg,
+                                    int n, int h, int w, int c4, int k, int P, int Q,
+                                    int8_t* __restrict__ ex) {
+    const int64_t total = (int64_t)n * P * Q * c4;
+    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
+         o += (int64_t)gridDim.x * blockDim.x) {
+        const int cg = (int)(o % c4);
+        int64_t t = o / c4;
+        const int j = (int)(t % Q); t /= Q;
+        const int i = (int)(t % P);
+        const int b = (int)(t / P);
+        const uint32_t ev = reinterpret_cast<const uint32_t*>(e)[o];
+        const uint32_t av = reinterpret_cast<const uint32_t*>(arg)[o];
+        for (int r = 0; r < k; r++) {
+            const int hh = i * k + r;
+            if (hh >= h) break;
+            for (int q = 0; q < k; q++) {
+                const int ww = j * k + q;
+                if (ww >= w) break;
+                const uint32_t tap = (uint32_t)(r * k + q);
+                uint32_t v = 0;
+#pragma unroll
+                for (int l = 0; l < 4; l++)
+                    if (((av >> (8 * l)) & 0xffu) == tap) v |= ev & (0xffu << (8 * l));
+                reinterpret_cast<uint32_t*>(ex)[(((int64_t)b * h + hh) * w + ww) * c4 + cg] = v;
+            }
+        }
+    }
+}
+
 __global__ void k_copy_scale(const double* __restrict__ a, double* __restrict__ b) { *b = *a; }
 __global__ void k_scale_pow2(const double* __restrict__ a, int e, double* __restrict__ out) {
     *out = ldexp(*a, e);
@@ -98,69 +130,59 @@ struct UpP {
     int n, h, w, c, R, st, pad, H, W;
 };
 
-__device__ __forceinline__ int up_acc(const UpP& u, const int8_t* __restrict__ x,
-                                      const int8_t* __restrict__ wt, int b, int Ho, int Wo,
-                                      int ch) {
-    int sum = 0;
-    // i*st <= Ho + pad < i*st + R
-    int i_hi = (Ho + u.pad) / u.st;
-    int j_hi = (Wo + u.pad) / u.st;
-    for (int i = i_hi; i >= 0; i--) {
+// One block per (n, output row, 32 output columns); one thread per channel.  The input
+// rows / columns reaching an output pixel are i = (Ho + pad - r) / st for the taps r of the
+// kernel with the right residue: at most ceil(R / st) of them per dimension.
+template <bool CODES>
+__global__ void k_up_fwd(UpP u, const int8_t* __restrict__ x, const int8_t* __restrict__ wT,
+                         unsigned long long* __restrict__ amax, const RqDiv* __restrict__ dv,
+                         int k, int8_t* __restrict__ out, int32_t* __restrict__ acc_out) {
+    const int Ho = blockIdx.y % u.H;
+    const int b = blockIdx.y / u.H;
+    const int Wo0 = blockIdx.x * 32;
+    const int ch = threadIdx.x;
+    RqDiv d;
+    if (CODES) d = *dv;
+    const int64_t lim = qmax(k);
+    uint64_t mx = 0;
+    // input rows of this output row
+    int rows_i[4], rows_r[4], nr = 0;
+    for (int i = (Ho + u.pad) / u.st; i >= 0 && nr < 4; i--) {
         int r = Ho + u.pad - i * u.st;
         if (r >= u.R) break;
-        if (i >= u.h) continue;
-        for (int j = j_hi; j >= 0; j--) {
-            int t = Wo + u.pad - j * u.st;
-            if (t >= u.R) break;
-            if (j >= u.w) continue;
-            sum += (int)x[(((int64_t)b * u.h + i) * u.w + j) * u.c + ch] *
-                   (int)wt[((int64_t)ch * u.R + r) * u.R + t];
+        if (i < u.h) { rows_i[nr] = i; rows_r[nr] = r; nr++; }
+    }
+    if (ch < u.c) {
+        for (int wo = 0; wo < 32; wo++) {
+            const int Wo = Wo0 + wo;
+            if (Wo >= u.W) break;
+            int sum = 0;
+            for (int j = (Wo + u.pad) / u.st; j >= 0; j--) {
+                int t = Wo + u.pad - j * u.st;
+                if (t >= u.R) break;
+                if (j >= u.w) continue;
+                for (int a = 0; a < nr; a++)
+                    sum += (int)x[(((int64_t)b * u.h + rows_i[a]) * u.w + j) * u.c + ch] *
+                           (int)wT[((int64_t)rows_r[a] * u.R + t) * u.c + ch];
+            }
+            const int64_t o = (((int64_t)b * u.H + Ho) * u.W + Wo) * u.c + ch;
+            if (CODES) {
+                if (acc_out) acc_out[o] = sum;
+                int64_t c = 0;
+                if (d.M) {
+                    uint64_t num = ((uint64_t)((int64_t)sum + (int64_t)d.M) << k) + d.M;
+                    c = clamp64((int64_t)udiv(num, d.div) - (int64_t(1) << (k - 1)), -lim, lim);
+                }
+                out[o] = (int8_t)c;
+            } else {
+                uint64_t a = (uint64_t)(sum < 0 ? -sum : sum);
+                mx = a > mx ? a : mx;
+            }
         }
     }
-    return sum;
-}
-
-__global__ void k_up_max(UpP u, const int8_t* __restrict__ x, const int8_t* __restrict__ wt,
-                         unsigned long long* __restrict__ amax) {
-    const int64_t total = (int64_t)u.n * u.H * u.W * u.c;
-    uint64_t mx = 0;
-    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
-         o += (int64_t)gridDim.x * blockDim.x) {
-        int ch = (int)(o % u.c);
-        int64_t t = o / u.c;
-        int Wo = (int)(t % u.W); t /= u.W;
-        int Ho = (int)(t % u.H);
-        int b = (int)(t / u.H);
-        int v = up_acc(u, x, wt, b, Ho, Wo, ch);
-        uint64_t a = (uint64_t)(v < 0 ? -v : v);
-        mx = a > mx ? a : mx;
-    }
-    mx = warp_max_u64(mx);
-    if ((threadIdx.x & 31) == 0 && mx) atomicMax(amax, (unsigned long long)mx);
-}
-
-// second pass: recompute and apply SQ with the divisor prepared by the requantizer
-__global__ void k_up_codes(UpP u, const int8_t* __restrict__ x, const int8_t* __restrict__ wt,
-                           const RqDiv* __restrict__ dv, int k, int8_t* __restrict__ out,
-                           int32_t* __restrict__ acc_out) {
-    const RqDiv d = *dv;
-    const int64_t lim = qmax(k);
-    const int64_t total = (int64_t)u.n * u.H * u.W * u.c;
-    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
-         o += (int64_t)gridDim.x * blockDim.x) {
-        int ch = (int)(o % u.c);
-        int64_t t = o / u.c;
-        int Wo = (int)(t % u.W); t /= u.W;
-        int Ho = (int)(t % u.H);
-        int b = (int)(t / u.H);
-        int v = up_acc(u, x, wt, b, Ho, Wo, ch);
-        if (acc_out) acc_out[o] = v;
-        int64_t c = 0;
-        if (d.M) {
-            uint64_t num = ((uint64_t)((int64_t)v + (int64_t)d.M) << k) + d.M;
-            c = clamp64((int64_t)udiv(num, d.div) - (int64_t(1) << (k - 1)), -lim, lim);
-        }
-        out[o] = (int8_t)c;
+    if (!CODES) {
+        mx = warp_max_u64(mx);
+        if ((threadIdx.x & 31) == 0 && mx) atomicMax(amax, (unsigned long long)mx);
     }
 }
 
@@ -248,12 +270,15 @@ struct MseP {
 // extremes of z for target (t=1) and non-target (t=0) elements: [max0, min0, max1, min1]
 __global__ void k_mse_stats(const int8_t* __restrict__ z, const uint8_t* __restrict__ lab,
                             int64_t npix, int c, int* __restrict__ ext) {
-    int mx0 = INT_MIN, mn0 = INT_MAX, mx1 = INT_MIN, mn1 = INT_MAX;
+    int mx0 = INT_MIN, mn0 = INT_MAX, mx1 = INT_MAX, mn1 = INT_MAX;
+    mx1 = INT_MIN;
+    const UDiv dc = make_udiv((uint64_t)c);
     const int64_t total = npix * c;
     for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
          o += (int64_t)gridDim.x * blockDim.x) {
         int v = z[o];
-        bool tgt = lab[o / c] == (uint8_t)(o % c);
+        const int64_t px = (int64_t)udiv((uint64_t)o, dc);
+        bool tgt = lab[px] == (uint8_t)(o - px * c);
         if (tgt) { mx1 = max(mx1, v); mn1 = min(mn1, v); }
         else { mx0 = max(mx0, v); mn0 = min(mn0, v); }
     }
@@ -314,10 +339,12 @@ __global__ void k_mse_codes(const int8_t* __restrict__ z, const uint8_t* __restr
                             int8_t* __restrict__ E) {
     const MseP p = *prm;
     const int64_t lim = qmax(k);
+    const UDiv dc = make_udiv((uint64_t)c);
     const int64_t total = npix * c;
     for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
          o += (int64_t)gridDim.x * blockDim.x) {
-        bool tgt = lab[o / c] == (uint8_t)(o % c);
+        const int64_t px = (int64_t)udiv((uint64_t)o, dc);
+        bool tgt = lab[px] == (uint8_t)(o - px * c);
         long long t = p.F * (long long)z[o] + (tgt ? p.B1 : p.B0);
         E[o] = (int8_t)clamp64(t >> p.P, -lim, lim);
     }
@@ -355,8 +382,15 @@ extern "C" iq_status iq_maxpool_bwd(const int8_t* e, const double* s_e, const ui
     int64_t total = (int64_t)n * h * w * c;
     if (k <= s) {
         // windows do not overlap: every input receives at most one error, same scale
-        k_maxpool_bwd<<<grid_for(total), kThreads, 0, st>>>(e, arg, n, h, w, c, k, s, p, P, Q,
-                                                            nullptr, ex, nullptr);
+        const bool tiled = k == s && p == 0 && c % 4 == 0 && h % k == 0 && w % k == 0 &&
+                           ((((uintptr_t)e) | (uintptr_t)arg | (uintptr_t)ex) & 3) == 0;
+        if (tiled) {
+            k_maxpool_bwd_tiled<<<grid_for((int64_t)n * P * Q * (c / 4)), kThreads, 0, st>>>(
+                e, arg, n, h, w, c / 4, k, P, Q, ex);
+        } else {
+            k_maxpool_bwd<<<grid_for(total), kThreads, 0, st>>>(e, arg, n, h, w, c, k, s, p, P,
+                                                                Q, nullptr, ex, nullptr);
+        }
         IQ_LAUNCH_CHECK();
         k_copy_scale<<<1, 1, 0, st>>>(s_e, s_ex);
         IQ_LAUNCH_CHECK();
@@ -401,6 +435,7 @@ extern "C" iq_status iq_upsample_fwd(const int8_t* x, const double* s_x, const i
     UpP u;
     if (!x || !s_x || !w || !out || !s_out || !up_dims(n, h, wd, c, R, stride, pad, &u))
         return IQ_ERR_INVALID_ARG;
+    if (c > 1024 || (R + stride - 1) / stride > 4) return IQ_ERR_UNSUPPORTED;
     size_t need = 0;
     iq_upsample_workspace_size(n, h, wd, c, R, &need);
     if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
@@ -409,15 +444,19 @@ extern "C" iq_status iq_upsample_fwd(const int8_t* x, const double* s_x, const i
     unsigned long long* cell = cur.take<unsigned long long>(1);
     RqDiv* dv = cur.take<RqDiv>(1);
     double* s_acc = cur.take<double>(1);
+    int8_t* wT = cur.take<int8_t>((size_t)c * R * R);
     IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, 8, st));
-    int64_t total = (int64_t)n * u.H * u.W * c;
-    k_up_max<<<grid_for(total), kThreads, 0, st>>>(u, x, w, cell);
+    k_up_wT<<<grid_for((int64_t)c * R * R), kThreads, 0, st>>>(w, wT, c, R);
+    IQ_LAUNCH_CHECK();
+    dim3 grid((unsigned)((u.W + 31) / 32), (unsigned)(n * u.H));
+    const int thr = (c + 31) / 32 * 32;
+    k_up_fwd<false><<<grid, thr, 0, st>>>(u, x, wT, cell, nullptr, 8, nullptr, nullptr);
     IQ_LAUNCH_CHECK();
     k_scale_pow2<<<1, 1, 0, st>>>(s_x, -7, s_acc);   // weights on the 8-bit grid
     IQ_LAUNCH_CHECK();
     k_sq_prepare<<<1, 1, 0, st>>>(cell, s_acc, 8, dv, s_out);
     IQ_LAUNCH_CHECK();
-    k_up_codes<<<grid_for(total), kThreads, 0, st>>>(u, x, w, dv, 8, out, acc_out);
+    k_up_fwd<true><<<grid, thr, 0, st>>>(u, x, wT, nullptr, dv, 8, out, acc_out);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }

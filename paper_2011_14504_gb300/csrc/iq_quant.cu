@@ -125,6 +125,30 @@ __global__ void k_rq_finalize(const unsigned long long* __restrict__ cell,
 
 // SQ: code = floor((2^k (q + M) + M) / (2M)) - 2^(k-1), the non-negative shift of
 // floor((2^k q + M) / (2M)); the numerator is < 2^(k+1) M + M < 2^57.
+__device__ __forceinline__ int64_t sq_code(int64_t v, const RqParams& p, int k, int relu,
+                                           int64_t lim) {
+    if (relu && v < 0) v = 0;
+    if (!p.M) return 0;
+    uint64_t num = ((uint64_t)(v + (int64_t)p.M) << k) + p.M;
+    return clamp64((int64_t)udiv(num, p.div) - (int64_t(1) << (k - 1)), -lim, lim);
+}
+
+// int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores)
+__global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int relu,
+                              const RqParams* __restrict__ prm, uint32_t* __restrict__ out) {
+    const RqParams p = *prm;
+    const int64_t lim = qmax(k);
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
+        int4 v = q[i];
+        uint32_t o = ((uint32_t)sq_code(v.x, p, k, relu, lim) & 0xffu) |
+                     (((uint32_t)sq_code(v.y, p, k, relu, lim) & 0xffu) << 8) |
+                     (((uint32_t)sq_code(v.z, p, k, relu, lim) & 0xffu) << 16) |
+                     (((uint32_t)sq_code(v.w, p, k, relu, lim) & 0xffu) << 24);
+        out[i] = o;
+    }
+}
+
 template <typename T>
 __global__ void k_sq_int(const T* __restrict__ q, int64_t n, int k, int relu,
                          const RqParams* __restrict__ prm, void* __restrict__ out, int dtype) {
@@ -189,7 +213,11 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
     IQ_LAUNCH_CHECK();
     if (n == 0) return IQ_OK;
     if (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) {
-        if (in_dtype == IQ_I32)
+        if (in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
+            (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0)
+            k_sq_i32_i8x4<<<grid_for(n / 4), kThreads, 0, st>>>((const int4*)q, n / 4, k, relu,
+                                                                prm, (uint32_t*)out);
+        else if (in_dtype == IQ_I32)
             k_sq_int<int32_t><<<g, kThreads, 0, st>>>((const int32_t*)q, n, k, relu, prm, out,
                                                       out_dtype);
         else
@@ -278,18 +306,25 @@ __global__ void k_weight_requant(const int32_t* __restrict__ m, int8_t* __restri
 }
 
 // Eq. (UQ2): dW = UQ(G_q lr, k_u) = clip(rhu(c s_g 2^(k_u-1-lr_log2))) (x2 grid: k_u-2),
-// m <- clip(m - dW), then wq = UQ(W_m, k_w).
+// m <- clip(m - dW), then wq = UQ(W_m, k_w).  A gradient code takes one of 255 values,
+// so each block first evaluates the fp64 product once per value (the same operations
+// every element with that code would perform) into a shared-memory table.
 __global__ void k_update(int32_t* __restrict__ master, int8_t* __restrict__ wq,
                          const int8_t* __restrict__ g, const double* __restrict__ s_g,
                          int64_t n, int sh, int k_u, int k_w) {
-    const double s = *s_g;
-    const double p2 = ldexp(1.0, sh);
+    __shared__ int32_t tab[256];
+    {
+        const double s = *s_g;
+        const double p2 = ldexp(1.0, sh);
+        for (int i = threadIdx.x; i < 255; i += blockDim.x)
+            tab[i] = (int32_t)code_of(__dmul_rn(__dmul_rn((double)(i - 127), s), p2), k_u);
+    }
+    __syncthreads();
     const int64_t lu = qmax(k_u), lw = qmax(k_w);
     const int dsh = k_u - k_w;
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
-        double t = __dmul_rn(__dmul_rn((double)g[i], s), p2);
-        int64_t du = code_of(t, k_u);
+        int64_t du = tab[(int)g[i] + 127];
         int64_t nm = clamp64((int64_t)master[i] - du, -lu, lu);
         master[i] = (int32_t)nm;
         int64_t v = (nm + (int64_t(1) << (dsh - 1))) >> dsh;
@@ -447,8 +482,8 @@ extern "C" iq_status iq_update(int32_t* master, int8_t* wq, const int8_t* g, con
     if (lr_log2 < 0 || lr_log2 > 60) return IQ_ERR_INVALID_ARG;
     if (n == 0) return IQ_OK;
     int sh = (x2 ? k_u - 2 : k_u - 1) - lr_log2;
-    k_update<<<grid_for(n), kThreads, 0, (cudaStream_t)stream>>>(master, wq, g, s_g, n, sh, k_u,
-                                                                  k_w);
+    k_update<<<grid_for(n, kThreads, 152 * 4), kThreads, 0, (cudaStream_t)stream>>>(
+        master, wq, g, s_g, n, sh, k_u, k_w);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }
