@@ -210,6 +210,23 @@ iq_status iq_bn_int_fwd(const int32_t* acc, int64_t m, int32_t c, const double* 
                         double* bn_scales, int64_t* bn_fixed, void* ws, size_t ws_bytes,
                         iq_stream stream);
 
+/* iq_bn_int_fwd_noalloc -- iq_bn_int_fwd without a workspace argument.  The paper has
+ * no counterpart: it serves callers that may not allocate device memory themselves (a
+ * plugin inside a host application that owns all device allocations, a real-time loop
+ * that must not allocate after start-up).  Its scratch is a fixed file-scope device
+ * array of 320 KB that every GPU loading the library keeps until process exit; it
+ * accepts c <= 4096 channels and returns IQ_ERR_UNSUPPORTED above that.  The first call
+ * on a device looks up that array's device address (one-time set-up, guarded by a
+ * lock); make that first call before any stream capture.  All calls share the one
+ * array: every call re-initialises the statistics it needs, but calls whose work
+ * overlaps on the GPU (different streams, no ordering) race on it.  Otherwise identical
+ * to iq_bn_int_fwd, with the same outputs. */
+iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_t c, const double* s_acc,
+                                const int32_t* gamma, const int32_t* beta,
+                                const iq_bn_bits* bits, int16_t* xhat, int8_t* a, double* s_a,
+                                int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
+                                iq_stream stream);
+
 /* iq_bn_int_bwd -- backward through Q_A/ReLU and the quantized L1BN (Sec. 3.3.1):
  *   e_y = e_a where a > 0 (ReLU mask of the stored activation codes);
  *   dbeta[c] = sum e_y (scale s_e), dgamma[c] = sum e_y X (scale s_e s_xhat), int64 out;

@@ -10,6 +10,7 @@
 #include "iq_internal.cuh"
 
 #include <climits>
+#include <mutex>
 
 namespace iq {
 
@@ -792,4 +793,52 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     if (dbeta)
         IQ_CUDA_CHECK(cudaMemcpyAsync(dbeta, w.sb, sizeof(int64_t) * c, cudaMemcpyDeviceToDevice, st));
     return IQ_OK;
+}
+
+// ==================================================================== no-allocation variant
+// For callers that may not allocate device memory themselves -- for example a plugin
+// running inside a host application that owns every device allocation, or a real-time
+// loop that must not allocate once it has started.  The scratch space lives in a
+// fixed-size file-scope device array instead of a caller-provided workspace.
+
+namespace {
+
+constexpr int32_t kBnNoAllocMaxC = 4096;          // largest channel count it accepts
+constexpr size_t kBnNoAllocBytes = 320 * 1024;    // scratch for up to kBnNoAllocMaxC channels
+
+static __device__ __align__(256) unsigned char g_bn_noalloc_scratch[kBnNoAllocBytes];
+
+std::mutex g_bn_noalloc_mu;
+void* g_bn_noalloc_ptr[256] = {};                 // device address of the array, per device
+
+}  // namespace
+
+extern "C" iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_t c,
+                                           const double* s_acc, const int32_t* gamma,
+                                           const int32_t* beta, const iq_bn_bits* bits,
+                                           int16_t* xhat, int8_t* a, double* s_a,
+                                           int32_t* bn_codes, double* bn_scales,
+                                           int64_t* bn_fixed, iq_stream stream) {
+    if (c > kBnNoAllocMaxC || bn_fwd_ws_bytes(c > 0 ? c : 1) > kBnNoAllocBytes)
+        return IQ_ERR_UNSUPPORTED;
+    int dev = -1;
+    IQ_CUDA_CHECK(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= 256) return IQ_ERR_UNSUPPORTED;
+    void* ws = nullptr;
+    {
+        // one-time set-up on this device: the host-side name of the array is not a device
+        // address, so ask the runtime for the address it has on the current device
+        std::lock_guard<std::mutex> lock(g_bn_noalloc_mu);
+        if (!g_bn_noalloc_ptr[dev]) {
+            void* p = nullptr;
+            cudaError_t e = cudaGetSymbolAddress(&p, g_bn_noalloc_scratch);
+            if (e != cudaSuccess || !p) return IQ_ERR_CUDA;
+            g_bn_noalloc_ptr[dev] = p;
+        }
+        ws = g_bn_noalloc_ptr[dev];
+    }
+    // the statistics in the scratch are re-initialised by every call (zero sums,
+    // min/max sentinels) before they are accumulated
+    return iq_bn_int_fwd(acc, m, c, s_acc, gamma, beta, bits, xhat, a, s_a, bn_codes, bn_scales,
+                         bn_fixed, ws, kBnNoAllocBytes, stream);
 }

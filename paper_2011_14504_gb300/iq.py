@@ -27,7 +27,7 @@ EXPORTS = [
     "iq_weight_requant", "iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad", "iq_bn_int_fwd",
     "iq_bn_int_bwd", "iq_relu_bwd", "iq_update", "iq_maxpool_fwd", "iq_maxpool_bwd",
     "iq_upsample_workspace_size", "iq_upsample_fwd", "iq_upsample_bwd", "iq_upsample_wgrad",
-    "iq_mse_grad",
+    "iq_mse_grad", "iq_bn_int_fwd_noalloc",
 ]
 
 
@@ -102,6 +102,8 @@ def load(path: str | None = None):
     L.iq_upsample_wgrad.argtypes = [_P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _I,
                                     _U64, _U64, _U64, _P, _P, _P, _P, _SZ, _P]
     L.iq_mse_grad.argtypes = [_P, _P, _P, _I64, _I32, _P, _P, _P, _SZ, _P]
+    L.iq_bn_int_fwd_noalloc.argtypes = [_P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _P, _P,
+                                        _P, _P, _P, _P, _P]
     for f in EXPORTS:
         if f not in ("iq_status_str", "iq_version", "iq_launch_count"):
             getattr(L, f).restype = _I
@@ -345,3 +347,15 @@ def iq_mse_grad(z, s_z, labels, E, s_e, ws=None, stream=None):
         ws = _ws(4096, z.device)
     _check("iq_mse_grad", load().iq_mse_grad(_p(z), _p(s_z), _p(labels), z.numel() // c, c, _p(E),
                                              _p(s_e), _p(ws), ws.numel(), _stream(stream)))
+
+
+def iq_bn_int_fwd_noalloc(acc, s_acc, gamma, beta, a, s_a, xhat=None, bn_codes=None,
+                          bn_scales=None, bn_fixed=None, bits=None, stream=None):
+    """iq_bn_int_fwd for callers that cannot allocate: no workspace argument."""
+    c = acc.shape[-1]
+    m = acc.numel() // c
+    _check("iq_bn_int_fwd_noalloc",
+           load().iq_bn_int_fwd_noalloc(_p(acc), m, c, _p(s_acc), _p(gamma), _p(beta),
+                                        C.byref(bits) if bits is not None else None, _p(xhat),
+                                        _p(a), _p(s_a), _p(bn_codes), _p(bn_scales),
+                                        _p(bn_fixed), _stream(stream)))
