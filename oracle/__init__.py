@@ -62,6 +62,13 @@ class BnOut(C.Structure):
                 ("m_y", C.c_double), ("p_x", C.c_int32), ("p_a", C.c_int32)]
 
 
+class Term(C.Structure):
+    _fields_ = [("codes", C.c_void_p), ("is16", C.c_int32), ("c", C.c_int32),
+                ("c_offset", C.c_int32), ("bcast", C.c_int32), ("scale", C.c_double),
+                ("gamma", C.c_void_p), ("beta", C.c_void_p), ("k_gamma", C.c_int32),
+                ("k_beta", C.c_int32)]
+
+
 _P = C.c_void_p
 _I64 = C.c_int64
 _I32 = C.c_int
@@ -104,6 +111,17 @@ def _declare(L):
     L.or_mse_grad.restype = _D
     L.or_u128_to_double.argtypes = [_U64, _U64]
     L.or_u128_to_double.restype = _D
+    L.or_combine.argtypes = [C.POINTER(Term), _I32, _I32, _I64, _I64, _I32, _I32, _P]
+    L.or_combine.restype = _D
+    L.or_spatial_sum.argtypes = [_P, _I64, _I64, _I32, _I32, _I32, _D, _I32, _P]
+    L.or_spatial_sum.restype = _D
+    L.or_bilinear_up.argtypes = [_P, _I32, _I32, _I32, _I32, _I32, _D, _P, _P]
+    L.or_bilinear_up.restype = _D
+    L.or_bilinear_up_bwd.argtypes = [_P, _I32, _I32, _I32, _I32, _I32, _D, _P, _P]
+    L.or_bilinear_up_bwd.restype = _D
+    L.or_exp_f32_n.argtypes = [_P, _I64, _P]
+    L.or_ce_grad.argtypes = [_P, _D, _P, _I64, _I32, _I32, _P, C.POINTER(C.c_int64)]
+    L.or_ce_grad.restype = _D
 
 
 def _ptr(a: np.ndarray):
@@ -369,3 +387,100 @@ def mse_grad(z, s_z: float, labels, k: int = 8):
     E = np.empty(z.shape, np.int8)
     s = lib().or_mse_grad(_ptr(z), z.size // c, c, float(s_z), _ptr(lab), k, _ptr(E))
     return E, s
+
+
+# ---------------------------------------------------------------- DeepLab glue
+
+@dataclass
+class CombineTerm:
+    """One operand of combine(): integer codes (int8 or int16) with real value
+    a_c v + b_c, a_c = scale (or gamma_q,c scale for a BN affine term), b_c = 0 (or beta_q,c).
+    codes are [n, hw, c] (or [n, c] with bcast: one value per image, broadcast over hw)."""
+    codes: np.ndarray
+    scale: float
+    c_offset: int = 0
+    bcast: bool = False
+    gamma: np.ndarray = None
+    beta: np.ndarray = None
+    k_gamma: int = 8
+    k_beta: int = 8
+
+
+def combine(terms, n: int, hw: int, c_out: int, concat: bool = False, relu: bool = False):
+    """Sum (or channel concatenation) of quantized tensors in real units, then SQ8
+    (Eqs. (AQ1)/(EQ) applied to a residual add, a sum of errors, the ASPP concat)."""
+    keep, arr = [], (Term * len(terms))()
+    for t, T in zip(terms, arr):
+        codes = np.ascontiguousarray(t.codes)
+        assert codes.dtype in (np.int8, np.int16)
+        keep.append(codes)
+        T.codes = codes.ctypes.data
+        T.is16 = int(codes.dtype == np.int16)
+        T.c = codes.shape[-1]
+        T.c_offset = t.c_offset
+        T.bcast = int(t.bcast)
+        T.scale = float(t.scale)
+        if t.gamma is not None:
+            g = _c(t.gamma, np.int32); b = _c(t.beta, np.int32)
+            keep += [g, b]
+            T.gamma, T.beta = g.ctypes.data, b.ctypes.data
+        else:
+            T.gamma = T.beta = None
+        T.k_gamma, T.k_beta = t.k_gamma, t.k_beta
+    out = np.empty((n * hw * c_out,), np.int8)
+    s = lib().or_combine(arr, len(terms), int(concat), n, hw, c_out, int(relu), _ptr(out))
+    return out, s
+
+
+def spatial_sum(x, s: float, mean: bool, c_offset: int = 0, c: int = None):
+    """Per image sum (mean) over the pixels of channels [c_offset, c_offset + c) of
+    x [n, h, w, c_total], then SQ8; returns ([n, c] codes, scale)."""
+    x = _c(x, np.int8)
+    n, c_total = x.shape[0], x.shape[-1]
+    hw = x.size // (n * c_total)
+    c = c_total - c_offset if c is None else c
+    out = np.empty((n, c), np.int8)
+    so = lib().or_spatial_sum(_ptr(x), n, hw, c_total, c_offset, c, float(s), int(mean), _ptr(out))
+    return out, so
+
+
+def bilinear_up(x, s: float, f: int):
+    """x8-style bilinear upsampling with aligned corners (exact integer numerators, then
+    SQ8); returns (codes [n, (h-1)f+1, (w-1)f+1, c], scale, numerators int32)."""
+    x = _c(x, np.int8)
+    n, h, w, c = x.shape
+    H, W = (h - 1) * f + 1, (w - 1) * f + 1
+    acc = np.empty((n, H, W, c), np.int32)
+    out = np.empty((n, H, W, c), np.int8)
+    so = lib().or_bilinear_up(_ptr(x), n, h, w, c, f, float(s), _ptr(acc), _ptr(out))
+    return out, so, acc
+
+
+def bilinear_up_bwd(e, s: float, f: int, in_shape):
+    e = _c(e, np.int8)
+    n, h, w, c = in_shape
+    assert e.shape == (n, (h - 1) * f + 1, (w - 1) * f + 1, c)
+    out = np.empty((n, h, w, c), np.int8)
+    acc = np.empty((n, h, w, c), np.int64)
+    so = lib().or_bilinear_up_bwd(_ptr(e), n, h, w, c, f, float(s), _ptr(acc), _ptr(out))
+    return out, so, acc
+
+
+def exp_f32(t) -> np.ndarray:
+    """The fp32 exponential of the softmax head (Cody-Waite reduction + degree-7 Taylor)."""
+    t = _c(t, np.float32)
+    out = np.empty(t.shape, np.float32)
+    lib().or_exp_f32_n(_ptr(t), t.size, _ptr(out))
+    return out
+
+
+def ce_grad(z, s_z: float, labels, ignore: int = 255):
+    """Softmax cross-entropy gradient on quantized logits, SQ8; returns (E, scale, n_valid)."""
+    z = _c(z, np.int8)
+    lab = _c(labels, np.uint8)
+    c = z.shape[-1]
+    E = np.empty(z.shape, np.int8)
+    nv = C.c_int64()
+    s = lib().or_ce_grad(_ptr(z), float(s_z), _ptr(lab), z.size // c, c, ignore, _ptr(E),
+                         C.byref(nv))
+    return E, s, nv.value

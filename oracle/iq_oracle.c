@@ -790,3 +790,271 @@ double or_mse_grad(const int8_t* z, int64_t npix, int c, double s_z, const uint8
         }
     return ldexp(M, 1 - k);
 }
+
+/* ------------------------------------------------------------------ */
+/* Network glue of the DeepLabv3-ResNet50 path                          */
+/* ------------------------------------------------------------------ */
+
+/* One operand of a combination: integer codes v (int8 or int16, [npix][c] or, when
+ * bcast != 0, [n][c] broadcast over the hw pixels of each image), real value
+ * a_c v + b_c with a_c = scale (or (gamma_c 2^(2-k_gamma)) * scale for a BN affine term)
+ * and b_c = 0 (or beta_c 2^(2-k_beta)). */
+typedef struct {
+    const void* codes;
+    int32_t is16, c, c_offset, bcast;
+    double scale;
+    const int32_t* gamma;
+    const int32_t* beta;
+    int32_t k_gamma, k_beta;
+} or_term;
+
+static double term_a(const or_term* t, int c) {
+    return t->gamma ? ((double)t->gamma[c] * ldexp(1.0, 2 - t->k_gamma)) * t->scale : t->scale;
+}
+static double term_b(const or_term* t, int c) {
+    return t->beta ? (double)t->beta[c] * ldexp(1.0, 2 - t->k_beta) : 0.0;
+}
+static int64_t term_v(const or_term* t, int64_t img, int64_t pix, int64_t hw, int c) {
+    int64_t idx = t->bcast ? img * t->c + c : (img * hw + pix) * t->c + c;
+    return t->is16 ? (int64_t)((const int16_t*)t->codes)[idx] : (int64_t)((const int8_t*)t->codes)[idx];
+}
+
+/* Sums (concat == 0: every term covers all c_out channels) or channel concatenations
+ * (concat != 0: term t fills channels [c_offset, c_offset + c)) of quantized tensors --
+ * the residual add of a bottleneck, the sum of the errors reaching one tensor, the ASPP
+ * concatenation -- followed by Q_A / Q_E = SQ(act(.), 8) (Eqs. (AQ1),(EQ)).  The real sum
+ * is carried in fixed point: z = sum_t (F_t,c v + B_t,c) with F = rhu(a 2^P),
+ * B = rhu(b 2^P) and P = 50 - exponent of sum_t max_c(|a| vmax + |b|), so |z| < 2^51;
+ * then SQ on the integer z (value z 2^-P) is exact: code = floor((256 z + M) / (2M)).
+ * Returns the output scale (M 2^-P) 2^-7. */
+double or_combine(const or_term* terms, int nt, int concat, int64_t n, int64_t hw, int c_out,
+                  int relu, int8_t* out) {
+    double bound = 0.0;
+    for (int t = 0; t < nt; t++) {
+        double vmax = terms[t].is16 ? 32767.0 : 127.0, lt = 0.0;
+        for (int c = 0; c < terms[t].c; c++) {
+            double l = fabs(term_a(&terms[t], c)) * vmax + fabs(term_b(&terms[t], c));
+            if (l > lt) lt = l;
+        }
+        bound = bound + lt;
+    }
+    int P = 50 - frexp_exp(bound + 1.0);
+    if (P > 62) P = 62;
+    int64_t* z = (int64_t*)malloc(sizeof(int64_t) * (size_t)(n * hw * c_out));
+    int64_t M = 0;
+    for (int64_t img = 0; img < n; img++)
+        for (int64_t pix = 0; pix < hw; pix++)
+            for (int co = 0; co < c_out; co++) {
+                i128 acc = 0;
+                for (int t = 0; t < nt; t++) {
+                    int c = co;
+                    if (concat) {
+                        c = co - terms[t].c_offset;
+                        if (c < 0 || c >= terms[t].c) continue;
+                    }
+                    int64_t F = (int64_t)rhu(ldexp(term_a(&terms[t], c), P));
+                    int64_t B = (int64_t)rhu(ldexp(term_b(&terms[t], c), P));
+                    acc += (i128)F * term_v(&terms[t], img, pix, hw, c) + B;
+                }
+                int64_t v = (int64_t)acc;
+                if (relu && v < 0) v = 0;
+                z[(img * hw + pix) * c_out + co] = v;
+                int64_t av = v < 0 ? -v : v;
+                if (av > M) M = av;
+            }
+    for (int64_t i = 0; i < n * hw * c_out; i++) {
+        if (M == 0) { out[i] = 0; continue; }
+        i128 q = floordiv128(((i128)z[i] << 8) + M, (i128)2 * M);
+        out[i] = (int8_t)clamp64((int64_t)q, -127, 127);
+    }
+    free(z);
+    return M ? ldexp((double)M, -P - 7) : ldexp(1.0, -P - 7);
+}
+
+/* Per image, the sum over its hw pixels of channels [c_off, c_off + c) of a tensor with
+ * c_total channels, then SQ8.  mean != 0: global average pooling (the ASPP image-pooling
+ * branch), real value s sum / hw; the 1/hw cancels in x / Scale(x), so the codes are SQ8
+ * of the integer sums and the scale is ((s M) / hw) 2^-7.  mean == 0: the backward of a
+ * broadcast over the pixels (the error of the pooled branch), scale (s M) 2^-7. */
+double or_spatial_sum(const int8_t* x, int64_t n, int64_t hw, int c_total, int c_off, int c,
+                      double s, int mean, int8_t* out) {
+    int64_t* sums = (int64_t*)malloc(sizeof(int64_t) * (size_t)(n * c + 1));
+    int64_t M = 0;
+    for (int64_t img = 0; img < n; img++)
+        for (int ch = 0; ch < c; ch++) {
+            int64_t acc = 0;
+            for (int64_t p = 0; p < hw; p++) acc += x[(img * hw + p) * c_total + c_off + ch];
+            sums[img * c + ch] = acc;
+            if ((acc < 0 ? -acc : acc) > M) M = acc < 0 ? -acc : acc;
+        }
+    for (int64_t i = 0; i < n * c; i++) {
+        if (M == 0) { out[i] = 0; continue; }
+        i128 q = floordiv128(((i128)sums[i] << 8) + M, (i128)2 * M);
+        out[i] = (int8_t)clamp64((int64_t)q, -127, 127);
+    }
+    free(sums);
+    double sm = M ? s * (double)M : s;
+    return ldexp(mean ? sm / (double)hw : sm, -7);
+}
+
+/* Bilinear upsampling by an integer factor f with aligned corners (output size
+ * (h-1) f + 1, the DeepLab logits 65 -> 513 for f = 8): output (f i + r, f j + t) is
+ * ((f-r)(f-t) x[i,j] + r(f-t) x[i+1,j] + (f-r) t x[i,j+1] + r t x[i+1,j+1]) / f^2, exact
+ * in integers; SQ8 of the integer numerators (the 1/f^2 cancels), scale ((s M)/f^2) 2^-7. */
+double or_bilinear_up(const int8_t* x, int n, int h, int w, int c, int f, double s,
+                      int32_t* acc_out, int8_t* out) {
+    int H = (h - 1) * f + 1, W = (w - 1) * f + 1;
+    int64_t total = (int64_t)n * H * W * c;
+    int32_t* a = acc_out ? acc_out : (int32_t*)malloc(sizeof(int32_t) * (size_t)total);
+    int64_t M = 0;
+    for (int b = 0; b < n; b++)
+        for (int I = 0; I < H; I++)
+            for (int J = 0; J < W; J++)
+                for (int ch = 0; ch < c; ch++) {
+                    int i = I / f, r = I % f, j = J / f, t = J % f;
+                    int i1 = i + 1 < h ? i + 1 : i, j1 = j + 1 < w ? j + 1 : j;
+#define XV(ii, jj) ((int64_t)x[(((int64_t)b * h + (ii)) * w + (jj)) * c + ch])
+                    int64_t v = (int64_t)(f - r) * (f - t) * XV(i, j) + (int64_t)r * (f - t) * XV(i1, j) +
+                                (int64_t)(f - r) * t * XV(i, j1) + (int64_t)r * t * XV(i1, j1);
+#undef XV
+                    a[(((int64_t)b * H + I) * W + J) * c + ch] = (int32_t)v;
+                    if ((v < 0 ? -v : v) > M) M = v < 0 ? -v : v;
+                }
+    for (int64_t i = 0; i < total; i++) {
+        if (M == 0) { out[i] = 0; continue; }
+        i128 q = floordiv128(((i128)a[i] << 8) + M, (i128)2 * M);
+        out[i] = (int8_t)clamp64((int64_t)q, -127, 127);
+    }
+    if (!acc_out) free(a);
+    return M ? ldexp((s * (double)M) / (double)(f * f), -7) : ldexp(s / (double)(f * f), -7);
+}
+
+/* Adjoint of or_bilinear_up: the error at low-resolution pixel (i, j) collects
+ * w_r w_t e[f i' + r, f j' + t] over every output that interpolates from it, with the same
+ * integer weights (f-r or r, f-t or t); SQ8 of the integer sums, scale ((s M)/f^2) 2^-7.
+ * Output row f i + r (0 < r < f) takes weight (f - r) from row i and r from row i + 1;
+ * the last row (h - 1) f takes weight f from row h - 1. */
+double or_bilinear_up_bwd(const int8_t* e, int n, int h, int w, int c, int f, double s,
+                          int64_t* acc_out, int8_t* out) {
+    int H = (h - 1) * f + 1, W = (w - 1) * f + 1;
+    int64_t total = (int64_t)n * h * w * c;
+    int64_t* a = (int64_t*)calloc((size_t)total, sizeof(int64_t));
+    for (int b = 0; b < n; b++)
+        for (int I = 0; I < H; I++)
+            for (int J = 0; J < W; J++)
+                for (int ch = 0; ch < c; ch++) {
+                    int i = I / f, r = I % f, j = J / f, t = J % f;
+                    int64_t ev = e[(((int64_t)b * H + I) * W + J) * c + ch];
+#define AX(ii, jj) a[(((int64_t)b * h + (ii)) * w + (jj)) * c + ch]
+                    AX(i, j) += (int64_t)(f - r) * (f - t) * ev;
+                    if (r) AX(i + 1, j) += (int64_t)r * (f - t) * ev;
+                    if (t) AX(i, j + 1) += (int64_t)(f - r) * t * ev;
+                    if (r && t) AX(i + 1, j + 1) += (int64_t)r * t * ev;
+#undef AX
+                }
+    int64_t M = 0;
+    for (int64_t i = 0; i < total; i++) {
+        int64_t v = a[i] < 0 ? -a[i] : a[i];
+        if (v > M) M = v;
+    }
+    for (int64_t i = 0; i < total; i++) {
+        if (M == 0) { out[i] = 0; continue; }
+        i128 q = floordiv128(((i128)a[i] << 8) + M, (i128)2 * M);
+        out[i] = (int8_t)clamp64((int64_t)q, -127, 127);
+    }
+    if (acc_out) memcpy(acc_out, a, sizeof(int64_t) * (size_t)total);
+    free(a);
+    return M ? ldexp((s * (double)M) / (double)(f * f), -7) : ldexp(s / (double)(f * f), -7);
+}
+
+/* fp32 exponential for t <= 0, written out so that any IEEE single-precision machine
+ * computes the same bits (no fused multiply-add).  Cody-Waite range reduction: k =
+ * rhu(t log2 e), r = (t - k c1) - k c2 with c1 + c2 = ln 2 and c1 carrying 15 significant
+ * bits, so k c1 is exact for |k| < 2^9; e^r from its Taylor series to degree 7 in Horner
+ * form (|r| <= ln2/2 + tiny, truncation below 8e-9 relative); times 2^k by building the
+ * exponent field.  t < -87 (and any k < -126) gives 0. */
+float or_exp_f32(float t) {
+    if (!(t >= -87.0f)) return 0.0f;
+    if (t > 0.0f) t = 0.0f;
+    const float log2e = 0x1.715476p+0f;   /* fp32 nearest to log2(e) */
+    const float c1 = 0x1.62e4p-1f;        /* ln 2 to 15 significant bits */
+    const float c2 = 0x1.7f7d1cp-20f;     /* ln 2 - c1, rounded to fp32 */
+    float kf = floorf(t * log2e + 0.5f);
+    float r = (t - kf * c1) - kf * c2;
+    /* Taylor coefficients 1/n!, each the nearest fp32 */
+    float p = 0x1.a01a02p-13f;            /* 1/5040 */
+    p = p * r + 0x1.6c16c2p-10f;          /* 1/720 */
+    p = p * r + 0x1.111112p-7f;           /* 1/120 */
+    p = p * r + 0x1.555556p-5f;           /* 1/24 */
+    p = p * r + 0x1.555556p-3f;           /* 1/6 */
+    p = p * r + 0.5f;
+    p = p * r + 1.0f;
+    p = p * r + 1.0f;
+    int k = (int)kf;
+    if (k < -126) return 0.0f;
+    union { uint32_t u; float f; } sc;
+    sc.u = (uint32_t)(k + 127) << 23;
+    return p * sc.f;
+}
+
+/* Softmax cross-entropy gradient on quantized logits (the DeepLab head; sum over
+ * classes, mean over labelled pixels): per pixel t_c = (z_c - max z) * (float)s_z,
+ * e_c = or_exp_f32(t_c), S = e_0 + e_1 + ... (class order), p_c = e_c / S,
+ * g_c = p_c - [c == label]; pixels labelled `ignore` give 0.  E = SQ8 of g as a float
+ * tensor (Scale = max|g|, Eq. (ScaleQ) on floats, code = rhu(fl(g / Scale) 128) clipped),
+ * and its scale is (Scale 2^-7) / n_valid, the 1/n_valid of the mean loss.  All-zero g:
+ * codes 0 and scale 2^-7 / max(n_valid, 1).  Returns the scale; *n_valid_out gets the
+ * count of labelled pixels. */
+double or_ce_grad(const int8_t* z, double s_z, const uint8_t* labels, int64_t npix, int c,
+                  int ignore, int8_t* E, int64_t* n_valid_out) {
+    float* g = (float*)malloc(sizeof(float) * (size_t)(npix * c + 1));
+    float* ex = (float*)malloc(sizeof(float) * (size_t)c);
+    const float sf = (float)s_z;
+    int64_t nv = 0;
+    float gmax = 0.0f;
+    for (int64_t p = 0; p < npix; p++) {
+        const int8_t* zp = z + p * c;
+        int lab = labels[p];
+        if (lab == ignore) {
+            for (int ch = 0; ch < c; ch++) g[p * c + ch] = 0.0f;
+            continue;
+        }
+        nv++;
+        int zm = -128;
+        for (int ch = 0; ch < c; ch++) if (zp[ch] > zm) zm = zp[ch];
+        float S = 0.0f;
+        for (int ch = 0; ch < c; ch++) {
+            float t = (float)(zp[ch] - zm) * sf;
+            ex[ch] = or_exp_f32(t);
+            S = S + ex[ch];
+        }
+        for (int ch = 0; ch < c; ch++) {
+            float pc = ex[ch] / S;
+            float gv = ch == lab ? pc - 1.0f : pc;
+            g[p * c + ch] = gv;
+            if (fabsf(gv) > gmax) gmax = fabsf(gv);
+        }
+    }
+    double scale;
+    if (gmax == 0.0f) {
+        for (int64_t i = 0; i < npix * c; i++) E[i] = 0;
+        scale = ldexp(1.0, -7) / (double)(nv > 0 ? nv : 1);
+    } else {
+        for (int64_t i = 0; i < npix * c; i++) {
+            float t = g[i] / gmax;
+            float y = t * 128.0f;
+            float f = floorf(y);
+            int64_t q = (int64_t)f + ((y - f) >= 0.5f ? 1 : 0);
+            E[i] = (int8_t)clamp64(q, -127, 127);
+        }
+        scale = ldexp((double)gmax, -7) / (double)nv;
+    }
+    if (n_valid_out) *n_valid_out = nv;
+    free(g); free(ex);
+    return scale;
+}
+
+/* or_exp_f32 over an array (for its tests). */
+void or_exp_f32_n(const float* t, int64_t n, float* out) {
+    for (int64_t i = 0; i < n; i++) out[i] = or_exp_f32(t[i]);
+}
