@@ -310,6 +310,124 @@ iq_status iq_mse_grad(const int8_t* z, const double* s_z, const uint8_t* labels,
                       int32_t c, int8_t* E, double* s_e, void* ws, size_t ws_bytes,
                       iq_stream stream);
 
+/* ---------------------------------------------------------------- DeepLab glue
+ * (Sec. 5, DeepLabv3-ResNet50: bottleneck residual adds, the ASPP concatenation and its
+ * image-pooling branch, the aligned-corner x8 bilinear upsampling of the logits and the
+ * softmax cross-entropy loss.  The paper does not say how these are quantized; each call
+ * evaluates the real-valued operation on the integer codes exactly (or in fixed point
+ * with a 2^-50 relative step) and requantizes with Q_A / Q_E = SQ(., 8).) */
+
+/* One operand of iq_combine.  Its real value per element is a_ch v + b_ch, with v the
+ * integer code, a_ch = scale (times gamma_q,ch when gamma is given) and b_ch = beta_q,ch
+ * (0 when beta is NULL): a plain quantized tensor, or the BN affine map gamma_q X s_X +
+ * beta_q of the X codes of a BN layer (pass the X codes, s_X = bn_scales[IQ_BN_S_XHAT]
+ * and the gamma/beta codes). */
+typedef struct {
+    const void* codes;      /* device codes, dtype IQ_I8 or IQ_I16; [n][hw][c], or
+                               [n][c] when bcast != 0 (one value per image and channel,
+                               the same at every pixel) */
+    int32_t dtype;
+    int32_t c;              /* channels of this operand */
+    int32_t c_offset;       /* concat: first output channel it fills (sum: must be 0) */
+    int32_t bcast;
+    const double* scale;    /* device double */
+    const int32_t* gamma;   /* optional device int32[c]: codes of gamma_q (scale 2^(2-k_gamma)) */
+    const int32_t* beta;    /* optional device int32[c]: codes of beta_q (scale 2^(2-k_beta)) */
+    int32_t k_gamma, k_beta;
+} iq_term;
+
+#define IQ_MAX_TERMS 8
+
+/* Workspace of iq_combine. */
+iq_status iq_combine_workspace_size(const iq_term* terms, int32_t n_terms, size_t* bytes);
+
+/* iq_combine -- out = SQ(act(sum of operands), 8), Eq. (AQ1) / (EQ), with act = ReLU when
+ * relu != 0.  concat == 0: every operand covers all c_out channels (the residual add of a
+ * bottleneck, the sum of the errors that reach one tensor); concat != 0: operand t covers
+ * channels [c_offset, c_offset + c) (the ASPP concatenation; overlapping ranges add).
+ * The sum is evaluated in fixed point: z = sum_t (F_t,ch v + B_t,ch), F = rhu(a 2^P),
+ * B = rhu(b 2^P), one shift P per call = 50 - (binary exponent of 1 + sum_t max_ch
+ * (|a| vmax + |b|)) (vmax 127 or 32767), at most 62; then code = floor((256 z + M)/(2M))
+ * clipped to +-127 with M = max |z|, and s_out = M 2^(-P-7) (M = 0: zero codes,
+ * s_out = 2^(-P-7)).  n images of hw pixels; terms is a host array of 1..IQ_MAX_TERMS
+ * descriptors (device pointers inside); out int8 [n][hw][c_out]; s_out device double. */
+iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t concat, int64_t n,
+                     int64_t hw, int32_t c_out, int32_t relu, int8_t* out, double* s_out,
+                     void* ws, size_t ws_bytes, iq_stream stream);
+
+/* Workspace of iq_spatial_sum. */
+iq_status iq_spatial_sum_workspace_size(int64_t n, int32_t c, size_t* bytes);
+
+/* iq_spatial_sum -- per image, the sum over its hw pixels of channels [c_off, c_off + c) of
+ * x [n][hw][c_total] (int8 codes, device scale s_x), then SQ(., 8) of the n x c sums.
+ *   mean != 0: global average pooling (the ASPP image-pooling branch): real value s_x
+ *              sum / hw, s_out = ((s_x M) / hw) 2^-7 (the 1/hw cancels in the codes);
+ *   mean == 0: the backward of a broadcast over the pixels, s_out = (s_x M) 2^-7.
+ * M = 0 gives zero codes and s_out = (s_x / hw or s_x) 2^-7.  out int8 [n][c]. */
+iq_status iq_spatial_sum(const int8_t* x, const double* s_x, int64_t n, int64_t hw,
+                         int32_t c_total, int32_t c_off, int32_t c, int32_t mean, int8_t* out,
+                         double* s_out, void* ws, size_t ws_bytes, iq_stream stream);
+
+/* iq_avgpool_bwd -- error of the input of a global average pooling: every pixel of image
+ * i gets the pooled error e[i][c] / hw.  s_ex = s_e / hw (IEEE division); when ex is not
+ * NULL the codes e are broadcast into ex [n][hw][c]; otherwise pass e as a bcast operand
+ * with scale s_ex to iq_combine. */
+iq_status iq_avgpool_bwd(const int8_t* e, const double* s_e, int64_t n, int64_t hw, int32_t c,
+                         int8_t* ex, double* s_ex, iq_stream stream);
+
+/* iq_channel_slice -- out[p][j] = x[p][c_off + j] for j < c (codes only: the error of one
+ * operand of a concatenation, whose scale is that of the concatenated error). */
+iq_status iq_channel_slice(const int8_t* x, int64_t npix, int32_t c_total, int32_t c_off,
+                           int32_t c, int8_t* out, iq_stream stream);
+
+/* Workspace of the two bilinear calls. */
+iq_status iq_bilinear_workspace_size(int32_t n, int32_t h, int32_t w, int32_t c, size_t* bytes);
+
+/* iq_bilinear_up_fwd -- bilinear upsampling by an integer factor f with aligned corners,
+ * output (h-1) f + 1 by (w-1) f + 1 (f = 8: the DeepLab logits 65 -> 513).  Output pixel
+ * (f i + r, f j + t) has the integer numerator (f-r)(f-t) x[i][j] + r(f-t) x[i+1][j] +
+ * (f-r) t x[i][j+1] + r t x[i+1][j+1] (real value numerator s_x / f^2), exact; codes =
+ * SQ(., 8) of the numerators, s_out = ((s_x M) / f^2) 2^-7.  x int8 [n][h][w][c];
+ * out int8 [n][H][W][c]. */
+iq_status iq_bilinear_up_fwd(const int8_t* x, const double* s_x, int32_t n, int32_t h,
+                             int32_t w, int32_t c, int32_t f, int8_t* out, double* s_out,
+                             void* ws, size_t ws_bytes, iq_stream stream);
+
+/* iq_bilinear_up_bwd -- its adjoint on errors: ex[i][j] = sum over the outputs that read
+ * x[i][j] of (integer weight) e, exact int32, then SQ(., 8); s_ex = ((s_e M) / f^2) 2^-7.
+ * e int8 [n][H][W][c]; ex int8 [n][h][w][c] (h, w the INPUT size of the forward). */
+iq_status iq_bilinear_up_bwd(const int8_t* e, const double* s_e, int32_t n, int32_t h,
+                             int32_t w, int32_t c, int32_t f, int8_t* ex, double* s_ex,
+                             void* ws, size_t ws_bytes, iq_stream stream);
+
+/* iq_ce_grad -- gradient of the softmax cross-entropy loss (mean over labelled pixels) on
+ * quantized logits, the DeepLab loss: per pixel t_c = (z_c - max z) * (float)s_z,
+ * e_c = exp(t_c) by a fixed fp32 sequence (Cody-Waite reduction with ln 2 split into
+ * 0x1.62e4p-1 + 0x1.7f7d1cp-20, k = floor(t log2e + 1/2), Taylor polynomial of degree 7
+ * in Horner form, no fused multiply-add, 0 below t = -87), S = sum of e_c in class order,
+ * p_c = e_c / S, g_c = p_c - [c == label]; pixels labelled `ignore` give g = 0.  Then
+ * Q_E on the float tensor: G = max |g|, code = rhu(fl(g / G) 128) clipped to +-127, and
+ * s_e = (G 2^-7) / n_valid (G = 0: zero codes, s_e = 2^-7 / max(n_valid, 1)).
+ *   z int8 [npix][c] (c <= 1024), device scale s_z; labels uint8 [npix]; E out int8
+ *   [npix][c]; s_e out device double; n_valid optional out device int64. */
+iq_status iq_ce_grad(const int8_t* z, const double* s_z, const uint8_t* labels, int64_t npix,
+                     int32_t c, int32_t ignore, int8_t* E, double* s_e, int64_t* n_valid,
+                     void* ws, size_t ws_bytes, iq_stream stream);
+
+/* iq_bn_update -- Sec. 3.3.3 for the L1BN parameters: the sums dgamma (scale s_e s_X,
+ * s_X = bn_scales[IQ_BN_S_XHAT]) and dbeta (scale s_e) from iq_bn_int_bwd are quantized
+ * with Eq. (GQ1) (RQ to 8 bits, Philox key (seed, layer), counter (i/8, step, tag, 0) with
+ * tag 1 for gamma and 2 for beta), then master <- clip(master - UQ(G_q lr, k_u)) on the
+ * x2 grid (value master 2^(2-k_u)), lr = 2^-lr_log2, and the codes gamma = UQ2(master,
+ * k_gamma), beta = UQ2(master, k_beta) used by the forward.  All arrays int32[c] on the
+ * device; gamma_master / beta_master in/out, gamma / beta out.  ws >= 4096 bytes + 2c. */
+iq_status iq_bn_update(int32_t* gamma_master, int32_t* beta_master, int32_t* gamma,
+                       int32_t* beta, const int64_t* dgamma, const int64_t* dbeta,
+                       const double* s_e, const double* bn_scales, int32_t c,
+                       const iq_bn_bits* bits, int lr_log2, int k_u, uint64_t seed,
+                       uint64_t layer, uint64_t step, void* ws, size_t ws_bytes,
+                       iq_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -842,3 +842,68 @@ extern "C" iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_
     return iq_bn_int_fwd(acc, m, c, s_acc, gamma, beta, bits, xhat, a, s_a, bn_codes, bn_scales,
                          bn_fixed, ws, kBnNoAllocBytes, stream);
 }
+
+// ---------------------------------------------------------------- parameter update
+
+namespace iq {
+namespace {
+
+__global__ void k_bn_grad_scale(const double* __restrict__ s_e, const double* __restrict__ bn_scales,
+                                double* __restrict__ out) {
+    out[0] = __dmul_rn(*s_e, bn_scales[IQ_BN_S_XHAT]);
+}
+
+// master <- clip(master - UQ(G_q s_g 2^sh, k_u)), codes = UQ2(master, k_w) on the x2 grid
+__global__ void k_bn_param_update(int32_t* __restrict__ master, int32_t* __restrict__ codes,
+                                  const int8_t* __restrict__ g, const double* __restrict__ s_g,
+                                  int32_t c, int sh, int k_u, int k_w) {
+    const double s = *s_g;
+    const double p2 = ldexp(1.0, sh);
+    const int64_t lu = qmax(k_u), lw = qmax(k_w);
+    const int dsh = k_u - k_w;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < c; i += gridDim.x * blockDim.x) {
+        const int64_t du = code_of(__dmul_rn(__dmul_rn((double)g[i], s), p2), k_u);
+        const int64_t nm = clamp64((int64_t)master[i] - du, -lu, lu);
+        master[i] = (int32_t)nm;
+        codes[i] = (int32_t)clamp64((nm + (int64_t(1) << (dsh - 1))) >> dsh, -lw, lw);
+    }
+}
+
+}  // namespace
+}  // namespace iq
+
+extern "C" iq_status iq_bn_update(int32_t* gamma_master, int32_t* beta_master, int32_t* gamma,
+                                  int32_t* beta, const int64_t* dgamma, const int64_t* dbeta,
+                                  const double* s_e, const double* bn_scales, int32_t c,
+                                  const iq_bn_bits* bits, int lr_log2, int k_u, uint64_t seed,
+                                  uint64_t layer, uint64_t step, void* ws, size_t ws_bytes,
+                                  iq_stream stream) {
+    using namespace iq;
+    if (!gamma_master || !beta_master || !gamma || !beta || !dgamma || !dbeta || !s_e ||
+        !bn_scales || c < 1)
+        return IQ_ERR_INVALID_ARG;
+    const iq_bn_bits b = bn_bits_or_default(bits);
+    if (!bn_bits_valid(b) || k_u <= b.k_gamma || k_u <= b.k_beta || k_u > 31) return IQ_ERR_INVALID_ARG;
+    if (lr_log2 < 0 || lr_log2 > 60) return IQ_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < 4096 + 2 * (size_t)c) return IQ_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    char* w = (char*)ws;
+    double* sc = (double*)(w + 1024);            // [0] s_e s_X, [1] s_G gamma, [2] s_G beta
+    int8_t* gg = (int8_t*)(w + 4096);
+    int8_t* gb = gg + c;
+    k_bn_grad_scale<<<1, 1, 0, st>>>(s_e, bn_scales, sc);
+    IQ_LAUNCH_CHECK();
+    iq_status r = requant_int(dgamma, IQ_I64, c, sc, 8, IQ_MODE_RQ_GQ1, seed, layer, step, 1, gg,
+                              IQ_I8, sc + 1, w, st);
+    if (r != IQ_OK) return r;
+    r = requant_int(dbeta, IQ_I64, c, s_e, 8, IQ_MODE_RQ_GQ1, seed, layer, step, 2, gb, IQ_I8,
+                    sc + 2, w, st);
+    if (r != IQ_OK) return r;
+    const int sh = (k_u - 2) - lr_log2;
+    const int g = (c + kThreads - 1) / kThreads;
+    k_bn_param_update<<<g, kThreads, 0, st>>>(gamma_master, gamma, gg, sc + 1, c, sh, k_u, b.k_gamma);
+    IQ_LAUNCH_CHECK();
+    k_bn_param_update<<<g, kThreads, 0, st>>>(beta_master, beta, gb, sc + 2, c, sh, k_u, b.k_beta);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}

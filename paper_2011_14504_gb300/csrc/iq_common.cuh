@@ -51,7 +51,7 @@ struct UDiv {
     uint64_t d;
 };
 
-__device__ inline UDiv make_udiv(uint64_t d) {
+__host__ __device__ inline UDiv make_udiv(uint64_t d) {
     int l = 0;
     while (l < 64 && (uint64_t(1) << l) < d) l++;
     UDiv u;

@@ -1,0 +1,371 @@
+// iq_merge.cu -- quantized sums and concatenations, spatial sums and channel slices:
+// the tensor joins of DeepLabv3-ResNet50 (bottleneck residual adds, the sums of the
+// errors that reach one tensor, the ASPP concatenation and its image-pooling branch).
+//
+// The paper (Sec. 5) runs DeepLabv3 fully quantized but does not say how its joins are
+// quantized; here each join evaluates the real-valued operation on the codes and then
+// applies Q_A / Q_E = SQ(., 8) (Eq. (ScaleQ) with Scale = max|.| of the whole tensor).
+#include <climits>
+
+#include "iq_internal.cuh"
+
+namespace iq {
+
+namespace {
+
+struct TermDev {
+    const void* codes;
+    const double* scale;
+    const int32_t* gamma;
+    const int32_t* beta;
+    int32_t is16, c, c_offset, bcast, k_gamma, k_beta, base;   // base: first table row
+};
+
+struct Terms {
+    TermDev t[IQ_MAX_TERMS];
+    int32_t n;
+};
+
+// Workspace: [0,256) header (max cell, shift P, output parameters), then F and B tables.
+struct CombHdr {
+    unsigned long long maxz;
+    int32_t P;
+    int32_t pad;
+    uint64_t M;
+    UDiv div;
+};
+
+__device__ __forceinline__ double term_a(const TermDev& t, double s, int ch) {
+    if (!t.gamma) return s;
+    return __dmul_rn(__dmul_rn((double)t.gamma[ch], ldexp(1.0, 2 - t.k_gamma)), s);
+}
+__device__ __forceinline__ double term_b(const TermDev& t, int ch) {
+    return t.beta ? __dmul_rn((double)t.beta[ch], ldexp(1.0, 2 - t.k_beta)) : 0.0;
+}
+
+// One block: per operand the bound max_ch(|a| vmax + |b|), the shift P from their sum (in
+// operand order), then the tables F = rhu(a 2^P), B = rhu(b 2^P).
+__global__ void k_comb_tables(Terms T, CombHdr* hdr, long long* F, long long* B) {
+    __shared__ unsigned long long lt[IQ_MAX_TERMS];
+    __shared__ int sP;
+    if (threadIdx.x < IQ_MAX_TERMS) lt[threadIdx.x] = 0ull;
+    __syncthreads();
+    for (int i = 0; i < T.n; i++) {
+        const TermDev& t = T.t[i];
+        const double s = *t.scale;
+        const double vmax = t.is16 ? 32767.0 : 127.0;
+        double l = 0.0;
+        for (int ch = threadIdx.x; ch < t.c; ch += blockDim.x) {
+            double v = __dadd_rn(__dmul_rn(fabs(term_a(t, s, ch)), vmax), fabs(term_b(t, ch)));
+            l = v > l ? v : l;
+        }
+        // non-negative doubles order as their bit patterns
+        atomicMax(&lt[i], (unsigned long long)__double_as_longlong(l));
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double bound = 0.0;
+        for (int i = 0; i < T.n; i++) bound = __dadd_rn(bound, __longlong_as_double((long long)lt[i]));
+        int e;
+        frexp(__dadd_rn(bound, 1.0), &e);
+        int P = 50 - e;
+        if (P > 62) P = 62;
+        sP = P;
+        hdr->P = P;
+        hdr->maxz = 0ull;
+    }
+    __syncthreads();
+    const int P = sP;
+    for (int i = 0; i < T.n; i++) {
+        const TermDev& t = T.t[i];
+        const double s = *t.scale;
+        for (int ch = threadIdx.x; ch < t.c; ch += blockDim.x) {
+            F[t.base + ch] = (long long)rhu(ldexp(term_a(t, s, ch), P));
+            B[t.base + ch] = (long long)rhu(ldexp(term_b(t, ch), P));
+        }
+    }
+}
+
+__device__ __forceinline__ int64_t load_code(const TermDev& t, int64_t idx) {
+    return t.is16 ? (int64_t)((const int16_t*)t.codes)[idx] : (int64_t)((const int8_t*)t.codes)[idx];
+}
+
+// Pass 0: max |z| over the tensor.  Pass 1: the SQ(., 8) codes.
+template <int PASS>
+__global__ void __launch_bounds__(kThreads) k_comb(Terms T, int concat, int64_t n, int64_t hw,
+                                                   int c_out, int relu,
+                                                   const long long* __restrict__ F,
+                                                   const long long* __restrict__ B,
+                                                   CombHdr* hdr, int8_t* __restrict__ out,
+                                                   UDiv dc, UDiv dhw) {
+    uint64_t M = 0;
+    UDiv d2m;
+    if (PASS == 1) {
+        M = hdr->M;
+        d2m = hdr->div;
+    }
+    const int64_t total = n * hw * (int64_t)c_out;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    uint64_t mx = 0;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += stride) {
+        const int64_t pix = (int64_t)udiv((uint64_t)e, dc);
+        const int co = (int)(e - pix * c_out);
+        const int64_t img = (int64_t)udiv((uint64_t)pix, dhw);
+        int64_t z = 0;
+        for (int i = 0; i < T.n; i++) {
+            const TermDev& t = T.t[i];
+            int ch = co;
+            if (concat) {
+                ch = co - t.c_offset;
+                if (ch < 0 || ch >= t.c) continue;
+            }
+            const int64_t idx = t.bcast ? img * t.c + ch : pix * t.c + ch;
+            z += (int64_t)F[t.base + ch] * load_code(t, idx) + (int64_t)B[t.base + ch];
+        }
+        if (relu && z < 0) z = 0;
+        if (PASS == 0) {
+            uint64_t a = (uint64_t)(z < 0 ? -z : z);
+            mx = a > mx ? a : mx;
+        } else {
+            int64_t c = 0;
+            if (M) {
+                uint64_t num = ((uint64_t)(z + (int64_t)M) << 8) + M;
+                c = clamp64((int64_t)udiv(num, d2m) - 128, -127, 127);
+            }
+            out[e] = (int8_t)c;
+        }
+    }
+    if (PASS == 0) {
+        mx = warp_max_u64(mx);
+        if ((threadIdx.x & 31) == 0 && mx) atomicMax(&hdr->maxz, (unsigned long long)mx);
+    }
+}
+
+__global__ void k_comb_params(CombHdr* hdr, double* s_out) {
+    const uint64_t M = hdr->maxz;
+    hdr->M = M;
+    hdr->div = make_udiv(M ? 2 * M : 1);
+    *s_out = M ? ldexp((double)M, -hdr->P - 7) : ldexp(1.0, -hdr->P - 7);
+}
+
+// ---------------------------------------------------------------- spatial sums
+
+// sums[i][j] += sum over a slice of image i's pixels of x[i][p][c_off + j]
+__global__ void k_ssum(const int8_t* __restrict__ x, int64_t hw, int c_total, int c_off, int c,
+                       int64_t pix_per_block, unsigned long long* __restrict__ sums) {
+    const int64_t img = blockIdx.y;
+    const int j = blockIdx.z * blockDim.x + threadIdx.x;
+    if (j >= c) return;
+    const int64_t p0 = (int64_t)blockIdx.x * pix_per_block;
+    const int64_t p1 = min(hw, p0 + pix_per_block);
+    const int8_t* src = x + (img * hw) * c_total + c_off + j;
+    int64_t acc = 0;
+    for (int64_t p = p0; p < p1; p++) acc += src[p * c_total];
+    if (acc) atomicAdd(&sums[img * c + j], (unsigned long long)acc);
+}
+
+// One block: M = max |sum|, the output scale in the oracle's order, then the codes.
+__global__ void k_ssum_finish(const unsigned long long* __restrict__ sums, int64_t count,
+                              const double* __restrict__ s_x, double den,
+                              int8_t* __restrict__ out, double* __restrict__ s_out) {
+    __shared__ unsigned long long sM;
+    __shared__ UDiv sdiv;
+    if (threadIdx.x == 0) sM = 0;
+    __syncthreads();
+    uint64_t mx = 0;
+    for (int64_t i = threadIdx.x; i < count; i += blockDim.x) {
+        int64_t v = (int64_t)sums[i];
+        uint64_t a = (uint64_t)(v < 0 ? -v : v);
+        mx = a > mx ? a : mx;
+    }
+    mx = warp_max_u64(mx);
+    if ((threadIdx.x & 31) == 0) atomicMax(&sM, (unsigned long long)mx);
+    __syncthreads();
+    const uint64_t M = sM;
+    if (threadIdx.x == 0) {
+        sdiv = make_udiv(M ? 2 * M : 1);
+        const double s = *s_x;
+        const double sm = M ? __dmul_rn(s, (double)M) : s;
+        *s_out = ldexp(__ddiv_rn(sm, den), -7);
+    }
+    __syncthreads();
+    const UDiv d = sdiv;
+    for (int64_t i = threadIdx.x; i < count; i += blockDim.x) {
+        int64_t c = 0;
+        if (M) {
+            uint64_t num = ((uint64_t)((int64_t)sums[i] + (int64_t)M) << 8) + M;
+            c = clamp64((int64_t)udiv(num, d) - 128, -127, 127);
+        }
+        out[i] = (int8_t)c;
+    }
+}
+
+__global__ void k_scale_div(const double* __restrict__ s, double den, double* __restrict__ out) {
+    *out = __ddiv_rn(*s, den);
+}
+
+__global__ void k_bcast(const int8_t* __restrict__ e, int64_t n, int64_t hw, int c,
+                        int8_t* __restrict__ ex, UDiv dhwc) {
+    const int64_t total = n * hw * c;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+        const int64_t img = (int64_t)udiv((uint64_t)i, dhwc);
+        const int64_t r = i - img * hw * c;
+        const int64_t pix = r / c;
+        ex[i] = e[img * c + (r - pix * c)];
+    }
+}
+
+__global__ void k_slice(const int8_t* __restrict__ x, int64_t npix, int c_total, int c_off, int c,
+                        int8_t* __restrict__ out, UDiv dc) {
+    const int64_t total = npix * c;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+        const int64_t p = (int64_t)udiv((uint64_t)i, dc);
+        out[i] = x[p * c_total + c_off + (i - p * c)];
+    }
+}
+
+bool terms_ok(const iq_term* terms, int32_t n_terms) {
+    if (!terms || n_terms < 1 || n_terms > IQ_MAX_TERMS) return false;
+    for (int i = 0; i < n_terms; i++) {
+        const iq_term& t = terms[i];
+        if (!t.codes || !t.scale || t.c < 1) return false;
+        if (t.dtype != IQ_I8 && t.dtype != IQ_I16) return false;
+        if ((t.gamma == nullptr) != (t.beta == nullptr)) return false;
+        if (t.gamma && (t.k_gamma < 2 || t.k_gamma > 16 || t.k_beta < 2 || t.k_beta > 16))
+            return false;
+    }
+    return true;
+}
+
+size_t comb_ws(const iq_term* terms, int32_t n_terms) {
+    size_t rows = 0;
+    for (int i = 0; i < n_terms; i++) rows += (size_t)terms[i].c;
+    return 256 + 2 * (((rows * 8) + 255) & ~size_t(255));
+}
+
+}  // namespace
+
+}  // namespace iq
+
+using namespace iq;
+
+extern "C" iq_status iq_combine_workspace_size(const iq_term* terms, int32_t n_terms,
+                                               size_t* bytes) {
+    if (!bytes || !terms_ok(terms, n_terms)) return IQ_ERR_INVALID_ARG;
+    *bytes = comb_ws(terms, n_terms);
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t concat, int64_t n,
+                                int64_t hw, int32_t c_out, int32_t relu, int8_t* out,
+                                double* s_out, void* ws, size_t ws_bytes, iq_stream stream) {
+    if (!terms_ok(terms, n_terms) || !out || !s_out || n < 1 || hw < 1 || c_out < 1)
+        return IQ_ERR_INVALID_ARG;
+    if (n * hw > (int64_t(1) << 40)) return IQ_ERR_INVALID_ARG;
+    Terms T;
+    T.n = n_terms;
+    int32_t base = 0;
+    for (int i = 0; i < n_terms; i++) {
+        const iq_term& s = terms[i];
+        if (concat) {
+            if (s.c_offset < 0 || s.c_offset + s.c > c_out) return IQ_ERR_INVALID_ARG;
+        } else if (s.c != c_out || s.c_offset != 0) {
+            return IQ_ERR_INVALID_ARG;
+        }
+        TermDev& t = T.t[i];
+        t.codes = s.codes;
+        t.scale = s.scale;
+        t.gamma = s.gamma;
+        t.beta = s.beta;
+        t.is16 = s.dtype == IQ_I16;
+        t.c = s.c;
+        t.c_offset = concat ? s.c_offset : 0;
+        t.bcast = s.bcast != 0;
+        t.k_gamma = s.k_gamma;
+        t.k_beta = s.k_beta;
+        t.base = base;
+        base += s.c;
+    }
+    if (!ws || ws_bytes < comb_ws(terms, n_terms)) return IQ_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    CombHdr* hdr = (CombHdr*)ws;
+    const size_t tab = (((size_t)base * 8) + 255) & ~size_t(255);
+    long long* F = (long long*)((char*)ws + 256);
+    long long* B = (long long*)((char*)ws + 256 + tab);
+    k_comb_tables<<<1, 1024, 0, st>>>(T, hdr, F, B);
+    IQ_LAUNCH_CHECK();
+    const int64_t total = n * hw * (int64_t)c_out;
+    const int g = grid_for(total, kThreads, 152 * 8);
+    const UDiv dc = make_udiv((uint64_t)c_out), dhw = make_udiv((uint64_t)hw);
+    k_comb<0><<<g, kThreads, 0, st>>>(T, concat != 0, n, hw, c_out, relu != 0, F, B, hdr, out,
+                                      dc, dhw);
+    IQ_LAUNCH_CHECK();
+    k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
+    IQ_LAUNCH_CHECK();
+    k_comb<1><<<g, kThreads, 0, st>>>(T, concat != 0, n, hw, c_out, relu != 0, F, B, hdr, out,
+                                      dc, dhw);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_spatial_sum_workspace_size(int64_t n, int32_t c, size_t* bytes) {
+    if (!bytes || n < 1 || c < 1) return IQ_ERR_INVALID_ARG;
+    *bytes = (((size_t)n * c * 8) + 255) & ~size_t(255);
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_spatial_sum(const int8_t* x, const double* s_x, int64_t n, int64_t hw,
+                                    int32_t c_total, int32_t c_off, int32_t c, int32_t mean,
+                                    int8_t* out, double* s_out, void* ws, size_t ws_bytes,
+                                    iq_stream stream) {
+    if (!x || !s_x || !out || !s_out || n < 1 || n > 65535 || hw < 1 || c < 1 || c_off < 0 ||
+        c_off + c > c_total)
+        return IQ_ERR_INVALID_ARG;
+    if (hw * 127 >= (int64_t(1) << 62) / 2) return IQ_ERR_INVALID_ARG;
+    const size_t need = (((size_t)n * c * 8) + 255) & ~size_t(255);
+    if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    unsigned long long* sums = (unsigned long long*)ws;
+    IQ_CUDA_CHECK(cudaMemsetAsync(sums, 0, (size_t)n * c * 8, st));
+    const int cz = (c + kThreads - 1) / kThreads;
+    // enough pixel slices that the grid covers the SMs a few times over
+    int64_t slices = (152 * 8 + n * cz - 1) / (n * cz);
+    if (slices > hw) slices = hw;
+    if (slices < 1) slices = 1;
+    if (slices > 65535) slices = 65535;
+    const int64_t per = (hw + slices - 1) / slices;
+    slices = (hw + per - 1) / per;
+    dim3 grid((unsigned)slices, (unsigned)n, (unsigned)cz);
+    k_ssum<<<grid, kThreads, 0, st>>>(x, hw, c_total, c_off, c, per, sums);
+    IQ_LAUNCH_CHECK();
+    k_ssum_finish<<<1, 1024, 0, st>>>(sums, n * c, s_x, mean ? (double)hw : 1.0, out, s_out);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_avgpool_bwd(const int8_t* e, const double* s_e, int64_t n, int64_t hw,
+                                    int32_t c, int8_t* ex, double* s_ex, iq_stream stream) {
+    if (!e || !s_e || !s_ex || n < 1 || hw < 1 || c < 1) return IQ_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    k_scale_div<<<1, 1, 0, st>>>(s_e, (double)hw, s_ex);
+    IQ_LAUNCH_CHECK();
+    if (ex) {
+        k_bcast<<<grid_for(n * hw * c), kThreads, 0, st>>>(e, n, hw, c, ex,
+                                                            make_udiv((uint64_t)(hw * c)));
+        IQ_LAUNCH_CHECK();
+    }
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_channel_slice(const int8_t* x, int64_t npix, int32_t c_total,
+                                      int32_t c_off, int32_t c, int8_t* out, iq_stream stream) {
+    if (!x || !out || npix < 0 || c < 1 || c_off < 0 || c_off + c > c_total)
+        return IQ_ERR_INVALID_ARG;
+    if (npix == 0) return IQ_OK;
+    k_slice<<<grid_for(npix * c), kThreads, 0, (cudaStream_t)stream>>>(x, npix, c_total, c_off, c,
+                                                                      out, make_udiv((uint64_t)c));
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}

@@ -27,7 +27,10 @@ EXPORTS = [
     "iq_weight_requant", "iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad", "iq_bn_int_fwd",
     "iq_bn_int_bwd", "iq_relu_bwd", "iq_update", "iq_maxpool_fwd", "iq_maxpool_bwd",
     "iq_upsample_workspace_size", "iq_upsample_fwd", "iq_upsample_bwd", "iq_upsample_wgrad",
-    "iq_mse_grad", "iq_bn_int_fwd_noalloc",
+    "iq_mse_grad", "iq_bn_int_fwd_noalloc", "iq_combine_workspace_size", "iq_combine",
+    "iq_spatial_sum_workspace_size", "iq_spatial_sum", "iq_avgpool_bwd", "iq_channel_slice",
+    "iq_bilinear_workspace_size", "iq_bilinear_up_fwd", "iq_bilinear_up_bwd", "iq_ce_grad",
+    "iq_bn_update",
 ]
 
 
@@ -45,6 +48,17 @@ class ConvDesc(C.Structure):
 
 class BnBits(C.Structure):
     _fields_ = [(n, C.c_int32) for n in ("k_mu", "k_sigma", "k_xhat", "k_gamma", "k_beta", "k_a")]
+
+
+class Term(C.Structure):
+    """iq_term: one operand of iq_combine (device pointers inside)."""
+    _fields_ = [("codes", C.c_void_p), ("dtype", C.c_int32), ("c", C.c_int32),
+                ("c_offset", C.c_int32), ("bcast", C.c_int32), ("scale", C.c_void_p),
+                ("gamma", C.c_void_p), ("beta", C.c_void_p), ("k_gamma", C.c_int32),
+                ("k_beta", C.c_int32)]
+
+
+IQ_MAX_TERMS = 8
 
 
 _P = C.c_void_p
@@ -104,6 +118,19 @@ def load(path: str | None = None):
     L.iq_mse_grad.argtypes = [_P, _P, _P, _I64, _I32, _P, _P, _P, _SZ, _P]
     L.iq_bn_int_fwd_noalloc.argtypes = [_P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _P, _P,
                                         _P, _P, _P, _P, _P]
+    L.iq_combine_workspace_size.argtypes = [C.POINTER(Term), _I32, C.POINTER(_SZ)]
+    L.iq_combine.argtypes = [C.POINTER(Term), _I32, _I32, _I64, _I64, _I32, _I32, _P, _P, _P, _SZ,
+                             _P]
+    L.iq_spatial_sum_workspace_size.argtypes = [_I64, _I32, C.POINTER(_SZ)]
+    L.iq_spatial_sum.argtypes = [_P, _P, _I64, _I64, _I32, _I32, _I32, _I32, _P, _P, _P, _SZ, _P]
+    L.iq_avgpool_bwd.argtypes = [_P, _P, _I64, _I64, _I32, _P, _P, _P]
+    L.iq_channel_slice.argtypes = [_P, _I64, _I32, _I32, _I32, _P, _P]
+    L.iq_bilinear_workspace_size.argtypes = [_I32, _I32, _I32, _I32, C.POINTER(_SZ)]
+    L.iq_bilinear_up_fwd.argtypes = [_P, _P, _I32, _I32, _I32, _I32, _I32, _P, _P, _P, _SZ, _P]
+    L.iq_bilinear_up_bwd.argtypes = [_P, _P, _I32, _I32, _I32, _I32, _I32, _P, _P, _P, _SZ, _P]
+    L.iq_ce_grad.argtypes = [_P, _P, _P, _I64, _I32, _I32, _P, _P, _P, _P, _SZ, _P]
+    L.iq_bn_update.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _I32, C.POINTER(BnBits), _I, _I,
+                               _U64, _U64, _U64, _P, _SZ, _P]
     for f in EXPORTS:
         if f not in ("iq_status_str", "iq_version", "iq_launch_count"):
             getattr(L, f).restype = _I
@@ -359,3 +386,100 @@ def iq_bn_int_fwd_noalloc(acc, s_acc, gamma, beta, a, s_a, xhat=None, bn_codes=N
                                         C.byref(bits) if bits is not None else None, _p(xhat),
                                         _p(a), _p(s_a), _p(bn_codes), _p(bn_scales),
                                         _p(bn_fixed), _stream(stream)))
+
+
+# ---------------------------------------------------------------- DeepLab glue
+
+def term(codes, scale, c_offset=0, bcast=False, gamma=None, beta=None, k_gamma=8, k_beta=8):
+    """An iq_term over device tensors: codes int8/int16 [..., c], scale a device double
+    (tensor, or an int device address such as bn_scales' IQ_BN_S_XHAT element)."""
+    dt = {torch.int8: IQ_I8, torch.int16: IQ_I16}[codes.dtype]
+    return Term(codes.data_ptr(), dt, codes.shape[-1], c_offset, int(bcast), _p(scale),
+                _p(gamma), _p(beta), k_gamma, k_beta)
+
+
+def iq_combine_workspace_size(terms) -> int:
+    arr = (Term * len(terms))(*terms)
+    b = _SZ()
+    _check("iq_combine_workspace_size", load().iq_combine_workspace_size(arr, len(terms), C.byref(b)))
+    return b.value
+
+
+def iq_combine(terms, n, hw, c_out, out, s_out, concat=False, relu=False, ws=None, stream=None):
+    arr = (Term * len(terms))(*terms)
+    if ws is None:
+        ws = _ws(iq_combine_workspace_size(terms), out.device)
+    _check("iq_combine", load().iq_combine(arr, len(terms), int(concat), n, hw, c_out, int(relu),
+                                           _p(out), _p(s_out), _p(ws), ws.numel(),
+                                           _stream(stream)))
+
+
+def iq_spatial_sum_workspace_size(n, c) -> int:
+    return _size("iq_spatial_sum_workspace_size", n, c)
+
+
+def iq_spatial_sum(x, s_x, out, s_out, mean=True, c_off=0, c=None, ws=None, stream=None):
+    n, c_total = x.shape[0], x.shape[-1]
+    hw = x.numel() // (n * c_total)
+    c = c_total - c_off if c is None else c
+    if ws is None:
+        ws = _ws(iq_spatial_sum_workspace_size(n, c), x.device)
+    _check("iq_spatial_sum", load().iq_spatial_sum(_p(x), _p(s_x), n, hw, c_total, c_off, c,
+                                                   int(mean), _p(out), _p(s_out), _p(ws),
+                                                   ws.numel(), _stream(stream)))
+
+
+def iq_avgpool_bwd(e, s_e, hw, s_ex, ex=None, stream=None):
+    n, c = e.shape[0], e.shape[-1]
+    _check("iq_avgpool_bwd", load().iq_avgpool_bwd(_p(e), _p(s_e), n, hw, c, _p(ex), _p(s_ex),
+                                                   _stream(stream)))
+
+
+def iq_channel_slice(x, c_off, c, out, stream=None):
+    c_total = x.shape[-1]
+    _check("iq_channel_slice", load().iq_channel_slice(_p(x), x.numel() // c_total, c_total, c_off,
+                                                       c, _p(out), _stream(stream)))
+
+
+def iq_bilinear_workspace_size(n, h, w, c) -> int:
+    return _size("iq_bilinear_workspace_size", n, h, w, c)
+
+
+def iq_bilinear_up_fwd(x, s_x, f, out, s_out, ws=None, stream=None):
+    n, h, w, c = x.shape
+    if ws is None:
+        ws = _ws(iq_bilinear_workspace_size(n, h, w, c), x.device)
+    _check("iq_bilinear_up_fwd", load().iq_bilinear_up_fwd(_p(x), _p(s_x), n, h, w, c, f, _p(out),
+                                                           _p(s_out), _p(ws), ws.numel(),
+                                                           _stream(stream)))
+
+
+def iq_bilinear_up_bwd(e, s_e, f, in_shape, ex, s_ex, ws=None, stream=None):
+    n, h, w, c = in_shape
+    if ws is None:
+        ws = _ws(iq_bilinear_workspace_size(n, h, w, c), e.device)
+    _check("iq_bilinear_up_bwd", load().iq_bilinear_up_bwd(_p(e), _p(s_e), n, h, w, c, f, _p(ex),
+                                                           _p(s_ex), _p(ws), ws.numel(),
+                                                           _stream(stream)))
+
+
+def iq_ce_grad(z, s_z, labels, E, s_e, n_valid=None, ignore=255, ws=None, stream=None):
+    c = z.shape[-1]
+    if ws is None:
+        ws = _ws(4096, z.device)
+    _check("iq_ce_grad", load().iq_ce_grad(_p(z), _p(s_z), _p(labels), z.numel() // c, c, ignore,
+                                           _p(E), _p(s_e), _p(n_valid), _p(ws), ws.numel(),
+                                           _stream(stream)))
+
+
+def iq_bn_update(gamma_master, beta_master, gamma, beta, dgamma, dbeta, s_e, bn_scales, lr_log2,
+                 seed, layer, step, k_u=24, bits=None, ws=None, stream=None):
+    c = gamma.numel()
+    if ws is None:
+        ws = _ws(4096 + 2 * c + 256, gamma.device)
+    _check("iq_bn_update", load().iq_bn_update(_p(gamma_master), _p(beta_master), _p(gamma),
+                                               _p(beta), _p(dgamma), _p(dbeta), _p(s_e),
+                                               _p(bn_scales), c,
+                                               C.byref(bits) if bits is not None else None,
+                                               lr_log2, k_u, seed, layer, step, _p(ws),
+                                               ws.numel(), _stream(stream)))

@@ -84,3 +84,36 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert rc == iq.IQ_ERR_UNSUPPORTED
     rc = lib.iq_update(1, 1, 1, 1, 10, -1, 24, 8, 0, None)
     assert rc == iq.IQ_ERR_INVALID_ARG
+
+
+def test_glue_arguments_rejected_before_launch(lib):
+    T = iq.Term
+    ok = T(16, iq.IQ_I8, 8, 0, 0, 16, None, None, 8, 8)
+    arr = (T * 9)(*([ok] * 9))
+    assert lib.iq_combine(arr, 0, 0, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_combine(arr, 9, 0, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    # a sum whose operand does not cover every output channel
+    assert lib.iq_combine(arr, 2, 0, 1, 4, 16, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    # a concatenation operand past the last channel
+    off = (T * 1)(T(16, iq.IQ_I8, 8, 4, 0, 16, None, None, 8, 8))
+    assert lib.iq_combine(off, 1, 1, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    # gamma without beta, bad dtype
+    half = (T * 1)(T(16, iq.IQ_I8, 8, 0, 0, 16, 16, None, 8, 8))
+    assert lib.iq_combine(half, 1, 0, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    wide = (T * 1)(T(16, iq.IQ_I32, 8, 0, 0, 16, None, None, 8, 8))
+    assert lib.iq_combine(wide, 1, 0, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    need = C.c_size_t()
+    assert lib.iq_combine_workspace_size(arr, 2, C.byref(need)) == 0 and need.value >= 256 + 2 * 128
+    assert lib.iq_combine(arr, 2, 0, 1, 4, 8, 0, 16, 16, 16, 64, None) == iq.IQ_ERR_WORKSPACE
+    assert lib.iq_spatial_sum(16, 16, 2, 9, 8, 4, 8, 1, 16, 16, 16, 4096, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_spatial_sum(16, 16, 2, 9, 8, 0, 8, 1, 16, 16, 16, 8, None) == iq.IQ_ERR_WORKSPACE
+    assert lib.iq_avgpool_bwd(None, 16, 2, 9, 8, None, 16, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_channel_slice(16, 10, 8, 6, 4, 16, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_bilinear_up_fwd(16, 16, 1, 4, 4, 3, 0, 16, 16, 16, 4096, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_bilinear_up_bwd(16, 16, 1, 4, 4, 3, 8, 16, 16, 16, 64, None) == iq.IQ_ERR_WORKSPACE
+    assert lib.iq_ce_grad(16, 16, 16, 10, 2000, 255, 16, 16, None, 16, 4096, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_ce_grad(16, 16, 16, 10, 21, 255, 16, 16, None, 16, 8, None) == iq.IQ_ERR_WORKSPACE
+    assert lib.iq_bn_update(16, 16, 16, 16, 16, None, 16, 16, 8, None, 10, 24, 0, 0, 0, 16, 1 << 16,
+                            None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_bn_update(16, 16, 16, 16, 16, 16, 16, 16, 8, None, 10, 24, 0, 0, 0, 16, 100,
+                            None) == iq.IQ_ERR_WORKSPACE

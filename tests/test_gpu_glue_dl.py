@@ -1,0 +1,213 @@
+"""GPU parity of the DeepLab glue calls against the oracle: every code bit-exact and every
+scale equal as fp64 (0 ULP), on seeded inputs that span several blocks and ragged tails,
+plus the full-size shapes of the DeepLabv3-ResNet50 head (65 -> 513, 21 classes)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2011_14504_gb300 import iq
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).to(DEV)
+
+
+def dscal(v):
+    return torch.tensor([v], dtype=torch.float64, device=DEV)
+
+
+def host(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+def scal():
+    return torch.zeros(1, dtype=torch.float64, device=DEV)
+
+
+# ---------------------------------------------------------------- combine
+
+def run_combine(specs, n, hw, c_out, concat, relu):
+    """specs: list of (codes np, scale, c_offset, bcast, gamma np|None, beta np|None)."""
+    keep, terms, oterms = [], [], []
+    for codes, s, off, bc, gam, bet in specs:
+        dc, ds = dev(codes), dscal(s)
+        dg = dev(gam) if gam is not None else None
+        db = dev(bet) if bet is not None else None
+        keep += [dc, ds, dg, db]
+        terms.append(iq.term(dc, ds, off, bc, dg, db))
+        oterms.append(O.CombineTerm(codes, s, off, bc, gam, bet))
+    out = torch.empty(n * hw * c_out, dtype=torch.int8, device=DEV)
+    so = scal()
+    iq.iq_combine(terms, n, hw, c_out, out, so, concat=concat, relu=relu)
+    ref, sref = O.combine(oterms, n, hw, c_out, concat=concat, relu=relu)
+    assert np.array_equal(host(out), ref)
+    assert host(so)[0] == sref
+
+
+def test_combine_residual_bn_affine_plus_shortcut():
+    g = np.random.default_rng(11)
+    n, hw, c = 2, 37 * 29, 96
+    X = g.integers(-32767, 32768, size=(n, hw, c)).astype(np.int16)
+    sc = g.integers(0, 128, size=(n, hw, c)).astype(np.int8)
+    gam = g.integers(-100, 128, size=c).astype(np.int32)
+    bet = g.integers(-127, 128, size=c).astype(np.int32)
+    run_combine([(X, 2.0 ** -15 * 3.7, 0, False, gam, bet), (sc, 0.041, 0, False, None, None)],
+                n, hw, c, False, True)
+
+
+def test_combine_two_bn_branches_downsample():
+    g = np.random.default_rng(12)
+    n, hw, c = 3, 17 * 17, 64
+    terms = []
+    for k in range(2):
+        X = g.integers(-32767, 32768, size=(n, hw, c)).astype(np.int16)
+        gam = g.integers(-127, 128, size=c).astype(np.int32)
+        bet = g.integers(-127, 128, size=c).astype(np.int32)
+        terms.append((X, 2.0 ** -15 * (1.5 + k), 0, False, gam, bet))
+    run_combine(terms, n, hw, c, False, True)
+
+
+def test_combine_sum_of_errors_with_broadcast():
+    """The error reaching the ASPP input: four branch errors plus the pooled one."""
+    g = np.random.default_rng(13)
+    n, hw, c = 2, 9 * 11, 40
+    specs = [(g.integers(-127, 128, size=(n, hw, c)).astype(np.int8), s, 0, False, None, None)
+             for s in (0.01, 0.3, 1e-4, 0.02)]
+    specs.append((g.integers(-127, 128, size=(n, c)).astype(np.int8), 0.5 / hw, 0, True, None, None))
+    run_combine(specs, n, hw, c, False, False)
+
+
+def test_combine_concat_aspp():
+    g = np.random.default_rng(14)
+    n, hw, cb = 2, 13 * 13, 32
+    specs = [(g.integers(0, 128, size=(n, hw, cb)).astype(np.int8), 0.01 * (k + 1), k * cb, False,
+              None, None) for k in range(4)]
+    specs.append((g.integers(0, 128, size=(n, cb)).astype(np.int8), 0.07, 4 * cb, True, None, None))
+    run_combine(specs, n, hw, 5 * cb, True, False)
+
+
+def test_combine_edge_cases():
+    # all zero, a single pixel, a single channel
+    run_combine([(np.zeros((1, 5, 8), np.int8), 0.5, 0, False, None, None)], 1, 5, 8, False, False)
+    run_combine([(np.full((1, 1, 3), -127, np.int8), 0.5, 0, False, None, None),
+                 (np.full((1, 1, 3), 127, np.int8), 0.25, 0, False, None, None)], 1, 1, 3, False,
+                False)
+    g = np.random.default_rng(15)
+    run_combine([(g.integers(-127, 128, size=(4, 33, 1)).astype(np.int8), 3.0, 0, False, None,
+                  None)], 4, 33, 1, False, True)
+
+
+# ---------------------------------------------------------------- spatial sums, slices
+
+@pytest.mark.parametrize("mean,n,h,w,ct,off,c", [(True, 2, 65, 65, 256, 0, 256),
+                                                  (True, 3, 7, 5, 40, 0, 40),
+                                                  (False, 2, 9, 9, 96, 64, 32),
+                                                  (False, 1, 1, 1, 8, 3, 5)])
+def test_spatial_sum(mean, n, h, w, ct, off, c):
+    g = np.random.default_rng(16)
+    x = g.integers(-127, 128, size=(n, h, w, ct)).astype(np.int8)
+    out = torch.empty((n, c), dtype=torch.int8, device=DEV)
+    so = scal()
+    iq.iq_spatial_sum(dev(x), dscal(0.013), out, so, mean=mean, c_off=off, c=c)
+    ref, sref = O.spatial_sum(x, 0.013, mean, c_offset=off, c=c)
+    assert np.array_equal(host(out), ref) and host(so)[0] == sref
+
+
+def test_avgpool_bwd_and_channel_slice():
+    g = np.random.default_rng(17)
+    e = g.integers(-127, 128, size=(3, 24)).astype(np.int8)
+    ex = torch.empty((3, 35, 24), dtype=torch.int8, device=DEV)
+    sx = scal()
+    iq.iq_avgpool_bwd(dev(e), dscal(0.37), 35, sx, ex=ex)
+    assert host(sx)[0] == 0.37 / 35
+    assert np.array_equal(host(ex), np.broadcast_to(e[:, None, :], (3, 35, 24)))
+    x = g.integers(-127, 128, size=(2, 5, 7, 48)).astype(np.int8)
+    out = torch.empty((2, 5, 7, 20), dtype=torch.int8, device=DEV)
+    iq.iq_channel_slice(dev(x), 17, 20, out)
+    assert np.array_equal(host(out), x[..., 17:37])
+
+
+# ---------------------------------------------------------------- bilinear, softmax head
+
+@pytest.mark.parametrize("n,h,w,c,f", [(2, 9, 9, 21, 8), (1, 5, 7, 3, 4), (3, 4, 3, 5, 1),
+                                       (2, 65, 65, 21, 8)])
+def test_bilinear_up_fwd_bwd(n, h, w, c, f):
+    g = np.random.default_rng(18)
+    x = g.integers(-127, 128, size=(n, h, w, c)).astype(np.int8)
+    H, W = (h - 1) * f + 1, (w - 1) * f + 1
+    out = torch.empty((n, H, W, c), dtype=torch.int8, device=DEV)
+    so = scal()
+    iq.iq_bilinear_up_fwd(dev(x), dscal(0.02), f, out, so)
+    ref, sref, _ = O.bilinear_up(x, 0.02, f)
+    assert np.array_equal(host(out), ref) and host(so)[0] == sref
+    e = g.integers(-127, 128, size=(n, H, W, c)).astype(np.int8)
+    ex = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
+    sx = scal()
+    iq.iq_bilinear_up_bwd(dev(e), dscal(0.003), f, (n, h, w, c), ex, sx)
+    refb, srefb, _ = O.bilinear_up_bwd(e, 0.003, f, (n, h, w, c))
+    assert np.array_equal(host(ex), refb) and host(sx)[0] == srefb
+
+
+@pytest.mark.parametrize("n,h,w,c,s", [(2, 33, 35, 21, 0.05), (1, 7, 9, 150, 0.5),
+                                       (2, 513, 513, 21, 0.03), (1, 3, 3, 2, 4.0)])
+def test_ce_grad(n, h, w, c, s):
+    g = np.random.default_rng(19)
+    z = g.integers(-127, 128, size=(n, h, w, c)).astype(np.int8)
+    lab = g.integers(0, c, size=(n, h, w)).astype(np.uint8)
+    lab[g.random(lab.shape) < 0.05] = 255
+    E = torch.empty_like(dev(z))
+    se = scal()
+    nv = torch.zeros(1, dtype=torch.int64, device=DEV)
+    iq.iq_ce_grad(dev(z), dscal(s), dev(lab), E, se, n_valid=nv)
+    ref, sref, nref = O.ce_grad(z, s, lab)
+    assert host(nv)[0] == nref
+    assert np.array_equal(host(E), ref) and host(se)[0] == sref
+
+
+def test_ce_grad_all_ignored_and_saturated():
+    z = np.zeros((1, 4, 4, 21), np.int8)
+    lab = np.full((1, 4, 4), 255, np.uint8)
+    E = torch.ones((1, 4, 4, 21), dtype=torch.int8, device=DEV)
+    se = scal()
+    iq.iq_ce_grad(dev(z), dscal(1.0), dev(lab), E, se)
+    ref, sref, _ = O.ce_grad(z, 1.0, lab)
+    assert not host(E).any() and host(se)[0] == sref
+    # logits far apart: exp underflows to 0 for every class but the max
+    z = np.full((1, 2, 2, 4), -127, np.int8)
+    z[..., 1] = 127
+    lab = np.array([[[0, 1], [1, 3]]], np.uint8)
+    E2 = torch.empty((1, 2, 2, 4), dtype=torch.int8, device=DEV)
+    iq.iq_ce_grad(dev(z), dscal(2.0), dev(lab), E2, se)
+    ref, sref, _ = O.ce_grad(z, 2.0, lab)
+    assert np.array_equal(host(E2), ref) and host(se)[0] == sref
+
+
+# ---------------------------------------------------------------- BN parameter update
+
+def test_bn_update_matches_oracle():
+    g = np.random.default_rng(20)
+    c = 300
+    gm = g.integers(-(2 ** 23) + 1, 2 ** 23, size=c).astype(np.int32)
+    bm = g.integers(-(2 ** 23) + 1, 2 ** 23, size=c).astype(np.int32)
+    dgam = g.integers(-(2 ** 35), 2 ** 35, size=c).astype(np.int64)
+    dbet = g.integers(-(2 ** 20), 2 ** 20, size=c).astype(np.int64)
+    s_e, s_x = 0.0123, 2.0 ** -15 * 1.7
+    bn_scales = np.zeros(8, np.float64)
+    bn_scales[0] = s_x
+    dgm, dbm = dev(gm), dev(bm)
+    dg, db = torch.empty(c, dtype=torch.int32, device=DEV), torch.empty(c, dtype=torch.int32, device=DEV)
+    seed, layer, step, lr = 5, 17, 3, 8
+    iq.iq_bn_update(dgm, dbm, dg, db, dev(dgam), dev(dbet), dscal(s_e), dev(bn_scales), lr, seed,
+                    layer, step)
+    qg, sg = O.rq_int(dgam, s_e * s_x, 8, 1, seed, layer, step, tag=1)
+    qb, sb = O.rq_int(dbet, s_e, 8, 1, seed, layer, step, tag=2)
+    rgm, rg = O.update(gm, qg, sg, lr, x2=True)
+    rbm, rb = O.update(bm, qb, sb, lr, x2=True)
+    assert np.array_equal(host(dgm), rgm) and np.array_equal(host(dg), rg)
+    assert np.array_equal(host(dbm), rbm) and np.array_equal(host(db), rb)
