@@ -9,6 +9,8 @@ uint8 RGB images, per-pixel class labels with an ignore value).
 """
 from __future__ import annotations
 
+from dataclasses import dataclass
+
 import numpy as np
 
 
@@ -120,3 +122,106 @@ def labels_voronoi(g: np.random.Generator, n: int, h: int, w: int, classes: int,
 
 def float_uniform(g: np.random.Generator, shape, lo: float = -1.0, hi: float = 1.0) -> np.ndarray:
     return g.uniform(lo, hi, size=shape).astype(np.float32)
+
+
+# ---------------------------------------------------------------- DeepLabv3-ResNet50
+
+@dataclass
+class ConvSpec:
+    """One convolution of the network: KRSC weights [cout][r][r][cin], square kernel."""
+    name: str
+    cin: int
+    cout: int
+    r: int
+    stride: int = 1
+    pad: int = 0
+    dil: int = 1
+    bn: bool = True
+
+
+@dataclass
+class Bottleneck:
+    name: str
+    conv1: ConvSpec
+    conv2: ConvSpec
+    conv3: ConvSpec
+    down: ConvSpec = None          # 1x1 projection shortcut (first block of a stage)
+
+
+@dataclass
+class DeepLabSpec:
+    classes: int
+    stem: ConvSpec                 # 7x7 stride 2, then 3x3 stride 2 max pool (padding 1)
+    blocks: list
+    aspp: list                     # 1x1 branch and the three atrous 3x3 branches
+    pool_conv: ConvSpec            # image-pooling branch: global mean -> 1x1 conv
+    project: ConvSpec              # 1x1 over the concatenation
+    head: ConvSpec                 # 3x3
+    cls: ConvSpec                  # 1x1 classifier, no BN, no ReLU
+    up: int = 8                    # bilinear factor, aligned corners
+
+    def convs(self):
+        """Every convolution in forward order (the layer ids of the RNG key)."""
+        out = [self.stem]
+        for b in self.blocks:
+            out += [b.conv1, b.conv2, b.conv3] + ([b.down] if b.down else [])
+        return out + list(self.aspp) + [self.pool_conv, self.project, self.head, self.cls]
+
+
+def deeplabv3_r50_spec(classes: int = 21, width: float = 1.0, blocks=(3, 4, 6, 3),
+                       rates=(12, 24, 36)) -> DeepLabSpec:
+    """DeepLabv3 on ResNet-50 at output stride 8: stages of (3, 4, 6, 3) bottlenecks with
+    stride 2 in the 3x3 convolution of stage 2's first block, stages 3 and 4 dilated (2 and
+    4; the first block of each keeps the previous dilation), ASPP with a 1x1 branch, 3x3
+    branches at rates 12/24/36 and an image-pooling branch (256 channels each), a 1x1
+    projection, a 3x3 head and a 1x1 classifier.  width scales every channel count
+    (multiples of 16, at least 16); the input has 4 channels (RGB padded)."""
+    def ch(c):
+        return max(16, int(round(c * width)) // 16 * 16)
+    stem = ConvSpec("stem", 4, ch(64), 7, 2, 3)
+    out_blocks, cin, dil = [], ch(64), 1
+    for si, (nb, mid, stride, new_dil) in enumerate(zip(blocks, (64, 128, 256, 512),
+                                                        (1, 2, 1, 1), (1, 1, 2, 4))):
+        cout = ch(mid * 4)
+        for bi in range(nb):
+            d = dil if bi == 0 else new_dil
+            s = stride if bi == 0 else 1
+            nm = f"layer{si + 1}.{bi}"
+            down = None
+            if bi == 0 and (s != 1 or cin != cout):
+                down = ConvSpec(nm + ".down", cin, cout, 1, s, 0)
+            out_blocks.append(Bottleneck(
+                nm, ConvSpec(nm + ".conv1", cin, ch(mid), 1),
+                ConvSpec(nm + ".conv2", ch(mid), ch(mid), 3, s, d, d),
+                ConvSpec(nm + ".conv3", ch(mid), cout, 1), down))
+            cin = cout
+        dil = new_dil
+    a = ch(256)
+    aspp = [ConvSpec("aspp.b0", cin, a, 1)] + [
+        ConvSpec(f"aspp.b{i + 1}", cin, a, 3, 1, r, r) for i, r in enumerate(rates)]
+    return DeepLabSpec(classes, stem, out_blocks, aspp, ConvSpec("aspp.pool", cin, a, 1),
+                       ConvSpec("aspp.project", 5 * a, a, 1), ConvSpec("head", a, a, 3, 1, 1),
+                       ConvSpec("cls", a, classes, 1, bn=False))
+
+
+def deeplabv3_r50_init(seed: int, spec: DeepLabSpec):
+    """Initial parameters: fp32 He weights per conv (input channel 3 of the stem, the RGB
+    padding, zero), and per BN conv the gamma / beta master codes on the 24-bit x2-scaled
+    grid (value m 2^-22), drawn as 8-bit codes (gamma in [0.5, 1.5], beta in [-0.5, 0.5])
+    times 2^16 so that the 8-bit codes the forward uses are exactly the drawn ones."""
+    g = rng(seed)
+    ws, gms, bms = [], [], []
+    for cv in spec.convs():
+        fan_in = (3 if cv.cin == 4 else cv.cin) * cv.r * cv.r
+        w = he_weights(g, (cv.cout, cv.r, cv.r, cv.cin), fan_in)
+        if cv.cin == 4:
+            w[..., 3] = 0.0
+        ws.append(w)
+        if cv.bn:
+            gam, bet = bn_gamma_beta_codes(g, cv.cout)
+            gms.append(gam.astype(np.int32) * np.int32(1 << 16))
+            bms.append(bet.astype(np.int32) * np.int32(1 << 16))
+        else:
+            gms.append(None)
+            bms.append(None)
+    return ws, gms, bms
