@@ -2,6 +2,12 @@
 paper's Sec. 3 dataflow) on synthetic 512x512 segmentation batches.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload fcn_vgg16_train|deeplabv3_r50_train|fcn_vgg16_infer|
+                              deeplabv3_r50_infer]
+
+The default workload is the FCN-VGG16 training step (batch 16, 512x512, 150 classes);
+the others are the DeepLabv3-ResNet50 training step (batch 16, 513x513, 21 classes, 5%
+ignored labels) and the two inference passes (batch 8).
 
 Prints one JSON line.  `value` is the int8 convolution throughput of the whole step in
 TOPS (2 x MACs of every forward, data-gradient and weight-gradient convolution, the
@@ -26,8 +32,69 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-BATCH, IMG, CLASSES, SITES = 16, 512, 150, 64
-WORKLOAD = "fcn_vgg16_train_step"
+SITES = 64
+
+
+class Workload:
+    """One benchmarked configuration: the network, its inputs and what a step counts."""
+
+    def __init__(self, name: str):
+        self.name = name
+        self.fcn = name.startswith("fcn")
+        self.train = name.endswith("train")
+        self.batch = 16 if self.train else 8
+        self.img = 512 if self.fcn else 513
+        self.classes = 150 if self.fcn else 21
+        self.labels = f"voronoi {SITES} sites" if self.fcn else "uniform, 5% ignore (255)"
+
+    def config(self, world: int) -> dict:
+        return {"workload": self.name + "_step" if self.train else self.name,
+                "global_batch": self.batch * world, "image": f"3x{self.img}x{self.img}",
+                "classes": self.classes, "labels": self.labels if self.train else None}
+
+    def inputs(self, g, n, h):
+        from paper_2011_14504_gb300 import synthetic as S
+        img = S.images_u8(g, n, h, h)
+        if not self.train:
+            return img, None
+        if self.fcn:
+            return img, S.labels_voronoi(g, n, h, h, self.classes, sites=SITES)
+        return img, S.labels_uniform_ignore(g, n, h, h, self.classes)
+
+    def build(self, dev, seed):
+        if self.fcn:
+            from paper_2011_14504_gb300.fcn import FcnVgg16
+            return FcnVgg16(self.batch, self.img, self.img, classes=self.classes, seed=seed,
+                            lr_log2=10, device=str(dev), train=self.train)
+        from paper_2011_14504_gb300.deeplab import DeepLabV3R50
+        return DeepLabV3R50(self.batch, self.img, self.img, classes=self.classes, seed=seed,
+                            lr_log2=10, device=str(dev), train=self.train)
+
+    def step(self, net, img, lab):
+        if self.train:
+            net.train_step(img, lab)
+        else:
+            net.forward(img)
+
+    def result(self, net):
+        """The scalar read back every end-to-end step: the loss-gradient scale (training)
+        or the logits scale (inference)."""
+        if self.train:
+            return net.s_Ez if self.fcn else net.s_E
+        return net.s_z
+
+    def macs(self, net) -> int:
+        return net.macs_step if self.train else net.macs_forward
+
+    def conv_macs(self, net) -> dict:
+        """MACs per step of each convolution entry point (the decoder of FCN excluded)."""
+        if self.fcn:
+            layers = [(L.macs, L.layer_id == 0) for L in net.convs]
+        else:
+            layers = [(L.macs, L is net.stem) for L in net.layers.values()]
+        f = sum(m for m, _ in layers)
+        return {"iq_conv_fwd": f, "iq_conv_dgrad": sum(m for m, first in layers if not first),
+                "iq_conv_wgrad": f}
 
 
 def peaks():
@@ -125,25 +192,75 @@ def max_over_ranks(v: float, world: int, device) -> float:
 
 # ------------------------------------------------------------------ oracle (CPU) leg
 
-def oracle_sample_step():
-    """One FCN-VGG16 training step of the CPU oracle on a bounded sample of the workload:
-    one image at 128x128 (the full-width network), about 10-30 s of CPU work."""
-    import numpy as np
-    from oracle.fcn import OracleFcn
+def oracle_sample_step(wl: Workload):
+    """One step of the CPU oracle on a bounded sample of the workload (the full-width
+    network, one image at 128x128 (FCN) or 129x129 (DeepLab), about 10-30 s of CPU work)."""
     from paper_2011_14504_gb300 import synthetic as S
-    n, h = 1, 128
-    chans = S.fcn_vgg16_channels(CLASSES, 1.0)
-    wts, up = S.fcn_vgg16_weights(0, CLASSES, 1.0)
-    ora = OracleFcn(chans, wts, up, CLASSES, seed=0)
     g = S.rng(1)
-    img = S.images_u8(g, n, h, h)
-    lab = S.labels_voronoi(g, n, h, h, CLASSES, sites=SITES)
-    macs = fcn_step_macs(n, h, h, CLASSES)
+    if wl.fcn:
+        from oracle.fcn import OracleFcn
+        n, h = 1, 128
+        chans = S.fcn_vgg16_channels(wl.classes, 1.0)
+        wts, up = S.fcn_vgg16_weights(0, wl.classes, 1.0)
+        ora = OracleFcn(chans, wts, up, wl.classes, seed=0)
+        macs = fcn_step_macs(n, h, h, wl.classes)
+        if not wl.train:
+            macs = fcn_forward_macs(n, h, h, wl.classes)
+        name = "FCN-VGG16"
+    else:
+        from oracle.deeplab import OracleDeepLab
+        n, h = 1, 129
+        sp = S.deeplabv3_r50_spec(wl.classes, 1.0)
+        w, gm, bm = S.deeplabv3_r50_init(0, sp)
+        ora = OracleDeepLab(sp, w, gm, bm, seed=0)
+        macs = deeplab_macs(sp, n, h, wl.train)
+        name = "DeepLabv3-ResNet50"
+    img, lab = wl.inputs(g, n, h)
 
     def run():
         tr = ora.forward(img)
-        ora.backward_update(tr, lab)
-    return run, macs, f"FCN-VGG16 train step, N={n}, {h}x{h}, full width, {CLASSES} classes"
+        if wl.train:
+            ora.backward_update(tr, lab)
+    kind = "train step" if wl.train else "inference"
+    return run, macs, f"{name} {kind}, N={n}, {h}x{h}, full width, {wl.classes} classes"
+
+
+def deeplab_macs(sp, n, h, train):
+    """Forward (+ data and weight gradient) MACs of the DeepLab convolutions for n images of
+    h x h, from the conv geometry alone."""
+    def out(sz, cv):
+        return (sz + 2 * cv.pad - cv.dil * (cv.r - 1) - 1) // cv.stride + 1
+    per = []
+    sz = out(h, sp.stem)
+    per.append((n * sz * sz * sp.stem.cout * 49 * 3, True))
+    sz = (sz + 2 - 3) // 2 + 1
+    for b in sp.blocks:
+        s1 = sz
+        for cv in (b.conv1, b.conv2, b.conv3):
+            o = out(s1, cv)
+            per.append((n * o * o * cv.cout * cv.r * cv.r * cv.cin, False))
+            s1 = o
+        if b.down:
+            per.append((n * s1 * s1 * b.down.cout * b.down.cin, False))
+        sz = s1
+    for cv in list(sp.aspp) + [sp.project, sp.head, sp.cls]:
+        per.append((n * sz * sz * cv.cout * cv.r * cv.r * cv.cin, False))
+    per.append((n * sp.pool_conv.cout * sp.pool_conv.cin, False))
+    f = sum(m for m, _ in per)
+    if not train:
+        return f
+    return f + sum(m for m, first in per if not first) + f
+
+
+def fcn_forward_macs(n, h, w, classes, width=1.0):
+    from paper_2011_14504_gb300 import synthetic as S
+    hh, ww, f = h, w, 0
+    for name, cin, cout, r, pad, relu in S.fcn_vgg16_channels(classes, width):
+        if name == "pool":
+            hh, ww = hh // 2, ww // 2
+            continue
+        f += n * hh * ww * cout * r * r * (3 if cin == 4 else cin)
+    return f + n * h * w * classes * 4
 
 
 def fcn_step_macs(n, h, w, classes, width=1.0):
@@ -174,7 +291,8 @@ def run_reference(args, rank, world):
         return 0
     import oracle
     oracle.build()
-    run, macs, sample = oracle_sample_step()
+    wl = Workload(args.workload)
+    run, macs, sample = oracle_sample_step(wl)
     for _ in range(min(args.warmup, 1)):
         run()
     times = []
@@ -184,17 +302,20 @@ def run_reference(args, rank, world):
         times.append(time.perf_counter() - t0)
     t = sum(times) / len(times)
     v = 2 * macs / t / 1e12
-    line = {"impl": "reference", "metric": "int8 conv TOPS (fwd+bwd)", "value": v, "unit": "TOPS",
+    line = {"impl": "reference", "metric": metric_name(wl), "value": v, "unit": "TOPS",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int8", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "global_batch": BATCH * args.gpus,
-                       "image": f"3x{IMG}x{IMG}", "classes": CLASSES},
+            "config": wl.config(args.gpus),
             "cpu_baseline": {"value": v, "unit": "TOPS", "cores": cpu_threads(), "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": v, "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
+
+
+def metric_name(wl: Workload) -> str:
+    return "int8 conv TOPS (fwd+bwd)" if wl.train else "int8 conv TOPS (fwd)"
 
 
 # ------------------------------------------------------------------ GPU leg
@@ -205,17 +326,16 @@ def run_ours(args, rank, world, local):
 
     from paper_2011_14504_gb300 import iq
     from paper_2011_14504_gb300 import synthetic as S
-    from paper_2011_14504_gb300.fcn import FcnVgg16
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     iq.load()
-    net = FcnVgg16(BATCH, IMG, IMG, classes=CLASSES, seed=rank, lr_log2=10, device=str(dev))
+    wl = Workload(args.workload)
+    net = wl.build(dev, rank)
     g = S.rng(1000 + rank)
-    img_np = S.images_u8(g, BATCH, IMG, IMG)
-    lab_np = S.labels_voronoi(g, BATCH, IMG, IMG, CLASSES, sites=SITES)
+    img_np, lab_np = wl.inputs(g, wl.batch, wl.img)
     img = torch.from_numpy(img_np).to(dev)
-    lab = torch.from_numpy(lab_np).to(dev)
+    lab = torch.from_numpy(lab_np).to(dev) if lab_np is not None else None
     stream = torch.cuda.current_stream(dev)
 
     # per-operation attribution with events on the launching stream
@@ -232,13 +352,12 @@ def run_ours(args, rank, world, local):
         return wrap
 
     for _ in range(args.warmup):
-        net.train_step(img, lab)
+        wl.step(net, img, lab)
     torch.cuda.synchronize(dev)
 
     orig = {k: getattr(iq, k) for k in ("iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad")}
-    import paper_2011_14504_gb300.fcn as fcn_mod
     for k, f in orig.items():
-        setattr(fcn_mod.iq, k, timed(k, f))
+        setattr(iq, k, timed(k, f))
     launches0 = iq.launch_count()
     barrier(world)
     torch.cuda.synchronize(dev)
@@ -247,17 +366,17 @@ def run_ours(args, rank, world, local):
         t_end = torch.cuda.Event(enable_timing=True)
         t_start.record(stream)
         for _ in range(args.steps):
-            net.train_step(img, lab)
+            wl.step(net, img, lab)
         t_end.record(stream)
         torch.cuda.synchronize(dev)
     barrier(world)
     launches = iq.launch_count() - launches0
     for k, f in orig.items():
-        setattr(fcn_mod.iq, k, f)
+        setattr(iq, k, f)
     ms_total = t_start.elapsed_time(t_end)
     ms_total = max_over_ranks(ms_total, world, dev)
     ms_step = ms_total / args.steps
-    macs = net.macs_step
+    macs = wl.macs(net)
     tops = 2 * macs * world / (ms_step * 1e-3) / 1e12
 
     # roofline of the dominant conv operation (per-call event durations)
@@ -265,9 +384,7 @@ def run_ours(args, rank, world, local):
     for kind, evs in op_events.items():
         per[kind] = sum(e0.elapsed_time(e1) for e0, e1, _ in evs)
     dom = max(per, key=per.get)
-    conv_macs = {"iq_conv_fwd": sum(L.macs for L in net.convs),
-                 "iq_conv_dgrad": sum(L.macs for L in net.convs if L.layer_id > 0),
-                 "iq_conv_wgrad": sum(L.macs for L in net.convs)}
+    conv_macs = wl.conv_macs(net)
     n_calls = len(op_events[dom]) // args.steps
     ms_call = per[dom] / len(op_events[dom])
     flops_call = 2 * conv_macs[dom] / n_calls
@@ -282,10 +399,10 @@ def run_ours(args, rank, world, local):
 
     # end to end: host (pinned) inputs copied in, a result scalar read back, every step
     img_h = torch.from_numpy(img_np).pin_memory()
-    lab_h = torch.from_numpy(lab_np).pin_memory()
+    lab_h = torch.from_numpy(lab_np).pin_memory() if lab is not None else None
     res_h = torch.empty(1, dtype=torch.float64).pin_memory()
     img_d = torch.empty_like(img)
-    lab_d = torch.empty_like(lab)
+    lab_d = torch.empty_like(lab) if lab is not None else None
     e2e_steps = max(1, min(args.steps, 3))
     barrier(world)
     torch.cuda.synchronize(dev)
@@ -294,9 +411,10 @@ def run_ours(args, rank, world, local):
     e0.record(stream)
     for _ in range(e2e_steps):
         img_d.copy_(img_h, non_blocking=True)
-        lab_d.copy_(lab_h, non_blocking=True)
-        net.train_step(img_d, lab_d)
-        res_h.copy_(net.s_Ez, non_blocking=True)     # max |z s_z - onehot| / 127
+        if lab_d is not None:
+            lab_d.copy_(lab_h, non_blocking=True)
+        wl.step(net, img_d, lab_d)
+        res_h.copy_(wl.result(net), non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize(dev)
     ms_e2e = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world, dev)
@@ -307,7 +425,7 @@ def run_ours(args, rank, world, local):
         try:
             import oracle
             oracle.build()
-            run, omacs, sample = oracle_sample_step()
+            run, omacs, sample = oracle_sample_step(wl)
             t0 = time.perf_counter()
             run()
             t = time.perf_counter() - t0
@@ -316,19 +434,19 @@ def run_ours(args, rank, world, local):
         except Exception as ex:   # the GPU number stands on its own
             cpu = {"value": None, "unit": "TOPS", "cores": cpu_threads(), "kind": "oracle",
                    "sample": f"failed: {ex}"}
-        line = {"metric": "int8 conv TOPS (fwd+bwd)", "value": tops, "unit": "TOPS",
+        cfg = wl.config(world)
+        cfg.update({"macs_per_image_step": macs // wl.batch, "parallelism": f"replicas x{world}",
+                    "l2": "working set >> 129 MB L2, no flush"})
+        line = {"metric": metric_name(wl), "value": tops, "unit": "TOPS",
                 "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
                 "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "int8", "data": "synthetic",
-                "images_per_s": BATCH * world / (ms_step * 1e-3),
-                "config": {"workload": WORKLOAD, "global_batch": BATCH * world,
-                           "image": f"3x{IMG}x{IMG}", "classes": CLASSES,
-                           "labels": f"voronoi {SITES} sites", "macs_per_image_step":
-                               macs // BATCH, "parallelism": f"replicas x{world}",
-                           "l2": "working set >> 129 MB L2, no flush"},
+                "images_per_s": wl.batch * world / (ms_step * 1e-3),
+                "config": cfg,
                 "e2e": {"value": tops_e2e, "unit": "TOPS",
-                        "h2d_bytes_per_step": img_h.numel() + lab_h.numel(),
-                        "d2h_bytes_per_step": 8, "images_per_s": BATCH * world /
+                        "h2d_bytes_per_step": img_h.numel() + (lab_h.numel() if lab_h is not None
+                                                               else 0),
+                        "d2h_bytes_per_step": 8, "images_per_s": wl.batch * world /
                         (ms_e2e * 1e-3)},
                 "gpu_launches": launches,
                 "roofline": roofline,
@@ -344,6 +462,9 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="fcn_vgg16_train",
+                    choices=["fcn_vgg16_train", "deeplabv3_r50_train", "fcn_vgg16_infer",
+                             "deeplabv3_r50_infer"])
     args = ap.parse_args()
     rank, world, local = dist_setup(args.gpus)
     if args.impl == "reference":
