@@ -67,6 +67,7 @@ BnStats bn_stats_carve(WsCursor& cur, int32_t C) {
     s.codes = cur.take<int>(2 * (size_t)C);
     s.px = cur.take<int>(4);
     s.scal = cur.take<double>(IQ_BN_SCALES);
+    s.red = cur.take<unsigned long long>(8);
     return s;
 }
 
@@ -74,6 +75,8 @@ __global__ void k_bn_init(BnStats s, int32_t C) {
     for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < C; c += gridDim.x * blockDim.x) {
         s.s1[c] = 0; s.dev[c] = 0; s.ngt[c] = 0;
         s.hi[c] = INT_MIN; s.lo[c] = INT_MAX;
+        if (c == 0)
+            for (int i = 0; i < 8; i++) s.red[i] = 0ull;
     }
 }
 
@@ -192,20 +195,6 @@ __global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__
 
 // ------------------------------------------------------------------ finalize (one block)
 
-__device__ double block_max_d(double v, double* sh) {
-    // v >= 0 on every thread
-    for (int o = 16; o > 0; o >>= 1) v = fmax(v, __shfl_xor_sync(0xffffffffu, v, o));
-    int w = threadIdx.x >> 5, l = threadIdx.x & 31;
-    __syncthreads();
-    if (l == 0) sh[w] = v;
-    __syncthreads();
-    double r = 0.0;
-    int nw = (blockDim.x + 31) >> 5;
-    for (int i = 0; i < nw; i++) r = fmax(r, sh[i]);
-    __syncthreads();
-    return r;
-}
-
 __device__ __forceinline__ int frexp_exp(double v) {
     int e;
     frexp(v, &e);
@@ -215,107 +204,158 @@ __device__ __forceinline__ int frexp_exp(double v) {
 // The fp64 steps below follow the oracle's operation order one for one:
 // mu_B = (S1 s_acc)/m, sigma_B = (T s_acc)/(m m), codes by rhu of v 2^(k-2),
 // xhat(v) = (v s_acc - mu_q)/den, a_c = (s_acc/den) qx, b_c = (-mu_q/den) qx, ...
-__global__ void __launch_bounds__(1024) k_bn_finalize(
-    BnStats s, int64_t m, int32_t C, const double* __restrict__ s_acc_p,
-    const int32_t* __restrict__ gam, const int32_t* __restrict__ bet, iq_bn_bits b,
-    int32_t* __restrict__ codes /* [2C] c_mu, c_sigma */) {
-    __shared__ double red[32];
+// The per-channel work is spread over C/64 blocks of 64 threads (the fp64 pipe of one SM
+// is narrow); each tensor-wide maximum of non-negative doubles is an atomicMax on its bit
+// pattern, and every stage that needs one is a separate launch.
+constexpr int kFinThreads = 64;
+
+__device__ __forceinline__ void red_max(unsigned long long* cell, double v) {
+    if (v > 0.0) atomicMax(cell, (unsigned long long)__double_as_longlong(v));
+}
+__device__ __forceinline__ double red_get(const unsigned long long* cell) {
+    return __longlong_as_double((long long)*cell);
+}
+
+// stage 1: mu_q / sigma_q codes; max |xhat| at the channel extremes (red[0]); max |acc| (red[1])
+__global__ void __launch_bounds__(kFinThreads) k_bn_fin1(BnStats s, int64_t m, int32_t C,
+                                                         const double* __restrict__ s_acc_p,
+                                                         iq_bn_bits b) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= C) return;
     const double s_acc = *s_acc_p;
     const double md = (double)m;
     const double mu_step = ldexp(1.0, 2 - b.k_mu), sg_step = ldexp(1.0, 2 - b.k_sigma);
-    double mx = 0.0, vmax = 0.0;
-    for (int c = threadIdx.x; c < C; c += blockDim.x) {
-        int64_t S1 = (int64_t)s.s1[c];
-        int64_t f = floordiv_i64(S1, m);
-        int64_t rho = S1 - f * m;
-        i128 T = (i128)m * (i128)(int64_t)s.dev[c] + (i128)rho * (i128)(m - 2 * (int64_t)s.ngt[c]);
-        double mu_b = __ddiv_rn(__dmul_rn((double)S1, s_acc), md);
-        double sg_b = __ddiv_rn(__dmul_rn(u128_to_double((u128)T), s_acc), __dmul_rn(md, md));
-        int64_t cm = code_of(ldexp(mu_b, b.k_mu - 2), b.k_mu);
-        int64_t cs = code_of(ldexp(sg_b, b.k_sigma - 2), b.k_sigma);
-        codes[c] = (int32_t)cm;
-        codes[C + c] = (int32_t)cs;
-        double muq = __dmul_rn((double)cm, mu_step);
-        double den = __dmul_rn((double)(cs + 1), sg_step);
-        double xh = __ddiv_rn(__dsub_rn(__dmul_rn((double)s.hi[c], s_acc), muq), den);
-        double xl = __ddiv_rn(__dsub_rn(__dmul_rn((double)s.lo[c], s_acc), muq), den);
-        mx = fmax(mx, fmax(fabs(xh), fabs(xl)));
-        vmax = fmax(vmax, fmax(fabs((double)s.hi[c]), fabs((double)s.lo[c])));
-    }
-    __syncthreads();
-    mx = block_max_d(mx, red);
-    vmax = block_max_d(vmax, red);
+    int64_t S1 = (int64_t)s.s1[c];
+    int64_t f = floordiv_i64(S1, m);
+    int64_t rho = S1 - f * m;
+    i128 T = (i128)m * (i128)(int64_t)s.dev[c] + (i128)rho * (i128)(m - 2 * (int64_t)s.ngt[c]);
+    double mu_b = __ddiv_rn(__dmul_rn((double)S1, s_acc), md);
+    double sg_b = __ddiv_rn(__dmul_rn(u128_to_double((u128)T), s_acc), __dmul_rn(md, md));
+    int64_t cm = code_of(ldexp(mu_b, b.k_mu - 2), b.k_mu);
+    int64_t cs = code_of(ldexp(sg_b, b.k_sigma - 2), b.k_sigma);
+    s.codes[c] = (int32_t)cm;
+    s.codes[C + c] = (int32_t)cs;
+    double muq = __dmul_rn((double)cm, mu_step);
+    double den = __dmul_rn((double)(cs + 1), sg_step);
+    double xh = __ddiv_rn(__dsub_rn(__dmul_rn((double)s.hi[c], s_acc), muq), den);
+    double xl = __ddiv_rn(__dsub_rn(__dmul_rn((double)s.lo[c], s_acc), muq), den);
+    red_max(&s.red[0], fmax(fabs(xh), fabs(xl)));
+    red_max(&s.red[1], fmax(fabs((double)s.hi[c]), fabs((double)s.lo[c])));
+}
+
+__device__ __forceinline__ void bn_xmap(const BnStats& s, int c, int32_t C, double s_acc,
+                                        double qx, const iq_bn_bits& b, double* a, double* bb) {
+    const double mu_step = ldexp(1.0, 2 - b.k_mu), sg_step = ldexp(1.0, 2 - b.k_sigma);
+    double muq = __dmul_rn((double)s.codes[c], mu_step);
+    double den = __dmul_rn((double)(s.codes[C + c] + 1), sg_step);
+    *a = __dmul_rn(__ddiv_rn(s_acc, den), qx);
+    *bb = __dmul_rn(__ddiv_rn(-muq, den), qx);
+}
+
+// stage 2: the bound of the acc -> X map (red[2])
+__global__ void __launch_bounds__(kFinThreads) k_bn_fin2(BnStats s, int32_t C,
+                                                         const double* __restrict__ s_acc_p,
+                                                         iq_bn_bits b) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    const double mx = red_get(&s.red[0]);
+    if (c >= C || !(mx > 0.0)) return;
+    const double qx = __ddiv_rn(ldexp(1.0, b.k_xhat - 1), mx);
+    double a, bb;
+    bn_xmap(s, c, C, *s_acc_p, qx, b, &a, &bb);
+    red_max(&s.red[2], __dadd_rn(__dmul_rn(fabs(a), red_get(&s.red[1])), fabs(bb)));
+}
+
+__device__ __forceinline__ int shift_of(double lmax) {
+    int p = 62 - frexp_exp(__dadd_rn(lmax, 1.0));
+    return p > 62 ? 62 : (p < 1 ? 1 : p);
+}
+
+// stage 3: F, B with the shift P_x; max ReLU(y) at the channel extremes (red[3])
+__global__ void __launch_bounds__(kFinThreads) k_bn_fin3(BnStats s, int32_t C,
+                                                         const double* __restrict__ s_acc_p,
+                                                         const int32_t* __restrict__ gam,
+                                                         const int32_t* __restrict__ bet,
+                                                         iq_bn_bits b) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= C) return;
+    const double mx = red_get(&s.red[0]);
     const double s_xhat = mx > 0.0 ? ldexp(mx, 1 - b.k_xhat) : ldexp(1.0, 1 - b.k_xhat);
     const int64_t xq = qmax(b.k_xhat);
     int px = 1;
     if (mx > 0.0) {
         const double qx = __ddiv_rn(ldexp(1.0, b.k_xhat - 1), mx);
-        double lmax = 0.0;
-        for (int c = threadIdx.x; c < C; c += blockDim.x) {
-            double muq = __dmul_rn((double)codes[c], mu_step);
-            double den = __dmul_rn((double)(codes[C + c] + 1), sg_step);
-            double a = __dmul_rn(__ddiv_rn(s_acc, den), qx);
-            double bb = __dmul_rn(__ddiv_rn(-muq, den), qx);
-            lmax = fmax(lmax, __dadd_rn(__dmul_rn(fabs(a), vmax), fabs(bb)));
-        }
-        lmax = block_max_d(lmax, red);
-        px = 62 - frexp_exp(__dadd_rn(lmax, 1.0));
-        px = px > 62 ? 62 : (px < 1 ? 1 : px);
-        for (int c = threadIdx.x; c < C; c += blockDim.x) {
-            double muq = __dmul_rn((double)codes[c], mu_step);
-            double den = __dmul_rn((double)(codes[C + c] + 1), sg_step);
-            double a = __dmul_rn(__ddiv_rn(s_acc, den), qx);
-            double bb = __dmul_rn(__ddiv_rn(-muq, den), qx);
-            s.F[c] = (long long)rhu(ldexp(a, px));
-            s.B[c] = (long long)rhu(ldexp(bb, px)) + (1LL << (px - 1));
-        }
+        px = shift_of(red_get(&s.red[2]));
+        double a, bb;
+        bn_xmap(s, c, C, *s_acc_p, qx, b, &a, &bb);
+        s.F[c] = (long long)rhu(ldexp(a, px));
+        s.B[c] = (long long)rhu(ldexp(bb, px)) + (1LL << (px - 1));
     } else {
-        for (int c = threadIdx.x; c < C; c += blockDim.x) { s.F[c] = 0; s.B[c] = 0; }
+        s.F[c] = 0;
+        s.B[c] = 0;
     }
-    __syncthreads();
     const double gstep = ldexp(1.0, 2 - b.k_gamma), bstep = ldexp(1.0, 2 - b.k_beta);
+    const int64_t xs[2] = {s.hi[c], s.lo[c]};
+    const double t1 = __dmul_rn(__dmul_rn((double)gam[c], gstep), s_xhat);
     double my = 0.0;
-    for (int c = threadIdx.x; c < C; c += blockDim.x) {
-        int64_t xs[2] = {s.hi[c], s.lo[c]};
-        double t1 = __dmul_rn(__dmul_rn((double)gam[c], gstep), s_xhat);
-        for (int j = 0; j < 2; j++) {
-            long long t = (long long)s.F[c] * xs[j] + s.B[c];
-            int64_t xc = clamp64(t >> px, -xq, xq);
-            double y = __dadd_rn(__dmul_rn(t1, (double)xc), __dmul_rn((double)bet[c], bstep));
-            my = fmax(my, y);
-        }
+    for (int j = 0; j < 2; j++) {
+        long long t = (long long)s.F[c] * xs[j] + s.B[c];
+        int64_t xc = clamp64(t >> px, -xq, xq);
+        double y = __dadd_rn(__dmul_rn(t1, (double)xc), __dmul_rn((double)bet[c], bstep));
+        my = fmax(my, y);
     }
-    my = block_max_d(my, red);
+    red_max(&s.red[3], my);
+}
+
+// stage 4: the bound of the X -> A map (red[4])
+__global__ void __launch_bounds__(kFinThreads) k_bn_fin4(BnStats s, int32_t C,
+                                                         const int32_t* __restrict__ gam,
+                                                         const int32_t* __restrict__ bet,
+                                                         iq_bn_bits b) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    const double my = red_get(&s.red[3]);
+    if (c >= C || !(my > 0.0)) return;
+    const double mx = red_get(&s.red[0]);
+    const double s_xhat = mx > 0.0 ? ldexp(mx, 1 - b.k_xhat) : ldexp(1.0, 1 - b.k_xhat);
+    const double gstep = ldexp(1.0, 2 - b.k_gamma), bstep = ldexp(1.0, 2 - b.k_beta);
+    const double qa = __ddiv_rn(ldexp(1.0, b.k_a - 1), my);
+    double t1 = __dmul_rn(__dmul_rn((double)gam[c], gstep), s_xhat);
+    double bq = __dmul_rn((double)bet[c], bstep);
+    red_max(&s.red[4], __dadd_rn(__dmul_rn(fabs(__dmul_rn(t1, qa)), (double)qmax(b.k_xhat)),
+                                 fabs(__dmul_rn(bq, qa))));
+}
+
+// stage 5: G, H with the shift P_a; the shifts and scales of the layer
+__global__ void __launch_bounds__(kFinThreads) k_bn_fin5(BnStats s, int32_t C,
+                                                         const double* __restrict__ s_acc_p,
+                                                         const int32_t* __restrict__ gam,
+                                                         const int32_t* __restrict__ bet,
+                                                         iq_bn_bits b) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    const double mx = red_get(&s.red[0]), my = red_get(&s.red[3]);
+    const double s_xhat = mx > 0.0 ? ldexp(mx, 1 - b.k_xhat) : ldexp(1.0, 1 - b.k_xhat);
     const double s_a = my > 0.0 ? ldexp(my, 1 - b.k_a) : ldexp(1.0, 1 - b.k_a);
     int pa = 1;
-    if (my > 0.0) {
-        const double qa = __ddiv_rn(ldexp(1.0, b.k_a - 1), my);
-        double lmax = 0.0;
-        for (int c = threadIdx.x; c < C; c += blockDim.x) {
-            double t1 = __dmul_rn(__dmul_rn((double)gam[c], gstep), s_xhat);
-            double bq = __dmul_rn((double)bet[c], bstep);
-            lmax = fmax(lmax, __dadd_rn(__dmul_rn(fabs(__dmul_rn(t1, qa)), (double)xq),
-                                        fabs(__dmul_rn(bq, qa))));
-        }
-        lmax = block_max_d(lmax, red);
-        pa = 62 - frexp_exp(__dadd_rn(lmax, 1.0));
-        pa = pa > 62 ? 62 : (pa < 1 ? 1 : pa);
-        for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    if (my > 0.0) pa = shift_of(red_get(&s.red[4]));
+    if (c < C) {
+        if (my > 0.0) {
+            const double gstep = ldexp(1.0, 2 - b.k_gamma), bstep = ldexp(1.0, 2 - b.k_beta);
+            const double qa = __ddiv_rn(ldexp(1.0, b.k_a - 1), my);
             double t1 = __dmul_rn(__dmul_rn((double)gam[c], gstep), s_xhat);
             double bq = __dmul_rn((double)bet[c], bstep);
             s.G[c] = (long long)rhu(ldexp(__dmul_rn(t1, qa), pa));
             s.H[c] = (long long)rhu(ldexp(__dmul_rn(bq, qa), pa)) + (1LL << (pa - 1));
+        } else {
+            s.G[c] = 0;
+            s.H[c] = 0;
         }
-    } else {
-        for (int c = threadIdx.x; c < C; c += blockDim.x) { s.G[c] = 0; s.H[c] = 0; }
     }
-    if (threadIdx.x == 0) {
-        s.px[0] = px;
+    if (c == 0) {
+        s.px[0] = mx > 0.0 ? shift_of(red_get(&s.red[2])) : 1;
         s.px[1] = pa;
         s.scal[IQ_BN_S_XHAT] = s_xhat;
         s.scal[IQ_BN_M_XHAT] = mx;
         s.scal[IQ_BN_M_Y] = my;
-        s.scal[IQ_BN_S_ACC] = s_acc;
+        s.scal[IQ_BN_S_ACC] = *s_acc_p;
         s.scal[IQ_BN_S_A] = s_a;
         for (int i = IQ_BN_S_A + 1; i < IQ_BN_SCALES; i++) s.scal[i] = 0.0;
     }
@@ -395,7 +435,16 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
     ChanGrid g = chan_grid(m, C / 4);
     k_bn_dev<<<g.blocks, kThreads, 0, st>>>(acc, m, C, s);
     IQ_LAUNCH_CHECK();
-    k_bn_finalize<<<1, 1024, 0, st>>>(s, m, C, s_acc, gamma, beta, b, s.codes);
+    const int fb = (C + kFinThreads - 1) / kFinThreads;
+    k_bn_fin1<<<fb, kFinThreads, 0, st>>>(s, m, C, s_acc, b);
+    IQ_LAUNCH_CHECK();
+    k_bn_fin2<<<fb, kFinThreads, 0, st>>>(s, C, s_acc, b);
+    IQ_LAUNCH_CHECK();
+    k_bn_fin3<<<fb, kFinThreads, 0, st>>>(s, C, s_acc, gamma, beta, b);
+    IQ_LAUNCH_CHECK();
+    k_bn_fin4<<<fb, kFinThreads, 0, st>>>(s, C, gamma, beta, b);
+    IQ_LAUNCH_CHECK();
+    k_bn_fin5<<<fb, kFinThreads, 0, st>>>(s, C, s_acc, gamma, beta, b);
     IQ_LAUNCH_CHECK();
     ChanGrid g2 = chan_grid(m, C / 4, 152 * 16);
     k_bn_requant<<<g2.blocks, kThreads, 0, st>>>(acc, m, C, s, b.k_xhat, b.k_a, xhat, a);
@@ -413,6 +462,17 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
 // fin 2 : d x_i = w_c (E_2 + kap_c sgn + lam_c); M = max |d x|; fixed-point SQ8 map
 // pass 3: e = clip(floor((fw E_2 + fk sgn + fl) / 2^P))
 
+// Division by 2M for E_2 = SQ(z, k_e2): the numerator 2^k (z + M) + M is below 2^32 for the
+// paper's widths (|z| <= 127 * 127, k_e2 <= 16), where a 32-bit invariant divisor (Granlund
+// & Montgomery, Sec. 4, at N = 32) replaces the 64-bit one.
+struct E2Div {
+    uint64_t M;
+    UDiv div;          // 64-bit divisor by 2M
+    uint32_t mp;       // 32-bit multiplier, shifts
+    int32_t sh1, sh2;
+    int32_t use32;
+};
+
 struct BnBwd {
     unsigned long long* sb;   // sum e_y
     unsigned long long* sg;   // sum e_y X
@@ -426,8 +486,12 @@ struct BnBwd {
     long long* fl;
     unsigned* zmax;           // [1]
     int* pe;                  // [1]
-    RqDiv* e2div;             // [1]
+    E2Div* e2div;             // [1]
     double* scal;             // [2]: s_e2, s_out
+    double* kap;              // [C] per-channel constants of d x (fin 2)
+    double* lam;
+    double* wc;
+    unsigned long long* red;  // [4]: maxima of non-negative doubles (bit patterns)
 };
 
 static BnBwd bnb_carve(WsCursor& cur, int32_t C) {
@@ -444,8 +508,12 @@ static BnBwd bnb_carve(WsCursor& cur, int32_t C) {
     w.fl = cur.take<long long>(C);
     w.zmax = cur.take<unsigned>(1);
     w.pe = cur.take<int>(1);
-    w.e2div = cur.take<RqDiv>(1);
+    w.e2div = cur.take<E2Div>(1);
     w.scal = cur.take<double>(2);
+    w.kap = cur.take<double>(C);
+    w.lam = cur.take<double>(C);
+    w.wc = cur.take<double>(C);
+    w.red = cur.take<unsigned long long>(4);
     return w;
 }
 
@@ -453,7 +521,10 @@ __global__ void k_bnb_init(BnBwd w, int32_t C) {
     for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < C; c += gridDim.x * blockDim.x) {
         w.sb[c] = 0; w.sg[c] = 0; w.se[c] = 0; w.sex[c] = 0; w.ss[c] = 0;
         for (int j = 0; j < 3; j++) { w.emin[3 * c + j] = INT_MAX; w.emax[3 * c + j] = INT_MIN; }
-        if (c == 0) *w.zmax = 0;
+        if (c == 0) {
+            *w.zmax = 0;
+            for (int i = 0; i < 4; i++) w.red[i] = 0ull;
+        }
     }
 }
 
@@ -493,7 +564,7 @@ __global__ void __launch_bounds__(kThreads) k_bnb_pass1(const int8_t* __restrict
         for (int j = 0; j < 4; j++) {
             int ey = am[j] > 0 ? e[j] : 0;
             sb[j] += ey;
-            sg[j] += (long long)ey * x[j];
+            sg[j] += (long long)(ey * x[j]);     // |ey x| < 2^22
             int z = ey * gm[j];
             zm = max(zm, (uint32_t)(z < 0 ? -z : z));
         }
@@ -520,16 +591,30 @@ __global__ void k_bnb_fin1(BnBwd w, const double* __restrict__ s_e, int k_gamma,
     uint32_t M2 = *w.zmax;
     double s_z = __dmul_rn(*s_e, ldexp(1.0, 2 - k_gamma));
     w.scal[0] = M2 ? ldexp(__dmul_rn(s_z, (double)M2), 1 - k_e2) : ldexp(s_z, 1 - k_e2);
-    RqDiv d;
+    E2Div d;
     d.M = M2;
-    d.div = make_udiv(M2 ? 2ull * M2 : 1ull);
+    const uint64_t dv = M2 ? 2ull * M2 : 1ull;
+    d.div = make_udiv(dv);
+    int l = 0;
+    while ((uint64_t(1) << l) < dv) l++;
+    d.use32 = (((uint64_t)2 * M2) << k_e2) + M2 < (uint64_t(1) << 32) && l <= 31;
+    d.mp = d.use32 ? (uint32_t)((((uint64_t(1) << l) - dv) << 32) / dv + 1) : 0u;
+    d.sh1 = l < 1 ? l : 1;
+    d.sh2 = l - 1 > 0 ? l - 1 : 0;
     *w.e2div = d;
 }
 
-__device__ __forceinline__ int e2_code(int z, const RqDiv& d, int k) {
+__device__ __forceinline__ int e2_code(int z, const E2Div& d, int k) {
     if (!d.M) return 0;
-    uint64_t num = ((uint64_t)((int64_t)z + (int64_t)d.M) << k) + d.M;
-    int64_t c = (int64_t)udiv(num, d.div) - (int64_t(1) << (k - 1));
+    int64_t c;
+    if (d.use32) {
+        const uint32_t num = ((uint32_t)(z + (int32_t)d.M) << k) + (uint32_t)d.M;
+        const uint32_t t = __umulhi(d.mp, num);
+        c = (int64_t)((t + ((num - t) >> d.sh1)) >> d.sh2) - (int64_t(1) << (k - 1));
+    } else {
+        uint64_t num = ((uint64_t)((int64_t)z + (int64_t)d.M) << k) + d.M;
+        c = (int64_t)udiv(num, d.div) - (int64_t(1) << (k - 1));
+    }
     return (int)clamp64(c, -qmax(k), qmax(k));
 }
 
@@ -548,7 +633,7 @@ __global__ void __launch_bounds__(kThreads) k_bnb_pass2(const int8_t* __restrict
             for (int j = 0; j < 3; j++) { sh_mn[3 * c + j] = INT_MAX; sh_mx[3 * c + j] = INT_MIN; }
         }
     __syncthreads();
-    const RqDiv d = *w.e2div;
+    const E2Div d = *w.e2div;
     const int64_t T = (int64_t)gridDim.x * blockDim.x;
     const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int g = (int)(t % C4);
@@ -571,7 +656,7 @@ __global__ void __launch_bounds__(kThreads) k_bnb_pass2(const int8_t* __restrict
             int e2 = e2_code(ey * gm[j], d, k_e2);
             int sgn = (x[j] > 0) - (x[j] < 0);
             se[j] += e2;
-            sx[j] += (long long)e2 * x[j];
+            sx[j] += (long long)(e2 * x[j]);     // |E_2 X| < 2^30
             ss[j] += sgn;
             int q = sgn + 1;
 #pragma unroll
@@ -606,69 +691,71 @@ __global__ void __launch_bounds__(kThreads) k_bnb_pass2(const int8_t* __restrict
 }
 
 // Per channel (oracle order): gx = (SEX s_x)/m; kap = -gx; lam = gx (SS/m) - SE/m;
-// w = s_e2 / ((c_sigma + 1) sg_step); d x = w ((E_2 + kap sgn) + lam).
-__global__ void __launch_bounds__(1024) k_bnb_fin2(BnBwd w, int64_t m, int32_t C,
-                                                   const int32_t* __restrict__ csig,
-                                                   const double* __restrict__ bn_scales,
-                                                   int k_sigma, int k_e2, int k_e,
-                                                   double* __restrict__ s_out) {
-    __shared__ double red[32];
+// w = s_e2 / ((c_sigma + 1) sg_step); d x = w ((E_2 + kap sgn) + lam).  Three launches of
+// C/64 blocks: M = max |d x| at the extremes of each sign class (red[0]), then the bound of
+// the fixed-point map (red[1]), then its constants.
+__global__ void __launch_bounds__(kFinThreads) k_bnb_fin2a(BnBwd w, int64_t m, int32_t C,
+                                                           const int32_t* __restrict__ csig,
+                                                           const double* __restrict__ bn_scales,
+                                                           int k_sigma) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= C) return;
     const double md = (double)m;
     const double s_x = bn_scales[IQ_BN_S_XHAT];
     const double s_e2 = w.scal[0];
     const double sg_step = ldexp(1.0, 2 - k_sigma);
+    double gx = __ddiv_rn(__dmul_rn((double)(long long)w.sex[c], s_x), md);
+    double kap = -gx;
+    double lam = __dsub_rn(__dmul_rn(gx, __ddiv_rn((double)(long long)w.ss[c], md)),
+                           __ddiv_rn((double)(long long)w.se[c], md));
+    double wc = __ddiv_rn(s_e2, __dmul_rn((double)(csig[c] + 1), sg_step));
+    w.kap[c] = kap;
+    w.lam[c] = lam;
+    w.wc[c] = wc;
     double M = 0.0;
-    for (int c = threadIdx.x; c < C; c += blockDim.x) {
-        double gx = __ddiv_rn(__dmul_rn((double)(long long)w.sex[c], s_x), md);
-        double kap = -gx;
-        double lam = __dsub_rn(__dmul_rn(gx, __ddiv_rn((double)(long long)w.ss[c], md)),
-                               __ddiv_rn((double)(long long)w.se[c], md));
-        double wc = __ddiv_rn(s_e2, __dmul_rn((double)(csig[c] + 1), sg_step));
-        for (int q = 0; q < 3; q++) {
-            int lo = w.emin[3 * c + q], hi = w.emax[3 * c + q];
-            if (lo > hi) continue;  // empty sign class
-            double sg = (double)(q - 1);
-            double ks = __dmul_rn(kap, sg);
-            double d0 = __dmul_rn(wc, __dadd_rn(__dadd_rn((double)lo, ks), lam));
-            double d1 = __dmul_rn(wc, __dadd_rn(__dadd_rn((double)hi, ks), lam));
-            M = fmax(M, fmax(fabs(d0), fabs(d1)));
-        }
+    for (int q = 0; q < 3; q++) {
+        int lo = w.emin[3 * c + q], hi = w.emax[3 * c + q];
+        if (lo > hi) continue;  // empty sign class
+        double sg = (double)(q - 1);
+        double ks = __dmul_rn(kap, sg);
+        double d0 = __dmul_rn(wc, __dadd_rn(__dadd_rn((double)lo, ks), lam));
+        double d1 = __dmul_rn(wc, __dadd_rn(__dadd_rn((double)hi, ks), lam));
+        M = fmax(M, fmax(fabs(d0), fabs(d1)));
     }
-    M = block_max_d(M, red);
-    if (M == 0.0) {
-        for (int c = threadIdx.x; c < C; c += blockDim.x) { w.fw[c] = 0; w.fk[c] = 0; w.fl[c] = 0; }
-        if (threadIdx.x == 0) { *w.pe = 1; w.scal[1] = ldexp(1.0, 1 - k_e); *s_out = w.scal[1]; }
-        return;
-    }
+    red_max(&w.red[0], M);
+}
+
+__global__ void __launch_bounds__(kFinThreads) k_bnb_fin2b(BnBwd w, int32_t C, int k_e2, int k_e) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    const double M = red_get(&w.red[0]);
+    if (c >= C || M == 0.0) return;
     const double qe = __ddiv_rn(ldexp(1.0, k_e - 1), M);
     const double emax = (double)qmax(k_e2);
-    double lmax = 0.0;
-    for (int c = threadIdx.x; c < C; c += blockDim.x) {
-        double gx = __ddiv_rn(__dmul_rn((double)(long long)w.sex[c], s_x), md);
-        double kap = -gx;
-        double lam = __dsub_rn(__dmul_rn(gx, __ddiv_rn((double)(long long)w.ss[c], md)),
-                               __ddiv_rn((double)(long long)w.se[c], md));
-        double wc = __ddiv_rn(s_e2, __dmul_rn((double)(csig[c] + 1), sg_step));
-        double om = __dmul_rn(wc, qe);
-        double l = __dadd_rn(__dadd_rn(__dmul_rn(fabs(om), emax), fabs(__dmul_rn(om, kap))),
-                             fabs(__dmul_rn(om, lam)));
-        lmax = fmax(lmax, l);
+    const double kap = w.kap[c], lam = w.lam[c];
+    double om = __dmul_rn(w.wc[c], qe);
+    red_max(&w.red[1], __dadd_rn(__dadd_rn(__dmul_rn(fabs(om), emax), fabs(__dmul_rn(om, kap))),
+                                 fabs(__dmul_rn(om, lam))));
+}
+
+__global__ void __launch_bounds__(kFinThreads) k_bnb_fin2c(BnBwd w, int32_t C, int k_e,
+                                                           double* __restrict__ s_out) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    const double M = red_get(&w.red[0]);
+    if (M == 0.0) {
+        if (c < C) { w.fw[c] = 0; w.fk[c] = 0; w.fl[c] = 0; }
+        if (c == 0) { *w.pe = 1; w.scal[1] = ldexp(1.0, 1 - k_e); *s_out = w.scal[1]; }
+        return;
     }
-    lmax = block_max_d(lmax, red);
-    int pe = 62 - frexp_exp(__dadd_rn(lmax, 1.0));
-    pe = pe > 62 ? 62 : (pe < 1 ? 1 : pe);
-    for (int c = threadIdx.x; c < C; c += blockDim.x) {
-        double gx = __ddiv_rn(__dmul_rn((double)(long long)w.sex[c], s_x), md);
-        double kap = -gx;
-        double lam = __dsub_rn(__dmul_rn(gx, __ddiv_rn((double)(long long)w.ss[c], md)),
-                               __ddiv_rn((double)(long long)w.se[c], md));
-        double wc = __ddiv_rn(s_e2, __dmul_rn((double)(csig[c] + 1), sg_step));
-        double om = __dmul_rn(wc, qe);
+    const int pe = shift_of(red_get(&w.red[1]));
+    if (c < C) {
+        const double qe = __ddiv_rn(ldexp(1.0, k_e - 1), M);
+        const double kap = w.kap[c], lam = w.lam[c];
+        double om = __dmul_rn(w.wc[c], qe);
         w.fw[c] = (long long)rhu(ldexp(om, pe));
         w.fk[c] = (long long)rhu(ldexp(__dmul_rn(om, kap), pe));
         w.fl[c] = (long long)rhu(ldexp(__dmul_rn(om, lam), pe)) + (1LL << (pe - 1));
     }
-    if (threadIdx.x == 0) { *w.pe = pe; w.scal[1] = ldexp(M, 1 - k_e); *s_out = w.scal[1]; }
+    if (c == 0) { *w.pe = pe; w.scal[1] = ldexp(M, 1 - k_e); *s_out = w.scal[1]; }
 }
 
 __global__ void __launch_bounds__(kThreads) k_bnb_pass3(const int8_t* __restrict__ ea,
@@ -677,7 +764,7 @@ __global__ void __launch_bounds__(kThreads) k_bnb_pass3(const int8_t* __restrict
                                                         const int32_t* __restrict__ gam,
                                                         int64_t m, int32_t C, int k_e2, int k_e,
                                                         BnBwd w, int8_t* __restrict__ out) {
-    const RqDiv d = *w.e2div;
+    const E2Div d = *w.e2div;
     const int pe = *w.pe;
     const int64_t eq = qmax(k_e);
     const int C4 = C >> 2;
@@ -783,7 +870,12 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     IQ_LAUNCH_CHECK();
     k_bnb_pass2<<<g.blocks, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, k_e2, w);
     IQ_LAUNCH_CHECK();
-    k_bnb_fin2<<<1, 1024, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma, k_e2, 8, s_e_out);
+    const int fb = (c + kFinThreads - 1) / kFinThreads;
+    k_bnb_fin2a<<<fb, kFinThreads, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma);
+    IQ_LAUNCH_CHECK();
+    k_bnb_fin2b<<<fb, kFinThreads, 0, st>>>(w, c, k_e2, 8);
+    IQ_LAUNCH_CHECK();
+    k_bnb_fin2c<<<fb, kFinThreads, 0, st>>>(w, c, 8, s_e_out);
     IQ_LAUNCH_CHECK();
     ChanGrid g3 = chan_grid(m, c / 4, 152 * 16);
     k_bnb_pass3<<<g3.blocks, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, k_e2, 8, w, e);

@@ -186,6 +186,115 @@ __global__ void k_up_fwd(UpP u, const int8_t* __restrict__ x, const int8_t* __re
     }
 }
 
+// 32-bit invariant division (Granlund & Montgomery, Sec. 4, N = 32) for SQ numerators that
+// fit 32 bits: q = floor(n / d) for n < 2^32, 1 <= d < 2^31.
+struct Div32 {
+    uint32_t mp;
+    int sh1, sh2;
+};
+__device__ __forceinline__ Div32 make_div32(uint32_t d) {
+    int l = 0;
+    while ((1u << l) < d && l < 31) l++;
+    if ((1u << l) < d) l = 32;
+    Div32 r;
+    r.mp = (uint32_t)(((((uint64_t)1 << l) - d) << 32) / d + 1);
+    r.sh1 = l < 1 ? l : 1;
+    r.sh2 = l - 1 > 0 ? l - 1 : 0;
+    return r;
+}
+__device__ __forceinline__ uint32_t div32(uint32_t n, const Div32& d) {
+    const uint32_t t = __umulhi(d.mp, n);
+    return (t + ((n - t) >> d.sh1)) >> d.sh2;
+}
+
+// The FCN decoder's shape -- kernel 64, stride 32, padding 16 -- as its own kernel.  Block
+// (q, r1, b) covers the output columns J = 32 q - 16 + t (t < 32) of the output rows
+// I = 32 p - 16 + r1: every such output reads the inputs (row p-1 or p, column q-1 or q)
+// through the taps (r1 + 32 or r1, t + 32 or t).  A thread (one channel) keeps the 4 taps
+// of every t packed in one word, so an output is one dp4a of those with the 4 inputs.
+template <bool CODES>
+__global__ void __launch_bounds__(256) k_up32_fwd(UpP u, const int8_t* __restrict__ x,
+                                                  const int8_t* __restrict__ w,
+                                                  unsigned long long* __restrict__ amax,
+                                                  const RqDiv* __restrict__ dv,
+                                                  int8_t* __restrict__ out,
+                                                  int32_t* __restrict__ acc_out) {
+    const int q = blockIdx.x, r1 = blockIdx.y, b = blockIdx.z, ch = threadIdx.x;
+    const bool act = ch < u.c;
+    uint32_t wt[32];
+    {
+        uint32_t w0[16], w1[16];     // tap rows r1 + 32 (input row p-1) and r1 (input row p)
+#pragma unroll
+        for (int k = 0; k < 4; k++) {
+            int4 a = make_int4(0, 0, 0, 0), c = make_int4(0, 0, 0, 0);
+            if (act) {
+                a = __ldg(reinterpret_cast<const int4*>(w + ((int64_t)ch * 64 + r1 + 32) * 64) + k);
+                c = __ldg(reinterpret_cast<const int4*>(w + ((int64_t)ch * 64 + r1) * 64) + k);
+            }
+            w0[4 * k] = a.x; w0[4 * k + 1] = a.y; w0[4 * k + 2] = a.z; w0[4 * k + 3] = a.w;
+            w1[4 * k] = c.x; w1[4 * k + 1] = c.y; w1[4 * k + 2] = c.z; w1[4 * k + 3] = c.w;
+        }
+        // wt[t] bytes: (w0[t+32], w0[t], w1[t+32], w1[t]) for inputs (p-1,q-1), (p-1,q),
+        // (p,q-1), (p,q)
+#pragma unroll
+        for (int t = 0; t < 32; t++) {
+            const uint32_t sh_hi = 8 * ((t + 32) & 3), sh_lo = 8 * (t & 3);
+            const uint32_t a0 = (w0[(t + 32) >> 2] >> sh_hi) & 0xffu;
+            const uint32_t a1 = (w0[t >> 2] >> sh_lo) & 0xffu;
+            const uint32_t a2 = (w1[(t + 32) >> 2] >> sh_hi) & 0xffu;
+            const uint32_t a3 = (w1[t >> 2] >> sh_lo) & 0xffu;
+            wt[t] = a0 | (a1 << 8) | (a2 << 16) | (a3 << 24);
+        }
+    }
+    uint32_t M = 0;
+    Div32 d32;
+    if (CODES) {
+        M = (uint32_t)dv->M;
+        d32 = make_div32(M ? 2 * M : 1);
+    }
+    uint32_t mx = 0;
+    const int Jb = 32 * q - 16;
+    const int t_lo = Jb < 0 ? -Jb : 0;
+    const int t_hi = Jb + 32 > u.W ? u.W - Jb : 32;
+    for (int p = 0; p <= u.h; p++) {
+        const int I = 32 * p - 16 + r1;
+        if (I < 0 || I >= u.H || !act) continue;
+        const bool rp = p >= 1, rc = p < u.h, cp = q >= 1, cc = q < u.w;
+        auto xin = [&](int i, int j) -> uint32_t {
+            return (uint8_t)x[(((int64_t)b * u.h + i) * u.w + j) * u.c + ch];
+        };
+        const uint32_t x00 = (rp && cp) ? xin(p - 1, q - 1) : 0u;
+        const uint32_t x01 = (rp && cc) ? xin(p - 1, q) : 0u;
+        const uint32_t x10 = (rc && cp) ? xin(p, q - 1) : 0u;
+        const uint32_t x11 = (rc && cc) ? xin(p, q) : 0u;
+        const int xv = (int)(x00 | (x01 << 8) | (x10 << 16) | (x11 << 24));
+        const int64_t row0 = ((int64_t)b * u.H + I) * u.W;
+#pragma unroll
+        for (int t = 0; t < 32; t++) {
+            if (t < t_lo || t >= t_hi) continue;
+            const int64_t o = (row0 + Jb + t) * u.c + ch;
+            const int sum = __dp4a(xv, (int)wt[t], 0);
+            if (CODES) {
+                int c = 0;
+                if (M) {
+                    const uint32_t num = ((uint32_t)(sum + (int)M) << 8) + M;
+                    c = (int)div32(num, d32) - 128;
+                    c = c > 127 ? 127 : (c < -127 ? -127 : c);
+                }
+                out[o] = (int8_t)c;
+                if (acc_out) acc_out[o] = sum;
+            } else {
+                const uint32_t a = (uint32_t)(sum < 0 ? -sum : sum);
+                mx = a > mx ? a : mx;
+            }
+        }
+    }
+    if (!CODES) {
+        mx = warp_max_u32(mx);
+        if ((threadIdx.x & 31) == 0 && mx) atomicMax(amax, (unsigned long long)mx);
+    }
+}
+
 __global__ void k_sq_prepare(const unsigned long long* __restrict__ cell,
                              const double* __restrict__ s_in, int k, RqDiv* __restrict__ dv,
                              double* __restrict__ s_out) {
@@ -267,20 +376,35 @@ struct MseP {
     double s_out;
 };
 
-// extremes of z for target (t=1) and non-target (t=0) elements: [max0, min0, max1, min1]
+// extremes of z for target (t=1) and non-target (t=0) elements: [max0, min0, max1, min1].
+// 16 elements per thread and step: one 16-byte load, the pixel / class of its first byte by
+// one division, then counters.
 __global__ void k_mse_stats(const int8_t* __restrict__ z, const uint8_t* __restrict__ lab,
-                            int64_t npix, int c, int* __restrict__ ext) {
-    int mx0 = INT_MIN, mn0 = INT_MAX, mx1 = INT_MAX, mn1 = INT_MAX;
-    mx1 = INT_MIN;
-    const UDiv dc = make_udiv((uint64_t)c);
+                            int64_t npix, int c, int* __restrict__ ext, UDiv dc, bool vec) {
+    int mx0 = INT_MIN, mn0 = INT_MAX, mx1 = INT_MIN, mn1 = INT_MAX;
     const int64_t total = npix * c;
-    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
-         o += (int64_t)gridDim.x * blockDim.x) {
-        int v = z[o];
+    const int64_t n16 = vec ? total / 16 : 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n16; u += stride) {
+        const int4 v = __ldg(reinterpret_cast<const int4*>(z) + u);
+        const int wv[4] = {v.x, v.y, v.z, v.w};
+        int64_t px = (int64_t)udiv((uint64_t)(u * 16), dc);
+        int ch = (int)(u * 16 - px * c);
+        int lb = lab[px];
+#pragma unroll
+        for (int j = 0; j < 16; j++) {
+            const int zv = (int)(int8_t)(wv[j >> 2] >> (8 * (j & 3)));
+            if (lb == ch) { mx1 = max(mx1, zv); mn1 = min(mn1, zv); }
+            else { mx0 = max(mx0, zv); mn0 = min(mn0, zv); }
+            if (++ch == c && j < 15) { ch = 0; px++; lb = lab[px]; }
+        }
+    }
+    for (int64_t o = n16 * 16 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
+         o += stride) {
+        const int zv = z[o];
         const int64_t px = (int64_t)udiv((uint64_t)o, dc);
-        bool tgt = lab[px] == (uint8_t)(o - px * c);
-        if (tgt) { mx1 = max(mx1, v); mn1 = min(mn1, v); }
-        else { mx0 = max(mx0, v); mn0 = min(mn0, v); }
+        if (lab[px] == (int)(o - px * c)) { mx1 = max(mx1, zv); mn1 = min(mn1, zv); }
+        else { mx0 = max(mx0, zv); mn0 = min(mn0, zv); }
     }
     for (int off = 16; off > 0; off >>= 1) {
         mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
@@ -334,19 +458,39 @@ __global__ void k_mse_fin(const int* __restrict__ ext, const double* __restrict_
     *s_out = p.s_out;
 }
 
+__device__ __forceinline__ int mse_code(int zv, bool tgt, const MseP& p, int64_t lim) {
+    long long t = p.F * (long long)zv + (tgt ? p.B1 : p.B0);
+    return (int)clamp64(t >> p.P, -lim, lim);
+}
+
 __global__ void k_mse_codes(const int8_t* __restrict__ z, const uint8_t* __restrict__ lab,
                             int64_t npix, int c, int k, const MseP* __restrict__ prm,
-                            int8_t* __restrict__ E) {
+                            int8_t* __restrict__ E, UDiv dc, bool vec) {
     const MseP p = *prm;
     const int64_t lim = qmax(k);
-    const UDiv dc = make_udiv((uint64_t)c);
     const int64_t total = npix * c;
-    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
-         o += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t px = (int64_t)udiv((uint64_t)o, dc);
-        bool tgt = lab[px] == (uint8_t)(o - px * c);
-        long long t = p.F * (long long)z[o] + (tgt ? p.B1 : p.B0);
-        E[o] = (int8_t)clamp64(t >> p.P, -lim, lim);
+    const int64_t n16 = vec ? total / 16 : 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n16; u += stride) {
+        const int4 v = __ldg(reinterpret_cast<const int4*>(z) + u);
+        const int wv[4] = {v.x, v.y, v.z, v.w};
+        int64_t px = (int64_t)udiv((uint64_t)(u * 16), dc);
+        int ch = (int)(u * 16 - px * c);
+        int lb = lab[px];
+        uint32_t o[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 16; j++) {
+            const int zv = (int)(int8_t)(wv[j >> 2] >> (8 * (j & 3)));
+            const int e = mse_code(zv, lb == ch, p, lim);
+            o[j >> 2] |= ((uint32_t)e & 0xffu) << (8 * (j & 3));
+            if (++ch == c && j < 15) { ch = 0; px++; lb = lab[px]; }
+        }
+        reinterpret_cast<int4*>(E)[u] = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+    }
+    for (int64_t i = n16 * 16 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += stride) {
+        const int64_t px = (int64_t)udiv((uint64_t)i, dc);
+        E[i] = (int8_t)mse_code(z[i], lab[px] == (int)(i - px * c), p, lim);
     }
 }
 
@@ -446,6 +590,21 @@ extern "C" iq_status iq_upsample_fwd(const int8_t* x, const double* s_x, const i
     double* s_acc = cur.take<double>(1);
     int8_t* wT = cur.take<int8_t>((size_t)c * R * R);
     IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, 8, st));
+    if (R == 64 && stride == 32 && pad == 16 && c <= 256 && ((uintptr_t)w & 15) == 0 &&
+        n <= 65535) {
+        // the FCN decoder shape: |sum| <= 4 * 127^2, so the SQ numerators fit 32 bits
+        dim3 g32((unsigned)(wd + 1), 32u, (unsigned)n);
+        const int thr = (c + 31) / 32 * 32;
+        k_up32_fwd<false><<<g32, thr, 0, st>>>(u, x, w, cell, nullptr, nullptr, nullptr);
+        IQ_LAUNCH_CHECK();
+        k_scale_pow2<<<1, 1, 0, st>>>(s_x, -7, s_acc);
+        IQ_LAUNCH_CHECK();
+        k_sq_prepare<<<1, 1, 0, st>>>(cell, s_acc, 8, dv, s_out);
+        IQ_LAUNCH_CHECK();
+        k_up32_fwd<true><<<g32, thr, 0, st>>>(u, x, w, nullptr, dv, out, acc_out);
+        IQ_LAUNCH_CHECK();
+        return IQ_OK;
+    }
     k_up_wT<<<grid_for((int64_t)c * R * R), kThreads, 0, st>>>(w, wT, c, R);
     IQ_LAUNCH_CHECK();
     dim3 grid((unsigned)((u.W + 31) / 32), (unsigned)(n * u.H));
@@ -536,11 +695,14 @@ extern "C" iq_status iq_mse_grad(const int8_t* z, const double* s_z, const uint8
     k_mse_init<<<1, 1, 0, st>>>(ext);
     IQ_LAUNCH_CHECK();
     int64_t total = npix * c;
-    k_mse_stats<<<grid_for(total), kThreads, 0, st>>>(z, labels, npix, c, ext);
+    const UDiv dc = make_udiv((uint64_t)c);
+    const bool vec = (((uintptr_t)z | (uintptr_t)E) & 15) == 0;
+    const int g = grid_for(vec ? total / 16 + 1 : total);
+    k_mse_stats<<<g, kThreads, 0, st>>>(z, labels, npix, c, ext, dc, vec);
     IQ_LAUNCH_CHECK();
     k_mse_fin<<<1, 1, 0, st>>>(ext, s_z, 8, prm, s_e);
     IQ_LAUNCH_CHECK();
-    k_mse_codes<<<grid_for(total), kThreads, 0, st>>>(z, labels, npix, c, 8, prm, E);
+    k_mse_codes<<<g, kThreads, 0, st>>>(z, labels, npix, c, 8, prm, E, dc, vec);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }

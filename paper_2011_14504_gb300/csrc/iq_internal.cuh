@@ -33,6 +33,7 @@ struct BnStats {
     int* codes;               // [2C]: mu_q codes, sigma_q codes
     int* px;                  // shifts [2]
     double* scal;             // IQ_BN_SCALES doubles (workspace copy)
+    unsigned long long* red;  // [8]: tensor-wide maxima of non-negative doubles (bit patterns)
 };
 
 size_t bn_fwd_ws_bytes(int32_t C);

@@ -112,7 +112,9 @@ __global__ void __launch_bounds__(kThreads) k_comb(Terms T, int concat, int64_t 
         const int co = (int)(e - pix * c_out);
         const int64_t img = (int64_t)udiv((uint64_t)pix, dhw);
         int64_t z = 0;
-        for (int i = 0; i < T.n; i++) {
+#pragma unroll
+        for (int i = 0; i < IQ_MAX_TERMS; i++) {
+            if (i >= T.n) break;
             const TermDev& t = T.t[i];
             int ch = co;
             if (concat) {
@@ -133,6 +135,95 @@ __global__ void __launch_bounds__(kThreads) k_comb(Terms T, int concat, int64_t 
                 c = clamp64((int64_t)udiv(num, d2m) - 128, -127, 127);
             }
             out[e] = (int8_t)c;
+        }
+    }
+    if (PASS == 0) {
+        mx = warp_max_u64(mx);
+        if ((threadIdx.x & 31) == 0 && mx) atomicMax(&hdr->maxz, (unsigned long long)mx);
+    }
+}
+
+// The same two passes, 8 channels per thread: every operand's channel count and offset
+// and c_out are multiples of 8 and the code pointers aligned, so each operand contributes
+// one 8-byte (int8) or 16-byte (int16) load and its F / B rows four 16-byte loads.
+__device__ __forceinline__ void load8(const TermDev& t, int64_t idx, int32_t v[8]) {
+    if (t.is16) {
+        const int4 q = __ldg(reinterpret_cast<const int4*>((const int16_t*)t.codes + idx));
+        const int w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            v[2 * j] = (int32_t)(int16_t)(w[j] & 0xffff);
+            v[2 * j + 1] = (int32_t)(w[j] >> 16);
+        }
+    } else {
+        const int2 q = __ldg(reinterpret_cast<const int2*>((const int8_t*)t.codes + idx));
+        const int w[2] = {q.x, q.y};
+#pragma unroll
+        for (int j = 0; j < 8; j++) v[j] = (int32_t)(int8_t)((w[j >> 2] >> (8 * (j & 3))) & 0xff);
+    }
+}
+
+template <int PASS>
+__global__ void __launch_bounds__(kThreads) k_comb8(Terms T, int concat, int64_t nvec, int cgs,
+                                                    int relu, const long long* __restrict__ F,
+                                                    const long long* __restrict__ B,
+                                                    CombHdr* hdr, int8_t* __restrict__ out,
+                                                    UDiv dcg, UDiv dhw, int any_bcast) {
+    uint64_t M = 0;
+    UDiv d2m;
+    if (PASS == 1) {
+        M = hdr->M;
+        d2m = hdr->div;
+    }
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    uint64_t mx = 0;
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < nvec; u += stride) {
+        const int64_t pix = (int64_t)udiv((uint64_t)u, dcg);
+        const int co0 = (int)(u - pix * cgs) * 8;
+        const int64_t img = any_bcast ? (int64_t)udiv((uint64_t)pix, dhw) : 0;
+        int64_t z[8];
+#pragma unroll
+        for (int j = 0; j < 8; j++) z[j] = 0;
+#pragma unroll
+        for (int i = 0; i < IQ_MAX_TERMS; i++) {
+            if (i >= T.n) break;
+            const TermDev& t = T.t[i];
+            int ch0 = co0;
+            if (concat) {
+                ch0 = co0 - t.c_offset;
+                if (ch0 < 0 || ch0 >= t.c) continue;
+            }
+            int32_t v[8];
+            load8(t, (t.bcast ? img : pix) * t.c + ch0, v);
+            const longlong2* f2 = reinterpret_cast<const longlong2*>(F + t.base + ch0);
+            const longlong2* b2 = reinterpret_cast<const longlong2*>(B + t.base + ch0);
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                const longlong2 f = __ldg(f2 + j), b = __ldg(b2 + j);
+                z[2 * j] += (int64_t)f.x * v[2 * j] + (int64_t)b.x;
+                z[2 * j + 1] += (int64_t)f.y * v[2 * j + 1] + (int64_t)b.y;
+            }
+        }
+        if (PASS == 0) {
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
+                uint64_t a = (uint64_t)(zz < 0 ? -zz : zz);
+                mx = a > mx ? a : mx;
+            }
+        } else {
+            uint32_t w[2] = {0u, 0u};
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
+                int64_t c = 0;
+                if (M) {
+                    uint64_t num = ((uint64_t)(zz + (int64_t)M) << 8) + M;
+                    c = clamp64((int64_t)udiv(num, d2m) - 128, -127, 127);
+                }
+                w[j >> 2] |= ((uint32_t)c & 0xffu) << (8 * (j & 3));
+            }
+            *reinterpret_cast<uint2*>(out + u * 8) = make_uint2(w[0], w[1]);
         }
     }
     if (PASS == 0) {
@@ -297,8 +388,31 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
     k_comb_tables<<<1, 1024, 0, st>>>(T, hdr, F, B);
     IQ_LAUNCH_CHECK();
     const int64_t total = n * hw * (int64_t)c_out;
+    bool vec = c_out % 8 == 0 && ((uintptr_t)out & 7) == 0;
+    bool any_bcast = false;
+    for (int i = 0; i < n_terms; i++) {
+        const TermDev& t = T.t[i];
+        vec = vec && t.c % 8 == 0 && t.c_offset % 8 == 0 &&
+              ((uintptr_t)t.codes & (t.is16 ? 15 : 7)) == 0;
+        any_bcast = any_bcast || t.bcast;
+    }
+    const UDiv dhw = make_udiv((uint64_t)hw);
+    if (vec) {
+        const int64_t nvec = total / 8;
+        const int g = grid_for(nvec, kThreads, 152 * 8);
+        const UDiv dcg = make_udiv((uint64_t)(c_out / 8));
+        k_comb8<0><<<g, kThreads, 0, st>>>(T, concat != 0, nvec, c_out / 8, relu != 0, F, B, hdr,
+                                           out, dcg, dhw, any_bcast);
+        IQ_LAUNCH_CHECK();
+        k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
+        IQ_LAUNCH_CHECK();
+        k_comb8<1><<<g, kThreads, 0, st>>>(T, concat != 0, nvec, c_out / 8, relu != 0, F, B, hdr,
+                                           out, dcg, dhw, any_bcast);
+        IQ_LAUNCH_CHECK();
+        return IQ_OK;
+    }
     const int g = grid_for(total, kThreads, 152 * 8);
-    const UDiv dc = make_udiv((uint64_t)c_out), dhw = make_udiv((uint64_t)hw);
+    const UDiv dc = make_udiv((uint64_t)c_out);
     k_comb<0><<<g, kThreads, 0, st>>>(T, concat != 0, n, hw, c_out, relu != 0, F, B, hdr, out,
                                       dc, dhw);
     IQ_LAUNCH_CHECK();
