@@ -390,7 +390,8 @@ def test_maxpool(k, s, p):
         assert np.array_equal(host(ex).astype(np.int32), want) and host(s_ex)[0] == ws_
 
 
-@pytest.mark.parametrize("n,h,c,R,st,pd", [(1, 2, 150, 64, 32, 16), (2, 3, 21, 16, 8, 4)])
+@pytest.mark.parametrize("n,h,c,R,st,pd", [(1, 2, 150, 64, 32, 16), (2, 3, 21, 16, 8, 4),
+                                           (2, 5, 150, 64, 32, 16), (1, 3, 40, 64, 32, 16)])
 def test_upsample_fwd_bwd_wgrad(n, h, c, R, st, pd):
     g = S.rng(c + R)
     H = (h - 1) * st - 2 * pd + R
@@ -424,6 +425,37 @@ def test_upsample_fwd_bwd_wgrad(n, h, c, R, st, pd):
     assert np.array_equal(host(gacc), want_g)
     want, ws_ = O.rq_int(want_g, 0.03 * 1e-3, 8, 2, 5, 19, 2, 0)
     assert np.array_equal(host(gq).astype(np.int32), want) and host(s_g)[0] == ws_
+
+
+def test_upsample_fcn_shape_extremes():
+    """Every sum at +-4 * 127^2: the largest SQ numerator of the decoder's 32-bit path."""
+    n, h, c = 2, 3, 150
+    H = 32 * h
+    cv = O.Conv(n, H, H, c, c, 64, 64, 32, 16, 1, c)
+    x = np.full((n, h, h, c), 127, np.int8)
+    x[1] = -127
+    w = np.full((c, 64, 64, 1), -127, np.int8)
+    out = torch.empty((n, H, H, c), dtype=torch.int8, device=DEV)
+    s_out = dscal()
+    iq.iq_upsample_fwd(dev(x), dscal(0.5), dev(w), 64, 32, 16, out, s_out)
+    want, ws_ = O.sq_int(O.conv_dgrad(cv, x, w), 0.5 * 2.0 ** -7, 8)
+    assert np.array_equal(host(out).astype(np.int32), want) and host(s_out)[0] == ws_
+
+
+@pytest.mark.parametrize("offset", [0, 1])
+def test_mse_grad_alignment(offset):
+    g = S.rng(78)
+    z = S.int8_uniform(g, (1, 16, 8, 150))
+    lab = S.labels_voronoi(g, 1, 16, 8, 150, sites=5)
+    zbuf = torch.empty(z.size + 16, dtype=torch.int8, device=DEV)
+    zbuf[offset:offset + z.size].copy_(dev(z).view(-1))
+    ebuf = torch.empty(z.size + 16, dtype=torch.int8, device=DEV)
+    s_e = dscal()
+    zt = zbuf[offset:offset + z.size].view(z.shape)
+    et = ebuf[offset:offset + z.size].view(z.shape)
+    iq.iq_mse_grad(zt, dscal(0.05), dev(lab), et, s_e)
+    want, ws_ = O.mse_grad(z, 0.05, lab)
+    assert np.array_equal(host(et), want) and host(s_e)[0] == ws_
 
 
 def test_mse_grad():
