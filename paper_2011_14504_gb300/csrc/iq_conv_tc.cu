@@ -521,6 +521,1106 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
 }
 
+// ---------------------------------------------------------------- persistent kernel
+// One CTA per SM walks a strided list of output tiles (m-tile fastest, then n-tile, then
+// K split) as one flat stream of k-blocks, so the producers run ahead across tile
+// boundaries.  Warps 0-3 gather A (and for WGRAD B), thread 0 issues the B TMA loads;
+// warp 12 issues the MMAs into one fp32 accumulator (TMEM columns [0, BN)); warps 4-11
+// fold every finished fp32 chunk into the int32 running sum (columns [BN, 2 BN)), each
+// warpgroup one half of the columns, and release the accumulator at once.  After a tile's
+// last fold they read the int32 sums back and write the output while the MMAs of the next
+// tile already run; the next tile's first fold overwrites the sums in the same threads'
+// program order, so no further handshake is needed.
+
+constexpr int THREADS_P = 416;
+
+struct BarsP {
+    uint64_t full_a[STAGES];
+    uint64_t full_b[STAGES];
+    uint64_t empty[STAGES];
+    uint64_t accf;
+    uint64_t acce;
+    uint64_t done;
+    uint32_t tmem_base;
+    int abort;
+    int never;
+};
+
+struct TileGrid {
+    int mt, nt, ns;      // m-tiles, n-tiles, splits
+    int total;
+};
+
+// k-block position in a CTA's stream of (tile, kb) pairs
+struct Pos {
+    int tile;            // linear tile index, >= total when past the end
+    int kb;              // k-block within the tile
+    int nkb;             // k-blocks of this tile
+    int64_t m0;
+    int n0, kb0;
+};
+
+__device__ __forceinline__ void pos_set_tile(Pos& q, int tile, const TcP& p, const TileGrid& g,
+                                             int BN) {
+    q.tile = tile;
+    q.kb = 0;
+    q.nkb = 0;
+    if (tile >= g.total) return;
+    const int mt = tile % g.mt;
+    const int rest = tile / g.mt;
+    const int nt = rest % g.nt;
+    const int sp = rest / g.nt;
+    q.m0 = (int64_t)mt * BM;
+    q.n0 = nt * BN;
+    q.kb0 = sp * p.kb_per_split;
+    int n = p.nkb_total - q.kb0;
+    q.nkb = n > p.kb_per_split ? p.kb_per_split : n;
+}
+
+__device__ __forceinline__ void pos_next(Pos& q, const TcP& p, const TileGrid& g, int BN) {
+    if (q.tile >= g.total) return;
+    if (++q.kb >= q.nkb) pos_set_tile(q, q.tile + gridDim.x, p, g, BN);
+}
+
+// output-pixel coordinates of one producer row, recomputed only when the tile changes
+struct RowCache {
+    int tile;
+    bool valid;
+    int n, pp, qq;
+};
+
+__device__ __forceinline__ void gather_fwd_pos(const TcP& p, const int8_t* __restrict__ x,
+                                               const Pos& q, int row, RowCache& rc,
+                                               uint32_t (&w)[16]) {
+    if (rc.tile != q.tile) {
+        rc.tile = q.tile;
+        const int64_t m = q.m0 + row;
+        rc.valid = q.nkb > 0 && m < p.M;
+        rc.n = rc.pp = rc.qq = 0;
+        if (rc.valid) {
+            const int64_t pq = (int64_t)p.P * p.Q;
+            rc.n = (int)(m / pq);
+            const int64_t rem = m - (int64_t)rc.n * pq;
+            rc.pp = (int)(rem / p.Q);
+            rc.qq = (int)(rem - (int64_t)rc.pp * p.Q);
+        }
+    }
+    gather_fwd(p, x, rc.valid, rc.n, rc.pp, rc.qq, q.kb0 + q.kb, w);
+}
+
+// fold the fp32 chunk into the int32 sums of this warpgroup's BN/2 columns
+template <int BN>
+__device__ __forceinline__ void fold_half(uint32_t tD, uint32_t tR, bool has_prev) {
+#pragma unroll 1
+    for (int cb = 0; cb < BN / 2; cb += 32) {
+        uint32_t d0[32], r0[32];
+        tc::tmem_ld_32x32b_x32(tD + cb, d0);
+        if (has_prev) tc::tmem_ld_32x32b_x32(tR + cb, r0);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; i++)
+            r0[i] = (uint32_t)((has_prev ? (int)r0[i] : 0) + __float2int_rn(__uint_as_float(d0[i])));
+        tc::tmem_st_32x32b_x32(tR + cb, r0);
+    }
+    tc::tmem_st_wait();
+}
+
+template <int BN>
+__device__ __forceinline__ void write_half(const TcP& p, uint32_t tR, int64_t m0, int n0, int row,
+                                           int lane, int32_t* __restrict__ out32,
+                                           long long* __restrict__ out64,
+                                           unsigned long long* __restrict__ s1,
+                                           int* __restrict__ hi_c, int* __restrict__ lo_c) {
+    const int64_t m = m0 + row;
+    const bool valid = m < p.M;
+    const bool any = __any_sync(0xffffffffu, valid);
+#pragma unroll 1
+    for (int cb = 0; cb < BN / 2; cb += 32) {
+        uint32_t r[32];
+        tc::tmem_ld_32x32b_x32(tR + cb, r);
+        tc::tmem_ld_wait();
+        if (!any) continue;
+        const int gc0 = n0 + cb;          // first global column of this block
+        if (p.out == OUT_STATS) {
+            if (valid) {
+                int32_t* dst = out32 + m * p.ncols + gc0;
+#pragma unroll
+                for (int i = 0; i < 8; i++)
+                    if (gc0 + 4 * i < p.ncols)
+                        reinterpret_cast<int4*>(dst)[i] =
+                            make_int4((int)r[4 * i], (int)r[4 * i + 1], (int)r[4 * i + 2],
+                                      (int)r[4 * i + 3]);
+            }
+            long long my_sum = 0;
+            int my_hi = INT_MIN, my_lo = INT_MAX;
+#pragma unroll
+            for (int j = 0; j < 32; j++) {
+                const int v = (int)r[j];
+                const int vh = valid ? v : INT_MIN, vl = valid ? v : INT_MAX;
+                const unsigned lo16 = valid ? ((unsigned)v & 0xffffu) : 0u;
+                const int hi16 = valid ? (v >> 16) : 0;
+                const int mx = __reduce_max_sync(0xffffffffu, vh);
+                const int mn = __reduce_min_sync(0xffffffffu, vl);
+                const unsigned sl = __reduce_add_sync(0xffffffffu, lo16);
+                const int sh = __reduce_add_sync(0xffffffffu, hi16);
+                if (lane == j) {
+                    my_hi = mx;
+                    my_lo = mn;
+                    my_sum = (long long)sh * 65536 + (long long)sl;
+                }
+            }
+            const int gcol = gc0 + lane;
+            if (gcol < p.ncols) {
+                atomicAdd(&s1[gcol], (unsigned long long)my_sum);
+                atomicMax(&hi_c[gcol], my_hi);
+                atomicMin(&lo_c[gcol], my_lo);
+            }
+        } else if (valid) {
+            long long* dst = out64 + m * p.ncols + gc0;
+#pragma unroll
+            for (int j = 0; j < 32; j++)
+                if ((int)r[j] != 0 && gc0 + j < p.ncols)
+                    atomicAdd(reinterpret_cast<unsigned long long*>(dst + j),
+                              (unsigned long long)(long long)(int)r[j]);
+        }
+    }
+}
+
+template <int BN>
+__global__ void __launch_bounds__(THREADS_P, 1)
+    k_conv_tcp(const __grid_constant__ CUtensorMap wmap, TcP p, TileGrid g,
+               const int8_t* __restrict__ xa, const int8_t* __restrict__ xb,
+               int32_t* __restrict__ out32, long long* __restrict__ out64,
+               unsigned long long* __restrict__ s1, int* __restrict__ hi_c,
+               int* __restrict__ lo_c, int* __restrict__ err) {
+    constexpr int STAGE_BYTES = Cfg<BN>::STAGE_BYTES;
+    constexpr int B_BYTES = Cfg<BN>::B_BYTES;
+    constexpr int TMEM_COLS = Cfg<BN>::TMEM_COLS;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    BarsP* bars = reinterpret_cast<BarsP*>(smem + STAGES * STAGE_BYTES);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    if (__syncthreads_or(tid == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    if ((int)blockIdx.x >= g.total) return;
+    const bool wg = p.mode == MODE_WGRAD;
+
+    if (tid == 0) {
+        for (int s = 0; s < STAGES; s++) {
+            tc::mbar_init(&bars->full_a[s], 128);
+            tc::mbar_init(&bars->full_b[s], 1);
+            tc::mbar_init(&bars->empty[s], 1);
+        }
+        tc::mbar_init(&bars->accf, 1);
+        tc::mbar_init(&bars->acce, 256);
+        tc::mbar_init(&bars->done, 1);
+        bars->abort = 0;
+        bars->never = 0;
+        tc::mbar_fence_init();
+        if (!wg) tc::tma_prefetch_desc(&wmap);
+    }
+    if (warp == 12) {
+        tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
+        tc::tmem_relinquish();
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
+    volatile int* abort_flag = &bars->abort;
+
+    if (warp < 4) {
+        // ================================================ producers
+        Pos cur, p1, p2;
+        pos_set_tile(cur, blockIdx.x, p, g, BN);
+        p1 = cur;
+        pos_next(p1, p, g, BN);
+        p2 = p1;
+        pos_next(p2, p, g, BN);
+        int issued_b = 0;
+        uint32_t kbc = 0;
+        if (!wg) {
+            const int row = tid;
+            uint32_t c0[16], c1[16], c2[16];
+            RowCache rc;
+            rc.tile = -1;
+            gather_fwd_pos(p, xa, cur, row, rc, c0);
+            gather_fwd_pos(p, xa, p1, row, rc, c1);
+            while (cur.tile < g.total) {
+                const int s = kbc % STAGES;
+                const uint32_t it = kbc / STAGES;
+                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                    bars->abort = 1;
+                    atomicExch(err, 1);
+                    break;
+                }
+                uint8_t* a_tile = smem + s * STAGE_BYTES;
+                if (tid == 0) {
+                    tc::mbar_expect_tx(&bars->full_b[s], B_BYTES);
+                    tc::tma_load_2d(a_tile + A_BYTES, &wmap, &bars->full_b[s],
+                                    (cur.kb0 + cur.kb) * BK, cur.n0);
+                    tc::mbar_arrive(&bars->full_b[s]);
+                    issued_b = (int)kbc + 1;
+                }
+                if (p2.tile < g.total) gather_fwd_pos(p, xa, p2, row, rc, c2);
+                store_kmajor_row(a_tile, row, c0);
+                tc::fence_proxy_async_smem();
+                tc::mbar_arrive(&bars->full_a[s]);
+#pragma unroll
+                for (int i = 0; i < 16; i++) { c0[i] = c1[i]; c1[i] = c2[i]; }
+                cur = p1;
+                p1 = p2;
+                pos_next(p2, p, g, BN);
+                kbc++;
+            }
+        } else {
+            const int j = tid >> 1, h = tid & 1;
+            uint4 a0[4], b0[BN / 32], a1[4], b1[BN / 32];
+            {
+                WgRow r0 = wg_row(p, (int64_t)(cur.kb0 + cur.kb) * BK + j);
+                gather_wgrad<BN>(p, xa, xb, cur.m0, cur.n0, r0, h, a0, b0);
+            }
+            while (cur.tile < g.total) {
+                const int s = kbc % STAGES;
+                const uint32_t it = kbc / STAGES;
+                if (p1.tile < g.total) {
+                    WgRow r1 = wg_row(p, (int64_t)(p1.kb0 + p1.kb) * BK + j);
+                    gather_wgrad<BN>(p, xa, xb, p1.m0, p1.n0, r1, h, a1, b1);
+                }
+                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                    bars->abort = 1;
+                    atomicExch(err, 1);
+                    break;
+                }
+                uint8_t* a_tile = smem + s * STAGE_BYTES;
+                uint8_t* b_tile = a_tile + A_BYTES;
+#pragma unroll
+                for (int i = 0; i < 4; i++)
+                    store_mnmajor_chunk(a_tile, j, 4 * h + i, a0[i].x, a0[i].y, a0[i].z, a0[i].w);
+#pragma unroll
+                for (int i = 0; i < BN / 32; i++)
+                    store_mnmajor_chunk(b_tile, j, h * (BN / 32) + i, b0[i].x, b0[i].y, b0[i].z,
+                                        b0[i].w);
+                tc::fence_proxy_async_smem();
+                tc::mbar_arrive(&bars->full_a[s]);
+                if (tid == 0) tc::mbar_arrive(&bars->full_b[s]);
+#pragma unroll
+                for (int i = 0; i < 4; i++) a0[i] = a1[i];
+#pragma unroll
+                for (int i = 0; i < BN / 32; i++) b0[i] = b1[i];
+                cur = p1;
+                pos_next(p1, p, g, BN);
+                kbc++;
+            }
+        }
+        if (!wg && tid == 0 && *abort_flag) {
+            for (int kb = (issued_b > STAGES ? issued_b - STAGES : 0); kb < issued_b; kb++)
+                tc::mbar_wait(&bars->full_b[kb % STAGES], (uint32_t)(kb / STAGES) & 1,
+                              &bars->never);
+        }
+    } else if (warp == 12) {
+        // ================================================ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_f16(BM, BN, wg);
+            bool ok = true;
+            uint32_t kbc = 0, cc = 0;
+            Pos q;
+            pos_set_tile(q, blockIdx.x, p, g, BN);
+            while (ok && q.tile < g.total) {
+                const int s = kbc % STAGES;
+                const uint32_t it = kbc / STAGES;
+                const bool first = (q.kb % CHUNK_KB) == 0;
+                const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
+                if (first && cc > 0 &&
+                    !tc::mbar_wait(&bars->acce, (cc - 1) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                if (!tc::mbar_wait(&bars->full_b[s], it & 1, abort_flag) ||
+                    !tc::mbar_wait(&bars->full_a[s], it & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc::tc_fence_after();
+                const uint32_t a_addr = tc::smem_u32(smem + s * STAGE_BYTES);
+                const uint32_t b_addr = a_addr + A_BYTES;
+#pragma unroll
+                for (int k = 0; k < BK / 16; k++) {
+                    uint64_t ad, bd;
+                    if (wg) {
+                        ad = sdesc_mnmajor_sw128(a_addr + 2 * 1024 * k);
+                        bd = sdesc_mnmajor_sw128(b_addr + 2 * 1024 * k);
+                    } else {
+                        ad = tc::sdesc_kmajor_sw128(a_addr + 32 * k);
+                        bd = tc::sdesc_kmajor_sw128(b_addr + 32 * k);
+                    }
+                    tc::umma_f16(tmem, ad, bd, idesc, (first && k == 0) ? 0u : 1u);
+                }
+                tc::umma_commit(&bars->empty[s]);
+                if (last) {
+                    tc::umma_commit(&bars->accf);
+                    cc++;
+                }
+                kbc++;
+                pos_next(q, p, g, BN);
+            }
+            if (!ok) {
+                bars->abort = 1;
+                atomicExch(err, 2);
+            }
+            tc::umma_commit(&bars->done);
+            tc::mbar_wait(&bars->done, 0, &bars->never);
+        }
+        __syncwarp();
+    } else {
+        // ================================================ epilogue (warps 4..11)
+        const int half = (warp - 4) >> 2;                 // column half
+        const int row = ((warp & 3) << 5) + lane;         // TMEM lane = tile row
+        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+        const uint32_t tD = tmem + lane_base + half * (BN / 2);
+        const uint32_t tR = tmem + lane_base + BN + half * (BN / 2);
+        uint32_t cc = 0;
+        bool ok = true;
+        Pos q;
+        pos_set_tile(q, blockIdx.x, p, g, BN);
+        while (ok && q.tile < g.total) {
+            const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
+            for (int c = 0; c < nch; c++) {
+                if (!tc::mbar_wait(&bars->accf, cc & 1, abort_flag)) {
+                    ok = false;
+                    bars->abort = 1;
+                    atomicExch(err, 3);
+                    break;
+                }
+                tc::tc_fence_after();
+                fold_half<BN>(tD, tR, c > 0);
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bars->acce);
+                cc++;
+            }
+            if (!ok || *abort_flag) break;
+            write_half<BN>(p, tR, q.m0, q.n0 + half * (BN / 2), row, lane, out32, out64, s1, hi_c,
+                           lo_c);
+            pos_set_tile(q, q.tile + gridDim.x, p, g, BN);
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 12) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+// ---------------------------------------------------------------- persistent forward kernel
+// The forward (and stride-1 data-gradient) GEMM for whole 64-channel k-blocks, persistent
+// like k_conv_tcp, with the fold spread over 16 epilogue warps (4 warpgroups, each a quarter
+// of the columns; warp w reads TMEM lanes 32 (w % 4) ..) so that the MMA warp waits only
+// briefly per 16 k-blocks, and the epilogue sleeping between its barrier probes.  Each
+// producer thread owns one A row: it copies its 64 int8 codes per k-block with cp.async
+// (zero fill for padding and rows past the end) into a private slot of a ring NST_Q
+// k-blocks deep, walks the taps with incremental counters (no divisions per k-block), and
+// widens the k-block NST_Q - 1 behind into the fp16 stage.
+
+constexpr int THREADS_Q = 672;       // warps 0-3 producers, 4-19 epilogue, 20 MMA
+constexpr int EPI_Q = 512;
+constexpr int STAGES_Q = 3;          // fp16 A + B stages
+constexpr int NST_Q = 6;             // int8 staging ring depth (k-blocks)
+constexpr int STG_PITCH = 80;        // bytes per staged row: 64 + 16 (conflict-free 16-B accesses)
+constexpr int STG_SLOT = BM * STG_PITCH;
+
+template <int BN>
+struct CfgQ {
+    static constexpr int STAGE_BYTES = Cfg<BN>::STAGE_BYTES;
+    static constexpr int STG_OFF = STAGES_Q * STAGE_BYTES;
+    static constexpr int BAR_OFF = STG_OFF + NST_Q * STG_SLOT;
+    static constexpr int SMEM = BAR_OFF + 1024 + 256;
+    static_assert(SMEM <= 232448, "shared memory");
+};
+
+struct BarsQ {
+    uint64_t full_a[STAGES_Q];
+    uint64_t full_b[STAGES_Q];
+    uint64_t empty[STAGES_Q];
+    uint64_t accf;
+    uint64_t acce;
+    uint64_t done;
+    uint32_t tmem_base;
+    int abort;
+    int never;
+};
+
+// a producer row's position in its k-block stream, with the tap counters of the k-block
+struct FwdCur {
+    Pos q;
+    bool valid;
+    int n, pp, qq;
+    int r, s, c0;      // tap mode: tap (r, s) and first channel of the k-block
+};
+
+__device__ __forceinline__ void fcur_tile(FwdCur& f, int tile, const TcP& p, const TileGrid& g,
+                                          int BN, int row) {
+    pos_set_tile(f.q, tile, p, g, BN);
+    f.valid = false;
+    f.n = f.pp = f.qq = 0;
+    f.r = f.s = f.c0 = 0;
+    if (f.q.tile >= g.total) return;
+    const int64_t m = f.q.m0 + row;
+    f.valid = m < p.M;
+    if (f.valid) {
+        const int64_t pq = (int64_t)p.P * p.Q;
+        f.n = (int)(m / pq);
+        const int64_t rem = m - (int64_t)f.n * pq;
+        f.pp = (int)(rem / p.Q);
+        f.qq = (int)(rem - (int64_t)f.pp * p.Q);
+    }
+    if (p.tap_mode) {
+        const int kpos = f.q.kb0 * BK;
+        const int tap = kpos / p.C;
+        f.c0 = kpos - tap * p.C;
+        f.r = tap / p.S;
+        f.s = tap - f.r * p.S;
+    }
+}
+
+__device__ __forceinline__ void fcur_next(FwdCur& f, const TcP& p, const TileGrid& g, int BN,
+                                          int row) {
+    if (f.q.tile >= g.total) return;
+    if (++f.q.kb >= f.q.nkb) {
+        fcur_tile(f, f.q.tile + gridDim.x, p, g, BN, row);
+        return;
+    }
+    if (p.tap_mode) {
+        f.c0 += BK;
+        if (f.c0 >= p.C) {
+            f.c0 = 0;
+            if (++f.s == p.S) {
+                f.s = 0;
+                f.r++;
+            }
+        }
+    }
+}
+
+// cp.async of this row's 64 codes of the cursor's k-block into a staging slot (tap mode)
+__device__ __forceinline__ void fcur_copy(const TcP& p, const int8_t* __restrict__ x,
+                                          const FwdCur& f, uint32_t dst) {
+    const int hh = f.pp * p.sh + f.r * p.dh - p.ph;
+    const int ww = f.qq * p.sw + f.s * p.dw - p.pw;
+    const bool in = f.valid && f.q.nkb > 0 && hh >= 0 && hh < p.H && ww >= 0 && ww < p.W;
+    const int8_t* src = in ? x + (((int64_t)f.n * p.H + hh) * p.W + ww) * p.cstride + p.cofs + f.c0
+                           : x;
+    const uint32_t nb = in ? 16u : 0u;
+#pragma unroll
+    for (int i = 0; i < 4; i++) tc::cp_async16(dst + 16 * i, src + 16 * i, nb);
+}
+
+// the output of 32 columns of one warpgroup's quarter: int32 stores and per-channel
+// statistics (OUT_STATS) or int64 atomic adds
+template <int CW>
+__device__ __forceinline__ void write_quarter(const TcP& p, const int (&sum)[CW], int64_t m0,
+                                              int c0, int row, int lane,
+                                              int32_t* __restrict__ out32,
+                                              long long* __restrict__ out64,
+                                              unsigned long long* __restrict__ s1,
+                                              int* __restrict__ hi_c, int* __restrict__ lo_c) {
+    const int64_t m = m0 + row;
+    const bool valid = m < p.M;
+    if (p.out == OUT_STATS) {
+        if (valid) {
+            int32_t* dst = out32 + m * p.ncols + c0;
+#pragma unroll
+            for (int i = 0; i < CW / 4; i++)
+                if (c0 + 4 * i < p.ncols)
+                    reinterpret_cast<int4*>(dst)[i] =
+                        make_int4(sum[4 * i], sum[4 * i + 1], sum[4 * i + 2], sum[4 * i + 3]);
+        }
+#pragma unroll
+        for (int cb = 0; cb < CW; cb += 32) {
+            long long my_sum = 0;
+            int my_hi = INT_MIN, my_lo = INT_MAX;
+#pragma unroll
+            for (int j = 0; j < 32 && cb + j < CW; j++) {
+                const int v = sum[cb + j];
+                const int mx = __reduce_max_sync(0xffffffffu, valid ? v : INT_MIN);
+                const int mn = __reduce_min_sync(0xffffffffu, valid ? v : INT_MAX);
+                const unsigned sl = __reduce_add_sync(0xffffffffu, valid ? ((unsigned)v & 0xffffu) : 0u);
+                const int sh = __reduce_add_sync(0xffffffffu, valid ? (v >> 16) : 0);
+                if (lane == j) {
+                    my_hi = mx;
+                    my_lo = mn;
+                    my_sum = (long long)sh * 65536 + (long long)sl;
+                }
+            }
+            const int gcol = c0 + cb + lane;
+            if (lane < CW - cb && gcol < p.ncols) {
+                atomicAdd(&s1[gcol], (unsigned long long)my_sum);
+                atomicMax(&hi_c[gcol], my_hi);
+                atomicMin(&lo_c[gcol], my_lo);
+            }
+        }
+    } else if (valid) {
+        long long* dst = out64 + m * p.ncols + c0;
+#pragma unroll
+        for (int j = 0; j < CW; j++)
+            if (sum[j] != 0 && c0 + j < p.ncols)
+                atomicAdd(reinterpret_cast<unsigned long long*>(dst + j),
+                          (unsigned long long)(long long)sum[j]);
+    }
+}
+
+// TMEM loads / stores of 16 or 32 columns
+template <int W>
+__device__ __forceinline__ void tmem_ld_w(uint32_t a, uint32_t (&r)[W]) {
+    if constexpr (W == 32) tc::tmem_ld_32x32b_x32(a, r);
+    else tc::tmem_ld_32x32b_x16(a, r);
+}
+template <int W>
+__device__ __forceinline__ void tmem_st_w(uint32_t a, const uint32_t (&r)[W]) {
+    if constexpr (W == 32) tc::tmem_st_32x32b_x32(a, r);
+    else tc::tmem_st_32x32b_x16(a, r);
+}
+
+template <int BN>
+__global__ void __launch_bounds__(THREADS_Q, 1)
+    k_conv_tcq(const __grid_constant__ CUtensorMap wmap, TcP p, TileGrid g,
+               const int8_t* __restrict__ xa, int32_t* __restrict__ out32,
+               long long* __restrict__ out64, unsigned long long* __restrict__ s1,
+               int* __restrict__ hi_c, int* __restrict__ lo_c, int* __restrict__ err) {
+    constexpr int STAGE_BYTES = CfgQ<BN>::STAGE_BYTES;
+    constexpr int B_BYTES = Cfg<BN>::B_BYTES;
+    constexpr int TMEM_COLS = Cfg<BN>::TMEM_COLS;     // fp32 chunk + int32 running sum
+    constexpr int CW = BN / 4;                         // columns per epilogue warpgroup
+    constexpr int LDW = 16;                            // columns per TMEM access
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    BarsQ* bars = reinterpret_cast<BarsQ*>(smem + CfgQ<BN>::BAR_OFF);
+    uint8_t* stg = smem + CfgQ<BN>::STG_OFF;
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    if (__syncthreads_or(tid == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    if ((int)blockIdx.x >= g.total) return;
+
+    if (tid == 0) {
+        for (int s = 0; s < STAGES_Q; s++) {
+            tc::mbar_init(&bars->full_a[s], 128);
+            tc::mbar_init(&bars->full_b[s], 1);
+            tc::mbar_init(&bars->empty[s], 1);
+        }
+        tc::mbar_init(&bars->accf, 1);
+        tc::mbar_init(&bars->acce, EPI_Q);
+        tc::mbar_init(&bars->done, 1);
+        bars->abort = 0;
+        bars->never = 0;
+        tc::mbar_fence_init();
+        tc::tma_prefetch_desc(&wmap);
+    }
+    if (warp == 20) {
+        tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
+        tc::tmem_relinquish();
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
+    volatile int* abort_flag = &bars->abort;
+
+    if (warp < 4) {
+        // ================================================ producers
+        const int row = tid;
+        const uint32_t my_stg = tc::smem_u32(stg) + row * STG_PITCH;
+        FwdCur cs, cg;
+        fcur_tile(cs, blockIdx.x, p, g, BN, row);
+        cg = cs;
+        // prologue: copies of the first NST_Q - 1 k-blocks in flight
+#pragma unroll 1
+        for (int i = 0; i < NST_Q - 1; i++) {
+            if (cg.q.tile < g.total) fcur_copy(p, xa, cg, my_stg + i * STG_SLOT);
+            tc::cp_async_commit();
+            fcur_next(cg, p, g, BN, row);
+        }
+        uint32_t kbc = 0;
+        int issued_b = 0;
+        while (cs.q.tile < g.total) {
+            // copy k-block kbc + NST_Q - 1, then wait until k-block kbc has landed
+            if (cg.q.tile < g.total)
+                fcur_copy(p, xa, cg, my_stg + ((kbc + NST_Q - 1) % NST_Q) * STG_SLOT);
+            tc::cp_async_commit();
+            fcur_next(cg, p, g, BN, row);
+            tc::cp_async_wait<NST_Q - 1>();
+            const uint8_t* src = stg + (kbc % NST_Q) * STG_SLOT + row * STG_PITCH;
+            uint32_t w[16];
+#pragma unroll
+            for (int i = 0; i < 4; i++) {
+                const uint4 v = *reinterpret_cast<const uint4*>(src + 16 * i);
+                w[4 * i] = v.x; w[4 * i + 1] = v.y; w[4 * i + 2] = v.z; w[4 * i + 3] = v.w;
+            }
+            const int s = kbc % STAGES_Q;
+            const uint32_t it = kbc / STAGES_Q;
+            if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                bars->abort = 1;
+                atomicExch(err, 1);
+                break;
+            }
+            uint8_t* a_tile = smem + s * STAGE_BYTES;
+            if (tid == 0) {
+                tc::mbar_expect_tx(&bars->full_b[s], B_BYTES);
+                tc::tma_load_2d(a_tile + A_BYTES, &wmap, &bars->full_b[s],
+                                (cs.q.kb0 + cs.q.kb) * BK, cs.q.n0);
+                tc::mbar_arrive(&bars->full_b[s]);
+                issued_b = (int)kbc + 1;
+            }
+            store_kmajor_row(a_tile, row, w);
+            tc::fence_proxy_async_smem();
+            tc::mbar_arrive(&bars->full_a[s]);
+            fcur_next(cs, p, g, BN, row);
+            kbc++;
+        }
+        tc::cp_async_wait<0>();
+        if (tid == 0 && *abort_flag) {
+            for (int kb = (issued_b > STAGES_Q ? issued_b - STAGES_Q : 0); kb < issued_b; kb++)
+                tc::mbar_wait(&bars->full_b[kb % STAGES_Q], (uint32_t)(kb / STAGES_Q) & 1,
+                              &bars->never);
+        }
+    } else if (warp == 20) {
+        // ================================================ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_f16(BM, BN, false);
+            bool ok = true;
+            uint32_t kbc = 0, cc = 0;
+            Pos q;
+            pos_set_tile(q, blockIdx.x, p, g, BN);
+            while (ok && q.tile < g.total) {
+                const int s = kbc % STAGES_Q;
+                const uint32_t it = kbc / STAGES_Q;
+                const bool first = (q.kb % CHUNK_KB) == 0;
+                const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
+                // the fp32 accumulator is free once the epilogue folded the previous chunk
+                if (first && cc > 0 && !tc::mbar_wait(&bars->acce, (cc - 1) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                if (!tc::mbar_wait(&bars->full_b[s], it & 1, abort_flag) ||
+                    !tc::mbar_wait(&bars->full_a[s], it & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc::tc_fence_after();
+                const uint32_t a_addr = tc::smem_u32(smem + s * STAGE_BYTES);
+                const uint32_t b_addr = a_addr + A_BYTES;
+#pragma unroll
+                for (int k = 0; k < BK / 16; k++)
+                    tc::umma_f16(tmem, tc::sdesc_kmajor_sw128(a_addr + 32 * k),
+                                 tc::sdesc_kmajor_sw128(b_addr + 32 * k), idesc,
+                                 (first && k == 0) ? 0u : 1u);
+                tc::umma_commit(&bars->empty[s]);
+                if (last) {
+                    tc::umma_commit(&bars->accf);
+                    cc++;
+                }
+                kbc++;
+                pos_next(q, p, g, BN);
+            }
+            if (!ok) {
+                bars->abort = 1;
+                atomicExch(err, 2);
+            }
+            tc::umma_commit(&bars->done);
+            tc::mbar_wait(&bars->done, 0, &bars->never);
+        }
+        __syncwarp();
+    } else {
+        // ================================================ epilogue (warps 4..19)
+        const int quarter = (warp - 4) >> 2;
+        const int row = ((warp & 3) << 5) + lane;
+        const uint32_t lb = (uint32_t)((warp & 3) * 32) << 16;
+        const uint32_t tD = tmem + lb + quarter * CW;          // fp32 chunk
+        const uint32_t tR = tmem + lb + BN + quarter * CW;     // int32 running sum
+        uint32_t cc = 0;
+        bool ok = true;
+        Pos q;
+        pos_set_tile(q, blockIdx.x, p, g, BN);
+        while (ok && q.tile < g.total) {
+            const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
+            for (int c = 0; c < nch; c++) {
+                if (!tc::mbar_wait_sleep(&bars->accf, cc & 1, abort_flag)) {
+                    ok = false;
+                    bars->abort = 1;
+                    atomicExch(err, 3);
+                    break;
+                }
+                tc::tc_fence_after();
+#pragma unroll
+                for (int cb = 0; cb < CW; cb += LDW) {
+                    uint32_t d[LDW], r[LDW];
+                    tmem_ld_w<LDW>(tD + cb, d);
+                    if (c > 0) tmem_ld_w<LDW>(tR + cb, r);
+                    tc::tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < LDW; i++)
+                        r[i] = (uint32_t)((c > 0 ? (int)r[i] : 0) +
+                                          __float2int_rn(__uint_as_float(d[i])));
+                    tmem_st_w<LDW>(tR + cb, r);
+                }
+                tc::tmem_st_wait();
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bars->acce);
+                cc++;
+            }
+            if (!ok || *abort_flag) break;
+            const int64_t m = q.m0 + row;
+            if (__any_sync(0xffffffffu, m < p.M)) {
+#pragma unroll
+                for (int cb = 0; cb < CW; cb += LDW) {
+                    uint32_t r[LDW];
+                    tmem_ld_w<LDW>(tR + cb, r);
+                    tc::tmem_ld_wait();
+                    write_quarter<LDW>(p, reinterpret_cast<const int(&)[LDW]>(r), q.m0,
+                                       q.n0 + quarter * CW + cb, row, lane, out32, out64, s1, hi_c,
+                                       lo_c);
+                }
+            }
+            pos_set_tile(q, q.tile + gridDim.x, p, g, BN);
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 20) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+// ---------------------------------------------------------------- all-TMA forward kernel
+// Stride-1/2 convolutions with whole 64-channel k-blocks, over fp16 carriers of the codes
+// (a pre-pass widens the input once per call).  The M tile is a BH x BW rectangle of one
+// image's output pixels; for k-block (tap r,s; channels c0..c0+63) its A rows are the input
+// box of that tap -- one 4-D TMA load (element strides = the conv strides, zero fill
+// outside the image = the padding) lands them directly in the K-major 128-byte-swizzled
+// UMMA layout, next to the B tile (fp16 weights, 2-D TMA).  Warp 0 issues the loads, warp
+// 1 the MMAs into two fp32 accumulators (chunk c in accumulator c % 2), and 16 epilogue
+// warps (4 warpgroups, a quarter of the columns each) fold every finished chunk into int32
+// sums held in registers, so neither the loads nor the folds stall the tensor pipe; a
+// tile's output is written while the next tile's MMAs run.  Persistent over the tiles.
+
+constexpr int THREADS_T = 640;       // warp 0 TMA, warp 1 MMA, warps 4-19 epilogue
+constexpr int EPI_T = 512;
+constexpr int STAGES_T = 4;
+
+template <int BN>
+struct CfgT {
+    static constexpr int STAGE_BYTES = A_BYTES + BN * 128;
+    static constexpr int BAR_OFF = STAGES_T * STAGE_BYTES;
+    static constexpr int SMEM = BAR_OFF + 1024 + 256;
+    static constexpr int TMEM_COLS = 2 * BN;
+    static_assert(SMEM <= 232448, "shared memory");
+};
+
+struct BarsT {
+    uint64_t full[STAGES_T];
+    uint64_t empty[STAGES_T];
+    uint64_t accf[2];
+    uint64_t acce[2];
+    uint64_t done;
+    uint32_t tmem_base;
+    int abort;
+    int never;
+};
+
+struct RectGrid {
+    int PT, QT, BW, BH;   // rectangles per image (rows x columns) and their size
+    int mt, nt, total;    // m-tiles (N * PT * QT), n-tiles, tiles
+};
+
+struct RectPos {
+    int tile, kb;
+    int n, p0, q0, n0;
+};
+
+__device__ __forceinline__ void rpos_set(RectPos& q, int tile, const RectGrid& g, int BN) {
+    q.tile = tile;
+    q.kb = 0;
+    if (tile >= g.total) return;
+    const int mt = tile % g.mt;
+    q.n0 = (tile / g.mt) * BN;
+    const int qt = mt % g.QT;
+    const int pt = (mt / g.QT) % g.PT;
+    q.n = mt / (g.QT * g.PT);
+    q.p0 = pt * g.BH;
+    q.q0 = qt * g.BW;
+}
+
+__device__ __forceinline__ void rpos_next(RectPos& q, const TcP& p, const RectGrid& g, int BN) {
+    if (q.tile >= g.total) return;
+    if (++q.kb >= p.nkb_total) rpos_set(q, q.tile + gridDim.x, g, BN);
+}
+
+// int32 stores and per-channel statistics (OUT_STATS) or int64 atomic adds of LDW columns
+// of one output row m (valid: the row exists)
+template <int LDW>
+__device__ __forceinline__ void write_row(const TcP& p, const uint32_t (&r)[LDW], int64_t m,
+                                          bool valid, int c0, int lane,
+                                          int32_t* __restrict__ out32,
+                                          long long* __restrict__ out64,
+                                          unsigned long long* __restrict__ s1,
+                                          int* __restrict__ hi_c, int* __restrict__ lo_c) {
+    if (p.out == OUT_STATS) {
+        if (valid) {
+            int32_t* dst = out32 + m * p.ncols + c0;
+#pragma unroll
+            for (int i = 0; i < LDW / 4; i++)
+                if (c0 + 4 * i < p.ncols)
+                    reinterpret_cast<int4*>(dst)[i] = make_int4((int)r[4 * i], (int)r[4 * i + 1],
+                                                                (int)r[4 * i + 2], (int)r[4 * i + 3]);
+        }
+        long long my_sum = 0;
+        int my_hi = INT_MIN, my_lo = INT_MAX;
+#pragma unroll
+        for (int j = 0; j < LDW; j++) {
+            const int v = (int)r[j];
+            const int mx = __reduce_max_sync(0xffffffffu, valid ? v : INT_MIN);
+            const int mn = __reduce_min_sync(0xffffffffu, valid ? v : INT_MAX);
+            const unsigned sl = __reduce_add_sync(0xffffffffu, valid ? ((unsigned)v & 0xffffu) : 0u);
+            const int sh = __reduce_add_sync(0xffffffffu, valid ? (v >> 16) : 0);
+            if (lane == j) {
+                my_hi = mx;
+                my_lo = mn;
+                my_sum = (long long)sh * 65536 + (long long)sl;
+            }
+        }
+        const int gcol = c0 + lane;
+        if (lane < LDW && gcol < p.ncols) {
+            atomicAdd(&s1[gcol], (unsigned long long)my_sum);
+            atomicMax(&hi_c[gcol], my_hi);
+            atomicMin(&lo_c[gcol], my_lo);
+        }
+    } else if (valid) {
+        long long* dst = out64 + m * p.ncols + c0;
+#pragma unroll
+        for (int j = 0; j < LDW; j++)
+            if ((int)r[j] != 0 && c0 + j < p.ncols)
+                atomicAdd(reinterpret_cast<unsigned long long*>(dst + j),
+                          (unsigned long long)(long long)(int)r[j]);
+    }
+}
+
+template <int BN>
+__global__ void __launch_bounds__(THREADS_T, 1)
+    k_conv_tct(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap amap,
+               TcP p, RectGrid g, int32_t* __restrict__ out32, long long* __restrict__ out64,
+               unsigned long long* __restrict__ s1, int* __restrict__ hi_c,
+               int* __restrict__ lo_c, int* __restrict__ err) {
+    constexpr int STAGE_BYTES = CfgT<BN>::STAGE_BYTES;
+    constexpr int TMEM_COLS = CfgT<BN>::TMEM_COLS;
+    constexpr int CW = BN / 4;                 // columns per epilogue warpgroup
+    constexpr int LDW = CW < 16 ? CW : 16;     // columns per TMEM load
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    BarsT* bars = reinterpret_cast<BarsT*>(smem + CfgT<BN>::BAR_OFF);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    if (__syncthreads_or(tid == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    if ((int)blockIdx.x >= g.total) return;
+
+    if (tid == 0) {
+        for (int s = 0; s < STAGES_T; s++) {
+            tc::mbar_init(&bars->full[s], 1);
+            tc::mbar_init(&bars->empty[s], 1);
+        }
+        for (int b = 0; b < 2; b++) {
+            tc::mbar_init(&bars->accf[b], 1);
+            tc::mbar_init(&bars->acce[b], EPI_T);
+        }
+        tc::mbar_init(&bars->done, 1);
+        bars->abort = 0;
+        bars->never = 0;
+        tc::mbar_fence_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
+        tc::tmem_relinquish();
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
+    volatile int* abort_flag = &bars->abort;
+
+    if (warp == 0) {
+        // ================================================ TMA issuer
+        if (lane == 0) {
+            tc::tma_prefetch_desc(&amap);
+            tc::tma_prefetch_desc(&wmap);
+            RectPos q;
+            rpos_set(q, blockIdx.x, g, BN);
+            int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
+            uint32_t kbc = 0;
+            int issued = 0;
+            while (q.tile < g.total) {
+                const int s = kbc % STAGES_T;
+                const uint32_t it = kbc / STAGES_T;
+                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                    bars->abort = 1;
+                    atomicExch(err, 4);
+                    break;
+                }
+                uint8_t* st = smem + s * STAGE_BYTES;
+                tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
+                tc::tma_load_4d(st, &amap, &bars->full[s], p.cofs + c0,
+                                q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph, q.n);
+                tc::tma_load_2d(st + A_BYTES, &wmap, &bars->full[s], q.kb * BK, q.n0);
+                tc::mbar_arrive(&bars->full[s]);
+                issued = (int)kbc + 1;
+                kbc++;
+                const int tile = q.tile;
+                rpos_next(q, p, g, BN);
+                if (q.tile != tile) {
+                    r = ss = c0 = 0;
+                } else {
+                    c0 += BK;
+                    if (c0 >= p.C) {
+                        c0 = 0;
+                        if (++ss == p.S) { ss = 0; r++; }
+                    }
+                }
+            }
+            if (*abort_flag) {
+                for (int kb = (issued > STAGES_T ? issued - STAGES_T : 0); kb < issued; kb++)
+                    tc::mbar_wait(&bars->full[kb % STAGES_T], (uint32_t)(kb / STAGES_T) & 1,
+                                  &bars->never);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ================================================ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_f16(BM, BN, false);
+            bool ok = true;
+            uint32_t kbc = 0, cc = 0;
+            RectPos q;
+            rpos_set(q, blockIdx.x, g, BN);
+            while (ok && q.tile < g.total) {
+                const int s = kbc % STAGES_T;
+                const uint32_t it = kbc / STAGES_T;
+                const bool first = (q.kb % CHUNK_KB) == 0;
+                const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == p.nkb_total - 1;
+                const uint32_t buf = cc & 1;
+                if (first && cc >= 2 &&
+                    !tc::mbar_wait(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                if (!tc::mbar_wait(&bars->full[s], it & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc::tc_fence_after();
+                const uint32_t a_addr = tc::smem_u32(smem + s * STAGE_BYTES);
+                const uint32_t b_addr = a_addr + A_BYTES;
+#pragma unroll
+                for (int k = 0; k < BK / 16; k++)
+                    tc::umma_f16(tmem + buf * BN, tc::sdesc_kmajor_sw128(a_addr + 32 * k),
+                                 tc::sdesc_kmajor_sw128(b_addr + 32 * k), idesc,
+                                 (first && k == 0) ? 0u : 1u);
+                tc::umma_commit(&bars->empty[s]);
+                if (last) {
+                    tc::umma_commit(&bars->accf[buf]);
+                    cc++;
+                }
+                kbc++;
+                rpos_next(q, p, g, BN);
+            }
+            if (!ok) {
+                bars->abort = 1;
+                atomicExch(err, 2);
+            }
+            tc::umma_commit(&bars->done);
+            tc::mbar_wait(&bars->done, 0, &bars->never);
+        }
+        __syncwarp();
+    } else if (warp >= 4) {
+        // ================================================ epilogue (warps 4..19)
+        const int quarter = (warp - 4) >> 2;
+        const int row = ((warp & 3) << 5) + lane;
+        const uint32_t taddr = tmem + ((uint32_t)((warp & 3) * 32) << 16) + quarter * CW;
+        const int dp = row / g.BW, dq = row - (row / g.BW) * g.BW;
+        uint32_t cc = 0;
+        bool ok = true;
+        RectPos q;
+        rpos_set(q, blockIdx.x, g, BN);
+        const int nch = (p.nkb_total + CHUNK_KB - 1) / CHUNK_KB;
+        int sum[CW];
+        while (ok && q.tile < g.total) {
+#pragma unroll
+            for (int i = 0; i < CW; i++) sum[i] = 0;
+            for (int c = 0; c < nch; c++) {
+                const uint32_t buf = cc & 1;
+                if (!tc::mbar_wait_sleep(&bars->accf[buf], (cc >> 1) & 1, abort_flag)) {
+                    ok = false;
+                    bars->abort = 1;
+                    atomicExch(err, 3);
+                    break;
+                }
+                tc::tc_fence_after();
+#pragma unroll
+                for (int cb = 0; cb < CW; cb += LDW) {
+                    uint32_t d[LDW];
+                    tmem_ld_w<LDW>(taddr + buf * BN + cb, d);
+                    tc::tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < LDW; i++) sum[cb + i] += __float2int_rn(__uint_as_float(d[i]));
+                }
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bars->acce[buf]);
+                cc++;
+            }
+            if (!ok || *abort_flag) break;
+            const int pp = q.p0 + dp, qq = q.q0 + dq;
+            const bool valid = pp < p.P && qq < p.Q;
+            const int64_t m = ((int64_t)q.n * p.P + pp) * p.Q + qq;
+            if (__any_sync(0xffffffffu, valid)) {
+#pragma unroll
+                for (int cb = 0; cb < CW; cb += LDW) {
+                    uint32_t v[LDW];
+#pragma unroll
+                    for (int i = 0; i < LDW; i++) v[i] = (uint32_t)sum[cb + i];
+                    write_row<LDW>(p, v, m, valid, q.n0 + quarter * CW + cb, lane, out32, out64,
+                                   s1, hi_c, lo_c);
+                }
+            }
+            rpos_set(q, q.tile + gridDim.x, g, BN);
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+// int8 codes [npix][cstride] -> exact fp16 carriers, 16 codes per thread
+__global__ void k_codes_to_f16(const int8_t* __restrict__ x, __half* __restrict__ xf, int64_t n16) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += stride) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4*>(x) + i);
+        uint32_t o[8];
+        tc::i8x4_to_f16x4(v.x, o[0], o[1]);
+        tc::i8x4_to_f16x4(v.y, o[2], o[3]);
+        tc::i8x4_to_f16x4(v.z, o[4], o[5]);
+        tc::i8x4_to_f16x4(v.w, o[6], o[7]);
+        uint4* dst = reinterpret_cast<uint4*>(xf) + 2 * i;
+        dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+        dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+    }
+}
+
 // ---------------------------------------------------------------- TMA-fed forward
 // Stride-1 convolutions with C % 64 == 0: the M tile is a BH x BW rectangle of output
 // pixels of one image (BH * BW = 128).  For k-block (tap r,s; channels c0..c0+63) the A
@@ -862,9 +1962,76 @@ iq_status launch_bn(const CUtensorMap& map, const TcP& p, int nsplit, const int8
 // N-tile width for a GEMM with `ncols` columns: the smallest of 64 / 128 / 256 covering it
 int pick_bn(int ncols) { return ncols <= 64 ? 64 : (ncols <= 128 ? 128 : 256); }
 
+int num_sms() {
+    static int n = 0;
+    if (!n) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+            n = 152;
+    }
+    return n;
+}
+
+template <int BN>
+iq_status launch_p(const CUtensorMap& map, const TcP& p, int nsplit, const int8_t* xa,
+                   const int8_t* xb, int32_t* out32, long long* out64, unsigned long long* s1,
+                   int* hi, int* lo, int* err, cudaStream_t st) {
+    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tcp<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Cfg<BN>::SMEM));
+    TileGrid g;
+    g.mt = (int)((p.M + BM - 1) / BM);
+    g.nt = (p.ncols + BN - 1) / BN;
+    g.ns = nsplit;
+    g.total = g.mt * g.nt * g.ns;
+    const int grid = g.total < num_sms() ? g.total : num_sms();
+    k_conv_tcp<BN><<<grid, THREADS_P, Cfg<BN>::SMEM, st>>>(map, p, g, xa, xb, out32, out64, s1, hi,
+                                                          lo, err);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+template <int BN>
+iq_status launch_q(const CUtensorMap& map, const TcP& p, const int8_t* xa, int32_t* out32,
+                   long long* out64, unsigned long long* s1, int* hi, int* lo, int* err,
+                   cudaStream_t st) {
+    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tcq<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       CfgQ<BN>::SMEM));
+    TileGrid g;
+    g.mt = (int)((p.M + BM - 1) / BM);
+    g.nt = (p.ncols + BN - 1) / BN;
+    g.ns = 1;
+    g.total = g.mt * g.nt;
+    const int grid = g.total < num_sms() ? g.total : num_sms();
+    k_conv_tcq<BN><<<grid, THREADS_Q, CfgQ<BN>::SMEM, st>>>(map, p, g, xa, out32, out64, s1, hi, lo,
+                                                           err);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+bool tc_persistent() {
+    const char* e = getenv("IQ_TC_TILE_PER_CTA");
+    return !(e && e[0] == '1');
+}
+
 iq_status launch(const CUtensorMap& map, const TcP& p, int nsplit, const int8_t* xa,
                  const int8_t* xb, int32_t* out32, long long* out64, unsigned long long* s1,
                  int* hi, int* lo, int* err, cudaStream_t st) {
+    if (tc_persistent() && p.mode == MODE_FWD && nsplit == 1 && p.tap_mode &&
+        p.cstride % 16 == 0 && p.cofs % 16 == 0 && ((uintptr_t)xa & 15) == 0) {
+        switch (pick_bn(p.ncols)) {
+            case 64: return launch_q<64>(map, p, xa, out32, out64, s1, hi, lo, err, st);
+            case 128: return launch_q<128>(map, p, xa, out32, out64, s1, hi, lo, err, st);
+            default: return launch_q<256>(map, p, xa, out32, out64, s1, hi, lo, err, st);
+        }
+    }
+    if (tc_persistent()) {
+        switch (pick_bn(p.ncols)) {
+            case 64: return launch_p<64>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
+            case 128: return launch_p<128>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
+            default: return launch_p<256>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
+        }
+    }
     switch (pick_bn(p.ncols)) {
         case 64: return launch_bn<64>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
         case 128: return launch_bn<128>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
@@ -943,6 +2110,80 @@ iq_status try_launch_tma(const CUtensorMap& wmap, const TcP& p, const int8_t* x,
     return r;
 }
 
+// 4-D map over the fp16 carriers [N][H][W][cstride]: box 64 channels x BW x BH pixels at
+// the conv strides (element strides), 128-byte swizzle, zero fill outside the tensor
+iq_status encode_acts16(const __half* xf, int N, int H, int W, int cstride, const TmaTile& t,
+                        int sh, int sw, CUtensorMap* map) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
+    if (!enc) return IQ_ERR_UNSUPPORTED;
+    cuuint64_t gdim[4] = {(cuuint64_t)cstride, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+    cuuint64_t gstride[3] = {(cuuint64_t)cstride * 2, (cuuint64_t)W * cstride * 2,
+                             (cuuint64_t)H * W * cstride * 2};
+    cuuint32_t box[4] = {64, (cuuint32_t)(t.BW * sw), (cuuint32_t)(t.BH * sh), 1};
+    cuuint32_t estr[4] = {1, (cuuint32_t)sw, (cuuint32_t)sh, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, (void*)xf, gdim, gstride, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
+}
+
+bool tma16_disabled() {
+    const char* e = getenv("IQ_TC_GATHER");
+    return e && e[0] == '1';
+}
+
+// Whether the all-TMA kernel takes this problem (whole 64-channel k-blocks, strides 1 or
+// 2, aligned slices, a rectangle tiling with little waste)
+bool tma16_ok(const TcP& p, TmaTile* t) {
+    if (tma16_disabled() || !p.tap_mode || p.sh > 2 || p.sw > 2 || (p.cstride % 8) ||
+        (p.cofs % 64))
+        return false;
+    if (!pick_tma_tile(p.P, p.Q, t)) return false;
+    return t->BW * p.sw <= 256 && t->BH * p.sh <= 256;
+}
+
+template <int BN>
+iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const TcP& p,
+                   const TmaTile& t, int32_t* out32, long long* out64, unsigned long long* s1,
+                   int* hi, int* lo, int* err, cudaStream_t st) {
+    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       CfgT<BN>::SMEM));
+    RectGrid g;
+    g.PT = t.PT; g.QT = t.QT; g.BW = t.BW; g.BH = t.BH;
+    g.mt = p.N * t.PT * t.QT;
+    g.nt = (p.ncols + BN - 1) / BN;
+    g.total = g.mt * g.nt;
+    const int grid = g.total < num_sms() ? g.total : num_sms();
+    k_conv_tct<BN><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(wmap, amap, p, g, out32, out64, s1,
+                                                           hi, lo, err);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+// widen the input codes into xf and run the all-TMA kernel; *used = false when not taken
+iq_status try_launch_t(const CUtensorMap& wmap, const TcP& p, const int8_t* x, __half* xf,
+                       bool convert, int32_t* out32, long long* out64, unsigned long long* s1,
+                       int* hi, int* lo, int* err, cudaStream_t st, bool* used) {
+    *used = false;
+    TmaTile t;
+    if (!xf || !tma16_ok(p, &t)) return IQ_OK;
+    if (convert) {
+        const int64_t n16 = (int64_t)p.N * p.H * p.W * p.cstride / 16;
+        k_codes_to_f16<<<grid_for(n16), kThreads, 0, st>>>(x, xf, n16);
+        IQ_LAUNCH_CHECK();
+    }
+    CUtensorMap amap;
+    iq_status r = encode_acts16(xf, p.N, p.H, p.W, p.cstride, t, p.sh, p.sw, &amap);
+    if (r != IQ_OK) return r;
+    switch (pick_bn(p.ncols)) {
+        case 64: r = launch_t<64>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
+        case 128: r = launch_t<128>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
+        default: r = launch_t<256>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
+    }
+    if (r == IQ_OK) *used = true;
+    return r;
+}
+
 void fill_geom(TcP& p, const iq_conv_desc* d) {
     p.N = d->n; p.H = d->h; p.W = d->w; p.C = d->c; p.K = d->k; p.R = d->r; p.S = d->s;
     p.sh = d->stride_h; p.sw = d->stride_w; p.ph = d->pad_h; p.pw = d->pad_w;
@@ -960,10 +2201,14 @@ constexpr int MAX_KB_INT32 = 133120 / 64;   // 2080 k-blocks: 133120 * 127^2 < 2
 
 // ================================================================ forward
 
+// fp16 weights, the error word, then the fp16 carriers of the input
+static size_t acts16_offset(size_t wbytes) { return (wbytes + 256 + 255) / 256 * 256; }
+
 size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d) {
     int64_t kdim = (int64_t)d->r * d->s * (d->c / d->groups);
     int64_t kpad = (kdim + 63) / 64 * 64;
-    return (size_t)(d->k * kpad * 2) + 512;
+    const size_t wb = (size_t)(d->k * kpad * 2);
+    return acts16_offset(wb) + (size_t)d->n * d->h * d->w * d->c * 2 + 512;
 }
 
 bool conv_fwd_tc_supported(const iq_conv_desc* d) {
@@ -999,8 +2244,13 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     CUtensorMap map;
     iq_status r = encode_weights(wf, p.K, p.kpad, pick_bn(p.ncols), &map);
     if (r != IQ_OK) return r;
+    __half* xf = reinterpret_cast<__half*>(wsb + acts16_offset((size_t)p.K * p.kpad * 2));
     bool used = false;
-    r = try_launch_tma(map, p, x, acc, nullptr, s1, hi, lo, err, st, &used);
+    if ((p.N * (int64_t)p.H * p.W * p.cstride) % 16 == 0) {
+        r = try_launch_t(map, p, x, xf, true, acc, nullptr, s1, hi, lo, err, st, &used);
+        if (r != IQ_OK) return r;
+    }
+    if (!used) r = try_launch_tma(map, p, x, acc, nullptr, s1, hi, lo, err, st, &used);
     if (r != IQ_OK) return r;
     if (!used) r = launch(map, p, 1, x, nullptr, acc, nullptr, s1, hi, lo, err, st);
     if (r == IQ_OK) *done = true;
@@ -1025,7 +2275,10 @@ size_t conv_dgrad_tc_ws_bytes(const iq_conv_desc* d) {
     int nsl = conv_dgrad_tc_slices(d);
     if (nsl < 1) nsl = 1;
     int64_t kpad = ((int64_t)d->r * d->s * (d->k / nsl) + 63) / 64 * 64;
-    return (size_t)(d->c * kpad * 2) + 512;
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    const size_t wb = (size_t)(d->c * kpad * 2);
+    return acts16_offset(wb) + (size_t)d->n * P * Q * d->k * 2 + 512;
 }
 
 bool conv_dgrad_tc_supported(const iq_conv_desc* d) {
@@ -1070,6 +2323,8 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
     __half* wf = reinterpret_cast<__half*>(wsb);
     int* err = reinterpret_cast<int*>(wsb + (size_t)d->c * p.kpad * 2);
     IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
+    __half* ef = reinterpret_cast<__half*>(wsb + acts16_offset((size_t)d->c * p.kpad * 2));
+    const bool ef_ok = ((int64_t)p.N * p.H * p.W * p.cstride) % 16 == 0;
     for (int sl = 0; sl < nsl; sl++) {
         k_widen_weights_dgrad<<<grid_for((int64_t)d->c * p.kpad), kThreads, 0, st>>>(
             w, wf, d->k, d->r, d->s, d->c, sl * kc, kc, p.kpad);
@@ -1079,7 +2334,11 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
         if (r != IQ_OK) return r;
         p.cofs = sl * kc;
         bool used = false;
-        r = try_launch_tma(map, p, e, out32, out64, s1, hi, lo, err, st, &used);
+        if (ef_ok) {
+            r = try_launch_t(map, p, e, ef, sl == 0, out32, out64, s1, hi, lo, err, st, &used);
+            if (r != IQ_OK) return r;
+        }
+        if (!used) r = try_launch_tma(map, p, e, out32, out64, s1, hi, lo, err, st, &used);
         if (r != IQ_OK) return r;
         if (!used) r = launch(map, p, 1, e, nullptr, out32, out64, s1, hi, lo, err, st);
         if (r != IQ_OK) return r;
