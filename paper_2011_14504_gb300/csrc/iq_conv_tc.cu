@@ -1408,7 +1408,62 @@ __device__ __forceinline__ void write_row(const TcP& p, const uint32_t (&r)[LDW]
     }
 }
 
-template <int BN>
+// weight-gradient tile position: (channel tile, column tile, K split) and k-block
+struct WgPos {
+    int tile, kb, nkb, kb0;
+    int64_t m0;
+    int n0;
+};
+
+__device__ __forceinline__ void wpos_set(WgPos& q, int tile, const TcP& p, const RectGrid& g,
+                                         int BN) {
+    q.tile = tile;
+    q.kb = 0;
+    q.nkb = 0;
+    if (tile >= g.total) return;
+    const int mt = tile % g.mt;
+    const int rest = tile / g.mt;
+    const int nt = rest % g.nt;
+    const int sp = rest / g.nt;
+    q.m0 = (int64_t)mt * BM;
+    q.n0 = nt * BN;
+    q.kb0 = sp * p.kb_per_split;
+    const int n = p.nkb_total - q.kb0;
+    q.nkb = n > p.kb_per_split ? p.kb_per_split : n;
+}
+
+__device__ __forceinline__ void wpos_next(WgPos& q, const TcP& p, const RectGrid& g, int BN) {
+    if (q.tile >= g.total) return;
+    if (++q.kb >= q.nkb) wpos_set(q, q.tile + gridDim.x, p, g, BN);
+}
+
+template <bool WG>
+struct TPos;
+
+template <>
+struct TPos<false> : RectPos {
+    int nkb;
+    __device__ void set(int t, const TcP& p, const RectGrid& g, int BN) {
+        rpos_set(*this, t, g, BN);
+        nkb = p.nkb_total;
+    }
+    __device__ void next(const TcP& p, const RectGrid& g, int BN) {
+        rpos_next(*this, p, g, BN);
+    }
+};
+
+template <>
+struct TPos<true> : WgPos {
+    __device__ void set(int t, const TcP& p, const RectGrid& g, int BN) { wpos_set(*this, t, p, g, BN); }
+    __device__ void next(const TcP& p, const RectGrid& g, int BN) { wpos_next(*this, p, g, BN); }
+};
+
+// WG: the weight gradient.  Then A = E^T (two 2-D boxes of 64 channels x 64 consecutive
+// pixels of the fp16 errors, map `wmap`) and B = the im2col of x (one 4-D box per 64-column
+// tap block: 64 channels x the k-block's 64 output pixels as a BW x BH rectangle at the conv
+// strides, map `amap`), both MN-major; tiles are (channel tile, column tile, K split) and
+// the epilogue adds its int32 sums into the int64 output.
+template <int BN, bool WG>
 __global__ void __launch_bounds__(THREADS_T, 1)
     k_conv_tct(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap amap,
                TcP p, RectGrid g, int32_t* __restrict__ out32, long long* __restrict__ out64,
@@ -1454,7 +1509,55 @@ __global__ void __launch_bounds__(THREADS_T, 1)
 
     if (warp == 0) {
         // ================================================ TMA issuer
-        if (lane == 0) {
+        if constexpr (WG) {
+          if (lane == 0) {
+            tc::tma_prefetch_desc(&amap);
+            tc::tma_prefetch_desc(&wmap);
+            WgPos q;
+            wpos_set(q, blockIdx.x, p, g, BN);
+            uint32_t kbc = 0;
+            int issued = 0;
+            const int64_t pq = (int64_t)p.P * p.Q;
+            while (q.tile < g.total) {
+                const int s = kbc % STAGES_T;
+                const uint32_t it = kbc / STAGES_T;
+                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                    bars->abort = 1;
+                    atomicExch(err, 4);
+                    break;
+                }
+                uint8_t* st = smem + s * STAGE_BYTES;
+                tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
+                const int64_t j0 = (int64_t)(q.kb0 + q.kb) * BK;     // first pixel of the k-block
+                // A: E[j0 .. j0+63][m0 .. m0+127] as two 64-channel boxes
+                tc::tma_load_2d(st, &wmap, &bars->full[s], (int)q.m0, (int)j0);
+                tc::tma_load_2d(st + 8192, &wmap, &bars->full[s], (int)q.m0 + 64, (int)j0);
+                // B: per 64-column block (one tap, 64 channels) the input box of the pixels
+                const int nimg = (int)(j0 / pq);
+                const int rem = (int)(j0 - (int64_t)nimg * pq);
+                const int pp = rem / p.Q, qq = rem - (rem / p.Q) * p.Q;
+#pragma unroll
+                for (int bb = 0; bb < BN / 64; bb++) {
+                    const int col = q.n0 + 64 * bb;
+                    const int tap = col / p.C;
+                    const int c0 = col - tap * p.C;
+                    const int r = tap / p.S, ss = tap - r * p.S;
+                    tc::tma_load_4d(st + A_BYTES + 8192 * bb, &amap, &bars->full[s], c0,
+                                    qq * p.sw + ss * p.dw - p.pw, pp * p.sh + r * p.dh - p.ph,
+                                    nimg);
+                }
+                tc::mbar_arrive(&bars->full[s]);
+                issued = (int)kbc + 1;
+                kbc++;
+                wpos_next(q, p, g, BN);
+            }
+            if (*abort_flag) {
+                for (int kb = (issued > STAGES_T ? issued - STAGES_T : 0); kb < issued; kb++)
+                    tc::mbar_wait(&bars->full[kb % STAGES_T], (uint32_t)(kb / STAGES_T) & 1,
+                                  &bars->never);
+            }
+          }
+        } else if (lane == 0) {
             tc::tma_prefetch_desc(&amap);
             tc::tma_prefetch_desc(&wmap);
             RectPos q;
@@ -1500,16 +1603,16 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     } else if (warp == 1) {
         // ================================================ MMA issuer
         if (lane == 0) {
-            const uint32_t idesc = idesc_f16(BM, BN, false);
+            const uint32_t idesc = idesc_f16(BM, BN, WG);
             bool ok = true;
             uint32_t kbc = 0, cc = 0;
-            RectPos q;
-            rpos_set(q, blockIdx.x, g, BN);
+            TPos<WG> q;
+            q.set(blockIdx.x, p, g, BN);
             while (ok && q.tile < g.total) {
                 const int s = kbc % STAGES_T;
                 const uint32_t it = kbc / STAGES_T;
                 const bool first = (q.kb % CHUNK_KB) == 0;
-                const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == p.nkb_total - 1;
+                const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
                 const uint32_t buf = cc & 1;
                 if (first && cc >= 2 &&
                     !tc::mbar_wait(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
@@ -1524,17 +1627,24 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 const uint32_t a_addr = tc::smem_u32(smem + s * STAGE_BYTES);
                 const uint32_t b_addr = a_addr + A_BYTES;
 #pragma unroll
-                for (int k = 0; k < BK / 16; k++)
-                    tc::umma_f16(tmem + buf * BN, tc::sdesc_kmajor_sw128(a_addr + 32 * k),
-                                 tc::sdesc_kmajor_sw128(b_addr + 32 * k), idesc,
-                                 (first && k == 0) ? 0u : 1u);
+                for (int k = 0; k < BK / 16; k++) {
+                    uint64_t ad, bd;
+                    if (WG) {
+                        ad = sdesc_mnmajor_sw128(a_addr + 2 * 1024 * k);
+                        bd = sdesc_mnmajor_sw128(b_addr + 2 * 1024 * k);
+                    } else {
+                        ad = tc::sdesc_kmajor_sw128(a_addr + 32 * k);
+                        bd = tc::sdesc_kmajor_sw128(b_addr + 32 * k);
+                    }
+                    tc::umma_f16(tmem + buf * BN, ad, bd, idesc, (first && k == 0) ? 0u : 1u);
+                }
                 tc::umma_commit(&bars->empty[s]);
                 if (last) {
                     tc::umma_commit(&bars->accf[buf]);
                     cc++;
                 }
                 kbc++;
-                rpos_next(q, p, g, BN);
+                q.next(p, g, BN);
             }
             if (!ok) {
                 bars->abort = 1;
@@ -1552,11 +1662,11 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         const int dp = row / g.BW, dq = row - (row / g.BW) * g.BW;
         uint32_t cc = 0;
         bool ok = true;
-        RectPos q;
-        rpos_set(q, blockIdx.x, g, BN);
-        const int nch = (p.nkb_total + CHUNK_KB - 1) / CHUNK_KB;
+        TPos<WG> q;
+        q.set(blockIdx.x, p, g, BN);
         int sum[CW];
         while (ok && q.tile < g.total) {
+            const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
 #pragma unroll
             for (int i = 0; i < CW; i++) sum[i] = 0;
             for (int c = 0; c < nch; c++) {
@@ -1581,9 +1691,16 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 cc++;
             }
             if (!ok || *abort_flag) break;
-            const int pp = q.p0 + dp, qq = q.q0 + dq;
-            const bool valid = pp < p.P && qq < p.Q;
-            const int64_t m = ((int64_t)q.n * p.P + pp) * p.Q + qq;
+            bool valid;
+            int64_t m;
+            if constexpr (WG) {
+                m = q.m0 + row;
+                valid = m < p.M;
+            } else {
+                const int pp = q.p0 + dp, qq = q.q0 + dq;
+                valid = pp < p.P && qq < p.Q;
+                m = ((int64_t)q.n * p.P + pp) * p.Q + qq;
+            }
             if (__any_sync(0xffffffffu, valid)) {
 #pragma unroll
                 for (int cb = 0; cb < CW; cb += LDW) {
@@ -1594,7 +1711,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                                    s1, hi_c, lo_c);
                 }
             }
-            rpos_set(q, q.tile + gridDim.x, g, BN);
+            q.set(q.tile + gridDim.x, p, g, BN);
         }
     }
     tc::tc_fence_before();
@@ -2146,16 +2263,16 @@ template <int BN>
 iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const TcP& p,
                    const TmaTile& t, int32_t* out32, long long* out64, unsigned long long* s1,
                    int* hi, int* lo, int* err, cudaStream_t st) {
-    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       CfgT<BN>::SMEM));
+    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN, false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, CfgT<BN>::SMEM));
     RectGrid g;
     g.PT = t.PT; g.QT = t.QT; g.BW = t.BW; g.BH = t.BH;
     g.mt = p.N * t.PT * t.QT;
     g.nt = (p.ncols + BN - 1) / BN;
     g.total = g.mt * g.nt;
     const int grid = g.total < num_sms() ? g.total : num_sms();
-    k_conv_tct<BN><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(wmap, amap, p, g, out32, out64, s1,
-                                                           hi, lo, err);
+    k_conv_tct<BN, false><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(wmap, amap, p, g, out32, out64,
+                                                                  s1, hi, lo, err);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }
@@ -2349,7 +2466,62 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
 
 // ================================================================ weight gradient
 
-size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc*) { return 512; }
+// the error word, then the fp16 carriers of the errors and of the input
+size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d) {
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    const size_t eb = ((size_t)d->n * P * Q * d->k * 2 + 255) / 256 * 256;
+    return 256 + eb + (size_t)d->n * d->h * d->w * d->c * 2 + 512;
+}
+
+namespace {
+
+// 2-D map over the fp16 errors [npq][K]: box 64 channels x 64 pixels, 128-byte swizzle
+iq_status encode_err16(const __half* ef, int64_t npq, int K, CUtensorMap* map) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
+    if (!enc) return IQ_ERR_UNSUPPORTED;
+    cuuint64_t gdim[2] = {(cuuint64_t)K, (cuuint64_t)npq};
+    cuuint64_t gstride[1] = {(cuuint64_t)K * 2};
+    cuuint32_t box[2] = {64, 64};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, (void*)ef, gdim, gstride, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
+}
+
+// the k-block's 64 output pixels as a rectangle of one image: whole 64-pixel runs of a row,
+// or whole rows when Q divides 64 (and the images hold whole rectangles)
+bool wgrad_rect(const TcP& p, TmaTile* t) {
+    if (p.Q % 64 == 0) {
+        t->BW = 64; t->BH = 1;
+    } else if (64 % p.Q == 0 && p.P % (64 / p.Q) == 0) {
+        t->BW = p.Q; t->BH = 64 / p.Q;
+    } else {
+        return false;
+    }
+    t->PT = t->QT = 1;
+    return t->BW * p.sw <= 256 && t->BH * p.sh <= 256;
+}
+
+template <int BN>
+iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP& p,
+                    const TmaTile& t, int nsplit, long long* G, int* err, cudaStream_t st) {
+    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN, true>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, CfgT<BN>::SMEM));
+    RectGrid g;
+    g.PT = 1; g.QT = 1; g.BW = t.BW; g.BH = t.BH;
+    g.mt = (int)((p.M + BM - 1) / BM);
+    g.nt = (p.ncols + BN - 1) / BN;
+    g.total = g.mt * g.nt * nsplit;
+    const int grid = g.total < num_sms() ? g.total : num_sms();
+    k_conv_tct<BN, true><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(emap, xmap, p, g, nullptr, G,
+                                                                 nullptr, nullptr, nullptr, err);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+}  // namespace
 
 bool conv_wgrad_tc_supported(const iq_conv_desc* d) {
     if (tc_env_disabled()) return false;
@@ -2374,16 +2546,45 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
     p.nkb_total = (int)nkb;
     const int bn = pick_bn(p.ncols);
     const int64_t tiles = ((p.M + BM - 1) / BM) * ((p.ncols + bn - 1) / bn);
-    // enough splits to fill the GPU twice over, each split within the int32 bound
-    int64_t want = (2 * 152 + tiles - 1) / tiles;
-    int64_t kbs = (nkb + want - 1) / want;
-    if (kbs < 32) kbs = 32;
-    if (kbs > MAX_KB_INT32) kbs = MAX_KB_INT32;
+    // the split of the reduction that minimises (tiles per SM) x (k-blocks per tile) on the
+    // persistent grid, each split within the int32 bound and at least 16 k-blocks long
+    const int64_t sms = num_sms();
+    int64_t best_cost = INT64_MAX, kbs = MAX_KB_INT32;
+    for (int64_t ns = 1; ns <= 256; ns++) {
+        const int64_t k = (nkb + ns - 1) / ns;
+        if (k > MAX_KB_INT32) continue;
+        if (k < 16 && ns > 1) break;
+        const int64_t nsr = (nkb + k - 1) / k;
+        const int64_t cost = ((tiles * nsr + sms - 1) / sms) * k;
+        if (cost < best_cost) { best_cost = cost; kbs = k; }
+    }
     p.kb_per_split = (int)kbs;
     const int nsplit = (int)((nkb + kbs - 1) / kbs);
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     int* err = reinterpret_cast<int*>(wsb);
     IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
+    TmaTile t;
+    const int64_t ne = p.npq * p.K, nx = (int64_t)p.N * p.H * p.W * p.C;
+    if (!tma16_disabled() && p.C % 64 == 0 && p.K % 8 == 0 && p.sh <= 2 && p.sw <= 2 &&
+        ne % 16 == 0 && nx % 16 == 0 && get_encode() && wgrad_rect(p, &t)) {
+        __half* ef = reinterpret_cast<__half*>(wsb + 256);
+        __half* xf = reinterpret_cast<__half*>(wsb + 256 + ((size_t)ne * 2 + 255) / 256 * 256);
+        k_codes_to_f16<<<grid_for(ne / 16), kThreads, 0, st>>>(e, ef, ne / 16);
+        IQ_LAUNCH_CHECK();
+        k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
+        IQ_LAUNCH_CHECK();
+        CUtensorMap emap, xmap;
+        iq_status r = encode_err16(ef, p.npq, p.K, &emap);
+        if (r == IQ_OK) r = encode_acts16(xf, p.N, p.H, p.W, p.C, t, p.sh, p.sw, &xmap);
+        if (r != IQ_OK) return r;
+        switch (bn) {
+            case 64: r = launch_tw<64>(emap, xmap, p, t, nsplit, G, err, st); break;
+            case 128: r = launch_tw<128>(emap, xmap, p, t, nsplit, G, err, st); break;
+            default: r = launch_tw<256>(emap, xmap, p, t, nsplit, G, err, st); break;
+        }
+        if (r == IQ_OK) *done = true;
+        return r;
+    }
     CUtensorMap dummy;
     memset(&dummy, 0, sizeof(dummy));
     iq_status r = launch(dummy, p, nsplit, e, x, nullptr, G, nullptr, nullptr, nullptr, err, st);
