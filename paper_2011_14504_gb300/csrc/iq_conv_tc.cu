@@ -1458,9 +1458,10 @@ struct TPos<true> : WgPos {
     __device__ void next(const TcP& p, const RectGrid& g, int BN) { wpos_next(*this, p, g, BN); }
 };
 
-// WG: the weight gradient.  Then A = E^T (two 2-D boxes of 64 channels x 64 consecutive
-// pixels of the fp16 errors, map `wmap`) and B = the im2col of x (one 4-D box per 64-column
-// tap block: 64 channels x the k-block's 64 output pixels as a BW x BH rectangle at the conv
+// WG: the weight gradient.  A k-block is a BW x BH rectangle of 64 output pixels of one
+// image (the rectangles tile every image; pixels outside it read zero errors).  A = E^T
+// (two 4-D boxes of 64 channels x the rectangle of the fp16 errors, map `wmap`) and B = the
+// im2col of x (one 4-D box per 64-column tap block: 64 channels x the rectangle at the conv
 // strides, map `amap`), both MN-major; tiles are (channel tile, column tile, K split) and
 // the epilogue adds its int32 sums into the int64 output.
 template <int BN, bool WG>
@@ -1517,7 +1518,6 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             wpos_set(q, blockIdx.x, p, g, BN);
             uint32_t kbc = 0;
             int issued = 0;
-            const int64_t pq = (int64_t)p.P * p.Q;
             while (q.tile < g.total) {
                 const int s = kbc % STAGES_T;
                 const uint32_t it = kbc / STAGES_T;
@@ -1528,14 +1528,15 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 }
                 uint8_t* st = smem + s * STAGE_BYTES;
                 tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
-                const int64_t j0 = (int64_t)(q.kb0 + q.kb) * BK;     // first pixel of the k-block
-                // A: E[j0 .. j0+63][m0 .. m0+127] as two 64-channel boxes
-                tc::tma_load_2d(st, &wmap, &bars->full[s], (int)q.m0, (int)j0);
-                tc::tma_load_2d(st + 8192, &wmap, &bars->full[s], (int)q.m0 + 64, (int)j0);
+                // the k-block's pixels: rectangle kb of the BW x BH tiling of the output
+                const int kr = q.kb0 + q.kb;
+                const int nimg = kr / (g.PT * g.QT);
+                const int rr = kr - nimg * (g.PT * g.QT);
+                const int pp = (rr / g.QT) * g.BH, qq = (rr - (rr / g.QT) * g.QT) * g.BW;
+                // A: E[rectangle][m0 .. m0+127] as two 64-channel boxes (zero outside P x Q)
+                tc::tma_load_4d(st, &wmap, &bars->full[s], (int)q.m0, qq, pp, nimg);
+                tc::tma_load_4d(st + 8192, &wmap, &bars->full[s], (int)q.m0 + 64, qq, pp, nimg);
                 // B: per 64-column block (one tap, 64 channels) the input box of the pixels
-                const int nimg = (int)(j0 / pq);
-                const int rem = (int)(j0 - (int64_t)nimg * pq);
-                const int pp = rem / p.Q, qq = rem - (rem / p.Q) * p.Q;
 #pragma unroll
                 for (int bb = 0; bb < BN / 64; bb++) {
                     const int col = q.n0 + 64 * bb;
@@ -2158,7 +2159,7 @@ iq_status launch(const CUtensorMap& map, const TcP& p, int nsplit, const int8_t*
 
 // Tile rectangle for the TMA-fed kernel: BW x BH = 128 output pixels; the shape with the
 // least padding waste, if that waste is small.
-bool pick_tma_tile(int P, int Q, TmaTile* t) {
+bool pick_tma_tile(int P, int Q, TmaTile* t, double min_util = 0.8) {
     double best = 0.0;
     for (int BW = 128; BW >= 16; BW /= 2) {
         const int BH = 128 / BW;
@@ -2169,7 +2170,7 @@ bool pick_tma_tile(int P, int Q, TmaTile* t) {
             t->BW = BW; t->BH = BH; t->PT = PT; t->QT = QT;
         }
     }
-    return best >= 0.8;
+    return best >= min_util;
 }
 
 iq_status encode_acts(const int8_t* x, int N, int H, int W, int cstride, const TmaTile& t,
@@ -2255,7 +2256,7 @@ bool tma16_ok(const TcP& p, TmaTile* t) {
     if (tma16_disabled() || !p.tap_mode || p.sh > 2 || p.sw > 2 || (p.cstride % 8) ||
         (p.cofs % 64))
         return false;
-    if (!pick_tma_tile(p.P, p.Q, t)) return false;
+    if (!pick_tma_tile(p.P, p.Q, t, 0.6)) return false;
     return t->BW * p.sw <= 256 && t->BH * p.sh <= 256;
 }
 
@@ -2476,32 +2477,21 @@ size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d) {
 
 namespace {
 
-// 2-D map over the fp16 errors [npq][K]: box 64 channels x 64 pixels, 128-byte swizzle
-iq_status encode_err16(const __half* ef, int64_t npq, int K, CUtensorMap* map) {
-    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
-    if (!enc) return IQ_ERR_UNSUPPORTED;
-    cuuint64_t gdim[2] = {(cuuint64_t)K, (cuuint64_t)npq};
-    cuuint64_t gstride[1] = {(cuuint64_t)K * 2};
-    cuuint32_t box[2] = {64, 64};
-    cuuint32_t estr[2] = {1, 1};
-    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, (void*)ef, gdim, gstride, box, estr,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
-}
-
-// the k-block's 64 output pixels as a rectangle of one image: whole 64-pixel runs of a row,
-// or whole rows when Q divides 64 (and the images hold whole rectangles)
+// the k-block rectangle of 64 output pixels (BW x BH) that wastes the fewest pixels at the
+// image borders
 bool wgrad_rect(const TcP& p, TmaTile* t) {
-    if (p.Q % 64 == 0) {
-        t->BW = 64; t->BH = 1;
-    } else if (64 % p.Q == 0 && p.P % (64 / p.Q) == 0) {
-        t->BW = p.Q; t->BH = 64 / p.Q;
-    } else {
-        return false;
+    double best = 0.0;
+    for (int BW = 64; BW >= 1; BW /= 2) {
+        const int BH = 64 / BW;
+        if (BW * p.sw > 256 || BH * p.sh > 256) continue;
+        const int PT = (p.P + BH - 1) / BH, QT = (p.Q + BW - 1) / BW;
+        const double util = (double)p.P * p.Q / ((double)PT * BH * QT * BW);
+        if (util > best + 1e-9) {
+            best = util;
+            t->BW = BW; t->BH = BH; t->PT = PT; t->QT = QT;
+        }
     }
-    t->PT = t->QT = 1;
-    return t->BW * p.sw <= 256 && t->BH * p.sh <= 256;
+    return best >= 0.5;
 }
 
 template <int BN>
@@ -2510,7 +2500,7 @@ iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP&
     IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN, true>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, CfgT<BN>::SMEM));
     RectGrid g;
-    g.PT = 1; g.QT = 1; g.BW = t.BW; g.BH = t.BH;
+    g.PT = t.PT; g.QT = t.QT; g.BW = t.BW; g.BH = t.BH;
     g.mt = (int)((p.M + BM - 1) / BM);
     g.nt = (p.ncols + BN - 1) / BN;
     g.total = g.mt * g.nt * nsplit;
@@ -2541,32 +2531,35 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
     p.ncols = p.R * p.S * p.C;
     p.npq = (int64_t)p.N * p.P * p.Q;
     p.kdim = 0; p.kpad = 0; p.tap_mode = 1;
-    const int64_t nkb = (p.npq + BK - 1) / BK;
-    if (nkb > INT_MAX) return IQ_OK;
-    p.nkb_total = (int)nkb;
     const int bn = pick_bn(p.ncols);
     const int64_t tiles = ((p.M + BM - 1) / BM) * ((p.ncols + bn - 1) / bn);
-    // the split of the reduction that minimises (tiles per SM) x (k-blocks per tile) on the
-    // persistent grid, each split within the int32 bound and at least 16 k-blocks long
-    const int64_t sms = num_sms();
-    int64_t best_cost = INT64_MAX, kbs = MAX_KB_INT32;
-    for (int64_t ns = 1; ns <= 256; ns++) {
-        const int64_t k = (nkb + ns - 1) / ns;
-        if (k > MAX_KB_INT32) continue;
-        if (k < 16 && ns > 1) break;
-        const int64_t nsr = (nkb + k - 1) / k;
-        const int64_t cost = ((tiles * nsr + sms - 1) / sms) * k;
-        if (cost < best_cost) { best_cost = cost; kbs = k; }
-    }
-    p.kb_per_split = (int)kbs;
-    const int nsplit = (int)((nkb + kbs - 1) / kbs);
+    // the split of the nkb k-blocks that minimises (tiles per SM) x (k-blocks per tile) on
+    // the persistent grid, each split within the int32 bound and at least 16 k-blocks long
+    auto split = [&](int64_t nkb) {
+        const int64_t sms = num_sms();
+        int64_t best_cost = INT64_MAX, kbs = MAX_KB_INT32;
+        for (int64_t ns = 1; ns <= 256; ns++) {
+            const int64_t k = (nkb + ns - 1) / ns;
+            if (k > MAX_KB_INT32) continue;
+            if (k < 16 && ns > 1) break;
+            const int64_t nsr = (nkb + k - 1) / k;
+            const int64_t cost = ((tiles * nsr + sms - 1) / sms) * k;
+            if (cost < best_cost) { best_cost = cost; kbs = k; }
+        }
+        p.nkb_total = (int)nkb;
+        p.kb_per_split = (int)kbs;
+        return (int)((nkb + kbs - 1) / kbs);
+    };
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     int* err = reinterpret_cast<int*>(wsb);
     IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
     TmaTile t;
     const int64_t ne = p.npq * p.K, nx = (int64_t)p.N * p.H * p.W * p.C;
     if (!tma16_disabled() && p.C % 64 == 0 && p.K % 8 == 0 && p.sh <= 2 && p.sw <= 2 &&
-        ne % 16 == 0 && nx % 16 == 0 && get_encode() && wgrad_rect(p, &t)) {
+        ne % 16 == 0 && nx % 16 == 0 && get_encode() && wgrad_rect(p, &t) &&
+        (int64_t)p.N * t.PT * t.QT <= INT_MAX) {
+        // k-blocks: the pixel rectangles of every image
+        const int nsplit = split((int64_t)p.N * t.PT * t.QT);
         __half* ef = reinterpret_cast<__half*>(wsb + 256);
         __half* xf = reinterpret_cast<__half*>(wsb + 256 + ((size_t)ne * 2 + 255) / 256 * 256);
         k_codes_to_f16<<<grid_for(ne / 16), kThreads, 0, st>>>(e, ef, ne / 16);
@@ -2574,7 +2567,7 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
         IQ_LAUNCH_CHECK();
         CUtensorMap emap, xmap;
-        iq_status r = encode_err16(ef, p.npq, p.K, &emap);
+        iq_status r = encode_acts16(ef, p.N, p.P, p.Q, p.K, t, 1, 1, &emap);
         if (r == IQ_OK) r = encode_acts16(xf, p.N, p.H, p.W, p.C, t, p.sh, p.sw, &xmap);
         if (r != IQ_OK) return r;
         switch (bn) {
@@ -2585,6 +2578,9 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         if (r == IQ_OK) *done = true;
         return r;
     }
+    const int64_t nkb = (p.npq + BK - 1) / BK;
+    if (nkb > INT_MAX) return IQ_OK;
+    const int nsplit = split(nkb);
     CUtensorMap dummy;
     memset(&dummy, 0, sizeof(dummy));
     iq_status r = launch(dummy, p, nsplit, e, x, nullptr, G, nullptr, nullptr, nullptr, err, st);
