@@ -368,6 +368,111 @@ __global__ void k_up_wgrad(UpP u, const int8_t* __restrict__ x, const int8_t* __
     }
 }
 
+// ---- the decoder's backward at kernel 64, stride 32, padding 16, on channel-major errors
+
+// NHWC -> NCHW bytes: block (n, row Ho, 128 columns): the 128 x c bytes of the row segment
+// come in as 16-byte loads, each channel's 128 bytes go out as 16-byte stores
+__global__ void k_up_tr(const int8_t* __restrict__ E, int8_t* __restrict__ Et, int H, int W,
+                        int c) {
+    extern __shared__ __align__(16) uint8_t tile[];
+    const int w0 = blockIdx.x * 128, Ho = blockIdx.y, b = blockIdx.z;
+    const int64_t src0 = (((int64_t)b * H + Ho) * W + w0) * c;
+    const int nbytes = 128 * c;
+    for (int i = threadIdx.x; i < nbytes / 16; i += blockDim.x)
+        reinterpret_cast<uint4*>(tile)[i] = __ldg(reinterpret_cast<const uint4*>(E + src0) + i);
+    __syncthreads();
+    for (int i = threadIdx.x; i < c * 8; i += blockDim.x) {
+        const int ch = i >> 3, seg = i & 7;
+        uint32_t w[4];
+#pragma unroll
+        for (int k = 0; k < 4; k++) {
+            uint32_t v = 0;
+#pragma unroll
+            for (int bb = 0; bb < 4; bb++)
+                v |= (uint32_t)tile[(seg * 16 + 4 * k + bb) * c + ch] << (8 * bb);
+            w[k] = v;
+        }
+        int8_t* dst = Et + (((int64_t)b * c + ch) * H + Ho) * W + w0 + seg * 16;
+        *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+// data gradient: thread per (n, c, i, j) with j fastest; each tap row r contributes the dot
+// product of 64 error bytes (4 x 16-byte loads of the channel-major row) with the weight row
+__global__ void __launch_bounds__(256) k_up32_bwd(UpP u, const int8_t* __restrict__ Et,
+                                                  const int8_t* __restrict__ w,
+                                                  int32_t* __restrict__ ex,
+                                                  unsigned long long* __restrict__ amax) {
+    const int64_t total = (int64_t)u.n * u.c * u.h * u.w;
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    uint32_t mx = 0;
+    if (idx < total) {
+        const int j = (int)(idx % u.w);
+        const int i = (int)((idx / u.w) % u.h);
+        const int ch = (int)((idx / ((int64_t)u.w * u.h)) % u.c);
+        const int b = (int)(idx / ((int64_t)u.w * u.h * u.c));
+        const int8_t* plane = Et + ((int64_t)b * u.c + ch) * u.H * u.W;
+        const int8_t* wr = w + (int64_t)ch * 64 * 64;
+        const int col0 = 32 * j - 16;
+        int sum = 0;
+        for (int r = 0; r < 64; r++) {
+            const int Ho = 32 * i + r - 16;
+            if (Ho < 0 || Ho >= u.H) continue;
+            const int8_t* row = plane + (int64_t)Ho * u.W;
+#pragma unroll
+            for (int q = 0; q < 4; q++) {
+                const int col = col0 + 16 * q;
+                if (col < 0 || col >= u.W) continue;
+                const int4 e = __ldg(reinterpret_cast<const int4*>(row + col));
+                const int4 f = __ldg(reinterpret_cast<const int4*>(wr + r * 64 + 16 * q));
+                sum = __dp4a(e.x, f.x, sum);
+                sum = __dp4a(e.y, f.y, sum);
+                sum = __dp4a(e.z, f.z, sum);
+                sum = __dp4a(e.w, f.w, sum);
+            }
+        }
+        ex[(((int64_t)b * u.h + i) * u.w + j) * u.c + ch] = sum;
+        mx = (uint32_t)(sum < 0 ? -sum : sum);
+    }
+    mx = warp_max_u32(mx);
+    if ((threadIdx.x & 31) == 0 && mx) atomicMax(amax, (unsigned long long)mx);
+}
+
+// weight gradient: block (c, 4 tap rows), 64 threads = 4 rows x 16 groups of 4 tap columns;
+// the channel's input codes sit in shared memory, each term is one 4-byte error load and
+// 4 products
+__global__ void __launch_bounds__(64) k_up32_wgrad(UpP u, const int8_t* __restrict__ x,
+                                                   const int8_t* __restrict__ Et,
+                                                   long long* __restrict__ g) {
+    extern __shared__ int8_t xs[];
+    const int ch = blockIdx.x, r = blockIdx.y * 4 + (threadIdx.x >> 4), q = threadIdx.x & 15;
+    const int nx = u.n * u.h * u.w;
+    for (int k = threadIdx.x; k < nx; k += blockDim.x) xs[k] = x[(int64_t)k * u.c + ch];
+    __syncthreads();
+    int s0 = 0, s1 = 0, s2 = 0, s3 = 0;
+    for (int b = 0; b < u.n; b++) {
+        const int8_t* plane = Et + ((int64_t)b * u.c + ch) * u.H * u.W;
+        for (int i = 0; i < u.h; i++) {
+            const int Ho = 32 * i + r - 16;
+            if (Ho < 0 || Ho >= u.H) continue;
+            const int8_t* row = plane + (int64_t)Ho * u.W;
+            const int8_t* xr = xs + (b * u.h + i) * u.w;
+            for (int j = 0; j < u.w; j++) {
+                const int col = 32 * j - 16 + 4 * q;
+                if (col < 0 || col >= u.W) continue;
+                const int xv = xr[j];
+                const int e = __ldg(reinterpret_cast<const int*>(row + col));
+                s0 += xv * (int)(int8_t)(e & 0xff);
+                s1 += xv * (int)(int8_t)((e >> 8) & 0xff);
+                s2 += xv * (int)(int8_t)((e >> 16) & 0xff);
+                s3 += xv * (int)(int8_t)(e >> 24);
+            }
+        }
+    }
+    long long* dst = g + ((int64_t)ch * 64 + r) * 64 + 4 * q;
+    dst[0] = s0; dst[1] = s1; dst[2] = s2; dst[3] = s3;
+}
+
 // ------------------------------------------------------------------ MSE loss gradient
 
 struct MseP {
@@ -567,8 +672,20 @@ static bool up_dims(int32_t n, int32_t h, int32_t w, int32_t c, int32_t R, int32
 extern "C" iq_status iq_upsample_workspace_size(int32_t n, int32_t h, int32_t w, int32_t c,
                                                 int32_t R, size_t* bytes) {
     if (!bytes || n <= 0 || h <= 0 || w <= 0 || c <= 0 || R <= 0) return IQ_ERR_INVALID_ARG;
-    *bytes = (size_t)c * R * R * 8 + (size_t)n * h * w * c * 4 + requant_ws_bytes() + 2048;
+    // + the channel-major copy of the errors used at kernel R, stride R/2 (H = h R/2)
+    *bytes = (size_t)c * R * R * 8 + (size_t)n * h * w * c * 4 + requant_ws_bytes() + 2048 +
+             (size_t)n * h * w * c * ((size_t)R / 2) * ((size_t)R / 2) + 256;
     return IQ_OK;
+}
+
+// whether the decoder backward can take the channel-major path: kernel 64, stride 32,
+// padding 16, output width a multiple of 128, aligned buffers, room in the workspace
+static bool up32_ok(const UpP& u, const void* E, const void* w, size_t ws_bytes, size_t used) {
+    return u.R == 64 && u.st == 32 && u.pad == 16 && u.W % 128 == 0 &&
+           (128 * (int64_t)u.c) % 16 == 0 && (((uintptr_t)E | (uintptr_t)w) & 15) == 0 &&
+           128 * u.c <= 48 * 1024 && u.n <= 65535 && u.H <= 65535 &&
+           (int64_t)u.n * u.h * u.w <= 48 * 1024 &&
+           ws_bytes >= used + (size_t)u.n * u.H * u.W * u.c + 256;
 }
 
 extern "C" iq_status iq_upsample_fwd(const int8_t* x, const double* s_x, const int8_t* w,
@@ -639,13 +756,23 @@ extern "C" iq_status iq_upsample_bwd(const int8_t* E, const double* s_e, const i
     void* rq = cur.take<char>(requant_ws_bytes());
     double* s_in = cur.take<double>(1);
     int32_t* acc = acc_out ? acc_out : sums;
-    k_up_wT<<<grid_for((int64_t)c * R * R), kThreads, 0, st>>>(w, wT, c, R);
-    IQ_LAUNCH_CHECK();
     unsigned long long* cell = (unsigned long long*)rq;
     IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, 8, st));
-    int thr = c >= 256 ? 256 : ((c + 31) / 32) * 32;
-    k_up_bwd<<<n * h * wd, thr, 0, st>>>(u, E, wT, acc, cell);
-    IQ_LAUNCH_CHECK();
+    if (up32_ok(u, E, w, ws_bytes, cur.off)) {
+        int8_t* Et = cur.take<int8_t>((size_t)n * u.H * u.W * c);
+        dim3 gt((unsigned)(u.W / 128), (unsigned)u.H, (unsigned)n);
+        k_up_tr<<<gt, 256, 128 * c, st>>>(E, Et, u.H, u.W, c);
+        IQ_LAUNCH_CHECK();
+        const int64_t total = (int64_t)n * c * h * wd;
+        k_up32_bwd<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(u, Et, w, acc, cell);
+        IQ_LAUNCH_CHECK();
+    } else {
+        k_up_wT<<<grid_for((int64_t)c * R * R), kThreads, 0, st>>>(w, wT, c, R);
+        IQ_LAUNCH_CHECK();
+        int thr = c >= 256 ? 256 : ((c + 31) / 32) * 32;
+        k_up_bwd<<<n * h * wd, thr, 0, st>>>(u, E, wT, acc, cell);
+        IQ_LAUNCH_CHECK();
+    }
     k_scale_pow2<<<1, 1, 0, st>>>(s_e, -7, s_in);
     IQ_LAUNCH_CHECK();
     return requant_apply(acc, IQ_I32, (int64_t)n * h * wd * c, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, ex,
@@ -672,9 +799,19 @@ extern "C" iq_status iq_upsample_wgrad(const int8_t* x, const double* s_x, const
     void* rq = cur.take<char>(requant_ws_bytes());
     double* s_in = cur.take<double>(1);
     int64_t* G = g_acc_out ? g_acc_out : gw;
-    int thr = c >= 256 ? 256 : ((c + 31) / 32) * 32;
-    k_up_wgrad<<<R * R, thr, 0, st>>>(u, x, E, (long long*)G);
-    IQ_LAUNCH_CHECK();
+    if (up32_ok(u, E, x, ws_bytes, cur.off)) {
+        int8_t* Et = cur.take<int8_t>((size_t)n * u.H * u.W * c);
+        dim3 gt((unsigned)(u.W / 128), (unsigned)u.H, (unsigned)n);
+        k_up_tr<<<gt, 256, 128 * c, st>>>(E, Et, u.H, u.W, c);
+        IQ_LAUNCH_CHECK();
+        k_up32_wgrad<<<dim3((unsigned)c, 16u), 64, (size_t)n * h * wd, st>>>(u, x, Et,
+                                                                          (long long*)G);
+        IQ_LAUNCH_CHECK();
+    } else {
+        int thr = c >= 256 ? 256 : ((c + 31) / 32) * 32;
+        k_up_wgrad<<<R * R, thr, 0, st>>>(u, x, E, (long long*)G);
+        IQ_LAUNCH_CHECK();
+    }
     k_scale_product<<<1, 1, 0, st>>>(s_x, s_e, s_in);
     IQ_LAUNCH_CHECK();
     return requant_int(G, IQ_I64, (int64_t)c * R * R, s_in, 8,

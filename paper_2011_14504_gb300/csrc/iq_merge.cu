@@ -232,6 +232,132 @@ __global__ void __launch_bounds__(kThreads) k_comb8(Terms T, int concat, int64_t
     }
 }
 
+// The same two passes with a fixed 8-channel group per thread: the launch has a multiple
+// of c_out / 8 threads, so thread t always owns group t % (c_out / 8) and keeps the F / B
+// rows of the (at most two) operands covering it in registers; it walks the pixels
+// t / (c_out / 8), + T / (c_out / 8), ...  Per 8 outputs the loads are one 8- or 16-byte
+// load per operand.
+struct Cover {
+    int n;              // operands covering the group (0..2)
+    int id0, id1;
+    int ch0, ch1;       // first channel of the group inside each operand
+};
+
+__device__ __forceinline__ void cover_of(const Terms& T, int concat, int co0, Cover& cv) {
+    cv.n = 0;
+    cv.id0 = cv.id1 = 0;
+    cv.ch0 = cv.ch1 = 0;
+#pragma unroll
+    for (int i = 0; i < IQ_MAX_TERMS; i++) {
+        if (i >= T.n) break;
+        const int ch = concat ? co0 - T.t[i].c_offset : co0;
+        if (ch < 0 || ch >= T.t[i].c) continue;
+        if (cv.n == 0) { cv.id0 = i; cv.ch0 = ch; }
+        else if (cv.n == 1) { cv.id1 = i; cv.ch1 = ch; }
+        cv.n++;
+    }
+}
+
+__device__ __forceinline__ const TermDev& term_at(const Terms& T, int i) {
+    switch (i) {
+        case 0: return T.t[0];
+        case 1: return T.t[1];
+        case 2: return T.t[2];
+        case 3: return T.t[3];
+        case 4: return T.t[4];
+        case 5: return T.t[5];
+        case 6: return T.t[6];
+        default: return T.t[7];
+    }
+}
+
+__device__ __forceinline__ void load8p(const void* codes, int is16, int64_t idx, int32_t v[8]) {
+    if (is16) {
+        const int4 q = __ldg(reinterpret_cast<const int4*>((const int16_t*)codes + idx));
+        const int w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            v[2 * j] = (int32_t)(int16_t)(w[j] & 0xffff);
+            v[2 * j + 1] = (int32_t)(w[j] >> 16);
+        }
+    } else {
+        const int2 q = __ldg(reinterpret_cast<const int2*>((const int8_t*)codes + idx));
+        const int w[2] = {q.x, q.y};
+#pragma unroll
+        for (int j = 0; j < 8; j++) v[j] = (int32_t)(int8_t)((w[j >> 2] >> (8 * (j & 3))) & 0xff);
+    }
+}
+
+template <int PASS>
+__global__ void __launch_bounds__(kThreads) k_comb8r(Terms T, int concat, int64_t npix, int cgs,
+                                                     int relu, const long long* __restrict__ F,
+                                                     const long long* __restrict__ B,
+                                                     CombHdr* hdr, int8_t* __restrict__ out,
+                                                     UDiv dhw, int any_bcast) {
+    uint64_t M = 0;
+    UDiv d2m;
+    if (PASS == 1) {
+        M = hdr->M;
+        d2m = hdr->div;
+    }
+    const int64_t tcount = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % cgs);
+    const int64_t pstride = tcount / cgs;
+    const int co0 = 8 * g;
+    Cover cv;
+    cover_of(T, concat, co0, cv);
+    long long f0[8], b0[8], f1[8], b1[8];
+    const TermDev& t0 = term_at(T, cv.id0);
+    const TermDev& t1 = term_at(T, cv.id1);
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+        f0[j] = cv.n > 0 ? F[t0.base + cv.ch0 + j] : 0;
+        b0[j] = cv.n > 0 ? B[t0.base + cv.ch0 + j] : 0;
+        f1[j] = cv.n > 1 ? F[t1.base + cv.ch1 + j] : 0;
+        b1[j] = cv.n > 1 ? B[t1.base + cv.ch1 + j] : 0;
+    }
+    const void* base0 = t0.codes;
+    const void* base1 = t1.codes;
+    const int is0 = t0.is16, is1 = t1.is16, c0 = t0.c, c1 = t1.c, bc0 = t0.bcast, bc1 = t1.bcast;
+    uint64_t mx = 0;
+    for (int64_t pix = t / cgs; pix < npix; pix += pstride) {
+        const int64_t img = any_bcast ? (int64_t)udiv((uint64_t)pix, dhw) : 0;
+        int32_t v0[8] = {0, 0, 0, 0, 0, 0, 0, 0}, v1[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        if (cv.n > 0) load8p(base0, is0, (bc0 ? img : pix) * c0 + cv.ch0, v0);
+        if (cv.n > 1) load8p(base1, is1, (bc1 ? img : pix) * c1 + cv.ch1, v1);
+        int64_t z[8];
+#pragma unroll
+        for (int j = 0; j < 8; j++)
+            z[j] = (int64_t)f0[j] * v0[j] + (int64_t)b0[j] + (int64_t)f1[j] * v1[j] + (int64_t)b1[j];
+        if (PASS == 0) {
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
+                uint64_t a = (uint64_t)(zz < 0 ? -zz : zz);
+                mx = a > mx ? a : mx;
+            }
+        } else {
+            uint32_t w[2] = {0u, 0u};
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
+                int64_t c = 0;
+                if (M) {
+                    uint64_t num = ((uint64_t)(zz + (int64_t)M) << 8) + M;
+                    c = clamp64((int64_t)udiv(num, d2m) - 128, -127, 127);
+                }
+                w[j >> 2] |= ((uint32_t)c & 0xffu) << (8 * (j & 3));
+            }
+            *reinterpret_cast<uint2*>(out + pix * (int64_t)cgs * 8 + co0) = make_uint2(w[0], w[1]);
+        }
+    }
+    if (PASS == 0) {
+        mx = warp_max_u64(mx);
+        if ((threadIdx.x & 31) == 0 && mx) atomicMax(&hdr->maxz, (unsigned long long)mx);
+    }
+}
+
 __global__ void k_comb_params(CombHdr* hdr, double* s_out) {
     const uint64_t M = hdr->maxz;
     hdr->M = M;
@@ -397,6 +523,40 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
         any_bcast = any_bcast || t.bcast;
     }
     const UDiv dhw = make_udiv((uint64_t)hw);
+    // at most two operands cover any 8-channel group: sums of up to two operands, and
+    // concatenations whose ranges overlap at most pairwise (checked per group on the host)
+    bool two = vec;
+    for (int co = 0; co < c_out && two; co += 8) {
+        int nc = 0;
+        for (int i = 0; i < n_terms; i++) {
+            const TermDev& t = T.t[i];
+            const int ch = concat ? co - t.c_offset : co;
+            if (ch >= 0 && ch < t.c) nc++;
+        }
+        two = nc <= 2;
+    }
+    if (two) {
+        const int cgs = c_out / 8;
+        const int64_t npix = n * hw;
+        // a multiple of cgs threads, about 8 blocks of 256 per SM
+        int64_t gcd = cgs, b2 = kThreads;
+        while (b2) { int64_t r = gcd % b2; gcd = b2; b2 = r; }
+        const int64_t unit = cgs / gcd;                 // blocks per whole number of groups
+        int64_t want = (npix * cgs + kThreads - 1) / kThreads;
+        if (want > 152 * 8) want = 152 * 8;
+        want = (want + unit - 1) / unit * unit;
+        if (want < unit) want = unit;
+        const int g = (int)want;
+        k_comb8r<0><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
+                                            dhw, any_bcast);
+        IQ_LAUNCH_CHECK();
+        k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
+        IQ_LAUNCH_CHECK();
+        k_comb8r<1><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
+                                            dhw, any_bcast);
+        IQ_LAUNCH_CHECK();
+        return IQ_OK;
+    }
     if (vec) {
         const int64_t nvec = total / 8;
         const int g = grid_for(nvec, kThreads, 152 * 8);

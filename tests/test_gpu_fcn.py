@@ -21,9 +21,10 @@ def host(t):
     return t.cpu().numpy()
 
 
-@pytest.mark.parametrize("classes,width,n", [(21, 0.125, 2), (150, 0.0625, 1)])
-def test_fcn_train_steps_match_oracle(classes, width, n):
-    h = w = 64
+@pytest.mark.parametrize("classes,width,n,h", [(21, 0.125, 2, 64), (150, 0.0625, 1, 64),
+                                               (150, 0.0625, 1, 128)])
+def test_fcn_train_steps_match_oracle(classes, width, n, h):
+    w = h
     seed = 3
     g = S.rng(100 + classes)
     net = FcnVgg16(n, h, w, classes=classes, width=width, seed=seed, lr_log2=6)

@@ -391,7 +391,8 @@ def test_maxpool(k, s, p):
 
 
 @pytest.mark.parametrize("n,h,c,R,st,pd", [(1, 2, 150, 64, 32, 16), (2, 3, 21, 16, 8, 4),
-                                           (2, 5, 150, 64, 32, 16), (1, 3, 40, 64, 32, 16)])
+                                           (2, 5, 150, 64, 32, 16), (1, 3, 40, 64, 32, 16),
+                                           (2, 4, 150, 64, 32, 16), (1, 8, 21, 64, 32, 16)])
 def test_upsample_fwd_bwd_wgrad(n, h, c, R, st, pd):
     g = S.rng(c + R)
     H = (h - 1) * st - 2 * pd + R
