@@ -51,7 +51,7 @@ struct Cfg {
 };
 
 enum { MODE_FWD = 0, MODE_WGRAD = 1 };
-enum { OUT_STATS = 0, OUT_ATOMIC64 = 1 };
+enum { OUT_STATS = 0, OUT_ATOMIC64 = 1, OUT_PART32 = 2 };
 
 struct TcP {
     int mode, out;
@@ -1368,6 +1368,17 @@ __device__ __forceinline__ void write_row(const TcP& p, const uint32_t (&r)[LDW]
                                           long long* __restrict__ out64,
                                           unsigned long long* __restrict__ s1,
                                           int* __restrict__ hi_c, int* __restrict__ lo_c) {
+    if (p.out == OUT_PART32) {
+        if (valid) {
+            int32_t* dst = out32 + m * p.ncols + c0;
+#pragma unroll
+            for (int i = 0; i < LDW / 4; i++)
+                if (c0 + 4 * i < p.ncols)
+                    reinterpret_cast<int4*>(dst)[i] = make_int4((int)r[4 * i], (int)r[4 * i + 1],
+                                                                (int)r[4 * i + 2], (int)r[4 * i + 3]);
+        }
+        return;
+    }
     if (p.out == OUT_STATS) {
         if (valid) {
             int32_t* dst = out32 + m * p.ncols + c0;
@@ -1702,13 +1713,19 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 valid = pp < p.P && qq < p.Q;
                 m = ((int64_t)q.n * p.P + pp) * p.Q + qq;
             }
+            int32_t* o32 = out32;
+            if constexpr (WG) {
+                // the split's own int32 slab (OUT_PART32): no atomics
+                if (p.out == OUT_PART32)
+                    o32 = out32 + (int64_t)(q.kb0 / p.kb_per_split) * p.M * p.ncols;
+            }
             if (__any_sync(0xffffffffu, valid)) {
 #pragma unroll
                 for (int cb = 0; cb < CW; cb += LDW) {
                     uint32_t v[LDW];
 #pragma unroll
                     for (int i = 0; i < LDW; i++) v[i] = (uint32_t)sum[cb + i];
-                    write_row<LDW>(p, v, m, valid, q.n0 + quarter * CW + cb, lane, out32, out64,
+                    write_row<LDW>(p, v, m, valid, q.n0 + quarter * CW + cb, lane, o32, out64,
                                    s1, hi_c, lo_c);
                 }
             }
@@ -1720,6 +1737,23 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     if (warp == 1) {
         tc::tc_fence_after();
         tc::tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+// G[i] += sum over the splits of their int32 partial sums (4 elements per thread)
+__global__ void k_split_sum(const int32_t* __restrict__ part, int ns, int64_t total4,
+                            long long* __restrict__ G) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total4; i += stride) {
+        long long a0 = 0, a1 = 0, a2 = 0, a3 = 0;
+        for (int sp = 0; sp < ns; sp++) {
+            const int4 v = __ldg(reinterpret_cast<const int4*>(part) + (int64_t)sp * total4 + i);
+            a0 += v.x; a1 += v.y; a2 += v.z; a3 += v.w;
+        }
+        longlong2* g2 = reinterpret_cast<longlong2*>(G) + 2 * i;
+        const longlong2 o0 = g2[0], o1 = g2[1];
+        g2[0] = make_longlong2(o0.x + a0, o0.y + a1);
+        g2[1] = make_longlong2(o1.x + a2, o1.y + a3);
     }
 }
 
@@ -2468,11 +2502,66 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
 // ================================================================ weight gradient
 
 // the error word, then the fp16 carriers of the errors and of the input
+namespace {
+
+// the split of nkb k-blocks that minimises (tiles per SM) x (k-blocks per tile) on the
+// persistent grid, each split within the int32 bound and at least 16 k-blocks long;
+// returns the number of splits, *kbs the k-blocks per split
+int choose_split(int64_t nkb, int64_t tiles, int64_t* kbs_out) {
+    const int64_t sms = num_sms();
+    int64_t best_cost = INT64_MAX, kbs = MAX_KB_INT32;
+    for (int64_t ns = 1; ns <= 256; ns++) {
+        const int64_t k = (nkb + ns - 1) / ns;
+        if (k > MAX_KB_INT32) continue;
+        if (k < 16 && ns > 1) break;
+        const int64_t nsr = (nkb + k - 1) / k;
+        const int64_t cost = ((tiles * nsr + sms - 1) / sms) * k;
+        if (cost < best_cost) { best_cost = cost; kbs = k; }
+    }
+    *kbs_out = kbs;
+    return (int)((nkb + kbs - 1) / kbs);
+}
+
+bool wgrad_rect(const TcP& p, TmaTile* t);
+
+// the all-TMA weight-gradient plan: geometry, k-block rectangles and splits
+bool wgrad_tma_plan(const iq_conv_desc* d, TcP* p, TmaTile* t, int* nsplit) {
+    fill_geom(*p, d);
+    p->mode = MODE_WGRAD;
+    p->M = p->K;
+    p->ncols = p->R * p->S * p->C;
+    p->npq = (int64_t)p->N * p->P * p->Q;
+    p->kdim = 0; p->kpad = 0; p->tap_mode = 1;
+    if (d->groups != 1 || p->C % 64 || p->K % 8 || p->sh > 2 || p->sw > 2) return false;
+    if ((p->npq * p->K) % 16 || ((int64_t)p->N * p->H * p->W * p->C) % 16) return false;
+    if (!wgrad_rect(*p, t)) return false;
+    const int64_t nkb = (int64_t)p->N * t->PT * t->QT;
+    if (nkb > INT_MAX) return false;
+    const int bn = pick_bn(p->ncols);
+    const int64_t tiles = ((p->M + BM - 1) / BM) * ((p->ncols + bn - 1) / bn);
+    int64_t kbs;
+    *nsplit = choose_split(nkb, tiles, &kbs);
+    p->nkb_total = (int)nkb;
+    p->kb_per_split = (int)kbs;
+    return true;
+}
+
+}  // namespace
+
+// the error word, the fp16 carriers of the errors and of the input, and the per-split
+// int32 partial sums of the all-TMA path
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d) {
     const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
     const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
     const size_t eb = ((size_t)d->n * P * Q * d->k * 2 + 255) / 256 * 256;
-    return 256 + eb + (size_t)d->n * d->h * d->w * d->c * 2 + 512;
+    const size_t xb = ((size_t)d->n * d->h * d->w * d->c * 2 + 255) / 256 * 256;
+    size_t parts = 0;
+    TcP p;
+    TmaTile t;
+    int ns = 1;
+    if (d->c > 0 && d->k > 0 && wgrad_tma_plan(d, &p, &t, &ns))
+        parts = (size_t)ns * d->k * d->r * d->s * d->c * 4;
+    return 256 + eb + xb + parts + 512;
 }
 
 namespace {
@@ -2496,7 +2585,7 @@ bool wgrad_rect(const TcP& p, TmaTile* t) {
 
 template <int BN>
 iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP& p,
-                    const TmaTile& t, int nsplit, long long* G, int* err, cudaStream_t st) {
+                    const TmaTile& t, int nsplit, int32_t* part, int* err, cudaStream_t st) {
     IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN, true>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, CfgT<BN>::SMEM));
     RectGrid g;
@@ -2505,7 +2594,7 @@ iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP&
     g.nt = (p.ncols + BN - 1) / BN;
     g.total = g.mt * g.nt * nsplit;
     const int grid = g.total < num_sms() ? g.total : num_sms();
-    k_conv_tct<BN, true><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(emap, xmap, p, g, nullptr, G,
+    k_conv_tct<BN, true><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(emap, xmap, p, g, part, nullptr,
                                                                  nullptr, nullptr, nullptr, err);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
@@ -2523,45 +2612,22 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
                         void* ws, cudaStream_t st, bool* done) {
     *done = false;
     if (!conv_wgrad_tc_supported(d) || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
-    TcP p;
-    fill_geom(p, d);
-    p.mode = MODE_WGRAD;
-    p.out = OUT_ATOMIC64;
-    p.M = p.K;
-    p.ncols = p.R * p.S * p.C;
-    p.npq = (int64_t)p.N * p.P * p.Q;
-    p.kdim = 0; p.kpad = 0; p.tap_mode = 1;
-    const int bn = pick_bn(p.ncols);
-    const int64_t tiles = ((p.M + BM - 1) / BM) * ((p.ncols + bn - 1) / bn);
-    // the split of the nkb k-blocks that minimises (tiles per SM) x (k-blocks per tile) on
-    // the persistent grid, each split within the int32 bound and at least 16 k-blocks long
-    auto split = [&](int64_t nkb) {
-        const int64_t sms = num_sms();
-        int64_t best_cost = INT64_MAX, kbs = MAX_KB_INT32;
-        for (int64_t ns = 1; ns <= 256; ns++) {
-            const int64_t k = (nkb + ns - 1) / ns;
-            if (k > MAX_KB_INT32) continue;
-            if (k < 16 && ns > 1) break;
-            const int64_t nsr = (nkb + k - 1) / k;
-            const int64_t cost = ((tiles * nsr + sms - 1) / sms) * k;
-            if (cost < best_cost) { best_cost = cost; kbs = k; }
-        }
-        p.nkb_total = (int)nkb;
-        p.kb_per_split = (int)kbs;
-        return (int)((nkb + kbs - 1) / kbs);
-    };
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     int* err = reinterpret_cast<int*>(wsb);
     IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
+    TcP p;
     TmaTile t;
-    const int64_t ne = p.npq * p.K, nx = (int64_t)p.N * p.H * p.W * p.C;
-    if (!tma16_disabled() && p.C % 64 == 0 && p.K % 8 == 0 && p.sh <= 2 && p.sw <= 2 &&
-        ne % 16 == 0 && nx % 16 == 0 && get_encode() && wgrad_rect(p, &t) &&
-        (int64_t)p.N * t.PT * t.QT <= INT_MAX) {
-        // k-blocks: the pixel rectangles of every image
-        const int nsplit = split((int64_t)p.N * t.PT * t.QT);
+    int nsplit = 1;
+    if (!tma16_disabled() && get_encode() && wgrad_tma_plan(d, &p, &t, &nsplit)) {
+        // k-blocks: the pixel rectangles of every image; each split writes its own int32
+        // partial sums, added into G afterwards
+        const int64_t ne = p.npq * p.K, nx = (int64_t)p.N * p.H * p.W * p.C;
+        const size_t eb = ((size_t)ne * 2 + 255) / 256 * 256;
+        const size_t xb = ((size_t)nx * 2 + 255) / 256 * 256;
         __half* ef = reinterpret_cast<__half*>(wsb + 256);
-        __half* xf = reinterpret_cast<__half*>(wsb + 256 + ((size_t)ne * 2 + 255) / 256 * 256);
+        __half* xf = reinterpret_cast<__half*>(wsb + 256 + eb);
+        int32_t* part = reinterpret_cast<int32_t*>(wsb + 256 + eb + xb);
+        p.out = OUT_PART32;
         k_codes_to_f16<<<grid_for(ne / 16), kThreads, 0, st>>>(e, ef, ne / 16);
         IQ_LAUNCH_CHECK();
         k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
@@ -2570,17 +2636,33 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         iq_status r = encode_acts16(ef, p.N, p.P, p.Q, p.K, t, 1, 1, &emap);
         if (r == IQ_OK) r = encode_acts16(xf, p.N, p.H, p.W, p.C, t, p.sh, p.sw, &xmap);
         if (r != IQ_OK) return r;
-        switch (bn) {
-            case 64: r = launch_tw<64>(emap, xmap, p, t, nsplit, G, err, st); break;
-            case 128: r = launch_tw<128>(emap, xmap, p, t, nsplit, G, err, st); break;
-            default: r = launch_tw<256>(emap, xmap, p, t, nsplit, G, err, st); break;
+        switch (pick_bn(p.ncols)) {
+            case 64: r = launch_tw<64>(emap, xmap, p, t, nsplit, part, err, st); break;
+            case 128: r = launch_tw<128>(emap, xmap, p, t, nsplit, part, err, st); break;
+            default: r = launch_tw<256>(emap, xmap, p, t, nsplit, part, err, st); break;
         }
-        if (r == IQ_OK) *done = true;
-        return r;
+        if (r != IQ_OK) return r;
+        const int64_t total4 = p.M * (int64_t)p.ncols / 4;
+        k_split_sum<<<grid_for(total4), kThreads, 0, st>>>(part, nsplit, total4, G);
+        IQ_LAUNCH_CHECK();
+        *done = true;
+        return IQ_OK;
     }
+    fill_geom(p, d);
+    p.mode = MODE_WGRAD;
+    p.out = OUT_ATOMIC64;
+    p.M = p.K;
+    p.ncols = p.R * p.S * p.C;
+    p.npq = (int64_t)p.N * p.P * p.Q;
+    p.kdim = 0; p.kpad = 0; p.tap_mode = 1;
     const int64_t nkb = (p.npq + BK - 1) / BK;
     if (nkb > INT_MAX) return IQ_OK;
-    const int nsplit = split(nkb);
+    const int bn = pick_bn(p.ncols);
+    const int64_t tiles = ((p.M + BM - 1) / BM) * ((p.ncols + bn - 1) / bn);
+    int64_t kbs;
+    nsplit = choose_split(nkb, tiles, &kbs);
+    p.nkb_total = (int)nkb;
+    p.kb_per_split = (int)kbs;
     CUtensorMap dummy;
     memset(&dummy, 0, sizeof(dummy));
     iq_status r = launch(dummy, p, nsplit, e, x, nullptr, G, nullptr, nullptr, nullptr, err, st);
