@@ -1757,6 +1757,55 @@ __global__ void k_split_sum(const int32_t* __restrict__ part, int ns, int64_t to
     }
 }
 
+// int8 codes [npix][K] -> fp16 carriers [npix][Kp], Kp = K rounded up to 8 (zeros beyond K),
+// 8 codes per thread
+__global__ void k_codes_to_f16_pad(const int8_t* __restrict__ x, __half* __restrict__ xf,
+                                   int64_t npix, int K, int Kp) {
+    const int kg = Kp / 8;
+    const int64_t total = npix * kg;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+        const int64_t pix = i / kg;
+        const int c0 = (int)(i - pix * kg) * 8;
+        uint32_t b[2] = {0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 8; j++)
+            if (c0 + j < K) b[j >> 2] |= ((uint32_t)(uint8_t)x[pix * K + c0 + j]) << (8 * (j & 3));
+        uint32_t o[4];
+        tc::i8x4_to_f16x4(b[0], o[0], o[1]);
+        tc::i8x4_to_f16x4(b[1], o[2], o[3]);
+        *reinterpret_cast<uint4*>(xf + pix * Kp + c0) = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
+// the im2col of a forward problem with few channels (C % 4 == 0) as fp16 [N P Q][kpad]:
+// column j = (r S + s) C + c (the widened weights' order), zeros for padding and
+// j >= R S C.  Block (output row pp, image n); a thread writes 4 columns (one tap, 4
+// channels: one 4-byte load, one 8-byte store) of one output pixel.
+__global__ void k_im2col_f16(const int8_t* __restrict__ x, TcP p, __half* __restrict__ A) {
+    const int g4 = p.kpad / 4;
+    const int pp = blockIdx.y, n = blockIdx.z;
+    const int per_row = p.Q * g4;
+    for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < per_row;
+         idx += gridDim.x * blockDim.x) {
+        const int qq = idx / g4, g = idx - (idx / g4) * g4;
+        const int j = 4 * g;
+        uint32_t v = 0;
+        if (j < p.kdim) {
+            const int tap = j / p.C, c = j - (j / p.C) * p.C;
+            const int r = tap / p.S, sx = tap - (tap / p.S) * p.S;
+            const int hh = pp * p.sh + r * p.dh - p.ph, ww = qq * p.sw + sx * p.dw - p.pw;
+            if (hh >= 0 && hh < p.H && ww >= 0 && ww < p.W)
+                v = __ldg(reinterpret_cast<const uint32_t*>(
+                    x + (((int64_t)n * p.H + hh) * p.W + ww) * p.cstride + p.cofs + c));
+        }
+        uint32_t o0, o1;
+        tc::i8x4_to_f16x4(v, o0, o1);
+        const int64_t m = ((int64_t)n * p.P + pp) * p.Q + qq;
+        *reinterpret_cast<uint2*>(A + m * p.kpad + j) = make_uint2(o0, o1);
+    }
+}
+
 // int8 codes [npix][cstride] -> exact fp16 carriers, 16 codes per thread
 __global__ void k_codes_to_f16(const int8_t* __restrict__ x, __half* __restrict__ xf, int64_t n16) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -2356,11 +2405,21 @@ constexpr int MAX_KB_INT32 = 133120 / 64;   // 2080 k-blocks: 133120 * 127^2 < 2
 // fp16 weights, the error word, then the fp16 carriers of the input
 static size_t acts16_offset(size_t wbytes) { return (wbytes + 256 + 255) / 256 * 256; }
 
+// inputs with few channels (C % 64 != 0, R S C <= 512) go through an fp16 im2col
+constexpr int IM2COL_MAX_K = 512;
+
 size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d) {
     int64_t kdim = (int64_t)d->r * d->s * (d->c / d->groups);
     int64_t kpad = (kdim + 63) / 64 * 64;
     const size_t wb = (size_t)(d->k * kpad * 2);
-    return acts16_offset(wb) + (size_t)d->n * d->h * d->w * d->c * 2 + 512;
+    size_t xb = (size_t)d->n * d->h * d->w * d->c * 2;
+    if (d->c % 64 != 0 && kpad <= IM2COL_MAX_K) {
+        const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+        const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+        const size_t ib = (size_t)d->n * P * Q * kpad * 2;
+        if (ib > xb) xb = ib;
+    }
+    return acts16_offset(wb) + xb + 512;
 }
 
 bool conv_fwd_tc_supported(const iq_conv_desc* d) {
@@ -2398,7 +2457,24 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     if (r != IQ_OK) return r;
     __half* xf = reinterpret_cast<__half*>(wsb + acts16_offset((size_t)p.K * p.kpad * 2));
     bool used = false;
-    if ((p.N * (int64_t)p.H * p.W * p.cstride) % 16 == 0) {
+    if (!p.tap_mode && p.kpad <= IM2COL_MAX_K && p.C % 4 == 0 && p.cstride % 4 == 0 &&
+        p.cofs % 4 == 0 && !tma16_disabled() && p.N <= 65535 && p.P <= 65535) {
+        // few input channels: the fp16 im2col, then a 1x1 problem over kpad channels
+        TcP q = p;
+        q.H = p.P; q.W = p.Q; q.C = p.kpad; q.cstride = p.kpad; q.cofs = 0;
+        q.R = q.S = 1; q.sh = q.sw = 1; q.ph = q.pw = 0; q.dh = q.dw = 1;
+        q.kdim = p.kpad; q.tap_mode = 1;
+        TmaTile tt;
+        if (tma16_ok(q, &tt)) {
+            const int per_row = p.Q * (p.kpad / 4);
+            dim3 gi((unsigned)((per_row + kThreads - 1) / kThreads), (unsigned)p.P, (unsigned)p.N);
+            k_im2col_f16<<<gi, kThreads, 0, st>>>(x, p, xf);
+            IQ_LAUNCH_CHECK();
+            r = try_launch_t(map, q, nullptr, xf, false, acc, nullptr, s1, hi, lo, err, st, &used);
+            if (r != IQ_OK) return r;
+        }
+    }
+    if (!used && (p.N * (int64_t)p.H * p.W * p.cstride) % 16 == 0) {
         r = try_launch_t(map, p, x, xf, true, acc, nullptr, s1, hi, lo, err, st, &used);
         if (r != IQ_OK) return r;
     }
@@ -2532,8 +2608,8 @@ bool wgrad_tma_plan(const iq_conv_desc* d, TcP* p, TmaTile* t, int* nsplit) {
     p->ncols = p->R * p->S * p->C;
     p->npq = (int64_t)p->N * p->P * p->Q;
     p->kdim = 0; p->kpad = 0; p->tap_mode = 1;
-    if (d->groups != 1 || p->C % 64 || p->K % 8 || p->sh > 2 || p->sw > 2) return false;
-    if ((p->npq * p->K) % 16 || ((int64_t)p->N * p->H * p->W * p->C) % 16) return false;
+    if (d->groups != 1 || p->C % 64 || p->sh > 2 || p->sw > 2) return false;
+    if (((int64_t)p->N * p->H * p->W * p->C) % 16) return false;
     if (!wgrad_rect(*p, t)) return false;
     const int64_t nkb = (int64_t)p->N * t->PT * t->QT;
     if (nkb > INT_MAX) return false;
@@ -2553,7 +2629,7 @@ bool wgrad_tma_plan(const iq_conv_desc* d, TcP* p, TmaTile* t, int* nsplit) {
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d) {
     const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
     const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
-    const size_t eb = ((size_t)d->n * P * Q * d->k * 2 + 255) / 256 * 256;
+    const size_t eb = ((size_t)d->n * P * Q * ((d->k + 7) / 8 * 8) * 2 + 255) / 256 * 256;
     const size_t xb = ((size_t)d->n * d->h * d->w * d->c * 2 + 255) / 256 * 256;
     size_t parts = 0;
     TcP p;
@@ -2611,7 +2687,7 @@ bool conv_wgrad_tc_supported(const iq_conv_desc* d) {
 iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
                         void* ws, cudaStream_t st, bool* done) {
     *done = false;
-    if (!conv_wgrad_tc_supported(d) || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
+    if (tc_env_disabled() || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     int* err = reinterpret_cast<int*>(wsb);
     IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
@@ -2621,19 +2697,25 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
     if (!tma16_disabled() && get_encode() && wgrad_tma_plan(d, &p, &t, &nsplit)) {
         // k-blocks: the pixel rectangles of every image; each split writes its own int32
         // partial sums, added into G afterwards
-        const int64_t ne = p.npq * p.K, nx = (int64_t)p.N * p.H * p.W * p.C;
+        const int Kp = (p.K + 7) / 8 * 8;     // fp16 error rows padded to 16 bytes
+        const int64_t ne = p.npq * Kp, nx = (int64_t)p.N * p.H * p.W * p.C;
         const size_t eb = ((size_t)ne * 2 + 255) / 256 * 256;
         const size_t xb = ((size_t)nx * 2 + 255) / 256 * 256;
         __half* ef = reinterpret_cast<__half*>(wsb + 256);
         __half* xf = reinterpret_cast<__half*>(wsb + 256 + eb);
         int32_t* part = reinterpret_cast<int32_t*>(wsb + 256 + eb + xb);
         p.out = OUT_PART32;
-        k_codes_to_f16<<<grid_for(ne / 16), kThreads, 0, st>>>(e, ef, ne / 16);
+        if (Kp == p.K && ne % 16 == 0) {
+            k_codes_to_f16<<<grid_for(ne / 16), kThreads, 0, st>>>(e, ef, ne / 16);
+        } else {
+            k_codes_to_f16_pad<<<grid_for(p.npq * (Kp / 8)), kThreads, 0, st>>>(e, ef, p.npq,
+                                                                              p.K, Kp);
+        }
         IQ_LAUNCH_CHECK();
         k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
         IQ_LAUNCH_CHECK();
         CUtensorMap emap, xmap;
-        iq_status r = encode_acts16(ef, p.N, p.P, p.Q, p.K, t, 1, 1, &emap);
+        iq_status r = encode_acts16(ef, p.N, p.P, p.Q, Kp, t, 1, 1, &emap);
         if (r == IQ_OK) r = encode_acts16(xf, p.N, p.H, p.W, p.C, t, p.sh, p.sw, &xmap);
         if (r != IQ_OK) return r;
         switch (pick_bn(p.ncols)) {
@@ -2648,6 +2730,7 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         *done = true;
         return IQ_OK;
     }
+    if (!conv_wgrad_tc_supported(d)) return IQ_OK;
     fill_geom(p, d);
     p.mode = MODE_WGRAD;
     p.out = OUT_ATOMIC64;

@@ -38,6 +38,43 @@ __global__ void k_maxpool_fwd(const int8_t* __restrict__ x, int n, int h, int w,
     }
 }
 
+// four channels per thread (c % 4 == 0): block (image b, output row i, a slice of the
+// row's Q x c/4 channel groups); 4-byte loads and stores, no 64-bit divisions
+__global__ void k_maxpool_fwd4(const int8_t* __restrict__ x, int h, int w, int c, int k, int s,
+                               int p, int P, int Q, int8_t* __restrict__ y,
+                               uint8_t* __restrict__ arg) {
+    const int c4 = c >> 2;
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= Q * c4) return;
+    const int i = blockIdx.y, b = blockIdx.z;
+    const int j = idx / c4, cg = idx - j * c4;
+    int best[4] = {-1000, -1000, -1000, -1000}, bi[4] = {255, 255, 255, 255};
+    for (int r = 0; r < k; r++) {
+        const int hh = i * s + r - p;
+        if (hh < 0 || hh >= h) continue;
+        const int8_t* row = x + (((int64_t)b * h + hh) * w) * c + 4 * cg;
+        for (int q = 0; q < k; q++) {
+            const int ww = j * s + q - p;
+            if (ww < 0 || ww >= w) continue;
+            const int v = __ldg(reinterpret_cast<const int*>(row + (int64_t)ww * c));
+#pragma unroll
+            for (int t = 0; t < 4; t++) {
+                const int vt = (int)(int8_t)((v >> (8 * t)) & 0xff);
+                if (vt > best[t]) { best[t] = vt; bi[t] = r * k + q; }
+            }
+        }
+    }
+    uint32_t yo = 0, ao = 0;
+#pragma unroll
+    for (int t = 0; t < 4; t++) {
+        yo |= ((uint32_t)(bi[t] == 255 ? 0 : best[t]) & 0xffu) << (8 * t);
+        ao |= ((uint32_t)bi[t] & 0xffu) << (8 * t);
+    }
+    const int64_t o = (((int64_t)b * P + i) * Q + j) * c + 4 * cg;
+    *reinterpret_cast<uint32_t*>(y + o) = yo;
+    *reinterpret_cast<uint32_t*>(arg + o) = ao;
+}
+
 // gather form of the backward: input position (hh, ww) sums the errors of the
 // windows whose first maximum it is (no atomics, deterministic)
 __global__ void k_maxpool_bwd(const int8_t* __restrict__ e, const uint8_t* __restrict__ arg,
@@ -613,6 +650,14 @@ extern "C" iq_status iq_maxpool_fwd(const int8_t* x, int32_t n, int32_t h, int32
         return IQ_ERR_INVALID_ARG;
     int P = (h + 2 * p - k) / s + 1, Q = (w + 2 * p - k) / s + 1;
     int64_t total = (int64_t)n * P * Q * c;
+    if (c % 4 == 0 && (((uintptr_t)x | (uintptr_t)y | (uintptr_t)arg) & 3) == 0 && n <= 65535 &&
+        P <= 65535) {
+        dim3 grid((unsigned)((Q * (c / 4) + kThreads - 1) / kThreads), (unsigned)P, (unsigned)n);
+        k_maxpool_fwd4<<<grid, kThreads, 0, (cudaStream_t)stream>>>(x, h, w, c, k, s, p, P, Q, y,
+                                                                   arg);
+        IQ_LAUNCH_CHECK();
+        return IQ_OK;
+    }
     k_maxpool_fwd<<<grid_for(total), kThreads, 0, (cudaStream_t)stream>>>(x, n, h, w, c, k, s, p,
                                                                           P, Q, y, arg);
     IQ_LAUNCH_CHECK();

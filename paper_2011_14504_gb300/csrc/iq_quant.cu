@@ -139,13 +139,20 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
     const RqParams p = *prm;
     const int64_t lim = qmax(k);
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
-        int4 v = q[i];
-        uint32_t o = ((uint32_t)sq_code(v.x, p, k, relu, lim) & 0xffu) |
-                     (((uint32_t)sq_code(v.y, p, k, relu, lim) & 0xffu) << 8) |
-                     (((uint32_t)sq_code(v.z, p, k, relu, lim) & 0xffu) << 16) |
-                     (((uint32_t)sq_code(v.w, p, k, relu, lim) & 0xffu) << 24);
-        out[i] = o;
+    // two 16-byte loads in flight per thread
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += 2 * stride) {
+        const int64_t i2 = i + stride;
+        const int4 v = __ldg(q + i);
+        const int4 v2 = i2 < n4 ? __ldg(q + i2) : make_int4(0, 0, 0, 0);
+        out[i] = ((uint32_t)sq_code(v.x, p, k, relu, lim) & 0xffu) |
+                 (((uint32_t)sq_code(v.y, p, k, relu, lim) & 0xffu) << 8) |
+                 (((uint32_t)sq_code(v.z, p, k, relu, lim) & 0xffu) << 16) |
+                 (((uint32_t)sq_code(v.w, p, k, relu, lim) & 0xffu) << 24);
+        if (i2 < n4)
+            out[i2] = ((uint32_t)sq_code(v2.x, p, k, relu, lim) & 0xffu) |
+                      (((uint32_t)sq_code(v2.y, p, k, relu, lim) & 0xffu) << 8) |
+                      (((uint32_t)sq_code(v2.z, p, k, relu, lim) & 0xffu) << 16) |
+                      (((uint32_t)sq_code(v2.w, p, k, relu, lim) & 0xffu) << 24);
     }
 }
 

@@ -309,6 +309,10 @@ TC_CASES = [
     (3, 9, 10, 64, 80, 1, 1, 1, 0, 1),      # 1x1, ragged
     (1, 33, 33, 256, 64, 3, 3, 2, 1, 1),    # stride 2 (data gradient on CUDA cores)
     (4, 40, 40, 64, 64, 3, 3, 1, 1, 1),     # weight gradient split over 100 k-blocks
+    (2, 24, 20, 64, 150, 1, 1, 1, 0, 1),    # 150 output channels (padded error rows)
+    (2, 31, 29, 4, 64, 3, 3, 1, 1, 1),      # 4 input channels (fp16 im2col forward)
+    (1, 35, 35, 4, 64, 7, 7, 2, 3, 1),      # stem: 7x7 stride 2 over 4 channels
+    (2, 17, 15, 128, 96, 3, 3, 1, 2, 2),    # dilation 2, rectangle tiles with waste
 ]
 
 
@@ -369,10 +373,10 @@ def test_conv_fwd_adversarial_full_scale(sign):
 
 # ----------------------------------------------------------------- network glue
 
-@pytest.mark.parametrize("k,s,p", [(2, 2, 0), (3, 2, 1)])
-def test_maxpool(k, s, p):
+@pytest.mark.parametrize("k,s,p,c", [(2, 2, 0, 24), (3, 2, 1, 24), (3, 2, 1, 6)])
+def test_maxpool(k, s, p, c):
     g = S.rng(k * 10 + s)
-    x = S.int8_uniform(g, (2, 37, 30, 24), -9, 9)
+    x = S.int8_uniform(g, (2, 37, 30, c), -9, 9)
     y_o, a_o = O.maxpool_fwd(x, k, s, p)
     y = torch.empty(y_o.shape, dtype=torch.int8, device=DEV)
     a = torch.empty(y_o.shape, dtype=torch.uint8, device=DEV)
