@@ -4,20 +4,27 @@
 // the codes travel as fp16 "carriers": every int8 code is exact in fp16, every product
 // |a b| <= 127^2 is exact, and fp32 accumulation of at most 1024 such products stays
 // below 2^24 and is therefore exact.  The K loop is cut into chunks of 16 k-blocks
-// (1024 products); the epilogue folds every fp32 chunk into an int32 running sum kept in
-// TMEM, so the result is the exact integer convolution.
+// (1024 products); the epilogue folds every fp32 chunk into an int32 running sum (in TMEM
+// or in registers), so the result is the exact integer convolution.
 //
-// One kernel, two operand layouts:
+// GEMM views of the three convolutions:
 //   FWD   (forward, and the stride-1 data gradient as a forward pass over the errors with
 //          flipped, transposed weights): D[M x N] = A[M x K] B[N x K]^T, M = output pixels,
-//          N = output channels, K = taps x channels.  A is gathered per output pixel
-//          (K-major), B (fp16 weights, widened once per call) arrives by TMA.
+//          N = output channels, K = taps x channels, both operands K-major.
 //   WGRAD (weight gradient): D[Kout x RSC] = sum over pixels of E^T X, both operands
-//          MN-major (channels contiguous), gathered per pixel.
-// Tile 128 x 256 x 64, 4 shared-memory stages.  Warps 0-3 gather / widen / store the
-// operands, warp 8 allocates TMEM and issues tcgen05.mma (M=128, N=256, K=16), warps 4-7
-// fold the chunks and run the epilogue: either int32 stores plus per-channel sum / max /
-// min, or int64 atomic adds (weight gradients and split reductions).
+//          MN-major (channels contiguous), the pixel sum split across CTAs.
+// Three persistent kernels (one CTA per SM, tiles 128 x BN x 64, BN in {64, 128, 256}):
+//   k_conv_tct  all operands by TMA from fp16 carrier copies (a pre-pass widens the codes
+//               once per call): 4-D boxes of the input per tap for FWD, error rectangles
+//               and im2col boxes for WGRAD.  The default whenever the shape allows it.
+//   k_conv_tcq  FWD with whole 64-channel k-blocks when no TMA tile rectangle fits well:
+//               producer threads copy int8 rows with cp.async and widen them in shared memory.
+//   k_conv_tcp  everything else (channel counts that are multiples of 8 or 16): producer
+//               warps gather int8 rows into registers and widen them on the way to shared
+//               memory.
+// In all three one elected thread issues tcgen05.mma (M=128, K=16) into TMEM and
+// epilogue warps fold the fp32 chunks into int32 and write either int32 outputs plus
+// per-channel sum / max / min (FWD), int32 split partials or int64 atomic adds (WGRAD).
 // Every mbarrier wait is bounded (about one second); on expiry the CTA records an error
 // word, drains what it issued and returns, and later CTAs of the launch exit at once.
 #include "iq_conv_tc.cuh"
@@ -36,7 +43,6 @@ constexpr int BK = 64;                    // fp16 elements per k-block = 128 byt
 constexpr int STAGES = 4;
 constexpr int CHUNK_KB = 16;              // 1024 products per fp32 chunk
 constexpr int A_BYTES = BM * 128;         // 16 KB
-constexpr int THREADS = 288;
 
 // Per N-tile width: B tile bytes, stage bytes, TMEM columns (fp32 chunk + int32 running
 // sum), dynamic shared memory, epilogue tile pitch.
@@ -45,9 +51,7 @@ struct Cfg {
     static constexpr int B_BYTES = BN * 128;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int TMEM_COLS = 2 * BN;
-    static constexpr int TILE_LD = BN + 1;
     static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
-    static_assert(BM * TILE_LD * 4 <= STAGES * STAGE_BYTES, "epilogue tile fits");
 };
 
 enum { MODE_FWD = 0, MODE_WGRAD = 1 };
@@ -67,23 +71,6 @@ struct TcP {
     int kb_per_split;
     int64_t npq;     // WGRAD: reduction length N*P*Q
 };
-
-struct Bars {
-    uint64_t full_a[STAGES];
-    uint64_t full_b[STAGES];
-    uint64_t empty[STAGES];
-    uint64_t accf;
-    uint64_t acce;
-    uint64_t done;
-    uint32_t tmem_base;
-    int abort;
-    int never;
-};
-
-__device__ __forceinline__ void record_abort(Bars* b, int* err, int code) {
-    b->abort = 1;
-    if (err) atomicExch(err, code);
-}
 
 // ---------------------------------------------------------------- FWD gather (K-major A)
 
@@ -247,278 +234,6 @@ __device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t saddr) {
 __host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool mn_major) {
     return (1u << 4) | ((mn_major ? 1u : 0u) << 15) | ((mn_major ? 1u : 0u) << 16) |
            ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
-
-// Fold one fp32 chunk (TMEM columns tD..tD+BN) into the int32 running sum (tR..): two
-// 32-column blocks per TMEM round trip.  On the last chunk the sums go to the thread's
-// row of the shared-memory tile instead.
-template <int BN>
-__device__ __forceinline__ void fold_chunk(uint32_t tD, uint32_t tR, bool has_prev, bool lastc,
-                                           int* tile_row) {
-#pragma unroll 1
-    for (int cb = 0; cb < BN / 32; cb += 2) {
-        uint32_t d0[32], d1[32], r0[32], r1[32];
-        tc::tmem_ld_32x32b_x32(tD + cb * 32, d0);
-        tc::tmem_ld_32x32b_x32(tD + cb * 32 + 32, d1);
-        if (has_prev) {
-            tc::tmem_ld_32x32b_x32(tR + cb * 32, r0);
-            tc::tmem_ld_32x32b_x32(tR + cb * 32 + 32, r1);
-        }
-        tc::tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 32; i++) {
-            r0[i] = (uint32_t)((has_prev ? (int)r0[i] : 0) + __float2int_rn(__uint_as_float(d0[i])));
-            r1[i] = (uint32_t)((has_prev ? (int)r1[i] : 0) + __float2int_rn(__uint_as_float(d1[i])));
-        }
-        if (!lastc) {
-            tc::tmem_st_32x32b_x32(tR + cb * 32, r0);
-            tc::tmem_st_32x32b_x32(tR + cb * 32 + 32, r1);
-        } else {
-#pragma unroll
-            for (int i = 0; i < 32; i++) {
-                tile_row[cb * 32 + i] = (int)r0[i];
-                tile_row[cb * 32 + 32 + i] = (int)r1[i];
-            }
-        }
-    }
-    if (!lastc) tc::tmem_st_wait();
-}
-
-// ---------------------------------------------------------------- the kernel
-
-template <int BN>
-__global__ void __launch_bounds__(THREADS, 1)
-    k_conv_tc(const __grid_constant__ CUtensorMap wmap, TcP p, const int8_t* __restrict__ xa,
-              const int8_t* __restrict__ xb, int32_t* __restrict__ out32,
-              long long* __restrict__ out64, unsigned long long* __restrict__ s1,
-              int* __restrict__ hi_c, int* __restrict__ lo_c, int* __restrict__ err) {
-    constexpr int STAGE_BYTES = Cfg<BN>::STAGE_BYTES;
-    constexpr int B_BYTES = Cfg<BN>::B_BYTES;
-    constexpr int TMEM_COLS = Cfg<BN>::TMEM_COLS;
-    constexpr int TILE_LD = Cfg<BN>::TILE_LD;
-    extern __shared__ __align__(1024) uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    Bars* bars = reinterpret_cast<Bars*>(smem + STAGES * STAGE_BYTES);
-
-    const int tid = threadIdx.x;
-    const int warp = tid >> 5, lane = tid & 31;
-    // a CTA that timed out earlier in this launch makes the rest leave at once; one
-    // thread reads the word so that the whole CTA takes the same branch
-    if (__syncthreads_or(tid == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
-    const int64_t m0 = (int64_t)blockIdx.x * BM;
-    const int n0 = blockIdx.y * BN;
-    const int kb0 = blockIdx.z * p.kb_per_split;
-    int nkb = p.nkb_total - kb0;
-    if (nkb > p.kb_per_split) nkb = p.kb_per_split;
-    if (nkb <= 0) return;
-    const int nchunks = (nkb + CHUNK_KB - 1) / CHUNK_KB;
-    const bool wg = p.mode == MODE_WGRAD;
-
-    if (tid == 0) {
-        for (int s = 0; s < STAGES; s++) {
-            tc::mbar_init(&bars->full_a[s], 128);
-            tc::mbar_init(&bars->full_b[s], 1);
-            tc::mbar_init(&bars->empty[s], 1);
-        }
-        tc::mbar_init(&bars->accf, 1);
-        tc::mbar_init(&bars->acce, 128);
-        tc::mbar_init(&bars->done, 1);
-        bars->abort = 0;
-        bars->never = 0;
-        tc::mbar_fence_init();
-        if (!wg) tc::tma_prefetch_desc(&wmap);
-    }
-    if (warp == 8) {
-        tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
-        tc::tmem_relinquish();
-    }
-    tc::tc_fence_before();
-    __syncthreads();
-    tc::tc_fence_after();
-    const uint32_t tmem = bars->tmem_base;
-    volatile int* abort_flag = &bars->abort;
-
-    if (warp < 4) {
-        // ================================================ producers
-        int issued_b = 0;
-        if (!wg) {
-            const int row = tid;
-            const int64_t m = m0 + row;
-            const bool valid = m < p.M;
-            int n = 0, pp = 0, qq = 0;
-            if (valid) {
-                const int64_t pq = (int64_t)p.P * p.Q;
-                n = (int)(m / pq);
-                const int64_t rem = m - (int64_t)n * pq;
-                pp = (int)(rem / p.Q);
-                qq = (int)(rem - (int64_t)pp * p.Q);
-            }
-            uint32_t c0[16], c1[16], c2[16];
-            gather_fwd(p, xa, valid, n, pp, qq, kb0, c0);
-            gather_fwd(p, xa, valid, n, pp, qq, kb0 + 1, c1);
-            for (int kb = 0; kb < nkb; kb++) {
-                const int s = kb % STAGES;
-                const uint32_t it = (uint32_t)(kb / STAGES);
-                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
-                    record_abort(bars, err, 1);
-                    break;
-                }
-                uint8_t* a_tile = smem + s * STAGE_BYTES;
-                if (tid == 0) {
-                    tc::mbar_expect_tx(&bars->full_b[s], B_BYTES);
-                    tc::tma_load_2d(a_tile + A_BYTES, &wmap, &bars->full_b[s], (kb0 + kb) * BK, n0);
-                    tc::mbar_arrive(&bars->full_b[s]);
-                    issued_b = kb + 1;
-                }
-                if (kb + 2 < nkb) gather_fwd(p, xa, valid, n, pp, qq, kb0 + kb + 2, c2);
-                store_kmajor_row(a_tile, row, c0);
-                tc::fence_proxy_async_smem();
-                tc::mbar_arrive(&bars->full_a[s]);
-#pragma unroll
-                for (int i = 0; i < 16; i++) { c0[i] = c1[i]; c1[i] = c2[i]; }
-            }
-        } else {
-            const int j = tid >> 1, h = tid & 1;
-            uint4 a0[4], b0[BN / 32], a1[4], b1[BN / 32];
-            WgRow r0 = wg_row(p, (int64_t)kb0 * BK + j);
-            gather_wgrad<BN>(p, xa, xb, m0, n0, r0, h, a0, b0);
-            for (int kb = 0; kb < nkb; kb++) {
-                const int s = kb % STAGES;
-                const uint32_t it = (uint32_t)(kb / STAGES);
-                if (kb + 1 < nkb) {
-                    WgRow r1 = wg_row(p, (int64_t)(kb0 + kb + 1) * BK + j);
-                    gather_wgrad<BN>(p, xa, xb, m0, n0, r1, h, a1, b1);
-                }
-                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
-                    record_abort(bars, err, 1);
-                    break;
-                }
-                uint8_t* a_tile = smem + s * STAGE_BYTES;
-                uint8_t* b_tile = a_tile + A_BYTES;
-#pragma unroll
-                for (int i = 0; i < 4; i++)
-                    store_mnmajor_chunk(a_tile, j, 4 * h + i, a0[i].x, a0[i].y, a0[i].z, a0[i].w);
-#pragma unroll
-                for (int i = 0; i < BN / 32; i++)
-                    store_mnmajor_chunk(b_tile, j, h * (BN / 32) + i, b0[i].x, b0[i].y, b0[i].z,
-                                        b0[i].w);
-                tc::fence_proxy_async_smem();
-                tc::mbar_arrive(&bars->full_a[s]);
-                if (tid == 0) tc::mbar_arrive(&bars->full_b[s]);
-#pragma unroll
-                for (int i = 0; i < 4; i++) a0[i] = a1[i];
-#pragma unroll
-                for (int i = 0; i < BN / 32; i++) b0[i] = b1[i];
-            }
-        }
-        if (!wg && tid == 0 && *abort_flag) {
-            for (int kb = (issued_b > STAGES ? issued_b - STAGES : 0); kb < issued_b; kb++)
-                tc::mbar_wait(&bars->full_b[kb % STAGES], (uint32_t)(kb / STAGES) & 1,
-                              &bars->never);
-        }
-    } else if (warp == 8) {
-        // ================================================ MMA issuer
-        if (lane == 0) {
-            const uint32_t idesc = idesc_f16(BM, BN, wg);
-            bool ok = true;
-            for (int kb = 0; kb < nkb && ok; kb++) {
-                const int s = kb % STAGES;
-                const uint32_t it = (uint32_t)(kb / STAGES);
-                const int chunk = kb / CHUNK_KB;
-                const bool first = (kb % CHUNK_KB) == 0;
-                const bool last = ((kb % CHUNK_KB) == CHUNK_KB - 1) || kb == nkb - 1;
-                // the fp32 buffer is free once the epilogue folded the previous chunk
-                if (first && chunk > 0 &&
-                    !tc::mbar_wait(&bars->acce, (uint32_t)(chunk - 1) & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                if (!tc::mbar_wait(&bars->full_b[s], it & 1, abort_flag) ||
-                    !tc::mbar_wait(&bars->full_a[s], it & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                tc::tc_fence_after();
-                const uint32_t a_addr = tc::smem_u32(smem + s * STAGE_BYTES);
-                const uint32_t b_addr = a_addr + A_BYTES;
-#pragma unroll
-                for (int k = 0; k < BK / 16; k++) {
-                    uint64_t ad, bd;
-                    if (wg) {
-                        ad = sdesc_mnmajor_sw128(a_addr + 2 * 1024 * k);
-                        bd = sdesc_mnmajor_sw128(b_addr + 2 * 1024 * k);
-                    } else {
-                        ad = tc::sdesc_kmajor_sw128(a_addr + 32 * k);
-                        bd = tc::sdesc_kmajor_sw128(b_addr + 32 * k);
-                    }
-                    tc::umma_f16(tmem, ad, bd, idesc, (first && k == 0) ? 0u : 1u);
-                }
-                tc::umma_commit(&bars->empty[s]);
-                if (last) tc::umma_commit(&bars->accf);
-            }
-            if (!ok) record_abort(bars, err, 2);
-            tc::umma_commit(&bars->done);
-            tc::mbar_wait(&bars->done, 0, &bars->never);
-        }
-        __syncwarp();
-    } else {
-        // ================================================ epilogue (warps 4..7)
-        const int row = tid - 128;
-        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-        const uint32_t tD = tmem + lane_base;            // fp32 chunk, columns [0, 256)
-        const uint32_t tR = tmem + lane_base + BN;       // int32 running sum, [256, 512)
-        int* tile = reinterpret_cast<int*>(smem);
-        bool ok = true;
-        for (int c = 0; c < nchunks; c++) {
-            if (!tc::mbar_wait(&bars->accf, (uint32_t)c & 1, abort_flag)) {
-                ok = false;
-                record_abort(bars, err, 3);
-                break;
-            }
-            tc::tc_fence_after();
-            // after the last chunk every MMA has completed (and with it every operand
-            // write and read), so the stage buffers are free for the epilogue tile
-            const bool lastc = c == nchunks - 1;
-            fold_chunk<BN>(tD, tR, c > 0, lastc, tile + row * TILE_LD);
-            tc::tc_fence_before();
-            tc::mbar_arrive(&bars->acce);
-        }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (ok && !*abort_flag) {
-            const int rows = (int)((p.M - m0) < BM ? (p.M - m0) : BM);
-            for (int col = row; col < BN; col += 128) {
-                const int gcol = n0 + col;
-                if (gcol >= p.ncols) continue;
-                if (p.out == OUT_STATS) {
-                    long long sum = 0;
-                    int h = INT_MIN, l = INT_MAX;
-                    for (int i = 0; i < rows; i++) {
-                        int v = tile[i * TILE_LD + col];
-                        sum += v; h = max(h, v); l = min(l, v);
-                        out32[(m0 + i) * p.ncols + gcol] = v;
-                    }
-                    atomicAdd(&s1[gcol], (unsigned long long)sum);
-                    atomicMax(&hi_c[gcol], h);
-                    atomicMin(&lo_c[gcol], l);
-                } else {
-                    for (int i = 0; i < rows; i++) {
-                        int v = tile[i * TILE_LD + col];
-                        if (v)
-                            atomicAdd(reinterpret_cast<unsigned long long*>(
-                                          &out64[(m0 + i) * p.ncols + gcol]),
-                                      (unsigned long long)(long long)v);
-                    }
-                }
-            }
-        }
-    }
-    tc::tc_fence_before();
-    __syncthreads();
-    if (warp == 8) {
-        tc::tc_fence_after();
-        tc::tmem_dealloc(tmem, TMEM_COLS);
-    }
 }
 
 // ---------------------------------------------------------------- persistent kernel
@@ -1822,268 +1537,10 @@ __global__ void k_codes_to_f16(const int8_t* __restrict__ x, __half* __restrict_
     }
 }
 
-// ---------------------------------------------------------------- TMA-fed forward
-// Stride-1 convolutions with C % 64 == 0: the M tile is a BH x BW rectangle of output
-// pixels of one image (BH * BW = 128).  For k-block (tap r,s; channels c0..c0+63) the A
-// rows are exactly the input box [c0, c0+64) x [q0 + s dw - pw, +BW) x [p0 + r dh - ph, +BH)
-// of image n, so one TMA load (zero fill outside the image = the padding, 64-byte
-// swizzle) brings them into a staging slot; converter warps widen it to fp16 in the
-// K-major 128-byte-swizzled UMMA layout.  Warp 9 issues the TMA loads (activations and
-// weights) ahead of the MMA warp; warps 4-7 run the epilogue as in k_conv_tc.
-
+// Tile rectangle of the TMA-fed kernels: BW x BH output pixels of one image.
 struct TmaTile {
     int BW, BH, PT, QT;
 };
-
-constexpr int STG_BYTES = 8192;     // 128 rows x 64 int8
-constexpr int TMA_THREADS = 320;
-
-struct TmaBars {
-    uint64_t full_a[STAGES];
-    uint64_t full_b[STAGES];
-    uint64_t empty[STAGES];
-    uint64_t stg_full[STAGES];
-    uint64_t stg_empty[STAGES];
-    uint64_t accf;
-    uint64_t acce;
-    uint64_t done;
-    uint32_t tmem_base;
-    int abort;
-    int never;
-};
-
-template <int BN>
-struct TmaCfg {
-    static constexpr int STAGE_BYTES = Cfg<BN>::STAGE_BYTES;
-    static constexpr int SMEM = STAGES * STAGE_BYTES + STAGES * STG_BYTES + 1024 + 512;
-};
-
-template <int BN>
-__global__ void __launch_bounds__(TMA_THREADS, 1)
-    k_conv_tc_tma(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap amap,
-                  TcP p, TmaTile tt, int32_t* __restrict__ out32, long long* __restrict__ out64,
-                  unsigned long long* __restrict__ s1, int* __restrict__ hi_c,
-                  int* __restrict__ lo_c, int* __restrict__ err) {
-    constexpr int STAGE_BYTES = Cfg<BN>::STAGE_BYTES;
-    constexpr int B_BYTES = Cfg<BN>::B_BYTES;
-    constexpr int TMEM_COLS = Cfg<BN>::TMEM_COLS;
-    constexpr int TILE_LD = Cfg<BN>::TILE_LD;
-    extern __shared__ __align__(1024) uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* staging = smem + STAGES * STAGE_BYTES;
-    TmaBars* bars = reinterpret_cast<TmaBars*>(staging + STAGES * STG_BYTES);
-
-    const int tid = threadIdx.x;
-    const int warp = tid >> 5, lane = tid & 31;
-    if (__syncthreads_or(tid == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
-    // tile: image n, output rows p0.., output columns q0..
-    const int qt = blockIdx.x % tt.QT;
-    const int pt = (blockIdx.x / tt.QT) % tt.PT;
-    const int n = blockIdx.x / (tt.QT * tt.PT);
-    const int p0 = pt * tt.BH, q0 = qt * tt.BW;
-    const int n0 = blockIdx.y * BN;
-    const int nkb = p.nkb_total;
-    const int nchunks = (nkb + CHUNK_KB - 1) / CHUNK_KB;
-
-    if (tid == 0) {
-        for (int s = 0; s < STAGES; s++) {
-            tc::mbar_init(&bars->full_a[s], 128);
-            tc::mbar_init(&bars->full_b[s], 1);
-            tc::mbar_init(&bars->empty[s], 1);
-            tc::mbar_init(&bars->stg_full[s], 1);
-            tc::mbar_init(&bars->stg_empty[s], 128);
-        }
-        tc::mbar_init(&bars->accf, 1);
-        tc::mbar_init(&bars->acce, 128);
-        tc::mbar_init(&bars->done, 1);
-        bars->abort = 0;
-        bars->never = 0;
-        tc::mbar_fence_init();
-    }
-    if (warp == 8) {
-        tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
-        tc::tmem_relinquish();
-    }
-    tc::tc_fence_before();
-    __syncthreads();
-    tc::tc_fence_after();
-    const uint32_t tmem = bars->tmem_base;
-    volatile int* abort_flag = &bars->abort;
-
-    if (warp == 9) {
-        // ================================================ TMA issuer
-        if (lane == 0) {
-            tc::tma_prefetch_desc(&amap);
-            tc::tma_prefetch_desc(&wmap);
-            int stg_issued = 0, b_issued = 0;
-            for (int kb = 0; kb < nkb; kb++) {
-                const int s = kb % STAGES;
-                const uint32_t ph = (uint32_t)(kb / STAGES) & 1;
-                if (!tc::mbar_wait(&bars->stg_empty[s], ph ^ 1, abort_flag)) {
-                    bars->abort = 1;
-                    atomicExch(err, 4);
-                    break;
-                }
-                const int kpos = kb * BK;
-                const int tap = kpos / p.C;
-                const int c0 = kpos - tap * p.C;
-                const int r = tap / p.S, ss = tap - r * p.S;
-                tc::mbar_expect_tx(&bars->stg_full[s], STG_BYTES);
-                tc::tma_load_4d(staging + s * STG_BYTES, &amap, &bars->stg_full[s], p.cofs + c0,
-                                q0 + ss * p.dw - p.pw, p0 + r * p.dh - p.ph, n);
-                tc::mbar_arrive(&bars->stg_full[s]);
-                stg_issued = kb + 1;
-                if (!tc::mbar_wait(&bars->empty[s], ph ^ 1, abort_flag)) {
-                    bars->abort = 1;
-                    atomicExch(err, 5);
-                    break;
-                }
-                tc::mbar_expect_tx(&bars->full_b[s], B_BYTES);
-                tc::tma_load_2d(smem + s * STAGE_BYTES + A_BYTES, &wmap, &bars->full_b[s], kb * BK,
-                                n0);
-                tc::mbar_arrive(&bars->full_b[s]);
-                b_issued = kb + 1;
-            }
-            if (*abort_flag) {
-                // let the loads already requested land before the CTA leaves
-                for (int kb = (stg_issued > STAGES ? stg_issued - STAGES : 0); kb < stg_issued; kb++)
-                    tc::mbar_wait(&bars->stg_full[kb % STAGES], (uint32_t)(kb / STAGES) & 1,
-                                  &bars->never);
-                for (int kb = (b_issued > STAGES ? b_issued - STAGES : 0); kb < b_issued; kb++)
-                    tc::mbar_wait(&bars->full_b[kb % STAGES], (uint32_t)(kb / STAGES) & 1,
-                                  &bars->never);
-            }
-        }
-        __syncwarp();
-    } else if (warp < 4) {
-        // ================================================ converters
-        const int row = tid;
-        const int rot = (row >> 1) & 3;          // the 64-byte swizzle of the staging rows
-        for (int kb = 0; kb < nkb; kb++) {
-            const int s = kb % STAGES;
-            const uint32_t ph = (uint32_t)(kb / STAGES) & 1;
-            if (!tc::mbar_wait(&bars->empty[s], ph ^ 1, abort_flag) ||
-                !tc::mbar_wait(&bars->stg_full[s], ph, abort_flag)) {
-                bars->abort = 1;
-                atomicExch(err, 1);
-                break;
-            }
-            const uint8_t* src = staging + s * STG_BYTES + row * 64;
-            uint8_t* dst = smem + s * STAGE_BYTES + row * 128;
-#pragma unroll
-            for (int i = 0; i < 4; i++) {
-                const uint4 v = *reinterpret_cast<const uint4*>(src + ((i ^ rot) << 4));
-                uint32_t o0, o1, o2, o3, o4, o5, o6, o7;
-                tc::i8x4_to_f16x4(v.x, o0, o1);
-                tc::i8x4_to_f16x4(v.y, o2, o3);
-                tc::i8x4_to_f16x4(v.z, o4, o5);
-                tc::i8x4_to_f16x4(v.w, o6, o7);
-                *reinterpret_cast<uint4*>(dst + (((2 * i) ^ (row & 7)) << 4)) =
-                    make_uint4(o0, o1, o2, o3);
-                *reinterpret_cast<uint4*>(dst + (((2 * i + 1) ^ (row & 7)) << 4)) =
-                    make_uint4(o4, o5, o6, o7);
-            }
-            tc::fence_proxy_async_smem();
-            tc::mbar_arrive(&bars->full_a[s]);
-            tc::mbar_arrive(&bars->stg_empty[s]);
-        }
-    } else if (warp == 8) {
-        // ================================================ MMA issuer
-        if (lane == 0) {
-            const uint32_t idesc = idesc_f16(BM, BN, false);
-            bool ok = true;
-            for (int kb = 0; kb < nkb && ok; kb++) {
-                const int s = kb % STAGES;
-                const uint32_t it = (uint32_t)(kb / STAGES);
-                const int chunk = kb / CHUNK_KB;
-                const bool first = (kb % CHUNK_KB) == 0;
-                const bool last = ((kb % CHUNK_KB) == CHUNK_KB - 1) || kb == nkb - 1;
-                if (first && chunk > 0 &&
-                    !tc::mbar_wait(&bars->acce, (uint32_t)(chunk - 1) & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                if (!tc::mbar_wait(&bars->full_b[s], it & 1, abort_flag) ||
-                    !tc::mbar_wait(&bars->full_a[s], it & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                tc::tc_fence_after();
-                const uint32_t a_addr = tc::smem_u32(smem + s * STAGE_BYTES);
-                const uint32_t b_addr = a_addr + A_BYTES;
-#pragma unroll
-                for (int k = 0; k < BK / 16; k++)
-                    tc::umma_f16(tmem, tc::sdesc_kmajor_sw128(a_addr + 32 * k),
-                                 tc::sdesc_kmajor_sw128(b_addr + 32 * k), idesc,
-                                 (first && k == 0) ? 0u : 1u);
-                tc::umma_commit(&bars->empty[s]);
-                if (last) tc::umma_commit(&bars->accf);
-            }
-            if (!ok) {
-                bars->abort = 1;
-                atomicExch(err, 2);
-            }
-            tc::umma_commit(&bars->done);
-            tc::mbar_wait(&bars->done, 0, &bars->never);
-        }
-        __syncwarp();
-    } else {
-        // ================================================ epilogue (warps 4..7)
-        const int row = tid - 128;
-        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-        const uint32_t tD = tmem + lane_base;
-        const uint32_t tR = tmem + lane_base + BN;
-        int* tile = reinterpret_cast<int*>(smem);
-        bool ok = true;
-        for (int c = 0; c < nchunks; c++) {
-            if (!tc::mbar_wait(&bars->accf, (uint32_t)c & 1, abort_flag)) {
-                ok = false;
-                bars->abort = 1;
-                atomicExch(err, 3);
-                break;
-            }
-            tc::tc_fence_after();
-            const bool lastc = c == nchunks - 1;
-            fold_chunk<BN>(tD, tR, c > 0, lastc, tile + row * TILE_LD);
-            tc::tc_fence_before();
-            tc::mbar_arrive(&bars->acce);
-        }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (ok && !*abort_flag) {
-            for (int col = row; col < BN; col += 128) {
-                const int gcol = n0 + col;
-                if (gcol >= p.ncols) continue;
-                long long sum = 0;
-                int h = INT_MIN, l = INT_MAX;
-                for (int i = 0; i < BM; i++) {
-                    const int pp = p0 + i / tt.BW, qq = q0 + i % tt.BW;
-                    if (pp >= p.P || qq >= p.Q) continue;
-                    const int64_t grow = ((int64_t)n * p.P + pp) * p.Q + qq;
-                    const int v = tile[i * TILE_LD + col];
-                    if (p.out == OUT_STATS) {
-                        sum += v; h = max(h, v); l = min(l, v);
-                        out32[grow * p.ncols + gcol] = v;
-                    } else if (v) {
-                        atomicAdd(reinterpret_cast<unsigned long long*>(&out64[grow * p.ncols + gcol]),
-                                  (unsigned long long)(long long)v);
-                    }
-                }
-                if (p.out == OUT_STATS) {
-                    atomicAdd(&s1[gcol], (unsigned long long)sum);
-                    atomicMax(&hi_c[gcol], h);
-                    atomicMin(&lo_c[gcol], l);
-                }
-            }
-        }
-    }
-    tc::tc_fence_before();
-    __syncthreads();
-    if (warp == 8) {
-        tc::tc_fence_after();
-        tc::tmem_dealloc(tmem, TMEM_COLS);
-    }
-}
 
 // int8 KRSC weights -> fp16 [K][kpad] (zero beyond R*S*C)
 __global__ void k_widen_weights(const int8_t* __restrict__ w, __half* __restrict__ wf, int K,
@@ -2146,20 +1603,6 @@ iq_status encode_weights(const __half* wf, int rows, int kpad, int box_rows, CUt
     return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
 }
 
-template <int BN>
-iq_status launch_bn(const CUtensorMap& map, const TcP& p, int nsplit, const int8_t* xa,
-                    const int8_t* xb, int32_t* out32, long long* out64, unsigned long long* s1,
-                    int* hi, int* lo, int* err, cudaStream_t st) {
-    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       Cfg<BN>::SMEM));
-    dim3 grid((unsigned)((p.M + BM - 1) / BM), (unsigned)((p.ncols + BN - 1) / BN),
-              (unsigned)nsplit);
-    k_conv_tc<BN><<<grid, THREADS, Cfg<BN>::SMEM, st>>>(map, p, xa, xb, out32, out64, s1, hi, lo,
-                                                        err);
-    IQ_LAUNCH_CHECK();
-    return IQ_OK;
-}
-
 // N-tile width for a GEMM with `ncols` columns: the smallest of 64 / 128 / 256 covering it
 int pick_bn(int ncols) { return ncols <= 64 ? 64 : (ncols <= 128 ? 128 : 256); }
 
@@ -2210,33 +1653,21 @@ iq_status launch_q(const CUtensorMap& map, const TcP& p, const int8_t* xa, int32
     return IQ_OK;
 }
 
-bool tc_persistent() {
-    const char* e = getenv("IQ_TC_TILE_PER_CTA");
-    return !(e && e[0] == '1');
-}
-
 iq_status launch(const CUtensorMap& map, const TcP& p, int nsplit, const int8_t* xa,
                  const int8_t* xb, int32_t* out32, long long* out64, unsigned long long* s1,
                  int* hi, int* lo, int* err, cudaStream_t st) {
-    if (tc_persistent() && p.mode == MODE_FWD && nsplit == 1 && p.tap_mode &&
-        p.cstride % 16 == 0 && p.cofs % 16 == 0 && ((uintptr_t)xa & 15) == 0) {
+    if (p.mode == MODE_FWD && nsplit == 1 && p.tap_mode && p.cstride % 16 == 0 &&
+        p.cofs % 16 == 0 && ((uintptr_t)xa & 15) == 0) {
         switch (pick_bn(p.ncols)) {
             case 64: return launch_q<64>(map, p, xa, out32, out64, s1, hi, lo, err, st);
             case 128: return launch_q<128>(map, p, xa, out32, out64, s1, hi, lo, err, st);
             default: return launch_q<256>(map, p, xa, out32, out64, s1, hi, lo, err, st);
         }
     }
-    if (tc_persistent()) {
-        switch (pick_bn(p.ncols)) {
-            case 64: return launch_p<64>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
-            case 128: return launch_p<128>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
-            default: return launch_p<256>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
-        }
-    }
     switch (pick_bn(p.ncols)) {
-        case 64: return launch_bn<64>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
-        case 128: return launch_bn<128>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
-        default: return launch_bn<256>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
+        case 64: return launch_p<64>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
+        case 128: return launch_p<128>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
+        default: return launch_p<256>(map, p, nsplit, xa, xb, out32, out64, s1, hi, lo, err, st);
     }
 }
 
@@ -2254,61 +1685,6 @@ bool pick_tma_tile(int P, int Q, TmaTile* t, double min_util = 0.8) {
         }
     }
     return best >= min_util;
-}
-
-iq_status encode_acts(const int8_t* x, int N, int H, int W, int cstride, const TmaTile& t,
-                      CUtensorMap* map) {
-    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
-    if (!enc) return IQ_ERR_UNSUPPORTED;
-    cuuint64_t gdim[4] = {(cuuint64_t)cstride, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
-    cuuint64_t gstride[3] = {(cuuint64_t)cstride, (cuuint64_t)W * cstride,
-                             (cuuint64_t)H * W * cstride};
-    cuuint32_t box[4] = {64, (cuuint32_t)t.BW, (cuuint32_t)t.BH, 1};
-    cuuint32_t estr[4] = {1, 1, 1, 1};
-    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, (void*)x, gdim, gstride, box, estr,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
-                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
-}
-
-template <int BN>
-iq_status launch_tma_bn(const CUtensorMap& wmap, const CUtensorMap& amap, const TcP& p,
-                        const TmaTile& t, int32_t* out32, long long* out64,
-                        unsigned long long* s1, int* hi, int* lo, int* err, cudaStream_t st) {
-    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tc_tma<BN>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       TmaCfg<BN>::SMEM));
-    dim3 grid((unsigned)(p.N * t.PT * t.QT), (unsigned)((p.ncols + BN - 1) / BN), 1);
-    k_conv_tc_tma<BN><<<grid, TMA_THREADS, TmaCfg<BN>::SMEM, st>>>(wmap, amap, p, t, out32,
-                                                                    out64, s1, hi, lo, err);
-    IQ_LAUNCH_CHECK();
-    return IQ_OK;
-}
-
-// the TMA-fed kernel when the problem allows it (stride 1, whole 64-channel k-blocks,
-// 16-byte aligned rows and a tile rectangle with little waste); *used = false otherwise
-iq_status try_launch_tma(const CUtensorMap& wmap, const TcP& p, const int8_t* x,
-                         int32_t* out32, long long* out64, unsigned long long* s1, int* hi,
-                         int* lo, int* err, cudaStream_t st, bool* used) {
-    *used = false;
-    // opt-in: the register gather moves fewer bytes through shared memory (measured faster)
-    const char* e = getenv("IQ_TMA_GATHER");
-    if (!e || e[0] != '1') return IQ_OK;
-    if (p.sh != 1 || p.sw != 1 || !p.tap_mode || (p.cstride % 16) || (p.cofs % 64) ||
-        ((uintptr_t)x & 15))
-        return IQ_OK;
-    TmaTile t;
-    if (!pick_tma_tile(p.P, p.Q, &t)) return IQ_OK;
-    CUtensorMap amap;
-    iq_status r = encode_acts(x, p.N, p.H, p.W, p.cstride, t, &amap);
-    if (r != IQ_OK) return IQ_OK;   // fall back to the gather kernel
-    switch (pick_bn(p.ncols)) {
-        case 64: r = launch_tma_bn<64>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
-        case 128: r = launch_tma_bn<128>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
-        default: r = launch_tma_bn<256>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
-    }
-    if (r == IQ_OK) *used = true;
-    return r;
 }
 
 // 4-D map over the fp16 carriers [N][H][W][cstride]: box 64 channels x BW x BH pixels at
@@ -2478,8 +1854,6 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
         r = try_launch_t(map, p, x, xf, true, acc, nullptr, s1, hi, lo, err, st, &used);
         if (r != IQ_OK) return r;
     }
-    if (!used) r = try_launch_tma(map, p, x, acc, nullptr, s1, hi, lo, err, st, &used);
-    if (r != IQ_OK) return r;
     if (!used) r = launch(map, p, 1, x, nullptr, acc, nullptr, s1, hi, lo, err, st);
     if (r == IQ_OK) *done = true;
     return r;
@@ -2566,8 +1940,6 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
             r = try_launch_t(map, p, e, ef, sl == 0, out32, out64, s1, hi, lo, err, st, &used);
             if (r != IQ_OK) return r;
         }
-        if (!used) r = try_launch_tma(map, p, e, out32, out64, s1, hi, lo, err, st, &used);
-        if (r != IQ_OK) return r;
         if (!used) r = launch(map, p, 1, e, nullptr, out32, out64, s1, hi, lo, err, st);
         if (r != IQ_OK) return r;
     }

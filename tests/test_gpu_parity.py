@@ -492,25 +492,3 @@ def test_conv_dgrad_int64_reduction():
     with pytest.raises(iq.IqError):
         iq.iq_conv_dgrad(d, dev(e), dscal(1e-4), dev(wq), dx, s_dx,
                          acc_out=torch.empty((n, h, w, c), dtype=torch.int32, device=DEV))
-
-
-@pytest.mark.parametrize("ci", [0, 1, 4])
-def test_conv_tc_tma_gather_path(ci, monkeypatch):
-    # the opt-in TMA-staged activation path must agree with the oracle as well
-    monkeypatch.setenv("IQ_TMA_GATHER", "1")
-    n, h, w, c, k, r, s, st, pd, dl = TC_CASES[ci]
-    cv = O.Conv(n, h, w, c, k, r, s, st, pd, dl)
-    d = iq.conv_desc(n, h, w, c, k, r, s, st, pd, dl)
-    g = S.rng(300 + ci)
-    x = S.int8_uniform(g, (n, h, w, c))
-    wq = O.requant_master(O.uq(S.he_weights(g, (k, r, s, c), c * r * s), 24)).astype(np.int8)
-    p, q = cv.pq
-    a = torch.empty((n, p, q, k), dtype=torch.int8, device=DEV)
-    acc = torch.empty((n, p, q, k), dtype=torch.int32, device=DEV)
-    iq.iq_conv_fwd(d, dev(x), dscal(0.01), dev(wq), a, dscal(), relu=True, acc_out=acc)
-    assert np.array_equal(host(acc), O.conv_fwd(cv, x, wq))
-    e = S.int8_uniform(g, (n, p, q, k))
-    dacc = torch.empty((n, h, w, c), dtype=torch.int32, device=DEV)
-    iq.iq_conv_dgrad(d, dev(e), dscal(1e-3), dev(wq), torch.empty((n, h, w, c), dtype=torch.int8,
-                     device=DEV), dscal(), acc_out=dacc)
-    assert np.array_equal(host(dacc), O.conv_dgrad(cv, e, wq))
