@@ -371,6 +371,7 @@ def run_ours(args, rank, world, local):
         torch.cuda.synchronize(dev)
     barrier(world)
     launches = iq.launch_count() - launches0
+    iq.iq_device_status(stream)     # raises if a bounded device wait gave up
     for k, f in orig.items():
         setattr(iq, k, f)
     ms_total = t_start.elapsed_time(t_end)
@@ -417,6 +418,7 @@ def run_ours(args, rank, world, local):
         res_h.copy_(wl.result(net), non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize(dev)
+    iq.iq_device_status(stream)
     ms_e2e = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world, dev)
     tops_e2e = 2 * macs * world / (ms_e2e * 1e-3) / 1e12
 

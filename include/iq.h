@@ -94,6 +94,16 @@ int iq_version(void);
  * paper has no counterpart -- it lets a caller count device launches in a region). */
 unsigned long long iq_launch_count(void);
 
+/* iq_device_status -- the library's sticky device status (the paper has no counterpart).
+ * Every wait inside the tensor-core convolution kernels is bounded (about one second); a
+ * wait that gives up records a code (1: operand loads, 2: MMA issue, 3: epilogue, 4: a
+ * TMA-fed producer), the kernel returns without completing its tiles, and every later
+ * launch of those kernels returns at once, so the outputs of that call and of all later
+ * calls are not valid.  This call synchronizes `stream`, stores the code in *code (0 when
+ * nothing gave up), clears it and returns IQ_ERR_TIMEOUT when it was set, else IQ_OK.
+ * Call it after a sequence of calls (a training step) to learn whether they completed. */
+iq_status iq_device_status(int32_t* code, iq_stream stream);
+
 /* Output size of a convolution (host-side, no device work). */
 iq_status iq_conv_out_size(const iq_conv_desc* d, int32_t* p, int32_t* q);
 

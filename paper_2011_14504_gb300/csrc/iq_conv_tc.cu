@@ -25,14 +25,16 @@
 // In all three one elected thread issues tcgen05.mma (M=128, K=16) into TMEM and
 // epilogue warps fold the fp32 chunks into int32 and write either int32 outputs plus
 // per-channel sum / max / min (FWD), int32 split partials or int64 atomic adds (WGRAD).
-// Every mbarrier wait is bounded (about one second); on expiry the CTA records an error
-// word, drains what it issued and returns, and later CTAs of the launch exit at once.
+// Every mbarrier wait is bounded (about one second); on expiry the CTA records a code in
+// the device's sticky status word, drains what it issued and returns, and every later
+// launch exits at once until the host reads the status (iq_device_status).
 #include "iq_conv_tc.cuh"
 #include "iq_tc_ptx.cuh"
 
 #include <climits>
 #include <cstring>
 #include <cudaTypedefs.h>
+#include <mutex>
 
 namespace iq {
 
@@ -1542,6 +1544,15 @@ struct TmaTile {
     int BW, BH, PT, QT;
 };
 
+// Sticky status of the tensor-core kernels on each device: 0, or the code of the first
+// bounded wait that gave up (1: operand loads, 2: MMA issue, 3: epilogue, 4: a TMA-fed
+// producer).  Set by the kernels, read and cleared by iq_device_status; while it is set,
+// every later launch of these kernels returns at once.
+__device__ int g_tc_status;
+
+std::mutex g_tc_status_mu;
+int* g_tc_status_ptr[256] = {};
+
 // int8 KRSC weights -> fp16 [K][kpad] (zero beyond R*S*C)
 __global__ void k_widen_weights(const int8_t* __restrict__ w, __half* __restrict__ wf, int K,
                                 int kdim, int kpad) {
@@ -1583,6 +1594,19 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
             fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
     }
     return fn;
+}
+
+// device address of g_tc_status on the current device (looked up once per device)
+int* tc_status_ptr() {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return nullptr;
+    std::lock_guard<std::mutex> lock(g_tc_status_mu);
+    if (!g_tc_status_ptr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_tc_status) != cudaSuccess || !p) return nullptr;
+        g_tc_status_ptr[dev] = static_cast<int*>(p);
+    }
+    return g_tc_status_ptr[dev];
 }
 
 bool tc_env_disabled() {
@@ -1778,7 +1802,7 @@ constexpr int MAX_KB_INT32 = 133120 / 64;   // 2080 k-blocks: 133120 * 127^2 < 2
 
 // ================================================================ forward
 
-// fp16 weights, the error word, then the fp16 carriers of the input
+// fp16 weights, a reserved 256-byte slot, then the fp16 carriers of the input
 static size_t acts16_offset(size_t wbytes) { return (wbytes + 256 + 255) / 256 * 256; }
 
 // inputs with few channels (C % 64 != 0, R S C <= 512) go through an fp16 im2col
@@ -1823,11 +1847,11 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     if (p.nkb_total > MAX_KB_INT32) return IQ_OK;   // cannot happen under the CRS bound
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     __half* wf = reinterpret_cast<__half*>(wsb);
-    int* err = reinterpret_cast<int*>(wsb + (size_t)p.K * p.kpad * 2);
+    int* err = tc_status_ptr();
+    if (!err) return IQ_ERR_CUDA;
     k_widen_weights<<<grid_for((int64_t)p.K * p.kpad), kThreads, 0, st>>>(w, wf, p.K, p.kdim,
                                                                          p.kpad);
     IQ_LAUNCH_CHECK();
-    IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
     CUtensorMap map;
     iq_status r = encode_weights(wf, p.K, p.kpad, pick_bn(p.ncols), &map);
     if (r != IQ_OK) return r;
@@ -1923,8 +1947,8 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
     if (p.P != d->h || p.Q != d->w) return IQ_OK;
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     __half* wf = reinterpret_cast<__half*>(wsb);
-    int* err = reinterpret_cast<int*>(wsb + (size_t)d->c * p.kpad * 2);
-    IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
+    int* err = tc_status_ptr();
+    if (!err) return IQ_ERR_CUDA;
     __half* ef = reinterpret_cast<__half*>(wsb + acts16_offset((size_t)d->c * p.kpad * 2));
     const bool ef_ok = ((int64_t)p.N * p.H * p.W * p.cstride) % 16 == 0;
     for (int sl = 0; sl < nsl; sl++) {
@@ -1949,7 +1973,7 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
 
 // ================================================================ weight gradient
 
-// the error word, then the fp16 carriers of the errors and of the input
+// a reserved 256-byte slot, then the fp16 carriers of the errors and of the input
 namespace {
 
 // the split of nkb k-blocks that minimises (tiles per SM) x (k-blocks per tile) on the
@@ -1996,7 +2020,7 @@ bool wgrad_tma_plan(const iq_conv_desc* d, TcP* p, TmaTile* t, int* nsplit) {
 
 }  // namespace
 
-// the error word, the fp16 carriers of the errors and of the input, and the per-split
+// a reserved 256-byte slot, the fp16 carriers of the errors and of the input, and the per-split
 // int32 partial sums of the all-TMA path
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d) {
     const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
@@ -2061,8 +2085,8 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
     *done = false;
     if (tc_env_disabled() || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
-    int* err = reinterpret_cast<int*>(wsb);
-    IQ_CUDA_CHECK(cudaMemsetAsync(err, 0, sizeof(int), st));
+    int* err = tc_status_ptr();
+    if (!err) return IQ_ERR_CUDA;
     TcP p;
     TmaTile t;
     int nsplit = 1;
@@ -2126,3 +2150,16 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
 }
 
 }  // namespace iq
+
+extern "C" iq_status iq_device_status(int32_t* code, iq_stream stream) {
+    if (!code) return IQ_ERR_INVALID_ARG;
+    int* p = iq::tc_status_ptr();
+    if (!p) return IQ_ERR_CUDA;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int v = 0;
+    IQ_CUDA_CHECK(cudaStreamSynchronize(st));
+    IQ_CUDA_CHECK(cudaMemcpy(&v, p, sizeof(int), cudaMemcpyDeviceToHost));
+    if (v != 0) IQ_CUDA_CHECK(cudaMemset(p, 0, sizeof(int)));
+    *code = v;
+    return v != 0 ? IQ_ERR_TIMEOUT : IQ_OK;
+}

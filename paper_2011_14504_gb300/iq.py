@@ -30,7 +30,7 @@ EXPORTS = [
     "iq_mse_grad", "iq_bn_int_fwd_noalloc", "iq_combine_workspace_size", "iq_combine",
     "iq_spatial_sum_workspace_size", "iq_spatial_sum", "iq_avgpool_bwd", "iq_channel_slice",
     "iq_bilinear_workspace_size", "iq_bilinear_up_fwd", "iq_bilinear_up_bwd", "iq_ce_grad",
-    "iq_bn_update",
+    "iq_bn_update", "iq_device_status",
 ]
 
 
@@ -131,6 +131,7 @@ def load(path: str | None = None):
     L.iq_ce_grad.argtypes = [_P, _P, _P, _I64, _I32, _I32, _P, _P, _P, _P, _SZ, _P]
     L.iq_bn_update.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _I32, C.POINTER(BnBits), _I, _I,
                                _U64, _U64, _U64, _P, _SZ, _P]
+    L.iq_device_status.argtypes = [C.POINTER(_I32), _P]
     for f in EXPORTS:
         if f not in ("iq_status_str", "iq_version", "iq_launch_count"):
             getattr(L, f).restype = _I
@@ -140,6 +141,15 @@ def load(path: str | None = None):
 
 def launch_count() -> int:
     return int(load().iq_launch_count())
+
+
+def iq_device_status(stream=None) -> int:
+    """Synchronize the stream, return and clear the sticky device status of the tensor-core
+    kernels (0: every bounded wait completed).  Raises IqError(IQ_ERR_TIMEOUT) when a wait
+    gave up, since the outputs since the last check are then not valid."""
+    code = _I32(0)
+    _check("iq_device_status", load().iq_device_status(C.byref(code), _stream(stream)))
+    return code.value
 
 
 def status_str(code: int) -> str:
