@@ -1457,6 +1457,226 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     }
 }
 
+// ---------------------------------------------------------------- channel-major forward
+// The forward (and stride-1 data-gradient) GEMM transposed, for layers with at most 128
+// output channels: D^T[channels x pixels] = W X^T with M = 128 output channels (weight rows
+// past the last channel are TMA zero fill) and N = 256 pixels (a BW x BH rectangle of one
+// image).  tcgen05 reaches its full rate only at N = 256; the pixel-major kernel would run
+// these layers at N = 64 or 128, a quarter or half of it.  TMEM lane = output channel,
+// column = pixel of the rectangle.  Each epilogue thread owns one channel and 64 pixels, so
+// a warp's int32 stores cover 32 consecutive channels of one pixel and the per-channel
+// statistics are per-thread sums (one atomic triple per thread and tile).  Loads, MMA
+// issue, accumulator handshake and bounded waits are those of k_conv_tct.
+constexpr int CM_PIX = 256;        // pixels per tile (GEMM N)
+constexpr int CM_CH = 128;         // output channels per tile (GEMM M)
+
+__global__ void __launch_bounds__(THREADS_T, 1)
+    k_conv_tcc(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap amap,
+               TcP p, RectGrid g, int bw_log2, int32_t* __restrict__ out32,
+               unsigned long long* __restrict__ s1, int* __restrict__ hi_c,
+               int* __restrict__ lo_c, int* __restrict__ err) {
+    constexpr int STAGE_BYTES = A_BYTES + CM_PIX * 128;
+    constexpr int TMEM_COLS = 2 * CM_PIX;
+    constexpr int CW = CM_PIX / 4;             // pixels per epilogue warpgroup
+    constexpr int LDW = 16;                    // columns per TMEM load
+    static_assert(STAGE_BYTES == CfgT<256>::STAGE_BYTES, "stage layout of CfgT<256>");
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    BarsT* bars = reinterpret_cast<BarsT*>(smem + CfgT<256>::BAR_OFF);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    if (__syncthreads_or(tid == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    if ((int)blockIdx.x >= g.total) return;
+
+    if (tid == 0) {
+        for (int s = 0; s < STAGES_T; s++) {
+            tc::mbar_init(&bars->full[s], 1);
+            tc::mbar_init(&bars->empty[s], 1);
+        }
+        for (int b = 0; b < 2; b++) {
+            tc::mbar_init(&bars->accf[b], 1);
+            tc::mbar_init(&bars->acce[b], EPI_T);
+        }
+        tc::mbar_init(&bars->done, 1);
+        bars->abort = 0;
+        bars->never = 0;
+        tc::mbar_fence_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
+        tc::tmem_relinquish();
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
+    volatile int* abort_flag = &bars->abort;
+
+    if (warp == 0) {
+        // ================================================ TMA issuer
+        if (lane == 0) {
+            tc::tma_prefetch_desc(&amap);
+            tc::tma_prefetch_desc(&wmap);
+            RectPos q;
+            rpos_set(q, blockIdx.x, g, CM_CH);
+            int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
+            uint32_t kbc = 0;
+            int issued = 0;
+            while (q.tile < g.total) {
+                const int s = kbc % STAGES_T;
+                const uint32_t it = kbc / STAGES_T;
+                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                    bars->abort = 1;
+                    atomicExch(err, 4);
+                    break;
+                }
+                uint8_t* st = smem + s * STAGE_BYTES;
+                tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
+                // A: weight rows n0 .. n0 + 127 (zero past the last channel)
+                tc::tma_load_2d(st, &wmap, &bars->full[s], q.kb * BK, q.n0);
+                // B: the 256 input pixels of tap (r, ss), channels c0 .. c0 + 63
+                tc::tma_load_4d(st + A_BYTES, &amap, &bars->full[s], p.cofs + c0,
+                                q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph, q.n);
+                tc::mbar_arrive(&bars->full[s]);
+                issued = (int)kbc + 1;
+                kbc++;
+                const int tile = q.tile;
+                rpos_next(q, p, g, CM_CH);
+                if (q.tile != tile) {
+                    r = ss = c0 = 0;
+                } else {
+                    c0 += BK;
+                    if (c0 >= p.C) {
+                        c0 = 0;
+                        if (++ss == p.S) { ss = 0; r++; }
+                    }
+                }
+            }
+            if (*abort_flag) {
+                for (int kb = (issued > STAGES_T ? issued - STAGES_T : 0); kb < issued; kb++)
+                    tc::mbar_wait(&bars->full[kb % STAGES_T], (uint32_t)(kb / STAGES_T) & 1,
+                                  &bars->never);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ================================================ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_f16(CM_CH, CM_PIX, false);
+            bool ok = true;
+            uint32_t kbc = 0, cc = 0;
+            TPos<false> q;
+            q.set(blockIdx.x, p, g, CM_CH);
+            while (ok && q.tile < g.total) {
+                const int s = kbc % STAGES_T;
+                const uint32_t it = kbc / STAGES_T;
+                const bool first = (q.kb % CHUNK_KB) == 0;
+                const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
+                const uint32_t buf = cc & 1;
+                if (first && cc >= 2 &&
+                    !tc::mbar_wait(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                if (!tc::mbar_wait(&bars->full[s], it & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc::tc_fence_after();
+                const uint32_t a_addr = tc::smem_u32(smem + s * STAGE_BYTES);
+                const uint32_t b_addr = a_addr + A_BYTES;
+#pragma unroll
+                for (int k = 0; k < BK / 16; k++)
+                    tc::umma_f16(tmem + buf * CM_PIX, tc::sdesc_kmajor_sw128(a_addr + 32 * k),
+                                 tc::sdesc_kmajor_sw128(b_addr + 32 * k), idesc,
+                                 (first && k == 0) ? 0u : 1u);
+                tc::umma_commit(&bars->empty[s]);
+                if (last) {
+                    tc::umma_commit(&bars->accf[buf]);
+                    cc++;
+                }
+                kbc++;
+                q.next(p, g, CM_CH);
+            }
+            if (!ok) {
+                bars->abort = 1;
+                atomicExch(err, 2);
+            }
+            tc::umma_commit(&bars->done);
+            tc::mbar_wait(&bars->done, 0, &bars->never);
+        }
+        __syncwarp();
+    } else if (warp >= 4) {
+        // ================================================ epilogue (warps 4..19)
+        const int quarter = (warp - 4) >> 2;          // pixels [64 quarter, 64 quarter + 64)
+        const int lq = warp & 3;                      // TMEM lanes (channels) 32 lq ..
+        const uint32_t taddr = tmem + ((uint32_t)(lq * 32) << 16) + quarter * CW;
+        const int bw_mask = g.BW - 1;
+        uint32_t cc = 0;
+        bool ok = true;
+        TPos<false> q;
+        q.set(blockIdx.x, p, g, CM_CH);
+        int sum[CW];
+        while (ok && q.tile < g.total) {
+            const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
+#pragma unroll
+            for (int i = 0; i < CW; i++) sum[i] = 0;
+            for (int c = 0; c < nch; c++) {
+                const uint32_t buf = cc & 1;
+                if (!tc::mbar_wait_sleep(&bars->accf[buf], (cc >> 1) & 1, abort_flag)) {
+                    ok = false;
+                    bars->abort = 1;
+                    atomicExch(err, 3);
+                    break;
+                }
+                tc::tc_fence_after();
+#pragma unroll
+                for (int cb = 0; cb < CW; cb += LDW) {
+                    uint32_t d[LDW];
+                    tc::tmem_ld_32x32b_x16(taddr + buf * CM_PIX + cb, d);
+                    tc::tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < LDW; i++) sum[cb + i] += __float2int_rn(__uint_as_float(d[i]));
+                }
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bars->acce[buf]);
+                cc++;
+            }
+            if (!ok || *abort_flag) break;
+            const int ch = q.n0 + lq * 32 + lane;
+            const bool chv = ch < p.ncols;
+            long long my_sum = 0;
+            int my_hi = INT_MIN, my_lo = INT_MAX;
+#pragma unroll
+            for (int j = 0; j < CW; j++) {
+                const int rr = quarter * CW + j;
+                const int pp = q.p0 + (rr >> bw_log2), qq = q.q0 + (rr & bw_mask);
+                if (pp < p.P && qq < p.Q) {          // the same pixel for the whole warp
+                    const int64_t m = ((int64_t)q.n * p.P + pp) * p.Q + qq;
+                    if (chv) out32[m * p.ncols + ch] = sum[j];
+                    my_sum += sum[j];
+                    my_hi = max(my_hi, sum[j]);
+                    my_lo = min(my_lo, sum[j]);
+                }
+            }
+            if (chv && my_hi != INT_MIN) {
+                atomicAdd(&s1[ch], (unsigned long long)my_sum);
+                atomicMax(&hi_c[ch], my_hi);
+                atomicMin(&lo_c[ch], my_lo);
+            }
+            q.set(q.tile + gridDim.x, p, g, CM_CH);
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
 // G[i] += sum over the splits of their int32 partial sums (4 elements per thread)
 __global__ void k_split_sum(const int32_t* __restrict__ part, int ns, int64_t total4,
                             long long* __restrict__ G) {
@@ -1695,12 +1915,12 @@ iq_status launch(const CUtensorMap& map, const TcP& p, int nsplit, const int8_t*
     }
 }
 
-// Tile rectangle for the TMA-fed kernel: BW x BH = 128 output pixels; the shape with the
+// Tile rectangle for the TMA-fed kernels: BW x BH = npix output pixels; the shape with the
 // least padding waste, if that waste is small.
-bool pick_tma_tile(int P, int Q, TmaTile* t, double min_util = 0.8) {
+bool pick_tma_tile(int P, int Q, TmaTile* t, double min_util = 0.8, int npix = 128) {
     double best = 0.0;
-    for (int BW = 128; BW >= 16; BW /= 2) {
-        const int BH = 128 / BW;
+    for (int BW = npix; BW >= 16; BW /= 2) {
+        const int BH = npix / BW;
         const int PT = (P + BH - 1) / BH, QT = (Q + BW - 1) / BW;
         const double util = (double)P * Q / ((double)PT * BH * QT * BW);
         if (util > best + 1e-9) {
@@ -1785,6 +2005,50 @@ iq_status try_launch_t(const CUtensorMap& wmap, const TcP& p, const int8_t* x, _
     return r;
 }
 
+// Whether the channel-major kernel takes this problem (at most 128 output channels, whole
+// 64-channel k-blocks, strides 1 or 2, aligned slices, a 256-pixel rectangle tiling with
+// little waste)
+bool cm_ok(const TcP& p, TmaTile* t) {
+    if (p.ncols > CM_CH || tma16_disabled() || !p.tap_mode || p.sh > 2 || p.sw > 2 ||
+        (p.cstride % 8) || (p.cofs % 64))
+        return false;
+    if (!pick_tma_tile(p.P, p.Q, t, 0.6, CM_PIX)) return false;
+    return t->BW * p.sw <= 256 && t->BH * p.sh <= 256;
+}
+
+// the channel-major kernel for problems with at most 128 output channels and int32 output
+// with statistics (wf: the fp16 weights [rows][kpad]); *used = false when not taken
+iq_status try_launch_c(const __half* wf, int rows, const TcP& p, const int8_t* x, __half* xf,
+                       bool convert, int32_t* out32, unsigned long long* s1, int* hi, int* lo,
+                       int* err, cudaStream_t st, bool* used) {
+    *used = false;
+    TmaTile t;
+    if (!xf || !out32 || !s1 || !cm_ok(p, &t)) return IQ_OK;
+    CUtensorMap wmap, amap;
+    if (encode_weights(wf, rows, p.kpad, CM_CH, &wmap) != IQ_OK) return IQ_OK;
+    if (encode_acts16(xf, p.N, p.H, p.W, p.cstride, t, p.sh, p.sw, &amap) != IQ_OK) return IQ_OK;
+    if (convert) {
+        const int64_t n16 = (int64_t)p.N * p.H * p.W * p.cstride / 16;
+        k_codes_to_f16<<<grid_for(n16), kThreads, 0, st>>>(x, xf, n16);
+        IQ_LAUNCH_CHECK();
+    }
+    IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tcc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       CfgT<256>::SMEM));
+    RectGrid g;
+    g.PT = t.PT; g.QT = t.QT; g.BW = t.BW; g.BH = t.BH;
+    g.mt = p.N * t.PT * t.QT;
+    g.nt = (p.ncols + CM_CH - 1) / CM_CH;
+    g.total = g.mt * g.nt;
+    int bw_log2 = 0;
+    while ((1 << bw_log2) < t.BW) bw_log2++;
+    const int grid = g.total < num_sms() ? g.total : num_sms();
+    k_conv_tcc<<<grid, THREADS_T, CfgT<256>::SMEM, st>>>(wmap, amap, p, g, bw_log2, out32, s1,
+                                                          hi, lo, err);
+    IQ_LAUNCH_CHECK();
+    *used = true;
+    return IQ_OK;
+}
+
 void fill_geom(TcP& p, const iq_conv_desc* d) {
     p.N = d->n; p.H = d->h; p.W = d->w; p.C = d->c; p.K = d->k; p.R = d->r; p.S = d->s;
     p.sh = d->stride_h; p.sw = d->stride_w; p.ph = d->pad_h; p.pw = d->pad_w;
@@ -1865,17 +2129,27 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
         q.R = q.S = 1; q.sh = q.sw = 1; q.ph = q.pw = 0; q.dh = q.dw = 1;
         q.kdim = p.kpad; q.tap_mode = 1;
         TmaTile tt;
-        if (tma16_ok(q, &tt)) {
+        const bool cm = cm_ok(q, &tt);
+        if (cm || tma16_ok(q, &tt)) {
             const int per_row = p.Q * (p.kpad / 4);
             dim3 gi((unsigned)((per_row + kThreads - 1) / kThreads), (unsigned)p.P, (unsigned)p.N);
             k_im2col_f16<<<gi, kThreads, 0, st>>>(x, p, xf);
             IQ_LAUNCH_CHECK();
-            r = try_launch_t(map, q, nullptr, xf, false, acc, nullptr, s1, hi, lo, err, st, &used);
-            if (r != IQ_OK) return r;
+            if (cm) {
+                r = try_launch_c(wf, p.K, q, nullptr, xf, false, acc, s1, hi, lo, err, st, &used);
+                if (r != IQ_OK) return r;
+            }
+            if (!used) {
+                r = try_launch_t(map, q, nullptr, xf, false, acc, nullptr, s1, hi, lo, err, st,
+                                 &used);
+                if (r != IQ_OK) return r;
+            }
         }
     }
     if (!used && (p.N * (int64_t)p.H * p.W * p.cstride) % 16 == 0) {
-        r = try_launch_t(map, p, x, xf, true, acc, nullptr, s1, hi, lo, err, st, &used);
+        r = try_launch_c(wf, p.K, p, x, xf, true, acc, s1, hi, lo, err, st, &used);
+        if (r != IQ_OK) return r;
+        if (!used) r = try_launch_t(map, p, x, xf, true, acc, nullptr, s1, hi, lo, err, st, &used);
         if (r != IQ_OK) return r;
     }
     if (!used) r = launch(map, p, 1, x, nullptr, acc, nullptr, s1, hi, lo, err, st);
@@ -1960,7 +2234,11 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
         if (r != IQ_OK) return r;
         p.cofs = sl * kc;
         bool used = false;
-        if (ef_ok) {
+        if (ef_ok && nsl == 1) {
+            r = try_launch_c(wf, d->c, p, e, ef, true, out32, s1, hi, lo, err, st, &used);
+            if (r != IQ_OK) return r;
+        }
+        if (ef_ok && !used) {
             r = try_launch_t(map, p, e, ef, sl == 0, out32, out64, s1, hi, lo, err, st, &used);
             if (r != IQ_OK) return r;
         }

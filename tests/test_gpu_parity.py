@@ -313,6 +313,12 @@ TC_CASES = [
     (2, 31, 29, 4, 64, 3, 3, 1, 1, 1),      # 4 input channels (fp16 im2col forward)
     (1, 35, 35, 4, 64, 7, 7, 2, 3, 1),      # stem: 7x7 stride 2 over 4 channels
     (2, 17, 15, 128, 96, 3, 3, 1, 2, 2),    # dilation 2, rectangle tiles with waste
+    # channel-major kernel (at most 128 output channels, 256-pixel rectangles)
+    (1, 64, 64, 64, 64, 3, 3, 1, 1, 1),     # conv1_2 shape: forward and data gradient
+    (2, 50, 48, 64, 72, 3, 3, 1, 1, 1),     # ragged channels (72) and 16 x 16 rectangles
+    (1, 64, 64, 128, 128, 3, 3, 2, 1, 1),   # stride 2, 128 output channels
+    (1, 32, 40, 64, 128, 3, 3, 1, 1, 1),    # 128 output channels, data gradient to 64
+    (2, 128, 160, 64, 64, 3, 3, 1, 1, 1),   # 160 tiles: persistent CTAs run two tiles
 ]
 
 
@@ -354,11 +360,11 @@ def test_conv_fwd_tc_shapes(ci):
     assert np.array_equal(host(gq).astype(np.int32), wg) and host(s_g)[0] == wgs
 
 
-@pytest.mark.parametrize("sign", [1, -1])
-def test_conv_fwd_adversarial_full_scale(sign):
+@pytest.mark.parametrize("sign,h,k", [(1, 6, 128), (-1, 6, 128), (1, 16, 64), (-1, 16, 64)])
+def test_conv_fwd_adversarial_full_scale(sign, h, k):
     # all codes at +-127: every fp32 chunk holds 1024 * 127^2 = 16,516,096 < 2^24 and
-    # the int32 total is 4608 * 127^2 for interior pixels
-    n, h, w, c, k = 1, 6, 6, 512, 128
+    # the int32 total is 4608 * 127^2 for interior pixels (16 x 16 x 64: channel-major kernel)
+    n, w, c = 1, h, 512
     cv = O.Conv(n, h, w, c, k, 3, 3, 1, 1)
     d = iq.conv_desc(n, h, w, c, k, 3, 3, 1, 1)
     x = np.full((n, h, w, c), 127, np.int8)
