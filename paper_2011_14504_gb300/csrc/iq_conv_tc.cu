@@ -1051,6 +1051,7 @@ struct BarsT {
 struct RectGrid {
     int PT, QT, BW, BH;   // rectangles per image (rows x columns) and their size
     int mt, nt, total;    // m-tiles (N * PT * QT), n-tiles, tiles
+    int nb;               // weight gradient: 64-channel blocks per im2col box
 };
 
 struct RectPos {
@@ -1188,10 +1189,12 @@ struct TPos<true> : WgPos {
 
 // WG: the weight gradient.  A k-block is a BW x BH rectangle of 64 output pixels of one
 // image (the rectangles tile every image; pixels outside it read zero errors).  A = E^T
-// (two 4-D boxes of 64 channels x the rectangle of the fp16 errors, map `wmap`) and B = the
-// im2col of x (one 4-D box per 64-column tap block: 64 channels x the rectangle at the conv
-// strides, map `amap`), both MN-major; tiles are (channel tile, column tile, K split) and
-// the epilogue adds its int32 sums into the int64 output.
+// (one 5-D box: 64 channels x the rectangle x 2 channel blocks of the fp16 errors, map
+// `wmap`) and B = the im2col of x (per tap, one 5-D box of 64 channels x the rectangle at
+// the conv strides x g.nb channel blocks, map `amap`), both MN-major: a box lands as
+// g.nb blocks of 64 rows of 128 bytes, the 8192-byte MN-block stride of the UMMA layout.
+// Tiles are (channel tile, column tile, K split); the epilogue writes each split's int32
+// sums to its own slab (OUT_PART32).
 template <int BN, bool WG>
 __global__ void __launch_bounds__(THREADS_T, 1)
     k_conv_tct(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap amap,
@@ -1246,7 +1249,28 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             wpos_set(q, blockIdx.x, p, g, BN);
             uint32_t kbc = 0;
             int issued = 0;
+            // per tile: the box coordinates of the B column runs (x and y offsets of the tap,
+            // first channel block); per k-block: the rectangle, advanced without divisions
+            int bx[4], by[4], bc[4];
+            int tile_seen = -1, nimg = 0, pt = 0, qt = 0;
             while (q.tile < g.total) {
+                if (q.tile != tile_seen) {
+                    tile_seen = q.tile;
+#pragma unroll
+                    for (int j = 0; j < 4; j++) {
+                        const int col = q.n0 + 64 * g.nb * j;
+                        const int tap = col / p.C;
+                        const int r = tap / p.S, ss = tap - r * p.S;
+                        bx[j] = ss * p.dw - p.pw;
+                        by[j] = r * p.dh - p.ph;
+                        bc[j] = (col - tap * p.C) >> 6;
+                    }
+                    const int kr = q.kb0;
+                    nimg = kr / (g.PT * g.QT);
+                    const int rr = kr - nimg * (g.PT * g.QT);
+                    pt = rr / g.QT;
+                    qt = rr - pt * g.QT;
+                }
                 const int s = kbc % STAGES_T;
                 const uint32_t it = kbc / STAGES_T;
                 if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
@@ -1256,24 +1280,22 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 }
                 uint8_t* st = smem + s * STAGE_BYTES;
                 tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
-                // the k-block's pixels: rectangle kb of the BW x BH tiling of the output
-                const int kr = q.kb0 + q.kb;
-                const int nimg = kr / (g.PT * g.QT);
-                const int rr = kr - nimg * (g.PT * g.QT);
-                const int pp = (rr / g.QT) * g.BH, qq = (rr - (rr / g.QT) * g.QT) * g.BW;
-                // A: E[rectangle][m0 .. m0+127] as two 64-channel boxes (zero outside P x Q)
-                tc::tma_load_4d(st, &wmap, &bars->full[s], (int)q.m0, qq, pp, nimg);
-                tc::tma_load_4d(st + 8192, &wmap, &bars->full[s], (int)q.m0 + 64, qq, pp, nimg);
-                // B: per 64-column block (one tap, 64 channels) the input box of the pixels
+                // the k-block's pixels: rectangle (pt, qt) of image nimg
+                const int pp = pt * g.BH, qq = qt * g.BW;
+                // A: E[rectangle][m0 .. m0+127], both 64-channel blocks in one box (zero
+                // outside P x Q and past the last channel block)
+                tc::tma_load_5d(st, &wmap, &bars->full[s], 0, qq, pp, (int)(q.m0 >> 6), nimg);
+                // B: per run of g.nb 64-column blocks (one tap, 64 g.nb channels) the input
+                // box of the pixels
 #pragma unroll
-                for (int bb = 0; bb < BN / 64; bb++) {
-                    const int col = q.n0 + 64 * bb;
-                    const int tap = col / p.C;
-                    const int c0 = col - tap * p.C;
-                    const int r = tap / p.S, ss = tap - r * p.S;
-                    tc::tma_load_4d(st + A_BYTES + 8192 * bb, &amap, &bars->full[s], c0,
-                                    qq * p.sw + ss * p.dw - p.pw, pp * p.sh + r * p.dh - p.ph,
-                                    nimg);
+                for (int j = 0; j < 4; j++) {
+                    if (j * g.nb >= BN / 64) break;
+                    tc::tma_load_5d(st + A_BYTES + 8192 * g.nb * j, &amap, &bars->full[s], 0,
+                                    qq * p.sw + bx[j], pp * p.sh + by[j], bc[j], nimg);
+                }
+                if (++qt == g.QT) {
+                    qt = 0;
+                    if (++pt == g.PT) { pt = 0; nimg++; }
                 }
                 tc::mbar_arrive(&bars->full[s]);
                 issued = (int)kbc + 1;
@@ -1948,6 +1970,27 @@ iq_status encode_acts16(const __half* xf, int N, int H, int W, int cstride, cons
     return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
 }
 
+// 5-D map over the fp16 carriers [N][H][W][cstride] with the channels split into 64-wide
+// blocks: dims (64 channels, W, H, cstride / 64 blocks, N), box 64 x BW x BH pixels (at the
+// conv strides) x nb blocks, so one load lands nb MN-major blocks of BW BH rows, 8192 bytes
+// apart when BW BH = 64.  cstride % 64 == 0.
+iq_status encode_acts16_blocks(const __half* xf, int N, int H, int W, int cstride,
+                               const TmaTile& t, int sh, int sw, int nb, CUtensorMap* map) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
+    if (!enc || cstride % 64) return IQ_ERR_UNSUPPORTED;
+    cuuint64_t gdim[5] = {64, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)(cstride / 64),
+                          (cuuint64_t)N};
+    cuuint64_t gstride[4] = {(cuuint64_t)cstride * 2, (cuuint64_t)W * cstride * 2, 128,
+                             (cuuint64_t)H * W * cstride * 2};
+    cuuint32_t box[5] = {64, (cuuint32_t)(t.BW * sw), (cuuint32_t)(t.BH * sh), (cuuint32_t)nb,
+                         1};
+    cuuint32_t estr[5] = {1, (cuuint32_t)sw, (cuuint32_t)sh, 1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, (void*)xf, gdim, gstride, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
+}
+
 bool tma16_disabled() {
     const char* e = getenv("IQ_TC_GATHER");
     return e && e[0] == '1';
@@ -1974,6 +2017,7 @@ iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const TcP& 
     g.mt = p.N * t.PT * t.QT;
     g.nt = (p.ncols + BN - 1) / BN;
     g.total = g.mt * g.nt;
+    g.nb = 1;
     const int grid = g.total < num_sms() ? g.total : num_sms();
     k_conv_tct<BN, false><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(wmap, amap, p, g, out32, out64,
                                                                   s1, hi, lo, err);
@@ -2039,6 +2083,7 @@ iq_status try_launch_c(const __half* wf, int rows, const TcP& p, const int8_t* x
     g.mt = p.N * t.PT * t.QT;
     g.nt = (p.ncols + CM_CH - 1) / CM_CH;
     g.total = g.mt * g.nt;
+    g.nb = 1;
     int bw_log2 = 0;
     while ((1 << bw_log2) < t.BW) bw_log2++;
     const int grid = g.total < num_sms() ? g.total : num_sms();
@@ -2303,7 +2348,7 @@ bool wgrad_tma_plan(const iq_conv_desc* d, TcP* p, TmaTile* t, int* nsplit) {
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d) {
     const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
     const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
-    const size_t eb = ((size_t)d->n * P * Q * ((d->k + 7) / 8 * 8) * 2 + 255) / 256 * 256;
+    const size_t eb = ((size_t)d->n * P * Q * ((d->k + 63) / 64 * 64) * 2 + 255) / 256 * 256;
     const size_t xb = ((size_t)d->n * d->h * d->w * d->c * 2 + 255) / 256 * 256;
     size_t parts = 0;
     TcP p;
@@ -2335,7 +2380,8 @@ bool wgrad_rect(const TcP& p, TmaTile* t) {
 
 template <int BN>
 iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP& p,
-                    const TmaTile& t, int nsplit, int32_t* part, int* err, cudaStream_t st) {
+                    const TmaTile& t, int nb, int nsplit, int32_t* part, int* err,
+                    cudaStream_t st) {
     IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN, true>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, CfgT<BN>::SMEM));
     RectGrid g;
@@ -2343,6 +2389,7 @@ iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP&
     g.mt = (int)((p.M + BM - 1) / BM);
     g.nt = (p.ncols + BN - 1) / BN;
     g.total = g.mt * g.nt * nsplit;
+    g.nb = nb < BN / 64 ? nb : BN / 64;
     const int grid = g.total < num_sms() ? g.total : num_sms();
     k_conv_tct<BN, true><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(emap, xmap, p, g, part, nullptr,
                                                                  nullptr, nullptr, nullptr, err);
@@ -2368,13 +2415,28 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
     TcP p;
     TmaTile t;
     int nsplit = 1;
+    CUtensorMap emap, xmap;
+    int nb = 1;
+    bool maps = false;
+    int Kp = 0;
+    size_t eb = 0, xb = 0;
     if (!tma16_disabled() && get_encode() && wgrad_tma_plan(d, &p, &t, &nsplit)) {
+        Kp = (p.K + 63) / 64 * 64;            // fp16 error rows padded to whole 64-channel blocks
+        eb = ((size_t)p.npq * Kp * 2 + 255) / 256 * 256;
+        xb = ((size_t)p.N * p.H * p.W * p.C * 2 + 255) / 256 * 256;
+        // channel blocks per im2col box: the tile's columns of one tap in as few boxes as
+        // the channel count allows
+        nb = p.C % 256 == 0 ? 4 : (p.C % 128 == 0 ? 2 : 1);
+        if (nb > pick_bn(p.ncols) / 64) nb = pick_bn(p.ncols) / 64;
+        maps = encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256), p.N, p.P, p.Q, Kp, t,
+                                    1, 1, 2, &emap) == IQ_OK &&
+               encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256 + eb), p.N, p.H, p.W,
+                                    p.C, t, p.sh, p.sw, nb, &xmap) == IQ_OK;
+    }
+    if (maps) {
         // k-blocks: the pixel rectangles of every image; each split writes its own int32
         // partial sums, added into G afterwards
-        const int Kp = (p.K + 7) / 8 * 8;     // fp16 error rows padded to 16 bytes
         const int64_t ne = p.npq * Kp, nx = (int64_t)p.N * p.H * p.W * p.C;
-        const size_t eb = ((size_t)ne * 2 + 255) / 256 * 256;
-        const size_t xb = ((size_t)nx * 2 + 255) / 256 * 256;
         __half* ef = reinterpret_cast<__half*>(wsb + 256);
         __half* xf = reinterpret_cast<__half*>(wsb + 256 + eb);
         int32_t* part = reinterpret_cast<int32_t*>(wsb + 256 + eb + xb);
@@ -2388,14 +2450,11 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         IQ_LAUNCH_CHECK();
         k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
         IQ_LAUNCH_CHECK();
-        CUtensorMap emap, xmap;
-        iq_status r = encode_acts16(ef, p.N, p.P, p.Q, Kp, t, 1, 1, &emap);
-        if (r == IQ_OK) r = encode_acts16(xf, p.N, p.H, p.W, p.C, t, p.sh, p.sw, &xmap);
-        if (r != IQ_OK) return r;
+        iq_status r = IQ_OK;
         switch (pick_bn(p.ncols)) {
-            case 64: r = launch_tw<64>(emap, xmap, p, t, nsplit, part, err, st); break;
-            case 128: r = launch_tw<128>(emap, xmap, p, t, nsplit, part, err, st); break;
-            default: r = launch_tw<256>(emap, xmap, p, t, nsplit, part, err, st); break;
+            case 64: r = launch_tw<64>(emap, xmap, p, t, nb, nsplit, part, err, st); break;
+            case 128: r = launch_tw<128>(emap, xmap, p, t, nb, nsplit, part, err, st); break;
+            default: r = launch_tw<256>(emap, xmap, p, t, nb, nsplit, part, err, st); break;
         }
         if (r != IQ_OK) return r;
         const int64_t total4 = p.M * (int64_t)p.ncols / 4;
