@@ -1012,6 +1012,24 @@ __global__ void __launch_bounds__(THREADS_Q, 1)
     }
 }
 
+// s[i] += the exact integer held in the fp32 value d[i] (|d| <= 1024 127^2 < 2^24).  When
+// every |d| < 2^22, d + 1.5 2^23 is exact and its bit pattern is 0x4B400000 + d, one add
+// and one integer add per value; otherwise the conversion instruction.
+template <int W>
+__device__ __forceinline__ void fold_f32(int* s, const uint32_t (&d)[W]) {
+    float mx = 0.0f;
+#pragma unroll
+    for (int i = 0; i < W; i++) mx = fmaxf(mx, fabsf(__uint_as_float(d[i])));
+    if (mx < 4194304.0f) {
+#pragma unroll
+        for (int i = 0; i < W; i++)
+            s[i] += __float_as_int(__uint_as_float(d[i]) + 12582912.0f) - 0x4B400000;
+    } else {
+#pragma unroll
+        for (int i = 0; i < W; i++) s[i] += __float2int_rn(__uint_as_float(d[i]));
+    }
+}
+
 // ---------------------------------------------------------------- all-TMA forward kernel
 // Stride-1/2 convolutions with whole 64-channel k-blocks, over fp16 carriers of the codes
 // (a pre-pass widens the input once per call).  The M tile is a BH x BW rectangle of one
@@ -1434,8 +1452,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                     uint32_t d[LDW];
                     tmem_ld_w<LDW>(taddr + buf * BN + cb, d);
                     tc::tmem_ld_wait();
-#pragma unroll
-                    for (int i = 0; i < LDW; i++) sum[cb + i] += __float2int_rn(__uint_as_float(d[i]));
+                    fold_f32<LDW>(sum + cb, d);
                 }
                 tc::tc_fence_before();
                 tc::mbar_arrive(&bars->acce[buf]);
@@ -1659,8 +1676,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                     uint32_t d[LDW];
                     tc::tmem_ld_32x32b_x16(taddr + buf * CM_PIX + cb, d);
                     tc::tmem_ld_wait();
-#pragma unroll
-                    for (int i = 0; i < LDW; i++) sum[cb + i] += __float2int_rn(__uint_as_float(d[i]));
+                    fold_f32<LDW>(sum + cb, d);
                 }
                 tc::tc_fence_before();
                 tc::mbar_arrive(&bars->acce[buf]);
@@ -1671,16 +1687,36 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             const bool chv = ch < p.ncols;
             long long my_sum = 0;
             int my_hi = INT_MIN, my_lo = INT_MAX;
+            if (g.BW >= CW) {
+                // the quarter's pixels are one run of one output row: pixel j at dst + j ncols
+                const int rr0 = quarter * CW;
+                const int pp = q.p0 + (rr0 >> bw_log2), qq0 = q.q0 + (rr0 & bw_mask);
+                int jlim = pp < p.P ? p.Q - qq0 : 0;
+                jlim = jlim < CW ? jlim : CW;
+                if (jlim > 0) {
+                    int32_t* dst = out32 + (((int64_t)q.n * p.P + pp) * p.Q + qq0) * p.ncols + ch;
 #pragma unroll
-            for (int j = 0; j < CW; j++) {
-                const int rr = quarter * CW + j;
-                const int pp = q.p0 + (rr >> bw_log2), qq = q.q0 + (rr & bw_mask);
-                if (pp < p.P && qq < p.Q) {          // the same pixel for the whole warp
-                    const int64_t m = ((int64_t)q.n * p.P + pp) * p.Q + qq;
-                    if (chv) out32[m * p.ncols + ch] = sum[j];
-                    my_sum += sum[j];
-                    my_hi = max(my_hi, sum[j]);
-                    my_lo = min(my_lo, sum[j]);
+                    for (int j = 0; j < CW; j++) {
+                        if (j < jlim) {               // the same pixel for the whole warp
+                            if (chv) dst[j * p.ncols] = sum[j];
+                            my_sum += sum[j];
+                            my_hi = max(my_hi, sum[j]);
+                            my_lo = min(my_lo, sum[j]);
+                        }
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < CW; j++) {
+                    const int rr = quarter * CW + j;
+                    const int pp = q.p0 + (rr >> bw_log2), qq = q.q0 + (rr & bw_mask);
+                    if (pp < p.P && qq < p.Q) {      // the same pixel for the whole warp
+                        const int64_t m = ((int64_t)q.n * p.P + pp) * p.Q + qq;
+                        if (chv) out32[m * p.ncols + ch] = sum[j];
+                        my_sum += sum[j];
+                        my_hi = max(my_hi, sum[j]);
+                        my_lo = min(my_lo, sum[j]);
+                    }
                 }
             }
             if (chv && my_hi != INT_MIN) {
