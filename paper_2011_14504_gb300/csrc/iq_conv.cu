@@ -589,18 +589,25 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
     double* s_in = cur.take<double>(1);
     void* tcws = cur.take<char>(conv_wgrad_tc_ws_bytes(d));
     int64_t* G = g_acc_out ? g_acc_out : gw;
-    IQ_CUDA_CHECK(cudaMemsetAsync(G, 0, sizeof(int64_t) * gn, st));
     k_scale_mul<<<1, 1, 0, st>>>(s_e, s_x, s_in);
     IQ_LAUNCH_CHECK();
     {
-        bool done = false;
-        iq_status r = conv_wgrad_tc(d, e, x, (long long*)G, tcws, st, &done);
+        // the tensor-core path writes every element of G and, usually, its max |G| into the
+        // requantizer's cell
+        bool done = false, amax_done = false;
+        unsigned long long* cell = (unsigned long long*)rq;
+        IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
+        iq_status r = conv_wgrad_tc(d, e, x, (long long*)G, tcws, st, &done, cell, &amax_done);
         if (r != IQ_OK) return r;
+        const int mode = gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2;
+        if (done && amax_done)
+            return requant_apply(G, IQ_I64, gn, s_in, 8, mode, seed, layer, step, 0, g, IQ_I8,
+                                 s_g, rq, st);
         if (done)
-            return requant_int(G, IQ_I64, gn, s_in, 8,
-                               gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2, seed, layer, step,
-                               0, g, IQ_I8, s_g, rq, st);
+            return requant_int(G, IQ_I64, gn, s_in, 8, mode, seed, layer, step, 0, g, IQ_I8,
+                               s_g, rq, st);
     }
+    IQ_CUDA_CHECK(cudaMemsetAsync(G, 0, sizeof(int64_t) * gn, st));
     cp.M = cp.Kg;
     cp.ncols = d->r * d->s * cp.Cg;
     int64_t tiles = ((cp.M + BM - 1) / BM) * ((cp.ncols + BN - 1) / BN) * cp.G;

@@ -1735,10 +1735,12 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     }
 }
 
-// G[i] += sum over the splits of their int32 partial sums (4 elements per thread)
+// G[i] = sum over the splits of their int32 partial sums (4 elements per thread), and
+// max |G| into *amax (zeroed by the caller)
 __global__ void k_split_sum(const int32_t* __restrict__ part, int ns, int64_t total4,
-                            long long* __restrict__ G) {
+                            long long* __restrict__ G, unsigned long long* __restrict__ amax) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    uint64_t m = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total4; i += stride) {
         long long a0 = 0, a1 = 0, a2 = 0, a3 = 0;
         for (int sp = 0; sp < ns; sp++) {
@@ -1746,14 +1748,18 @@ __global__ void k_split_sum(const int32_t* __restrict__ part, int ns, int64_t to
             a0 += v.x; a1 += v.y; a2 += v.z; a3 += v.w;
         }
         longlong2* g2 = reinterpret_cast<longlong2*>(G) + 2 * i;
-        const longlong2 o0 = g2[0], o1 = g2[1];
-        g2[0] = make_longlong2(o0.x + a0, o0.y + a1);
-        g2[1] = make_longlong2(o1.x + a2, o1.y + a3);
+        g2[0] = make_longlong2(a0, a1);
+        g2[1] = make_longlong2(a2, a3);
+        const uint64_t b0 = (uint64_t)(a0 < 0 ? -a0 : a0), b1 = (uint64_t)(a1 < 0 ? -a1 : a1);
+        const uint64_t b2 = (uint64_t)(a2 < 0 ? -a2 : a2), b3 = (uint64_t)(a3 < 0 ? -a3 : a3);
+        const uint64_t c0 = b0 > b1 ? b0 : b1, c1 = b2 > b3 ? b2 : b3;
+        const uint64_t c = c0 > c1 ? c0 : c1;
+        m = c > m ? c : m;
     }
+    m = warp_max_u64(m);
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(amax, (unsigned long long)m);
 }
 
-// int8 codes [npix][K] -> fp16 carriers [npix][Kp], Kp = K rounded up to 8 (zeros beyond K),
-// 8 codes per thread
 __global__ void k_codes_to_f16_pad(const int8_t* __restrict__ x, __half* __restrict__ xf,
                                    int64_t npix, int K, int Kp) {
     const int kg = Kp / 8;
@@ -1832,32 +1838,55 @@ std::mutex g_tc_status_mu;
 int* g_tc_status_ptr[256] = {};
 
 // int8 KRSC weights -> fp16 [K][kpad] (zero beyond R*S*C)
+// int8 KRSC weights -> fp16 [K][kpad] (zero beyond R*S*C): blocks (x, rows y, y + gridDim.y,
+// ...), each thread 8 consecutive columns (one 16-byte store)
 __global__ void k_widen_weights(const int8_t* __restrict__ w, __half* __restrict__ wf, int K,
                                 int kdim, int kpad) {
-    int64_t total = (int64_t)K * kpad;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        int k = (int)(i / kpad), j = (int)(i - (int64_t)k * kpad);
-        wf[i] = __int2half_rn(j < kdim ? (int)w[(int64_t)k * kdim + j] : 0);
+    const int j0 = (blockIdx.x * blockDim.x + threadIdx.x) * 8;
+    if (j0 >= kpad) return;
+    for (int k = blockIdx.y; k < K; k += gridDim.y) {
+        const int8_t* src = w + (int64_t)k * kdim;
+        uint32_t b[2] = {0u, 0u};
+#pragma unroll
+        for (int t = 0; t < 8; t++)
+            if (j0 + t < kdim) b[t >> 2] |= (uint32_t)(uint8_t)src[j0 + t] << (8 * (t & 3));
+        uint32_t o[4];
+        tc::i8x4_to_f16x4(b[0], o[0], o[1]);
+        tc::i8x4_to_f16x4(b[1], o[2], o[3]);
+        *reinterpret_cast<uint4*>(wf + (int64_t)k * kpad + j0) = make_uint4(o[0], o[1], o[2], o[3]);
     }
 }
 
-// data-gradient weights: w[K][R][S][C] -> [C][R][S][kc] flipped in r and s, fp16, for the
-// K-channel slice [kofs, kofs + kc); rows of kpad >= R*S*kc
+// data-gradient weights: wf[c][(r s) kc + k] = w[kofs + k][R-1-r][S-1-s][c] (zero for the
+// padding columns j >= R S kc), one 32 x 32 (k, c) transpose through shared memory per block
+// and tap: block (c tile, k tile, tap), 32 x 8 threads
 __global__ void k_widen_weights_dgrad(const int8_t* __restrict__ w, __half* __restrict__ wf, int K,
                                       int R, int S, int C, int kofs, int kc, int kpad) {
-    int64_t total = (int64_t)C * kpad;
-    const int kdim = R * S * kc;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        int c = (int)(i / kpad), j = (int)(i - (int64_t)c * kpad);
-        int v = 0;
-        if (j < kdim) {
-            int k = j % kc, rs = j / kc;
-            int r = rs / S, s = rs % S;
-            v = w[(((int64_t)(kofs + k) * R + (R - 1 - r)) * S + (S - 1 - s)) * C + c];
+    __shared__ int8_t tile[32][33];
+    const int c0 = blockIdx.x * 32, k0 = blockIdx.y * 32, tap = blockIdx.z;
+    const int r = tap / S, s = tap - r * S;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+#pragma unroll
+    for (int i = 0; i < 32; i += 8) {
+        const int k = k0 + ty + i, c = c0 + tx;
+        tile[ty + i][tx] = (k < kc && c < C)
+            ? w[(((int64_t)(kofs + k) * R + (R - 1 - r)) * S + (S - 1 - s)) * C + c] : (int8_t)0;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < 32; i += 8) {
+        const int c = c0 + ty + i, k = k0 + tx;
+        if (c < C && k < kc) wf[(int64_t)c * kpad + (int64_t)tap * kc + k] = __int2half_rn(tile[tx][ty + i]);
+    }
+    // the padding columns of row c (written by the first tap's blocks of the first k tile)
+    if (tap == 0 && blockIdx.y == 0) {
+        const int kdim = R * S * kc;
+#pragma unroll
+        for (int i = 0; i < 32; i += 8) {
+            const int c = c0 + ty + i;
+            if (c < C)
+                for (int j = kdim + tx; j < kpad; j += 32) wf[(int64_t)c * kpad + j] = __float2half(0.0f);
         }
-        wf[i] = __int2half_rn(v);
     }
 }
 
@@ -2194,8 +2223,9 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     __half* wf = reinterpret_cast<__half*>(wsb);
     int* err = tc_status_ptr();
     if (!err) return IQ_ERR_CUDA;
-    k_widen_weights<<<grid_for((int64_t)p.K * p.kpad), kThreads, 0, st>>>(w, wf, p.K, p.kdim,
-                                                                         p.kpad);
+    k_widen_weights<<<dim3((unsigned)((p.kpad / 8 + kThreads - 1) / kThreads),
+                           (unsigned)(p.K < 65535 ? p.K : 65535)),
+                      kThreads, 0, st>>>(w, wf, p.K, p.kdim, p.kpad);
     IQ_LAUNCH_CHECK();
     CUtensorMap map;
     iq_status r = encode_weights(wf, p.K, p.kpad, pick_bn(p.ncols), &map);
@@ -2307,7 +2337,8 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
     __half* ef = reinterpret_cast<__half*>(wsb + acts16_offset((size_t)d->c * p.kpad * 2));
     const bool ef_ok = ((int64_t)p.N * p.H * p.W * p.cstride) % 16 == 0;
     for (int sl = 0; sl < nsl; sl++) {
-        k_widen_weights_dgrad<<<grid_for((int64_t)d->c * p.kpad), kThreads, 0, st>>>(
+        k_widen_weights_dgrad<<<dim3((unsigned)((d->c + 31) / 32), (unsigned)((kc + 31) / 32),
+                                     (unsigned)(d->r * d->s)), dim3(32, 8), 0, st>>>(
             w, wf, d->k, d->r, d->s, d->c, sl * kc, kc, p.kpad);
         IQ_LAUNCH_CHECK();
         CUtensorMap map;
@@ -2442,8 +2473,10 @@ bool conv_wgrad_tc_supported(const iq_conv_desc* d) {
 
 // G (int64 KRSC, zeroed by the caller) += E^T im2col(x)
 iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
-                        void* ws, cudaStream_t st, bool* done) {
+                        void* ws, cudaStream_t st, bool* done, unsigned long long* amax,
+                        bool* amax_done) {
     *done = false;
+    *amax_done = false;
     if (tc_env_disabled() || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     int* err = tc_status_ptr();
@@ -2494,9 +2527,10 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         }
         if (r != IQ_OK) return r;
         const int64_t total4 = p.M * (int64_t)p.ncols / 4;
-        k_split_sum<<<grid_for(total4), kThreads, 0, st>>>(part, nsplit, total4, G);
+        k_split_sum<<<grid_for(total4), kThreads, 0, st>>>(part, nsplit, total4, G, amax);
         IQ_LAUNCH_CHECK();
         *done = true;
+        *amax_done = true;
         return IQ_OK;
     }
     if (!conv_wgrad_tc_supported(d)) return IQ_OK;
@@ -2517,6 +2551,7 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
     p.kb_per_split = (int)kbs;
     CUtensorMap dummy;
     memset(&dummy, 0, sizeof(dummy));
+    IQ_CUDA_CHECK(cudaMemsetAsync(G, 0, sizeof(long long) * (size_t)p.M * p.ncols, st));
     iq_status r = launch(dummy, p, nsplit, e, x, nullptr, G, nullptr, nullptr, nullptr, err, st);
     if (r == IQ_OK) *done = true;
     return r;

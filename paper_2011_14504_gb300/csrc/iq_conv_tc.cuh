@@ -25,10 +25,12 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
                         long long* out64, unsigned long long* s1, int* hi, int* lo, void* ws,
                         cudaStream_t st, bool* done);
 
-// Weight gradient: adds the exact int64 sums into G (KRSC, zeroed by the caller).
+// Weight gradient: writes the exact int64 sums to G (KRSC).  When *amax_done, max |G| has
+// also been folded into *amax (an atomicMax cell the caller zeroed).
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d);
 bool conv_wgrad_tc_supported(const iq_conv_desc* d);
 iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
-                        void* ws, cudaStream_t st, bool* done);
+                        void* ws, cudaStream_t st, bool* done, unsigned long long* amax,
+                        bool* amax_done);
 
 }  // namespace iq

@@ -103,6 +103,7 @@ struct RqParams {
     uint64_t M;
     UDiv div;      // by 2M (SQ) or by M (RQ)
     double s_out;
+    uint32_t R8;   // SQ with k = 8 and 128 < M <= 2^31: floor(2^39 / M), else 0
 };
 
 size_t requant_ws_bytes() { return 512; }
@@ -116,6 +117,8 @@ __global__ void k_rq_finalize(const unsigned long long* __restrict__ cell,
     p.M = M;
     bool rq = mode == IQ_MODE_RQ_GQ1 || mode == IQ_MODE_RQ_GQ2;
     p.div = make_udiv(M == 0 ? 1 : (rq ? M : 2 * M));
+    p.R8 = (!rq && k == 8 && M > 128 && M <= (uint64_t(1) << 31))
+               ? (uint32_t)((uint64_t(1) << 39) / M) : 0u;
     double Md = (double)M;
     if (mode == IQ_MODE_RQ_GQ2) p.s_out = ldexp(1.0, 1 - k);
     else p.s_out = M ? ldexp(__dmul_rn(s, Md), 1 - k) : ldexp(s, 1 - k);
@@ -133,12 +136,48 @@ __device__ __forceinline__ int64_t sq_code(int64_t v, const RqParams& p, int k, 
     return clamp64((int64_t)udiv(num, p.div) - (int64_t(1) << (k - 1)), -lim, lim);
 }
 
+// SQ with k = 8 for int32 codes and 128 < M <= 2^31, in 32-bit arithmetic: with u = v + M
+// in [0, 2M] the code is q - 128 for q = floor((256 u + M) / (2M)) = floor(128 u / M + 1/2).
+// t = floor(u R8 / 2^32), R8 = floor(2^39 / M), lies in [floor(128 u / M) - 1,
+// floor(128 u / M)], so q = t + [(2t + 1) M <= 256 u] + [(2t + 3) M <= 256 u] exactly (both
+// sides below 2^41).  Clipping to +-127 is q in [1, 255]; the code byte is q ^ 0x80.
+__device__ __forceinline__ uint32_t sq8_byte(int v, uint32_t M, uint32_t R8, int relu) {
+    if (relu && v < 0) v = 0;
+    const uint32_t u = (uint32_t)v + M;
+    const uint32_t t = __umulhi(u, R8);
+    const uint64_t rhs = (uint64_t)u << 8;
+    const uint64_t l1 = (uint64_t)(2 * t + 1) * M;
+    uint32_t q = t + (l1 <= rhs ? 1u : 0u) + (l1 + 2 * (uint64_t)M <= rhs ? 1u : 0u);
+    q = q < 1u ? 1u : (q > 255u ? 255u : q);
+    return q ^ 0x80u;
+}
+
+__device__ __forceinline__ uint32_t sq8_word(const int4& v, uint32_t M, uint32_t R8, int relu) {
+    return sq8_byte(v.x, M, R8, relu) | (sq8_byte(v.y, M, R8, relu) << 8) |
+           (sq8_byte(v.z, M, R8, relu) << 16) | (sq8_byte(v.w, M, R8, relu) << 24);
+}
+
 // int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores)
 __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int relu,
                               const RqParams* __restrict__ prm, uint32_t* __restrict__ out) {
     const RqParams p = *prm;
     const int64_t lim = qmax(k);
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    if (p.R8) {
+        // four 16-byte loads in flight per thread
+        const uint32_t M = (uint32_t)p.M;
+        for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
+             i += 4 * stride) {
+            int4 v[4];
+#pragma unroll
+            for (int j = 0; j < 4; j++)
+                v[j] = i + j * stride < n4 ? __ldg(q + i + j * stride) : make_int4(0, 0, 0, 0);
+#pragma unroll
+            for (int j = 0; j < 4; j++)
+                if (i + j * stride < n4) out[i + j * stride] = sq8_word(v[j], M, p.R8, relu);
+        }
+        return;
+    }
     // two 16-byte loads in flight per thread
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += 2 * stride) {
         const int64_t i2 = i + stride;
