@@ -1735,6 +1735,28 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     }
 }
 
+// G[k ncols_out + j] = sum over the splits of the partial sums [k][j] of rows of ncols_in
+// columns, j < ncols_out (the weight gradient computed over an im2col with padded columns),
+// and max |G| into *amax (zeroed by the caller)
+__global__ void k_split_sum_cols(const int32_t* __restrict__ part, int ns, int64_t rows,
+                                 int ncols_in, int ncols_out, long long* __restrict__ G,
+                                 unsigned long long* __restrict__ amax) {
+    const int64_t total = rows * ncols_out, slab = rows * ncols_in;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    uint64_t m = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+        const int64_t k = i / ncols_out;
+        const int64_t src = k * ncols_in + (i - k * ncols_out);
+        long long a = 0;
+        for (int sp = 0; sp < ns; sp++) a += __ldg(part + sp * slab + src);
+        G[i] = a;
+        const uint64_t b = (uint64_t)(a < 0 ? -a : a);
+        m = b > m ? b : m;
+    }
+    m = warp_max_u64(m);
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(amax, (unsigned long long)m);
+}
+
 // G[i] = sum over the splits of their int32 partial sums (4 elements per thread), and
 // max |G| into *amax (zeroed by the caller)
 __global__ void k_split_sum(const int32_t* __restrict__ part, int ns, int64_t total4,
@@ -1781,33 +1803,46 @@ __global__ void k_codes_to_f16_pad(const int8_t* __restrict__ x, __half* __restr
 
 // the im2col of a forward problem with few channels (C % 4 == 0) as fp16 [N P Q][kpad]:
 // column j = (r S + s) C + c (the widened weights' order), zeros for padding and
-// j >= R S C.  Block (output row pp, image n); a thread writes 4 columns (one tap, 4
-// channels: one 4-byte load, one 8-byte store) of one output pixel.
+// j >= R S C.  Blocks (pixel range, output row pp, image n); a thread writes 4 columns (one
+// tap, 4 channels: one 4-byte load, one 8-byte store) of several output pixels.
 __global__ void k_im2col_f16(const int8_t* __restrict__ x, TcP p, __half* __restrict__ A) {
-    const int g4 = p.kpad / 4;
+    // thread (g, y): columns 4g .. 4g + 3 (one tap, 4 channels) of the pixels q = y, y +
+    // blockDim.y, ... of output row blockIdx.y of image blockIdx.z; the tap is decoded once
+    const int j = 4 * threadIdx.x;
     const int pp = blockIdx.y, n = blockIdx.z;
-    const int per_row = p.Q * g4;
-    for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < per_row;
-         idx += gridDim.x * blockDim.x) {
-        const int qq = idx / g4, g = idx - (idx / g4) * g4;
-        const int j = 4 * g;
+    bool ok = j < p.kdim;
+    int dx = 0, c = 0, hh = 0;
+    if (ok) {
+        const int tap = j / p.C;
+        c = j - tap * p.C;
+        const int r = tap / p.S, sx = tap - r * p.S;
+        hh = pp * p.sh + r * p.dh - p.ph;
+        dx = sx * p.dw - p.pw;
+        ok = hh >= 0 && hh < p.H;
+    }
+    const int8_t* xrow = x + (((int64_t)n * p.H + (ok ? hh : 0)) * p.W) * p.cstride + p.cofs + c;
+    __half* arow = A + ((int64_t)n * p.P + pp) * p.Q * p.kpad + j;
+    for (int qq = blockIdx.x * blockDim.y + threadIdx.y; qq < p.Q; qq += gridDim.x * blockDim.y) {
+        const int ww = qq * p.sw + dx;
         uint32_t v = 0;
-        if (j < p.kdim) {
-            const int tap = j / p.C, c = j - (j / p.C) * p.C;
-            const int r = tap / p.S, sx = tap - (tap / p.S) * p.S;
-            const int hh = pp * p.sh + r * p.dh - p.ph, ww = qq * p.sw + sx * p.dw - p.pw;
-            if (hh >= 0 && hh < p.H && ww >= 0 && ww < p.W)
-                v = __ldg(reinterpret_cast<const uint32_t*>(
-                    x + (((int64_t)n * p.H + hh) * p.W + ww) * p.cstride + p.cofs + c));
-        }
+        if (ok && ww >= 0 && ww < p.W)
+            v = __ldg(reinterpret_cast<const uint32_t*>(xrow + (int64_t)ww * p.cstride));
         uint32_t o0, o1;
         tc::i8x4_to_f16x4(v, o0, o1);
-        const int64_t m = ((int64_t)n * p.P + pp) * p.Q + qq;
-        *reinterpret_cast<uint2*>(A + m * p.kpad + j) = make_uint2(o0, o1);
+        *reinterpret_cast<uint2*>(arow + (int64_t)qq * p.kpad) = make_uint2(o0, o1);
     }
 }
 
 // int8 codes [npix][cstride] -> exact fp16 carriers, 16 codes per thread
+// launch k_im2col_f16 for the geometry in p (kpad / 4 <= 128 column groups per pixel)
+void launch_im2col(const int8_t* x, const TcP& p, __half* A, cudaStream_t st) {
+    const int g4 = p.kpad / 4;
+    const int by = 256 / g4 > 0 ? 256 / g4 : 1;
+    dim3 block((unsigned)g4, (unsigned)by);
+    dim3 grid((unsigned)((p.Q + by - 1) / by), (unsigned)p.P, (unsigned)p.N);
+    k_im2col_f16<<<grid, block, 0, st>>>(x, p, A);
+}
+
 __global__ void k_codes_to_f16(const int8_t* __restrict__ x, __half* __restrict__ xf, int64_t n16) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += stride) {
@@ -2242,9 +2277,7 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
         TmaTile tt;
         const bool cm = cm_ok(q, &tt);
         if (cm || tma16_ok(q, &tt)) {
-            const int per_row = p.Q * (p.kpad / 4);
-            dim3 gi((unsigned)((per_row + kThreads - 1) / kThreads), (unsigned)p.P, (unsigned)p.N);
-            k_im2col_f16<<<gi, kThreads, 0, st>>>(x, p, xf);
+            launch_im2col(x, p, xf, st);
             IQ_LAUNCH_CHECK();
             if (cm) {
                 r = try_launch_c(wf, p.K, q, nullptr, xf, false, acc, s1, hi, lo, err, st, &used);
@@ -2412,17 +2445,42 @@ bool wgrad_tma_plan(const iq_conv_desc* d, TcP* p, TmaTile* t, int* nsplit) {
 
 // a reserved 256-byte slot, the fp16 carriers of the errors and of the input, and the per-split
 // int32 partial sums of the all-TMA path
+// The weight gradient of a convolution with few input channels (C % 4 == 0, C < 64) as that
+// of a 1 x 1 convolution over its fp16 im2col (kpad = R S C rounded up to 64 channels per
+// output pixel, the forward's im2col layout); false when the shape does not qualify.
+bool wgrad_im2col_desc(const iq_conv_desc* d, iq_conv_desc* d2) {
+    if (d->groups != 1 || d->c % 4 || d->c >= 64) return false;
+    const int kpad = (d->r * d->s * d->c + 63) / 64 * 64;
+    if (kpad > IM2COL_MAX_K) return false;
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    if (P > 65535 || d->n > 65535) return false;
+    *d2 = *d;
+    d2->h = P; d2->w = Q; d2->c = kpad;
+    d2->r = d2->s = 1;
+    d2->stride_h = d2->stride_w = 1;
+    d2->pad_h = d2->pad_w = 0;
+    d2->dil_h = d2->dil_w = 1;
+    return true;
+}
+
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d) {
     const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
     const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
     const size_t eb = ((size_t)d->n * P * Q * ((d->k + 63) / 64 * 64) * 2 + 255) / 256 * 256;
-    const size_t xb = ((size_t)d->n * d->h * d->w * d->c * 2 + 255) / 256 * 256;
+    size_t xb = ((size_t)d->n * d->h * d->w * d->c * 2 + 255) / 256 * 256;
     size_t parts = 0;
     TcP p;
     TmaTile t;
     int ns = 1;
-    if (d->c > 0 && d->k > 0 && wgrad_tma_plan(d, &p, &t, &ns))
+    iq_conv_desc d2;
+    if (d->c > 0 && d->k > 0 && wgrad_tma_plan(d, &p, &t, &ns)) {
         parts = (size_t)ns * d->k * d->r * d->s * d->c * 4;
+    } else if (d->c > 0 && d->k > 0 && wgrad_im2col_desc(d, &d2) &&
+               wgrad_tma_plan(&d2, &p, &t, &ns)) {
+        xb = ((size_t)d->n * P * Q * d2.c * 2 + 255) / 256 * 256;
+        parts = (size_t)ns * d->k * d2.c * 4;
+    }
     return 256 + eb + xb + parts + 512;
 }
 
@@ -2502,6 +2560,26 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
                encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256 + eb), p.N, p.H, p.W,
                                     p.C, t, p.sh, p.sw, nb, &xmap) == IQ_OK;
     }
+    // few input channels: the 1 x 1 problem over the im2col of x (pc: the conv's own geometry)
+    iq_conv_desc d2;
+    bool im2col = false;
+    TcP pc;
+    if (!maps && !tma16_disabled() && get_encode() && wgrad_im2col_desc(d, &d2) &&
+        wgrad_tma_plan(&d2, &p, &t, &nsplit)) {
+        Kp = (p.K + 63) / 64 * 64;
+        eb = ((size_t)p.npq * Kp * 2 + 255) / 256 * 256;
+        xb = ((size_t)p.npq * p.C * 2 + 255) / 256 * 256;
+        nb = p.C % 256 == 0 ? 4 : (p.C % 128 == 0 ? 2 : 1);
+        if (nb > pick_bn(p.ncols) / 64) nb = pick_bn(p.ncols) / 64;
+        maps = encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256), p.N, p.P, p.Q, Kp, t,
+                                    1, 1, 2, &emap) == IQ_OK &&
+               encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256 + eb), p.N, p.H, p.W,
+                                    p.C, t, 1, 1, nb, &xmap) == IQ_OK;
+        im2col = maps;
+        fill_geom(pc, d);
+        pc.kdim = d->r * d->s * d->c;
+        pc.kpad = p.C;
+    }
     if (maps) {
         // k-blocks: the pixel rectangles of every image; each split writes its own int32
         // partial sums, added into G afterwards
@@ -2517,7 +2595,10 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
                                                                               p.K, Kp);
         }
         IQ_LAUNCH_CHECK();
-        k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
+        if (im2col)
+            launch_im2col(x, pc, xf, st);
+        else
+            k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
         IQ_LAUNCH_CHECK();
         iq_status r = IQ_OK;
         switch (pick_bn(p.ncols)) {
@@ -2526,8 +2607,14 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
             default: r = launch_tw<256>(emap, xmap, p, t, nb, nsplit, part, err, st); break;
         }
         if (r != IQ_OK) return r;
-        const int64_t total4 = p.M * (int64_t)p.ncols / 4;
-        k_split_sum<<<grid_for(total4), kThreads, 0, st>>>(part, nsplit, total4, G, amax);
+        if (im2col) {
+            const int kdim = d->r * d->s * d->c;
+            k_split_sum_cols<<<grid_for(p.M * (int64_t)kdim), kThreads, 0, st>>>(
+                part, nsplit, p.M, p.ncols, kdim, G, amax);
+        } else {
+            const int64_t total4 = p.M * (int64_t)p.ncols / 4;
+            k_split_sum<<<grid_for(total4), kThreads, 0, st>>>(part, nsplit, total4, G, amax);
+        }
         IQ_LAUNCH_CHECK();
         *done = true;
         *amax_done = true;

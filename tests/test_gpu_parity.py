@@ -104,6 +104,28 @@ def test_requantize_sq_int32(relu):
     assert host(so)[0] == ws
 
 
+@pytest.mark.parametrize("relu", [False, True])
+@pytest.mark.parametrize("M", [128, 129, 255, 256 * 1000, 2 ** 30 + 3, 2 ** 31])
+def test_requantize_sq_int32_vector_path(relu, M):
+    # the 4-wide int32 -> int8 kernel (n % 4 == 0, aligned), across its 32-bit branch (M > 128)
+    # and the 64-bit one (M <= 128): random values, both extremes, and exact half-step ties
+    g = S.rng(M % 1000 + relu)
+    vals = [-M, M - 1 if M == 2 ** 31 else M, 0, 1, -1]
+    if M % 256 == 0:
+        vals += [(2 * k + 1) * M // 256 - M for k in range(0, 256, 5)]
+    q = np.concatenate([np.array(vals, np.int64),
+                        g.integers(-M, min(M, 2 ** 31 - 1) + 1, size=4000)])
+    q = q[: len(q) // 4 * 4].astype(np.int32)
+    assert np.abs(q.astype(np.int64)).max() == M
+    out = torch.empty(q.size, dtype=torch.int8, device=DEV)
+    so = dscal()
+    iq.iq_requantize(dev(q), dscal(2.0 ** -20), 8, iq.IQ_MODE_SQ_RELU if relu else iq.IQ_MODE_SQ,
+                     out, so)
+    want, ws = O.sq_int(q, 2.0 ** -20, 8, relu)
+    assert np.array_equal(host(out).astype(np.int32), want)
+    assert host(so)[0] == ws
+
+
 @pytest.mark.parametrize("mode,gq", [(iq.IQ_MODE_RQ_GQ1, 1), (iq.IQ_MODE_RQ_GQ2, 2)])
 def test_requantize_rq_int64(mode, gq):
     g = S.rng(4)
