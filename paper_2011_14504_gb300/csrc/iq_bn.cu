@@ -537,51 +537,93 @@ __device__ __forceinline__ void load4_e_a_x(int64_t v, const int8_t* ea, const i
     x[2] = (int)(int16_t)(xv.y & 0xffffu); x[3] = (int)(int16_t)(xv.y >> 16);
 }
 
+// Launch shape of the reduction passes of the backward: blocks of CG channel groups (4
+// channels each) x RL row lanes (CG RL = 256), grid (channel-group tiles, row tiles).  A warp
+// reads 4 CG consecutive channels of one row; the RL lanes of a channel group are combined
+// in shared memory, so each block adds one partial per channel to the global accumulators.
+struct RowGrid {
+    int cg, rl;
+    dim3 grid;
+};
+
+RowGrid row_grid(int64_t m, int32_t C4, int target_blocks = 152 * 8) {
+    RowGrid g;
+    g.cg = 32;
+    while (g.cg > 1 && g.cg > C4) g.cg >>= 1;
+    g.rl = kThreads / g.cg;
+    const int64_t bx = (C4 + g.cg - 1) / g.cg;
+    int64_t by = (m + g.rl - 1) / g.rl;
+    int64_t cap = target_blocks / bx;
+    if (cap < 1) cap = 1;
+    if (by > cap) by = cap;
+    if (by > 65535) by = 65535;
+    g.grid = dim3((unsigned)bx, (unsigned)by);
+    return g;
+}
+
+// sum e_y and sum e_y X per channel (e_y = e_a [A > 0]), max |e_y gamma|
 __global__ void __launch_bounds__(kThreads) k_bnb_pass1(const int8_t* __restrict__ ea,
                                                         const int8_t* __restrict__ a,
                                                         const int16_t* __restrict__ X,
                                                         const int32_t* __restrict__ gam,
-                                                        int64_t m, int32_t C, BnBwd w) {
-    __shared__ unsigned long long sh_b[1024], sh_g[1024];
+                                                        int64_t m, int32_t C, int CG, BnBwd w) {
+    __shared__ long long sh_b[kThreads * 4], sh_g[kThreads * 4];
     const int C4 = C >> 2;
-    const bool use_sh = C <= 1024;
-    if (use_sh)
-        for (int c = threadIdx.x; c < C; c += blockDim.x) { sh_b[c] = 0; sh_g[c] = 0; }
-    __syncthreads();
-    const int64_t T = (int64_t)gridDim.x * blockDim.x;
-    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int g = (int)(t % C4);
-    const int64_t rstride = T / C4;
-    int gm[4];
+    const int cg = threadIdx.x % CG, rl = threadIdx.x / CG, RL = blockDim.x / CG;
+    const int g = blockIdx.x * CG + cg;
+    const bool act = g < C4;
+    int gm[4] = {0, 0, 0, 0};
+    if (act) {
 #pragma unroll
-    for (int j = 0; j < 4; j++) gm[j] = gam[4 * g + j];
+        for (int j = 0; j < 4; j++) gm[j] = gam[4 * g + j];
+    }
     long long sb[4] = {0, 0, 0, 0}, sg[4] = {0, 0, 0, 0};
     uint32_t zm = 0;
-    for (int64_t r = t / C4; r < m; r += rstride) {
-        int e[4], am[4], x[4];
-        load4_e_a_x(r * C4 + g, ea, a, X, e, am, x);
+    const int64_t step = (int64_t)gridDim.y * RL;
+    if (act) {
+        int64_t r = (int64_t)blockIdx.y * RL + rl;
+        // two rows per iteration: both rows' loads are in flight together
+        for (; r + step < m; r += 2 * step) {
+            int e0[4], a0[4], x0[4], e1[4], a1[4], x1[4];
+            load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
+            load4_e_a_x((r + step) * C4 + g, ea, a, X, e1, a1, x1);
 #pragma unroll
-        for (int j = 0; j < 4; j++) {
-            int ey = am[j] > 0 ? e[j] : 0;
-            sb[j] += ey;
-            sg[j] += (long long)(ey * x[j]);     // |ey x| < 2^22
-            int z = ey * gm[j];
-            zm = max(zm, (uint32_t)(z < 0 ? -z : z));
+            for (int j = 0; j < 4; j++) {
+                const int ey0 = a0[j] > 0 ? e0[j] : 0, ey1 = a1[j] > 0 ? e1[j] : 0;
+                sb[j] += ey0 + ey1;
+                sg[j] += (long long)(ey0 * x0[j]) + (long long)(ey1 * x1[j]);   // |ey X| < 2^22
+                const int z0 = ey0 * gm[j], z1 = ey1 * gm[j];
+                zm = max(zm, max((uint32_t)abs(z0), (uint32_t)abs(z1)));
+            }
+        }
+        if (r < m) {
+            int e0[4], a0[4], x0[4];
+            load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                const int ey0 = a0[j] > 0 ? e0[j] : 0;
+                sb[j] += ey0;
+                sg[j] += (long long)(ey0 * x0[j]);
+                zm = max(zm, (uint32_t)abs(ey0 * gm[j]));
+            }
         }
     }
     zm = warp_max_u32(zm);
     if ((threadIdx.x & 31) == 0 && zm) atomicMax(w.zmax, zm);
 #pragma unroll
     for (int j = 0; j < 4; j++) {
-        int c = 4 * g + j;
-        if (use_sh) { atomicAdd(&sh_b[c], (unsigned long long)sb[j]); atomicAdd(&sh_g[c], (unsigned long long)sg[j]); }
-        else { atomicAdd(&w.sb[c], (unsigned long long)sb[j]); atomicAdd(&w.sg[c], (unsigned long long)sg[j]); }
+        sh_b[rl * CG * 4 + 4 * cg + j] = sb[j];
+        sh_g[rl * CG * 4 + 4 * cg + j] = sg[j];
     }
-    if (use_sh) {
-        __syncthreads();
-        for (int c = threadIdx.x; c < C; c += blockDim.x) {
-            atomicAdd(&w.sb[c], sh_b[c]);
-            atomicAdd(&w.sg[c], sh_g[c]);
+    __syncthreads();
+    const int col = threadIdx.x;                 // one channel of the block's 4 CG
+    if (col < CG * 4) {
+        const int c = 4 * blockIdx.x * CG + col;
+        if (c < C) {
+            long long tb = 0, tg = 0;
+            for (int i = 0; i < RL; i++) { tb += sh_b[i * CG * 4 + col]; tg += sh_g[i * CG * 4 + col]; }
+            atomicAdd(&w.sb[c], (unsigned long long)tb);
+            atomicAdd(&w.sg[c], (unsigned long long)tg);
         }
     }
 }
@@ -618,78 +660,102 @@ __device__ __forceinline__ int e2_code(int z, const E2Div& d, int k) {
     return (int)clamp64(c, -qmax(k), qmax(k));
 }
 
-__global__ void __launch_bounds__(kThreads) k_bnb_pass2(const int8_t* __restrict__ ea,
+// E_2 = SQ_kE2(e_y gamma): per channel sum E_2, sum E_2 X, sum sign X, and the extremes of
+// E_2 per sign class of X (-1, 0, +1).  The extremes travel packed as (max, -min) int16
+// pairs (|E_2| <= 2^15 - 1), one __vmaxs2 per class.
+__global__ void __launch_bounds__(kThreads, 3) k_bnb_pass2(const int8_t* __restrict__ ea,
                                                         const int8_t* __restrict__ a,
                                                         const int16_t* __restrict__ X,
                                                         const int32_t* __restrict__ gam,
-                                                        int64_t m, int32_t C, int k_e2, BnBwd w) {
-    __shared__ unsigned long long sh_e[512], sh_x[512], sh_s[512];
-    __shared__ int sh_mn[3 * 512], sh_mx[3 * 512];
+                                                        int64_t m, int32_t C, int CG, int k_e2,
+                                                        BnBwd w) {
+    __shared__ long long sh_e[kThreads * 4], sh_x[kThreads * 4];
+    __shared__ int sh_s[kThreads * 4];
+    __shared__ uint32_t sh_p[3][kThreads * 4];
     const int C4 = C >> 2;
-    const bool use_sh = C <= 512;
-    if (use_sh)
-        for (int c = threadIdx.x; c < C; c += blockDim.x) {
-            sh_e[c] = 0; sh_x[c] = 0; sh_s[c] = 0;
-            for (int j = 0; j < 3; j++) { sh_mn[3 * c + j] = INT_MAX; sh_mx[3 * c + j] = INT_MIN; }
-        }
-    __syncthreads();
+    const int cg = threadIdx.x % CG, rl = threadIdx.x / CG, RL = blockDim.x / CG;
+    const int g = blockIdx.x * CG + cg;
+    const bool act = g < C4;
     const E2Div d = *w.e2div;
-    const int64_t T = (int64_t)gridDim.x * blockDim.x;
-    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int g = (int)(t % C4);
-    const int64_t rstride = T / C4;
-    int gm[4];
+    constexpr uint32_t kEmpty = 0x80008000u;      // (-32768, -32768): no element yet
+    int gm[4] = {0, 0, 0, 0};
+    if (act) {
 #pragma unroll
-    for (int j = 0; j < 4; j++) gm[j] = gam[4 * g + j];
-    long long se[4] = {0, 0, 0, 0}, sx[4] = {0, 0, 0, 0}, ss[4] = {0, 0, 0, 0};
-    int mn[4][3], mx[4][3];
+        for (int j = 0; j < 4; j++) gm[j] = gam[4 * g + j];
+    }
+    long long se64[4] = {0, 0, 0, 0}, sx[4] = {0, 0, 0, 0};
+    int ss[4] = {0, 0, 0, 0};
+    uint32_t pk[4][3];
 #pragma unroll
     for (int j = 0; j < 4; j++)
 #pragma unroll
-        for (int q = 0; q < 3; q++) { mn[j][q] = INT_MAX; mx[j][q] = INT_MIN; }
-    for (int64_t r = t / C4; r < m; r += rstride) {
-        int e[4], am[4], x[4];
-        load4_e_a_x(r * C4 + g, ea, a, X, e, am, x);
+        for (int q = 0; q < 3; q++) pk[j][q] = kEmpty;
+    const int64_t step = (int64_t)gridDim.y * RL;
+    if (act) {
+        int64_t r = (int64_t)blockIdx.y * RL + rl;
+        while (r < m) {
+            // int32 partial sums of E_2 over at most 2^15 rows (|E_2| < 2^15)
+            int se[4] = {0, 0, 0, 0};
+            for (int it = 0; it < 32768 && r < m; it++, r += step) {
+                int e0[4], a0[4], x0[4];
+                load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
 #pragma unroll
-        for (int j = 0; j < 4; j++) {
-            int ey = am[j] > 0 ? e[j] : 0;
-            int e2 = e2_code(ey * gm[j], d, k_e2);
-            int sgn = (x[j] > 0) - (x[j] < 0);
-            se[j] += e2;
-            sx[j] += (long long)(e2 * x[j]);     // |E_2 X| < 2^30
-            ss[j] += sgn;
-            int q = sgn + 1;
+                for (int j = 0; j < 4; j++) {
+                    const int ey = a0[j] > 0 ? e0[j] : 0;
+                    const int e2 = e2_code(ey * gm[j], d, k_e2);
+                    const int sgn = (x0[j] > 0) - (x0[j] < 0);
+                    se[j] += e2;
+                    sx[j] += (long long)(e2 * x0[j]);     // |E_2 X| < 2^30
+                    ss[j] += sgn;
+                    const uint32_t cand = ((uint32_t)e2 & 0xffffu) | ((uint32_t)(-e2) << 16);
+                    if (sgn < 0) pk[j][0] = __vmaxs2(pk[j][0], cand);
+                    else if (sgn == 0) pk[j][1] = __vmaxs2(pk[j][1], cand);
+                    else pk[j][2] = __vmaxs2(pk[j][2], cand);
+                }
+            }
 #pragma unroll
-            for (int qq = 0; qq < 3; qq++)
-                if (qq == q) { mn[j][qq] = min(mn[j][qq], e2); mx[j][qq] = max(mx[j][qq], e2); }
+            for (int j = 0; j < 4; j++) se64[j] += se[j];
         }
     }
 #pragma unroll
     for (int j = 0; j < 4; j++) {
-        int c = 4 * g + j;
-        if (use_sh) {
-            atomicAdd(&sh_e[c], (unsigned long long)se[j]);
-            atomicAdd(&sh_x[c], (unsigned long long)sx[j]);
-            atomicAdd(&sh_s[c], (unsigned long long)ss[j]);
-            for (int q = 0; q < 3; q++) { atomicMin(&sh_mn[3 * c + q], mn[j][q]); atomicMax(&sh_mx[3 * c + q], mx[j][q]); }
-        } else {
-            atomicAdd(&w.se[c], (unsigned long long)se[j]);
-            atomicAdd(&w.sex[c], (unsigned long long)sx[j]);
-            atomicAdd(&w.ss[c], (unsigned long long)ss[j]);
-            for (int q = 0; q < 3; q++) { atomicMin(&w.emin[3 * c + q], mn[j][q]); atomicMax(&w.emax[3 * c + q], mx[j][q]); }
-        }
+        const int i = rl * CG * 4 + 4 * cg + j;
+        sh_e[i] = se64[j];
+        sh_x[i] = sx[j];
+        sh_s[i] = ss[j];
+#pragma unroll
+        for (int q = 0; q < 3; q++) sh_p[q][i] = pk[j][q];
     }
-    if (use_sh) {
-        __syncthreads();
-        for (int c = threadIdx.x; c < C; c += blockDim.x) {
-            atomicAdd(&w.se[c], sh_e[c]);
-            atomicAdd(&w.sex[c], sh_x[c]);
-            atomicAdd(&w.ss[c], sh_s[c]);
-            for (int q = 0; q < 3; q++) { atomicMin(&w.emin[3 * c + q], sh_mn[3 * c + q]); atomicMax(&w.emax[3 * c + q], sh_mx[3 * c + q]); }
+    __syncthreads();
+    const int col = threadIdx.x;
+    if (col < CG * 4) {
+        const int c = 4 * blockIdx.x * CG + col;
+        if (c < C) {
+            long long te = 0, tx = 0;
+            long long ts = 0;
+            uint32_t tp[3] = {kEmpty, kEmpty, kEmpty};
+            for (int i = 0; i < RL; i++) {
+                const int k = i * CG * 4 + col;
+                te += sh_e[k];
+                tx += sh_x[k];
+                ts += sh_s[k];
+#pragma unroll
+                for (int q = 0; q < 3; q++) tp[q] = __vmaxs2(tp[q], sh_p[q][k]);
+            }
+            atomicAdd(&w.se[c], (unsigned long long)te);
+            atomicAdd(&w.sex[c], (unsigned long long)tx);
+            atomicAdd(&w.ss[c], (unsigned long long)ts);
+#pragma unroll
+            for (int q = 0; q < 3; q++) {
+                if (tp[q] == kEmpty) continue;
+                const int hi = (int)(int16_t)(tp[q] & 0xffffu);
+                const int lo = -(int)(int16_t)(tp[q] >> 16);
+                atomicMin(&w.emin[3 * c + q], lo);
+                atomicMax(&w.emax[3 * c + q], hi);
+            }
         }
     }
 }
-
 // Per channel (oracle order): gx = (SEX s_x)/m; kap = -gx; lam = gx (SS/m) - SE/m;
 // w = s_e2 / ((c_sigma + 1) sg_step); d x = w ((E_2 + kap sgn) + lam).  Three launches of
 // C/64 blocks: M = max |d x| at the extremes of each sign class (red[0]), then the bound of
@@ -863,12 +929,12 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     BnBwd w = bnb_carve(cur, c);
     k_bnb_init<<<(c + 255) / 256, 256, 0, st>>>(w, c);
     IQ_LAUNCH_CHECK();
-    ChanGrid g = chan_grid(m, c / 4);
-    k_bnb_pass1<<<g.blocks, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, w);
+    RowGrid rg = row_grid(m, c / 4);
+    k_bnb_pass1<<<rg.grid, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, rg.cg, w);
     IQ_LAUNCH_CHECK();
     k_bnb_fin1<<<1, 1, 0, st>>>(w, s_e, b.k_gamma, k_e2);
     IQ_LAUNCH_CHECK();
-    k_bnb_pass2<<<g.blocks, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, k_e2, w);
+    k_bnb_pass2<<<rg.grid, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, rg.cg, k_e2, w);
     IQ_LAUNCH_CHECK();
     const int fb = (c + kFinThreads - 1) / kFinThreads;
     k_bnb_fin2a<<<fb, kFinThreads, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma);
