@@ -171,12 +171,18 @@ iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_
  *   bn_codes  out device int32[2k]: mu_q codes then sigma_q codes (bn only, may be NULL)
  *   bn_scales out device double[IQ_BN_SCALES] (bn only, may be NULL)
  *   acc_out   optional out int32 [n][p][q][k]: the raw accumulators
+ *   x_f16     optional out fp16 [n][h][w][c] (16-byte aligned, n h w c % 16 == 0, else
+ *             IQ_ERR_INVALID_ARG): the exact fp16 copy of the codes x that the tensor-core
+ *             kernels read (every int8 code is exact in fp16).  When given it is written first
+ *             and the kernels read it; keep it for iq_conv_wgrad of the same layer, which then
+ *             skips its own conversion of x.  (The paper has no counterpart: it is the
+ *             operand format of this implementation's tensor-core path.)
  * Returns IQ_ERR_OVERFLOW_RISK when (c/groups) r s 127^2 >= 2^31. */
 iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
                       const int8_t* w, const int32_t* gamma, const int32_t* beta,
                       const iq_bn_bits* bits, int use_bn, int relu, int8_t* a, double* s_a,
                       int16_t* xhat, int32_t* bn_codes, double* bn_scales, int32_t* acc_out,
-                      void* ws, size_t ws_bytes, iq_stream stream);
+                      void* x_f16, void* ws, size_t ws_bytes, iq_stream stream);
 
 /* iq_conv_dgrad -- error of the layer input (Sec. 3.3.1, Eq. (EQ)):
  * dx = conv_transpose(e, w) in exact int32, then E_1 = SQ(dx, 8).
@@ -184,10 +190,12 @@ iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
  *   w    int8 KRSC forward weights (scale 2^-7)
  *   dx   out int8 NHWC [n][h][w][c]; s_dx out device double = (s_e 2^-7 M) 2^-7
  *   acc_out optional out int32 [n][h][w][c]; must be NULL when (k/groups) r s 127^2 >= 2^31,
- *           where the sums are accumulated in int64 (IQ_ERR_UNSUPPORTED otherwise) */
+ *           where the sums are accumulated in int64 (IQ_ERR_UNSUPPORTED otherwise)
+ *   e_f16   optional out fp16 [n][p][q][k], as x_f16 of iq_conv_fwd for the errors e: written
+ *           first and read by the kernels; pass it to iq_conv_wgrad of the same layer */
 iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
-                        const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out, void* ws,
-                        size_t ws_bytes, iq_stream stream);
+                        const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
+                        void* e_f16, void* ws, size_t ws_bytes, iq_stream stream);
 
 /* iq_conv_wgrad -- weight gradient and its quantization (Sec. 3.3.2):
  * G[k][r][s][c] = sum_{n,p,q} e[n,p,q,k] x[n, h(p,r), w(q,s), c] in exact int64, then
@@ -196,11 +204,15 @@ iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_
  *   x, s_x  the forward input codes and their scale (s_G = s_e s_x)
  *   seed, layer, step  Philox key/counter words of the stochastic rounding (tag 0)
  *   g       out int8 KRSC gradient codes;  s_g out device double
- *   g_acc_out optional out int64 KRSC: the exact sums */
+ *   g_acc_out optional out int64 KRSC: the exact sums
+ *   e_f16, x_f16  optional fp16 copies of e and x written by iq_conv_dgrad (e_f16) and
+ *           iq_conv_fwd (x_f16) for these same codes (16-byte aligned); used instead of
+ *           converting e and x again.  Results are undefined if they do not hold e and x. */
 iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
                         const int8_t* x, const double* s_x, int gq_mode, uint64_t seed,
                         uint64_t layer, uint64_t step, int8_t* g, double* s_g,
-                        int64_t* g_acc_out, void* ws, size_t ws_bytes, iq_stream stream);
+                        int64_t* g_acc_out, const void* e_f16, const void* x_f16, void* ws,
+                        size_t ws_bytes, iq_stream stream);
 
 /* iq_bn_int_fwd -- quantized L1BN + ReLU + Q_A on int32 accumulators acc[m][c] with
  * scale s_acc (Sec. 3.2.2, Eqs. (BN2),(BN4),(BN5), QBN block, Eq. (AQ1)):

@@ -38,6 +38,30 @@ ChanGrid chan_grid(int64_t m, int32_t C4, int max_blocks = 152 * 8) {
     return g;
 }
 
+// Launch shape of the per-channel reduction passes (L1 deviation, backward sums): blocks of CG channel groups (4
+// channels each) x RL row lanes (CG RL = 256), grid (channel-group tiles, row tiles).  A warp
+// reads 4 CG consecutive channels of one row; the RL lanes of a channel group are combined
+// in shared memory, so each block adds one partial per channel to the global accumulators.
+struct RowGrid {
+    int cg, rl;
+    dim3 grid;
+};
+
+RowGrid row_grid(int64_t m, int32_t C4, int target_blocks = 152 * 8) {
+    RowGrid g;
+    g.cg = 32;
+    while (g.cg > 1 && g.cg > C4) g.cg >>= 1;
+    g.rl = kThreads / g.cg;
+    const int64_t bx = (C4 + g.cg - 1) / g.cg;
+    int64_t by = (m + g.rl - 1) / g.rl;
+    int64_t cap = target_blocks / bx;
+    if (cap < 1) cap = 1;
+    if (by > cap) by = cap;
+    if (by > 65535) by = 65535;
+    g.grid = dim3((unsigned)bx, (unsigned)by);
+    return g;
+}
+
 __device__ __forceinline__ void unpack4_i8(int v, int out[4]) {
 #pragma unroll
     for (int j = 0; j < 4; j++) out[j] = (int)(int8_t)(v >> (8 * j));
@@ -152,43 +176,55 @@ __device__ __forceinline__ int64_t floordiv_i64(int64_t a, int64_t b) {
 }
 
 __global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__ acc, int64_t m,
-                                                     int32_t C, BnStats s) {
-    __shared__ unsigned long long sh_d[1024], sh_n[1024];
+                                                     int32_t C, int CG, BnStats s) {
+    __shared__ unsigned long long sh_d[kThreads * 4], sh_n[kThreads * 4];
     const int C4 = C >> 2;
-    const bool use_sh = C <= 1024;
-    if (use_sh)
-        for (int c = threadIdx.x; c < C; c += blockDim.x) { sh_d[c] = 0; sh_n[c] = 0; }
-    __syncthreads();
-    const int64_t T = (int64_t)gridDim.x * blockDim.x;
-    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int g = (int)(t % C4);
-    const int64_t rstride = T / C4;
-    int64_t f[4];
+    const int cg = threadIdx.x % CG, rl = threadIdx.x / CG, RL = blockDim.x / CG;
+    const int g = blockIdx.x * CG + cg;
+    const bool act = g < C4;
+    int64_t f[4] = {0, 0, 0, 0};
+    if (act) {
 #pragma unroll
-    for (int j = 0; j < 4; j++) f[j] = floordiv_i64((int64_t)s.s1[4 * g + j], m);
+        for (int j = 0; j < 4; j++) f[j] = floordiv_i64((int64_t)s.s1[4 * g + j], m);
+    }
     unsigned long long d[4] = {0, 0, 0, 0}, n[4] = {0, 0, 0, 0};
     const int4* a4 = reinterpret_cast<const int4*>(acc);
-    for (int64_t r = t / C4; r < m; r += rstride) {
-        int4 v = a4[r * C4 + g];
-        int vs[4] = {v.x, v.y, v.z, v.w};
+    const int64_t step = (int64_t)gridDim.y * RL;
+    if (act) {
+        int64_t r = (int64_t)blockIdx.y * RL + rl;
+        // two rows per iteration: both loads in flight together
+        for (; r < m; r += 2 * step) {
+            const bool two = r + step < m;
+            const int4 v0 = a4[r * C4 + g];
+            const int4 v1 = two ? a4[(r + step) * C4 + g] : make_int4(0, 0, 0, 0);
+            const int vs0[4] = {v0.x, v0.y, v0.z, v0.w}, vs1[4] = {v1.x, v1.y, v1.z, v1.w};
 #pragma unroll
-        for (int j = 0; j < 4; j++) {
-            int64_t dv = (int64_t)vs[j] - f[j];
-            d[j] += (unsigned long long)(dv < 0 ? -dv : dv);
-            n[j] += dv > 0;
+            for (int j = 0; j < 4; j++) {
+                const int64_t dv0 = (int64_t)vs0[j] - f[j];
+                d[j] += (unsigned long long)(dv0 < 0 ? -dv0 : dv0);
+                n[j] += dv0 > 0;
+                if (two) {
+                    const int64_t dv1 = (int64_t)vs1[j] - f[j];
+                    d[j] += (unsigned long long)(dv1 < 0 ? -dv1 : dv1);
+                    n[j] += dv1 > 0;
+                }
+            }
         }
     }
 #pragma unroll
     for (int j = 0; j < 4; j++) {
-        int c = 4 * g + j;
-        if (use_sh) { atomicAdd(&sh_d[c], d[j]); atomicAdd(&sh_n[c], n[j]); }
-        else { atomicAdd(&s.dev[c], d[j]); atomicAdd(&s.ngt[c], n[j]); }
+        sh_d[rl * CG * 4 + 4 * cg + j] = d[j];
+        sh_n[rl * CG * 4 + 4 * cg + j] = n[j];
     }
-    if (use_sh) {
-        __syncthreads();
-        for (int c = threadIdx.x; c < C; c += blockDim.x) {
-            atomicAdd(&s.dev[c], sh_d[c]);
-            atomicAdd(&s.ngt[c], sh_n[c]);
+    __syncthreads();
+    const int col = threadIdx.x;
+    if (col < CG * 4) {
+        const int c = 4 * blockIdx.x * CG + col;
+        if (c < C) {
+            unsigned long long td = 0, tn = 0;
+            for (int i = 0; i < RL; i++) { td += sh_d[i * CG * 4 + col]; tn += sh_n[i * CG * 4 + col]; }
+            atomicAdd(&s.dev[c], td);
+            atomicAdd(&s.ngt[c], tn);
         }
     }
 }
@@ -432,8 +468,8 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
                              const BnStats& s, int16_t* xhat, int8_t* a, double* s_a,
                              int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
                              cudaStream_t st) {
-    ChanGrid g = chan_grid(m, C / 4);
-    k_bn_dev<<<g.blocks, kThreads, 0, st>>>(acc, m, C, s);
+    RowGrid rg = row_grid(m, C / 4);
+    k_bn_dev<<<rg.grid, kThreads, 0, st>>>(acc, m, C, rg.cg, s);
     IQ_LAUNCH_CHECK();
     const int fb = (C + kFinThreads - 1) / kFinThreads;
     k_bn_fin1<<<fb, kFinThreads, 0, st>>>(s, m, C, s_acc, b);
@@ -535,30 +571,6 @@ __device__ __forceinline__ void load4_e_a_x(int64_t v, const int8_t* ea, const i
     uint2 xv = reinterpret_cast<const uint2*>(X)[v];
     x[0] = (int)(int16_t)(xv.x & 0xffffu); x[1] = (int)(int16_t)(xv.x >> 16);
     x[2] = (int)(int16_t)(xv.y & 0xffffu); x[3] = (int)(int16_t)(xv.y >> 16);
-}
-
-// Launch shape of the reduction passes of the backward: blocks of CG channel groups (4
-// channels each) x RL row lanes (CG RL = 256), grid (channel-group tiles, row tiles).  A warp
-// reads 4 CG consecutive channels of one row; the RL lanes of a channel group are combined
-// in shared memory, so each block adds one partial per channel to the global accumulators.
-struct RowGrid {
-    int cg, rl;
-    dim3 grid;
-};
-
-RowGrid row_grid(int64_t m, int32_t C4, int target_blocks = 152 * 8) {
-    RowGrid g;
-    g.cg = 32;
-    while (g.cg > 1 && g.cg > C4) g.cg >>= 1;
-    g.rl = kThreads / g.cg;
-    const int64_t bx = (C4 + g.cg - 1) / g.cg;
-    int64_t by = (m + g.rl - 1) / g.rl;
-    int64_t cap = target_blocks / bx;
-    if (cap < 1) cap = 1;
-    if (by > cap) by = cap;
-    if (by > 65535) by = 65535;
-    g.grid = dim3((unsigned)bx, (unsigned)by);
-    return g;
 }
 
 // sum e_y and sum e_y X per channel (e_y = e_a [A > 0]), max |e_y gamma|

@@ -450,8 +450,11 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
                                  const int8_t* w, const int32_t* gamma, const int32_t* beta,
                                  const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
                                  double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
-                                 int32_t* acc_out, void* ws, size_t ws_bytes, iq_stream stream) {
+                                 int32_t* acc_out, void* x_f16, void* ws, size_t ws_bytes,
+                                 iq_stream stream) {
     if (!desc_ok(d) || !x || !s_x || !w || !a || !s_a) return IQ_ERR_INVALID_ARG;
+    const int64_t nx = (int64_t)d->n * d->h * d->w * d->c;
+    if (x_f16 && (nx % 16 || (((uintptr_t)x | (uintptr_t)x_f16) & 15))) return IQ_ERR_INVALID_ARG;
     if (crs_overflow(d)) return IQ_ERR_OVERFLOW_RISK;
     iq_bn_bits b = bn_bits_or_default(bits);
     if (use_bn) {
@@ -475,7 +478,12 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     k_scale_mul_pow2<<<1, 1, 0, st>>>(s_x, -7, L.s_acc);  // s_acc = s_x * 2^-7 (W_q step)
     IQ_LAUNCH_CHECK();
     bool done = false;
-    r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done);
+    if (x_f16) {
+        r = codes_to_f16(x, (__half*)x_f16, nx, st);
+        if (r != IQ_OK) return r;
+    }
+    r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done,
+                    (const __half*)x_f16);
     if (r != IQ_OK) return r;
     if (!done) {
         dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
@@ -497,7 +505,7 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
 
 extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
                                    const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
-                                   void* ws, size_t ws_bytes, iq_stream stream) {
+                                   void* e_f16, void* ws, size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d) || !e || !s_e || !w || !dx || !s_dx) return IQ_ERR_INVALID_ARG;
     const bool wide = dgrad_wide(d);
     if (wide && acc_out) return IQ_ERR_UNSUPPORTED;   // the sums need 64 bits: no int32 copy
@@ -520,6 +528,11 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, -7, s_in);
     IQ_LAUNCH_CHECK();
     int32_t* acc = acc_out ? acc_out : reinterpret_cast<int32_t*>(accw);
+    if (e_f16) {
+        const int64_t ne = (int64_t)d->n * cp.P * cp.Q * d->k;
+        iq_status r0 = codes_to_f16(e, (__half*)e_f16, ne, st);
+        if (r0 != IQ_OK) return r0;
+    }
     // tensor-core path: stride 1, as a forward pass over the errors
     if (conv_dgrad_tc_supported(d)) {
         bool done = false;
@@ -527,7 +540,7 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
         if (wide) {
             IQ_CUDA_CHECK(cudaMemsetAsync(accw, 0, sizeof(int64_t) * total, st));
             r = conv_dgrad_tc(d, e, w, nullptr, (long long*)accw, nullptr, nullptr, nullptr, tcws,
-                              st, &done);
+                              st, &done, (const __half*)e_f16);
             if (r != IQ_OK) return r;
             if (done)
                 return requant_int(accw, IQ_I64, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
@@ -535,7 +548,8 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
         } else {
             r = bn_stats_init(stats, d->c, st);
             if (r != IQ_OK) return r;
-            r = conv_dgrad_tc(d, e, w, acc, nullptr, stats.s1, stats.hi, stats.lo, tcws, st, &done);
+            r = conv_dgrad_tc(d, e, w, acc, nullptr, stats.s1, stats.hi, stats.lo, tcws, st, &done,
+                              (const __half*)e_f16);
             if (r != IQ_OK) return r;
             if (done) {
                 IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
@@ -571,8 +585,9 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
 extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
                                    const int8_t* x, const double* s_x, int gq_mode, uint64_t seed,
                                    uint64_t layer, uint64_t step, int8_t* g, double* s_g,
-                                   int64_t* g_acc_out, void* ws, size_t ws_bytes,
-                                   iq_stream stream) {
+                                   int64_t* g_acc_out, const void* e_f16, const void* x_f16,
+                                   void* ws, size_t ws_bytes, iq_stream stream) {
+    if ((((uintptr_t)e_f16 | (uintptr_t)x_f16) & 15)) return IQ_ERR_INVALID_ARG;
     if (!desc_ok(d) || !e || !s_e || !x || !s_x || !g || !s_g) return IQ_ERR_INVALID_ARG;
     if (gq_mode != 1 && gq_mode != 2) return IQ_ERR_INVALID_ARG;
     size_t need = 0;
@@ -597,7 +612,8 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
         bool done = false, amax_done = false;
         unsigned long long* cell = (unsigned long long*)rq;
         IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
-        iq_status r = conv_wgrad_tc(d, e, x, (long long*)G, tcws, st, &done, cell, &amax_done);
+        iq_status r = conv_wgrad_tc(d, e, x, (long long*)G, tcws, st, &done, cell, &amax_done,
+                                    (const __half*)e_f16, (const __half*)x_f16);
         if (r != IQ_OK) return r;
         const int mode = gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2;
         if (done && amax_done)

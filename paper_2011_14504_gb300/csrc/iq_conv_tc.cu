@@ -2217,6 +2217,14 @@ static size_t acts16_offset(size_t wbytes) { return (wbytes + 256 + 255) / 256 *
 // inputs with few channels (C % 64 != 0, R S C <= 512) go through an fp16 im2col
 constexpr int IM2COL_MAX_K = 512;
 
+iq_status codes_to_f16(const int8_t* x, __half* xf, int64_t n, cudaStream_t st) {
+    if (n % 16 || (((uintptr_t)x | (uintptr_t)xf) & 15)) return IQ_ERR_INVALID_ARG;
+    if (n == 0) return IQ_OK;
+    k_codes_to_f16<<<grid_for(n / 16), kThreads, 0, st>>>(x, xf, n / 16);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
 size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d) {
     int64_t kdim = (int64_t)d->r * d->s * (d->c / d->groups);
     int64_t kpad = (kdim + 63) / 64 * 64;
@@ -2238,7 +2246,7 @@ bool conv_fwd_tc_supported(const iq_conv_desc* d) {
 
 iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, int32_t* acc,
                       unsigned long long* s1, int* hi, int* lo, void* ws, cudaStream_t st,
-                      bool* done) {
+                      bool* done, const __half* xf_given) {
     *done = false;
     if (!conv_fwd_tc_supported(d) || ((uintptr_t)x & 15) != 0 || !get_encode()) return IQ_OK;
     TcP p;
@@ -2291,9 +2299,12 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
         }
     }
     if (!used && (p.N * (int64_t)p.H * p.W * p.cstride) % 16 == 0) {
-        r = try_launch_c(wf, p.K, p, x, xf, true, acc, s1, hi, lo, err, st, &used);
+        // the fp16 carrier of x: the caller's copy, or converted into the workspace
+        __half* xc = xf_given ? const_cast<__half*>(xf_given) : xf;
+        const bool convert = xf_given == nullptr;
+        r = try_launch_c(wf, p.K, p, x, xc, convert, acc, s1, hi, lo, err, st, &used);
         if (r != IQ_OK) return r;
-        if (!used) r = try_launch_t(map, p, x, xf, true, acc, nullptr, s1, hi, lo, err, st, &used);
+        if (!used) r = try_launch_t(map, p, x, xc, convert, acc, nullptr, s1, hi, lo, err, st, &used);
         if (r != IQ_OK) return r;
     }
     if (!used) r = launch(map, p, 1, x, nullptr, acc, nullptr, s1, hi, lo, err, st);
@@ -2335,7 +2346,7 @@ bool conv_dgrad_tc_supported(const iq_conv_desc* d) {
 
 iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w, int32_t* out32,
                         long long* out64, unsigned long long* s1, int* hi, int* lo, void* ws,
-                        cudaStream_t st, bool* done) {
+                        cudaStream_t st, bool* done, const __half* ef_given) {
     *done = false;
     if (!conv_dgrad_tc_supported(d) || ((uintptr_t)e & 15) != 0 || !get_encode()) return IQ_OK;
     const int nsl = conv_dgrad_tc_slices(d);
@@ -2367,7 +2378,9 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
     __half* wf = reinterpret_cast<__half*>(wsb);
     int* err = tc_status_ptr();
     if (!err) return IQ_ERR_CUDA;
-    __half* ef = reinterpret_cast<__half*>(wsb + acts16_offset((size_t)d->c * p.kpad * 2));
+    __half* ef = ef_given ? const_cast<__half*>(ef_given)
+                          : reinterpret_cast<__half*>(wsb + acts16_offset((size_t)d->c * p.kpad * 2));
+    const bool convert = ef_given == nullptr;
     const bool ef_ok = ((int64_t)p.N * p.H * p.W * p.cstride) % 16 == 0;
     for (int sl = 0; sl < nsl; sl++) {
         k_widen_weights_dgrad<<<dim3((unsigned)((d->c + 31) / 32), (unsigned)((kc + 31) / 32),
@@ -2380,11 +2393,12 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
         p.cofs = sl * kc;
         bool used = false;
         if (ef_ok && nsl == 1) {
-            r = try_launch_c(wf, d->c, p, e, ef, true, out32, s1, hi, lo, err, st, &used);
+            r = try_launch_c(wf, d->c, p, e, ef, convert, out32, s1, hi, lo, err, st, &used);
             if (r != IQ_OK) return r;
         }
         if (ef_ok && !used) {
-            r = try_launch_t(map, p, e, ef, sl == 0, out32, out64, s1, hi, lo, err, st, &used);
+            r = try_launch_t(map, p, e, ef, convert && sl == 0, out32, out64, s1, hi, lo, err, st,
+                             &used);
             if (r != IQ_OK) return r;
         }
         if (!used) r = launch(map, p, 1, e, nullptr, out32, out64, s1, hi, lo, err, st);
@@ -2532,7 +2546,7 @@ bool conv_wgrad_tc_supported(const iq_conv_desc* d) {
 // G (int64 KRSC, zeroed by the caller) += E^T im2col(x)
 iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
                         void* ws, cudaStream_t st, bool* done, unsigned long long* amax,
-                        bool* amax_done) {
+                        bool* amax_done, const __half* ef_given, const __half* xf_given) {
     *done = false;
     *amax_done = false;
     if (tc_env_disabled() || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
@@ -2547,6 +2561,7 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
     bool maps = false;
     int Kp = 0;
     size_t eb = 0, xb = 0;
+    bool use_ef = false, use_xf = false;   // read the caller's carriers instead of converting
     if (!tma16_disabled() && get_encode() && wgrad_tma_plan(d, &p, &t, &nsplit)) {
         Kp = (p.K + 63) / 64 * 64;            // fp16 error rows padded to whole 64-channel blocks
         eb = ((size_t)p.npq * Kp * 2 + 255) / 256 * 256;
@@ -2555,10 +2570,12 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         // the channel count allows
         nb = p.C % 256 == 0 ? 4 : (p.C % 128 == 0 ? 2 : 1);
         if (nb > pick_bn(p.ncols) / 64) nb = pick_bn(p.ncols) / 64;
-        maps = encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256), p.N, p.P, p.Q, Kp, t,
-                                    1, 1, 2, &emap) == IQ_OK &&
-               encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256 + eb), p.N, p.H, p.W,
-                                    p.C, t, p.sh, p.sw, nb, &xmap) == IQ_OK;
+        use_ef = ef_given && Kp == p.K;
+        use_xf = xf_given != nullptr;
+        maps = encode_acts16_blocks(use_ef ? ef_given : reinterpret_cast<__half*>(wsb + 256), p.N,
+                                    p.P, p.Q, Kp, t, 1, 1, 2, &emap) == IQ_OK &&
+               encode_acts16_blocks(use_xf ? xf_given : reinterpret_cast<__half*>(wsb + 256 + eb),
+                                    p.N, p.H, p.W, p.C, t, p.sh, p.sw, nb, &xmap) == IQ_OK;
     }
     // few input channels: the 1 x 1 problem over the im2col of x (pc: the conv's own geometry)
     iq_conv_desc d2;
@@ -2571,8 +2588,10 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         xb = ((size_t)p.npq * p.C * 2 + 255) / 256 * 256;
         nb = p.C % 256 == 0 ? 4 : (p.C % 128 == 0 ? 2 : 1);
         if (nb > pick_bn(p.ncols) / 64) nb = pick_bn(p.ncols) / 64;
-        maps = encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256), p.N, p.P, p.Q, Kp, t,
-                                    1, 1, 2, &emap) == IQ_OK &&
+        use_ef = ef_given && Kp == p.K;
+        use_xf = false;
+        maps = encode_acts16_blocks(use_ef ? ef_given : reinterpret_cast<__half*>(wsb + 256), p.N,
+                                    p.P, p.Q, Kp, t, 1, 1, 2, &emap) == IQ_OK &&
                encode_acts16_blocks(reinterpret_cast<__half*>(wsb + 256 + eb), p.N, p.H, p.W,
                                     p.C, t, 1, 1, nb, &xmap) == IQ_OK;
         im2col = maps;
@@ -2588,18 +2607,22 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         __half* xf = reinterpret_cast<__half*>(wsb + 256 + eb);
         int32_t* part = reinterpret_cast<int32_t*>(wsb + 256 + eb + xb);
         p.out = OUT_PART32;
-        if (Kp == p.K && ne % 16 == 0) {
-            k_codes_to_f16<<<grid_for(ne / 16), kThreads, 0, st>>>(e, ef, ne / 16);
-        } else {
-            k_codes_to_f16_pad<<<grid_for(p.npq * (Kp / 8)), kThreads, 0, st>>>(e, ef, p.npq,
-                                                                              p.K, Kp);
+        if (!use_ef) {
+            if (Kp == p.K && ne % 16 == 0) {
+                k_codes_to_f16<<<grid_for(ne / 16), kThreads, 0, st>>>(e, ef, ne / 16);
+            } else {
+                k_codes_to_f16_pad<<<grid_for(p.npq * (Kp / 8)), kThreads, 0, st>>>(e, ef, p.npq,
+                                                                                  p.K, Kp);
+            }
+            IQ_LAUNCH_CHECK();
         }
-        IQ_LAUNCH_CHECK();
-        if (im2col)
+        if (im2col) {
             launch_im2col(x, pc, xf, st);
-        else
+            IQ_LAUNCH_CHECK();
+        } else if (!use_xf) {
             k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
-        IQ_LAUNCH_CHECK();
+            IQ_LAUNCH_CHECK();
+        }
         iq_status r = IQ_OK;
         switch (pick_bn(p.ncols)) {
             case 64: r = launch_tw<64>(emap, xmap, p, t, nb, nsplit, part, err, st); break;

@@ -3,17 +3,24 @@
 
 #include "iq_internal.cuh"
 
+#include <cuda_fp16.h>
+
 namespace iq {
 
 // Forward convolution on the 5th-generation tensor cores when the shape is
 // supported; sets *done = false (and enqueues nothing) otherwise.  Writes the int32
 // accumulators and the per-channel sum / max / min like the CUDA-core path.
 // `ws` must hold conv_fwd_tc_ws_bytes(d) bytes (the fp16 copy of the weights).
+// xf (optional): the fp16 carrier of x already written by codes_to_f16, read instead of
+// converting x again.
 size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d);
 bool conv_fwd_tc_supported(const iq_conv_desc* d);
 iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, int32_t* acc,
                       unsigned long long* s1, int* hi, int* lo, void* ws, cudaStream_t st,
-                      bool* done);
+                      bool* done, const __half* xf = nullptr);
+
+// x (int8 codes, n elements, n % 16 == 0, 16-byte aligned) -> xf (fp16, 16-byte aligned)
+iq_status codes_to_f16(const int8_t* x, __half* xf, int64_t n, cudaStream_t st);
 
 // Stride-1 data gradient as a forward pass over the errors with flipped, transposed
 // weights.  Writes int32 sums to out32 plus per-channel sum/max/min when the reduction
@@ -23,14 +30,15 @@ bool conv_dgrad_tc_supported(const iq_conv_desc* d);
 int conv_dgrad_tc_slices(const iq_conv_desc* d);
 iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w, int32_t* out32,
                         long long* out64, unsigned long long* s1, int* hi, int* lo, void* ws,
-                        cudaStream_t st, bool* done);
+                        cudaStream_t st, bool* done, const __half* ef = nullptr);
 
 // Weight gradient: writes the exact int64 sums to G (KRSC).  When *amax_done, max |G| has
 // also been folded into *amax (an atomicMax cell the caller zeroed).
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d);
 bool conv_wgrad_tc_supported(const iq_conv_desc* d);
+// ef, xf (optional): fp16 carriers of e and x written by codes_to_f16.
 iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
                         void* ws, cudaStream_t st, bool* done, unsigned long long* amax,
-                        bool* amax_done);
+                        bool* amax_done, const __half* ef = nullptr, const __half* xf = nullptr);
 
 }  // namespace iq

@@ -40,6 +40,7 @@ class Layer:
                                  spec.pad, spec.dil)
         p, q = iq.iq_conv_out_size(self.desc)
         self.out_shape = (n, p, q, spec.cout)
+        self.x16 = None
         self.master = net.master(w_fp32)
         self.wq = torch.empty((spec.cout, spec.r, spec.r, spec.cin), dtype=torch.int8, device=dev)
         iq.iq_weight_requant(self.master, self.wq)
@@ -89,10 +90,10 @@ class Layer:
         if self.spec.bn:
             iq.iq_conv_fwd(self.desc, self.x, self.s_x, self.wq, self.a, self.s_a, self.gamma,
                            self.beta, use_bn=True, relu=True, xhat=self.X, bn_codes=self.bn_codes,
-                           bn_scales=self.bn_scales, ws=ws, stream=stream)
+                           bn_scales=self.bn_scales, x_f16=self.x16, ws=ws, stream=stream)
         else:
             iq.iq_conv_fwd(self.desc, self.x, self.s_x, self.wq, self.a, self.s_a, relu=False,
-                           ws=ws, stream=stream)
+                           x_f16=self.x16, ws=ws, stream=stream)
 
     def backward(self, net, e_a, s_ea, mask=None, need_dx=True, stream=None):
         """From the error of the output codes (before the ReLU mask) to the error of the
@@ -105,10 +106,13 @@ class Layer:
             e, s_e = self.e, self.s_e
         else:
             e, s_e = e_a, s_ea
-        iq.iq_conv_wgrad(self.desc, e, s_e, self.x, self.s_x, self.g, self.s_g, gq_mode=1,
-                         seed=seed, layer=self.lid, step=step, ws=ws, stream=stream)
+        e16 = net.e16 if need_dx and self.spec.cout % 64 == 0 else None
         if need_dx:
-            iq.iq_conv_dgrad(self.desc, e, s_e, self.wq, self.ex, self.s_ex, ws=ws, stream=stream)
+            iq.iq_conv_dgrad(self.desc, e, s_e, self.wq, self.ex, self.s_ex, e_f16=e16, ws=ws,
+                             stream=stream)
+        iq.iq_conv_wgrad(self.desc, e, s_e, self.x, self.s_x, self.g, self.s_g, gq_mode=1,
+                         seed=seed, layer=self.lid, step=step, e_f16=e16, x_f16=self.x16, ws=ws,
+                         stream=stream)
         iq.iq_update(self.master, self.wq, self.g, self.s_g, lr, stream=stream)
         if self.spec.bn:
             iq.iq_bn_update(self.gm, self.bm, self.gamma, self.beta, self.dgamma, self.dbeta,
@@ -196,6 +200,21 @@ class DeepLabV3R50:
             self.s_e_c4 = self.scal()
             self.e_stem = torch.empty(self.stem.out_shape, dtype=torch.int8, device=dev)
             self.s_e_stem = self.scal()
+        if train:
+            # fp16 copies of the codes the tensor-core kernels read: one per distinct conv
+            # input (written by the forward of each layer reading it, reused by their weight
+            # gradients) and one error buffer (written by a layer's data gradient, reused by its
+            # weight gradient)
+            x16, e16 = {}, 0
+            for L in self.layers.values():
+                if L.spec.cin % 64 == 0 and L.x.numel() % 16 == 0:
+                    key = L.x.data_ptr()
+                    if key not in x16:
+                        x16[key] = torch.empty(L.x.numel(), dtype=torch.float16, device=dev)
+                    L.x16 = x16[key]
+                if L.spec.cout % 64 == 0:
+                    e16 = max(e16, L.a.numel())
+            self.e16 = torch.empty(max(e16, 16), dtype=torch.float16, device=dev)
         self.ws = torch.empty(self._ws_bytes(), dtype=torch.uint8, device=dev)
 
     # ------------------------------------------------------------------ helpers

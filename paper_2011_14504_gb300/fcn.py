@@ -49,6 +49,7 @@ class Conv:
     e: torch.Tensor = None        # error after the ReLU mask
     ex: torch.Tensor = None       # error of the input (dgrad output)
     s_ex: torch.Tensor = None
+    x16: torch.Tensor = None      # fp16 copy of x written by the forward, read by the wgrad
     macs: int = 0
 
 
@@ -160,6 +161,16 @@ class FcnVgg16:
             if isinstance(P, Pool):
                 P.ex = torch.empty_like(P.x)
                 P.s_ex = torch.zeros(1, dtype=torch.float64, device=dev)
+        # fp16 copies of the codes that the tensor-core kernels read: each conv input (written by
+        # the forward, reused by the weight gradient) and one error buffer (written by the data
+        # gradient, reused by the weight gradient of the same layer)
+        e16 = 0
+        for L in self.convs:
+            if L.cin % 64 == 0 and L.x.numel() % 16 == 0:
+                L.x16 = torch.empty(L.x.numel(), dtype=torch.float16, device=dev)
+            if L.layer_id > 0 and L.cout % 64 == 0:
+                e16 = max(e16, L.a.numel())
+        self.e16 = torch.empty(max(e16, 16), dtype=torch.float16, device=dev)
 
     def _ws_bytes(self) -> int:
         b = iq.iq_quantize_workspace_size(self.img_codes.numel())
@@ -193,8 +204,8 @@ class FcnVgg16:
                 iq.iq_maxpool_fwd(item.x, 2, 2, 0, item.y, item.arg, stream=stream)
                 continue
             L = item
-            iq.iq_conv_fwd(L.desc, L.x, L.s_x, L.wq, L.a, L.s_a, relu=L.relu, ws=ws,
-                           stream=stream)
+            iq.iq_conv_fwd(L.desc, L.x, L.s_x, L.wq, L.a, L.s_a, relu=L.relu, x_f16=L.x16,
+                           ws=ws, stream=stream)
         iq.iq_upsample_fwd(self.score, self.s_score, self.up_wq, UP_R, UP_STRIDE, UP_PAD, self.z,
                            self.s_z, ws=ws, stream=stream)
 
@@ -223,10 +234,13 @@ class FcnVgg16:
                 e = L.e
             else:
                 e = err
+            e16 = self.e16 if L.layer_id > 0 and L.cout % 64 == 0 else None
             if L.layer_id > 0:
-                iq.iq_conv_dgrad(L.desc, e, s_err, L.wq, L.ex, L.s_ex, ws=ws, stream=stream)
+                iq.iq_conv_dgrad(L.desc, e, s_err, L.wq, L.ex, L.s_ex, e_f16=e16, ws=ws,
+                                 stream=stream)
             iq.iq_conv_wgrad(L.desc, e, s_err, L.x, L.s_x, L.g, L.s_g, gq_mode=2, seed=seed,
-                             layer=L.layer_id, step=step, ws=ws, stream=stream)
+                             layer=L.layer_id, step=step, e_f16=e16, x_f16=L.x16, ws=ws,
+                             stream=stream)
             iq.iq_update(L.master, L.wq, L.g, L.s_g, lr, stream=stream)
             if L.layer_id > 0:
                 err, s_err = L.ex, L.s_ex

@@ -95,10 +95,10 @@ def load(path: str | None = None):
                                 _SZ, _P]
     L.iq_weight_requant.argtypes = [_P, _P, _I64, _I, _I, _P]
     L.iq_conv_fwd.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, C.POINTER(BnBits), _I, _I,
-                              _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
-    L.iq_conv_dgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
+                              _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
+    L.iq_conv_dgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
     L.iq_conv_wgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _I, _U64, _U64, _U64, _P, _P,
-                                _P, _P, _SZ, _P]
+                                _P, _P, _P, _P, _SZ, _P]
     L.iq_bn_int_fwd.argtypes = [_P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _P, _P, _P, _P, _P,
                                 _P, _P, _SZ, _P]
     L.iq_bn_int_bwd.argtypes = [_P, _P, _P, _P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _I, _P,
@@ -263,33 +263,34 @@ def iq_weight_requant(master, wq, k_u=24, k_w=8, stream=None):
 
 
 def iq_conv_fwd(d: ConvDesc, x, s_x, w, a, s_a, gamma=None, beta=None, bits=None, use_bn=False,
-                relu=True, xhat=None, bn_codes=None, bn_scales=None, acc_out=None, ws=None,
-                stream=None):
+                relu=True, xhat=None, bn_codes=None, bn_scales=None, acc_out=None, x_f16=None,
+                ws=None, stream=None):
     if ws is None:
         ws = _ws(iq_conv_fwd_workspace_size(d, use_bn), x.device)
     _check("iq_conv_fwd",
            load().iq_conv_fwd(C.byref(d), _p(x), _p(s_x), _p(w), _p(gamma), _p(beta),
                               C.byref(bits) if bits is not None else None, int(use_bn),
                               int(relu), _p(a), _p(s_a), _p(xhat), _p(bn_codes), _p(bn_scales),
-                              _p(acc_out), _p(ws), ws.numel(), _stream(stream)))
+                              _p(acc_out), _p(x_f16), _p(ws), ws.numel(), _stream(stream)))
 
 
-def iq_conv_dgrad(d: ConvDesc, e, s_e, w, dx, s_dx, acc_out=None, ws=None, stream=None):
+def iq_conv_dgrad(d: ConvDesc, e, s_e, w, dx, s_dx, acc_out=None, e_f16=None, ws=None,
+                  stream=None):
     if ws is None:
         ws = _ws(iq_conv_dgrad_workspace_size(d), e.device)
     _check("iq_conv_dgrad",
            load().iq_conv_dgrad(C.byref(d), _p(e), _p(s_e), _p(w), _p(dx), _p(s_dx), _p(acc_out),
-                                _p(ws), ws.numel(), _stream(stream)))
+                                _p(e_f16), _p(ws), ws.numel(), _stream(stream)))
 
 
 def iq_conv_wgrad(d: ConvDesc, e, s_e, x, s_x, g, s_g, gq_mode=1, seed=0, layer=0, step=0,
-                  g_acc_out=None, ws=None, stream=None):
+                  g_acc_out=None, e_f16=None, x_f16=None, ws=None, stream=None):
     if ws is None:
         ws = _ws(iq_conv_wgrad_workspace_size(d), e.device)
     _check("iq_conv_wgrad",
            load().iq_conv_wgrad(C.byref(d), _p(e), _p(s_e), _p(x), _p(s_x), gq_mode, seed, layer,
-                                step, _p(g), _p(s_g), _p(g_acc_out), _p(ws), ws.numel(),
-                                _stream(stream)))
+                                step, _p(g), _p(s_g), _p(g_acc_out), _p(e_f16), _p(x_f16),
+                                _p(ws), ws.numel(), _stream(stream)))
 
 
 def iq_bn_int_fwd(acc, s_acc, gamma, beta, a, s_a, xhat=None, bn_codes=None, bn_scales=None,

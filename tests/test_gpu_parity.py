@@ -382,6 +382,40 @@ def test_conv_fwd_tc_shapes(ci):
     assert np.array_equal(host(gq).astype(np.int32), wg) and host(s_g)[0] == wgs
 
 
+@pytest.mark.parametrize("ci", [0, 4, 9, 11])
+def test_conv_fp16_carriers_reused(ci):
+    # the forward writes the fp16 copy of x, the data gradient that of e, and the weight
+    # gradient reads both instead of converting: every output still equals the oracle's
+    n, h, w, c, k, r, s, st, pd, dl = TC_CASES[ci]
+    cv = O.Conv(n, h, w, c, k, r, s, st, pd, dl)
+    d = iq.conv_desc(n, h, w, c, k, r, s, st, pd, dl)
+    g = S.rng(400 + ci)
+    x = S.int8_uniform(g, (n, h, w, c))
+    wq = O.requant_master(O.uq(S.he_weights(g, (k, r, s, c), c * r * s), 24)).astype(np.int8)
+    p, q = cv.pq
+    x16 = torch.full((n * h * w * c,), float("nan"), dtype=torch.float16, device=DEV)
+    e16 = torch.full((n * p * q * k,), float("nan"), dtype=torch.float16, device=DEV)
+    acc = torch.empty((n, p, q, k), dtype=torch.int32, device=DEV)
+    iq.iq_conv_fwd(d, dev(x), dscal(0.01), dev(wq), torch.empty((n, p, q, k), dtype=torch.int8,
+                   device=DEV), dscal(), relu=True, acc_out=acc, x_f16=x16)
+    assert np.array_equal(host(acc), O.conv_fwd(cv, x, wq))
+    assert np.array_equal(host(x16).astype(np.int64), x.reshape(-1).astype(np.int64))
+    e = S.int8_uniform(g, (n, p, q, k))
+    if st == 1:
+        dacc = torch.empty((n, h, w, c), dtype=torch.int32, device=DEV)
+        iq.iq_conv_dgrad(d, dev(e), dscal(1e-3), dev(wq), torch.empty((n, h, w, c),
+                         dtype=torch.int8, device=DEV), dscal(), acc_out=dacc, e_f16=e16)
+        assert np.array_equal(host(dacc), O.conv_dgrad(cv, e, wq))
+    else:
+        e16.copy_(dev(e).view(-1).to(torch.float16))
+    assert np.array_equal(host(e16).astype(np.int64), e.reshape(-1).astype(np.int64))
+    gacc = torch.empty(wq.shape, dtype=torch.int64, device=DEV)
+    iq.iq_conv_wgrad(d, dev(e), dscal(1e-3), dev(x), dscal(0.01), torch.empty(wq.shape,
+                     dtype=torch.int8, device=DEV), dscal(), gq_mode=1, seed=1, layer=ci, step=0,
+                     g_acc_out=gacc, e_f16=e16, x_f16=x16)
+    assert np.array_equal(host(gacc), O.conv_wgrad(cv, e, x))
+
+
 @pytest.mark.parametrize("sign,h,k", [(1, 6, 128), (-1, 6, 128), (1, 16, 64), (-1, 16, 64)])
 def test_conv_fwd_adversarial_full_scale(sign, h, k):
     # all codes at +-127: every fp32 chunk holds 1024 * 127^2 = 16,516,096 < 2^24 and
