@@ -612,10 +612,15 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
         bool done = false, amax_done = false;
         unsigned long long* cell = (unsigned long long*)rq;
         IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
+        const int32_t* g32 = nullptr;
         iq_status r = conv_wgrad_tc(d, e, x, (long long*)G, tcws, st, &done, cell, &amax_done,
-                                    (const __half*)e_f16, (const __half*)x_f16);
+                                    (const __half*)e_f16, (const __half*)x_f16,
+                                    g_acc_out ? nullptr : &g32);
         if (r != IQ_OK) return r;
         const int mode = gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2;
+        if (done && g32)
+            return requant_apply(g32, IQ_I32, gn, s_in, 8, mode, seed, layer, step, 0, g, IQ_I8,
+                                 s_g, rq, st);
         if (done && amax_done)
             return requant_apply(G, IQ_I64, gn, s_in, 8, mode, seed, layer, step, 0, g, IQ_I8,
                                  s_g, rq, st);

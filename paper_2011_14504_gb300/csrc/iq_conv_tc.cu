@@ -72,6 +72,8 @@ struct TcP {
     int nkb_total;   // k-blocks of the whole reduction
     int kb_per_split;
     int64_t npq;     // WGRAD: reduction length N*P*Q
+    int slices;      // FWD on the all-TMA kernel: reduction slices (channel ranges of C
+    int slice_rows;  // channels each) run as separate tiles; weight rows per slice
 };
 
 // ---------------------------------------------------------------- FWD gather (K-major A)
@@ -1075,6 +1077,7 @@ struct RectGrid {
 struct RectPos {
     int tile, kb;
     int n, p0, q0, n0;
+    int slice;            // reduction slice (tiles beyond mt nt)
 };
 
 __device__ __forceinline__ void rpos_set(RectPos& q, int tile, const RectGrid& g, int BN) {
@@ -1082,7 +1085,9 @@ __device__ __forceinline__ void rpos_set(RectPos& q, int tile, const RectGrid& g
     q.kb = 0;
     if (tile >= g.total) return;
     const int mt = tile % g.mt;
-    q.n0 = (tile / g.mt) * BN;
+    const int rest = tile / g.mt;
+    q.n0 = (rest % g.nt) * BN;
+    q.slice = rest / g.nt;
     const int qt = mt % g.QT;
     const int pt = (mt / g.QT) % g.PT;
     q.n = mt / (g.QT * g.PT);
@@ -1344,9 +1349,10 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 }
                 uint8_t* st = smem + s * STAGE_BYTES;
                 tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
-                tc::tma_load_4d(st, &amap, &bars->full[s], p.cofs + c0,
+                tc::tma_load_4d(st, &amap, &bars->full[s], p.cofs + q.slice * p.C + c0,
                                 q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph, q.n);
-                tc::tma_load_2d(st + A_BYTES, &wmap, &bars->full[s], q.kb * BK, q.n0);
+                tc::tma_load_2d(st + A_BYTES, &wmap, &bars->full[s], q.kb * BK,
+                                q.slice * p.slice_rows + q.n0);
                 tc::mbar_arrive(&bars->full[s]);
                 issued = (int)kbc + 1;
                 kbc++;
@@ -1434,6 +1440,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         TPos<WG> q;
         q.set(blockIdx.x, p, g, BN);
         int sum[CW];
+        uint32_t amax_t = 0;      // WG with a single split: max |G| of this thread's outputs
         while (ok && q.tile < g.total) {
             const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
 #pragma unroll
@@ -1474,6 +1481,13 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 // the split's own int32 slab (OUT_PART32): no atomics
                 if (p.out == OUT_PART32)
                     o32 = out32 + (int64_t)(q.kb0 / p.kb_per_split) * p.M * p.ncols;
+                // a single split: its slab is the result, and s1 collects max |G|
+                if (s1 && valid) {
+#pragma unroll
+                    for (int i = 0; i < CW; i++)
+                        if (q.n0 + quarter * CW + i < p.ncols)
+                            amax_t = max(amax_t, (uint32_t)abs(sum[i]));
+                }
             }
             if (__any_sync(0xffffffffu, valid)) {
 #pragma unroll
@@ -1486,6 +1500,12 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 }
             }
             q.set(q.tile + gridDim.x, p, g, BN);
+        }
+        if constexpr (WG) {
+            if (s1) {
+                amax_t = warp_max_u32(amax_t);
+                if (lane == 0 && amax_t) atomicMax(s1, (unsigned long long)amax_t);
+            }
         }
     }
     tc::tc_fence_before();
@@ -2116,7 +2136,7 @@ iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const TcP& 
     g.PT = t.PT; g.QT = t.QT; g.BW = t.BW; g.BH = t.BH;
     g.mt = p.N * t.PT * t.QT;
     g.nt = (p.ncols + BN - 1) / BN;
-    g.total = g.mt * g.nt;
+    g.total = g.mt * g.nt * (p.slices > 1 ? p.slices : 1);
     g.nb = 1;
     const int grid = g.total < num_sms() ? g.total : num_sms();
     k_conv_tct<BN, false><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(wmap, amap, p, g, out32, out64,
@@ -2202,6 +2222,8 @@ void fill_geom(TcP& p, const iq_conv_desc* d) {
     p.Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
     p.cstride = d->c;
     p.cofs = 0;
+    p.slices = 1;
+    p.slice_rows = 0;
 }
 
 // k-blocks per split so that each split's int32 running sum cannot overflow
@@ -2332,7 +2354,7 @@ size_t conv_dgrad_tc_ws_bytes(const iq_conv_desc* d) {
     int64_t kpad = ((int64_t)d->r * d->s * (d->k / nsl) + 63) / 64 * 64;
     const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
     const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
-    const size_t wb = (size_t)(d->c * kpad * 2);
+    const size_t wb = (size_t)nsl * d->c * kpad * 2;    // every slice's widened weights
     return acts16_offset(wb) + (size_t)d->n * P * Q * d->k * 2 + 512;
 }
 
@@ -2379,9 +2401,35 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
     int* err = tc_status_ptr();
     if (!err) return IQ_ERR_CUDA;
     __half* ef = ef_given ? const_cast<__half*>(ef_given)
-                          : reinterpret_cast<__half*>(wsb + acts16_offset((size_t)d->c * p.kpad * 2));
+                          : reinterpret_cast<__half*>(
+                                wsb + acts16_offset((size_t)nsl * d->c * p.kpad * 2));
     const bool convert = ef_given == nullptr;
     const bool ef_ok = ((int64_t)p.N * p.H * p.W * p.cstride) % 16 == 0;
+    TmaTile tt;
+    if (nsl > 1 && ef_ok && tma16_ok(p, &tt)) {
+        // every slice in one launch of the all-TMA kernel: slice sl's weights are rows
+        // [sl C, (sl + 1) C) of one matrix, its errors channels [sl kc, (sl + 1) kc)
+        for (int sl = 0; sl < nsl; sl++) {
+            k_widen_weights_dgrad<<<dim3((unsigned)((d->c + 31) / 32), (unsigned)((kc + 31) / 32),
+                                         (unsigned)(d->r * d->s)), dim3(32, 8), 0, st>>>(
+                w, wf + (size_t)sl * d->c * p.kpad, d->k, d->r, d->s, d->c, sl * kc, kc, p.kpad);
+            IQ_LAUNCH_CHECK();
+        }
+        CUtensorMap map;
+        iq_status r = encode_weights(wf, nsl * d->c, p.kpad, pick_bn(p.ncols), &map);
+        if (r != IQ_OK) return r;
+        TcP ps = p;
+        ps.cofs = 0;
+        ps.slices = nsl;
+        ps.slice_rows = d->c;
+        bool used = false;
+        r = try_launch_t(map, ps, e, ef, convert, out32, out64, s1, hi, lo, err, st, &used);
+        if (r != IQ_OK) return r;
+        if (used) {
+            *done = true;
+            return IQ_OK;
+        }
+    }
     for (int sl = 0; sl < nsl; sl++) {
         k_widen_weights_dgrad<<<dim3((unsigned)((d->c + 31) / 32), (unsigned)((kc + 31) / 32),
                                      (unsigned)(d->r * d->s)), dim3(32, 8), 0, st>>>(
@@ -2520,7 +2568,7 @@ bool wgrad_rect(const TcP& p, TmaTile* t) {
 template <int BN>
 iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP& p,
                     const TmaTile& t, int nb, int nsplit, int32_t* part, int* err,
-                    cudaStream_t st) {
+                    cudaStream_t st, unsigned long long* amax = nullptr) {
     IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN, true>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, CfgT<BN>::SMEM));
     RectGrid g;
@@ -2531,7 +2579,7 @@ iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP&
     g.nb = nb < BN / 64 ? nb : BN / 64;
     const int grid = g.total < num_sms() ? g.total : num_sms();
     k_conv_tct<BN, true><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(emap, xmap, p, g, part, nullptr,
-                                                                 nullptr, nullptr, nullptr, err);
+                                                                 amax, nullptr, nullptr, err);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }
@@ -2546,9 +2594,11 @@ bool conv_wgrad_tc_supported(const iq_conv_desc* d) {
 // G (int64 KRSC, zeroed by the caller) += E^T im2col(x)
 iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
                         void* ws, cudaStream_t st, bool* done, unsigned long long* amax,
-                        bool* amax_done, const __half* ef_given, const __half* xf_given) {
+                        bool* amax_done, const __half* ef_given, const __half* xf_given,
+                        const int32_t** g32_out) {
     *done = false;
     *amax_done = false;
+    if (g32_out) *g32_out = nullptr;
     if (tc_env_disabled() || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     int* err = tc_status_ptr();
@@ -2624,12 +2674,22 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
             IQ_LAUNCH_CHECK();
         }
         iq_status r = IQ_OK;
+        // one split and no column compaction: the int32 slab is the result (max |G| from the
+        // epilogue), no int64 copy
+        const bool direct = g32_out && nsplit == 1 && !im2col;
+        unsigned long long* am = direct ? amax : nullptr;
         switch (pick_bn(p.ncols)) {
-            case 64: r = launch_tw<64>(emap, xmap, p, t, nb, nsplit, part, err, st); break;
-            case 128: r = launch_tw<128>(emap, xmap, p, t, nb, nsplit, part, err, st); break;
-            default: r = launch_tw<256>(emap, xmap, p, t, nb, nsplit, part, err, st); break;
+            case 64: r = launch_tw<64>(emap, xmap, p, t, nb, nsplit, part, err, st, am); break;
+            case 128: r = launch_tw<128>(emap, xmap, p, t, nb, nsplit, part, err, st, am); break;
+            default: r = launch_tw<256>(emap, xmap, p, t, nb, nsplit, part, err, st, am); break;
         }
         if (r != IQ_OK) return r;
+        if (direct) {
+            *g32_out = part;
+            *done = true;
+            *amax_done = true;
+            return IQ_OK;
+        }
         if (im2col) {
             const int kdim = d->r * d->s * d->c;
             k_split_sum_cols<<<grid_for(p.M * (int64_t)kdim), kThreads, 0, st>>>(

@@ -36,9 +36,12 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
 // also been folded into *amax (an atomicMax cell the caller zeroed).
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d);
 bool conv_wgrad_tc_supported(const iq_conv_desc* d);
-// ef, xf (optional): fp16 carriers of e and x written by codes_to_f16.
+// ef, xf (optional): fp16 carriers of e and x written by codes_to_f16.  g32 (optional):
+// when the sums fit one int32 slab (a single split) they are left there, *g32 points at them
+// ([K][R S C]) and G is not written.
 iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x, long long* G,
                         void* ws, cudaStream_t st, bool* done, unsigned long long* amax,
-                        bool* amax_done, const __half* ef = nullptr, const __half* xf = nullptr);
+                        bool* amax_done, const __half* ef = nullptr, const __half* xf = nullptr,
+                        const int32_t** g32 = nullptr);
 
 }  // namespace iq

@@ -369,12 +369,30 @@ __global__ void k_update(int32_t* __restrict__ master, int8_t* __restrict__ wq,
     const int64_t lu = qmax(k_u), lw = qmax(k_w);
     const int dsh = k_u - k_w;
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
-        int64_t du = tab[(int)g[i] + 127];
-        int64_t nm = clamp64((int64_t)master[i] - du, -lu, lu);
-        master[i] = (int32_t)nm;
-        int64_t v = (nm + (int64_t(1) << (dsh - 1))) >> dsh;
-        wq[i] = (int8_t)clamp64(v, -lw, lw);
+    auto one = [&](int32_t m, int8_t gv, int8_t& w) -> int32_t {
+        const int64_t nm = clamp64((int64_t)m - tab[(int)gv + 127], -lu, lu);
+        w = (int8_t)clamp64((nm + (int64_t(1) << (dsh - 1))) >> dsh, -lw, lw);
+        return (int32_t)nm;
+    };
+    const bool vec = ((((uintptr_t)master | (uintptr_t)wq | (uintptr_t)g) & 15) == 0);
+    const int64_t n4 = vec ? n / 4 : 0;
+    // 4 parameters per thread: one 16-byte master load/store, 4-byte gradient and code words
+    for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < n4; v += stride) {
+        int4 m = reinterpret_cast<int4*>(master)[v];
+        const uint32_t gw = reinterpret_cast<const uint32_t*>(g)[v];
+        int8_t w0, w1, w2, w3;
+        m.x = one(m.x, (int8_t)(gw & 0xffu), w0);
+        m.y = one(m.y, (int8_t)((gw >> 8) & 0xffu), w1);
+        m.z = one(m.z, (int8_t)((gw >> 16) & 0xffu), w2);
+        m.w = one(m.w, (int8_t)(gw >> 24), w3);
+        reinterpret_cast<int4*>(master)[v] = m;
+        reinterpret_cast<uint32_t*>(wq)[v] = (uint32_t)(uint8_t)w0 | ((uint32_t)(uint8_t)w1 << 8) |
+                                              ((uint32_t)(uint8_t)w2 << 16) | ((uint32_t)(uint8_t)w3 << 24);
+    }
+    for (int64_t i = n4 * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        int8_t w;
+        master[i] = one(master[i], g[i], w);
+        wq[i] = w;
     }
 }
 
@@ -528,7 +546,7 @@ extern "C" iq_status iq_update(int32_t* master, int8_t* wq, const int8_t* g, con
     if (lr_log2 < 0 || lr_log2 > 60) return IQ_ERR_INVALID_ARG;
     if (n == 0) return IQ_OK;
     int sh = (x2 ? k_u - 2 : k_u - 1) - lr_log2;
-    k_update<<<grid_for(n, kThreads, 152 * 4), kThreads, 0, (cudaStream_t)stream>>>(
+    k_update<<<grid_for(n / 4 + 1, kThreads, 152 * 8), kThreads, 0, (cudaStream_t)stream>>>(
         master, wq, g, s_g, n, sh, k_u, k_w);
     IQ_LAUNCH_CHECK();
     return IQ_OK;

@@ -382,6 +382,26 @@ def test_conv_fwd_tc_shapes(ci):
     assert np.array_equal(host(gq).astype(np.int32), wg) and host(s_g)[0] == wgs
 
 
+def test_conv_dgrad_int64_slices_one_launch():
+    # an fc6-like data gradient, (k/groups) r s 127^2 >= 2^31: two reduction slices of 2048
+    # channels run as tiles of one all-TMA launch, int64 sums
+    n, h, w, c, k = 1, 16, 16, 64, 4096
+    cv = O.Conv(n, h, w, c, k, 7, 7, 1, 3)
+    d = iq.conv_desc(n, h, w, c, k, 7, 7, 1, 3)
+    g = S.rng(501)
+    e = np.full((n, h, w, k), 127, np.int8)
+    e[0, :, :, g.integers(0, k, 300)] = -127
+    wq = np.full((k, 7, 7, c), 127, np.int8)
+    wq[:, :, :, 5] = -127
+    dx = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
+    s_dx = dscal()
+    iq.iq_conv_dgrad(d, dev(e), dscal(1e-4), dev(wq), dx, s_dx)
+    want_acc = O.conv_dgrad(cv, e, wq)
+    assert np.abs(want_acc).max() > 2 ** 31
+    want, ws_ = O.sq_int(want_acc, 1e-4 * 2.0 ** -7, 8)
+    assert np.array_equal(host(dx).astype(np.int32), want) and host(s_dx)[0] == ws_
+
+
 @pytest.mark.parametrize("ci", [0, 4, 9, 11])
 def test_conv_fp16_carriers_reused(ci):
     # the forward writes the fp16 copy of x, the data gradient that of e, and the weight
@@ -413,7 +433,15 @@ def test_conv_fp16_carriers_reused(ci):
     iq.iq_conv_wgrad(d, dev(e), dscal(1e-3), dev(x), dscal(0.01), torch.empty(wq.shape,
                      dtype=torch.int8, device=DEV), dscal(), gq_mode=1, seed=1, layer=ci, step=0,
                      g_acc_out=gacc, e_f16=e16, x_f16=x16)
-    assert np.array_equal(host(gacc), O.conv_wgrad(cv, e, x))
+    want_g = O.conv_wgrad(cv, e, x)
+    assert np.array_equal(host(gacc), want_g)
+    # without the int64 copy (a single split requantizes its int32 sums directly)
+    gq = torch.empty(wq.shape, dtype=torch.int8, device=DEV)
+    s_g = dscal()
+    iq.iq_conv_wgrad(d, dev(e), dscal(1e-3), dev(x), dscal(0.01), gq, s_g, gq_mode=1, seed=1,
+                     layer=ci, step=0, e_f16=e16, x_f16=x16)
+    wg, wgs = O.rq_int(want_g, 1e-3 * 0.01, 8, 1, 1, ci, 0, 0)
+    assert np.array_equal(host(gq).astype(np.int32), wg) and host(s_g)[0] == wgs
 
 
 @pytest.mark.parametrize("sign,h,k", [(1, 6, 128), (-1, 6, 128), (1, 16, 64), (-1, 16, 64)])
