@@ -2462,8 +2462,9 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
 namespace {
 
 // the split of nkb k-blocks that minimises (tiles per SM) x (k-blocks per tile) on the
-// persistent grid, each split within the int32 bound and at least 16 k-blocks long;
-// returns the number of splits, *kbs the k-blocks per split
+// persistent grid, each split within the int32 bound and at least 16 k-blocks long; a split
+// count only wins if it beats every smaller one by more than 10% (each extra split costs a
+// partial slab and its sum).  Returns the number of splits, *kbs the k-blocks per split.
 int choose_split(int64_t nkb, int64_t tiles, int64_t* kbs_out) {
     const int64_t sms = num_sms();
     int64_t best_cost = INT64_MAX, kbs = MAX_KB_INT32;
@@ -2473,7 +2474,7 @@ int choose_split(int64_t nkb, int64_t tiles, int64_t* kbs_out) {
         if (k < 16 && ns > 1) break;
         const int64_t nsr = (nkb + k - 1) / k;
         const int64_t cost = ((tiles * nsr + sms - 1) / sms) * k;
-        if (cost < best_cost) { best_cost = cost; kbs = k; }
+        if (best_cost == INT64_MAX || cost * 10 < best_cost * 9) { best_cost = cost; kbs = k; }
     }
     *kbs_out = kbs;
     return (int)((nkb + kbs - 1) / kbs);

@@ -224,26 +224,55 @@ __global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
     const RqParams p = *prm;
     const int64_t lim = qmax(k);
     const int64_t nb = (n + 7) / 8;
+    // u M < rem 2^32  <=>  floor(u M / 2^32) < rem (rem an integer), and with M = Mh 2^32 + Ml
+    // floor(u M / 2^32) = u Mh + umulhi(u, Ml): two 32-bit products instead of 128-bit ones
+    const uint64_t Mh = p.M >> 32;
+    const uint32_t Ml = (uint32_t)p.M;
+    // 8 consecutive elements per thread: 16-byte loads and, for int8 codes, one 8-byte store
+    const bool vec = ((((uintptr_t)q) & 15) == 0) && (dtype != IQ_I8 || (((uintptr_t)out) & 7) == 0);
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nb; b += stride) {
         uint64_t w[4];
         philox4x64_10((uint64_t)b, step, tag, 0, seed, layer, w);
+        const bool full = vec && b * 8 + 8 <= n;
+        T v[8];
+        if (full) {
+            const uint4* src = reinterpret_cast<const uint4*>(q + b * 8);
+#pragma unroll
+            for (int j = 0; j < (int)(8 * sizeof(T) / 16); j++)
+                reinterpret_cast<uint4*>(v)[j] = __ldg(src + j);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 8; j++) v[j] = b * 8 + j < n ? q[b * 8 + j] : T(0);
+        }
+        int64_t c8[8];
 #pragma unroll
         for (int j = 0; j < 8; j++) {
-            int64_t i = b * 8 + j;
-            if (i >= n) break;
             int64_t c = 0;
             if (p.M) {
-                uint64_t num = (uint64_t)((int64_t)q[i] + (int64_t)p.M) << (k - 1);
-                uint64_t fq = udiv(num, p.div);
-                uint64_t rem = num - fq * p.M;
-                uint64_t word = w[j >> 1];
-                uint32_t u = (j & 1) ? (uint32_t)(word >> 32) : (uint32_t)word;
-                bool up = ((u128)u * p.M) < ((u128)rem << 32);
-                c = (int64_t)fq - (int64_t(1) << (k - 1)) + (up ? 1 : 0);
+                const uint64_t num = (uint64_t)((int64_t)v[j] + (int64_t)p.M) << (k - 1);
+                const uint64_t fq = udiv(num, p.div);
+                const uint64_t rem = num - fq * p.M;
+                const uint64_t word = w[j >> 1];
+                const uint32_t u = (j & 1) ? (uint32_t)(word >> 32) : (uint32_t)word;
+                const uint64_t hi = (uint64_t)u * Mh + __umulhi(u, Ml);
+                c = (int64_t)fq - (int64_t(1) << (k - 1)) + (hi < rem ? 1 : 0);
                 c = clamp64(c, -lim, lim);
             }
-            store_code(out, dtype, i, c);
+            c8[j] = c;
+        }
+        if (full && dtype == IQ_I8) {
+            uint32_t lo = 0, hi = 0;
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                lo |= ((uint32_t)c8[j] & 0xffu) << (8 * j);
+                hi |= ((uint32_t)c8[4 + j] & 0xffu) << (8 * j);
+            }
+            reinterpret_cast<uint2*>(out)[b] = make_uint2(lo, hi);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 8; j++)
+                if (b * 8 + j < n) store_code(out, dtype, b * 8 + j, c8[j]);
         }
     }
 }
