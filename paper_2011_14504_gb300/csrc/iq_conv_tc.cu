@@ -1859,7 +1859,8 @@ void launch_im2col(const int8_t* x, const TcP& p, __half* A, cudaStream_t st) {
     const int g4 = p.kpad / 4;
     const int by = 256 / g4 > 0 ? 256 / g4 : 1;
     dim3 block((unsigned)g4, (unsigned)by);
-    dim3 grid((unsigned)((p.Q + by - 1) / by), (unsigned)p.P, (unsigned)p.N);
+    // about 8 pixels per thread: long-lived blocks rather than one pixel each
+    dim3 grid((unsigned)((p.Q + 8 * by - 1) / (8 * by)), (unsigned)p.P, (unsigned)p.N);
     k_im2col_f16<<<grid, block, 0, st>>>(x, p, A);
 }
 

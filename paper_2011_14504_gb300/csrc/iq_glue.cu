@@ -306,6 +306,22 @@ __global__ void __launch_bounds__(256) k_up32_fwd(UpP u, const int8_t* __restric
         const uint32_t x11 = (rc && cc) ? xin(p, q) : 0u;
         const int xv = (int)(x00 | (x01 << 8) | (x10 << 16) | (x11 << 24));
         const int64_t row0 = ((int64_t)b * u.H + I) * u.W;
+        if (CODES && t_lo == 0 && t_hi == 32 && !acc_out) {
+            // a whole 32-column segment: the codes of column t at ob[t c]
+            int8_t* ob = out + (row0 + Jb) * u.c + ch;
+#pragma unroll
+            for (int t = 0; t < 32; t++) {
+                const int sum = __dp4a(xv, (int)wt[t], 0);
+                int c = 0;
+                if (M) {
+                    const uint32_t num = ((uint32_t)(sum + (int)M) << 8) + M;
+                    c = (int)div32(num, d32) - 128;
+                    c = c > 127 ? 127 : (c < -127 ? -127 : c);
+                }
+                ob[t * u.c] = (int8_t)c;
+            }
+            continue;
+        }
 #pragma unroll
         for (int t = 0; t < 32; t++) {
             if (t < t_lo || t >= t_hi) continue;
@@ -518,27 +534,74 @@ struct MseP {
     double s_out;
 };
 
+__device__ __forceinline__ uint32_t word_of(const uint32_t (&w)[4], int t) {
+    return t < 8 ? (t < 4 ? w[0] : w[1]) : (t < 12 ? w[2] : w[3]);
+}
+__device__ __forceinline__ int sbyte_of(const uint32_t (&w)[4], int t) {
+    return (int)(int8_t)(word_of(w, t) >> (8 * (t & 3)));
+}
+__device__ __forceinline__ void set_byte(uint32_t (&w)[4], int t, uint32_t v) {
+    const uint32_t sh = 8 * (t & 3), m = ~(0xffu << sh);
+#pragma unroll
+    for (int k = 0; k < 4; k++)
+        if ((t >> 2) == k) w[k] = (w[k] & m) | ((v & 0xffu) << sh);
+}
+
 // extremes of z for target (t=1) and non-target (t=0) elements: [max0, min0, max1, min1].
-// 16 elements per thread and step: one 16-byte load, the pixel / class of its first byte by
-// one division, then counters.
+// 16 elements per thread and step (one 16-byte load).  With c >= 16 a step holds at most two
+// target elements (one per pixel it touches): they are taken out one by one, replaced by a
+// non-target byte of the same step, and the 16 bytes go through packed __vmaxs4 / __vmins4.
 __global__ void k_mse_stats(const int8_t* __restrict__ z, const uint8_t* __restrict__ lab,
                             int64_t npix, int c, int* __restrict__ ext, UDiv dc, bool vec) {
     int mx0 = INT_MIN, mn0 = INT_MAX, mx1 = INT_MIN, mn1 = INT_MAX;
+    uint32_t pmx = 0x80808080u, pmn = 0x7f7f7f7fu;     // packed running extremes (non-target)
     const int64_t total = npix * c;
     const int64_t n16 = vec ? total / 16 : 0;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n16; u += stride) {
         const int4 v = __ldg(reinterpret_cast<const int4*>(z) + u);
-        const int wv[4] = {v.x, v.y, v.z, v.w};
+        uint32_t w[4] = {(uint32_t)v.x, (uint32_t)v.y, (uint32_t)v.z, (uint32_t)v.w};
         int64_t px = (int64_t)udiv((uint64_t)(u * 16), dc);
-        int ch = (int)(u * 16 - px * c);
-        int lb = lab[px];
+        const int ch0 = (int)(u * 16 - px * c);
+        if (c >= 16) {
+            const int n0 = c - ch0 < 16 ? c - ch0 : 16;    // bytes of pixel px
+            const int t1 = (int)lab[px] - ch0;
+            const bool v1 = t1 >= 0 && t1 < n0;
+            int t2 = 16;
+            if (n0 < 16) {
+                const int l2 = lab[px + 1];
+                if (l2 < 16 - n0) t2 = n0 + l2;
+            }
+            const bool v2 = t2 < 16;
+            if (v1) { const int x = sbyte_of(w, t1); mx1 = max(mx1, x); mn1 = min(mn1, x); }
+            if (v2) { const int x = sbyte_of(w, t2); mx1 = max(mx1, x); mn1 = min(mn1, x); }
+            if (v1 || v2) {
+                int r = 0;
+                if ((v1 && t1 == r) || (v2 && t2 == r)) r = 1;
+                if ((v1 && t1 == r) || (v2 && t2 == r)) r = 2;
+                const uint32_t rb = (uint32_t)sbyte_of(w, r) & 0xffu;
+                if (v1) set_byte(w, t1, rb);
+                if (v2) set_byte(w, t2, rb);
+            }
+            pmx = __vmaxs4(pmx, __vmaxs4(__vmaxs4(w[0], w[1]), __vmaxs4(w[2], w[3])));
+            pmn = __vmins4(pmn, __vmins4(__vmins4(w[0], w[1]), __vmins4(w[2], w[3])));
+        } else {
+            int ch = ch0;
+            int lb = lab[px];
 #pragma unroll
-        for (int j = 0; j < 16; j++) {
-            const int zv = (int)(int8_t)(wv[j >> 2] >> (8 * (j & 3)));
-            if (lb == ch) { mx1 = max(mx1, zv); mn1 = min(mn1, zv); }
-            else { mx0 = max(mx0, zv); mn0 = min(mn0, zv); }
-            if (++ch == c && j < 15) { ch = 0; px++; lb = lab[px]; }
+            for (int j = 0; j < 16; j++) {
+                const int zv = (int)(int8_t)(w[j >> 2] >> (8 * (j & 3)));
+                if (lb == ch) { mx1 = max(mx1, zv); mn1 = min(mn1, zv); }
+                else { mx0 = max(mx0, zv); mn0 = min(mn0, zv); }
+                if (++ch == c && j < 15) { ch = 0; px++; lb = lab[px]; }
+            }
+        }
+    }
+    if (n16 > 0 && c >= 16 && (int64_t)blockIdx.x * blockDim.x + threadIdx.x < n16) {
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            mx0 = max(mx0, (int)(int8_t)(pmx >> (8 * j)));
+            mn0 = min(mn0, (int)(int8_t)(pmn >> (8 * j)));
         }
     }
     for (int64_t o = n16 * 16 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < total;
@@ -608,23 +671,30 @@ __device__ __forceinline__ int mse_code(int zv, bool tgt, const MseP& p, int64_t
 __global__ void k_mse_codes(const int8_t* __restrict__ z, const uint8_t* __restrict__ lab,
                             int64_t npix, int c, int k, const MseP* __restrict__ prm,
                             int8_t* __restrict__ E, UDiv dc, bool vec) {
-    const MseP p = *prm;
-    const int64_t lim = qmax(k);
+    // the code of every (z, target) pair, from the fixed-point map: one table per block
+    __shared__ int8_t tab[512];
+    {
+        const MseP p = *prm;
+        const int64_t lim = qmax(k);
+        for (int i = threadIdx.x; i < 512; i += blockDim.x)
+            tab[i] = (int8_t)mse_code((int)(int8_t)(i & 0xff), i >= 256, p, lim);
+    }
+    __syncthreads();
     const int64_t total = npix * c;
     const int64_t n16 = vec ? total / 16 : 0;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n16; u += stride) {
         const int4 v = __ldg(reinterpret_cast<const int4*>(z) + u);
-        const int wv[4] = {v.x, v.y, v.z, v.w};
+        const uint32_t wv[4] = {(uint32_t)v.x, (uint32_t)v.y, (uint32_t)v.z, (uint32_t)v.w};
         int64_t px = (int64_t)udiv((uint64_t)(u * 16), dc);
         int ch = (int)(u * 16 - px * c);
         int lb = lab[px];
         uint32_t o[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
         for (int j = 0; j < 16; j++) {
-            const int zv = (int)(int8_t)(wv[j >> 2] >> (8 * (j & 3)));
-            const int e = mse_code(zv, lb == ch, p, lim);
-            o[j >> 2] |= ((uint32_t)e & 0xffu) << (8 * (j & 3));
+            const uint32_t zb = (wv[j >> 2] >> (8 * (j & 3))) & 0xffu;
+            const uint32_t e = (uint8_t)tab[zb | (lb == ch ? 256u : 0u)];
+            o[j >> 2] |= e << (8 * (j & 3));
             if (++ch == c && j < 15) { ch = 0; px++; lb = lab[px]; }
         }
         reinterpret_cast<int4*>(E)[u] = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
@@ -632,7 +702,8 @@ __global__ void k_mse_codes(const int8_t* __restrict__ z, const uint8_t* __restr
     for (int64_t i = n16 * 16 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += stride) {
         const int64_t px = (int64_t)udiv((uint64_t)i, dc);
-        E[i] = (int8_t)mse_code(z[i], lab[px] == (int)(i - px * c), p, lim);
+        const uint32_t zb = (uint8_t)z[i];
+        E[i] = tab[zb | (lab[px] == (int)(i - px * c) ? 256u : 0u)];
     }
 }
 

@@ -553,10 +553,11 @@ def test_mse_grad_alignment(offset):
     assert np.array_equal(host(et), want) and host(s_e)[0] == ws_
 
 
-def test_mse_grad():
-    g = S.rng(77)
-    z = S.int8_uniform(g, (2, 33, 17, 150))
-    lab = S.labels_voronoi(g, 2, 33, 17, 150, sites=8)
+@pytest.mark.parametrize("c", [150, 21, 16, 5])
+def test_mse_grad(c):
+    g = S.rng(77 + c)
+    z = S.int8_uniform(g, (2, 33, 17, c))
+    lab = S.labels_voronoi(g, 2, 33, 17, c, sites=8)
     E = torch.empty(z.shape, dtype=torch.int8, device=DEV)
     s_e = dscal()
     iq.iq_mse_grad(dev(z), dscal(0.0123), dev(lab), E, s_e)
