@@ -442,7 +442,8 @@ iq_status iq_ce_grad(const int8_t* z, const double* s_z, const uint8_t* labels, 
  * tag 1 for gamma and 2 for beta), then master <- clip(master - UQ(G_q lr, k_u)) on the
  * x2 grid (value master 2^(2-k_u)), lr = 2^-lr_log2, and the codes gamma = UQ2(master,
  * k_gamma), beta = UQ2(master, k_beta) used by the forward.  All arrays int32[c] on the
- * device; gamma_master / beta_master in/out, gamma / beta out.  ws >= 4096 bytes + 2c. */
+ * device (c <= 4096, else IQ_ERR_UNSUPPORTED); gamma_master / beta_master in/out, gamma /
+ * beta out.  ws >= 4096 bytes + 2c (reserved).  One launch. */
 iq_status iq_bn_update(int32_t* gamma_master, int32_t* beta_master, int32_t* gamma,
                        int32_t* beta, const int64_t* dgamma, const int64_t* dbeta,
                        const double* s_e, const double* bn_scales, int32_t c,

@@ -1018,21 +1018,62 @@ extern "C" iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_
 namespace iq {
 namespace {
 
-__global__ void k_bn_grad_scale(const double* __restrict__ s_e, const double* __restrict__ bn_scales,
-                                double* __restrict__ out) {
-    out[0] = __dmul_rn(*s_e, bn_scales[IQ_BN_S_XHAT]);
-}
-
-// master <- clip(master - UQ(G_q s_g 2^sh, k_u)), codes = UQ2(master, k_w) on the x2 grid
-__global__ void k_bn_param_update(int32_t* __restrict__ master, int32_t* __restrict__ codes,
-                                  const int8_t* __restrict__ g, const double* __restrict__ s_g,
-                                  int32_t c, int sh, int k_u, int k_w) {
-    const double s = *s_g;
+// The whole parameter update of one L1BN layer in one launch: block 0 updates gamma (gradient
+// scale s_e s_X, Philox tag 1), block 1 beta (scale s_e, tag 2).  Each block takes M = max |d|
+// of its c sums, quantizes them by RQ to 8 bits with GQ1's scale (s M) 2^-7, then updates
+// the x2-grid masters and codes; the same steps as requantize + update, one element per
+// thread (c <= 4096).
+__global__ void __launch_bounds__(1024) k_bn_update_fused(int32_t* __restrict__ gmaster,
+                                                          int32_t* __restrict__ bmaster,
+                                                          int32_t* __restrict__ gcodes,
+                                                          int32_t* __restrict__ bcodes,
+                                                          const int64_t* __restrict__ dgam,
+                                                          const int64_t* __restrict__ dbet,
+                                                          const double* __restrict__ s_e,
+                                                          const double* __restrict__ bn_scales,
+                                                          int32_t c, int sh, int k_u, int kg,
+                                                          int kb, uint64_t seed, uint64_t layer,
+                                                          uint64_t step) {
+    __shared__ unsigned long long red[32];
+    const int b = blockIdx.x;
+    const int64_t* d = b ? dbet : dgam;
+    int32_t* master = b ? bmaster : gmaster;
+    int32_t* codes = b ? bcodes : gcodes;
+    const int kw = b ? kb : kg;
+    const uint64_t tag = (uint64_t)b + 1;
+    uint64_t m = 0;
+    for (int i = threadIdx.x; i < c; i += blockDim.x) {
+        const int64_t v = d[i];
+        const uint64_t a = (uint64_t)(v < 0 ? -v : v);
+        m = a > m ? a : m;
+    }
+    m = warp_max_u64(m);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        uint64_t r = threadIdx.x < (blockDim.x + 31) / 32 ? red[threadIdx.x] : 0;
+        r = warp_max_u64(r);
+        if (threadIdx.x == 0) red[0] = r;
+    }
+    __syncthreads();
+    const uint64_t M = red[0];
+    const double s_in = b ? *s_e : __dmul_rn(*s_e, bn_scales[IQ_BN_S_XHAT]);
+    // GQ1 scale (s M) 2^(1-k), k = 8
+    const double s_g = M ? ldexp(__dmul_rn(s_in, (double)M), -7) : ldexp(s_in, -7);
+    const UDiv div = make_udiv(M ? M : 1);
     const double p2 = ldexp(1.0, sh);
-    const int64_t lu = qmax(k_u), lw = qmax(k_w);
-    const int dsh = k_u - k_w;
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < c; i += gridDim.x * blockDim.x) {
-        const int64_t du = code_of(__dmul_rn(__dmul_rn((double)g[i], s), p2), k_u);
+    const int64_t lu = qmax(k_u), lw = qmax(kw);
+    const int dsh = k_u - kw;
+    for (int i = threadIdx.x; i < c; i += blockDim.x) {
+        int64_t q = 0;
+        if (M) {
+            uint64_t w[4];
+            philox4x64_10((uint64_t)(i / 8), step, tag, 0, seed, layer, w);
+            const int j = i & 7;
+            const uint32_t u = (j & 1) ? (uint32_t)(w[j >> 1] >> 32) : (uint32_t)w[j >> 1];
+            q = rq_code(d[i], M, div, 8, u);
+        }
+        const int64_t du = code_of(__dmul_rn(__dmul_rn((double)q, s_g), p2), k_u);
         const int64_t nm = clamp64((int64_t)master[i] - du, -lu, lu);
         master[i] = (int32_t)nm;
         codes[i] = (int32_t)clamp64((nm + (int64_t(1) << (dsh - 1))) >> dsh, -lw, lw);
@@ -1056,24 +1097,12 @@ extern "C" iq_status iq_bn_update(int32_t* gamma_master, int32_t* beta_master, i
     if (!bn_bits_valid(b) || k_u <= b.k_gamma || k_u <= b.k_beta || k_u > 31) return IQ_ERR_INVALID_ARG;
     if (lr_log2 < 0 || lr_log2 > 60) return IQ_ERR_INVALID_ARG;
     if (!ws || ws_bytes < 4096 + 2 * (size_t)c) return IQ_ERR_WORKSPACE;
+    if (c > 4096) return IQ_ERR_UNSUPPORTED;
     cudaStream_t st = (cudaStream_t)stream;
-    char* w = (char*)ws;
-    double* sc = (double*)(w + 1024);            // [0] s_e s_X, [1] s_G gamma, [2] s_G beta
-    int8_t* gg = (int8_t*)(w + 4096);
-    int8_t* gb = gg + c;
-    k_bn_grad_scale<<<1, 1, 0, st>>>(s_e, bn_scales, sc);
-    IQ_LAUNCH_CHECK();
-    iq_status r = requant_int(dgamma, IQ_I64, c, sc, 8, IQ_MODE_RQ_GQ1, seed, layer, step, 1, gg,
-                              IQ_I8, sc + 1, w, st);
-    if (r != IQ_OK) return r;
-    r = requant_int(dbeta, IQ_I64, c, s_e, 8, IQ_MODE_RQ_GQ1, seed, layer, step, 2, gb, IQ_I8,
-                    sc + 2, w, st);
-    if (r != IQ_OK) return r;
     const int sh = (k_u - 2) - lr_log2;
-    const int g = (c + kThreads - 1) / kThreads;
-    k_bn_param_update<<<g, kThreads, 0, st>>>(gamma_master, gamma, gg, sc + 1, c, sh, k_u, b.k_gamma);
-    IQ_LAUNCH_CHECK();
-    k_bn_param_update<<<g, kThreads, 0, st>>>(beta_master, beta, gb, sc + 2, c, sh, k_u, b.k_beta);
+    k_bn_update_fused<<<2, 1024, 0, st>>>(gamma_master, beta_master, gamma, beta, dgamma, dbeta,
+                                          s_e, bn_scales, c, sh, k_u, b.k_gamma, b.k_beta, seed,
+                                          layer, step);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }

@@ -68,6 +68,20 @@ __device__ __forceinline__ uint64_t udiv(uint64_t n, const UDiv& u) {
     return (t + ((n - t) >> u.sh1)) >> u.sh2;
 }
 
+// RQ_k of one integer code v (Eqs. (SQ),(SR)) with M = max|v| > 0 and div = the divisor by M:
+// f = floor((v + M) 2^(k-1) / M), rem the remainder; up iff u M < rem 2^32 for the element's
+// 32-bit random word u, i.e. floor(u M / 2^32) < rem, evaluated as u Mh + umulhi(u, Ml) with
+// M = Mh 2^32 + Ml.  Returns the clipped code.
+__device__ __forceinline__ int64_t rq_code(int64_t v, uint64_t M, const UDiv& div, int k,
+                                           uint32_t u) {
+    const uint64_t num = (uint64_t)(v + (int64_t)M) << (k - 1);
+    const uint64_t fq = udiv(num, div);
+    const uint64_t rem = num - fq * M;
+    const uint64_t hi = (uint64_t)u * (M >> 32) + __umulhi(u, (uint32_t)M);
+    const int64_t c = (int64_t)fq - (int64_t(1) << (k - 1)) + (hi < rem ? 1 : 0);
+    return clamp64(c, -qmax(k), qmax(k));
+}
+
 // A tensor-wide max |q| together with the divisor derived from it.
 struct RqDiv {
     uint64_t M;

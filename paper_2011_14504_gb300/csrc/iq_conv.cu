@@ -326,8 +326,13 @@ __global__ void k_scale_mul(const double* __restrict__ a, const double* __restri
     *out = __dmul_rn(*a, *b);
 }
 // M for SQ of the conv output from the per-channel extremes
+// One block: M = max |acc| (of ReLU(acc) when relu) from the per-channel extremes, then the
+// SQ_8 parameters and the output scale s_in M 2^-7 (the requantizer's finalize step).
 __global__ void k_max_from_stats(const int* __restrict__ hi, const int* __restrict__ lo, int C,
-                                 int relu, unsigned long long* __restrict__ cell) {
+                                 int relu, const double* __restrict__ s_in,
+                                 unsigned long long* __restrict__ cell, RqParams* __restrict__ prm,
+                                 double* __restrict__ s_out) {
+    __shared__ unsigned long long red[32];
     uint64_t m = 0;
     for (int c = threadIdx.x; c < C; c += blockDim.x) {
         int64_t h = hi[c], l = lo[c];
@@ -336,7 +341,18 @@ __global__ void k_max_from_stats(const int* __restrict__ hi, const int* __restri
         m = v > m ? v : m;
     }
     m = warp_max_u64(m);
-    if ((threadIdx.x & 31) == 0 && m) atomicMax(cell, (unsigned long long)m);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        uint64_t r = threadIdx.x < (blockDim.x + 31) / 32 ? red[threadIdx.x] : 0;
+        r = warp_max_u64(r);
+        if (threadIdx.x == 0) {
+            *cell = r;
+            const RqParams p = rq_params_make(r, *s_in, 8, relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ);
+            *prm = p;
+            *s_out = p.s_out;
+        }
+    }
 }
 
 // ------------------------------------------------------------------ geometry helpers
@@ -496,11 +512,12 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
                                   bn_codes, bn_scales, nullptr, st);
     // Q_A = SQ(act(acc), 8) with M from the per-channel extremes
     unsigned long long* cell = (unsigned long long*)L.rq;
-    IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
-    k_max_from_stats<<<1, 1024, 0, st>>>(L.st.hi, L.st.lo, cp.K, relu, cell);
+    k_max_from_stats<<<1, 1024, 0, st>>>(L.st.hi, L.st.lo, cp.K, relu, L.s_acc, cell,
+                                         rq_params_slot(L.rq), s_a);
     IQ_LAUNCH_CHECK();
     return requant_apply(acc, IQ_I32, cp.npq * cp.K, L.s_acc, 8,
-                         relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ, 0, 0, 0, 0, a, IQ_I8, s_a, L.rq, st);
+                         relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ, 0, 0, 0, 0, a, IQ_I8, s_a, L.rq, st,
+                         true);
 }
 
 extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
@@ -552,11 +569,11 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
                               (const __half*)e_f16);
             if (r != IQ_OK) return r;
             if (done) {
-                IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
-                k_max_from_stats<<<1, 1024, 0, st>>>(stats.hi, stats.lo, d->c, 0, cell);
+                k_max_from_stats<<<1, 1024, 0, st>>>(stats.hi, stats.lo, d->c, 0, s_in, cell,
+                                                     rq_params_slot(rq), s_dx);
                 IQ_LAUNCH_CHECK();
                 return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx,
-                                     IQ_I8, s_dx, rq, st);
+                                     IQ_I8, s_dx, rq, st, true);
             }
         }
     }

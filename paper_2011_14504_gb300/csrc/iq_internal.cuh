@@ -14,10 +14,35 @@ iq_status requant_int(const void* q, int in_dtype, int64_t n, const double* s_in
                       int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
                       void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st);
 
-// The same with max |q| already in the first 8 bytes of ws (an unsigned long long).
+// Quantizer parameters of SQ_k / RQ_k for a tensor with max |q| = M and input scale s.
+struct RqParams {
+    uint64_t M;
+    UDiv div;      // by 2M (SQ) or by M (RQ)
+    double s_out;
+    uint32_t R8;   // SQ with k = 8 and 128 < M <= 2^31: floor(2^39 / M), else 0
+};
+
+__device__ inline RqParams rq_params_make(uint64_t M, double s, int k, int mode) {
+    RqParams p;
+    p.M = M;
+    const bool rq = mode == IQ_MODE_RQ_GQ1 || mode == IQ_MODE_RQ_GQ2;
+    p.div = make_udiv(M == 0 ? 1 : (rq ? M : 2 * M));
+    p.R8 = (!rq && k == 8 && M > 128 && M <= (uint64_t(1) << 31))
+               ? (uint32_t)((uint64_t(1) << 39) / M) : 0u;
+    if (mode == IQ_MODE_RQ_GQ2) p.s_out = ldexp(1.0, 1 - k);
+    else p.s_out = M ? ldexp(__dmul_rn(s, (double)M), 1 - k) : ldexp(s, 1 - k);
+    return p;
+}
+
+// where requant_apply keeps the parameters in its workspace
+inline RqParams* rq_params_slot(void* ws) { return (RqParams*)((char*)ws + 256); }
+
+// The same with max |q| already in the first 8 bytes of ws (an unsigned long long); with
+// params_ready the parameters (rq_params_slot) and *s_out have been written as well.
 iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
-                        void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st);
+                        void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st,
+                        bool params_ready = false);
 
 // Per-channel statistics buffers of a BN layer, in the workspace.
 struct BnStats {

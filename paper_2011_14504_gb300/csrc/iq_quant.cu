@@ -99,29 +99,13 @@ __global__ void k_sq_f32_scale(const unsigned* __restrict__ cell, int k, double*
 
 // ------------------------------------------------------------------ SQ / RQ on integer codes
 
-struct RqParams {
-    uint64_t M;
-    UDiv div;      // by 2M (SQ) or by M (RQ)
-    double s_out;
-    uint32_t R8;   // SQ with k = 8 and 128 < M <= 2^31: floor(2^39 / M), else 0
-};
 
 size_t requant_ws_bytes() { return 512; }
 
 __global__ void k_rq_finalize(const unsigned long long* __restrict__ cell,
                               const double* __restrict__ s_in, int k, int mode,
                               RqParams* __restrict__ prm, double* __restrict__ s_out) {
-    uint64_t M = *cell;
-    double s = s_in ? *s_in : 1.0;
-    RqParams p;
-    p.M = M;
-    bool rq = mode == IQ_MODE_RQ_GQ1 || mode == IQ_MODE_RQ_GQ2;
-    p.div = make_udiv(M == 0 ? 1 : (rq ? M : 2 * M));
-    p.R8 = (!rq && k == 8 && M > 128 && M <= (uint64_t(1) << 31))
-               ? (uint32_t)((uint64_t(1) << 39) / M) : 0u;
-    double Md = (double)M;
-    if (mode == IQ_MODE_RQ_GQ2) p.s_out = ldexp(1.0, 1 - k);
-    else p.s_out = M ? ldexp(__dmul_rn(s, Md), 1 - k) : ldexp(s, 1 - k);
+    const RqParams p = rq_params_make(*cell, s_in ? *s_in : 1.0, k, mode);
     *prm = p;
     if (s_out) *s_out = p.s_out;
 }
@@ -222,12 +206,7 @@ __global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
                          const RqParams* __restrict__ prm, uint64_t seed, uint64_t layer,
                          uint64_t step, uint64_t tag, void* __restrict__ out, int dtype) {
     const RqParams p = *prm;
-    const int64_t lim = qmax(k);
     const int64_t nb = (n + 7) / 8;
-    // u M < rem 2^32  <=>  floor(u M / 2^32) < rem (rem an integer), and with M = Mh 2^32 + Ml
-    // floor(u M / 2^32) = u Mh + umulhi(u, Ml): two 32-bit products instead of 128-bit ones
-    const uint64_t Mh = p.M >> 32;
-    const uint32_t Ml = (uint32_t)p.M;
     // 8 consecutive elements per thread: 16-byte loads and, for int8 codes, one 8-byte store
     const bool vec = ((((uintptr_t)q) & 15) == 0) && (dtype != IQ_I8 || (((uintptr_t)out) & 7) == 0);
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -250,14 +229,9 @@ __global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
         for (int j = 0; j < 8; j++) {
             int64_t c = 0;
             if (p.M) {
-                const uint64_t num = (uint64_t)((int64_t)v[j] + (int64_t)p.M) << (k - 1);
-                const uint64_t fq = udiv(num, p.div);
-                const uint64_t rem = num - fq * p.M;
                 const uint64_t word = w[j >> 1];
                 const uint32_t u = (j & 1) ? (uint32_t)(word >> 32) : (uint32_t)word;
-                const uint64_t hi = (uint64_t)u * Mh + __umulhi(u, Ml);
-                c = (int64_t)fq - (int64_t(1) << (k - 1)) + (hi < rem ? 1 : 0);
-                c = clamp64(c, -lim, lim);
+                c = rq_code((int64_t)v[j], p.M, p.div, k, u);
             }
             c8[j] = c;
         }
@@ -279,13 +253,16 @@ __global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
 
 iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
-                        void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st) {
+                        void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st,
+                        bool params_ready) {
     unsigned long long* cell = (unsigned long long*)ws;
-    RqParams* prm = (RqParams*)((char*)ws + 256);
+    RqParams* prm = rq_params_slot(ws);
     bool relu = mode == IQ_MODE_SQ_RELU;
     int g = grid_for(n);
-    k_rq_finalize<<<1, 1, 0, st>>>(cell, s_in, k, mode, prm, s_out);
-    IQ_LAUNCH_CHECK();
+    if (!params_ready) {
+        k_rq_finalize<<<1, 1, 0, st>>>(cell, s_in, k, mode, prm, s_out);
+        IQ_LAUNCH_CHECK();
+    }
     if (n == 0) return IQ_OK;
     if (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) {
         if (in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
