@@ -104,6 +104,14 @@ unsigned long long iq_launch_count(void);
  * Call it after a sequence of calls (a training step) to learn whether they completed. */
 iq_status iq_device_status(int32_t* code, iq_stream stream);
 
+/* The stochastic rounding of Eqs. (SQ),(SR) draws, for element i, the Philox4x64-10 block with
+ * key (seed, layer) and counter (i/8, step, tag, epoch).  epoch is a device-resident word of
+ * the library, 0 until changed: iq_rq_epoch_advance adds 1 to it as a stream operation (so a
+ * training step captured in a CUDA graph, with the advance at its end, draws new numbers on
+ * every replay); iq_rq_epoch_set sets it.  (The paper has no counterpart: it fixes no RNG.) */
+iq_status iq_rq_epoch_advance(iq_stream stream);
+iq_status iq_rq_epoch_set(uint64_t value, iq_stream stream);
+
 /* Output size of a convolution (host-side, no device work). */
 iq_status iq_conv_out_size(const iq_conv_desc* d, int32_t* p, int32_t* q);
 

@@ -1033,7 +1033,8 @@ __global__ void __launch_bounds__(1024) k_bn_update_fused(int32_t* __restrict__ 
                                                           const double* __restrict__ bn_scales,
                                                           int32_t c, int sh, int k_u, int kg,
                                                           int kb, uint64_t seed, uint64_t layer,
-                                                          uint64_t step) {
+                                                          uint64_t step,
+                                                          const unsigned long long* __restrict__ epoch) {
     __shared__ unsigned long long red[32];
     const int b = blockIdx.x;
     const int64_t* d = b ? dbet : dgam;
@@ -1068,7 +1069,7 @@ __global__ void __launch_bounds__(1024) k_bn_update_fused(int32_t* __restrict__ 
         int64_t q = 0;
         if (M) {
             uint64_t w[4];
-            philox4x64_10((uint64_t)(i / 8), step, tag, 0, seed, layer, w);
+            philox4x64_10((uint64_t)(i / 8), step, tag, *epoch, seed, layer, w);
             const int j = i & 7;
             const uint32_t u = (j & 1) ? (uint32_t)(w[j >> 1] >> 32) : (uint32_t)w[j >> 1];
             q = rq_code(d[i], M, div, 8, u);
@@ -1100,9 +1101,11 @@ extern "C" iq_status iq_bn_update(int32_t* gamma_master, int32_t* beta_master, i
     if (c > 4096) return IQ_ERR_UNSUPPORTED;
     cudaStream_t st = (cudaStream_t)stream;
     const int sh = (k_u - 2) - lr_log2;
+    const unsigned long long* ep = rq_epoch_ptr();
+    if (!ep) return IQ_ERR_CUDA;
     k_bn_update_fused<<<2, 1024, 0, st>>>(gamma_master, beta_master, gamma, beta, dgamma, dbeta,
                                           s_e, bn_scales, c, sh, k_u, b.k_gamma, b.k_beta, seed,
-                                          layer, step);
+                                          layer, step, ep);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }

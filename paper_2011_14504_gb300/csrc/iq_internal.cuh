@@ -8,6 +8,9 @@ namespace iq {
 // Scratch needed by requant_int (bytes).
 size_t requant_ws_bytes();
 
+// Device address of the stochastic-rounding epoch (the fourth Philox counter word), or NULL.
+unsigned long long* rq_epoch_ptr();
+
 // SQ / RQ of an integer-coded tensor (see iq_requantize in iq.h).  `relu` applies
 // to the SQ modes only.  `out` has out_dtype elements.
 iq_status requant_int(const void* q, int in_dtype, int64_t n, const double* s_in, int k,

@@ -6,12 +6,36 @@
 #include "iq_internal.cuh"
 
 #include <atomic>
+#include <mutex>
 #include <climits>
 
 namespace iq {
 
 static std::atomic<unsigned long long> g_launches{0};
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+// The fourth Philox counter word of every stochastic rounding: 0 unless advanced on the device
+// (iq_rq_epoch_advance), so that a captured training step replayed as a graph draws new
+// random numbers on each replay.
+static __device__ unsigned long long g_rq_epoch;
+static std::mutex g_epoch_mu;
+static unsigned long long* g_epoch_ptr[256] = {};
+
+unsigned long long* rq_epoch_ptr() {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return nullptr;
+    std::lock_guard<std::mutex> lock(g_epoch_mu);
+    if (!g_epoch_ptr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_rq_epoch) != cudaSuccess || !p) return nullptr;
+        g_epoch_ptr[dev] = static_cast<unsigned long long*>(p);
+    }
+    return g_epoch_ptr[dev];
+}
+
+__global__ void k_epoch_update(unsigned long long* e, unsigned long long v, int set) {
+    *e = set ? v : *e + v;
+}
 
 // ------------------------------------------------------------------ absmax
 
@@ -204,15 +228,17 @@ __global__ void k_sq_int(const T* __restrict__ q, int64_t n, int k, int relu,
 template <typename T>
 __global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
                          const RqParams* __restrict__ prm, uint64_t seed, uint64_t layer,
-                         uint64_t step, uint64_t tag, void* __restrict__ out, int dtype) {
+                         uint64_t step, uint64_t tag, const unsigned long long* __restrict__ epoch,
+                         void* __restrict__ out, int dtype) {
     const RqParams p = *prm;
+    const uint64_t ep = *epoch;
     const int64_t nb = (n + 7) / 8;
     // 8 consecutive elements per thread: 16-byte loads and, for int8 codes, one 8-byte store
     const bool vec = ((((uintptr_t)q) & 15) == 0) && (dtype != IQ_I8 || (((uintptr_t)out) & 7) == 0);
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nb; b += stride) {
         uint64_t w[4];
-        philox4x64_10((uint64_t)b, step, tag, 0, seed, layer, w);
+        philox4x64_10((uint64_t)b, step, tag, ep, seed, layer, w);
         const bool full = vec && b * 8 + 8 <= n;
         T v[8];
         if (full) {
@@ -277,12 +303,14 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
                                                       out_dtype);
     } else {
         int gb = grid_for((n + 7) / 8);
+        const unsigned long long* ep = rq_epoch_ptr();
+        if (!ep) return IQ_ERR_CUDA;
         if (in_dtype == IQ_I32)
             k_rq_int<int32_t><<<gb, kThreads, 0, st>>>((const int32_t*)q, n, k, prm, seed, layer,
-                                                       step, tag, out, out_dtype);
+                                                       step, tag, ep, out, out_dtype);
         else
             k_rq_int<int64_t><<<gb, kThreads, 0, st>>>((const int64_t*)q, n, k, prm, seed, layer,
-                                                       step, tag, out, out_dtype);
+                                                       step, tag, ep, out, out_dtype);
     }
     IQ_LAUNCH_CHECK();
     return IQ_OK;
@@ -450,6 +478,22 @@ extern "C" const char* iq_status_str(iq_status s) {
 extern "C" int iq_version(void) { return 1; }
 
 extern "C" unsigned long long iq_launch_count(void) { return g_launches.load(); }
+
+extern "C" iq_status iq_rq_epoch_advance(iq_stream stream) {
+    unsigned long long* e = iq::rq_epoch_ptr();
+    if (!e) return IQ_ERR_CUDA;
+    iq::k_epoch_update<<<1, 1, 0, (cudaStream_t)stream>>>(e, 1ull, 0);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_rq_epoch_set(uint64_t value, iq_stream stream) {
+    unsigned long long* e = iq::rq_epoch_ptr();
+    if (!e) return IQ_ERR_CUDA;
+    iq::k_epoch_update<<<1, 1, 0, (cudaStream_t)stream>>>(e, (unsigned long long)value, 1);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
 
 extern "C" iq_status iq_quantize_workspace_size(int64_t n, size_t* bytes) {
     if (!bytes || n < 0) return IQ_ERR_INVALID_ARG;

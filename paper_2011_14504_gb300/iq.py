@@ -30,7 +30,7 @@ EXPORTS = [
     "iq_mse_grad", "iq_bn_int_fwd_noalloc", "iq_combine_workspace_size", "iq_combine",
     "iq_spatial_sum_workspace_size", "iq_spatial_sum", "iq_avgpool_bwd", "iq_channel_slice",
     "iq_bilinear_workspace_size", "iq_bilinear_up_fwd", "iq_bilinear_up_bwd", "iq_ce_grad",
-    "iq_bn_update", "iq_device_status",
+    "iq_bn_update", "iq_device_status", "iq_rq_epoch_advance", "iq_rq_epoch_set",
 ]
 
 
@@ -132,6 +132,8 @@ def load(path: str | None = None):
     L.iq_bn_update.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _I32, C.POINTER(BnBits), _I, _I,
                                _U64, _U64, _U64, _P, _SZ, _P]
     L.iq_device_status.argtypes = [C.POINTER(_I32), _P]
+    L.iq_rq_epoch_advance.argtypes = [_P]
+    L.iq_rq_epoch_set.argtypes = [_U64, _P]
     for f in EXPORTS:
         if f not in ("iq_status_str", "iq_version", "iq_launch_count"):
             getattr(L, f).restype = _I
@@ -150,6 +152,15 @@ def iq_device_status(stream=None) -> int:
     code = _I32(0)
     _check("iq_device_status", load().iq_device_status(C.byref(code), _stream(stream)))
     return code.value
+
+
+def iq_rq_epoch_advance(stream=None):
+    """Add 1 to the stochastic-rounding epoch (the fourth Philox counter word) on the stream."""
+    _check("iq_rq_epoch_advance", load().iq_rq_epoch_advance(_stream(stream)))
+
+
+def iq_rq_epoch_set(value: int, stream=None):
+    _check("iq_rq_epoch_set", load().iq_rq_epoch_set(value, _stream(stream)))
 
 
 def status_str(code: int) -> str:

@@ -126,6 +126,34 @@ def test_requantize_sq_int32_vector_path(relu, M):
     assert host(so)[0] == ws
 
 
+def test_rq_epoch_changes_only_the_draws():
+    # the epoch is the fourth Philox counter word: 0 reproduces the oracle; another value gives
+    # other draws of the same stochastic rounding (every code within one of the exact value)
+    g = S.rng(91)
+    q = g.integers(-(2 ** 40), 2 ** 40, size=50000).astype(np.int64)
+    out = torch.empty(q.size, dtype=torch.int8, device=DEV)
+    so = dscal()
+    want, _ = O.rq_int(q, 1e-9, 8, 1, 77, 3, 5)
+    try:
+        iq.iq_requantize(dev(q), dscal(1e-9), 8, iq.IQ_MODE_RQ_GQ1, out, so, seed=77, layer=3,
+                         step=5)
+        assert np.array_equal(host(out).astype(np.int32), want)
+        iq.iq_rq_epoch_set(7)
+        iq.iq_requantize(dev(q), dscal(1e-9), 8, iq.IQ_MODE_RQ_GQ1, out, so, seed=77, layer=3,
+                         step=5)
+        got = host(out).astype(np.int32)
+        assert np.abs(got - want).max() <= 1 and (got != want).mean() > 0.2
+        iq.iq_rq_epoch_advance()
+        iq.iq_requantize(dev(q), dscal(1e-9), 8, iq.IQ_MODE_RQ_GQ1, out, so, seed=77, layer=3,
+                         step=5)
+        got8 = host(out).astype(np.int32)
+        assert np.abs(got8 - want).max() <= 1 and (got8 != got).mean() > 0.2
+    finally:
+        iq.iq_rq_epoch_set(0)
+    iq.iq_requantize(dev(q), dscal(1e-9), 8, iq.IQ_MODE_RQ_GQ1, out, so, seed=77, layer=3, step=5)
+    assert np.array_equal(host(out).astype(np.int32), want)
+
+
 @pytest.mark.parametrize("mode,gq", [(iq.IQ_MODE_RQ_GQ1, 1), (iq.IQ_MODE_RQ_GQ2, 2)])
 def test_requantize_rq_int64(mode, gq):
     g = S.rng(4)
