@@ -1264,10 +1264,12 @@ __global__ void __launch_bounds__(THREADS_T, 1)
 
     if (warp == 0) {
         // ================================================ TMA issuer
-        if constexpr (WG) {
-          if (lane == 0) {
+        if (lane == 0) {
             tc::tma_prefetch_desc(&amap);
             tc::tma_prefetch_desc(&wmap);
+        }
+        if constexpr (WG) {
+          {
             WgPos q;
             wpos_set(q, blockIdx.x, p, g, BN);
             uint32_t kbc = 0;
@@ -1296,31 +1298,31 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 }
                 const int s = kbc % STAGES_T;
                 const uint32_t it = kbc / STAGES_T;
-                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
                     bars->abort = 1;
                     atomicExch(err, 4);
                     break;
                 }
                 uint8_t* st = smem + s * STAGE_BYTES;
-                tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
+                tc::mbar_expect_tx_e(&bars->full[s], STAGE_BYTES);
                 // the k-block's pixels: rectangle (pt, qt) of image nimg
                 const int pp = pt * g.BH, qq = qt * g.BW;
                 // A: E[rectangle][m0 .. m0+127], both 64-channel blocks in one box (zero
                 // outside P x Q and past the last channel block)
-                tc::tma_load_5d(st, &wmap, &bars->full[s], 0, qq, pp, (int)(q.m0 >> 6), nimg);
+                tc::tma_load_5d_e(st, &wmap, &bars->full[s], 0, qq, pp, (int)(q.m0 >> 6), nimg);
                 // B: per run of g.nb 64-column blocks (one tap, 64 g.nb channels) the input
                 // box of the pixels
 #pragma unroll
                 for (int j = 0; j < 4; j++) {
                     if (j * g.nb >= BN / 64) break;
-                    tc::tma_load_5d(st + A_BYTES + 8192 * g.nb * j, &amap, &bars->full[s], 0,
+                    tc::tma_load_5d_e(st + A_BYTES + 8192 * g.nb * j, &amap, &bars->full[s], 0,
                                     qq * p.sw + bx[j], pp * p.sh + by[j], bc[j], nimg);
                 }
                 if (++qt == g.QT) {
                     qt = 0;
                     if (++pt == g.PT) { pt = 0; nimg++; }
                 }
-                tc::mbar_arrive(&bars->full[s]);
+                tc::mbar_arrive_e(&bars->full[s]);
                 issued = (int)kbc + 1;
                 kbc++;
                 wpos_next(q, p, g, BN);
@@ -1331,9 +1333,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                                   &bars->never);
             }
           }
-        } else if (lane == 0) {
-            tc::tma_prefetch_desc(&amap);
-            tc::tma_prefetch_desc(&wmap);
+        } else {
             RectPos q;
             rpos_set(q, blockIdx.x, g, BN);
             int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
@@ -1342,18 +1342,18 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             while (q.tile < g.total) {
                 const int s = kbc % STAGES_T;
                 const uint32_t it = kbc / STAGES_T;
-                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
                     bars->abort = 1;
                     atomicExch(err, 4);
                     break;
                 }
                 uint8_t* st = smem + s * STAGE_BYTES;
-                tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
-                tc::tma_load_4d(st, &amap, &bars->full[s], p.cofs + q.slice * p.C + c0,
+                tc::mbar_expect_tx_e(&bars->full[s], STAGE_BYTES);
+                tc::tma_load_4d_e(st, &amap, &bars->full[s], p.cofs + q.slice * p.C + c0,
                                 q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph, q.n);
-                tc::tma_load_2d(st + A_BYTES, &wmap, &bars->full[s], q.kb * BK,
+                tc::tma_load_2d_e(st + A_BYTES, &wmap, &bars->full[s], q.kb * BK,
                                 q.slice * p.slice_rows + q.n0);
-                tc::mbar_arrive(&bars->full[s]);
+                tc::mbar_arrive_e(&bars->full[s]);
                 issued = (int)kbc + 1;
                 kbc++;
                 const int tile = q.tile;
@@ -1377,7 +1377,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         __syncwarp();
     } else if (warp == 1) {
         // ================================================ MMA issuer
-        if (lane == 0) {
+        {
             const uint32_t idesc = idesc_f16(BM, BN, WG);
             bool ok = true;
             uint32_t kbc = 0, cc = 0;
@@ -1390,11 +1390,11 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
                 const uint32_t buf = cc & 1;
                 if (first && cc >= 2 &&
-                    !tc::mbar_wait(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
+                    !tc::mbar_wait_warp(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
-                if (!tc::mbar_wait(&bars->full[s], it & 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->full[s], it & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
@@ -1411,11 +1411,11 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                         ad = tc::sdesc_kmajor_sw128(a_addr + 32 * k);
                         bd = tc::sdesc_kmajor_sw128(b_addr + 32 * k);
                     }
-                    tc::umma_f16(tmem + buf * BN, ad, bd, idesc, (first && k == 0) ? 0u : 1u);
+                    tc::umma_f16_e(tmem + buf * BN, ad, bd, idesc, (first && k == 0) ? 0u : 1u);
                 }
-                tc::umma_commit(&bars->empty[s]);
+                tc::umma_commit_e(&bars->empty[s]);
                 if (last) {
-                    tc::umma_commit(&bars->accf[buf]);
+                    tc::umma_commit_e(&bars->accf[buf]);
                     cc++;
                 }
                 kbc++;
@@ -1425,7 +1425,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 bars->abort = 1;
                 atomicExch(err, 2);
             }
-            tc::umma_commit(&bars->done);
+            tc::umma_commit_e(&bars->done);
             tc::mbar_wait(&bars->done, 0, &bars->never);
         }
         __syncwarp();
@@ -1578,6 +1578,8 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         if (lane == 0) {
             tc::tma_prefetch_desc(&amap);
             tc::tma_prefetch_desc(&wmap);
+        }
+        {
             RectPos q;
             rpos_set(q, blockIdx.x, g, CM_CH);
             int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
@@ -1586,19 +1588,19 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             while (q.tile < g.total) {
                 const int s = kbc % STAGES_T;
                 const uint32_t it = kbc / STAGES_T;
-                if (!tc::mbar_wait(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
                     bars->abort = 1;
                     atomicExch(err, 4);
                     break;
                 }
                 uint8_t* st = smem + s * STAGE_BYTES;
-                tc::mbar_expect_tx(&bars->full[s], STAGE_BYTES);
+                tc::mbar_expect_tx_e(&bars->full[s], STAGE_BYTES);
                 // A: weight rows n0 .. n0 + 127 (zero past the last channel)
-                tc::tma_load_2d(st, &wmap, &bars->full[s], q.kb * BK, q.n0);
+                tc::tma_load_2d_e(st, &wmap, &bars->full[s], q.kb * BK, q.n0);
                 // B: the 256 input pixels of tap (r, ss), channels c0 .. c0 + 63
-                tc::tma_load_4d(st + A_BYTES, &amap, &bars->full[s], p.cofs + c0,
+                tc::tma_load_4d_e(st + A_BYTES, &amap, &bars->full[s], p.cofs + c0,
                                 q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph, q.n);
-                tc::mbar_arrive(&bars->full[s]);
+                tc::mbar_arrive_e(&bars->full[s]);
                 issued = (int)kbc + 1;
                 kbc++;
                 const int tile = q.tile;
@@ -1622,7 +1624,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         __syncwarp();
     } else if (warp == 1) {
         // ================================================ MMA issuer
-        if (lane == 0) {
+        {
             const uint32_t idesc = idesc_f16(CM_CH, CM_PIX, false);
             bool ok = true;
             uint32_t kbc = 0, cc = 0;
@@ -1635,11 +1637,11 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
                 const uint32_t buf = cc & 1;
                 if (first && cc >= 2 &&
-                    !tc::mbar_wait(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
+                    !tc::mbar_wait_warp(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
-                if (!tc::mbar_wait(&bars->full[s], it & 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->full[s], it & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
@@ -1648,12 +1650,12 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 const uint32_t b_addr = a_addr + A_BYTES;
 #pragma unroll
                 for (int k = 0; k < BK / 16; k++)
-                    tc::umma_f16(tmem + buf * CM_PIX, tc::sdesc_kmajor_sw128(a_addr + 32 * k),
+                    tc::umma_f16_e(tmem + buf * CM_PIX, tc::sdesc_kmajor_sw128(a_addr + 32 * k),
                                  tc::sdesc_kmajor_sw128(b_addr + 32 * k), idesc,
                                  (first && k == 0) ? 0u : 1u);
-                tc::umma_commit(&bars->empty[s]);
+                tc::umma_commit_e(&bars->empty[s]);
                 if (last) {
-                    tc::umma_commit(&bars->accf[buf]);
+                    tc::umma_commit_e(&bars->accf[buf]);
                     cc++;
                 }
                 kbc++;
@@ -1663,7 +1665,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 bars->abort = 1;
                 atomicExch(err, 2);
             }
-            tc::umma_commit(&bars->done);
+            tc::umma_commit_e(&bars->done);
             tc::mbar_wait(&bars->done, 0, &bars->never);
         }
         __syncwarp();
