@@ -58,9 +58,12 @@ struct Cfg {
 
 enum { MODE_FWD = 0, MODE_WGRAD = 1 };
 enum { OUT_STATS = 0, OUT_ATOMIC64 = 1, OUT_PART32 = 2 };
+// the column sums of 32 rows fit one 32-bit warp reduction (R S C <= 4095: 32 4095 128^2 < 2^31)
+constexpr int ST_SUM32 = 4;
 
 struct TcP {
     int mode, out;
+    int st_mask;     // OUT_STATS: TC_STATS_SUM / TC_STATS_LO wanted, ST_SUM32 (see write_row)
     // geometry of the convolution whose operands are gathered
     int N, H, W, C, K, R, S, sh, sw, ph, pw, dh, dw, P, Q;
     int cstride;     // FWD: channel stride of x (>= C) and channel offset of the slice
@@ -1014,9 +1017,13 @@ __global__ void __launch_bounds__(THREADS_Q, 1)
     }
 }
 
-// s[i] += the exact integer held in the fp32 value d[i] (|d| <= 1024 127^2 < 2^24).  When
-// every |d| < 2^22, d + 1.5 2^23 is exact and its bit pattern is 0x4B400000 + d, one add
-// and one integer add per value; otherwise the conversion instruction.
+// s[i] += 0x4B400000 + the exact integer held in the fp32 value d[i] (|d| <= 1024 127^2 <
+// 2^24), modulo 2^32; the caller subtracts 0x4B400000 per folded chunk at the end.  When
+// every |d| < 2^22, d + 1.5 2^23 is exact and its bit pattern is that sum, one add and one
+// integer add per value; otherwise the conversion instruction and the constant.  (The
+// kernels start each tile's sums at -nch FOLD_BIAS.)
+constexpr uint32_t FOLD_BIAS = 0x4B400000u;
+
 template <int W>
 __device__ __forceinline__ void fold_f32(int* s, const uint32_t (&d)[W]) {
     float mx = 0.0f;
@@ -1025,10 +1032,12 @@ __device__ __forceinline__ void fold_f32(int* s, const uint32_t (&d)[W]) {
     if (mx < 4194304.0f) {
 #pragma unroll
         for (int i = 0; i < W; i++)
-            s[i] += __float_as_int(__uint_as_float(d[i]) + 12582912.0f) - 0x4B400000;
+            s[i] = (int)((uint32_t)s[i] + __float_as_uint(__uint_as_float(d[i]) + 12582912.0f));
     } else {
 #pragma unroll
-        for (int i = 0; i < W; i++) s[i] += __float2int_rn(__uint_as_float(d[i]));
+        for (int i = 0; i < W; i++)
+            s[i] = (int)((uint32_t)s[i] + (uint32_t)__float2int_rn(__uint_as_float(d[i])) +
+                         FOLD_BIAS);
     }
 }
 
@@ -1038,28 +1047,32 @@ __device__ __forceinline__ void fold_f32(int* s, const uint32_t (&d)[W]) {
 // image's output pixels; for k-block (tap r,s; channels c0..c0+63) its A rows are the input
 // box of that tap -- one 4-D TMA load (element strides = the conv strides, zero fill
 // outside the image = the padding) lands them directly in the K-major 128-byte-swizzled
-// UMMA layout, next to the B tile (fp16 weights, 2-D TMA).  Warp 0 issues the loads, warp
-// 1 the MMAs into two fp32 accumulators (chunk c in accumulator c % 2), and 16 epilogue
+// UMMA layout, next to the B tile (fp16 weights, 2-D TMA).  Warps 0 and 2 issue the A and
+// the B loads, warp 1 the MMAs into two fp32 accumulators (chunk c in accumulator c % 2), and 16 epilogue
 // warps (4 warpgroups, a quarter of the columns each) fold every finished chunk into int32
 // sums held in registers, so neither the loads nor the folds stall the tensor pipe; a
 // tile's output is written while the next tile's MMAs run.  Persistent over the tiles.
 
-constexpr int THREADS_T = 640;       // warp 0 TMA, warp 1 MMA, warps 4-19 epilogue
+constexpr int THREADS_T = 640;       // warps 0, 2 TMA, warp 1 MMA, warps 4-19 epilogue
 constexpr int EPI_T = 512;
-constexpr int STAGES_T = 4;
+constexpr int STAGES_MAX = 8;
 
 template <int BN>
 struct CfgT {
     static constexpr int STAGE_BYTES = A_BYTES + BN * 128;
-    static constexpr int BAR_OFF = STAGES_T * STAGE_BYTES;
+    // as many stages as 192 KB hold: 4 at BN = 256, 6 at 128, 8 at 64 (the k-blocks in
+    // flight are what hide the load -> MMA -> release round trip)
+    static constexpr int STAGES =
+        196608 / STAGE_BYTES < STAGES_MAX ? 196608 / STAGE_BYTES : STAGES_MAX;
+    static constexpr int BAR_OFF = STAGES * STAGE_BYTES;
     static constexpr int SMEM = BAR_OFF + 1024 + 256;
     static constexpr int TMEM_COLS = 2 * BN;
     static_assert(SMEM <= 232448, "shared memory");
 };
 
 struct BarsT {
-    uint64_t full[STAGES_T];
-    uint64_t empty[STAGES_T];
+    uint64_t full[STAGES_MAX];      // count 2: the A and the B issuer
+    uint64_t empty[STAGES_MAX];
     uint64_t accf[2];
     uint64_t acce[2];
     uint64_t done;
@@ -1129,26 +1142,39 @@ __device__ __forceinline__ void write_row(const TcP& p, const uint32_t (&r)[LDW]
                     reinterpret_cast<int4*>(dst)[i] = make_int4((int)r[4 * i], (int)r[4 * i + 1],
                                                                 (int)r[4 * i + 2], (int)r[4 * i + 3]);
         }
+        // per column over the warp's 32 rows: the maximum always, the minimum and the sum
+        // when the caller consumes them (the sum as one signed reduction when it fits 32 bits,
+        // else as two of its 16-bit halves)
         long long my_sum = 0;
         int my_hi = INT_MIN, my_lo = INT_MAX;
+        const bool want_lo = p.st_mask & TC_STATS_LO, want_sum = p.st_mask & TC_STATS_SUM;
+        const bool sum32 = p.st_mask & ST_SUM32;
 #pragma unroll
         for (int j = 0; j < LDW; j++) {
             const int v = (int)r[j];
             const int mx = __reduce_max_sync(0xffffffffu, valid ? v : INT_MIN);
-            const int mn = __reduce_min_sync(0xffffffffu, valid ? v : INT_MAX);
-            const unsigned sl = __reduce_add_sync(0xffffffffu, valid ? ((unsigned)v & 0xffffu) : 0u);
-            const int sh = __reduce_add_sync(0xffffffffu, valid ? (v >> 16) : 0);
-            if (lane == j) {
-                my_hi = mx;
-                my_lo = mn;
-                my_sum = (long long)sh * 65536 + (long long)sl;
+            if (lane == j) my_hi = mx;
+            if (want_lo) {
+                const int mn = __reduce_min_sync(0xffffffffu, valid ? v : INT_MAX);
+                if (lane == j) my_lo = mn;
+            }
+            if (want_sum) {
+                if (sum32) {
+                    const int sm = __reduce_add_sync(0xffffffffu, valid ? v : 0);
+                    if (lane == j) my_sum = sm;
+                } else {
+                    const unsigned sl =
+                        __reduce_add_sync(0xffffffffu, valid ? ((unsigned)v & 0xffffu) : 0u);
+                    const int sh = __reduce_add_sync(0xffffffffu, valid ? (v >> 16) : 0);
+                    if (lane == j) my_sum = (long long)sh * 65536 + (long long)sl;
+                }
             }
         }
         const int gcol = c0 + lane;
         if (lane < LDW && gcol < p.ncols) {
-            atomicAdd(&s1[gcol], (unsigned long long)my_sum);
             atomicMax(&hi_c[gcol], my_hi);
-            atomicMin(&lo_c[gcol], my_lo);
+            if (want_lo) atomicMin(&lo_c[gcol], my_lo);
+            if (want_sum) atomicAdd(&s1[gcol], (unsigned long long)my_sum);
         }
     } else if (valid) {
         long long* dst = out64 + m * p.ncols + c0;
@@ -1225,6 +1251,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                unsigned long long* __restrict__ s1, int* __restrict__ hi_c,
                int* __restrict__ lo_c, int* __restrict__ err) {
     constexpr int STAGE_BYTES = CfgT<BN>::STAGE_BYTES;
+    constexpr int NST = CfgT<BN>::STAGES;
     constexpr int TMEM_COLS = CfgT<BN>::TMEM_COLS;
     constexpr int CW = BN / 4;                 // columns per epilogue warpgroup
     constexpr int LDW = CW < 16 ? CW : 16;     // columns per TMEM load
@@ -1239,8 +1266,8 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     if ((int)blockIdx.x >= g.total) return;
 
     if (tid == 0) {
-        for (int s = 0; s < STAGES_T; s++) {
-            tc::mbar_init(&bars->full[s], 1);
+        for (int s = 0; s < NST; s++) {
+            tc::mbar_init(&bars->full[s], 2);
             tc::mbar_init(&bars->empty[s], 1);
         }
         for (int b = 0; b < 2; b++) {
@@ -1262,18 +1289,21 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     const uint32_t tmem = bars->tmem_base;
     volatile int* abort_flag = &bars->abort;
 
-    if (warp == 0) {
-        // ================================================ TMA issuer
-        if (lane == 0) {
-            tc::tma_prefetch_desc(&amap);
-            tc::tma_prefetch_desc(&wmap);
-        }
+    if (warp == 0 || warp == 2) {
+        // ================================================ TMA issuers
+        // Warp 0 loads the A tiles and warp 2 the B tiles of the same k-blocks; each adds
+        // its bytes to the stage's full barrier and arrives once (count 2), so the two
+        // issue chains run side by side.
+        const bool side_a = warp == 0;
+        if (lane == 0) tc::tma_prefetch_desc(side_a == WG ? &wmap : &amap);
+        const uint32_t tx = side_a ? (uint32_t)A_BYTES : (uint32_t)(STAGE_BYTES - A_BYTES);
+        int s = 0;
+        uint32_t ph = 0;
+        uint32_t kbc = 0;
+        int issued = 0;
         if constexpr (WG) {
-          {
             WgPos q;
             wpos_set(q, blockIdx.x, p, g, BN);
-            uint32_t kbc = 0;
-            int issued = 0;
             // per tile: the box coordinates of the B column runs (x and y offsets of the tap,
             // first channel block); per k-block: the rectangle, advanced without divisions
             int bx[4], by[4], bc[4];
@@ -1296,27 +1326,29 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                     pt = rr / g.QT;
                     qt = rr - pt * g.QT;
                 }
-                const int s = kbc % STAGES_T;
-                const uint32_t it = kbc / STAGES_T;
-                if (!tc::mbar_wait_warp(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->empty[s], ph ^ 1, abort_flag)) {
                     bars->abort = 1;
                     atomicExch(err, 4);
                     break;
                 }
                 uint8_t* st = smem + s * STAGE_BYTES;
-                tc::mbar_expect_tx_e(&bars->full[s], STAGE_BYTES);
+                tc::mbar_expect_tx_e(&bars->full[s], tx);
                 // the k-block's pixels: rectangle (pt, qt) of image nimg
                 const int pp = pt * g.BH, qq = qt * g.BW;
-                // A: E[rectangle][m0 .. m0+127], both 64-channel blocks in one box (zero
-                // outside P x Q and past the last channel block)
-                tc::tma_load_5d_e(st, &wmap, &bars->full[s], 0, qq, pp, (int)(q.m0 >> 6), nimg);
-                // B: per run of g.nb 64-column blocks (one tap, 64 g.nb channels) the input
-                // box of the pixels
+                if (side_a) {
+                    // A: E[rectangle][m0 .. m0+127], both 64-channel blocks in one box (zero
+                    // outside P x Q and past the last channel block)
+                    tc::tma_load_5d_e(st, &wmap, &bars->full[s], 0, qq, pp, (int)(q.m0 >> 6),
+                                      nimg);
+                } else {
+                    // B: per run of g.nb 64-column blocks (one tap, 64 g.nb channels) the
+                    // input box of the pixels
 #pragma unroll
-                for (int j = 0; j < 4; j++) {
-                    if (j * g.nb >= BN / 64) break;
-                    tc::tma_load_5d_e(st + A_BYTES + 8192 * g.nb * j, &amap, &bars->full[s], 0,
-                                    qq * p.sw + bx[j], pp * p.sh + by[j], bc[j], nimg);
+                    for (int j = 0; j < 4; j++) {
+                        if (j * g.nb >= BN / 64) break;
+                        tc::tma_load_5d_e(st + A_BYTES + 8192 * g.nb * j, &amap, &bars->full[s],
+                                          0, qq * p.sw + bx[j], pp * p.sh + by[j], bc[j], nimg);
+                    }
                 }
                 if (++qt == g.QT) {
                     qt = 0;
@@ -1325,37 +1357,32 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 tc::mbar_arrive_e(&bars->full[s]);
                 issued = (int)kbc + 1;
                 kbc++;
+                if (++s == NST) { s = 0; ph ^= 1; }
                 wpos_next(q, p, g, BN);
             }
-            if (*abort_flag) {
-                for (int kb = (issued > STAGES_T ? issued - STAGES_T : 0); kb < issued; kb++)
-                    tc::mbar_wait(&bars->full[kb % STAGES_T], (uint32_t)(kb / STAGES_T) & 1,
-                                  &bars->never);
-            }
-          }
         } else {
             RectPos q;
             rpos_set(q, blockIdx.x, g, BN);
             int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
-            uint32_t kbc = 0;
-            int issued = 0;
             while (q.tile < g.total) {
-                const int s = kbc % STAGES_T;
-                const uint32_t it = kbc / STAGES_T;
-                if (!tc::mbar_wait_warp(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->empty[s], ph ^ 1, abort_flag)) {
                     bars->abort = 1;
                     atomicExch(err, 4);
                     break;
                 }
                 uint8_t* st = smem + s * STAGE_BYTES;
-                tc::mbar_expect_tx_e(&bars->full[s], STAGE_BYTES);
-                tc::tma_load_4d_e(st, &amap, &bars->full[s], p.cofs + q.slice * p.C + c0,
-                                q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph, q.n);
-                tc::tma_load_2d_e(st + A_BYTES, &wmap, &bars->full[s], q.kb * BK,
-                                q.slice * p.slice_rows + q.n0);
+                tc::mbar_expect_tx_e(&bars->full[s], tx);
+                if (side_a)
+                    tc::tma_load_4d_e(st, &amap, &bars->full[s], p.cofs + q.slice * p.C + c0,
+                                      q.q0 * p.sw + ss * p.dw - p.pw,
+                                      q.p0 * p.sh + r * p.dh - p.ph, q.n);
+                else
+                    tc::tma_load_2d_e(st + A_BYTES, &wmap, &bars->full[s], q.kb * BK,
+                                      q.slice * p.slice_rows + q.n0);
                 tc::mbar_arrive_e(&bars->full[s]);
                 issued = (int)kbc + 1;
                 kbc++;
+                if (++s == NST) { s = 0; ph ^= 1; }
                 const int tile = q.tile;
                 rpos_next(q, p, g, BN);
                 if (q.tile != tile) {
@@ -1368,11 +1395,11 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                     }
                 }
             }
-            if (*abort_flag) {
-                for (int kb = (issued > STAGES_T ? issued - STAGES_T : 0); kb < issued; kb++)
-                    tc::mbar_wait(&bars->full[kb % STAGES_T], (uint32_t)(kb / STAGES_T) & 1,
-                                  &bars->never);
-            }
+        }
+        if (*abort_flag) {
+            // let this warp's copies in flight land before the CTA leaves
+            for (int kb = (issued > NST ? issued - NST : 0); kb < issued; kb++)
+                tc::mbar_wait(&bars->full[kb % NST], (uint32_t)(kb / NST) & 1, &bars->never);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -1381,11 +1408,11 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             const uint32_t idesc = idesc_f16(BM, BN, WG);
             bool ok = true;
             uint32_t kbc = 0, cc = 0;
+            int s = 0;
+            uint32_t ph = 0;
             TPos<WG> q;
             q.set(blockIdx.x, p, g, BN);
             while (ok && q.tile < g.total) {
-                const int s = kbc % STAGES_T;
-                const uint32_t it = kbc / STAGES_T;
                 const bool first = (q.kb % CHUNK_KB) == 0;
                 const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
                 const uint32_t buf = cc & 1;
@@ -1394,7 +1421,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                     ok = false;
                     break;
                 }
-                if (!tc::mbar_wait_warp(&bars->full[s], it & 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->full[s], ph, abort_flag)) {
                     ok = false;
                     break;
                 }
@@ -1419,6 +1446,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                     cc++;
                 }
                 kbc++;
+                if (++s == NST) { s = 0; ph ^= 1; }
                 q.next(p, g, BN);
             }
             if (!ok) {
@@ -1443,8 +1471,10 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         uint32_t amax_t = 0;      // WG with a single split: max |G| of this thread's outputs
         while (ok && q.tile < g.total) {
             const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
+            // the sums start at minus the FOLD_BIAS of the tile's nch chunks
+            const int sum0 = (int)(0u - (uint32_t)nch * FOLD_BIAS);
 #pragma unroll
-            for (int i = 0; i < CW; i++) sum[i] = 0;
+            for (int i = 0; i < CW; i++) sum[i] = sum0;
             for (int c = 0; c < nch; c++) {
                 const uint32_t buf = cc & 1;
                 if (!tc::mbar_wait_sleep(&bars->accf[buf], (cc >> 1) & 1, abort_flag)) {
@@ -1535,6 +1565,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                unsigned long long* __restrict__ s1, int* __restrict__ hi_c,
                int* __restrict__ lo_c, int* __restrict__ err) {
     constexpr int STAGE_BYTES = A_BYTES + CM_PIX * 128;
+    constexpr int NST = CfgT<256>::STAGES;
     constexpr int TMEM_COLS = 2 * CM_PIX;
     constexpr int CW = CM_PIX / 4;             // pixels per epilogue warpgroup
     constexpr int LDW = 16;                    // columns per TMEM load
@@ -1550,8 +1581,8 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     if ((int)blockIdx.x >= g.total) return;
 
     if (tid == 0) {
-        for (int s = 0; s < STAGES_T; s++) {
-            tc::mbar_init(&bars->full[s], 1);
+        for (int s = 0; s < NST; s++) {
+            tc::mbar_init(&bars->full[s], 2);
             tc::mbar_init(&bars->empty[s], 1);
         }
         for (int b = 0; b < 2; b++) {
@@ -1573,53 +1604,52 @@ __global__ void __launch_bounds__(THREADS_T, 1)
     const uint32_t tmem = bars->tmem_base;
     volatile int* abort_flag = &bars->abort;
 
-    if (warp == 0) {
-        // ================================================ TMA issuer
-        if (lane == 0) {
-            tc::tma_prefetch_desc(&amap);
-            tc::tma_prefetch_desc(&wmap);
-        }
-        {
-            RectPos q;
-            rpos_set(q, blockIdx.x, g, CM_CH);
-            int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
-            uint32_t kbc = 0;
-            int issued = 0;
-            while (q.tile < g.total) {
-                const int s = kbc % STAGES_T;
-                const uint32_t it = kbc / STAGES_T;
-                if (!tc::mbar_wait_warp(&bars->empty[s], (it & 1) ^ 1, abort_flag)) {
-                    bars->abort = 1;
-                    atomicExch(err, 4);
-                    break;
-                }
-                uint8_t* st = smem + s * STAGE_BYTES;
-                tc::mbar_expect_tx_e(&bars->full[s], STAGE_BYTES);
-                // A: weight rows n0 .. n0 + 127 (zero past the last channel)
+    if (warp == 0 || warp == 2) {
+        // ================================================ TMA issuers
+        // warp 0 the weight tiles (A), warp 2 the pixel tiles (B); full barriers count 2
+        const bool side_a = warp == 0;
+        if (lane == 0) tc::tma_prefetch_desc(side_a ? &wmap : &amap);
+        const uint32_t tx = side_a ? (uint32_t)A_BYTES : (uint32_t)(STAGE_BYTES - A_BYTES);
+        int s = 0;
+        uint32_t ph = 0;
+        RectPos q;
+        rpos_set(q, blockIdx.x, g, CM_CH);
+        int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
+        uint32_t kbc = 0;
+        int issued = 0;
+        while (q.tile < g.total) {
+            if (!tc::mbar_wait_warp(&bars->empty[s], ph ^ 1, abort_flag)) {
+                bars->abort = 1;
+                atomicExch(err, 4);
+                break;
+            }
+            uint8_t* st = smem + s * STAGE_BYTES;
+            tc::mbar_expect_tx_e(&bars->full[s], tx);
+            if (side_a)     // A: weight rows n0 .. n0 + 127 (zero past the last channel)
                 tc::tma_load_2d_e(st, &wmap, &bars->full[s], q.kb * BK, q.n0);
-                // B: the 256 input pixels of tap (r, ss), channels c0 .. c0 + 63
+            else            // B: the 256 input pixels of tap (r, ss), channels c0 .. c0 + 63
                 tc::tma_load_4d_e(st + A_BYTES, &amap, &bars->full[s], p.cofs + c0,
-                                q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph, q.n);
-                tc::mbar_arrive_e(&bars->full[s]);
-                issued = (int)kbc + 1;
-                kbc++;
-                const int tile = q.tile;
-                rpos_next(q, p, g, CM_CH);
-                if (q.tile != tile) {
-                    r = ss = c0 = 0;
-                } else {
-                    c0 += BK;
-                    if (c0 >= p.C) {
-                        c0 = 0;
-                        if (++ss == p.S) { ss = 0; r++; }
-                    }
+                                  q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph,
+                                  q.n);
+            tc::mbar_arrive_e(&bars->full[s]);
+            issued = (int)kbc + 1;
+            kbc++;
+            if (++s == NST) { s = 0; ph ^= 1; }
+            const int tile = q.tile;
+            rpos_next(q, p, g, CM_CH);
+            if (q.tile != tile) {
+                r = ss = c0 = 0;
+            } else {
+                c0 += BK;
+                if (c0 >= p.C) {
+                    c0 = 0;
+                    if (++ss == p.S) { ss = 0; r++; }
                 }
             }
-            if (*abort_flag) {
-                for (int kb = (issued > STAGES_T ? issued - STAGES_T : 0); kb < issued; kb++)
-                    tc::mbar_wait(&bars->full[kb % STAGES_T], (uint32_t)(kb / STAGES_T) & 1,
-                                  &bars->never);
-            }
+        }
+        if (*abort_flag) {
+            for (int kb = (issued > NST ? issued - NST : 0); kb < issued; kb++)
+                tc::mbar_wait(&bars->full[kb % NST], (uint32_t)(kb / NST) & 1, &bars->never);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -1628,11 +1658,11 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             const uint32_t idesc = idesc_f16(CM_CH, CM_PIX, false);
             bool ok = true;
             uint32_t kbc = 0, cc = 0;
+            int s = 0;
+            uint32_t ph = 0;
             TPos<false> q;
             q.set(blockIdx.x, p, g, CM_CH);
             while (ok && q.tile < g.total) {
-                const int s = kbc % STAGES_T;
-                const uint32_t it = kbc / STAGES_T;
                 const bool first = (q.kb % CHUNK_KB) == 0;
                 const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
                 const uint32_t buf = cc & 1;
@@ -1641,7 +1671,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                     ok = false;
                     break;
                 }
-                if (!tc::mbar_wait_warp(&bars->full[s], it & 1, abort_flag)) {
+                if (!tc::mbar_wait_warp(&bars->full[s], ph, abort_flag)) {
                     ok = false;
                     break;
                 }
@@ -1659,6 +1689,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                     cc++;
                 }
                 kbc++;
+                if (++s == NST) { s = 0; ph ^= 1; }
                 q.next(p, g, CM_CH);
             }
             if (!ok) {
@@ -1682,8 +1713,10 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         int sum[CW];
         while (ok && q.tile < g.total) {
             const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
+            // the sums start at minus the FOLD_BIAS of the tile's nch chunks
+            const int sum0 = (int)(0u - (uint32_t)nch * FOLD_BIAS);
 #pragma unroll
-            for (int i = 0; i < CW; i++) sum[i] = 0;
+            for (int i = 0; i < CW; i++) sum[i] = sum0;
             for (int c = 0; c < nch; c++) {
                 const uint32_t buf = cc & 1;
                 if (!tc::mbar_wait_sleep(&bars->accf[buf], (cc >> 1) & 1, abort_flag)) {
@@ -2227,6 +2260,7 @@ void fill_geom(TcP& p, const iq_conv_desc* d) {
     p.cofs = 0;
     p.slices = 1;
     p.slice_rows = 0;
+    p.st_mask = TC_STATS_SUM | TC_STATS_LO;
 }
 
 // k-blocks per split so that each split's int32 running sum cannot overflow
@@ -2271,7 +2305,7 @@ bool conv_fwd_tc_supported(const iq_conv_desc* d) {
 
 iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, int32_t* acc,
                       unsigned long long* s1, int* hi, int* lo, void* ws, cudaStream_t st,
-                      bool* done, const __half* xf_given) {
+                      bool* done, const __half* xf_given, unsigned st_mask) {
     *done = false;
     if (!conv_fwd_tc_supported(d) || ((uintptr_t)x & 15) != 0 || !get_encode()) return IQ_OK;
     TcP p;
@@ -2281,6 +2315,7 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     p.M = (int64_t)p.N * p.P * p.Q;
     p.ncols = p.K;
     p.kdim = d->r * d->s * d->c;
+    p.st_mask = (int)(st_mask & (TC_STATS_SUM | TC_STATS_LO)) | (p.kdim <= 4095 ? ST_SUM32 : 0);
     p.kpad = (p.kdim + 63) / 64 * 64;
     p.tap_mode = (d->c % 64) == 0;
     p.nkb_total = p.kpad / 64;
@@ -2393,6 +2428,7 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
     p.M = (int64_t)d->n * d->h * d->w;
     p.ncols = d->c;
     p.kdim = d->r * d->s * kc;
+    p.st_mask = TC_STATS_LO;    // the requantizer of dx reads the extremes only
     p.kpad = (p.kdim + 63) / 64 * 64;
     p.tap_mode = (kc % 64) == 0;
     p.nkb_total = p.kpad / 64;

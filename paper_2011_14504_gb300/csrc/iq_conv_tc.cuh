@@ -7,9 +7,14 @@
 
 namespace iq {
 
+// per-channel statistics of the forward beyond the maximum (always written)
+constexpr unsigned TC_STATS_SUM = 1;   // the column sums (the batch-norm mean)
+constexpr unsigned TC_STATS_LO = 2;    // the column minima
+
 // Forward convolution on the 5th-generation tensor cores when the shape is
 // supported; sets *done = false (and enqueues nothing) otherwise.  Writes the int32
-// accumulators and the per-channel sum / max / min like the CUDA-core path.
+// accumulators and the per-channel max, plus the sum and the min selected by st_mask
+// (TC_STATS_*; the CUDA-core path writes all three).
 // `ws` must hold conv_fwd_tc_ws_bytes(d) bytes (the fp16 copy of the weights).
 // xf (optional): the fp16 carrier of x already written by codes_to_f16, read instead of
 // converting x again.
@@ -17,14 +22,16 @@ size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d);
 bool conv_fwd_tc_supported(const iq_conv_desc* d);
 iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, int32_t* acc,
                       unsigned long long* s1, int* hi, int* lo, void* ws, cudaStream_t st,
-                      bool* done, const __half* xf = nullptr);
+                      bool* done, const __half* xf = nullptr,
+                      unsigned st_mask = TC_STATS_SUM | TC_STATS_LO);
 
 // x (int8 codes, n elements, n % 16 == 0, 16-byte aligned) -> xf (fp16, 16-byte aligned)
 iq_status codes_to_f16(const int8_t* x, __half* xf, int64_t n, cudaStream_t st);
 
 // Stride-1 data gradient as a forward pass over the errors with flipped, transposed
-// weights.  Writes int32 sums to out32 plus per-channel sum/max/min when the reduction
-// (k r s) fits int32, else adds int64 sums into out64 (zeroed by the caller).
+// weights.  Writes int32 sums to out32 plus the per-channel max/min (the channel-major
+// kernel also the sums) when the reduction (k r s) fits int32, else adds int64 sums into
+// out64 (zeroed by the caller).
 size_t conv_dgrad_tc_ws_bytes(const iq_conv_desc* d);
 bool conv_dgrad_tc_supported(const iq_conv_desc* d);
 int conv_dgrad_tc_slices(const iq_conv_desc* d);
