@@ -336,6 +336,9 @@ __global__ void k_max_from_stats(const int* __restrict__ hi, const int* __restri
     uint64_t m = 0;
     for (int c = threadIdx.x; c < C; c += blockDim.x) {
         int64_t h = hi[c], l = lo[c];
+        // a channel no extreme was written to (kernels that keep only the extremes of the
+        // whole output write channel 0; under ReLU only the maxima, INT_MIN when untouched)
+        if (!relu && h < l) continue;
         uint64_t v = relu ? (uint64_t)(h > 0 ? h : 0)
                           : (uint64_t)max(h < 0 ? -h : h, l < 0 ? -l : l);
         m = v > m ? v : m;

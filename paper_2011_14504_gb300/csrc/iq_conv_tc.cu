@@ -60,10 +60,14 @@ enum { MODE_FWD = 0, MODE_WGRAD = 1 };
 enum { OUT_STATS = 0, OUT_ATOMIC64 = 1, OUT_PART32 = 2 };
 // the column sums of 32 rows fit one 32-bit warp reduction (R S C <= 4095: 32 4095 128^2 < 2^31)
 constexpr int ST_SUM32 = 4;
+// only the extremes over the whole output are read (SQ without batch norm): the kernel keeps
+// per-thread extremes and writes them to channel 0 once per warp
+constexpr int ST_GMAX = 8;
 
 struct TcP {
     int mode, out;
-    int st_mask;     // OUT_STATS: TC_STATS_SUM / TC_STATS_LO wanted, ST_SUM32 (see write_row)
+    int st_mask;     // OUT_STATS: TC_STATS_SUM / TC_STATS_LO wanted, ST_SUM32, ST_GMAX
+    int tma_out;     // all-TMA forward: the int32 output leaves through TMA stores (map omap)
     // geometry of the convolution whose operands are gathered
     int N, H, W, C, K, R, S, sh, sw, ph, pw, dh, dw, P, Q;
     int cstride;     // FWD: channel stride of x (>= C) and channel offset of the slice
@@ -1065,7 +1069,10 @@ struct CfgT {
     static constexpr int STAGES =
         196608 / STAGE_BYTES < STAGES_MAX ? 196608 / STAGE_BYTES : STAGES_MAX;
     static constexpr int BAR_OFF = STAGES * STAGE_BYTES;
-    static constexpr int SMEM = BAR_OFF + 1024 + 256;
+    // per epilogue warp a 2 KB box (32 rows x 16 int32, 64-byte swizzle) staging the TMA
+    // stores of the int32 output
+    static constexpr int OUT_OFF = BAR_OFF + 1024;
+    static constexpr int SMEM = OUT_OFF + 16 * 2048 + 1024;
     static constexpr int TMEM_COLS = 2 * BN;
     static_assert(SMEM <= 232448, "shared memory");
 };
@@ -1186,6 +1193,78 @@ __device__ __forceinline__ void write_row(const TcP& p, const uint32_t (&r)[LDW]
     }
 }
 
+// per-channel statistics of LDW columns over the warp's 32 rows (OUT_STATS): the maximum,
+// and the minimum and the sum when st_mask asks for them (the sum as one signed 32-bit
+// reduction under ST_SUM32, else as two 16-bit halves)
+template <int LDW>
+__device__ __forceinline__ void col_stats(const TcP& p, const int* r, bool valid, int c0,
+                                          int lane, unsigned long long* __restrict__ s1,
+                                          int* __restrict__ hi_c, int* __restrict__ lo_c) {
+    long long my_sum = 0;
+    int my_hi = INT_MIN, my_lo = INT_MAX;
+    const bool want_lo = p.st_mask & TC_STATS_LO, want_sum = p.st_mask & TC_STATS_SUM;
+    const bool sum32 = p.st_mask & ST_SUM32;
+#pragma unroll
+    for (int j = 0; j < LDW; j++) {
+        const int v = r[j];
+        const int mx = __reduce_max_sync(0xffffffffu, valid ? v : INT_MIN);
+        if (lane == j) my_hi = mx;
+        if (want_lo) {
+            const int mn = __reduce_min_sync(0xffffffffu, valid ? v : INT_MAX);
+            if (lane == j) my_lo = mn;
+        }
+        if (want_sum) {
+            if (sum32) {
+                const int sm = __reduce_add_sync(0xffffffffu, valid ? v : 0);
+                if (lane == j) my_sum = sm;
+            } else {
+                const unsigned sl =
+                    __reduce_add_sync(0xffffffffu, valid ? ((unsigned)v & 0xffffu) : 0u);
+                const int sh = __reduce_add_sync(0xffffffffu, valid ? (v >> 16) : 0);
+                if (lane == j) my_sum = (long long)sh * 65536 + (long long)sl;
+            }
+        }
+    }
+    const int gcol = c0 + lane;
+    if (lane < LDW && gcol < p.ncols && my_hi != INT_MIN) {
+        atomicMax(&hi_c[gcol], my_hi);
+        if (want_lo) atomicMin(&lo_c[gcol], my_lo);
+        if (want_sum) atomicAdd(&s1[gcol], (unsigned long long)my_sum);
+    }
+}
+
+// The warp's 32 output rows (tile rows 32 (warp % 4) .. + 31) are a box of pixels, min(BW,
+// 32) wide and 32 / min(BW, 32) high, starting at output pixel (pp0, qq0) of image n.  Per
+// 16 columns the lanes write their 64-byte rows into the warp's 2 KB staging box in the
+// 64-byte-swizzled layout of map `omap` (16-byte chunk i of row l at chunk i ^ ((l >> 1) & 3):
+// eight lanes of a store phase hit eight distinct bank groups) and lane 0 issues one TMA
+// store, which writes only the part inside the tensor.  The box is reused once the previous
+// store has read it.
+template <int CW>
+__device__ __forceinline__ void tile_store(const CUtensorMap* omap, const int (&sum)[CW],
+                                           uint8_t* stg, int c0, int pp0, int qq0, int n,
+                                           const TcP& p, int lane) {
+    const bool box_in = pp0 < p.P && qq0 < p.Q;
+    const uint32_t sw = (uint32_t)((lane >> 1) & 3);
+#pragma unroll
+    for (int cb = 0; cb < CW; cb += 16) {
+        if (lane == 0) tc::bulk_wait_read_all();
+        __syncwarp();
+        uint8_t* row = stg + lane * 64;
+#pragma unroll
+        for (int i = 0; i < 4; i++)
+            *reinterpret_cast<int4*>(row + (((uint32_t)i ^ sw) << 4)) =
+                make_int4(sum[cb + 4 * i], sum[cb + 4 * i + 1], sum[cb + 4 * i + 2],
+                          sum[cb + 4 * i + 3]);
+        tc::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0 && box_in && c0 + cb < p.ncols) {
+            tc::tma_store_4d(omap, stg, c0 + cb, qq0, pp0, n);
+            tc::bulk_commit();
+        }
+    }
+}
+
 // weight-gradient tile position: (channel tile, column tile, K split) and k-block
 struct WgPos {
     int tile, kb, nkb, kb0;
@@ -1247,6 +1326,7 @@ struct TPos<true> : WgPos {
 template <int BN, bool WG>
 __global__ void __launch_bounds__(THREADS_T, 1)
     k_conv_tct(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap amap,
+               const __grid_constant__ CUtensorMap omap,
                TcP p, RectGrid g, int32_t* __restrict__ out32, long long* __restrict__ out64,
                unsigned long long* __restrict__ s1, int* __restrict__ hi_c,
                int* __restrict__ lo_c, int* __restrict__ err) {
@@ -1469,6 +1549,9 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         q.set(blockIdx.x, p, g, BN);
         int sum[CW];
         uint32_t amax_t = 0;      // WG with a single split: max |G| of this thread's outputs
+        int gmx = INT_MIN, gmn = INT_MAX;     // ST_GMAX: this thread's extremes
+        const int wr0 = (warp & 3) << 5;      // first tile row (pixel) of the warp
+        uint8_t* stg = smem + CfgT<BN>::OUT_OFF + (warp - 4) * 2048;
         while (ok && q.tile < g.total) {
             const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
             // the sums start at minus the FOLD_BIAS of the tile's nch chunks
@@ -1519,7 +1602,27 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                             amax_t = max(amax_t, (uint32_t)abs(sum[i]));
                 }
             }
-            if (__any_sync(0xffffffffu, valid)) {
+            if (!WG && p.tma_out) {
+                if constexpr (!WG) {
+                    if (p.st_mask & ST_GMAX) {
+                        // columns past ncols hold zeros (zero-filled weight rows): harmless
+                        if (valid) {
+#pragma unroll
+                            for (int i = 0; i < CW; i++) {
+                                gmx = max(gmx, sum[i]);
+                                gmn = min(gmn, sum[i]);
+                            }
+                        }
+                    } else {
+#pragma unroll
+                        for (int cb = 0; cb < CW; cb += LDW)
+                            col_stats<LDW>(p, sum + cb, valid, q.n0 + quarter * CW + cb, lane, s1,
+                                           hi_c, lo_c);
+                    }
+                    tile_store<CW>(&omap, sum, stg, q.n0 + quarter * CW, q.p0 + wr0 / g.BW,
+                                   q.q0 + wr0 % g.BW, q.n, p, lane);
+                }
+            } else if (__any_sync(0xffffffffu, valid)) {
 #pragma unroll
                 for (int cb = 0; cb < CW; cb += LDW) {
                     uint32_t v[LDW];
@@ -1530,6 +1633,19 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 }
             }
             q.set(q.tile + gridDim.x, p, g, BN);
+        }
+        if (!WG && p.tma_out) {
+            // the last stores leave the staging box before the CTA does; the global extremes
+            if (lane == 0) tc::bulk_wait_all();
+            __syncwarp();
+            if (p.st_mask & ST_GMAX) {
+                gmx = __reduce_max_sync(0xffffffffu, gmx);
+                gmn = __reduce_min_sync(0xffffffffu, gmn);
+                if (lane == 0 && gmx >= gmn) {
+                    atomicMax(&hi_c[0], gmx);
+                    if (p.st_mask & TC_STATS_LO) atomicMin(&lo_c[0], gmn);
+                }
+            }
         }
         if constexpr (WG) {
             if (s1) {
@@ -2126,6 +2242,26 @@ iq_status encode_acts16(const __half* xf, int N, int H, int W, int cstride, cons
     return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
 }
 
+// 4-D map over the int32 output [N][P][Q][ncols] for the epilogue's TMA stores: box 16
+// channels x min(BW, 32) x 32 / min(BW, 32) pixels (one warp's 32 tile rows), 64-byte
+// swizzle.  Needs ncols % 4 == 0 and a 16-byte-aligned base.
+iq_status encode_out32(int32_t* out, int N, int P, int Q, int ncols, const TmaTile& t,
+                       CUtensorMap* map) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
+    if (!enc || ncols % 4 || ((uintptr_t)out & 15) || t.BW < 16 || 32 % (t.BW < 32 ? t.BW : 32))
+        return IQ_ERR_UNSUPPORTED;
+    const int bw = t.BW < 32 ? t.BW : 32;
+    cuuint64_t gdim[4] = {(cuuint64_t)ncols, (cuuint64_t)Q, (cuuint64_t)P, (cuuint64_t)N};
+    cuuint64_t gstride[3] = {(cuuint64_t)ncols * 4, (cuuint64_t)Q * ncols * 4,
+                             (cuuint64_t)P * Q * ncols * 4};
+    cuuint32_t box[4] = {16, (cuuint32_t)bw, (cuuint32_t)(32 / bw), 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_INT32, 4, (void*)out, gdim, gstride, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                     CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_UNSUPPORTED;
+}
+
 // 5-D map over the fp16 carriers [N][H][W][cstride] with the channels split into 64-wide
 // blocks: dims (64 channels, W, H, cstride / 64 blocks, N), box 64 x BW x BH pixels (at the
 // conv strides) x nb blocks, so one load lands nb MN-major blocks of BW BH rows, 8192 bytes
@@ -2163,9 +2299,9 @@ bool tma16_ok(const TcP& p, TmaTile* t) {
 }
 
 template <int BN>
-iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const TcP& p,
-                   const TmaTile& t, int32_t* out32, long long* out64, unsigned long long* s1,
-                   int* hi, int* lo, int* err, cudaStream_t st) {
+iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const CUtensorMap& omap,
+                   const TcP& p, const TmaTile& t, int32_t* out32, long long* out64,
+                   unsigned long long* s1, int* hi, int* lo, int* err, cudaStream_t st) {
     IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tct<BN, false>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, CfgT<BN>::SMEM));
     RectGrid g;
@@ -2175,8 +2311,8 @@ iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const TcP& 
     g.total = g.mt * g.nt * (p.slices > 1 ? p.slices : 1);
     g.nb = 1;
     const int grid = g.total < num_sms() ? g.total : num_sms();
-    k_conv_tct<BN, false><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(wmap, amap, p, g, out32, out64,
-                                                                  s1, hi, lo, err);
+    k_conv_tct<BN, false><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(wmap, amap, omap, p, g, out32,
+                                                                  out64, s1, hi, lo, err);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }
@@ -2193,13 +2329,18 @@ iq_status try_launch_t(const CUtensorMap& wmap, const TcP& p, const int8_t* x, _
         k_codes_to_f16<<<grid_for(n16), kThreads, 0, st>>>(x, xf, n16);
         IQ_LAUNCH_CHECK();
     }
-    CUtensorMap amap;
+    CUtensorMap amap, omap;
     iq_status r = encode_acts16(xf, p.N, p.H, p.W, p.cstride, t, p.sh, p.sw, &amap);
     if (r != IQ_OK) return r;
+    TcP q = p;
+    // int32 output with statistics: TMA stores of the warps' pixel boxes
+    q.tma_out = p.out == OUT_STATS && out32 && p.slices <= 1 &&
+                encode_out32(out32, p.N, p.P, p.Q, p.ncols, t, &omap) == IQ_OK;
+    if (!q.tma_out) omap = amap;    // not read
     switch (pick_bn(p.ncols)) {
-        case 64: r = launch_t<64>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
-        case 128: r = launch_t<128>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
-        default: r = launch_t<256>(wmap, amap, p, t, out32, out64, s1, hi, lo, err, st); break;
+        case 64: r = launch_t<64>(wmap, amap, omap, q, t, out32, out64, s1, hi, lo, err, st); break;
+        case 128: r = launch_t<128>(wmap, amap, omap, q, t, out32, out64, s1, hi, lo, err, st); break;
+        default: r = launch_t<256>(wmap, amap, omap, q, t, out32, out64, s1, hi, lo, err, st); break;
     }
     if (r == IQ_OK) *used = true;
     return r;
@@ -2261,6 +2402,7 @@ void fill_geom(TcP& p, const iq_conv_desc* d) {
     p.slices = 1;
     p.slice_rows = 0;
     p.st_mask = TC_STATS_SUM | TC_STATS_LO;
+    p.tma_out = 0;
 }
 
 // k-blocks per split so that each split's int32 running sum cannot overflow
@@ -2316,6 +2458,7 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     p.ncols = p.K;
     p.kdim = d->r * d->s * d->c;
     p.st_mask = (int)(st_mask & (TC_STATS_SUM | TC_STATS_LO)) | (p.kdim <= 4095 ? ST_SUM32 : 0);
+    if (!(st_mask & TC_STATS_SUM)) p.st_mask |= ST_GMAX;   // no batch norm: one scale only
     p.kpad = (p.kdim + 63) / 64 * 64;
     p.tap_mode = (d->c % 64) == 0;
     p.nkb_total = p.kpad / 64;
@@ -2428,7 +2571,7 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
     p.M = (int64_t)d->n * d->h * d->w;
     p.ncols = d->c;
     p.kdim = d->r * d->s * kc;
-    p.st_mask = TC_STATS_LO;    // the requantizer of dx reads the extremes only
+    p.st_mask = TC_STATS_LO | ST_GMAX;   // the requantizer of dx reads the extremes only
     p.kpad = (p.kdim + 63) / 64 * 64;
     p.tap_mode = (kc % 64) == 0;
     p.nkb_total = p.kpad / 64;
@@ -2618,8 +2761,10 @@ iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP&
     g.total = g.mt * g.nt * nsplit;
     g.nb = nb < BN / 64 ? nb : BN / 64;
     const int grid = g.total < num_sms() ? g.total : num_sms();
-    k_conv_tct<BN, true><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(emap, xmap, p, g, part, nullptr,
-                                                                 amax, nullptr, nullptr, err);
+    // (the output map is not read: the weight gradient writes its slabs with plain stores)
+    k_conv_tct<BN, true><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(emap, xmap, emap, p, g, part,
+                                                                 nullptr, amax, nullptr, nullptr,
+                                                                 err);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }

@@ -194,6 +194,33 @@ __device__ __forceinline__ void tma_load_5d_e(void* dst, const CUtensorMap* map,
         : "memory");
 }
 
+// ---------------------------------------------------------------- bulk tensor stores
+// 4-D tiled store from shared memory (dense box, no swizzle); elements outside the tensor are
+// not written.  The caller fences the generic-proxy writes of the box first
+// (fence_proxy_async_smem) and every coordinate is >= 0.
+__device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, const void* src, int c0,
+                                             int c1, int c2, int c3) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%2, %3, %4, %5}], [%1];" ::
+            "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2),
+        "r"(c3)
+        : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() {
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+// the bulk stores of this thread have finished reading their shared-memory sources
+__device__ __forceinline__ void bulk_wait_read_all() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+
+// the bulk stores of this thread are complete (written to global memory)
+__device__ __forceinline__ void bulk_wait_all() {
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }

@@ -1,12 +1,16 @@
-"""Time one integer 3x3 convolution layer (stride 1, padding 1) through the C ABI.
+"""Time one integer 3x3 convolution layer (stride 1, padding 1), or one integer L1BN,
+through the C ABI.
 
     python -m paper_2011_14504_gb300.layer_bench [N,H,C,K] [time|once]
+    python -m paper_2011_14504_gb300.layer_bench bn M,C [time|once]
 
 Runs iq_conv_fwd (with ReLU and the SQ8 requantisation of the output), iq_conv_dgrad and
 iq_conv_wgrad (GQ8 gradient) of an N x H x H x C -> K layer on random 8-bit codes.  "time"
 (the default) prints each call's CUDA-event duration over 10 calls after 3 warm-up calls and
 the int8 multiply-accumulate rate it implies (2 ops per MAC); "once" makes one call of each,
-which is the form used under a profiler.
+which is the form used under a profiler.  The bn form runs iq_bn_int_fwd on M x C random
+int32 accumulators (L1BN, ReLU, Q_A) and iq_bn_int_bwd on random 8-bit errors, and prints
+each call's duration and its DRAM bytes per element over that time.
 """
 import sys
 
@@ -15,8 +19,60 @@ import torch
 from . import iq
 
 
+def _time(f, mode):
+    if mode != "time":
+        f()
+        return None
+    for _ in range(3):
+        f()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(10):
+        f()
+    t1.record()
+    torch.cuda.synchronize()
+    return t0.elapsed_time(t1) / 10
+
+
+def bn_main(argv):
+    m, c = [int(v) for v in (argv[0] if argv else "67600,1024").split(",")]
+    mode = argv[1] if len(argv) > 1 else "time"
+    dev = "cuda"
+    g = torch.Generator(device=dev)
+    g.manual_seed(1)
+    acc = (torch.randn((m, c), generator=g, device=dev) * 4000).to(torch.int32)
+    gam = torch.randint(-127, 128, (c,), generator=g, device=dev, dtype=torch.int32)
+    bet = torch.randint(-127, 128, (c,), generator=g, device=dev, dtype=torch.int32)
+    ea = torch.randint(-127, 128, (m, c), generator=g, device=dev, dtype=torch.int8)
+    s_acc = torch.tensor([2.0 ** -14], dtype=torch.float64, device=dev)
+    s_e = torch.tensor([2.0 ** -21], dtype=torch.float64, device=dev)
+    a = torch.empty((m, c), dtype=torch.int8, device=dev)
+    x = torch.empty((m, c), dtype=torch.int16, device=dev)
+    e = torch.empty((m, c), dtype=torch.int8, device=dev)
+    codes = torch.empty(2 * c, dtype=torch.int32, device=dev)
+    scal = torch.empty(iq.IQ_BN_SCALES, dtype=torch.float64, device=dev)
+    s_a, s_out = torch.empty_like(s_acc), torch.empty_like(s_acc)
+    ws = torch.empty(iq.iq_bn_int_workspace_size(m, c), dtype=torch.uint8, device=dev)
+    fwd = lambda: iq.iq_bn_int_fwd(acc, s_acc, gam, bet, a, s_a, xhat=x, bn_codes=codes,
+                                   bn_scales=scal, ws=ws)
+    bwd = lambda: iq.iq_bn_int_bwd(ea, s_e, a, x, gam, codes, scal, e, s_out, ws=ws)
+    # bytes per element: fwd reads the int32 sums three times (sums, deviation,
+    # requantisation) and
+    # writes X (int16) and A (int8); bwd reads e_a, A, X three times and writes E (int8)
+    for name, f, nb in (("bn_fwd", fwd, 15), ("bn_bwd", bwd, 13)):
+        ms = _time(f, mode)
+        if ms is not None:
+            print(f"{name}: {ms:.3f} ms  {nb * m * c / ms / 1e6:.0f} GB/s at {nb} B/element")
+    torch.cuda.synchronize()
+    print("ok")
+
+
 def main(argv=None):
     argv = sys.argv[1:] if argv is None else argv
+    if argv and argv[0] == "bn":
+        return bn_main(argv[1:])
     n, h, c, k = [int(v) for v in (argv[0] if argv else "8,128,256,256").split(",")]
     mode = argv[1] if len(argv) > 1 else "time"
     dev = "cuda"
