@@ -178,6 +178,7 @@ __device__ __forceinline__ int64_t floordiv_i64(int64_t a, int64_t b) {
 __global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__ acc, int64_t m,
                                                      int32_t C, int CG, BnStats s) {
     __shared__ unsigned long long sh_d[kThreads * 4], sh_n[kThreads * 4];
+    __shared__ int sh_h[kThreads * 4], sh_l[kThreads * 4];
     const int C4 = C >> 2;
     const int cg = threadIdx.x % CG, rl = threadIdx.x / CG, RL = blockDim.x / CG;
     const int g = blockIdx.x * CG + cg;
@@ -188,6 +189,8 @@ __global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__
         for (int j = 0; j < 4; j++) f[j] = floordiv_i64((int64_t)s.s1[4 * g + j], m);
     }
     unsigned long long d[4] = {0, 0, 0, 0}, n[4] = {0, 0, 0, 0};
+    // the per-channel extremes too (the conv epilogue may leave them to this pass)
+    int hi[4] = {INT_MIN, INT_MIN, INT_MIN, INT_MIN}, lo[4] = {INT_MAX, INT_MAX, INT_MAX, INT_MAX};
     const int4* a4 = reinterpret_cast<const int4*>(acc);
     const int64_t step = (int64_t)gridDim.y * RL;
     if (act) {
@@ -196,13 +199,15 @@ __global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__
         for (; r < m; r += 2 * step) {
             const bool two = r + step < m;
             const int4 v0 = a4[r * C4 + g];
-            const int4 v1 = two ? a4[(r + step) * C4 + g] : make_int4(0, 0, 0, 0);
+            const int4 v1 = two ? a4[(r + step) * C4 + g] : v0;
             const int vs0[4] = {v0.x, v0.y, v0.z, v0.w}, vs1[4] = {v1.x, v1.y, v1.z, v1.w};
 #pragma unroll
             for (int j = 0; j < 4; j++) {
                 const int64_t dv0 = (int64_t)vs0[j] - f[j];
                 d[j] += (unsigned long long)(dv0 < 0 ? -dv0 : dv0);
                 n[j] += dv0 > 0;
+                hi[j] = max(hi[j], max(vs0[j], vs1[j]));
+                lo[j] = min(lo[j], min(vs0[j], vs1[j]));
                 if (two) {
                     const int64_t dv1 = (int64_t)vs1[j] - f[j];
                     d[j] += (unsigned long long)(dv1 < 0 ? -dv1 : dv1);
@@ -215,6 +220,8 @@ __global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__
     for (int j = 0; j < 4; j++) {
         sh_d[rl * CG * 4 + 4 * cg + j] = d[j];
         sh_n[rl * CG * 4 + 4 * cg + j] = n[j];
+        sh_h[rl * CG * 4 + 4 * cg + j] = hi[j];
+        sh_l[rl * CG * 4 + 4 * cg + j] = lo[j];
     }
     __syncthreads();
     const int col = threadIdx.x;
@@ -222,9 +229,19 @@ __global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__
         const int c = 4 * blockIdx.x * CG + col;
         if (c < C) {
             unsigned long long td = 0, tn = 0;
-            for (int i = 0; i < RL; i++) { td += sh_d[i * CG * 4 + col]; tn += sh_n[i * CG * 4 + col]; }
+            int th = INT_MIN, tl = INT_MAX;
+            for (int i = 0; i < RL; i++) {
+                td += sh_d[i * CG * 4 + col];
+                tn += sh_n[i * CG * 4 + col];
+                th = max(th, sh_h[i * CG * 4 + col]);
+                tl = min(tl, sh_l[i * CG * 4 + col]);
+            }
             atomicAdd(&s.dev[c], td);
             atomicAdd(&s.ngt[c], tn);
+            if (th >= tl) {
+                atomicMax(&s.hi[c], th);
+                atomicMin(&s.lo[c], tl);
+            }
         }
     }
 }

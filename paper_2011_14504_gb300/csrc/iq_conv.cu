@@ -502,7 +502,8 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
         if (r != IQ_OK) return r;
     }
     // batch norm reads the sums and both extremes; SQ of ReLU(acc) only the maxima
-    const unsigned want = use_bn ? (TC_STATS_SUM | TC_STATS_LO) : (relu ? 0u : TC_STATS_LO);
+    // (the batch-norm deviation pass computes the per-channel extremes itself)
+    const unsigned want = use_bn ? (TC_STATS_SUM | TC_STATS_NOEXT) : (relu ? 0u : TC_STATS_LO);
     r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done,
                     (const __half*)x_f16, want);
     if (r != IQ_OK) return r;

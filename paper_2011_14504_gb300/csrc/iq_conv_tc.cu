@@ -63,6 +63,8 @@ constexpr int ST_SUM32 = 4;
 // only the extremes over the whole output are read (SQ without batch norm): the kernel keeps
 // per-thread extremes and writes them to channel 0 once per warp
 constexpr int ST_GMAX = 8;
+// no extremes at all (TC_STATS_NOEXT: batch norm's deviation pass takes them)
+constexpr int ST_NOEXT = (int)TC_STATS_NOEXT;
 
 struct TcP {
     int mode, out;
@@ -1202,13 +1204,16 @@ __device__ __forceinline__ void col_stats(const TcP& p, const int* r, bool valid
                                           int* __restrict__ hi_c, int* __restrict__ lo_c) {
     long long my_sum = 0;
     int my_hi = INT_MIN, my_lo = INT_MAX;
-    const bool want_lo = p.st_mask & TC_STATS_LO, want_sum = p.st_mask & TC_STATS_SUM;
-    const bool sum32 = p.st_mask & ST_SUM32;
+    const bool want_hi = !(p.st_mask & ST_NOEXT);
+    const bool want_lo = want_hi && (p.st_mask & TC_STATS_LO);
+    const bool want_sum = p.st_mask & TC_STATS_SUM, sum32 = p.st_mask & ST_SUM32;
 #pragma unroll
     for (int j = 0; j < LDW; j++) {
         const int v = r[j];
-        const int mx = __reduce_max_sync(0xffffffffu, valid ? v : INT_MIN);
-        if (lane == j) my_hi = mx;
+        if (want_hi) {
+            const int mx = __reduce_max_sync(0xffffffffu, valid ? v : INT_MIN);
+            if (lane == j) my_hi = mx;
+        }
         if (want_lo) {
             const int mn = __reduce_min_sync(0xffffffffu, valid ? v : INT_MAX);
             if (lane == j) my_lo = mn;
@@ -1226,10 +1231,10 @@ __device__ __forceinline__ void col_stats(const TcP& p, const int* r, bool valid
         }
     }
     const int gcol = c0 + lane;
-    if (lane < LDW && gcol < p.ncols && my_hi != INT_MIN) {
-        atomicMax(&hi_c[gcol], my_hi);
-        if (want_lo) atomicMin(&lo_c[gcol], my_lo);
-        if (want_sum) atomicAdd(&s1[gcol], (unsigned long long)my_sum);
+    if (lane < LDW && gcol < p.ncols) {
+        if (want_hi && my_hi != INT_MIN) atomicMax(&hi_c[gcol], my_hi);
+        if (want_lo && my_lo != INT_MAX) atomicMin(&lo_c[gcol], my_lo);
+        if (want_sum && my_sum) atomicAdd(&s1[gcol], (unsigned long long)my_sum);
     }
 }
 
@@ -2457,7 +2462,8 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     p.M = (int64_t)p.N * p.P * p.Q;
     p.ncols = p.K;
     p.kdim = d->r * d->s * d->c;
-    p.st_mask = (int)(st_mask & (TC_STATS_SUM | TC_STATS_LO)) | (p.kdim <= 4095 ? ST_SUM32 : 0);
+    p.st_mask = (int)(st_mask & (TC_STATS_SUM | TC_STATS_LO | TC_STATS_NOEXT)) |
+                (p.kdim <= 4095 ? ST_SUM32 : 0);
     if (!(st_mask & TC_STATS_SUM)) p.st_mask |= ST_GMAX;   // no batch norm: one scale only
     p.kpad = (p.kdim + 63) / 64 * 64;
     p.tap_mode = (d->c % 64) == 0;

@@ -10,6 +10,7 @@ namespace iq {
 // per-channel statistics of the forward beyond the maximum (always written)
 constexpr unsigned TC_STATS_SUM = 1;   // the column sums (the batch-norm mean)
 constexpr unsigned TC_STATS_LO = 2;    // the column minima
+constexpr unsigned TC_STATS_NOEXT = 16; // no extremes either: a later pass computes them
 
 // Forward convolution on the 5th-generation tensor cores when the shape is
 // supported; sets *done = false (and enqueues nothing) otherwise.  Writes the int32
