@@ -232,11 +232,7 @@ __global__ void __launch_bounds__(kThreads) k_comb8(Terms T, int concat, int64_t
     }
 }
 
-// The same two passes with a fixed 8-channel group per thread: the launch has a multiple
-// of c_out / 8 threads, so thread t always owns group t % (c_out / 8) and keeps the F / B
-// rows of the (at most two) operands covering it in registers; it walks the pixels
-// t / (c_out / 8), + T / (c_out / 8), ...  Per 8 outputs the loads are one 8- or 16-byte
-// load per operand.
+// The operands covering a channel group of the output (at most two in k_comb4r).
 struct Cover {
     int n;              // operands covering the group (0..2)
     int id0, id1;
@@ -271,25 +267,38 @@ __device__ __forceinline__ const TermDev& term_at(const Terms& T, int i) {
     }
 }
 
-__device__ __forceinline__ void load8p(const void* codes, int is16, int64_t idx, int32_t v[8]) {
+// 4 channels of one pixel as int32 (int16 codes: one 8-byte load, int8: one 4-byte load)
+__device__ __forceinline__ void load4p(const void* codes, int is16, int64_t idx, int32_t v[4]) {
     if (is16) {
-        const int4 q = __ldg(reinterpret_cast<const int4*>((const int16_t*)codes + idx));
-        const int w[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-        for (int j = 0; j < 4; j++) {
-            v[2 * j] = (int32_t)(int16_t)(w[j] & 0xffff);
-            v[2 * j + 1] = (int32_t)(w[j] >> 16);
-        }
+        const int2 q = __ldg(reinterpret_cast<const int2*>((const int16_t*)codes + idx));
+        v[0] = (int32_t)(int16_t)(q.x & 0xffff);
+        v[1] = q.x >> 16;
+        v[2] = (int32_t)(int16_t)(q.y & 0xffff);
+        v[3] = q.y >> 16;
     } else {
-        const int2 q = __ldg(reinterpret_cast<const int2*>((const int8_t*)codes + idx));
-        const int w[2] = {q.x, q.y};
+        const int q = __ldg(reinterpret_cast<const int*>((const int8_t*)codes + idx));
 #pragma unroll
-        for (int j = 0; j < 8; j++) v[j] = (int32_t)(int8_t)((w[j >> 2] >> (8 * (j & 3))) & 0xff);
+        for (int j = 0; j < 4; j++) v[j] = (int32_t)(int8_t)((q >> (8 * j)) & 0xff);
     }
 }
 
+// z of 4 channels: F0 v0 + F1 v1 + (B0 + B1), exact in int64 (|z| < 2^50 by the choice of
+// P, and the two offsets are added first, which changes no sum)
+__device__ __forceinline__ void comb_z4(const long long (&f0)[4], const long long (&f1)[4],
+                                        const long long (&bs)[4], const int32_t (&v0)[4],
+                                        const int32_t (&v1)[4], int64_t (&z)[4]) {
+#pragma unroll
+    for (int j = 0; j < 4; j++) z[j] = (int64_t)f0[j] * v0[j] + (int64_t)f1[j] * v1[j] + bs[j];
+}
+
+// The two passes with a fixed 4-channel group per thread: the launch has a multiple of
+// c_out / 4 threads, so thread t always owns group t % (c_out / 4), keeps the F rows of the
+// (at most two) operands covering it and their summed B rows in registers (24 registers,
+// about half of an 8-channel group's, for twice the resident warps), and walks the pixels
+// t / (c_out / 4), + T / (c_out / 4), ... two at a time, both pixels' loads in flight
+// together.
 template <int PASS>
-__global__ void __launch_bounds__(kThreads) k_comb8r(Terms T, int concat, int64_t npix, int cgs,
+__global__ void __launch_bounds__(kThreads, 3) k_comb4r(Terms T, int concat, int64_t npix, int cgs,
                                                      int relu, const long long* __restrict__ F,
                                                      const long long* __restrict__ B,
                                                      CombHdr* hdr, int8_t* __restrict__ out,
@@ -304,53 +313,72 @@ __global__ void __launch_bounds__(kThreads) k_comb8r(Terms T, int concat, int64_
     const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int g = (int)(t % cgs);
     const int64_t pstride = tcount / cgs;
-    const int co0 = 8 * g;
+    const int co0 = 4 * g;
     Cover cv;
     cover_of(T, concat, co0, cv);
-    long long f0[8], b0[8], f1[8], b1[8];
+    long long f0[4], f1[4], bs[4];
     const TermDev& t0 = term_at(T, cv.id0);
     const TermDev& t1 = term_at(T, cv.id1);
 #pragma unroll
-    for (int j = 0; j < 8; j++) {
+    for (int j = 0; j < 4; j++) {
         f0[j] = cv.n > 0 ? F[t0.base + cv.ch0 + j] : 0;
-        b0[j] = cv.n > 0 ? B[t0.base + cv.ch0 + j] : 0;
         f1[j] = cv.n > 1 ? F[t1.base + cv.ch1 + j] : 0;
-        b1[j] = cv.n > 1 ? B[t1.base + cv.ch1 + j] : 0;
+        bs[j] = (cv.n > 0 ? B[t0.base + cv.ch0 + j] : 0) + (cv.n > 1 ? B[t1.base + cv.ch1 + j] : 0);
     }
     const void* base0 = t0.codes;
     const void* base1 = t1.codes;
     const int is0 = t0.is16, is1 = t1.is16, c0 = t0.c, c1 = t1.c, bc0 = t0.bcast, bc1 = t1.bcast;
+    const int n0 = cv.n;
     uint64_t mx = 0;
-    for (int64_t pix = t / cgs; pix < npix; pix += pstride) {
-        const int64_t img = any_bcast ? (int64_t)udiv((uint64_t)pix, dhw) : 0;
-        int32_t v0[8] = {0, 0, 0, 0, 0, 0, 0, 0}, v1[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-        if (cv.n > 0) load8p(base0, is0, (bc0 ? img : pix) * c0 + cv.ch0, v0);
-        if (cv.n > 1) load8p(base1, is1, (bc1 ? img : pix) * c1 + cv.ch1, v1);
-        int64_t z[8];
-#pragma unroll
-        for (int j = 0; j < 8; j++)
-            z[j] = (int64_t)f0[j] * v0[j] + (int64_t)b0[j] + (int64_t)f1[j] * v1[j] + (int64_t)b1[j];
+    auto one = [&](int64_t pix, const int32_t (&v0)[4], const int32_t (&v1)[4]) {
+        int64_t z[4];
+        comb_z4(f0, f1, bs, v0, v1, z);
         if (PASS == 0) {
 #pragma unroll
-            for (int j = 0; j < 8; j++) {
-                int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
-                uint64_t a = (uint64_t)(zz < 0 ? -zz : zz);
+            for (int j = 0; j < 4; j++) {
+                const int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
+                const uint64_t a = (uint64_t)(zz < 0 ? -zz : zz);
                 mx = a > mx ? a : mx;
             }
         } else {
-            uint32_t w[2] = {0u, 0u};
+            uint32_t w = 0u;
 #pragma unroll
-            for (int j = 0; j < 8; j++) {
-                int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
+            for (int j = 0; j < 4; j++) {
+                const int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
                 int64_t c = 0;
                 if (M) {
-                    uint64_t num = ((uint64_t)(zz + (int64_t)M) << 8) + M;
+                    const uint64_t num = ((uint64_t)(zz + (int64_t)M) << 8) + M;
                     c = clamp64((int64_t)udiv(num, d2m) - 128, -127, 127);
                 }
-                w[j >> 2] |= ((uint32_t)c & 0xffu) << (8 * (j & 3));
+                w |= ((uint32_t)c & 0xffu) << (8 * j);
             }
-            *reinterpret_cast<uint2*>(out + pix * (int64_t)cgs * 8 + co0) = make_uint2(w[0], w[1]);
+            *reinterpret_cast<uint32_t*>(out + pix * (int64_t)cgs * 4 + co0) = w;
         }
+    };
+    int64_t pix = t / cgs;
+    for (; pix + pstride < npix; pix += 2 * pstride) {
+        const int64_t pb = pix + pstride;
+        const int64_t ia = any_bcast ? (int64_t)udiv((uint64_t)pix, dhw) : 0;
+        const int64_t ib = any_bcast ? (int64_t)udiv((uint64_t)pb, dhw) : 0;
+        int32_t a0[4] = {0, 0, 0, 0}, a1[4] = {0, 0, 0, 0}, b0[4] = {0, 0, 0, 0},
+                b1[4] = {0, 0, 0, 0};
+        if (n0 > 0) {
+            load4p(base0, is0, (bc0 ? ia : pix) * c0 + cv.ch0, a0);
+            load4p(base0, is0, (bc0 ? ib : pb) * c0 + cv.ch0, b0);
+        }
+        if (n0 > 1) {
+            load4p(base1, is1, (bc1 ? ia : pix) * c1 + cv.ch1, a1);
+            load4p(base1, is1, (bc1 ? ib : pb) * c1 + cv.ch1, b1);
+        }
+        one(pix, a0, a1);
+        one(pb, b0, b1);
+    }
+    if (pix < npix) {
+        const int64_t ia = any_bcast ? (int64_t)udiv((uint64_t)pix, dhw) : 0;
+        int32_t a0[4] = {0, 0, 0, 0}, a1[4] = {0, 0, 0, 0};
+        if (n0 > 0) load4p(base0, is0, (bc0 ? ia : pix) * c0 + cv.ch0, a0);
+        if (n0 > 1) load4p(base1, is1, (bc1 ? ia : pix) * c1 + cv.ch1, a1);
+        one(pix, a0, a1);
     }
     if (PASS == 0) {
         mx = warp_max_u64(mx);
@@ -515,18 +543,21 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
     IQ_LAUNCH_CHECK();
     const int64_t total = n * hw * (int64_t)c_out;
     bool vec = c_out % 8 == 0 && ((uintptr_t)out & 7) == 0;
+    bool vec4 = c_out % 4 == 0 && ((uintptr_t)out & 3) == 0;
     bool any_bcast = false;
     for (int i = 0; i < n_terms; i++) {
         const TermDev& t = T.t[i];
         vec = vec && t.c % 8 == 0 && t.c_offset % 8 == 0 &&
               ((uintptr_t)t.codes & (t.is16 ? 15 : 7)) == 0;
+        vec4 = vec4 && t.c % 4 == 0 && t.c_offset % 4 == 0 &&
+               ((uintptr_t)t.codes & (t.is16 ? 7 : 3)) == 0;
         any_bcast = any_bcast || t.bcast;
     }
     const UDiv dhw = make_udiv((uint64_t)hw);
-    // at most two operands cover any 8-channel group: sums of up to two operands, and
+    // at most two operands cover any 4-channel group: sums of up to two operands, and
     // concatenations whose ranges overlap at most pairwise (checked per group on the host)
-    bool two = vec;
-    for (int co = 0; co < c_out && two; co += 8) {
+    bool two = vec4;
+    for (int co = 0; co < c_out && two; co += 4) {
         int nc = 0;
         for (int i = 0; i < n_terms; i++) {
             const TermDev& t = T.t[i];
@@ -536,7 +567,7 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
         two = nc <= 2;
     }
     if (two) {
-        const int cgs = c_out / 8;
+        const int cgs = c_out / 4;
         const int64_t npix = n * hw;
         // a multiple of cgs threads, about 8 blocks of 256 per SM
         int64_t gcd = cgs, b2 = kThreads;
@@ -547,12 +578,12 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
         want = (want + unit - 1) / unit * unit;
         if (want < unit) want = unit;
         const int g = (int)want;
-        k_comb8r<0><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
+        k_comb4r<0><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
                                             dhw, any_bcast);
         IQ_LAUNCH_CHECK();
         k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
         IQ_LAUNCH_CHECK();
-        k_comb8r<1><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
+        k_comb4r<1><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
                                             dhw, any_bcast);
         IQ_LAUNCH_CHECK();
         return IQ_OK;

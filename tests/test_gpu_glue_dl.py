@@ -92,6 +92,22 @@ def test_combine_concat_aspp():
     run_combine(specs, n, hw, 5 * cb, True, False)
 
 
+@pytest.mark.parametrize("n,hw,c", [(3, 7 * 13, 36), (2, 65 * 65, 256)])
+def test_combine_four_channel_groups(n, hw, c):
+    # c_out a multiple of 4 (not of 8 in the first case) and an odd pixel count: the
+    # 4-channel kernel, its pairs of pixels and its single-pixel tail; then a full-size
+    # bottleneck join (65 x 65 x 256)
+    g = np.random.default_rng(18 + c)
+    X = g.integers(-32767, 32768, size=(n, hw, c)).astype(np.int16)
+    sc = g.integers(-127, 128, size=(n, hw, c)).astype(np.int8)
+    gam = g.integers(-127, 128, size=c).astype(np.int32)
+    bet = g.integers(-127, 128, size=c).astype(np.int32)
+    run_combine([(X, 2.0 ** -15 * 1.9, 0, False, gam, bet), (sc, 0.013, 0, False, None, None)],
+                n, hw, c, False, True)
+    run_combine([(sc, 0.02, 0, False, None, None), (X, 2.0 ** -15, 0, False, gam, bet)],
+                n, hw, c, False, False)
+
+
 def test_combine_edge_cases():
     # all zero, a single pixel, a single channel
     run_combine([(np.zeros((1, 5, 8), np.int8), 0.5, 0, False, None, None)], 1, 5, 8, False, False)
