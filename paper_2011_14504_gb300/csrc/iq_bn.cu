@@ -47,9 +47,9 @@ struct RowGrid {
     dim3 grid;
 };
 
-RowGrid row_grid(int64_t m, int32_t C4, int target_blocks = 152 * 8) {
+RowGrid row_grid(int64_t m, int32_t C4, int target_blocks = 152 * 8, int cg_max = 32) {
     RowGrid g;
-    g.cg = 32;
+    g.cg = cg_max;
     while (g.cg > 1 && g.cg > C4) g.cg >>= 1;
     g.rl = kThreads / g.cg;
     const int64_t bx = (C4 + g.cg - 1) / g.cg;
@@ -518,6 +518,13 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
 // Division by 2M for E_2 = SQ(z, k_e2): the numerator 2^k (z + M) + M is below 2^32 for the
 // paper's widths (|z| <= 127 * 127, k_e2 <= 16), where a 32-bit invariant divisor (Granlund
 // & Montgomery, Sec. 4, at N = 32) replaces the 64-bit one.
+// Per channel, E_2 depends on e_y alone and the output code on (sign X, e_y) alone, so
+// both are tabulated once per call (k_bnb_tab2 / k_bnb_tab3, the same arithmetic as the
+// per-element form) and passes 2 and 3 look them up in shared memory.
+constexpr int kTab2 = 256;          // entries per channel: e_y + 128
+constexpr int kTab3 = 3 * 256;      // (sign X + 1) 256 + e_y + 128
+constexpr int kTabCG = 8;           // channel groups (32 channels) per block of passes 2 / 3
+
 struct E2Div {
     uint64_t M;
     UDiv div;          // 64-bit divisor by 2M
@@ -540,6 +547,8 @@ struct BnBwd {
     unsigned* zmax;           // [1]
     int* pe;                  // [1]
     E2Div* e2div;             // [1]
+    int16_t* t2;              // [C][256]: E_2 of e_y = -128 .. 127
+    int8_t* t3;               // [C][3][256]: the output code of (sign X, e_y)
     double* scal;             // [2]: s_e2, s_out
     double* kap;              // [C] per-channel constants of d x (fin 2)
     double* lam;
@@ -567,6 +576,8 @@ static BnBwd bnb_carve(WsCursor& cur, int32_t C) {
     w.lam = cur.take<double>(C);
     w.wc = cur.take<double>(C);
     w.red = cur.take<unsigned long long>(4);
+    w.t2 = cur.take<int16_t>((size_t)kTab2 * C);
+    w.t3 = cur.take<int8_t>((size_t)kTab3 * C);
     return w;
 }
 
@@ -689,29 +700,49 @@ __device__ __forceinline__ int e2_code(int z, const E2Div& d, int k) {
     return (int)clamp64(c, -qmax(k), qmax(k));
 }
 
-// E_2 = SQ_kE2(e_y gamma): per channel sum E_2, sum E_2 X, sum sign X, and the extremes of
-// E_2 per sign class of X (-1, 0, +1).  The extremes travel packed as (max, -min) int16
-// pairs (|E_2| <= 2^15 - 1), one __vmaxs2 per class.
+// the E_2 table: t2[c][e_y + 128] = SQ_kE2(e_y gamma_c)
+__global__ void k_bnb_tab2(const int32_t* __restrict__ gam, int32_t C, int k_e2, BnBwd w) {
+    const E2Div d = *w.e2div;
+    const int64_t n = (int64_t)C * kTab2;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i >> 8), ey = (int)(i & 255) - 128;
+        w.t2[i] = (int16_t)e2_code(ey * gam[c], d, k_e2);
+    }
+}
+
+// the block's 32 channel tables (rows of `row` bytes) into shared memory, 16 bytes a thread
+__device__ __forceinline__ void load_tables(const void* __restrict__ src, int64_t c0, int nch,
+                                            int row, uint8_t* dst) {
+    const int4* s4 = reinterpret_cast<const int4*>((const uint8_t*)src + c0 * row);
+    int4* d4 = reinterpret_cast<int4*>(dst);
+    const int n16 = nch * row / 16;
+    for (int i = threadIdx.x; i < n16; i += blockDim.x) d4[i] = s4[i];
+}
+
+// E_2 = SQ_kE2(e_y gamma) (from the table): per channel sum E_2, sum E_2 X, sum sign X, and
+// the extremes of E_2 per sign class of X (-1, 0, +1).  The extremes travel packed as (max,
+// -min) int16 pairs (|E_2| <= 2^15 - 1), one __vmaxs2 per class.
 __global__ void __launch_bounds__(kThreads, 3) k_bnb_pass2(const int8_t* __restrict__ ea,
                                                         const int8_t* __restrict__ a,
                                                         const int16_t* __restrict__ X,
-                                                        const int32_t* __restrict__ gam,
-                                                        int64_t m, int32_t C, int CG, int k_e2,
-                                                        BnBwd w) {
+                                                        int64_t m, int32_t C, int CG, BnBwd w) {
     __shared__ long long sh_e[kThreads * 4], sh_x[kThreads * 4];
+    __shared__ __align__(16) int16_t tab[4 * kTabCG * kTab2];
     __shared__ int sh_s[kThreads * 4];
     __shared__ uint32_t sh_p[3][kThreads * 4];
     const int C4 = C >> 2;
     const int cg = threadIdx.x % CG, rl = threadIdx.x / CG, RL = blockDim.x / CG;
     const int g = blockIdx.x * CG + cg;
     const bool act = g < C4;
-    const E2Div d = *w.e2div;
     constexpr uint32_t kEmpty = 0x80008000u;      // (-32768, -32768): no element yet
-    int gm[4] = {0, 0, 0, 0};
-    if (act) {
-#pragma unroll
-        for (int j = 0; j < 4; j++) gm[j] = gam[4 * g + j];
+    {
+        const int64_t c0 = 4 * (int64_t)blockIdx.x * CG;
+        const int nch = (int)min((int64_t)4 * CG, (int64_t)C - c0);
+        load_tables(w.t2, c0, nch, 2 * kTab2, reinterpret_cast<uint8_t*>(tab));
     }
+    __syncthreads();
+    const int16_t* tb = tab + 4 * cg * kTab2;
     long long se64[4] = {0, 0, 0, 0}, sx[4] = {0, 0, 0, 0};
     int ss[4] = {0, 0, 0, 0};
     uint32_t pk[4][3];
@@ -725,13 +756,11 @@ __global__ void __launch_bounds__(kThreads, 3) k_bnb_pass2(const int8_t* __restr
         while (r < m) {
             // int32 partial sums of E_2 over at most 2^15 rows (|E_2| < 2^15)
             int se[4] = {0, 0, 0, 0};
-            for (int it = 0; it < 32768 && r < m; it++, r += step) {
-                int e0[4], a0[4], x0[4];
-                load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
+            auto row = [&](const int (&e0)[4], const int (&a0)[4], const int (&x0)[4]) {
 #pragma unroll
                 for (int j = 0; j < 4; j++) {
                     const int ey = a0[j] > 0 ? e0[j] : 0;
-                    const int e2 = e2_code(ey * gm[j], d, k_e2);
+                    const int e2 = tb[j * kTab2 + ey + 128];
                     const int sgn = (x0[j] > 0) - (x0[j] < 0);
                     se[j] += e2;
                     sx[j] += (long long)(e2 * x0[j]);     // |E_2 X| < 2^30
@@ -741,6 +770,21 @@ __global__ void __launch_bounds__(kThreads, 3) k_bnb_pass2(const int8_t* __restr
                     else if (sgn == 0) pk[j][1] = __vmaxs2(pk[j][1], cand);
                     else pk[j][2] = __vmaxs2(pk[j][2], cand);
                 }
+            };
+            // two rows per iteration, both rows' loads in flight together
+            int it = 0;
+            for (; it < 32767 && r + step < m; it += 2, r += 2 * step) {
+                int e0[4], a0[4], x0[4], e1[4], a1[4], x1[4];
+                load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
+                load4_e_a_x((r + step) * C4 + g, ea, a, X, e1, a1, x1);
+                row(e0, a0, x0);
+                row(e1, a1, x1);
+            }
+            if (it < 32768 && r < m) {
+                int e0[4], a0[4], x0[4];
+                load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
+                row(e0, a0, x0);
+                r += step;
             }
 #pragma unroll
             for (int j = 0; j < 4; j++) se64[j] += se[j];
@@ -853,42 +897,67 @@ __global__ void __launch_bounds__(kFinThreads) k_bnb_fin2c(BnBwd w, int32_t C, i
     if (c == 0) { *w.pe = pe; w.scal[1] = ldexp(M, 1 - k_e); *s_out = w.scal[1]; }
 }
 
-__global__ void __launch_bounds__(kThreads) k_bnb_pass3(const int8_t* __restrict__ ea,
-                                                        const int8_t* __restrict__ a,
-                                                        const int16_t* __restrict__ X,
-                                                        const int32_t* __restrict__ gam,
-                                                        int64_t m, int32_t C, int k_e2, int k_e,
-                                                        BnBwd w, int8_t* __restrict__ out) {
+// the output-code table: t3[c][(s + 1) 256 + e_y + 128] = clip(floor((fw E_2 + fk s + fl) /
+// 2^P)) with E_2 = SQ_kE2(e_y gamma_c)
+__global__ void k_bnb_tab3(const int32_t* __restrict__ gam, int32_t C, int k_e2, int k_e,
+                           BnBwd w) {
     const E2Div d = *w.e2div;
     const int pe = *w.pe;
     const int64_t eq = qmax(k_e);
-    const int C4 = C >> 2;
-    const int64_t T = (int64_t)gridDim.x * blockDim.x;
-    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int g = (int)(t % C4);
-    const int64_t rstride = T / C4;
-    int gm[4];
-    long long fw[4], fk[4], fl[4];
-#pragma unroll
-    for (int j = 0; j < 4; j++) {
-        gm[j] = gam[4 * g + j];
-        fw[j] = w.fw[4 * g + j]; fk[j] = w.fk[4 * g + j]; fl[j] = w.fl[4 * g + j];
+    const int64_t n = (int64_t)C * kTab3;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i / kTab3), r = (int)(i - (int64_t)c * kTab3);
+        const int sgn = (r >> 8) - 1, ey = (r & 255) - 128;
+        const int e2 = e2_code(ey * gam[c], d, k_e2);
+        const long long tt = w.fw[c] * (long long)e2 + w.fk[c] * (long long)sgn + w.fl[c];
+        w.t3[i] = (int8_t)clamp64(tt >> pe, -eq, eq);
     }
-    for (int64_t r = t / C4; r < m; r += rstride) {
-        int64_t v = r * C4 + g;
-        int e[4], am[4], x[4];
-        load4_e_a_x(v, ea, a, X, e, am, x);
+}
+
+// e = the output code of (sign X, e_y) per element, from the block's tables in shared memory
+__global__ void __launch_bounds__(kThreads) k_bnb_pass3(const int8_t* __restrict__ ea,
+                                                        const int8_t* __restrict__ a,
+                                                        const int16_t* __restrict__ X,
+                                                        int64_t m, int32_t C, int CG, BnBwd w,
+                                                        int8_t* __restrict__ out) {
+    __shared__ __align__(16) int8_t tab[4 * kTabCG * kTab3];
+    const int C4 = C >> 2;
+    const int cg = threadIdx.x % CG, rl = threadIdx.x / CG, RL = blockDim.x / CG;
+    const int g = blockIdx.x * CG + cg;
+    {
+        const int64_t c0 = 4 * (int64_t)blockIdx.x * CG;
+        const int nch = (int)min((int64_t)4 * CG, (int64_t)C - c0);
+        load_tables(w.t3, c0, nch, kTab3, reinterpret_cast<uint8_t*>(tab));
+    }
+    __syncthreads();
+    if (g >= C4) return;
+    const int8_t* tb = tab + 4 * cg * kTab3;
+    const int64_t step = (int64_t)gridDim.y * RL;
+    auto code4 = [&](const int (&e)[4], const int (&am)[4], const int (&x)[4]) {
         uint32_t o = 0;
 #pragma unroll
         for (int j = 0; j < 4; j++) {
-            int ey = am[j] > 0 ? e[j] : 0;
-            int e2 = e2_code(ey * gm[j], d, k_e2);
-            int sgn = (x[j] > 0) - (x[j] < 0);
-            long long tt = fw[j] * (long long)e2 + fk[j] * (long long)sgn + fl[j];
-            int64_t c = clamp64(tt >> pe, -eq, eq);
-            o |= ((uint32_t)c & 0xffu) << (8 * j);
+            const int ey = am[j] > 0 ? e[j] : 0;
+            const int sg = (x[j] > 0) - (x[j] < 0);
+            o |= ((uint32_t)(uint8_t)tb[j * kTab3 + (sg + 1) * 256 + ey + 128]) << (8 * j);
         }
-        reinterpret_cast<uint32_t*>(out)[v] = o;
+        return o;
+    };
+    int64_t r = (int64_t)blockIdx.y * RL + rl;
+    // four rows per iteration: all their loads in flight together
+    for (; r + 3 * step < m; r += 4 * step) {
+        int e[4][4], am[4][4], x[4][4];
+#pragma unroll
+        for (int u = 0; u < 4; u++) load4_e_a_x((r + u * step) * C4 + g, ea, a, X, e[u], am[u], x[u]);
+#pragma unroll
+        for (int u = 0; u < 4; u++)
+            reinterpret_cast<uint32_t*>(out)[(r + u * step) * C4 + g] = code4(e[u], am[u], x[u]);
+    }
+    for (; r < m; r += step) {
+        int e[4], am[4], x[4];
+        load4_e_a_x(r * C4 + g, ea, a, X, e, am, x);
+        reinterpret_cast<uint32_t*>(out)[r * C4 + g] = code4(e, am, x);
     }
 }
 
@@ -963,7 +1032,11 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     IQ_LAUNCH_CHECK();
     k_bnb_fin1<<<1, 1, 0, st>>>(w, s_e, b.k_gamma, k_e2);
     IQ_LAUNCH_CHECK();
-    k_bnb_pass2<<<rg.grid, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, rg.cg, k_e2, w);
+    const int tb2 = (int)(((int64_t)c * kTab2 + kThreads - 1) / kThreads);
+    k_bnb_tab2<<<tb2 < 152 * 4 ? tb2 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, w);
+    IQ_LAUNCH_CHECK();
+    RowGrid rt = row_grid(m, c / 4, 152 * 8, kTabCG);
+    k_bnb_pass2<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w);
     IQ_LAUNCH_CHECK();
     const int fb = (c + kFinThreads - 1) / kFinThreads;
     k_bnb_fin2a<<<fb, kFinThreads, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma);
@@ -972,8 +1045,10 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     IQ_LAUNCH_CHECK();
     k_bnb_fin2c<<<fb, kFinThreads, 0, st>>>(w, c, 8, s_e_out);
     IQ_LAUNCH_CHECK();
-    ChanGrid g3 = chan_grid(m, c / 4, 152 * 16);
-    k_bnb_pass3<<<g3.blocks, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, k_e2, 8, w, e);
+    const int tb3 = (int)(((int64_t)c * kTab3 + kThreads - 1) / kThreads);
+    k_bnb_tab3<<<tb3 < 152 * 4 ? tb3 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, 8, w);
+    IQ_LAUNCH_CHECK();
+    k_bnb_pass3<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w, e);
     IQ_LAUNCH_CHECK();
     if (dgamma)
         IQ_CUDA_CHECK(cudaMemcpyAsync(dgamma, w.sg, sizeof(int64_t) * c, cudaMemcpyDeviceToDevice, st));
