@@ -405,12 +405,15 @@ def run_ours(args, rank, world, local):
     iq.iq_device_status(stream)     # raises if a bounded device wait gave up
 
     # per-operation attribution (eager steps, CUDA events around each conv call on the stream)
+    # and, inside those calls, events around every launch of the tensor-core conv kernels
     orig = {k: getattr(iq, k) for k in ("iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad")}
     for k, f in orig.items():
         setattr(iq, k, timed(k, f))
+    iq.iq_kernel_timing_begin()
     for _ in range(args.steps):
         wl.step(net, img, lab)
     torch.cuda.synchronize(dev)
+    ktimes = iq.iq_kernel_timing_end()
     for k, f in orig.items():
         setattr(iq, k, f)
     ms_total = t_start.elapsed_time(t_end)
@@ -419,22 +422,32 @@ def run_ours(args, rank, world, local):
     macs = wl.macs(net)
     tops = 2 * macs * world / (ms_step * 1e-3) / 1e12
 
-    # roofline of the dominant conv operation (per-call event durations)
+    # roofline of the dominant kernel: the tensor-core conv kernel with the largest summed
+    # event time over the attribution steps; achieved = its algorithmic flops (2 x the MACs
+    # of the calls that launched it) / its summed launch time
     per = {}
     for kind, evs in op_events.items():
         per[kind] = sum(e0.elapsed_time(e1) for e0, e1, _ in evs)
-    dom = max(per, key=per.get)
-    conv_macs = wl.conv_macs(net)
-    n_calls = len(op_events[dom]) // args.steps
-    ms_call = per[dom] / len(op_events[dom])
-    flops_call = 2 * conv_macs[dom] / n_calls
+    byk = {}
+    for r in ktimes:
+        t = byk.setdefault(r["kernel"], {"ms": 0.0, "macs": 0.0, "launches": 0})
+        t["ms"] += r["ms"]
+        t["macs"] += r["macs"]
+        t["launches"] += r["launches"]
     pk, pk_kind = peaks()
     peak_tf = pk.get("bf16_tflops_sustained", pk.get("bf16_tflops"))
-    achieved = flops_call / (ms_call * 1e-3) / 1e12
-    roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak_tf,
-                "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": None,
+    dk = max(byk, key=lambda k: byk[k]["ms"])
+    kt = byk[dk]
+    achieved = 2 * kt["macs"] / (kt["ms"] * 1e-3) / 1e12
+    roofline = {"bound": "tensor", "kernel": iq.KERNEL_NAMES.get(dk, str(dk)),
+                "achieved": achieved, "peak": peak_tf, "unit": "TFLOP/s",
+                "frac": achieved / peak_tf, "traffic": None,
                 "peak_source": f"{pk_kind} fp16/bf16 dense sustained (MEASURED_PEAKS.json)",
-                "share_of_step": per[dom] / ms_total,
+                "launches_per_step": kt["launches"] / args.steps,
+                "kernel_ms_per_step": kt["ms"] / args.steps,
+                "share_of_step": kt["ms"] / args.steps / (ms_total / args.steps),
+                "kernels_ms_per_step": {iq.KERNEL_NAMES.get(k, str(k)): v["ms"] / args.steps
+                                        for k, v in byk.items()},
                 "op_ms_per_step": {k: v / args.steps for k, v in per.items()}}
 
     # end to end: host (pinned) inputs copied in, a result scalar read back, every step

@@ -104,6 +104,31 @@ unsigned long long iq_launch_count(void);
  * Call it after a sequence of calls (a training step) to learn whether they completed. */
 iq_status iq_device_status(int32_t* code, iq_stream stream);
 
+/* Kernel timing -- a measurement aid (the paper has no counterpart).  Between
+ * iq_kernel_timing_begin and iq_kernel_timing_end, every launch of a tensor-core convolution
+ * kernel (up to 4096 of them) is bracketed by a pair of CUDA events recorded on its launching
+ * stream, and tagged with the kernel, the calling operation and the operation's algorithmic
+ * multiply-accumulates N P Q K R S C / groups (counted once per call, on its first bracketed
+ * launch).  Use it on eagerly launched calls, not inside a CUDA graph capture.
+ * iq_kernel_timing_end waits for the recorded events, writes one iq_kernel_time per
+ * (kernel, op) pair seen (at most `capacity`, the count in *n_out), and stops recording.
+ * Errors: IQ_ERR_INVALID_ARG for null pointers, IQ_ERR_CUDA when an event call fails. */
+enum {
+    IQ_KERNEL_CONV_PIXEL_MAJOR = 1,    /* all-TMA kernel, forward / data gradient (k_conv_tct)  */
+    IQ_KERNEL_CONV_CHANNEL_MAJOR = 2,  /* channel-major kernel, <= 128 output channels (k_conv_tcc) */
+    IQ_KERNEL_CONV_WGRAD = 3           /* all-TMA kernel, weight gradient                       */
+};
+typedef struct iq_kernel_time {
+    int32_t kernel;     /* IQ_KERNEL_CONV_* */
+    int32_t op;         /* 1 iq_conv_fwd, 2 iq_conv_dgrad, 3 iq_conv_wgrad */
+    int32_t launches;   /* bracketed launches */
+    int32_t pad;
+    double ms;          /* summed event time of those launches, milliseconds */
+    double macs;        /* summed algorithmic multiply-accumulates of their calls */
+} iq_kernel_time;
+iq_status iq_kernel_timing_begin(void);
+iq_status iq_kernel_timing_end(iq_kernel_time* out, int32_t capacity, int32_t* n_out);
+
 /* The stochastic rounding of Eqs. (SQ),(SR) draws, for element i, the Philox4x64-10 block with
  * key (seed, layer) and counter (i/8, step, tag, epoch).  epoch is a device-resident word of
  * the library, 0 until changed: iq_rq_epoch_advance adds 1 to it as a stream operation (so a

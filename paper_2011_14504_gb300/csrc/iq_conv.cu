@@ -465,6 +465,109 @@ static bool crs_overflow(const iq_conv_desc* d) {
     return crs * 127 * 127 >= (int64_t(1) << 31);
 }
 
+// algorithmic multiply-accumulates of one convolution pass: N P Q K R S C / groups
+static double conv_macs(const iq_conv_desc* d) {
+    const int64_t P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    const int64_t Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    return (double)d->n * P * Q * d->k * d->r * d->s * (double)(d->c / d->groups);
+}
+
+// ------------------------------------------------------------------ kernel timing
+
+namespace iq {
+namespace {
+
+constexpr int kKtCap = 4096;
+
+struct KtState {
+    bool on = false;
+    int n = 0;
+    int op = 0;
+    double pending_macs = 0.0;      // the current call's MACs, given to its first launch
+    cudaEvent_t ev[2 * kKtCap] = {};
+    int kernel[kKtCap] = {};
+    int opv[kKtCap] = {};
+    double macs[kKtCap] = {};
+};
+
+KtState& kt() {
+    static KtState* s = new KtState();
+    return *s;
+}
+
+}  // namespace
+
+void kt_set_op(int op, double macs) {
+    KtState& k = kt();
+    k.op = op;
+    k.pending_macs = macs;
+}
+
+void kt_pre(cudaStream_t st) {
+    KtState& k = kt();
+    if (!k.on || k.n >= kKtCap) return;
+    cudaEvent_t& e = k.ev[2 * k.n];
+    if (!e && cudaEventCreate(&e) != cudaSuccess) { e = nullptr; return; }
+    cudaEventRecord(e, st);
+}
+
+void kt_post(cudaStream_t st, int kernel) {
+    KtState& k = kt();
+    if (!k.on || k.n >= kKtCap || !k.ev[2 * k.n]) return;
+    cudaEvent_t& e = k.ev[2 * k.n + 1];
+    if (!e && cudaEventCreate(&e) != cudaSuccess) { e = nullptr; return; }
+    cudaEventRecord(e, st);
+    k.kernel[k.n] = kernel;
+    k.opv[k.n] = k.op;
+    k.macs[k.n] = k.pending_macs;
+    k.pending_macs = 0.0;
+    k.n++;
+}
+
+}  // namespace iq
+
+extern "C" iq_status iq_kernel_timing_begin(void) {
+    KtState& k = kt();
+    k.on = true;
+    k.n = 0;
+    k.pending_macs = 0.0;
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_kernel_timing_end(iq_kernel_time* out, int32_t capacity, int32_t* n_out) {
+    if (!out || !n_out || capacity < 0) return IQ_ERR_INVALID_ARG;
+    KtState& k = kt();
+    k.on = false;
+    int nout = 0;
+    iq_status r = IQ_OK;
+    for (int i = 0; i < k.n; i++) {
+        float ms = 0.0f;
+        if (cudaEventSynchronize(k.ev[2 * i + 1]) != cudaSuccess ||
+            cudaEventElapsedTime(&ms, k.ev[2 * i], k.ev[2 * i + 1]) != cudaSuccess) {
+            r = IQ_ERR_CUDA;
+            continue;
+        }
+        int j = 0;
+        while (j < nout && !(out[j].kernel == k.kernel[i] && out[j].op == k.opv[i])) j++;
+        if (j == nout) {
+            if (nout == capacity) continue;
+            out[j].kernel = k.kernel[i];
+            out[j].op = k.opv[i];
+            out[j].launches = 0;
+            out[j].pad = 0;
+            out[j].ms = 0.0;
+            out[j].macs = 0.0;
+            nout++;
+        }
+        out[j].launches++;
+        out[j].ms += ms;
+        out[j].macs += k.macs[i];
+    }
+    k.n = 0;
+    *n_out = nout;
+    return r;
+}
+
 extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
                                  const int8_t* w, const int32_t* gamma, const int32_t* beta,
                                  const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
@@ -475,6 +578,7 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     const int64_t nx = (int64_t)d->n * d->h * d->w * d->c;
     if (x_f16 && (nx % 16 || (((uintptr_t)x | (uintptr_t)x_f16) & 15))) return IQ_ERR_INVALID_ARG;
     if (crs_overflow(d)) return IQ_ERR_OVERFLOW_RISK;
+    kt_set_op(1, conv_macs(d));
     iq_bn_bits b = bn_bits_or_default(bits);
     if (use_bn) {
         if (!gamma || !beta || !bn_bits_valid(b)) return IQ_ERR_INVALID_ARG;
@@ -537,6 +641,7 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     size_t need = 0;
     iq_conv_dgrad_workspace_size(d, &need);
     if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    kt_set_op(2, conv_macs(d));
     cudaStream_t st = (cudaStream_t)stream;
     ConvP cp = make_params(d);
     WsCursor cur(ws, ws_bytes);
@@ -616,6 +721,7 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
     size_t need = 0;
     iq_conv_wgrad_workspace_size(d, &need);
     if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    kt_set_op(3, conv_macs(d));
     ConvP cp = make_params(d);
     // |G| < npq 127^2 must stay below 2^40 for the requantizer
     if ((double)cp.npq * 16129.0 >= 1099511627776.0) return IQ_ERR_OVERFLOW_RISK;

@@ -2316,9 +2316,11 @@ iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const CUten
     g.total = g.mt * g.nt * (p.slices > 1 ? p.slices : 1);
     g.nb = 1;
     const int grid = g.total < num_sms() ? g.total : num_sms();
+    kt_pre(st);
     k_conv_tct<BN, false><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(wmap, amap, omap, p, g, out32,
                                                                   out64, s1, hi, lo, err);
     IQ_LAUNCH_CHECK();
+    kt_post(st, IQ_KERNEL_CONV_PIXEL_MAJOR);
     return IQ_OK;
 }
 
@@ -2389,9 +2391,11 @@ iq_status try_launch_c(const __half* wf, int rows, const TcP& p, const int8_t* x
     int bw_log2 = 0;
     while ((1 << bw_log2) < t.BW) bw_log2++;
     const int grid = g.total < num_sms() ? g.total : num_sms();
+    kt_pre(st);
     k_conv_tcc<<<grid, THREADS_T, CfgT<256>::SMEM, st>>>(wmap, amap, p, g, bw_log2, out32, s1,
                                                           hi, lo, err);
     IQ_LAUNCH_CHECK();
+    kt_post(st, IQ_KERNEL_CONV_CHANNEL_MAJOR);
     *used = true;
     return IQ_OK;
 }
@@ -2768,10 +2772,12 @@ iq_status launch_tw(const CUtensorMap& emap, const CUtensorMap& xmap, const TcP&
     g.nb = nb < BN / 64 ? nb : BN / 64;
     const int grid = g.total < num_sms() ? g.total : num_sms();
     // (the output map is not read: the weight gradient writes its slabs with plain stores)
+    kt_pre(st);
     k_conv_tct<BN, true><<<grid, THREADS_T, CfgT<BN>::SMEM, st>>>(emap, xmap, emap, p, g, part,
                                                                  nullptr, amax, nullptr, nullptr,
                                                                  err);
     IQ_LAUNCH_CHECK();
+    kt_post(st, IQ_KERNEL_CONV_WGRAD);
     return IQ_OK;
 }
 

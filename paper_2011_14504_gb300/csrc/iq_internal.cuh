@@ -91,4 +91,11 @@ inline bool bn_bits_valid(const iq_bn_bits& b) {
            b.k_beta >= 2 && b.k_beta <= 16 && b.k_a >= 2 && b.k_a <= 8;
 }
 
+
+// kernel timing (iq_kernel_timing_begin / _end): the conv entry points name the operation
+// and its algorithmic MACs, the launchers bracket their main kernel with kt_pre / kt_post
+void kt_set_op(int op, double macs);
+void kt_pre(cudaStream_t st);
+void kt_post(cudaStream_t st, int kernel);
+
 }  // namespace iq

@@ -31,7 +31,11 @@ EXPORTS = [
     "iq_spatial_sum_workspace_size", "iq_spatial_sum", "iq_avgpool_bwd", "iq_channel_slice",
     "iq_bilinear_workspace_size", "iq_bilinear_up_fwd", "iq_bilinear_up_bwd", "iq_ce_grad",
     "iq_bn_update", "iq_device_status", "iq_rq_epoch_advance", "iq_rq_epoch_set",
+    "iq_kernel_timing_begin", "iq_kernel_timing_end",
 ]
+IQ_KERNEL_CONV_PIXEL_MAJOR, IQ_KERNEL_CONV_CHANNEL_MAJOR, IQ_KERNEL_CONV_WGRAD = 1, 2, 3
+KERNEL_NAMES = {1: "k_conv_tct (forward / data gradient)", 2: "k_conv_tcc (channel-major)",
+                3: "k_conv_tct (weight gradient)"}
 
 
 class IqError(RuntimeError):
@@ -56,6 +60,12 @@ class Term(C.Structure):
                 ("c_offset", C.c_int32), ("bcast", C.c_int32), ("scale", C.c_void_p),
                 ("gamma", C.c_void_p), ("beta", C.c_void_p), ("k_gamma", C.c_int32),
                 ("k_beta", C.c_int32)]
+
+
+class KernelTime(C.Structure):
+    """iq_kernel_time: summed event time and MACs of one (kernel, operation) pair."""
+    _fields_ = [("kernel", C.c_int32), ("op", C.c_int32), ("launches", C.c_int32),
+                ("pad", C.c_int32), ("ms", C.c_double), ("macs", C.c_double)]
 
 
 IQ_MAX_TERMS = 8
@@ -132,6 +142,8 @@ def load(path: str | None = None):
     L.iq_bn_update.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _I32, C.POINTER(BnBits), _I, _I,
                                _U64, _U64, _U64, _P, _SZ, _P]
     L.iq_device_status.argtypes = [C.POINTER(_I32), _P]
+    L.iq_kernel_timing_begin.argtypes = []
+    L.iq_kernel_timing_end.argtypes = [C.POINTER(KernelTime), _I32, C.POINTER(_I32)]
     L.iq_rq_epoch_advance.argtypes = [_P]
     L.iq_rq_epoch_set.argtypes = [_U64, _P]
     for f in EXPORTS:
@@ -143,6 +155,20 @@ def load(path: str | None = None):
 
 def launch_count() -> int:
     return int(load().iq_launch_count())
+
+
+def iq_kernel_timing_begin():
+    """Start bracketing every tensor-core conv kernel launch with CUDA events (eager calls)."""
+    _check("iq_kernel_timing_begin", load().iq_kernel_timing_begin())
+
+
+def iq_kernel_timing_end(capacity=16):
+    """Stop, wait for the events and return [{kernel, op, launches, ms, macs}] per (kernel, op)."""
+    out = (KernelTime * capacity)()
+    n = _I32(0)
+    _check("iq_kernel_timing_end", load().iq_kernel_timing_end(out, capacity, C.byref(n)))
+    return [{"kernel": out[i].kernel, "op": out[i].op, "launches": out[i].launches,
+             "ms": out[i].ms, "macs": out[i].macs} for i in range(n.value)]
 
 
 def iq_device_status(stream=None) -> int:

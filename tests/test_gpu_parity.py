@@ -611,3 +611,31 @@ def test_conv_dgrad_int64_reduction():
     with pytest.raises(iq.IqError):
         iq.iq_conv_dgrad(d, dev(e), dscal(1e-4), dev(wq), dx, s_dx,
                          acc_out=torch.empty((n, h, w, c), dtype=torch.int32, device=DEV))
+
+
+def test_kernel_timing_brackets_the_conv_kernels():
+    # one forward, data-gradient and weight-gradient call of a 3x3 layer: each operation's
+    # main kernel bracketed once, with the layer's algorithmic MACs
+    n, h, c, k = 2, 32, 64, 128
+    d = iq.conv_desc(n, h, h, c, k, 3, 3, 1, 1)
+    g = S.rng(77)
+    x = dev(S.int8_uniform(g, (n, h, h, c)))
+    wq = dev(S.int8_uniform(g, (k, 3, 3, c)))
+    e = dev(S.int8_uniform(g, (n, h, h, k)))
+    a = torch.empty((n, h, h, k), dtype=torch.int8, device=DEV)
+    dx = torch.empty((n, h, h, c), dtype=torch.int8, device=DEV)
+    gw = torch.empty((k, 3, 3, c), dtype=torch.int8, device=DEV)
+    iq.iq_kernel_timing_begin()
+    iq.iq_conv_fwd(d, x, dscal(0.01), wq, a, dscal(0.0), relu=True)
+    iq.iq_conv_dgrad(d, e, dscal(0.01), wq, dx, dscal(0.0))
+    iq.iq_conv_wgrad(d, e, dscal(0.01), x, dscal(0.01), gw, dscal(0.0), gq_mode=2)
+    rows = iq.iq_kernel_timing_end()
+    macs = float(n * h * h * k * 9 * c)
+    ops = {r["op"]: r for r in rows}
+    assert sorted(ops) == [1, 2, 3]
+    for r in rows:
+        assert r["launches"] == 1 and r["macs"] == macs and r["ms"] > 0
+    assert ops[1]["kernel"] in (iq.IQ_KERNEL_CONV_PIXEL_MAJOR, iq.IQ_KERNEL_CONV_CHANNEL_MAJOR)
+    assert ops[2]["kernel"] in (iq.IQ_KERNEL_CONV_PIXEL_MAJOR, iq.IQ_KERNEL_CONV_CHANNEL_MAJOR)
+    assert ops[3]["kernel"] == iq.IQ_KERNEL_CONV_WGRAD
+    assert iq.iq_kernel_timing_end() == []      # stopped: nothing recorded since
