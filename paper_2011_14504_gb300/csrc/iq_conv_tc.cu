@@ -2435,6 +2435,23 @@ iq_status codes_to_f16(const int8_t* x, __half* xf, int64_t n, cudaStream_t st) 
     return IQ_OK;
 }
 
+// A stride-1, unpadded 1 x 1 convolution treats every pixel alike, so its N x H x W pixels
+// can run as one image of 1 x (N H W) pixels -- the same memory layout for the input, the
+// errors and the output.  The rectangle tilings then take runs of 128 (256, 64) consecutive
+// pixels and waste none at the image borders (at 65 x 65, 128-pixel rectangles of one
+// image cover 27% padding).  Returns d itself when the convolution is not of that kind.
+static const iq_conv_desc* flat_pointwise(const iq_conv_desc* d, iq_conv_desc* tmp) {
+    if (d->r != 1 || d->s != 1 || d->stride_h != 1 || d->stride_w != 1 || d->pad_h || d->pad_w)
+        return d;
+    const int64_t pix = (int64_t)d->n * d->h * d->w;
+    if (pix > INT_MAX || (d->n == 1 && d->h == 1)) return d;
+    *tmp = *d;
+    tmp->n = 1;
+    tmp->h = 1;
+    tmp->w = (int32_t)pix;
+    return tmp;
+}
+
 size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d) {
     int64_t kdim = (int64_t)d->r * d->s * (d->c / d->groups);
     int64_t kpad = (kdim + 63) / 64 * 64;
@@ -2459,6 +2476,8 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
                       bool* done, const __half* xf_given, unsigned st_mask) {
     *done = false;
     if (!conv_fwd_tc_supported(d) || ((uintptr_t)x & 15) != 0 || !get_encode()) return IQ_OK;
+    iq_conv_desc dflat;
+    d = flat_pointwise(d, &dflat);
     TcP p;
     fill_geom(p, d);
     p.mode = MODE_FWD;
@@ -2562,6 +2581,8 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
                         cudaStream_t st, bool* done, const __half* ef_given) {
     *done = false;
     if (!conv_dgrad_tc_supported(d) || ((uintptr_t)e & 15) != 0 || !get_encode()) return IQ_OK;
+    iq_conv_desc dflat;
+    d = flat_pointwise(d, &dflat);
     const int nsl = conv_dgrad_tc_slices(d);
     if (nsl > 1 && !out64) return IQ_OK;
     if (nsl == 1 && !out32) return IQ_OK;
@@ -2720,6 +2741,8 @@ bool wgrad_im2col_desc(const iq_conv_desc* d, iq_conv_desc* d2) {
 }
 
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d) {
+    iq_conv_desc dflat;
+    d = flat_pointwise(d, &dflat);      // the tiling (and split count) conv_wgrad_tc uses
     const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
     const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
     const size_t eb = ((size_t)d->n * P * Q * ((d->k + 63) / 64 * 64) * 2 + 255) / 256 * 256;
@@ -2797,6 +2820,8 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
     *amax_done = false;
     if (g32_out) *g32_out = nullptr;
     if (tc_env_disabled() || (((uintptr_t)e | (uintptr_t)x) & 15) != 0) return IQ_OK;
+    iq_conv_desc dflat;
+    d = flat_pointwise(d, &dflat);
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     int* err = tc_status_ptr();
     if (!err) return IQ_ERR_CUDA;
