@@ -108,6 +108,23 @@ def test_combine_four_channel_groups(n, hw, c):
                 n, hw, c, False, False)
 
 
+def test_combine_small_values_and_negative_relu():
+    # values far below the fixed-point bound (int16 codes in [-3, 3]): M < 2^37, so the
+    # float estimate cannot decide and every element takes the exact form; then a ReLU join
+    # whose sums are all negative (max 0, every code 0)
+    g = np.random.default_rng(19)
+    n, hw, c = 2, 23 * 19, 48
+    X = g.integers(-3, 4, size=(n, hw, c)).astype(np.int16)
+    sc = g.integers(-127, 128, size=(n, hw, c)).astype(np.int8)
+    gam = g.integers(-127, 128, size=c).astype(np.int32)
+    bet = np.zeros(c, np.int32)
+    run_combine([(X, 2.0 ** -15, 0, False, gam, bet), (sc, 2.0 ** -30, 0, False, None, None)],
+                n, hw, c, False, False)
+    neg = -np.abs(g.integers(1, 128, size=(n, hw, c))).astype(np.int8)
+    run_combine([(neg, 0.01, 0, False, None, None), (neg, 0.02, 0, False, None, None)],
+                n, hw, c, False, True)
+
+
 def test_combine_edge_cases():
     # all zero, a single pixel, a single channel
     run_combine([(np.zeros((1, 5, 8), np.int8), 0.5, 0, False, None, None)], 1, 5, 8, False, False)
