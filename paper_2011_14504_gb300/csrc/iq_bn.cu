@@ -193,28 +193,28 @@ __global__ void __launch_bounds__(kThreads) k_bn_dev(const int32_t* __restrict__
     int hi[4] = {INT_MIN, INT_MIN, INT_MIN, INT_MIN}, lo[4] = {INT_MAX, INT_MAX, INT_MAX, INT_MAX};
     const int4* a4 = reinterpret_cast<const int4*>(acc);
     const int64_t step = (int64_t)gridDim.y * RL;
+    auto row = [&](const int4 v) {
+        const int vs[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            const int64_t dv = (int64_t)vs[j] - f[j];
+            d[j] += (unsigned long long)(dv < 0 ? -dv : dv);
+            n[j] += dv > 0;
+            hi[j] = max(hi[j], vs[j]);
+            lo[j] = min(lo[j], vs[j]);
+        }
+    };
     if (act) {
         int64_t r = (int64_t)blockIdx.y * RL + rl;
-        // two rows per iteration: both loads in flight together
-        for (; r < m; r += 2 * step) {
-            const bool two = r + step < m;
-            const int4 v0 = a4[r * C4 + g];
-            const int4 v1 = two ? a4[(r + step) * C4 + g] : v0;
-            const int vs0[4] = {v0.x, v0.y, v0.z, v0.w}, vs1[4] = {v1.x, v1.y, v1.z, v1.w};
+        // four rows per iteration: their loads in flight together
+        for (; r + 3 * step < m; r += 4 * step) {
+            int4 v[4];
 #pragma unroll
-            for (int j = 0; j < 4; j++) {
-                const int64_t dv0 = (int64_t)vs0[j] - f[j];
-                d[j] += (unsigned long long)(dv0 < 0 ? -dv0 : dv0);
-                n[j] += dv0 > 0;
-                hi[j] = max(hi[j], max(vs0[j], vs1[j]));
-                lo[j] = min(lo[j], min(vs0[j], vs1[j]));
-                if (two) {
-                    const int64_t dv1 = (int64_t)vs1[j] - f[j];
-                    d[j] += (unsigned long long)(dv1 < 0 ? -dv1 : dv1);
-                    n[j] += dv1 > 0;
-                }
-            }
+            for (int u = 0; u < 4; u++) v[u] = a4[(r + u * step) * C4 + g];
+#pragma unroll
+            for (int u = 0; u < 4; u++) row(v[u]);
         }
+        for (; r < m; r += step) row(a4[r * C4 + g]);
     }
 #pragma unroll
     for (int j = 0; j < 4; j++) {
@@ -436,10 +436,8 @@ __global__ void __launch_bounds__(kThreads) k_bn_requant(const int32_t* __restri
         G[j] = s.G[4 * g + j]; H[j] = s.H[4 * g + j];
     }
     const int4* a4 = reinterpret_cast<const int4*>(acc);
-    for (int64_t r = t / C4; r < m; r += rstride) {
-        int64_t v = r * C4 + g;
-        int4 in = a4[v];
-        int vs[4] = {in.x, in.y, in.z, in.w};
+    auto row = [&](int64_t v, const int4 in) {
+        const int vs[4] = {in.x, in.y, in.z, in.w};
         int xo[4];
         uint32_t ao = 0;
 #pragma unroll
@@ -458,7 +456,16 @@ __global__ void __launch_bounds__(kThreads) k_bn_requant(const int32_t* __restri
             reinterpret_cast<uint2*>(X)[v] = xv;
         }
         reinterpret_cast<uint32_t*>(A)[v] = ao;
+    };
+    int64_t r = t / C4;
+    // two rows per iteration: both loads in flight together
+    for (; r + rstride < m; r += 2 * rstride) {
+        const int64_t v0 = r * C4 + g, v1 = (r + rstride) * C4 + g;
+        const int4 in0 = a4[v0], in1 = a4[v1];
+        row(v0, in0);
+        row(v1, in1);
     }
+    if (r < m) row(r * C4 + g, a4[r * C4 + g]);
 }
 
 __global__ void k_bn_export(BnStats s, int32_t C, const int32_t* __restrict__ codes_ws,
