@@ -1122,79 +1122,6 @@ __device__ __forceinline__ void rpos_next(RectPos& q, const TcP& p, const RectGr
     if (++q.kb >= p.nkb_total) rpos_set(q, q.tile + gridDim.x, g, BN);
 }
 
-// int32 stores and per-channel statistics (OUT_STATS) or int64 atomic adds of LDW columns
-// of one output row m (valid: the row exists)
-template <int LDW>
-__device__ __forceinline__ void write_row(const TcP& p, const uint32_t (&r)[LDW], int64_t m,
-                                          bool valid, int c0, int lane,
-                                          int32_t* __restrict__ out32,
-                                          long long* __restrict__ out64,
-                                          unsigned long long* __restrict__ s1,
-                                          int* __restrict__ hi_c, int* __restrict__ lo_c) {
-    if (p.out == OUT_PART32) {
-        if (valid) {
-            int32_t* dst = out32 + m * p.ncols + c0;
-#pragma unroll
-            for (int i = 0; i < LDW / 4; i++)
-                if (c0 + 4 * i < p.ncols)
-                    reinterpret_cast<int4*>(dst)[i] = make_int4((int)r[4 * i], (int)r[4 * i + 1],
-                                                                (int)r[4 * i + 2], (int)r[4 * i + 3]);
-        }
-        return;
-    }
-    if (p.out == OUT_STATS) {
-        if (valid) {
-            int32_t* dst = out32 + m * p.ncols + c0;
-#pragma unroll
-            for (int i = 0; i < LDW / 4; i++)
-                if (c0 + 4 * i < p.ncols)
-                    reinterpret_cast<int4*>(dst)[i] = make_int4((int)r[4 * i], (int)r[4 * i + 1],
-                                                                (int)r[4 * i + 2], (int)r[4 * i + 3]);
-        }
-        // per column over the warp's 32 rows: the maximum always, the minimum and the sum
-        // when the caller consumes them (the sum as one signed reduction when it fits 32 bits,
-        // else as two of its 16-bit halves)
-        long long my_sum = 0;
-        int my_hi = INT_MIN, my_lo = INT_MAX;
-        const bool want_lo = p.st_mask & TC_STATS_LO, want_sum = p.st_mask & TC_STATS_SUM;
-        const bool sum32 = p.st_mask & ST_SUM32;
-#pragma unroll
-        for (int j = 0; j < LDW; j++) {
-            const int v = (int)r[j];
-            const int mx = __reduce_max_sync(0xffffffffu, valid ? v : INT_MIN);
-            if (lane == j) my_hi = mx;
-            if (want_lo) {
-                const int mn = __reduce_min_sync(0xffffffffu, valid ? v : INT_MAX);
-                if (lane == j) my_lo = mn;
-            }
-            if (want_sum) {
-                if (sum32) {
-                    const int sm = __reduce_add_sync(0xffffffffu, valid ? v : 0);
-                    if (lane == j) my_sum = sm;
-                } else {
-                    const unsigned sl =
-                        __reduce_add_sync(0xffffffffu, valid ? ((unsigned)v & 0xffffu) : 0u);
-                    const int sh = __reduce_add_sync(0xffffffffu, valid ? (v >> 16) : 0);
-                    if (lane == j) my_sum = (long long)sh * 65536 + (long long)sl;
-                }
-            }
-        }
-        const int gcol = c0 + lane;
-        if (lane < LDW && gcol < p.ncols) {
-            atomicMax(&hi_c[gcol], my_hi);
-            if (want_lo) atomicMin(&lo_c[gcol], my_lo);
-            if (want_sum) atomicAdd(&s1[gcol], (unsigned long long)my_sum);
-        }
-    } else if (valid) {
-        long long* dst = out64 + m * p.ncols + c0;
-#pragma unroll
-        for (int j = 0; j < LDW; j++)
-            if ((int)r[j] != 0 && c0 + j < p.ncols)
-                atomicAdd(reinterpret_cast<unsigned long long*>(dst + j),
-                          (unsigned long long)(long long)(int)r[j]);
-    }
-}
-
 // per-channel statistics of LDW columns over the warp's 32 rows (OUT_STATS): the maximum,
 // and the minimum and the sum when st_mask asks for them (the sum as one signed 32-bit
 // reduction under ST_SUM32, else as two 16-bit halves)
@@ -1235,6 +1162,46 @@ __device__ __forceinline__ void col_stats(const TcP& p, const int* r, bool valid
         if (want_hi && my_hi != INT_MIN) atomicMax(&hi_c[gcol], my_hi);
         if (want_lo && my_lo != INT_MAX) atomicMin(&lo_c[gcol], my_lo);
         if (want_sum && my_sum) atomicAdd(&s1[gcol], (unsigned long long)my_sum);
+    }
+}
+
+// int32 stores and per-channel statistics (OUT_STATS) or int64 atomic adds of LDW columns
+// of one output row m (valid: the row exists)
+template <int LDW>
+__device__ __forceinline__ void write_row(const TcP& p, const uint32_t (&r)[LDW], int64_t m,
+                                          bool valid, int c0, int lane,
+                                          int32_t* __restrict__ out32,
+                                          long long* __restrict__ out64,
+                                          unsigned long long* __restrict__ s1,
+                                          int* __restrict__ hi_c, int* __restrict__ lo_c) {
+    if (p.out == OUT_PART32) {
+        if (valid) {
+            int32_t* dst = out32 + m * p.ncols + c0;
+#pragma unroll
+            for (int i = 0; i < LDW / 4; i++)
+                if (c0 + 4 * i < p.ncols)
+                    reinterpret_cast<int4*>(dst)[i] = make_int4((int)r[4 * i], (int)r[4 * i + 1],
+                                                                (int)r[4 * i + 2], (int)r[4 * i + 3]);
+        }
+        return;
+    }
+    if (p.out == OUT_STATS) {
+        if (valid) {
+            int32_t* dst = out32 + m * p.ncols + c0;
+#pragma unroll
+            for (int i = 0; i < LDW / 4; i++)
+                if (c0 + 4 * i < p.ncols)
+                    reinterpret_cast<int4*>(dst)[i] = make_int4((int)r[4 * i], (int)r[4 * i + 1],
+                                                                (int)r[4 * i + 2], (int)r[4 * i + 3]);
+        }
+        col_stats<LDW>(p, reinterpret_cast<const int*>(r), valid, c0, lane, s1, hi_c, lo_c);
+    } else if (valid) {
+        long long* dst = out64 + m * p.ncols + c0;
+#pragma unroll
+        for (int j = 0; j < LDW; j++)
+            if ((int)r[j] != 0 && c0 + j < p.ncols)
+                atomicAdd(reinterpret_cast<unsigned long long*>(dst + j),
+                          (unsigned long long)(long long)(int)r[j]);
     }
 }
 
