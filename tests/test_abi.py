@@ -55,6 +55,19 @@ def test_conv_out_size_and_workspace_queries(lib):
     assert iq.iq_bn_int_workspace_size(1024, 64) > 0
 
 
+def test_kernel_timing_host_side(lib):
+    # with nothing launched between begin and end: no rows, no device work; null outputs
+    # are rejected
+    iq.iq_kernel_timing_begin()
+    assert iq.iq_kernel_timing_end() == []
+    n = C.c_int32(0)
+    assert lib.iq_kernel_timing_end(None, 4, C.byref(n)) == iq.IQ_ERR_INVALID_ARG
+    out = (iq.KernelTime * 2)()
+    assert lib.iq_kernel_timing_end(out, 2, None) == iq.IQ_ERR_INVALID_ARG
+    # the struct layout the header declares: 4 int32 then 2 doubles
+    assert C.sizeof(iq.KernelTime) == 32
+
+
 def test_invalid_arguments_rejected_before_launch(lib):
     bad = iq.conv_desc(1, 8, 8, 6, 4, 3, 3, 1, 1, 1, 4)        # C not divisible by groups
     with pytest.raises(iq.IqError) as e:
