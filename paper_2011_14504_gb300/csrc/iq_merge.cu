@@ -386,6 +386,92 @@ __global__ void __launch_bounds__(kThreads, 3) k_comb4r(Terms T, int concat, int
     }
 }
 
+// The two passes for a sum of up to 6 operands that each cover all c_out channels (the ASPP
+// error sum: four branch errors and the broadcast pooled one).  As in k_comb4r each thread
+// owns one 4-channel group, (blockIdx.x 256 + tid) % (c_out / 4), and walks pixels; the
+// operands' F rows of the block's 256 groups are staged once per block in shared memory
+// (n 8 KB), their B rows summed per thread in registers, so per 4 outputs an operand costs
+// one 4- or 8-byte code load and two 16-byte shared loads.
+template <int PASS>
+__global__ void __launch_bounds__(kThreads) k_combNs(Terms T, int64_t npix, int cgs, int relu,
+                                                     const long long* __restrict__ F,
+                                                     const long long* __restrict__ B,
+                                                     CombHdr* hdr, int8_t* __restrict__ out,
+                                                     UDiv dhw, int any_bcast) {
+    extern __shared__ __align__(16) long long sF[];     // [n][256 groups][4]
+    const int n = T.n, c_out = 4 * cgs;
+    const int w0 = (int)(((int64_t)blockIdx.x * blockDim.x) % cgs);   // the block's first group
+    for (int k = threadIdx.x; k < n * kThreads * 4; k += blockDim.x) {
+        const int ti = k / (kThreads * 4), r = k - ti * (kThreads * 4);
+        const int grp = (w0 + (r >> 2)) % cgs;
+        sF[k] = F[term_at(T, ti).base + 4 * grp + (r & 3)];
+    }
+    __syncthreads();
+    uint64_t M = 0;
+    UDiv d2m;
+    if (PASS == 1) {
+        M = hdr->M;
+        d2m = hdr->div;
+    }
+    const int64_t tcount = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % cgs);
+    const int64_t pstride = tcount / cgs;
+    const int co0 = 4 * g;
+    long long bs[4] = {0, 0, 0, 0};
+#pragma unroll
+    for (int i = 0; i < IQ_MAX_TERMS; i++) {
+        if (i >= n) break;
+        const TermDev& ti = term_at(T, i);
+#pragma unroll
+        for (int j = 0; j < 4; j++) bs[j] += B[ti.base + co0 + j];
+    }
+    uint64_t mx = 0;
+    for (int64_t pix = t / cgs; pix < npix; pix += pstride) {
+        const int64_t img = any_bcast ? (int64_t)udiv((uint64_t)pix, dhw) : 0;
+        int64_t z[4] = {bs[0], bs[1], bs[2], bs[3]};
+#pragma unroll
+        for (int i = 0; i < IQ_MAX_TERMS; i++) {
+            if (i >= n) break;
+            const TermDev& ti = term_at(T, i);
+            int32_t v[4];
+            load4p(ti.codes, ti.is16, (ti.bcast ? img : pix) * c_out + co0, v);
+            const longlong2* f2 =
+                reinterpret_cast<const longlong2*>(sF + (i * kThreads + threadIdx.x) * 4);
+            const longlong2 fa = f2[0], fb = f2[1];
+            z[0] += (int64_t)fa.x * v[0];
+            z[1] += (int64_t)fa.y * v[1];
+            z[2] += (int64_t)fb.x * v[2];
+            z[3] += (int64_t)fb.y * v[3];
+        }
+        if (PASS == 0) {
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                const int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
+                const uint64_t a = (uint64_t)(zz < 0 ? -zz : zz);
+                mx = a > mx ? a : mx;
+            }
+        } else {
+            uint32_t w = 0u;
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                const int64_t zz = (relu && z[j] < 0) ? 0 : z[j];
+                int64_t c = 0;
+                if (M) {
+                    const uint64_t num = ((uint64_t)(zz + (int64_t)M) << 8) + M;
+                    c = clamp64((int64_t)udiv(num, d2m) - 128, -127, 127);
+                }
+                w |= ((uint32_t)c & 0xffu) << (8 * j);
+            }
+            *reinterpret_cast<uint32_t*>(out + pix * (int64_t)c_out + co0) = w;
+        }
+    }
+    if (PASS == 0) {
+        mx = warp_max_u64(mx);
+        if ((threadIdx.x & 31) == 0 && mx) atomicMax(&hdr->maxz, (unsigned long long)mx);
+    }
+}
+
 __global__ void k_comb_params(CombHdr* hdr, double* s_out) {
     const uint64_t M = hdr->maxz;
     hdr->M = M;
@@ -585,6 +671,31 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
         IQ_LAUNCH_CHECK();
         k_comb4r<1><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
                                             dhw, any_bcast);
+        IQ_LAUNCH_CHECK();
+        return IQ_OK;
+    }
+    // sums whose operands all cover every channel, F rows of all of them in shared memory
+    bool all_cover = vec4 && !concat && n_terms <= 6;
+    for (int i = 0; i < n_terms && all_cover; i++) all_cover = T.t[i].c == c_out;
+    if (all_cover) {
+        const int cgs = c_out / 4;
+        const int64_t npix = n * hw;
+        int64_t gcd = cgs, b2 = kThreads;
+        while (b2) { int64_t r = gcd % b2; gcd = b2; b2 = r; }
+        const int64_t unit = cgs / gcd;
+        int64_t want = (npix * cgs + kThreads - 1) / kThreads;
+        if (want > 152 * 8) want = 152 * 8;
+        want = (want + unit - 1) / unit * unit;
+        if (want < unit) want = unit;
+        const int g = (int)want;
+        const size_t sm = (size_t)n_terms * kThreads * 4 * 8;   // <= 48 KB
+        k_combNs<0><<<g, kThreads, sm, st>>>(T, npix, cgs, relu != 0, F, B, hdr, out, dhw,
+                                             any_bcast);
+        IQ_LAUNCH_CHECK();
+        k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
+        IQ_LAUNCH_CHECK();
+        k_combNs<1><<<g, kThreads, sm, st>>>(T, npix, cgs, relu != 0, F, B, hdr, out, dhw,
+                                             any_bcast);
         IQ_LAUNCH_CHECK();
         return IQ_OK;
     }

@@ -83,6 +83,23 @@ def test_combine_sum_of_errors_with_broadcast():
     run_combine(specs, n, hw, c, False, False)
 
 
+def test_combine_sum_of_many_operands_all_channels():
+    # three to six operands covering every channel (the shared-memory row kernel): int16
+    # with the BN affine, int8, and a broadcast term, with and without ReLU
+    g = np.random.default_rng(20)
+    n, hw, c = 3, 33 * 31, 64
+    X = g.integers(-32767, 32768, size=(n, hw, c)).astype(np.int16)
+    gam = g.integers(-127, 128, size=c).astype(np.int32)
+    bet = g.integers(-127, 128, size=c).astype(np.int32)
+    specs = [(X, 2.0 ** -15 * 2.1, 0, False, gam, bet),
+             (g.integers(-127, 128, size=(n, hw, c)).astype(np.int8), 0.03, 0, False, None, None),
+             (g.integers(-127, 128, size=(n, c)).astype(np.int8), 0.2, 0, True, None, None)]
+    run_combine(specs, n, hw, c, False, True)
+    more = specs + [(g.integers(-127, 128, size=(n, hw, c)).astype(np.int8), s, 0, False, None,
+                     None) for s in (0.5, 1e-3, 0.07)]
+    run_combine(more, n, hw, c, False, False)
+
+
 def test_combine_concat_aspp():
     g = np.random.default_rng(14)
     n, hw, cb = 2, 13 * 13, 32
