@@ -13,18 +13,22 @@
 //          N = output channels, K = taps x channels, both operands K-major.
 //   WGRAD (weight gradient): D[Kout x RSC] = sum over pixels of E^T X, both operands
 //          MN-major (channels contiguous), the pixel sum split across CTAs.
-// Three persistent kernels (one CTA per SM, tiles 128 x BN x 64, BN in {64, 128, 256}):
+// Four persistent kernels (one CTA per SM, tiles 128 x BN x 64, BN in {64, 128, 256}):
 //   k_conv_tct  all operands by TMA from fp16 carrier copies (a pre-pass widens the codes
 //               once per call): 4-D boxes of the input per tap for FWD, error rectangles
-//               and im2col boxes for WGRAD.  The default whenever the shape allows it.
+//               and im2col boxes for WGRAD.  The default whenever the shape allows it; its
+//               FWD epilogue writes the int32 output through TMA stores.
+//   k_conv_tcc  FWD with at most 128 output channels, channel-major (M = output channels,
+//               N = 256 pixels), the same TMA loads.
 //   k_conv_tcq  FWD with whole 64-channel k-blocks when no TMA tile rectangle fits well:
 //               producer threads copy int8 rows with cp.async and widen them in shared memory.
 //   k_conv_tcp  everything else (channel counts that are multiples of 8 or 16): producer
 //               warps gather int8 rows into registers and widen them on the way to shared
 //               memory.
-// In all three one elected thread issues tcgen05.mma (M=128, K=16) into TMEM and
-// epilogue warps fold the fp32 chunks into int32 and write either int32 outputs plus
-// per-channel sum / max / min (FWD), int32 split partials or int64 atomic adds (WGRAD).
+// In all of them one thread (in k_conv_tct / k_conv_tcc: one lane elected in a converged
+// warp) issues tcgen05.mma (M=128, K=16) into TMEM, and epilogue warps fold the fp32 chunks
+// into int32 and write either int32 outputs plus per-channel statistics (FWD; which ones
+// the caller reads, TcP::st_mask), int32 split partials or int64 atomic adds (WGRAD).
 // Every mbarrier wait is bounded (about one second); on expiry the CTA records a code in
 // the device's sticky status word, drains what it issued and returns, and every later
 // launch exits at once until the host reads the status (iq_device_status).

@@ -293,8 +293,8 @@ __device__ __forceinline__ void comb_z4(const long long (&f0)[4], const long lon
 
 // The two passes with a fixed 4-channel group per thread: the launch has a multiple of
 // c_out / 4 threads, so thread t always owns group t % (c_out / 4), keeps the F rows of the
-// (at most two) operands covering it and their summed B rows in registers (24 registers,
-// about half of an 8-channel group's, for twice the resident warps), and walks the pixels
+// (at most two) operands covering it and their summed B rows in registers (24 registers;
+// the kernel fits 3 blocks of 256 threads per SM), and walks the pixels
 // t / (c_out / 4), + T / (c_out / 4), ... two at a time, both pixels' loads in flight
 // together.
 template <int PASS>
