@@ -1,0 +1,104 @@
+"""Pins of the oracle's network composition (oracle/fcn.py) by exact symmetries.
+
+The layer functions are pinned one by one elsewhere; these tests fix how the FCN-VGG16
+step composes them, with properties that hold for the correct dataflow and fail for a
+dropped layer, a wrong index, a transposed axis or a pool / decoder misplacement:
+
+- Horizontal flip.  Take every convolution kernel and the decoder filters mirror-symmetric
+  (w[.., s, ..] = w[.., S-1-s, ..]).  Then each step commutes with flipping the image
+  width:
+  - the image quantizer and SQ_8 use global maxima;
+  - the convolutions pad symmetrically;
+  - 2 x 2 max pools on even widths map windows onto windows;
+  - the 32x decoder (kernel 64, stride 32, padding 16) maps output column y to
+    W - 1 - y;
+  - the MSE error is elementwise.
+  So the flipped image and labels give the flipped forward trace and error. The backward
+  gives the mirrored raw weight gradients and the flipped errors down to the last pool
+  (the pools' argmax ties and the stochastic rounding of G_q, indexed by element, are not
+  symmetric and are not compared).
+- Batch order.  Every scale is a maximum over the whole batch and every gradient a sum over
+  it, so permuting three images cyclically permutes every activation and error and leaves
+  the raw gradients unchanged.
+"""
+import numpy as np
+
+from oracle.fcn import OracleFcn
+from paper_2011_14504_gb300 import synthetic as S
+
+CLASSES, WIDTH, SEED = 21, 0.125, 5
+
+
+def _mirrored_weights():
+    wts, up = S.fcn_vgg16_weights(SEED, CLASSES, WIDTH)
+    wts = [0.5 * (w + w[:, :, ::-1, :]) for w in wts]        # KRSC: mirror the S axis
+    up = 0.5 * (up + up[..., ::-1])
+    return wts, up
+
+
+def _inputs(n=2, h=64, w=64):
+    g = S.rng(41)
+    return S.images_u8(g, n, h, w), S.labels_voronoi(g, n, h, w, CLASSES, sites=6)
+
+
+def _net(wts, up):
+    return OracleFcn(S.fcn_vgg16_channels(CLASSES, WIDTH), wts, up, CLASSES, seed=SEED,
+                     lr_log2=6)
+
+
+def _fw(a):           # flip the width axis of an NHWC / NHW array
+    return a[:, :, ::-1, ...]
+
+
+def test_fcn_step_commutes_with_a_horizontal_flip():
+    wts, up = _mirrored_weights()
+    img, lab = _inputs()
+    a, b = _net(wts, up), _net(wts, up)
+    ta = a.forward(img)
+    tb = b.forward(np.ascontiguousarray(_fw(img)))
+    assert np.array_equal(tb["img"][0], _fw(ta["img"][0])) and tb["img"][1] == ta["img"][1]
+    for la, lb in zip(ta["layers"], tb["layers"]):
+        if la[0] == "pool":
+            assert np.array_equal(lb[3], _fw(la[3]))
+            continue
+        assert np.array_equal(lb[6], _fw(la[6])), la[2]          # int32 accumulators
+        assert np.array_equal(lb[7], _fw(la[7])) and lb[8] == la[8]
+    za, zb = ta["up"], tb["up"]
+    assert np.array_equal(zb[4], _fw(za[4])) and np.array_equal(zb[5], _fw(za[5]))
+    assert zb[6] == za[6]
+    oa = a.backward_update(ta, lab)
+    ob = b.backward_update(tb, np.ascontiguousarray(_fw(lab)))
+    assert np.array_equal(ob["E"][0], _fw(oa["E"][0])) and ob["E"][1] == oa["E"][1]
+    assert np.array_equal(ob["e_score"][0], _fw(oa["e_score"][0]))
+    assert np.array_equal(ob["up_g"][0], oa["up_g"][0][..., ::-1])  # decoder kernel mirrored
+    # layers after the last pool: raw gradients mirrored, errors flipped
+    chans = S.fcn_vgg16_channels(CLASSES, WIDTH)
+    last_pool = max(i for i, c in enumerate(chans) if c[0] == "pool")
+    tail = [sum(1 for c in chans[:i] if c[0] != "pool") for i in range(last_pool + 1, len(chans))]
+    assert tail
+    for li in tail:
+        assert np.array_equal(ob["grads"][li][0], oa["grads"][li][0][:, :, ::-1, :]), li
+        if li in oa.get("ex", {}):
+            assert np.array_equal(ob["ex"][li][0], _fw(oa["ex"][li][0])), li
+            assert ob["ex"][li][1] == oa["ex"][li][1]
+
+
+def test_fcn_step_is_equivariant_to_the_batch_order():
+    wts, up = S.fcn_vgg16_weights(SEED, CLASSES, WIDTH)
+    img, lab = _inputs(n=3)
+    swap = [1, 2, 0]        # a 3-cycle: no reversal or swap of the batch commutes with it
+    a, b = _net(wts, up), _net(wts, up)
+    ta = a.forward(img)
+    tb = b.forward(np.ascontiguousarray(img[swap]))
+    for la, lb in zip(ta["layers"], tb["layers"]):
+        if la[0] == "conv":
+            assert np.array_equal(lb[7], la[7][swap]) and lb[8] == la[8], la[2]
+    assert np.array_equal(tb["up"][5], ta["up"][5][swap]) and tb["up"][6] == ta["up"][6]
+    oa = a.backward_update(ta, lab)
+    ob = b.backward_update(tb, np.ascontiguousarray(lab[swap]))
+    assert np.array_equal(ob["E"][0], oa["E"][0][swap])
+    assert np.array_equal(ob["up_g"][0], oa["up_g"][0])
+    for li, (G, _, _) in oa["grads"].items():
+        assert np.array_equal(ob["grads"][li][0], G), li
+    for li, (ex, s) in oa.get("ex", {}).items():
+        assert np.array_equal(ob["ex"][li][0], ex[swap]) and ob["ex"][li][1] == s, li
