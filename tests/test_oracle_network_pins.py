@@ -102,3 +102,86 @@ def test_fcn_step_is_equivariant_to_the_batch_order():
         assert np.array_equal(ob["grads"][li][0], G), li
     for li, (ex, s) in oa.get("ex", {}).items():
         assert np.array_equal(ob["ex"][li][0], ex[swap]) and ob["ex"][li][1] == s, li
+
+
+# ---------------------------------------------------------------- DeepLabv3-ResNet50
+
+def _deeplab(mirror, blocks=(1, 1, 2, 1), width=0.0625):
+    from oracle.deeplab import OracleDeepLab
+    sp = S.deeplabv3_r50_spec(21, width, blocks)
+    w, gm, bm = S.deeplabv3_r50_init(6, sp)
+    if mirror:
+        w = [0.5 * (x + x[:, :, ::-1, :]) for x in w]
+    return sp, (lambda: OracleDeepLab(sp, w, gm, bm, seed=6, lr_log2=6))
+
+
+def _conv_records(tr):
+    return {k: v for k, v in tr.items() if isinstance(v, dict) and "a" in v}
+
+
+def test_deeplab_step_commutes_with_a_horizontal_flip():
+    # 33 x 33: every stride-2 stage (stem, its 3 x 3 pool, stage 2) sees an odd width, so
+    # output column x takes input column 2x on both sides of the flip; the dilated and ASPP
+    # convolutions pad by their rates, BN statistics, the image pooling and the scales are
+    # sums and maxima over the whole tensor, and the x8 bilinear maps 5 -> 33 corner to
+    # corner.  The stem's pool backward (overlapping windows, argmax ties) is not compared.
+    sp, mk = _deeplab(True)
+    g = S.rng(43)
+    img = S.images_u8(g, 1, 33, 33)
+    lab = S.labels_uniform_ignore(g, 1, 33, 33, 21)
+    a, b = mk(), mk()
+    ta = a.forward(img)
+    tb = b.forward(np.ascontiguousarray(_fw(img)))
+    ra, rb = _conv_records(ta), _conv_records(tb)
+    assert ra.keys() == rb.keys() and len(ra) > 10
+    for name in ra:
+        assert np.array_equal(rb[name]["a"], _fw(ra[name]["a"])), name
+        assert rb[name]["s_a"] == ra[name]["s_a"], name
+        if "X" in ra[name]:
+            assert np.array_equal(rb[name]["X"], _fw(ra[name]["X"])), name
+    for blk in sp.blocks:
+        assert np.array_equal(tb[blk.name]["out"][0], _fw(ta[blk.name]["out"][0])), blk.name
+        assert tb[blk.name]["out"][1] == ta[blk.name]["out"][1]
+    assert np.array_equal(tb["cat"][0], _fw(ta["cat"][0])) and tb["cat"][1] == ta["cat"][1]
+    assert np.array_equal(tb["z"][0], _fw(ta["z"][0])) and tb["z"][1] == ta["z"][1]
+    oa = a.backward_update(ta, lab)
+    ob = b.backward_update(tb, np.ascontiguousarray(_fw(lab)))
+    assert np.array_equal(ob["E"][0], _fw(oa["E"][0])) and ob["E"][1] == oa["E"][1]
+    assert np.array_equal(ob["e_cls"][0], _fw(oa["e_cls"][0]))
+    for name, rec in ra.items():
+        if name == sp.stem.name:
+            continue
+        shp = rec["a"].shape
+        ea, eb = oa[name]["e"], ob[name]["e"]
+        assert np.array_equal(eb[0].reshape(shp), _fw(ea[0].reshape(shp))), name
+        assert eb[1] == ea[1], name
+        if "ex" in oa[name]:
+            xs = rec["x"].shape
+            assert np.array_equal(ob[name]["ex"][0].reshape(xs),
+                                  _fw(oa[name]["ex"][0].reshape(xs))), name
+        if "dgb" in oa[name]:
+            assert all(np.array_equal(p, q) for p, q in zip(ob[name]["dgb"], oa[name]["dgb"]))
+    for blk in sp.blocks:
+        assert np.array_equal(ob[blk.name][0], _fw(oa[blk.name][0])), blk.name
+
+
+def test_deeplab_step_is_equivariant_to_the_batch_order():
+    sp, mk = _deeplab(False)
+    g = S.rng(44)
+    img = S.images_u8(g, 3, 33, 33)
+    lab = S.labels_uniform_ignore(g, 3, 33, 33, 21)
+    cyc = [1, 2, 0]
+    a, b = mk(), mk()
+    ta = a.forward(img)
+    tb = b.forward(np.ascontiguousarray(img[cyc]))
+    for name, rec in _conv_records(ta).items():
+        assert np.array_equal(tb[name]["a"], rec["a"][cyc]) and tb[name]["s_a"] == rec["s_a"], name
+    assert np.array_equal(tb["z"][0], ta["z"][0][cyc]) and tb["z"][1] == ta["z"][1]
+    oa = a.backward_update(ta, lab)
+    ob = b.backward_update(tb, np.ascontiguousarray(lab[cyc]))
+    assert np.array_equal(ob["E"][0], oa["E"][0][cyc])
+    for name, rec in _conv_records(ta).items():
+        shp = rec["a"].shape
+        assert np.array_equal(ob[name]["e"][0].reshape(shp), oa[name]["e"][0].reshape(shp)[cyc]), name
+        if "dgb" in oa[name]:
+            assert all(np.array_equal(p, q) for p, q in zip(ob[name]["dgb"], oa[name]["dgb"]))
