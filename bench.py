@@ -1,28 +1,34 @@
-"""Benchmark: the FCN-VGG16 quantized training step (int8 conv fwd + dgrad + wgrad, the
-paper's Sec. 3 dataflow) on synthetic 512x512 segmentation batches.
+"""Benchmark of the integer quantized convolution hot path (Sec. 3 of the paper: int8 conv
+forward, data gradient and weight gradient with integer L1BN, ReLU and requantization).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--workload fcn_vgg16_train|deeplabv3_r50_train|fcn_vgg16_infer|
-                              deeplabv3_r50_infer]
+                  [--workload deeplabv3_r50_train|fcn_vgg16_train|deeplabv3_r50_infer|
+                              fcn_vgg16_infer|single_layer]
 
-The default workload is the FCN-VGG16 training step (batch 16, 512x512, 150 classes);
-the others are the DeepLabv3-ResNet50 training step (batch 16, 513x513, 21 classes, 5%
-ignored labels) and the two inference passes (batch 8).
+The default workload is the largest single-GPU configuration, the DeepLabv3-ResNet50
+training step (batch 16, 3x513x513, 21 classes, 5% ignored labels, output stride 8).  The
+others are the FCN-VGG16 training step (batch 16, 3x512x512, 150 classes), the two
+inference passes (batch 8) and one quantized conv layer (N=1, 64 -> 64 channels, 32x32,
+3x3, L1BN + ReLU + Q_A forward, data gradient and weight gradient).
 
 Prints one JSON line.  `value` is the int8 convolution throughput of the whole step in
-TOPS (2 x MACs of every forward, data-gradient and weight-gradient convolution, the
-decoder included, divided by the device time of the step), summed over all ranks.
-Inputs are resident in HBM during the timed region; the working set of a step (several
-GB) is far larger than the 129 MB L2, so no flush is needed between steps.  With
---gpus N > 1 (torchrun) every rank trains its own replica on its own batch (weak
-scaling, no data-path collective).  --impl reference times the CPU oracle on a bounded
-sample of the same workload.
+TOPS: 2 x the in-bounds multiply-accumulates (taps that read inside the input; zero
+padding does no work) of every forward, data-gradient and weight-gradient convolution,
+the FCN decoder included, divided by the device time of the step, summed over all ranks.
+The dense count (every tap) is reported beside it.  Inputs are resident in HBM during
+the timed region; the working set of a network step (several GB) is far larger than the
+129 MB L2, so no flush is needed between steps (the single layer flushes L2 before each of
+its steps).  With --gpus N > 1 (torchrun) every rank trains its own replica on its own
+batch (weak scaling, no data-path collective).  --impl reference times the CPU oracle on a
+bounded sample of the same workload.
 """
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -33,10 +39,68 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 SITES = 64
+WORKLOADS = ["deeplabv3_r50_train", "fcn_vgg16_train", "deeplabv3_r50_infer", "fcn_vgg16_infer",
+             "single_layer"]
 
+
+# ------------------------------------------------------------------ layer geometry
+
+def fcn_layers(n, h, w, classes, width=1.0):
+    """(n, h, w, cin (real channels), cout, r, stride, pad, dil, first) of every FCN conv."""
+    from paper_2011_14504_gb300 import synthetic as S
+    out, hh, ww = [], h, w
+    for name, cin, cout, r, pad, relu in S.fcn_vgg16_channels(classes, width):
+        if name == "pool":
+            hh, ww = hh // 2, ww // 2
+            continue
+        out.append((n, hh, ww, 3 if cin == 4 else cin, cout, r, 1, pad, 1, cin == 4))
+    return out, (hh, ww)
+
+
+def deeplab_layers(sp, n, h):
+    """The same for every DeepLab conv, from the spec's geometry alone."""
+    from paper_2011_14504_gb300.work import out_size
+    per = []
+    sz = out_size(h, sp.stem.r, sp.stem.stride, sp.stem.pad, sp.stem.dil)
+    per.append((n, h, h, 3, sp.stem.cout, sp.stem.r, sp.stem.stride, sp.stem.pad, 1, True))
+    sz = (sz + 2 - 3) // 2 + 1
+    for b in sp.blocks:
+        s1 = sz
+        for cv in (b.conv1, b.conv2, b.conv3):
+            per.append((n, s1, s1, cv.cin, cv.cout, cv.r, cv.stride, cv.pad, cv.dil, False))
+            s1 = out_size(s1, cv.r, cv.stride, cv.pad, cv.dil)
+        if b.down:
+            per.append((n, sz, sz, b.down.cin, b.down.cout, 1, b.down.stride, 0, 1, False))
+        sz = s1
+    for cv in list(sp.aspp) + [sp.project, sp.head, sp.cls]:
+        per.append((n, sz, sz, cv.cin, cv.cout, cv.r, cv.stride, cv.pad, cv.dil, False))
+    per.append((n, 1, 1, sp.pool_conv.cin, sp.pool_conv.cout, 1, 1, 0, 1, False))
+    return per
+
+
+def step_macs(layers, train, extra=(0, 0)):
+    """(in-bounds, dense) MACs of an inference pass or a training step over `layers`;
+    `extra` is the (in-bounds, dense) MACs of one pass of the FCN decoder."""
+    from paper_2011_14504_gb300.work import conv_macs
+    f = [0, 0]
+    dg = [0, 0]
+    for (n, h, w, cin, cout, r, st, pad, dil, first) in layers:
+        m = conv_macs(n, h, w, cin, cout, r, st, pad, dil)
+        for i in range(2):
+            f[i] += m[i]
+            if not first:
+                dg[i] += m[i]
+    if not train:
+        return f[0] + extra[0], f[1] + extra[1]
+    return tuple(2 * f[i] + dg[i] + 3 * extra[i] for i in range(2))
+
+
+# ------------------------------------------------------------------ workloads
 
 class Workload:
-    """One benchmarked configuration: the network, its inputs and what a step counts."""
+    """One network configuration: the network, its inputs and what a step counts."""
+
+    single = False
 
     def __init__(self, name: str):
         self.name = name
@@ -46,6 +110,9 @@ class Workload:
         self.img = 512 if self.fcn else 513
         self.classes = 150 if self.fcn else 21
         self.labels = f"voronoi {SITES} sites" if self.fcn else "uniform, 5% ignore (255)"
+
+    def metric(self) -> str:
+        return "int8 conv TOPS (fwd+bwd)" if self.train else "int8 conv TOPS (fwd)"
 
     def config(self, world: int) -> dict:
         return {"workload": self.name + "_step" if self.train else self.name,
@@ -83,19 +150,98 @@ class Workload:
             return net.s_Ez if self.fcn else net.s_E
         return net.s_z
 
-    def macs(self, net) -> int:
-        return net.macs_step if self.train else net.macs_forward
+    def macs(self, net):
+        """(in-bounds, dense) MACs of one step."""
+        if self.train:
+            return net.macs_step, net.macs_step_dense
+        return net.macs_forward, net.macs_forward_dense
 
-    def conv_macs(self, net) -> dict:
-        """MACs per step of each convolution entry point (the decoder of FCN excluded)."""
-        if self.fcn:
-            layers = [(L.macs, L.layer_id == 0) for L in net.convs]
-        else:
-            layers = [(L.macs, L is net.stem) for L in net.layers.values()]
-        f = sum(m for m, _ in layers)
-        return {"iq_conv_fwd": f, "iq_conv_dgrad": sum(m for m, first in layers if not first),
-                "iq_conv_wgrad": f}
 
+class SingleLayer:
+    """One quantized conv layer: N=1, 64 -> 64 channels, 32x32, 3x3, stride 1, padding 1;
+    forward with integer L1BN + ReLU + Q_A, data gradient (SQ8) and weight gradient (GQ1).
+    Inputs: activations and errors int8 uniform on [-127, 127], weights UQ(UQ(N(0,
+    sqrt(2/576)), 24), 8), gamma / beta codes drawn on the 8-bit x2 grid, s_x = s_e = 2^-7."""
+
+    single = True
+    name = "single_layer"
+    train = True
+    batch = 1
+    N, H, C, K = 1, 32, 64, 64
+
+    def metric(self) -> str:
+        return "int8 conv TOPS (fwd+bwd)"
+
+    def config(self, world: int) -> dict:
+        return {"workload": "single_layer", "global_batch": self.N * world,
+                "layer": f"N={self.N} C={self.C} {self.H}x{self.H} K={self.K} 3x3 s1 p1",
+                "epilogue": "integer L1BN + ReLU + Q_A"}
+
+    def macs(self, layer=None):
+        from paper_2011_14504_gb300.work import conv_macs
+        inb, dense = conv_macs(self.N, self.H, self.H, self.C, self.K, 3, 1, 1)
+        return 3 * inb, 3 * dense
+
+    def host_inputs(self, seed=0):
+        import numpy as np
+        from paper_2011_14504_gb300 import synthetic as S
+        g = S.rng(seed)
+        x = S.int8_uniform(g, (self.N, self.H, self.H, self.C))
+        w = S.he_weights(g, (self.K, 3, 3, self.C), 9 * self.C)
+        gam, bet = S.bn_gamma_beta_codes(g, self.K)
+        e = S.int8_uniform(g, (self.N, self.H, self.H, self.K))
+        return x, w, gam.astype(np.int32), bet.astype(np.int32), e
+
+
+class LayerRun:
+    """Device buffers and the three calls of the single-layer workload."""
+
+    def __init__(self, sl: SingleLayer, dev):
+        import torch
+        from paper_2011_14504_gb300 import iq
+        x, w, gam, bet, e = sl.host_inputs(0)
+        self.iq = iq
+        t = lambda a: torch.from_numpy(a).to(dev)
+        sc = lambda v=0.0: torch.tensor([v], dtype=torch.float64, device=dev)
+        n, h, c, k = sl.N, sl.H, sl.C, sl.K
+        self.d = iq.conv_desc(n, h, h, c, k, 3, 3, 1, 1)
+        wf = t(w)
+        self.master = torch.empty(wf.shape, dtype=torch.int32, device=dev)
+        iq.iq_quantize(wf, 24, iq.IQ_MODE_UQ, self.master, sc())
+        self.wq = torch.empty(wf.shape, dtype=torch.int8, device=dev)
+        iq.iq_weight_requant(self.master, self.wq)
+        self.x, self.e = t(x), t(e)
+        self.gam, self.bet = t(gam), t(bet)
+        self.s_x, self.s_e = sc(2.0 ** -7), sc(2.0 ** -7)
+        self.a = torch.empty((n, h, h, k), dtype=torch.int8, device=dev)
+        self.X = torch.empty((n, h, h, k), dtype=torch.int16, device=dev)
+        self.dx = torch.empty((n, h, h, c), dtype=torch.int8, device=dev)
+        self.g = torch.empty_like(self.wq)
+        self.s_a, self.s_dx, self.s_g = sc(), sc(), sc()
+        self.codes = torch.empty(2 * k, dtype=torch.int32, device=dev)
+        self.scal = torch.zeros(iq.IQ_BN_SCALES, dtype=torch.float64, device=dev)
+        self.x16 = torch.empty(self.x.numel(), dtype=torch.float16, device=dev)
+        self.e16 = torch.empty(self.e.numel(), dtype=torch.float16, device=dev)
+        wsz = max(iq.iq_conv_fwd_workspace_size(self.d, True),
+                  iq.iq_conv_dgrad_workspace_size(self.d), iq.iq_conv_wgrad_workspace_size(self.d))
+        self.ws = torch.empty(wsz, dtype=torch.uint8, device=dev)
+
+    def step(self):
+        iq = self.iq
+        iq.iq_conv_fwd(self.d, self.x, self.s_x, self.wq, self.a, self.s_a, self.gam, self.bet,
+                       use_bn=True, relu=True, xhat=self.X, bn_codes=self.codes,
+                       bn_scales=self.scal, x_f16=self.x16, ws=self.ws)
+        iq.iq_conv_dgrad(self.d, self.e, self.s_e, self.wq, self.dx, self.s_dx, e_f16=self.e16,
+                         ws=self.ws)
+        iq.iq_conv_wgrad(self.d, self.e, self.s_e, self.x, self.s_x, self.g, self.s_g, gq_mode=1,
+                         seed=0, layer=0, step=0, e_f16=self.e16, x_f16=self.x16, ws=self.ws)
+
+
+def make_workload(name):
+    return SingleLayer() if name == "single_layer" else Workload(name)
+
+
+# ------------------------------------------------------------------ environment
 
 def peaks():
     try:
@@ -105,6 +251,30 @@ def peaks():
     except Exception:
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, \
             "fallback"
+
+
+def kernel_source_sha() -> str:
+    p = os.path.join(ROOT, "paper_2011_14504_gb300", "csrc", "iq_conv_tc.cu")
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def recorded_traffic(workload: str, kernel: int):
+    """DRAM bytes per launch of `kernel` in `workload`, from the committed ncu summary
+    profiles/traffic_<workload>.md, or None when there is none or the kernel source has
+    changed since the counters were taken."""
+    p = os.path.join(ROOT, "profiles", f"traffic_{workload}.md")
+    if not os.path.exists(p):
+        return None, None
+    txt = open(p).read()
+    sha = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", txt)
+    row = re.search(rf"^traffic kernel {kernel}:\s*([0-9.eE+]+) bytes per launch, "
+                    rf"([0-9.eE+]+) launches", txt, re.M)
+    if not sha or not row:
+        return None, None
+    if sha.group(1) != kernel_source_sha():
+        return None, "kernel source changed since the capture"
+    return float(row.group(1)), os.path.relpath(p, ROOT)
 
 
 class ClockSampler:
@@ -190,22 +360,32 @@ def max_over_ranks(v: float, world: int, device) -> float:
     return float(t.item())
 
 
+def cpu_threads():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
 # ------------------------------------------------------------------ oracle (CPU) leg
 
-def oracle_sample_step(wl: Workload):
-    """One step of the CPU oracle on a bounded sample of the workload (the full-width
-    network, one image at 128x128 (FCN) or 129x129 (DeepLab), about 10-30 s of CPU work)."""
+def oracle_sample_step(wl):
+    """One step of the CPU oracle on a bounded sample of the workload: the full-width network
+    on one image at 128x128 (FCN) or 129x129 (DeepLab), about 10-30 s of CPU work, or the
+    single layer itself.  Returns (run, in-bounds MACs of one run, description)."""
     from paper_2011_14504_gb300 import synthetic as S
+    if wl.single:
+        return oracle_single_layer(wl)
     g = S.rng(1)
     if wl.fcn:
         from oracle.fcn import OracleFcn
+        from paper_2011_14504_gb300.work import transposed_macs
         n, h = 1, 128
         chans = S.fcn_vgg16_channels(wl.classes, 1.0)
         wts, up = S.fcn_vgg16_weights(0, wl.classes, 1.0)
         ora = OracleFcn(chans, wts, up, wl.classes, seed=0)
-        macs = fcn_step_macs(n, h, h, wl.classes)
-        if not wl.train:
-            macs = fcn_forward_macs(n, h, h, wl.classes)
+        layers, (hs, ws_) = fcn_layers(n, h, h, wl.classes)
+        macs = step_macs(layers, wl.train, transposed_macs(n, hs, ws_, wl.classes, 64, 32, 16))[0]
         name = "FCN-VGG16"
     else:
         from oracle.deeplab import OracleDeepLab
@@ -213,7 +393,7 @@ def oracle_sample_step(wl: Workload):
         sp = S.deeplabv3_r50_spec(wl.classes, 1.0)
         w, gm, bm = S.deeplabv3_r50_init(0, sp)
         ora = OracleDeepLab(sp, w, gm, bm, seed=0)
-        macs = deeplab_macs(sp, n, h, wl.train)
+        macs = step_macs(deeplab_layers(sp, n, h), wl.train)[0]
         name = "DeepLabv3-ResNet50"
     img, lab = wl.inputs(g, n, h)
 
@@ -225,65 +405,22 @@ def oracle_sample_step(wl: Workload):
     return run, macs, f"{name} {kind}, N={n}, {h}x{h}, full width, {wl.classes} classes"
 
 
-def deeplab_macs(sp, n, h, train):
-    """Forward (+ data and weight gradient) MACs of the DeepLab convolutions for n images of
-    h x h, from the conv geometry alone."""
-    def out(sz, cv):
-        return (sz + 2 * cv.pad - cv.dil * (cv.r - 1) - 1) // cv.stride + 1
-    per = []
-    sz = out(h, sp.stem)
-    per.append((n * sz * sz * sp.stem.cout * 49 * 3, True))
-    sz = (sz + 2 - 3) // 2 + 1
-    for b in sp.blocks:
-        s1 = sz
-        for cv in (b.conv1, b.conv2, b.conv3):
-            o = out(s1, cv)
-            per.append((n * o * o * cv.cout * cv.r * cv.r * cv.cin, False))
-            s1 = o
-        if b.down:
-            per.append((n * s1 * s1 * b.down.cout * b.down.cin, False))
-        sz = s1
-    for cv in list(sp.aspp) + [sp.project, sp.head, sp.cls]:
-        per.append((n * sz * sz * cv.cout * cv.r * cv.r * cv.cin, False))
-    per.append((n * sp.pool_conv.cout * sp.pool_conv.cin, False))
-    f = sum(m for m, _ in per)
-    if not train:
-        return f
-    return f + sum(m for m, first in per if not first) + f
+def oracle_single_layer(sl: SingleLayer):
+    """The single layer on the oracle: conv, L1BN + ReLU + Q_A, data gradient + SQ8, weight
+    gradient + RQ8, repeated 250 times (one run, about 10 s on 8 to 16 cores)."""
+    import oracle as O
+    x, w, gam, bet, e = sl.host_inputs(0)
+    wq = O.requant_master(O.uq(w, 24)).astype("int8")
+    cv = O.Conv(sl.N, sl.H, sl.H, sl.C, sl.K, 3, 3, 1, 1)
+    reps = 250
 
-
-def fcn_forward_macs(n, h, w, classes, width=1.0):
-    from paper_2011_14504_gb300 import synthetic as S
-    hh, ww, f = h, w, 0
-    for name, cin, cout, r, pad, relu in S.fcn_vgg16_channels(classes, width):
-        if name == "pool":
-            hh, ww = hh // 2, ww // 2
-            continue
-        f += n * hh * ww * cout * r * r * (3 if cin == 4 else cin)
-    return f + n * h * w * classes * 4
-
-
-def fcn_step_macs(n, h, w, classes, width=1.0):
-    from paper_2011_14504_gb300 import synthetic as S
-    hh, ww = h, w
-    f = dg = 0
-    for name, cin, cout, r, pad, relu in S.fcn_vgg16_channels(classes, width):
-        if name == "pool":
-            hh, ww = hh // 2, ww // 2
-            continue
-        m = n * hh * ww * cout * r * r * (3 if cin == 4 else cin)
-        f += m
-        if cin != 4:
-            dg += m
-    up = n * h * w * classes * 4
-    return f + dg + f + 3 * up
-
-
-def cpu_threads():
-    try:
-        return len(os.sched_getaffinity(0))
-    except Exception:
-        return os.cpu_count() or 1
+    def run():
+        for _ in range(reps):
+            acc = O.conv_fwd(cv, x, wq)
+            O.bn_fwd(acc.reshape(-1, sl.K), 2.0 ** -14, gam, bet)
+            O.sq_int(O.conv_dgrad(cv, e, wq), 2.0 ** -14, 8)
+            O.rq_int(O.conv_wgrad(cv, e, x), 2.0 ** -14, 8, 1, 0, 0, 0, 0)
+    return run, reps * sl.macs()[0], f"single layer x{reps}: fwd + L1BN + dgrad + wgrad"
 
 
 def run_reference(args, rank, world):
@@ -291,7 +428,7 @@ def run_reference(args, rank, world):
         return 0
     import oracle
     oracle.build()
-    wl = Workload(args.workload)
+    wl = make_workload(args.workload)
     run, macs, sample = oracle_sample_step(wl)
     for _ in range(min(args.warmup, 1)):
         run()
@@ -302,7 +439,7 @@ def run_reference(args, rank, world):
         times.append(time.perf_counter() - t0)
     t = sum(times) / len(times)
     v = 2 * macs / t / 1e12
-    line = {"impl": "reference", "metric": metric_name(wl), "value": v, "unit": "TOPS",
+    line = {"impl": "reference", "metric": wl.metric(), "value": v, "unit": "TOPS",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int8", "data": "synthetic",
@@ -314,45 +451,71 @@ def run_reference(args, rank, world):
     return 0
 
 
-def metric_name(wl: Workload) -> str:
-    return "int8 conv TOPS (fwd+bwd)" if wl.train else "int8 conv TOPS (fwd)"
-
-
 # ------------------------------------------------------------------ GPU leg
 
+HBM_KERNELS = (10, 11, 12, 13, 14, 15, 16, 17, 18, 19, 20)
+
+
+def summarize_kernels(iq, ktimes, steps, ms_step, pk):
+    """Per-kernel figures of the attribution steps: the dominant conv kernel's roofline and
+    the bandwidth kernels' achieved GB/s against the HBM peak."""
+    byk = {}
+    for r in ktimes:
+        t = byk.setdefault(r["kernel"], {"ms": 0.0, "macs": 0.0, "dense": 0.0, "bytes": 0.0,
+                                         "launches": 0})
+        t["ms"] += r["ms"]
+        t["macs"] += r["macs"]
+        t["dense"] += r["dense_macs"]
+        t["bytes"] += r["bytes"]
+        t["launches"] += r["launches"]
+    conv = {k: v for k, v in byk.items() if k in iq.CONV_KERNELS}
+    hbm = pk.get("hbm_gbs", 6800.0)
+    table = {}
+    for k, v in sorted(byk.items()):
+        if k not in HBM_KERNELS or v["ms"] <= 0:
+            continue
+        gbs = v["bytes"] / (v["ms"] * 1e-3) / 1e9
+        table[iq.KERNEL_NAMES.get(k, str(k))] = {
+            "launches_per_step": v["launches"] / steps, "ms_per_step": v["ms"] / steps,
+            "gb_per_step": v["bytes"] / steps / 1e9, "achieved_gbs": gbs,
+            "frac_of_hbm": gbs / hbm}
+    return byk, conv, table
+
+
 def run_ours(args, rank, world, local):
-    import numpy as np
     import torch
 
     from paper_2011_14504_gb300 import iq
-    from paper_2011_14504_gb300 import synthetic as S
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     iq.load()
-    wl = Workload(args.workload)
-    net = wl.build(dev, rank)
-    g = S.rng(1000 + rank)
-    img_np, lab_np = wl.inputs(g, wl.batch, wl.img)
-    img = torch.from_numpy(img_np).to(dev)
-    lab = torch.from_numpy(lab_np).to(dev) if lab_np is not None else None
+    wl = make_workload(args.workload)
     stream = torch.cuda.current_stream(dev)
+    pk, pk_kind = peaks()
 
-    # per-operation attribution with events on the launching stream
-    op_events = {}
-
-    def timed(kind, fn):
-        def wrap(*a, **k):
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            fn(*a, **k)
-            e1.record(stream)
-            op_events.setdefault(kind, []).append((e0, e1, a[0]))
-        return wrap
+    if wl.single:
+        run = LayerRun(wl, dev)
+        step_fn = run.step
+        inputs_h = [(run.x, run.x.cpu().pin_memory()), (run.e, run.e.cpu().pin_memory())]
+        result = run.s_a
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    else:
+        from paper_2011_14504_gb300 import synthetic as S
+        net = wl.build(dev, rank)
+        g = S.rng(1000 + rank)
+        img_np, lab_np = wl.inputs(g, wl.batch, wl.img)
+        img = torch.from_numpy(img_np).to(dev)
+        lab = torch.from_numpy(lab_np).to(dev) if lab_np is not None else None
+        step_fn = lambda: wl.step(net, img, lab)
+        inputs_h = [(img, torch.from_numpy(img_np).pin_memory())]
+        if lab is not None:
+            inputs_h.append((lab, torch.from_numpy(lab_np).pin_memory()))
+        result = wl.result(net)
+        flush = None
 
     for _ in range(args.warmup):
-        wl.step(net, img, lab)
+        step_fn()
     torch.cuda.synchronize(dev)
 
     # The step as a CUDA graph (one captured step, replayed): every kernel of the step is
@@ -364,13 +527,13 @@ def run_ours(args, rank, world, local):
         side = torch.cuda.Stream(dev)
         side.wait_stream(stream)
         with torch.cuda.stream(side):
-            wl.step(net, img, lab)
+            step_fn()
         stream.wait_stream(side)
         torch.cuda.synchronize(dev)
         graph = torch.cuda.CUDAGraph()
         l0 = iq.launch_count()
         with torch.cuda.graph(graph):
-            wl.step(net, img, lab)
+            step_fn()
             iq.iq_rq_epoch_advance()
         graph_launches = iq.launch_count() - l0
         graph.replay()
@@ -386,99 +549,103 @@ def run_ours(args, rank, world, local):
         if graph is not None:
             graph.replay()
         else:
-            wl.step(net, img, lab)
+            step_fn()
 
     launches0 = iq.launch_count()
     barrier(world)
     torch.cuda.synchronize(dev)
     with ClockSampler(local) as clk:
-        t_start = torch.cuda.Event(enable_timing=True)
-        t_end = torch.cuda.Event(enable_timing=True)
-        t_start.record(stream)
-        for _ in range(args.steps):
-            run_step()
-        t_end.record(stream)
-        torch.cuda.synchronize(dev)
+        if flush is None:
+            t_start = torch.cuda.Event(enable_timing=True)
+            t_end = torch.cuda.Event(enable_timing=True)
+            t_start.record(stream)
+            for _ in range(args.steps):
+                run_step()
+            t_end.record(stream)
+            torch.cuda.synchronize(dev)
+            ms_total = t_start.elapsed_time(t_end)
+        else:
+            # a small layer: flush L2 (write 256 MB) before each step, time the step alone
+            evs = []
+            for _ in range(args.steps):
+                flush.fill_(1)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                run_step()
+                e1.record(stream)
+                evs.append((e0, e1))
+            torch.cuda.synchronize(dev)
+            ms_total = sum(a.elapsed_time(b) for a, b in evs)
     barrier(world)
     launches = (graph_launches * args.steps if graph is not None
                 else iq.launch_count() - launches0)
     iq.iq_device_status(stream)     # raises if a bounded device wait gave up
 
-    # per-operation attribution (eager steps, CUDA events around each conv call on the stream)
-    # and, inside those calls, events around every launch of the tensor-core conv kernels
-    orig = {k: getattr(iq, k) for k in ("iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad")}
-    for k, f in orig.items():
-        setattr(iq, k, timed(k, f))
+    # per-kernel attribution: eager steps with the library's kernel timing on (CUDA events
+    # on the launching stream around every conv and bandwidth kernel launch)
     iq.iq_kernel_timing_begin()
     for _ in range(args.steps):
-        wl.step(net, img, lab)
+        if flush is not None:
+            flush.fill_(1)
+        step_fn()
     torch.cuda.synchronize(dev)
     ktimes = iq.iq_kernel_timing_end()
-    for k, f in orig.items():
-        setattr(iq, k, f)
-    ms_total = t_start.elapsed_time(t_end)
     ms_total = max_over_ranks(ms_total, world, dev)
     ms_step = ms_total / args.steps
-    macs = wl.macs(net)
+    macs, macs_dense = wl.macs(run if wl.single else net)
     tops = 2 * macs * world / (ms_step * 1e-3) / 1e12
+    tops_dense = 2 * macs_dense * world / (ms_step * 1e-3) / 1e12
 
-    # roofline of the dominant kernel: the tensor-core conv kernel with the largest summed
-    # event time over the attribution steps; achieved = its algorithmic flops (2 x the MACs
-    # of the calls that launched it) / its summed launch time
-    per = {}
-    for kind, evs in op_events.items():
-        per[kind] = sum(e0.elapsed_time(e1) for e0, e1, _ in evs)
-    byk = {}
-    for r in ktimes:
-        t = byk.setdefault(r["kernel"], {"ms": 0.0, "macs": 0.0, "launches": 0})
-        t["ms"] += r["ms"]
-        t["macs"] += r["macs"]
-        t["launches"] += r["launches"]
-    pk, pk_kind = peaks()
-    peak_tf = pk.get("bf16_tflops_sustained", pk.get("bf16_tflops"))
-    dk = max(byk, key=lambda k: byk[k]["ms"])
-    kt = byk[dk]
+    # roofline of the dominant kernel: the conv kernel with the largest summed event time
+    # over the attribution steps; achieved = 2 x the in-bounds MACs of the calls that
+    # launched it / its summed launch time
+    byk, conv, hbm_table = summarize_kernels(iq, ktimes, args.steps, ms_step, pk)
+    peak_s = pk.get("bf16_tflops_sustained", pk.get("bf16_tflops"))
+    peak_b = pk.get("bf16_tflops", peak_s)
+    dk = max(conv, key=lambda k: conv[k]["ms"])
+    kt = conv[dk]
     achieved = 2 * kt["macs"] / (kt["ms"] * 1e-3) / 1e12
+    traffic, traffic_src = recorded_traffic(wl.config(1)["workload"], dk)
     roofline = {"bound": "tensor", "kernel": iq.KERNEL_NAMES.get(dk, str(dk)),
-                "achieved": achieved, "peak": peak_tf, "unit": "TFLOP/s",
-                "frac": achieved / peak_tf, "traffic": None,
-                "peak_source": f"{pk_kind} fp16/bf16 dense sustained (MEASURED_PEAKS.json)",
+                "achieved": achieved, "peak": peak_s, "unit": "TFLOP/s",
+                "frac": achieved / peak_s, "traffic": traffic,
+                "traffic_source": traffic_src,
+                "peak_source": f"{pk_kind} fp16/bf16 dense sustained (MEASURED_PEAKS.json); "
+                               "the int8 codes ride exactly on the fp16 tensor pipe",
+                "frac_of_burst_peak": achieved / peak_b,
+                "achieved_dense_macs": 2 * kt["dense"] / (kt["ms"] * 1e-3) / 1e12,
                 "launches_per_step": kt["launches"] / args.steps,
                 "kernel_ms_per_step": kt["ms"] / args.steps,
-                "share_of_step": kt["ms"] / args.steps / (ms_total / args.steps),
+                "share_of_step": kt["ms"] / args.steps / ms_step,
                 "kernels_ms_per_step": {iq.KERNEL_NAMES.get(k, str(k)): v["ms"] / args.steps
-                                        for k, v in byk.items()},
-                "op_ms_per_step": {k: v / args.steps for k, v in per.items()}}
+                                        for k, v in sorted(conv.items())},
+                "kernels_tflops": {iq.KERNEL_NAMES.get(k, str(k)):
+                                   2 * v["macs"] / (v["ms"] * 1e-3) / 1e12
+                                   for k, v in sorted(conv.items()) if v["ms"] > 0}}
 
     # end to end: host (pinned) inputs copied in, a result scalar read back, every step
-    img_h = torch.from_numpy(img_np).pin_memory()
-    lab_h = torch.from_numpy(lab_np).pin_memory() if lab is not None else None
     res_h = torch.empty(1, dtype=torch.float64).pin_memory()
-    img_d = torch.empty_like(img)
-    lab_d = torch.empty_like(lab) if lab is not None else None
     e2e_steps = max(1, min(args.steps, 3))
     barrier(world)
     torch.cuda.synchronize(dev)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
+    evs = []
     for _ in range(e2e_steps):
-        if graph is not None:
-            # the captured step reads the static input buffers
-            img.copy_(img_h, non_blocking=True)
-            if lab is not None:
-                lab.copy_(lab_h, non_blocking=True)
-            graph.replay()
-        else:
-            img_d.copy_(img_h, non_blocking=True)
-            if lab_d is not None:
-                lab_d.copy_(lab_h, non_blocking=True)
-            wl.step(net, img_d, lab_d)
-        res_h.copy_(wl.result(net), non_blocking=True)
-    e1.record(stream)
+        if flush is not None:
+            flush.fill_(1)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        # the captured step reads the static input buffers
+        for d_t, h_t in inputs_h:
+            d_t.copy_(h_t, non_blocking=True)
+        run_step()
+        res_h.copy_(result, non_blocking=True)
+        e1.record(stream)
+        evs.append((e0, e1))
     torch.cuda.synchronize(dev)
     iq.iq_device_status(stream)
-    ms_e2e = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world, dev)
+    ms_e2e = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs) / e2e_steps, world, dev)
     tops_e2e = 2 * macs * world / (ms_e2e * 1e-3) / 1e12
 
     if rank == 0:
@@ -486,9 +653,9 @@ def run_ours(args, rank, world, local):
         try:
             import oracle
             oracle.build()
-            run, omacs, sample = oracle_sample_step(wl)
+            orun, omacs, sample = oracle_sample_step(wl)
             t0 = time.perf_counter()
-            run()
+            orun()
             t = time.perf_counter() - t0
             cpu = {"value": 2 * omacs / t / 1e12, "unit": "TOPS", "cores": cpu_threads(),
                    "kind": "oracle", "sample": sample, "seconds": t}
@@ -496,25 +663,33 @@ def run_ours(args, rank, world, local):
             cpu = {"value": None, "unit": "TOPS", "cores": cpu_threads(), "kind": "oracle",
                    "sample": f"failed: {ex}"}
         cfg = wl.config(world)
-        cfg.update({"macs_per_image_step": macs // wl.batch, "parallelism": f"replicas x{world}",
-                    "l2": "working set >> 129 MB L2, no flush",
+        cfg.update({"parallelism": f"replicas x{world}",
+                    "l2": ("flushed before each step (256 MB write)" if flush is not None
+                           else "working set >> 129 MB L2, no flush"),
                     "launch": "cuda graph of one step, replayed" if graph is not None
                     else "eager"})
-        line = {"metric": metric_name(wl), "value": tops, "unit": "TOPS",
+        if not wl.single:
+            cfg["macs_per_image_step"] = macs // wl.batch
+        line = {"metric": wl.metric(), "value": tops, "unit": "TOPS",
                 "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
                 "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+                "value_dense_macs": tops_dense,
+                "macs_per_step": {"in_bounds": macs, "dense": macs_dense},
                 "images_per_s": wl.batch * world / (ms_step * 1e-3),
                 "config": cfg,
                 "e2e": {"value": tops_e2e, "unit": "TOPS",
-                        "h2d_bytes_per_step": img_h.numel() + (lab_h.numel() if lab_h is not None
-                                                               else 0),
+                        "h2d_bytes_per_step": sum(h.numel() * h.element_size()
+                                                  for _, h in inputs_h),
                         "d2h_bytes_per_step": 8, "images_per_s": wl.batch * world /
-                        (ms_e2e * 1e-3)},
+                        (ms_e2e * 1e-3), "ms_per_step": ms_e2e},
                 "gpu_launches": launches,
                 "roofline": roofline,
+                "hbm_kernels": hbm_table,
                 "clocks": clk.summary(),
                 "cpu_baseline": cpu}
+        if wl.single:
+            line["us_per_step"] = ms_step * 1e3
         print(json.dumps(line))
     return 0
 
@@ -525,9 +700,7 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="fcn_vgg16_train",
-                    choices=["fcn_vgg16_train", "deeplabv3_r50_train", "fcn_vgg16_infer",
-                             "deeplabv3_r50_infer"])
+    ap.add_argument("--workload", default="deeplabv3_r50_train", choices=WORKLOADS)
     args = ap.parse_args()
     rank, world, local = dist_setup(args.gpus)
     if args.impl == "reference":

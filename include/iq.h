@@ -105,26 +105,45 @@ unsigned long long iq_launch_count(void);
 iq_status iq_device_status(int32_t* code, iq_stream stream);
 
 /* Kernel timing -- a measurement aid (the paper has no counterpart).  Between
- * iq_kernel_timing_begin and iq_kernel_timing_end, every launch of a tensor-core convolution
- * kernel (up to 4096 of them) is bracketed by a pair of CUDA events recorded on its launching
- * stream, and tagged with the kernel, the calling operation and the operation's algorithmic
- * multiply-accumulates N P Q K R S C / groups (counted once per call, on its first bracketed
- * launch).  Use it on eagerly launched calls, not inside a CUDA graph capture.
+ * iq_kernel_timing_begin and iq_kernel_timing_end, every launch of a convolution kernel and
+ * of the main bandwidth-bound kernels (up to 8192 launches) is bracketed by a pair of CUDA
+ * events recorded on its launching stream.  A convolution launch is tagged with its kernel,
+ * the calling operation and the operation's multiply-accumulates (counted once per call, on
+ * its first bracketed launch): `macs` counts the in-bounds products only (the taps that read
+ * inside the input), `dense_macs` every tap N P Q K R S C / groups.  A bandwidth launch is
+ * tagged with its kernel and `bytes`, the bytes its pass must read and write (each operand
+ * once).  Use it on eagerly launched calls, not inside a CUDA graph capture.
  * iq_kernel_timing_end waits for the recorded events, writes one iq_kernel_time per
  * (kernel, op) pair seen (at most `capacity`, the count in *n_out), and stops recording.
  * Errors: IQ_ERR_INVALID_ARG for null pointers, IQ_ERR_CUDA when an event call fails. */
 enum {
     IQ_KERNEL_CONV_PIXEL_MAJOR = 1,    /* all-TMA kernel, forward / data gradient (k_conv_tct)  */
     IQ_KERNEL_CONV_CHANNEL_MAJOR = 2,  /* channel-major kernel, <= 128 output channels (k_conv_tcc) */
-    IQ_KERNEL_CONV_WGRAD = 3           /* all-TMA kernel, weight gradient                       */
+    IQ_KERNEL_CONV_WGRAD = 3,          /* all-TMA kernel, weight gradient                       */
+    IQ_KERNEL_CONV_CPASYNC = 4,        /* cp.async-fed forward kernel (k_conv_tcq)               */
+    IQ_KERNEL_CONV_GATHER = 5,         /* register-gather kernel (k_conv_tcp)                    */
+    IQ_KERNEL_CONV_SIMT = 6,           /* CUDA-core kernel (k_conv_simt)                         */
+    IQ_KERNEL_BN_DEV = 10,             /* L1BN deviation pass (k_bn_dev)                         */
+    IQ_KERNEL_BN_REQUANT = 11,         /* L1BN acc -> X -> A pass (k_bn_requant)                 */
+    IQ_KERNEL_BNB_PASS1 = 12,          /* L1BN backward passes (k_bnb_pass1..3)                  */
+    IQ_KERNEL_BNB_PASS2 = 13,
+    IQ_KERNEL_BNB_PASS3 = 14,
+    IQ_KERNEL_COMBINE_MAX = 15,        /* iq_combine, max |z| pass                               */
+    IQ_KERNEL_COMBINE_CODES = 16,      /* iq_combine, codes pass                                 */
+    IQ_KERNEL_SQ_CODES = 17,           /* SQ codes of int32 / int64 sums (k_sq_i32_i8x4, k_sq_int) */
+    IQ_KERNEL_CODES_TO_F16 = 18,       /* fp16 carrier copy of int8 codes (k_codes_to_f16)       */
+    IQ_KERNEL_ABSMAX = 19,             /* max |q| pass of SQ / RQ (k_absmax_int)                 */
+    IQ_KERNEL_RQ_CODES = 20            /* RQ codes (k_rq_int)                                    */
 };
 typedef struct iq_kernel_time {
-    int32_t kernel;     /* IQ_KERNEL_CONV_* */
-    int32_t op;         /* 1 iq_conv_fwd, 2 iq_conv_dgrad, 3 iq_conv_wgrad */
+    int32_t kernel;     /* IQ_KERNEL_* */
+    int32_t op;         /* 1 iq_conv_fwd, 2 iq_conv_dgrad, 3 iq_conv_wgrad; 0 bandwidth kernels */
     int32_t launches;   /* bracketed launches */
     int32_t pad;
     double ms;          /* summed event time of those launches, milliseconds */
-    double macs;        /* summed algorithmic multiply-accumulates of their calls */
+    double macs;        /* summed in-bounds multiply-accumulates of their calls */
+    double dense_macs;  /* summed dense multiply-accumulates of their calls */
+    double bytes;       /* summed algorithmic bytes of the bandwidth launches */
 } iq_kernel_time;
 iq_status iq_kernel_timing_begin(void);
 iq_status iq_kernel_timing_end(iq_kernel_time* out, int32_t capacity, int32_t* n_out);
@@ -270,12 +289,14 @@ iq_status iq_bn_int_fwd(const int32_t* acc, int64_t m, int32_t c, const double* 
  * plugin inside a host application that owns all device allocations, a real-time loop
  * that must not allocate after start-up).  Its scratch is a fixed file-scope device
  * array of 320 KB that every GPU loading the library keeps until process exit; it
- * accepts c <= 4096 channels and returns IQ_ERR_UNSUPPORTED above that.  The first call
- * on a device looks up that array's device address (one-time set-up, guarded by a
- * lock); make that first call before any stream capture.  All calls share the one
- * array: every call re-initialises the statistics it needs, but calls whose work
- * overlaps on the GPU (different streams, no ordering) race on it.  Otherwise identical
- * to iq_bn_int_fwd, with the same outputs. */
+ * accepts c <= 4096 channels and returns IQ_ERR_UNSUPPORTED above that.  Every call looks
+ * up that array's device address in the CUDA context current at the call (the address
+ * belongs to a context, not to a device, so a context the host application made current,
+ * or one created after a reset, is served correctly); the first call in a context also
+ * loads the library's device code there, so make it before any stream capture.  All calls
+ * share the one array: every call re-initialises the statistics it needs, but calls whose
+ * work overlaps on the GPU (different streams, no ordering) race on it.  Otherwise
+ * identical to iq_bn_int_fwd, with the same outputs. */
 iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_t c, const double* s_acc,
                                 const int32_t* gamma, const int32_t* beta,
                                 const iq_bn_bits* bits, int16_t* xhat, int8_t* a, double* s_a,
@@ -476,7 +497,8 @@ iq_status iq_ce_grad(const int8_t* z, const double* s_z, const uint8_t* labels, 
  * x2 grid (value master 2^(2-k_u)), lr = 2^-lr_log2, and the codes gamma = UQ2(master,
  * k_gamma), beta = UQ2(master, k_beta) used by the forward.  All arrays int32[c] on the
  * device (c <= 4096, else IQ_ERR_UNSUPPORTED); gamma_master / beta_master in/out, gamma /
- * beta out.  ws >= 4096 bytes + 2c (reserved).  One launch. */
+ * beta out.  ws / ws_bytes are reserved: the update needs no scratch, and NULL / 0 are
+ * accepted.  One launch. */
 iq_status iq_bn_update(int32_t* gamma_master, int32_t* beta_master, int32_t* gamma,
                        int32_t* beta, const int64_t* dgamma, const int64_t* dbeta,
                        const double* s_e, const double* bn_scales, int32_t c,

@@ -10,7 +10,6 @@
 #include "iq_internal.cuh"
 
 #include <climits>
-#include <mutex>
 
 namespace iq {
 
@@ -493,8 +492,10 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
                              int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
                              cudaStream_t st) {
     RowGrid rg = row_grid(m, C / 4);
+    kt_pre(st);
     k_bn_dev<<<rg.grid, kThreads, 0, st>>>(acc, m, C, rg.cg, s);
     IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, IQ_KERNEL_BN_DEV, 4.0 * (double)m * C);
     const int fb = (C + kFinThreads - 1) / kFinThreads;
     k_bn_fin1<<<fb, kFinThreads, 0, st>>>(s, m, C, s_acc, b);
     IQ_LAUNCH_CHECK();
@@ -507,8 +508,10 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
     k_bn_fin5<<<fb, kFinThreads, 0, st>>>(s, C, s_acc, gamma, beta, b);
     IQ_LAUNCH_CHECK();
     ChanGrid g2 = chan_grid(m, C / 4, 152 * 16);
+    kt_pre(st);
     k_bn_requant<<<g2.blocks, kThreads, 0, st>>>(acc, m, C, s, b.k_xhat, b.k_a, xhat, a);
     IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, IQ_KERNEL_BN_REQUANT, (double)m * C * (xhat ? 7.0 : 5.0));
     k_bn_export<<<(C + 255) / 256, 256, 0, st>>>(s, C, s.codes, s_a, bn_codes, bn_scales,
                                                  bn_fixed);
     IQ_LAUNCH_CHECK();
@@ -1035,16 +1038,20 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     k_bnb_init<<<(c + 255) / 256, 256, 0, st>>>(w, c);
     IQ_LAUNCH_CHECK();
     RowGrid rg = row_grid(m, c / 4);
+    kt_pre(st);
     k_bnb_pass1<<<rg.grid, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, rg.cg, w);
     IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, IQ_KERNEL_BNB_PASS1, 4.0 * (double)m * c);
     k_bnb_fin1<<<1, 1, 0, st>>>(w, s_e, b.k_gamma, k_e2);
     IQ_LAUNCH_CHECK();
     const int tb2 = (int)(((int64_t)c * kTab2 + kThreads - 1) / kThreads);
     k_bnb_tab2<<<tb2 < 152 * 4 ? tb2 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, w);
     IQ_LAUNCH_CHECK();
     RowGrid rt = row_grid(m, c / 4, 152 * 8, kTabCG);
+    kt_pre(st);
     k_bnb_pass2<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w);
     IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, IQ_KERNEL_BNB_PASS2, 4.0 * (double)m * c);
     const int fb = (c + kFinThreads - 1) / kFinThreads;
     k_bnb_fin2a<<<fb, kFinThreads, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma);
     IQ_LAUNCH_CHECK();
@@ -1055,8 +1062,10 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     const int tb3 = (int)(((int64_t)c * kTab3 + kThreads - 1) / kThreads);
     k_bnb_tab3<<<tb3 < 152 * 4 ? tb3 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, 8, w);
     IQ_LAUNCH_CHECK();
+    kt_pre(st);
     k_bnb_pass3<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w, e);
     IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, IQ_KERNEL_BNB_PASS3, 5.0 * (double)m * c);
     if (dgamma)
         IQ_CUDA_CHECK(cudaMemcpyAsync(dgamma, w.sg, sizeof(int64_t) * c, cudaMemcpyDeviceToDevice, st));
     if (dbeta)
@@ -1077,9 +1086,6 @@ constexpr size_t kBnNoAllocBytes = 320 * 1024;    // scratch for up to kBnNoAllo
 
 static __device__ __align__(256) unsigned char g_bn_noalloc_scratch[kBnNoAllocBytes];
 
-std::mutex g_bn_noalloc_mu;
-void* g_bn_noalloc_ptr[256] = {};                 // device address of the array, per device
-
 }  // namespace
 
 extern "C" iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_t c,
@@ -1090,22 +1096,14 @@ extern "C" iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_
                                            int64_t* bn_fixed, iq_stream stream) {
     if (c > kBnNoAllocMaxC || bn_fwd_ws_bytes(c > 0 ? c : 1) > kBnNoAllocBytes)
         return IQ_ERR_UNSUPPORTED;
-    int dev = -1;
-    IQ_CUDA_CHECK(cudaGetDevice(&dev));
-    if (dev < 0 || dev >= 256) return IQ_ERR_UNSUPPORTED;
+    // The host-side name of the array is not a device address.  Its device address belongs
+    // to the CUDA context that is current now (the primary context of the current device for
+    // runtime-API callers, or a context the host application made current itself), and it
+    // changes when that context is destroyed and another one created.  So it is looked up on
+    // every call, in the current context -- a host-side table lookup, no device work.
     void* ws = nullptr;
-    {
-        // one-time set-up on this device: the host-side name of the array is not a device
-        // address, so ask the runtime for the address it has on the current device
-        std::lock_guard<std::mutex> lock(g_bn_noalloc_mu);
-        if (!g_bn_noalloc_ptr[dev]) {
-            void* p = nullptr;
-            cudaError_t e = cudaGetSymbolAddress(&p, g_bn_noalloc_scratch);
-            if (e != cudaSuccess || !p) return IQ_ERR_CUDA;
-            g_bn_noalloc_ptr[dev] = p;
-        }
-        ws = g_bn_noalloc_ptr[dev];
-    }
+    cudaError_t e = cudaGetSymbolAddress(&ws, g_bn_noalloc_scratch);
+    if (e != cudaSuccess || !ws) return IQ_ERR_CUDA;
     // the statistics in the scratch are re-initialised by every call (zero sums,
     // min/max sentinels) before they are accumulated
     return iq_bn_int_fwd(acc, m, c, s_acc, gamma, beta, bits, xhat, a, s_a, bn_codes, bn_scales,
@@ -1196,7 +1194,8 @@ extern "C" iq_status iq_bn_update(int32_t* gamma_master, int32_t* beta_master, i
     const iq_bn_bits b = bn_bits_or_default(bits);
     if (!bn_bits_valid(b) || k_u <= b.k_gamma || k_u <= b.k_beta || k_u > 31) return IQ_ERR_INVALID_ARG;
     if (lr_log2 < 0 || lr_log2 > 60) return IQ_ERR_INVALID_ARG;
-    if (!ws || ws_bytes < 4096 + 2 * (size_t)c) return IQ_ERR_WORKSPACE;
+    (void)ws;        // reserved: the update needs no scratch (NULL and any size accepted)
+    (void)ws_bytes;
     if (c > 4096) return IQ_ERR_UNSUPPORTED;
     cudaStream_t st = (cudaStream_t)stream;
     const int sh = (k_u - 2) - lr_log2;

@@ -465,11 +465,34 @@ static bool crs_overflow(const iq_conv_desc* d) {
     return crs * 127 * 127 >= (int64_t(1) << 31);
 }
 
-// algorithmic multiply-accumulates of one convolution pass: N P Q K R S C / groups
-static double conv_macs(const iq_conv_desc* d) {
+// multiply-accumulates of one convolution pass, dense: N P Q K R S C / groups (every tap,
+// the zero padding included)
+static double conv_macs_dense(const iq_conv_desc* d) {
     const int64_t P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
     const int64_t Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
     return (double)d->n * P * Q * d->k * d->r * d->s * (double)(d->c / d->groups);
+}
+
+// number of (output index, tap) pairs of one spatial dimension whose input index
+// o stride + t dil - pad lies inside [0, extent)
+static int64_t inbounds_pairs(int64_t extent, int64_t out, int taps, int stride, int dil,
+                              int pad) {
+    int64_t n = 0;
+    for (int t = 0; t < taps; t++)
+        for (int64_t o = 0; o < out; o++) {
+            const int64_t i = o * stride + (int64_t)t * dil - pad;
+            n += i >= 0 && i < extent;
+        }
+    return n;
+}
+
+// the algorithmic multiply-accumulates: only the taps that read inside the input
+static double conv_macs(const iq_conv_desc* d) {
+    const int64_t P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    const int64_t Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    return (double)d->n * d->k * (double)(d->c / d->groups) *
+           (double)inbounds_pairs(d->h, P, d->r, d->stride_h, d->dil_h, d->pad_h) *
+           (double)inbounds_pairs(d->w, Q, d->s, d->stride_w, d->dil_w, d->pad_w);
 }
 
 // ------------------------------------------------------------------ kernel timing
@@ -477,17 +500,20 @@ static double conv_macs(const iq_conv_desc* d) {
 namespace iq {
 namespace {
 
-constexpr int kKtCap = 4096;
+constexpr int kKtCap = 8192;
 
 struct KtState {
     bool on = false;
     int n = 0;
     int op = 0;
     double pending_macs = 0.0;      // the current call's MACs, given to its first launch
+    double pending_dense = 0.0;
     cudaEvent_t ev[2 * kKtCap] = {};
     int kernel[kKtCap] = {};
     int opv[kKtCap] = {};
     double macs[kKtCap] = {};
+    double dense[kKtCap] = {};
+    double bytes[kKtCap] = {};
 };
 
 KtState& kt() {
@@ -495,12 +521,27 @@ KtState& kt() {
     return *s;
 }
 
+void kt_record(cudaStream_t st, int kernel, double macs, double dense, double bytes, int op) {
+    KtState& k = kt();
+    if (!k.on || k.n >= kKtCap || !k.ev[2 * k.n]) return;
+    cudaEvent_t& e = k.ev[2 * k.n + 1];
+    if (!e && cudaEventCreate(&e) != cudaSuccess) { e = nullptr; return; }
+    cudaEventRecord(e, st);
+    k.kernel[k.n] = kernel;
+    k.opv[k.n] = op;
+    k.macs[k.n] = macs;
+    k.dense[k.n] = dense;
+    k.bytes[k.n] = bytes;
+    k.n++;
+}
+
 }  // namespace
 
-void kt_set_op(int op, double macs) {
+void kt_set_op(int op, double macs, double dense) {
     KtState& k = kt();
     k.op = op;
     k.pending_macs = macs;
+    k.pending_dense = dense;
 }
 
 void kt_pre(cudaStream_t st) {
@@ -513,15 +554,14 @@ void kt_pre(cudaStream_t st) {
 
 void kt_post(cudaStream_t st, int kernel) {
     KtState& k = kt();
-    if (!k.on || k.n >= kKtCap || !k.ev[2 * k.n]) return;
-    cudaEvent_t& e = k.ev[2 * k.n + 1];
-    if (!e && cudaEventCreate(&e) != cudaSuccess) { e = nullptr; return; }
-    cudaEventRecord(e, st);
-    k.kernel[k.n] = kernel;
-    k.opv[k.n] = k.op;
-    k.macs[k.n] = k.pending_macs;
+    if (!k.on) return;
+    kt_record(st, kernel, k.pending_macs, k.pending_dense, 0.0, k.op);
     k.pending_macs = 0.0;
-    k.n++;
+    k.pending_dense = 0.0;
+}
+
+void kt_post_bytes(cudaStream_t st, int kernel, double bytes) {
+    kt_record(st, kernel, 0.0, 0.0, bytes, 0);
 }
 
 }  // namespace iq
@@ -531,6 +571,7 @@ extern "C" iq_status iq_kernel_timing_begin(void) {
     k.on = true;
     k.n = 0;
     k.pending_macs = 0.0;
+    k.pending_dense = 0.0;
     return IQ_OK;
 }
 
@@ -557,11 +598,15 @@ extern "C" iq_status iq_kernel_timing_end(iq_kernel_time* out, int32_t capacity,
             out[j].pad = 0;
             out[j].ms = 0.0;
             out[j].macs = 0.0;
+            out[j].dense_macs = 0.0;
+            out[j].bytes = 0.0;
             nout++;
         }
         out[j].launches++;
         out[j].ms += ms;
         out[j].macs += k.macs[i];
+        out[j].dense_macs += k.dense[i];
+        out[j].bytes += k.bytes[i];
     }
     k.n = 0;
     *n_out = nout;
@@ -578,7 +623,7 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     const int64_t nx = (int64_t)d->n * d->h * d->w * d->c;
     if (x_f16 && (nx % 16 || (((uintptr_t)x | (uintptr_t)x_f16) & 15))) return IQ_ERR_INVALID_ARG;
     if (crs_overflow(d)) return IQ_ERR_OVERFLOW_RISK;
-    kt_set_op(1, conv_macs(d));
+    kt_set_op(1, conv_macs(d), conv_macs_dense(d));
     iq_bn_bits b = bn_bits_or_default(bits);
     if (use_bn) {
         if (!gamma || !beta || !bn_bits_valid(b)) return IQ_ERR_INVALID_ARG;
@@ -613,9 +658,11 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     if (r != IQ_OK) return r;
     if (!done) {
         dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
+        kt_pre(st);
         k_conv_simt<OP_FWD, false><<<grid, 256, 0, st>>>(cp, x, w, acc, nullptr, L.st.s1, L.st.hi,
                                                   L.st.lo, nullptr);
         IQ_LAUNCH_CHECK();
+        kt_post(st, IQ_KERNEL_CONV_SIMT);
     }
     if (use_bn)
         return bn_fwd_after_stats(acc, cp.M, cp.K, L.s_acc, gamma, beta, b, L.st, xhat, a, s_a,
@@ -641,7 +688,7 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     size_t need = 0;
     iq_conv_dgrad_workspace_size(d, &need);
     if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
-    kt_set_op(2, conv_macs(d));
+    kt_set_op(2, conv_macs(d), conv_macs_dense(d));
     cudaStream_t st = (cudaStream_t)stream;
     ConvP cp = make_params(d);
     WsCursor cur(ws, ws_bytes);
@@ -697,15 +744,19 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     cp.kin = (int)roundup(cp.Kg, BK);
     dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
     if (wide) {
+        kt_pre(st);
         k_conv_simt<OP_DGRAD, true><<<grid, 256, 0, st>>>(cp, e, wt, nullptr, (long long*)accw,
                                                           nullptr, nullptr, nullptr, cell);
         IQ_LAUNCH_CHECK();
+        kt_post(st, IQ_KERNEL_CONV_SIMT);
         return requant_apply(accw, IQ_I64, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
                              s_dx, rq, st);
     }
+    kt_pre(st);
     k_conv_simt<OP_DGRAD, false><<<grid, 256, 0, st>>>(cp, e, wt, acc, nullptr, nullptr, nullptr,
                                                        nullptr, cell);
     IQ_LAUNCH_CHECK();
+    kt_post(st, IQ_KERNEL_CONV_SIMT);
     return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8, s_dx, rq,
                          st);
 }
@@ -721,7 +772,7 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
     size_t need = 0;
     iq_conv_wgrad_workspace_size(d, &need);
     if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
-    kt_set_op(3, conv_macs(d));
+    kt_set_op(3, conv_macs(d), conv_macs_dense(d));
     ConvP cp = make_params(d);
     // |G| < npq 127^2 must stay below 2^40 for the requantizer
     if ((double)cp.npq * 16129.0 >= 1099511627776.0) return IQ_ERR_OVERFLOW_RISK;
@@ -770,9 +821,11 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
     cp.nsplit = (int)((cp.npq + cp.chunk - 1) / cp.chunk);
     dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN),
               (unsigned)(cp.G * cp.nsplit));
+    kt_pre(st);
     k_conv_simt<OP_WGRAD, false><<<grid, 256, 0, st>>>(cp, e, x, nullptr, (long long*)G, nullptr,
                                                        nullptr, nullptr, nullptr);
     IQ_LAUNCH_CHECK();
+    kt_post(st, IQ_KERNEL_CONV_SIMT);
     return requant_int(G, IQ_I64, gn, s_in, 8, gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2,
                        seed, layer, step, 0, g, IQ_I8, s_g, rq, st);
 }

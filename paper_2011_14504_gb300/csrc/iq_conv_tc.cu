@@ -2143,9 +2143,11 @@ iq_status launch_p(const CUtensorMap& map, const TcP& p, int nsplit, const int8_
     g.ns = nsplit;
     g.total = g.mt * g.nt * g.ns;
     const int grid = g.total < num_sms() ? g.total : num_sms();
+    kt_pre(st);
     k_conv_tcp<BN><<<grid, THREADS_P, Cfg<BN>::SMEM, st>>>(map, p, g, xa, xb, out32, out64, s1, hi,
                                                           lo, err);
     IQ_LAUNCH_CHECK();
+    kt_post(st, IQ_KERNEL_CONV_GATHER);
     return IQ_OK;
 }
 
@@ -2161,9 +2163,11 @@ iq_status launch_q(const CUtensorMap& map, const TcP& p, const int8_t* xa, int32
     g.ns = 1;
     g.total = g.mt * g.nt;
     const int grid = g.total < num_sms() ? g.total : num_sms();
+    kt_pre(st);
     k_conv_tcq<BN><<<grid, THREADS_Q, CfgQ<BN>::SMEM, st>>>(map, p, g, xa, out32, out64, s1, hi, lo,
                                                            err);
     IQ_LAUNCH_CHECK();
+    kt_post(st, IQ_KERNEL_CONV_CPASYNC);
     return IQ_OK;
 }
 
@@ -2304,7 +2308,9 @@ iq_status try_launch_t(const CUtensorMap& wmap, const TcP& p, const int8_t* x, _
     if (!xf || !tma16_ok(p, &t)) return IQ_OK;
     if (convert) {
         const int64_t n16 = (int64_t)p.N * p.H * p.W * p.cstride / 16;
+        kt_pre(st);
         k_codes_to_f16<<<grid_for(n16), kThreads, 0, st>>>(x, xf, n16);
+        kt_post_bytes(st, IQ_KERNEL_CODES_TO_F16, 48.0 * (double)(n16));
         IQ_LAUNCH_CHECK();
     }
     CUtensorMap amap, omap;
@@ -2348,7 +2354,9 @@ iq_status try_launch_c(const __half* wf, int rows, const TcP& p, const int8_t* x
     if (encode_acts16(xf, p.N, p.H, p.W, p.cstride, t, p.sh, p.sw, &amap) != IQ_OK) return IQ_OK;
     if (convert) {
         const int64_t n16 = (int64_t)p.N * p.H * p.W * p.cstride / 16;
+        kt_pre(st);
         k_codes_to_f16<<<grid_for(n16), kThreads, 0, st>>>(x, xf, n16);
+        kt_post_bytes(st, IQ_KERNEL_CODES_TO_F16, 48.0 * (double)(n16));
         IQ_LAUNCH_CHECK();
     }
     IQ_CUDA_CHECK(cudaFuncSetAttribute(k_conv_tcc, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -2401,7 +2409,9 @@ constexpr int IM2COL_MAX_K = 512;
 iq_status codes_to_f16(const int8_t* x, __half* xf, int64_t n, cudaStream_t st) {
     if (n % 16 || (((uintptr_t)x | (uintptr_t)xf) & 15)) return IQ_ERR_INVALID_ARG;
     if (n == 0) return IQ_OK;
+    kt_pre(st);
     k_codes_to_f16<<<grid_for(n / 16), kThreads, 0, st>>>(x, xf, n / 16);
+    kt_post_bytes(st, IQ_KERNEL_CODES_TO_F16, 48.0 * (double)(n / 16));
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }
@@ -2852,7 +2862,9 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
         p.out = OUT_PART32;
         if (!use_ef) {
             if (Kp == p.K && ne % 16 == 0) {
+                kt_pre(st);
                 k_codes_to_f16<<<grid_for(ne / 16), kThreads, 0, st>>>(e, ef, ne / 16);
+                kt_post_bytes(st, IQ_KERNEL_CODES_TO_F16, 48.0 * (double)(ne / 16));
             } else {
                 k_codes_to_f16_pad<<<grid_for(p.npq * (Kp / 8)), kThreads, 0, st>>>(e, ef, p.npq,
                                                                                   p.K, Kp);
@@ -2863,7 +2875,9 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
             launch_im2col(x, pc, xf, st);
             IQ_LAUNCH_CHECK();
         } else if (!use_xf) {
+            kt_pre(st);
             k_codes_to_f16<<<grid_for(nx / 16), kThreads, 0, st>>>(x, xf, nx / 16);
+            kt_post_bytes(st, IQ_KERNEL_CODES_TO_F16, 48.0 * (double)(nx / 16));
             IQ_LAUNCH_CHECK();
         }
         iq_status r = IQ_OK;

@@ -93,9 +93,12 @@ inline bool bn_bits_valid(const iq_bn_bits& b) {
 
 
 // kernel timing (iq_kernel_timing_begin / _end): the conv entry points name the operation
-// and its algorithmic MACs, the launchers bracket their main kernel with kt_pre / kt_post
-void kt_set_op(int op, double macs);
+// and its algorithmic (in-bounds) and dense MACs, the launchers bracket their main kernel
+// with kt_pre / kt_post; a bandwidth kernel is bracketed with kt_pre / kt_post_bytes and
+// tagged with the bytes its pass must read and write
+void kt_set_op(int op, double macs, double dense);
 void kt_pre(cudaStream_t st);
 void kt_post(cudaStream_t st, int kernel);
+void kt_post_bytes(cudaStream_t st, int kernel, double bytes);
 
 }  // namespace iq

@@ -639,6 +639,11 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
                ((uintptr_t)t.codes & (t.is16 ? 7 : 3)) == 0;
         any_bcast = any_bcast || t.bcast;
     }
+    // the bytes each pass must move: every operand's codes once (+ the output codes)
+    double in_b = 0.0;
+    for (int i = 0; i < n_terms; i++)
+        in_b += (double)(T.t[i].bcast ? n : n * hw) * T.t[i].c * (T.t[i].is16 ? 2.0 : 1.0);
+    const double out_b = (double)total;
     const UDiv dhw = make_udiv((uint64_t)hw);
     // at most two operands cover any 4-channel group: sums of up to two operands, and
     // concatenations whose ranges overlap at most pairwise (checked per group on the host)
@@ -664,14 +669,18 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
         want = (want + unit - 1) / unit * unit;
         if (want < unit) want = unit;
         const int g = (int)want;
+        kt_pre(st);
         k_comb4r<0><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
                                             dhw, any_bcast);
         IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_COMBINE_MAX, in_b);
         k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
         IQ_LAUNCH_CHECK();
+        kt_pre(st);
         k_comb4r<1><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
                                             dhw, any_bcast);
         IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b);
         return IQ_OK;
     }
     // sums whose operands all cover every channel, F rows of all of them in shared memory
@@ -689,40 +698,52 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
         if (want < unit) want = unit;
         const int g = (int)want;
         const size_t sm = (size_t)n_terms * kThreads * 4 * 8;   // <= 48 KB
+        kt_pre(st);
         k_combNs<0><<<g, kThreads, sm, st>>>(T, npix, cgs, relu != 0, F, B, hdr, out, dhw,
                                              any_bcast);
         IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_COMBINE_MAX, in_b);
         k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
         IQ_LAUNCH_CHECK();
+        kt_pre(st);
         k_combNs<1><<<g, kThreads, sm, st>>>(T, npix, cgs, relu != 0, F, B, hdr, out, dhw,
                                              any_bcast);
         IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b);
         return IQ_OK;
     }
     if (vec) {
         const int64_t nvec = total / 8;
         const int g = grid_for(nvec, kThreads, 152 * 8);
         const UDiv dcg = make_udiv((uint64_t)(c_out / 8));
+        kt_pre(st);
         k_comb8<0><<<g, kThreads, 0, st>>>(T, concat != 0, nvec, c_out / 8, relu != 0, F, B, hdr,
                                            out, dcg, dhw, any_bcast);
         IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_COMBINE_MAX, in_b);
         k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
         IQ_LAUNCH_CHECK();
+        kt_pre(st);
         k_comb8<1><<<g, kThreads, 0, st>>>(T, concat != 0, nvec, c_out / 8, relu != 0, F, B, hdr,
                                            out, dcg, dhw, any_bcast);
         IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b);
         return IQ_OK;
     }
     const int g = grid_for(total, kThreads, 152 * 8);
     const UDiv dc = make_udiv((uint64_t)c_out);
+    kt_pre(st);
     k_comb<0><<<g, kThreads, 0, st>>>(T, concat != 0, n, hw, c_out, relu != 0, F, B, hdr, out,
                                       dc, dhw);
     IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, IQ_KERNEL_COMBINE_MAX, in_b);
     k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
     IQ_LAUNCH_CHECK();
+    kt_pre(st);
     k_comb<1><<<g, kThreads, 0, st>>>(T, concat != 0, n, hw, c_out, relu != 0, F, B, hdr, out,
                                       dc, dhw);
     IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b);
     return IQ_OK;
 }
 

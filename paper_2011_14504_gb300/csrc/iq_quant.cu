@@ -290,6 +290,9 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
         IQ_LAUNCH_CHECK();
     }
     if (n == 0) return IQ_OK;
+    const double isz = in_dtype == IQ_I64 ? 8.0 : 4.0;
+    const double osz = out_dtype == IQ_I8 ? 1.0 : (out_dtype == IQ_I16 ? 2.0 : 4.0);
+    kt_pre(st);
     if (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) {
         if (in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
             (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0)
@@ -313,6 +316,9 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
                                                        step, tag, ep, out, out_dtype);
     }
     IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) ? IQ_KERNEL_SQ_CODES
+                                                                       : IQ_KERNEL_RQ_CODES,
+                  (double)n * (isz + osz));
     return IQ_OK;
 }
 
@@ -324,11 +330,13 @@ iq_status requant_int(const void* q, int in_dtype, int64_t n, const double* s_in
     IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, sizeof(unsigned long long), st));
     if (n > 0) {
         int g = grid_for(n);
+        kt_pre(st);
         if (in_dtype == IQ_I32)
             k_absmax_int<int32_t><<<g, kThreads, 0, st>>>((const int32_t*)q, n, relu, cell);
         else
             k_absmax_int<int64_t><<<g, kThreads, 0, st>>>((const int64_t*)q, n, relu, cell);
         IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_ABSMAX, (double)n * (in_dtype == IQ_I64 ? 8.0 : 4.0));
     }
     return requant_apply(q, in_dtype, n, s_in, k, mode, seed, layer, step, tag, out, out_dtype,
                          s_out, ws, st);

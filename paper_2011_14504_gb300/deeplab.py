@@ -24,6 +24,7 @@ import torch
 
 from . import iq
 from . import synthetic as S
+from .work import conv_macs
 
 K_E2 = 16
 
@@ -46,7 +47,11 @@ class Layer:
         iq.iq_weight_requant(self.master, self.wq)
         self.a = torch.empty(self.out_shape, dtype=torch.int8, device=dev)
         self.s_a = net.scal()
-        self.macs = n * p * q * spec.cout * spec.r * spec.r * (3 if spec.cin == 4 else spec.cin)
+        # in-bounds and dense multiply-accumulates of one pass (the stem's fourth input
+        # channel is the zero RGB padding: no work)
+        self.macs, self.macs_dense = conv_macs(n, h, w, 3 if spec.cin == 4 else spec.cin,
+                                               spec.cout, spec.r, spec.stride, spec.pad,
+                                               spec.dil)
         if spec.bn:
             self.gm = torch.from_numpy(gm).to(dev)
             self.bm = torch.from_numpy(bm).to(dev)
@@ -266,12 +271,24 @@ class DeepLabV3R50:
 
     @property
     def macs_forward(self) -> int:
+        """In-bounds multiply-accumulates of the inference pass."""
         return sum(L.macs for L in self.layers.values())
 
     @property
     def macs_step(self) -> int:
+        """In-bounds multiply-accumulates of a training step: forward, data gradient (not for
+        the stem) and weight gradient of every conv."""
         f = self.macs_forward
         return f + (f - self.stem.macs) + f
+
+    @property
+    def macs_forward_dense(self) -> int:
+        return sum(L.macs_dense for L in self.layers.values())
+
+    @property
+    def macs_step_dense(self) -> int:
+        f = self.macs_forward_dense
+        return f + (f - self.stem.macs_dense) + f
 
     def forward(self, img_u8: torch.Tensor, stream=None):
         ws = self.ws

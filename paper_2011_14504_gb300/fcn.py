@@ -22,6 +22,7 @@ import torch
 
 from . import iq
 from . import synthetic as S
+from .work import conv_macs, transposed_macs
 
 UP_R, UP_STRIDE, UP_PAD = 64, 32, 16
 
@@ -50,7 +51,8 @@ class Conv:
     ex: torch.Tensor = None       # error of the input (dgrad output)
     s_ex: torch.Tensor = None
     x16: torch.Tensor = None      # fp16 copy of x written by the forward, read by the wgrad
-    macs: int = 0
+    macs: int = 0                 # in-bounds multiply-accumulates of one pass
+    macs_dense: int = 0           # every tap, the zero padding included
 
 
 @dataclass
@@ -115,7 +117,10 @@ class FcnVgg16:
             self.up_s_g = scal()
             self.e_score = torch.empty_like(self.score)
             self.s_e_score = scal()
-        self.up_macs = n * h * w * classes * 4   # <= 2 x 2 taps per output pixel
+        # the decoder: (in-bounds, dense) multiply-accumulates, <= 2 x 2 taps per output pixel
+        self.up_macs, self.up_macs_dense = transposed_macs(n, self.score_hw[0],
+                                                           self.score_hw[1], classes, UP_R,
+                                                           UP_STRIDE, UP_PAD)
         self._alloc_backward()
         self.ws = torch.empty(self._ws_bytes(), dtype=torch.uint8, device=dev)
 
@@ -139,7 +144,8 @@ class FcnVgg16:
         L.x, L.s_x = x, s_x
         L.a = torch.empty((n, hh, ww, cout), dtype=torch.int8, device=dev)
         L.s_a = torch.zeros(1, dtype=torch.float64, device=dev)
-        L.macs = n * hh * ww * cout * r * r * (3 if cin == 4 else cin)
+        # the first layer's fourth input channel is the zero RGB padding: no work
+        L.macs, L.macs_dense = conv_macs(n, hh, ww, 3 if cin == 4 else cin, cout, r, 1, pad)
         self.layers.append(L)
         self.convs.append(L)
         return L.a, L.s_a
@@ -187,14 +193,27 @@ class FcnVgg16:
 
     @property
     def macs_forward(self) -> int:
+        """In-bounds multiply-accumulates of the inference pass."""
         return sum(L.macs for L in self.convs) + self.up_macs
 
     @property
     def macs_step(self) -> int:
-        # forward, data gradient (not for the first layer) and weight gradient of every conv
-        f = sum(L.macs for L in self.convs)
-        dg = sum(L.macs for L in self.convs if L.layer_id > 0)
-        return f + dg + f + 3 * self.up_macs
+        """In-bounds multiply-accumulates of a training step: forward, data gradient (not for
+        the first layer) and weight gradient of every conv, the decoder included."""
+        return self._step(lambda L: L.macs, self.up_macs)
+
+    @property
+    def macs_forward_dense(self) -> int:
+        return sum(L.macs_dense for L in self.convs) + self.up_macs_dense
+
+    @property
+    def macs_step_dense(self) -> int:
+        return self._step(lambda L: L.macs_dense, self.up_macs_dense)
+
+    def _step(self, get, up) -> int:
+        f = sum(get(L) for L in self.convs)
+        dg = sum(get(L) for L in self.convs if L.layer_id > 0)
+        return f + dg + f + 3 * up
 
     def forward(self, img_u8: torch.Tensor, stream=None):
         ws = self.ws

@@ -34,8 +34,17 @@ EXPORTS = [
     "iq_kernel_timing_begin", "iq_kernel_timing_end",
 ]
 IQ_KERNEL_CONV_PIXEL_MAJOR, IQ_KERNEL_CONV_CHANNEL_MAJOR, IQ_KERNEL_CONV_WGRAD = 1, 2, 3
+IQ_KERNEL_CONV_CPASYNC, IQ_KERNEL_CONV_GATHER, IQ_KERNEL_CONV_SIMT = 4, 5, 6
+(IQ_KERNEL_BN_DEV, IQ_KERNEL_BN_REQUANT, IQ_KERNEL_BNB_PASS1, IQ_KERNEL_BNB_PASS2,
+ IQ_KERNEL_BNB_PASS3, IQ_KERNEL_COMBINE_MAX, IQ_KERNEL_COMBINE_CODES, IQ_KERNEL_SQ_CODES,
+ IQ_KERNEL_CODES_TO_F16, IQ_KERNEL_ABSMAX, IQ_KERNEL_RQ_CODES) = range(10, 21)
 KERNEL_NAMES = {1: "k_conv_tct (forward / data gradient)", 2: "k_conv_tcc (channel-major)",
-                3: "k_conv_tct (weight gradient)"}
+                3: "k_conv_tct (weight gradient)", 4: "k_conv_tcq", 5: "k_conv_tcp",
+                6: "k_conv_simt", 10: "k_bn_dev", 11: "k_bn_requant", 12: "k_bnb_pass1",
+                13: "k_bnb_pass2", 14: "k_bnb_pass3", 15: "iq_combine max pass",
+                16: "iq_combine codes pass", 17: "SQ codes (k_sq_i32_i8x4 / k_sq_int)",
+                18: "k_codes_to_f16", 19: "k_absmax_int", 20: "k_rq_int"}
+CONV_KERNELS = (1, 2, 3, 4, 5, 6)
 
 
 class IqError(RuntimeError):
@@ -65,7 +74,8 @@ class Term(C.Structure):
 class KernelTime(C.Structure):
     """iq_kernel_time: summed event time and MACs of one (kernel, operation) pair."""
     _fields_ = [("kernel", C.c_int32), ("op", C.c_int32), ("launches", C.c_int32),
-                ("pad", C.c_int32), ("ms", C.c_double), ("macs", C.c_double)]
+                ("pad", C.c_int32), ("ms", C.c_double), ("macs", C.c_double),
+                ("dense_macs", C.c_double), ("bytes", C.c_double)]
 
 
 IQ_MAX_TERMS = 8
@@ -162,13 +172,15 @@ def iq_kernel_timing_begin():
     _check("iq_kernel_timing_begin", load().iq_kernel_timing_begin())
 
 
-def iq_kernel_timing_end(capacity=16):
-    """Stop, wait for the events and return [{kernel, op, launches, ms, macs}] per (kernel, op)."""
+def iq_kernel_timing_end(capacity=64):
+    """Stop, wait for the events and return [{kernel, op, launches, ms, macs, dense_macs,
+    bytes}] per (kernel, op)."""
     out = (KernelTime * capacity)()
     n = _I32(0)
     _check("iq_kernel_timing_end", load().iq_kernel_timing_end(out, capacity, C.byref(n)))
     return [{"kernel": out[i].kernel, "op": out[i].op, "launches": out[i].launches,
-             "ms": out[i].ms, "macs": out[i].macs} for i in range(n.value)]
+             "ms": out[i].ms, "macs": out[i].macs, "dense_macs": out[i].dense_macs,
+             "bytes": out[i].bytes} for i in range(n.value)]
 
 
 def iq_device_status(stream=None) -> int:
@@ -522,12 +534,11 @@ def iq_ce_grad(z, s_z, labels, E, s_e, n_valid=None, ignore=255, ws=None, stream
 
 def iq_bn_update(gamma_master, beta_master, gamma, beta, dgamma, dbeta, s_e, bn_scales, lr_log2,
                  seed, layer, step, k_u=24, bits=None, ws=None, stream=None):
+    """ws is accepted for compatibility and ignored: the update needs no scratch."""
     c = gamma.numel()
-    if ws is None:
-        ws = _ws(4096 + 2 * c + 256, gamma.device)
     _check("iq_bn_update", load().iq_bn_update(_p(gamma_master), _p(beta_master), _p(gamma),
                                                _p(beta), _p(dgamma), _p(dbeta), _p(s_e),
                                                _p(bn_scales), c,
                                                C.byref(bits) if bits is not None else None,
-                                               lr_log2, k_u, seed, layer, step, _p(ws),
-                                               ws.numel(), _stream(stream)))
+                                               lr_log2, k_u, seed, layer, step, None, 0,
+                                               _stream(stream)))

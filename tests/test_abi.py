@@ -64,8 +64,8 @@ def test_kernel_timing_host_side(lib):
     assert lib.iq_kernel_timing_end(None, 4, C.byref(n)) == iq.IQ_ERR_INVALID_ARG
     out = (iq.KernelTime * 2)()
     assert lib.iq_kernel_timing_end(out, 2, None) == iq.IQ_ERR_INVALID_ARG
-    # the struct layout the header declares: 4 int32 then 2 doubles
-    assert C.sizeof(iq.KernelTime) == 32
+    # the struct layout the header declares: 4 int32 then 4 doubles
+    assert C.sizeof(iq.KernelTime) == 48
 
 
 def test_invalid_arguments_rejected_before_launch(lib):
@@ -132,5 +132,6 @@ def test_glue_arguments_rejected_before_launch(lib):
     assert lib.iq_ce_grad(16, 16, 16, 10, 21, 255, 16, 16, None, 16, 8, None) == iq.IQ_ERR_WORKSPACE
     assert lib.iq_bn_update(16, 16, 16, 16, 16, None, 16, 16, 8, None, 10, 24, 0, 0, 0, 16, 1 << 16,
                             None) == iq.IQ_ERR_INVALID_ARG
-    assert lib.iq_bn_update(16, 16, 16, 16, 16, 16, 16, 16, 8, None, 10, 24, 0, 0, 0, 16, 100,
-                            None) == iq.IQ_ERR_WORKSPACE
+    # more channels than the one-launch update takes (its workspace is reserved: NULL is fine)
+    assert lib.iq_bn_update(16, 16, 16, 16, 16, 16, 16, 16, 4097, None, 10, 24, 0, 0, 0, None, 0,
+                            None) == iq.IQ_ERR_UNSUPPORTED

@@ -630,12 +630,20 @@ def test_kernel_timing_brackets_the_conv_kernels():
     iq.iq_conv_dgrad(d, e, dscal(0.01), wq, dx, dscal(0.0))
     iq.iq_conv_wgrad(d, e, dscal(0.01), x, dscal(0.01), gw, dscal(0.0), gq_mode=2)
     rows = iq.iq_kernel_timing_end()
-    macs = float(n * h * h * k * 9 * c)
-    ops = {r["op"]: r for r in rows}
-    assert sorted(ops) == [1, 2, 3]
-    for r in rows:
-        assert r["launches"] == 1 and r["macs"] == macs and r["ms"] > 0
+    dense = float(n * h * h * k * 9 * c)
+    inb = float(n * k * c * (3 * h - 2) ** 2)      # taps that read inside the 32 x 32 input
+    conv = [r for r in rows if r["op"] != 0]
+    ops = {r["op"]: r for r in conv}
+    assert sorted(ops) == [1, 2, 3] and len(conv) == 3
+    for r in conv:
+        assert r["launches"] == 1 and r["macs"] == inb and r["dense_macs"] == dense
+        assert r["ms"] > 0 and r["bytes"] == 0
     assert ops[1]["kernel"] in (iq.IQ_KERNEL_CONV_PIXEL_MAJOR, iq.IQ_KERNEL_CONV_CHANNEL_MAJOR)
     assert ops[2]["kernel"] in (iq.IQ_KERNEL_CONV_PIXEL_MAJOR, iq.IQ_KERNEL_CONV_CHANNEL_MAJOR)
     assert ops[3]["kernel"] == iq.IQ_KERNEL_CONV_WGRAD
+    # the bandwidth passes around them: the SQ codes of the forward and data-gradient sums,
+    # each tagged with its int32 read and int8 write
+    bw = {r["kernel"]: r for r in rows if r["op"] == 0}
+    sq = bw[iq.IQ_KERNEL_SQ_CODES]
+    assert sq["launches"] == 2 and sq["bytes"] == 5.0 * n * h * h * (k + c)
     assert iq.iq_kernel_timing_end() == []      # stopped: nothing recorded since

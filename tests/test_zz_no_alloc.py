@@ -31,17 +31,36 @@ def _run(fn, acc, s_acc, gam, bet, **kw):
     return [t.cpu().numpy() for t in (X, A, codes, scal, fixed, s_a)]
 
 
+def _case(g, m, c, spread, call):
+    acc = torch.from_numpy((g.standard_normal((m, c)) * spread +
+                            g.integers(-2000, 2001, c)).astype(np.int32)).to(DEV)
+    gam, bet = (torch.from_numpy(v).to(DEV) for v in S.bn_gamma_beta_codes(g, c))
+    s_acc = torch.tensor([2.0 ** -14 * (call + 1.5)], dtype=torch.float64, device=DEV)
+    return acc, s_acc, gam, bet
+
+
 def test_noalloc_matches_workspace_version_twice():
+    """A larger channel count, then a smaller one: the second call reuses the bytes the
+    first one left in the shared array."""
     g = S.rng(2024)
-    for call, (m, c, spread) in enumerate([(4096, 256, 3000.0), (777, 4096, 90000.0)]):
-        acc = torch.from_numpy((g.standard_normal((m, c)) * spread +
-                                g.integers(-2000, 2001, c)).astype(np.int32)).to(DEV)
-        gam, bet = (torch.from_numpy(v).to(DEV) for v in S.bn_gamma_beta_codes(g, c))
-        s_acc = torch.tensor([2.0 ** -14 * (call + 1.5)], dtype=torch.float64, device=DEV)
+    for call, (m, c, spread) in enumerate([(777, 4096, 90000.0), (4096, 256, 3000.0)]):
+        acc, s_acc, gam, bet = _case(g, m, c, spread, call)
         want = _run(iq.iq_bn_int_fwd, acc, s_acc, gam, bet)
         got = _run(iq.iq_bn_int_fwd_noalloc, acc, s_acc, gam, bet)
         for w, h in zip(want, got):
             assert np.array_equal(w, h), call
+
+
+def test_noalloc_identical_calls_in_a_row():
+    """The same call twice: a statistic that is not reset between calls (a sum that
+    doubles, an extreme that sticks) would change the second result."""
+    g = S.rng(7)
+    acc, s_acc, gam, bet = _case(g, 3000, 512, 20000.0, 0)
+    want = _run(iq.iq_bn_int_fwd, acc, s_acc, gam, bet)
+    for rep in range(2):
+        got = _run(iq.iq_bn_int_fwd_noalloc, acc, s_acc, gam, bet)
+        for w, h in zip(want, got):
+            assert np.array_equal(w, h), rep
 
 
 def test_noalloc_rejects_too_many_channels():
