@@ -94,6 +94,11 @@ def _declare(L):
     L.or_conv_out_size.argtypes = [C.POINTER(ConvDesc)]
     for f in ("or_conv_fwd", "or_conv_dgrad", "or_conv_wgrad"):
         getattr(L, f).argtypes = [C.POINTER(ConvDesc), _P, _P, _P]
+        getattr(L, f + "_at").argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _I64, _P]
+    L.or_sq_at.argtypes = [_P, _I64, _I64, _D, _I32, _I32, _P]
+    L.or_sq_at.restype = _D
+    L.or_rq_at.argtypes = [_P, _P, _I64, _I64, _D, _I32, _I32, _U64, _U64, _U64, _U64, _P]
+    L.or_rq_at.restype = _D
     L.or_bn_fwd.argtypes = [_I64, _I32, _P, _D, _P, _P, C.POINTER(BnBits), _P, _P, _P, _P,
                             _P, _P, _P, _P, C.POINTER(BnOut)]
     L.or_bn_fwd.restype = _I32
@@ -164,6 +169,28 @@ def sq_int(q, s: float, k: int, relu: bool = False):
     q = _c(q, np.int64)
     out = np.empty(q.shape, np.int32)
     so = lib().or_sq_int64(_ptr(q), q.size, float(s), k, int(relu), _ptr(out))
+    return out, so
+
+
+def sq_at(q, M: int, s: float, k: int, relu: bool = False):
+    """Eq. (ScaleQ) codes of selected elements q of a tensor whose max |q| (after ReLU when
+    relu) is M, and the output scale: the values sq_int gives at those elements."""
+    q = _c(q, np.int64)
+    out = np.empty(q.shape, np.int32)
+    so = lib().or_sq_at(_ptr(q), q.size, int(M), float(s), k, int(relu), _ptr(out))
+    return out, so
+
+
+def rq_at(q, idx, M: int, s: float, k: int, gq_mode: int, seed: int, layer: int, step: int,
+          tag: int = 0):
+    """Eqs. (SQ),(SR),(GQ1)/(GQ2) codes of selected elements q (flat indices idx) of a tensor
+    whose max |q| is M, and the output scale: the values rq_int gives at those elements."""
+    q = _c(q, np.int64)
+    idx = _c(idx, np.int64)
+    assert q.shape == idx.shape
+    out = np.empty(q.shape, np.int32)
+    so = lib().or_rq_at(_ptr(q), _ptr(idx), q.size, int(M), float(s), k, gq_mode, seed, layer,
+                        step, tag, _ptr(out))
     return out, so
 
 
@@ -269,6 +296,31 @@ def conv_wgrad(cv: Conv, e, x) -> np.ndarray:
     out = np.empty((cv.k, cv.r, cv.s, cv.c // cv.groups), np.int64)
     lib().or_conv_wgrad(C.byref(d), _ptr(e), _ptr(x), _ptr(out))
     return out
+
+
+def _at(fname, cv: Conv, a, b, idx):
+    d = cv.desc()
+    a = _c(a, np.int8)
+    b = _c(b, np.int8)
+    idx = _c(idx, np.int64).ravel()
+    out = np.empty(idx.shape, np.int64)
+    getattr(lib(), fname)(C.byref(d), _ptr(a), _ptr(b), _ptr(idx), idx.size, _ptr(out))
+    return out
+
+
+def conv_fwd_at(cv: Conv, x, w, idx) -> np.ndarray:
+    """conv_fwd at the flat NPQK output indices idx only (int64 sums), one by one."""
+    return _at("or_conv_fwd_at", cv, x, w, idx)
+
+
+def conv_dgrad_at(cv: Conv, e, w, idx) -> np.ndarray:
+    """conv_dgrad at the flat NHWC input indices idx only."""
+    return _at("or_conv_dgrad_at", cv, e, w, idx)
+
+
+def conv_wgrad_at(cv: Conv, e, x, idx) -> np.ndarray:
+    """conv_wgrad at the flat KRSC weight indices idx only."""
+    return _at("or_conv_wgrad_at", cv, e, x, idx)
 
 
 # ---------------------------------------------------------------- L1BN

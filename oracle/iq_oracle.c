@@ -230,6 +230,44 @@ double or_rq_int64(const int64_t* q, int64_t n, double s, int k, int gq_mode,
     return gq_mode == 1 ? ldexp(s * (double)M, 1 - k) : ldexp(1.0, 1 - k);
 }
 
+/* Eq. (ScaleQ) and Eqs. (SQ),(SR) for selected elements of a tensor whose
+ * max |q| (after ReLU for SQ of ReLU) is M: the codes that or_sq_int64 and
+ * or_rq_int64 give at those elements, and the output scale.  idx[j] is the
+ * flat index of element q[j] in its tensor (the stochastic rounding's
+ * counter).  For checking a large tensor at sampled positions. */
+double or_sq_at(const int64_t* q, int64_t m, int64_t M, double s, int k, int relu,
+                int32_t* code) {
+    if (M == 0) {
+        for (int64_t j = 0; j < m; j++) code[j] = 0;
+        return ldexp(s, 1 - k);
+    }
+    for (int64_t j = 0; j < m; j++) {
+        int64_t v = q[j];
+        if (relu && v < 0) v = 0;
+        i128 c = floordiv128(((i128)v << k) + M, (i128)2 * M);
+        code[j] = (int32_t)clamp64((int64_t)c, -qmax(k), qmax(k));
+    }
+    return ldexp(s * (double)M, 1 - k);
+}
+
+double or_rq_at(const int64_t* q, const int64_t* idx, int64_t m, int64_t M, double s,
+                int k, int gq_mode, uint64_t seed, uint64_t layer, uint64_t step,
+                uint64_t tag, int32_t* code) {
+    if (M == 0) {
+        for (int64_t j = 0; j < m; j++) code[j] = 0;
+        return gq_mode == 1 ? ldexp(s, 1 - k) : ldexp(1.0, 1 - k);
+    }
+    for (int64_t j = 0; j < m; j++) {
+        i128 num = (i128)q[j] << (k - 1);
+        i128 f = floordiv128(num, (i128)M);
+        i128 rem = num - f * M;
+        uint32_t u = or_rq_uniform(seed, layer, step, tag, (uint64_t)idx[j]);
+        int up = ((u128)u * (u128)M) < ((u128)rem << 32);
+        code[j] = (int32_t)clamp64((int64_t)(f + up), -qmax(k), qmax(k));
+    }
+    return gq_mode == 1 ? ldexp(s * (double)M, 1 - k) : ldexp(1.0, 1 - k);
+}
+
 /* ------------------------------------------------------------------ */
 /* Sec. 3.2.1: weights                                                 */
 /* ------------------------------------------------------------------ */
@@ -360,6 +398,95 @@ void or_conv_wgrad(const or_conv* d, const int8_t* e, const int8_t* x,
                         }
                     gw[(((int64_t)k * d->r + r) * d->s + s) * cg + c] = sum;
                 }
+    }
+}
+
+/* Selected outputs of the three convolutions, one at a time: out[j] is the
+ * sum that or_conv_fwd / or_conv_dgrad / or_conv_wgrad would store at the
+ * flat output index idx[j] (NPQK, NHWC and KRSC order respectively), written
+ * out from the same definitions.  They let a tensor too large for the full
+ * loops be checked at sampled positions. */
+void or_conv_fwd_at(const or_conv* d, const int8_t* x, const int8_t* wt,
+                    const int64_t* idx, int64_t m, int64_t* out) {
+    const int cg = d->c / d->groups, kg = d->k / d->groups;
+    #pragma omp parallel for schedule(static)
+    for (int64_t j = 0; j < m; j++) {
+        int64_t t = idx[j];
+        int k = (int)(t % d->k); t /= d->k;
+        int q = (int)(t % d->q); t /= d->q;
+        int p = (int)(t % d->p);
+        int n = (int)(t / d->p);
+        int g = k / kg;
+        int64_t sum = 0;
+        for (int r = 0; r < d->r; r++) {
+            int hh = p * d->stride_h + r * d->dil_h - d->pad_h;
+            if (hh < 0 || hh >= d->h) continue;
+            for (int s = 0; s < d->s; s++) {
+                int ww = q * d->stride_w + s * d->dil_w - d->pad_w;
+                if (ww < 0 || ww >= d->w) continue;
+                for (int c = 0; c < cg; c++)
+                    sum += (int64_t)X_AT(n, hh, ww, g * cg + c) * (int64_t)W_AT(k, r, s, c);
+            }
+        }
+        out[j] = sum;
+    }
+}
+
+/* dx[n,h,w,c]: every (p, r) with p*sh + r*dh - ph = h and every (q, s) alike,
+ * over the output channels k of c's group. */
+void or_conv_dgrad_at(const or_conv* d, const int8_t* e, const int8_t* wt,
+                      const int64_t* idx, int64_t m, int64_t* out) {
+    const int cg = d->c / d->groups, kg = d->k / d->groups;
+    #pragma omp parallel for schedule(static)
+    for (int64_t j = 0; j < m; j++) {
+        int64_t t = idx[j];
+        int c = (int)(t % d->c); t /= d->c;
+        int w = (int)(t % d->w); t /= d->w;
+        int h = (int)(t % d->h);
+        int n = (int)(t / d->h);
+        int g = c / cg;
+        int64_t sum = 0;
+        for (int r = 0; r < d->r; r++) {
+            int num_p = h + d->pad_h - r * d->dil_h;
+            if (num_p < 0 || num_p % d->stride_h) continue;
+            int p = num_p / d->stride_h;
+            if (p >= d->p) continue;
+            for (int s = 0; s < d->s; s++) {
+                int num_q = w + d->pad_w - s * d->dil_w;
+                if (num_q < 0 || num_q % d->stride_w) continue;
+                int q = num_q / d->stride_w;
+                if (q >= d->q) continue;
+                for (int k = g * kg; k < (g + 1) * kg; k++)
+                    sum += (int64_t)e[Y_AT(n, p, q, k)] * (int64_t)W_AT(k, r, s, c - g * cg);
+            }
+        }
+        out[j] = sum;
+    }
+}
+
+void or_conv_wgrad_at(const or_conv* d, const int8_t* e, const int8_t* x,
+                      const int64_t* idx, int64_t m, int64_t* out) {
+    const int cg = d->c / d->groups, kg = d->k / d->groups;
+    #pragma omp parallel for schedule(static)
+    for (int64_t j = 0; j < m; j++) {
+        int64_t t = idx[j];
+        int c = (int)(t % cg); t /= cg;
+        int s = (int)(t % d->s); t /= d->s;
+        int r = (int)(t % d->r);
+        int k = (int)(t / d->r);
+        int g = k / kg;
+        int64_t sum = 0;
+        for (int n = 0; n < d->n; n++)
+            for (int p = 0; p < d->p; p++) {
+                int hh = p * d->stride_h + r * d->dil_h - d->pad_h;
+                if (hh < 0 || hh >= d->h) continue;
+                for (int q = 0; q < d->q; q++) {
+                    int ww = q * d->stride_w + s * d->dil_w - d->pad_w;
+                    if (ww < 0 || ww >= d->w) continue;
+                    sum += (int64_t)e[Y_AT(n, p, q, k)] * (int64_t)X_AT(n, hh, ww, g * cg + c);
+                }
+            }
+        out[j] = sum;
     }
 }
 
