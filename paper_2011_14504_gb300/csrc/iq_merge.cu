@@ -33,6 +33,8 @@ struct CombHdr {
     int32_t pad;
     uint64_t M;
     UDiv div;
+    float kq;      // fl(128 / M) (0 when M = 0)
+    float c130;    // 130 / M rounded up
 };
 
 __device__ __forceinline__ double term_a(const TermDev& t, double s, int ch) {
@@ -472,10 +474,288 @@ __global__ void __launch_bounds__(kThreads) k_combNs(Terms T, int64_t npix, int 
     }
 }
 
+// ---------------------------------------------------------------- fp32-decided joins
+//
+// The two passes with a fixed group of CPT channels per thread (as k_comb4r with 4), for up
+// to NC operands covering each group, with each element first evaluated in fp32:
+// zf = fma(F_k, v_k, ...) over the covering operands from fl(sum B), with F_k rounded to
+// fp32.  With u = 2^-24 and, over the thread's channels, S = max |sum B| +
+// sum_k |F_k| vmax_k, every |zf - z| <= (nc + 2) u S (the B sum and each F converted with a
+// relative error of at most 2u, one rounding per fma, every partial sum below S); the
+// kernel takes E = (nc + 3) u S, evaluated in fp32 rounded upward, so it bounds the exact
+// value.  The exact int64 z is formed only where fp32 cannot decide:
+//  - max pass: an element whose |zf| is within 3E_w of the largest |zf| its warp has seen,
+//    E_w the largest E of the warp's lanes.  No |zf| of the warp exceeds M + E_w, M = max
+//    |z|, and an element with |z| = M has |zf| >= M - E_w, so that element is evaluated
+//    exactly (the third E_w covers the rounding of the threshold); the largest exact value
+//    over all evaluated elements is M;
+//  - codes pass: y = fl(zf fl(128/M) + 1/2) is within D = 130 E / M + 2^-14 of the exact
+//    128 z / M + 1/2 (the ratio's and the fma's roundings add at most 2^-15); when
+//    floor(y - D) == floor(y + D) that is the code, otherwise the code is
+//    floor((256 z + M) / (2M)) with the 64-bit invariant division, as in k_comb4r.
+// UNR pixels per iteration keep UNR x NC loads of 8 or 16 bytes in flight per thread; the
+// codes stay packed in registers until they are used.
+
+template <int NC>
+struct Cover4 {
+    int n;
+    int id[NC];
+    int ch[NC];
+};
+
+template <int NC>
+__device__ __forceinline__ void cover4_of(const Terms& T, int concat, int co0, Cover4<NC>& cv) {
+    cv.n = 0;
+#pragma unroll
+    for (int k = 0; k < NC; k++) { cv.id[k] = 0; cv.ch[k] = 0; }
+#pragma unroll
+    for (int i = 0; i < IQ_MAX_TERMS; i++) {
+        if (i >= T.n) break;
+        const int ch = concat ? co0 - T.t[i].c_offset : co0;
+        if (ch < 0 || ch >= T.t[i].c) continue;
+#pragma unroll
+        for (int k = 0; k < NC; k++)
+            if (k == cv.n) { cv.id[k] = i; cv.ch[k] = ch; }
+        cv.n++;
+    }
+}
+
+// int64 -> fp32 through the two 32-bit halves of |v| (64-bit conversions run on the narrow
+// FP64 pipe of this part): |v| = hi 2^32 + lo with hi < 2^24 (|v| < 2^56) is exact in
+// hi 2^32, so fma(hi, 2^32, fl(lo)) is fl(lo) when hi = 0 and otherwise within
+// 2^8 + u |v| <= 2u |v| of |v| (u = 2^-24): a relative error of at most 2u.
+__device__ __forceinline__ float f32_of_i64(long long v) {
+    const unsigned long long a = (unsigned long long)(v < 0 ? -v : v);
+    const float f = fmaf((float)(uint32_t)(a >> 32), 0x1p32f, __uint2float_rn((uint32_t)a));
+    return v < 0 ? -f : f;
+}
+// an fp32 upper bound of |v|
+__device__ __forceinline__ float f32_abs_up(long long v) {
+    const unsigned long long a = (unsigned long long)(v < 0 ? -v : v);
+    return __fmaf_ru(__uint2float_ru((uint32_t)(a >> 32)), 0x1p32f,
+                     __uint2float_ru((uint32_t)a));
+}
+
+// CPT codes of one operand as loaded: 16 bytes (CPT = 8 int16 or 16 int8 codes) or
+// 8 bytes (CPT = 8 int8 codes)
+struct Raw16 {
+    uint32_t w[4];
+};
+
+template <int CPT>
+__device__ __forceinline__ Raw16 load_raw(const char* p, int is16) {
+    Raw16 r;
+    if (CPT == 16 || is16) {
+        const int4 q = __ldg(reinterpret_cast<const int4*>(p));
+        r.w[0] = (uint32_t)q.x; r.w[1] = (uint32_t)q.y; r.w[2] = (uint32_t)q.z; r.w[3] = (uint32_t)q.w;
+    } else {
+        const int2 q = __ldg(reinterpret_cast<const int2*>(p));
+        r.w[0] = (uint32_t)q.x; r.w[1] = (uint32_t)q.y; r.w[2] = 0u; r.w[3] = 0u;
+    }
+    return r;
+}
+
+template <int CPT>
+__device__ __forceinline__ int32_t raw_code(const Raw16& r, int is16, int j) {
+    if (CPT == 8 && is16) {
+        const uint32_t w = r.w[j >> 1];
+        return (j & 1) ? (int32_t)w >> 16 : (int32_t)(int16_t)(w & 0xffffu);
+    }
+    return (int32_t)(int8_t)((r.w[j >> 2] >> (8 * (j & 3))) & 0xffu);
+}
+
+// The two passes with CPT channels per thread.  PLAIN: every operand is int8 codes
+// without gamma / beta, so each has one F for all its channels and B = 0 (the sums of
+// errors and the ASPP concatenation); otherwise (the residual joins) F and B are
+// per channel, codes int16 or int8, CPT = 8.
+template <int PASS, int NC, int CPT, int UNR, bool PLAIN>
+__global__ void __launch_bounds__(kThreads, (PLAIN && NC <= 2) ? 3 : 2) k_comb4f(Terms T, int concat, int64_t npix, int cgs,
+                                                     int relu, const long long* __restrict__ F,
+                                                     const long long* __restrict__ B,
+                                                     CombHdr* hdr, int8_t* __restrict__ out,
+                                                     UDiv dhw, int any_bcast) {
+    constexpr int FW = PLAIN ? 1 : CPT;      // F values held per operand
+    const int64_t tcount = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % cgs);
+    const int64_t pstride = tcount / cgs;
+    const int co0 = CPT * g;
+    Cover4<NC> cv;
+    cover4_of<NC>(T, concat, co0, cv);
+    const int nc = cv.n;
+    // per covering operand: its codes at the group's first channel, row bytes, type,
+    // broadcast flag, first row of F / B, fp32 F; the fp32 B sums; the bound S
+    const char* base[NC];
+    int rowb[NC], is16[NC], bc[NC], fo[NC];
+    float ff[NC][FW];
+    float bf[FW];
+    long long fi[NC];          // PLAIN: the exact F of each operand
+    float S = 0.f;             // fp32 with upward rounding: an upper bound of the exact S
+    {
+        long long bs[FW];
+        float sv[FW];
+#pragma unroll
+        for (int j = 0; j < FW; j++) { bs[j] = 0; sv[j] = 0.f; }
+#pragma unroll
+        for (int k = 0; k < NC; k++) {
+            const TermDev& tt = term_at(T, cv.id[k]);
+            const bool on = k < nc;
+            is16[k] = PLAIN ? 0 : tt.is16;
+            bc[k] = tt.bcast;
+            rowb[k] = tt.c * (tt.is16 ? 2 : 1);
+            base[k] = (const char*)tt.codes + (size_t)cv.ch[k] * (tt.is16 ? 2 : 1);
+            fo[k] = tt.base + cv.ch[k];
+            const float vmax = tt.is16 ? 32767.f : 127.f;
+#pragma unroll
+            for (int j = 0; j < FW; j++) {
+                const long long f = on ? F[fo[k] + j] : 0;
+                ff[k][j] = f32_of_i64(f);
+                if (PLAIN) fi[k] = f;
+                if (!PLAIN) bs[j] += on ? B[fo[k] + j] : 0;
+                sv[j] = __fmaf_ru(f32_abs_up(f), vmax, sv[j]);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < FW; j++) {
+            bf[j] = f32_of_i64(bs[j]);
+            const float sj = __fadd_ru(sv[j], f32_abs_up(bs[j]));
+            S = fmaxf(S, sj);
+        }
+    }
+    const float E = __fmul_ru(__fmul_ru((float)(nc + 3), 0x1p-24f), S);
+    // the max pass shares its running maximum across the warp, so its margin covers the
+    // largest E of the warp's lanes
+    float E3 = __fmul_ru(3.f, E);
+    if (PASS == 0) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) E3 = fmaxf(E3, __shfl_xor_sync(0xffffffffu, E3, o));
+    }
+    uint64_t M = 0;
+    float kq = 0.f, D = 0.f;
+    if (PASS == 1) {
+        M = hdr->M;
+        kq = hdr->kq;
+        D = __fmaf_ru(E, hdr->c130, 0x1p-14f);
+    }
+    // exact z of channel j of a pixel from its loaded codes (F and B re-read: a rare path)
+    auto exact = [&](const Raw16 (&r)[NC], int j) -> int64_t {
+        int64_t z = 0;
+#pragma unroll
+        for (int k = 0; k < NC; k++)
+            if (k < nc) {
+                const int64_t f = PLAIN ? fi[k] : F[fo[k] + j];
+                z += f * raw_code<CPT>(r[k], is16[k], j);
+                if (!PLAIN) z += B[fo[k] + j];
+            }
+        return (relu && z < 0) ? 0 : z;
+    };
+    float fmx = 0.f;
+    uint64_t mx = 0;
+    auto one = [&](int64_t pix, const Raw16 (&r)[NC]) {
+        const bool valid = pix < npix;
+        float zf[CPT];
+#pragma unroll
+        for (int j = 0; j < CPT; j++) zf[j] = PLAIN ? 0.f : bf[PLAIN ? 0 : j];
+#pragma unroll
+        for (int k = 0; k < NC; k++)
+            if (k < nc) {
+#pragma unroll
+                for (int j = 0; j < CPT; j++)
+                    zf[j] = fmaf(ff[k][PLAIN ? 0 : j], (float)raw_code<CPT>(r[k], is16[k], j),
+                                 zf[j]);
+            }
+        if (PASS == 0) {
+            // the pixel's largest |zf| first, so that only elements near the running maximum
+            // (usually none of the pixel's) take the exact form
+            float a[CPT], am = 0.f;
+#pragma unroll
+            for (int j = 0; j < CPT; j++) {
+                a[j] = fabsf(relu ? fmaxf(zf[j], 0.f) : zf[j]);
+                am = fmaxf(am, a[j]);
+            }
+            if (!valid) am = 0.f;
+            fmx = fmaxf(fmx, am);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) fmx = fmaxf(fmx, __shfl_xor_sync(0xffffffffu, fmx, o));
+            const float thr = fmx - E3;
+            if (valid && am >= thr) {
+#pragma unroll
+                for (int j = 0; j < CPT; j++)
+                    if (a[j] >= thr) {
+                        const int64_t z = exact(r, j);
+                        const uint64_t az = (uint64_t)(z < 0 ? -z : z);
+                        mx = az > mx ? az : mx;
+                    }
+            }
+        } else {
+            uint32_t w[CPT / 4];
+#pragma unroll
+            for (int q = 0; q < CPT / 4; q++) w[q] = 0u;
+            if (M) {
+#pragma unroll
+                for (int j = 0; j < CPT; j++) {
+                    const float y = fmaf(relu ? fmaxf(zf[j], 0.f) : zf[j], kq, 0.5f);
+                    const float lo = floorf(y - D), hi = floorf(y + D);
+                    int64_t c;
+                    if (lo == hi) {      // only when D < 1/2, so |y| < 130
+                        c = min(max((int)lo, -127), 127);
+                    } else {
+                        const UDiv d2m = hdr->div;
+                        const uint64_t num = ((uint64_t)(exact(r, j) + (int64_t)M) << 8) + M;
+                        c = clamp64((int64_t)udiv(num, d2m) - 128, -127, 127);
+                    }
+                    w[j >> 2] |= ((uint32_t)c & 0xffu) << (8 * (j & 3));
+                }
+            }
+            int8_t* o = out + pix * (int64_t)cgs * CPT + co0;
+            if (!valid) return;
+            if (CPT == 16)
+                *reinterpret_cast<uint4*>(o) = make_uint4(w[0], w[1], w[2], w[3]);
+            else
+                *reinterpret_cast<uint2*>(o) = make_uint2(w[0], w[1]);
+        }
+    };
+    auto load = [&](int64_t pix, Raw16 (&r)[NC]) {
+        const bool valid = pix < npix;
+        const int64_t img = (any_bcast && valid) ? (int64_t)udiv((uint64_t)pix, dhw) : 0;
+#pragma unroll
+        for (int k = 0; k < NC; k++) {
+            if (k < nc && valid) {
+                r[k] = load_raw<CPT>(base[k] + (bc[k] ? img : pix) * rowb[k], is16[k]);
+            } else {
+#pragma unroll
+                for (int q = 0; q < 4; q++) r[k].w[q] = 0u;
+            }
+        }
+    };
+    // every lane of a warp runs the warp's largest number of pixel steps (the max pass
+    // shuffles inside the loop); steps past the tensor's end load and store nothing
+    const int64_t p0 = t / cgs;
+    int64_t steps = p0 < npix ? (npix - p0 + pstride - 1) / pstride : 0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const int64_t w = __shfl_xor_sync(0xffffffffu, steps, o);
+        steps = w > steps ? w : steps;
+    }
+    for (int64_t k0 = 0; k0 < steps; k0 += UNR) {
+        Raw16 r[UNR][NC];
+#pragma unroll
+        for (int u = 0; u < UNR; u++) load(p0 + (k0 + u) * pstride, r[u]);
+#pragma unroll
+        for (int u = 0; u < UNR; u++) one(p0 + (k0 + u) * pstride, r[u]);
+    }
+    if (PASS == 0) {
+        mx = warp_max_u64(mx);
+        if ((threadIdx.x & 31) == 0 && mx) atomicMax(&hdr->maxz, (unsigned long long)mx);
+    }
+}
+
 __global__ void k_comb_params(CombHdr* hdr, double* s_out) {
     const uint64_t M = hdr->maxz;
     hdr->M = M;
     hdr->div = make_udiv(M ? 2 * M : 1);
+    hdr->kq = M ? (float)(128.0 / (double)M) : 0.f;
+    hdr->c130 = M ? __double2float_ru(__ddiv_ru(130.0, (double)M)) : 0.f;
     *s_out = M ? ldexp((double)M, -hdr->P - 7) : ldexp(1.0, -hdr->P - 7);
 }
 
@@ -645,6 +925,80 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
         in_b += (double)(T.t[i].bcast ? n : n * hw) * T.t[i].c * (T.t[i].is16 ? 2.0 : 1.0);
     const double out_b = (double)total;
     const UDiv dhw = make_udiv((uint64_t)hw);
+    // the wide kernels: every operand's channel count and offset and c_out a multiple of the
+    // channels per thread, codes 16-byte (8-byte for int8 at 8 channels) aligned; the most
+    // operands covering any group (checked per group on the host) and whether all are plain
+    // int8 codes decide the variant
+    bool plain = true, any16 = false;
+    for (int i = 0; i < n_terms; i++) {
+        plain = plain && !T.t[i].gamma && !T.t[i].beta && !T.t[i].is16;
+        any16 = any16 || T.t[i].is16;
+    }
+    const int cpt = plain ? 16 : 8;
+    bool wide = c_out % cpt == 0 && ((uintptr_t)out & (cpt - 1)) == 0;
+    for (int i = 0; i < n_terms && wide; i++) {
+        const TermDev& t = T.t[i];
+        const uintptr_t al = (cpt == 16 || t.is16) ? 15 : 7;
+        wide = t.c % cpt == 0 && t.c_offset % cpt == 0 && ((uintptr_t)t.codes & al) == 0;
+    }
+    int maxcover = 0;
+    for (int co = 0; co < c_out && wide; co += cpt) {
+        int nc = 0;
+        for (int i = 0; i < n_terms; i++) {
+            const TermDev& t = T.t[i];
+            const int ch = concat ? co - t.c_offset : co;
+            if (ch >= 0 && ch < t.c) nc++;
+        }
+        maxcover = nc > maxcover ? nc : maxcover;
+    }
+    (void)any16;
+    if (wide && (plain ? maxcover <= 6 : maxcover <= 2)) {
+        const int cgs = c_out / cpt;
+        const int64_t npix = n * hw;
+        // a multiple of cgs threads, about 8 blocks of 256 per SM
+        int64_t gcd = cgs, b2 = kThreads;
+        while (b2) { int64_t r = gcd % b2; gcd = b2; b2 = r; }
+        const int64_t unit = cgs / gcd;                 // blocks per whole number of groups
+        int64_t want = (npix * cgs + kThreads - 1) / kThreads;
+        if (want > 152 * 8) want = 152 * 8;
+        want = (want + unit - 1) / unit * unit;
+        if (want < unit) want = unit;
+        const int g = (int)want;
+        const int cc = concat != 0, rl = relu != 0;
+        for (int pass = 0; pass < 2; pass++) {
+            kt_pre(st);
+            if (!plain) {
+                if (pass == 0)
+                    k_comb4f<0, 2, 8, 2, false><<<g, kThreads, 0, st>>>(T, cc, npix, cgs, rl, F, B,
+                                                                        hdr, out, dhw, any_bcast);
+                else
+                    k_comb4f<1, 2, 8, 2, false><<<g, kThreads, 0, st>>>(T, cc, npix, cgs, rl, F, B,
+                                                                        hdr, out, dhw, any_bcast);
+            } else if (maxcover <= 2) {
+                if (pass == 0)
+                    k_comb4f<0, 2, 16, 2, true><<<g, kThreads, 0, st>>>(T, cc, npix, cgs, rl, F, B,
+                                                                        hdr, out, dhw, any_bcast);
+                else
+                    k_comb4f<1, 2, 16, 2, true><<<g, kThreads, 0, st>>>(T, cc, npix, cgs, rl, F, B,
+                                                                        hdr, out, dhw, any_bcast);
+            } else {
+                if (pass == 0)
+                    k_comb4f<0, 6, 16, 1, true><<<g, kThreads, 0, st>>>(T, cc, npix, cgs, rl, F, B,
+                                                                        hdr, out, dhw, any_bcast);
+                else
+                    k_comb4f<1, 6, 16, 1, true><<<g, kThreads, 0, st>>>(T, cc, npix, cgs, rl, F, B,
+                                                                        hdr, out, dhw, any_bcast);
+            }
+            IQ_LAUNCH_CHECK();
+            kt_post_bytes(st, pass == 0 ? IQ_KERNEL_COMBINE_MAX : IQ_KERNEL_COMBINE_CODES,
+                          pass == 0 ? in_b : in_b + out_b);
+            if (pass == 0) {
+                k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
+                IQ_LAUNCH_CHECK();
+            }
+        }
+        return IQ_OK;
+    }
     // at most two operands cover any 4-channel group: sums of up to two operands, and
     // concatenations whose ranges overlap at most pairwise (checked per group on the host)
     bool two = vec4;
@@ -679,35 +1033,6 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
         kt_pre(st);
         k_comb4r<1><<<g, kThreads, 0, st>>>(T, concat != 0, npix, cgs, relu != 0, F, B, hdr, out,
                                             dhw, any_bcast);
-        IQ_LAUNCH_CHECK();
-        kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b);
-        return IQ_OK;
-    }
-    // sums whose operands all cover every channel, F rows of all of them in shared memory
-    bool all_cover = vec4 && !concat && n_terms <= 6;
-    for (int i = 0; i < n_terms && all_cover; i++) all_cover = T.t[i].c == c_out;
-    if (all_cover) {
-        const int cgs = c_out / 4;
-        const int64_t npix = n * hw;
-        int64_t gcd = cgs, b2 = kThreads;
-        while (b2) { int64_t r = gcd % b2; gcd = b2; b2 = r; }
-        const int64_t unit = cgs / gcd;
-        int64_t want = (npix * cgs + kThreads - 1) / kThreads;
-        if (want > 152 * 8) want = 152 * 8;
-        want = (want + unit - 1) / unit * unit;
-        if (want < unit) want = unit;
-        const int g = (int)want;
-        const size_t sm = (size_t)n_terms * kThreads * 4 * 8;   // <= 48 KB
-        kt_pre(st);
-        k_combNs<0><<<g, kThreads, sm, st>>>(T, npix, cgs, relu != 0, F, B, hdr, out, dhw,
-                                             any_bcast);
-        IQ_LAUNCH_CHECK();
-        kt_post_bytes(st, IQ_KERNEL_COMBINE_MAX, in_b);
-        k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
-        IQ_LAUNCH_CHECK();
-        kt_pre(st);
-        k_combNs<1><<<g, kThreads, sm, st>>>(T, npix, cgs, relu != 0, F, B, hdr, out, dhw,
-                                             any_bcast);
         IQ_LAUNCH_CHECK();
         kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b);
         return IQ_OK;

@@ -32,11 +32,22 @@ def scal():
 
 # ---------------------------------------------------------------- combine
 
-def run_combine(specs, n, hw, c_out, concat, relu):
-    """specs: list of (codes np, scale, c_offset, bcast, gamma np|None, beta np|None)."""
+def dev_offset(a, elems):
+    """A device copy of `a` that starts `elems` elements into a larger buffer (an address
+    that is not 16-byte aligned when elems * itemsize is not a multiple of 16)."""
+    flat = np.ascontiguousarray(a).ravel()
+    buf = torch.zeros(flat.size + elems, dtype=dev(flat[:1]).dtype, device=DEV)
+    buf[elems:] = dev(flat)
+    return buf[elems:].view(a.shape)
+
+
+def run_combine(specs, n, hw, c_out, concat, relu, misalign=False):
+    """specs: list of (codes np, scale, c_offset, bcast, gamma np|None, beta np|None).
+    misalign: operands 8 bytes past a 16-byte boundary."""
     keep, terms, oterms = [], [], []
     for codes, s, off, bc, gam, bet in specs:
-        dc, ds = dev(codes), dscal(s)
+        dc = dev_offset(codes, 8 // codes.itemsize) if misalign else dev(codes)
+        ds = dscal(s)
         dg = dev(gam) if gam is not None else None
         db = dev(bet) if bet is not None else None
         keep += [dc, ds, dg, db]
@@ -123,6 +134,24 @@ def test_combine_four_channel_groups(n, hw, c):
                 n, hw, c, False, True)
     run_combine([(sc, 0.02, 0, False, None, None), (X, 2.0 ** -15, 0, False, gam, bet)],
                 n, hw, c, False, False)
+
+
+def test_combine_unaligned_operands():
+    """Operands whose codes start 8 bytes past a 16-byte boundary (4-byte loads of int8
+    codes, 8-byte loads of int16 codes stay aligned): a two-operand residual join and a
+    five-operand sum with a broadcast operand."""
+    g = np.random.default_rng(21)
+    n, hw, c = 2, 21 * 23, 64
+    X = g.integers(-32767, 32768, size=(n, hw, c)).astype(np.int16)
+    sc = g.integers(-127, 128, size=(n, hw, c)).astype(np.int8)
+    gam = g.integers(-127, 128, size=c).astype(np.int32)
+    bet = g.integers(-127, 128, size=c).astype(np.int32)
+    run_combine([(X, 2.0 ** -15 * 1.3, 0, False, gam, bet), (sc, 0.017, 0, False, None, None)],
+                n, hw, c, False, True, misalign=True)
+    specs = [(g.integers(-127, 128, size=(n, hw, c)).astype(np.int8), s, 0, False, None, None)
+             for s in (0.01, 0.3, 1e-4, 0.02)]
+    specs.append((g.integers(-127, 128, size=(n, c)).astype(np.int8), 0.5 / hw, 0, True, None, None))
+    run_combine(specs, n, hw, c, False, False, misalign=True)
 
 
 def test_combine_small_values_and_negative_relu():
