@@ -971,6 +971,84 @@ __global__ void __launch_bounds__(kThreads) k_bnb_pass3(const int8_t* __restrict
     }
 }
 
+// int8 / int16 code j of a packed row segment
+__device__ __forceinline__ int code8(const uint32_t* o, int j) {
+    return (int)(int8_t)((o[j >> 2] >> (8 * (j & 3))) & 0xffu);
+}
+__device__ __forceinline__ int code16(const uint32_t* o, int j) {
+    const uint32_t v = o[j >> 1];
+    return (j & 1) ? (int)v >> 16 : (int)(int16_t)(v & 0xffffu);
+}
+
+// Pass 3 with 16 channels per thread (C % 16 == 0): 16-byte loads of the errors and
+// activation codes, two of the X codes, one 16-byte store.  A block is 4 channel groups
+// (64 channels) x 64 row lanes; the 64 channels' tables sit in shared memory in rows of
+// 772 bytes (the 768-byte rows padded by one word, so that the rows of neighbouring
+// channels start in different banks).
+constexpr int kTab3P = kTab3 + 4;
+
+__global__ void __launch_bounds__(kThreads, 4) k_bnb_p3w(const int8_t* __restrict__ ea,
+                                                         const int8_t* __restrict__ a,
+                                                         const int16_t* __restrict__ X,
+                                                         int64_t m, int32_t C, BnBwd w,
+                                                         int8_t* __restrict__ out) {
+    extern __shared__ __align__(16) uint32_t tab3w[];   // [64][kTab3P / 4]
+    const int64_t cb = 64 * (int64_t)blockIdx.x;
+    const int nch = (int)min((int64_t)64, (int64_t)C - cb);
+    {
+        const uint32_t* src = reinterpret_cast<const uint32_t*>(w.t3 + cb * kTab3);
+        for (int i = threadIdx.x; i < nch * (kTab3 / 4); i += blockDim.x) {
+            const int ch = i / (kTab3 / 4), k = i - ch * (kTab3 / 4);
+            tab3w[ch * (kTab3P / 4) + k] = src[i];
+        }
+    }
+    __syncthreads();
+    const int cg = threadIdx.x & 3, rl = threadIdx.x >> 2;
+    if (16 * cg >= nch) return;
+    const int64_t c0 = cb + 16 * cg;
+    const int8_t* tb = reinterpret_cast<const int8_t*>(tab3w) + 16 * cg * kTab3P;
+    const int64_t step = (int64_t)gridDim.y * 64;
+    auto code16x = [&](const int4 e, const int4 am, const int4 x0, const int4 x1) {
+        const uint32_t ev[4] = {(uint32_t)e.x, (uint32_t)e.y, (uint32_t)e.z, (uint32_t)e.w};
+        const uint32_t av[4] = {(uint32_t)am.x, (uint32_t)am.y, (uint32_t)am.z, (uint32_t)am.w};
+        const uint32_t xv[8] = {(uint32_t)x0.x, (uint32_t)x0.y, (uint32_t)x0.z, (uint32_t)x0.w,
+                                (uint32_t)x1.x, (uint32_t)x1.y, (uint32_t)x1.z, (uint32_t)x1.w};
+        uint32_t o[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 16; j++) {
+            const int ey = code8(av, j) > 0 ? code8(ev, j) : 0;
+            const int xx = code16(xv, j);
+            const int sg = (xx > 0) - (xx < 0);
+            o[j >> 2] |= ((uint32_t)(uint8_t)tb[j * kTab3P + (sg + 1) * 256 + ey + 128])
+                         << (8 * (j & 3));
+        }
+        return make_uint4(o[0], o[1], o[2], o[3]);
+    };
+    int64_t r = (int64_t)blockIdx.y * 64 + rl;
+    // two rows per iteration: all their loads in flight together
+    for (; r + step < m; r += 2 * step) {
+        const int64_t o0 = r * C + c0, o1 = (r + step) * C + c0;
+        const int4 e0 = __ldg(reinterpret_cast<const int4*>(ea + o0));
+        const int4 a0 = __ldg(reinterpret_cast<const int4*>(a + o0));
+        const int4 x00 = __ldg(reinterpret_cast<const int4*>(X + o0));
+        const int4 x01 = __ldg(reinterpret_cast<const int4*>(X + o0 + 8));
+        const int4 e1 = __ldg(reinterpret_cast<const int4*>(ea + o1));
+        const int4 a1 = __ldg(reinterpret_cast<const int4*>(a + o1));
+        const int4 x10 = __ldg(reinterpret_cast<const int4*>(X + o1));
+        const int4 x11 = __ldg(reinterpret_cast<const int4*>(X + o1 + 8));
+        *reinterpret_cast<uint4*>(out + o0) = code16x(e0, a0, x00, x01);
+        *reinterpret_cast<uint4*>(out + o1) = code16x(e1, a1, x10, x11);
+    }
+    if (r < m) {
+        const int64_t o0 = r * C + c0;
+        *reinterpret_cast<uint4*>(out + o0) =
+            code16x(__ldg(reinterpret_cast<const int4*>(ea + o0)),
+                    __ldg(reinterpret_cast<const int4*>(a + o0)),
+                    __ldg(reinterpret_cast<const int4*>(X + o0)),
+                    __ldg(reinterpret_cast<const int4*>(X + o0 + 8)));
+    }
+}
+
 size_t bn_bwd_ws_bytes(int32_t C) {
     WsCursor c(nullptr, 0);
     bnb_carve(c, C);
@@ -1063,7 +1141,24 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     k_bnb_tab3<<<tb3 < 152 * 4 ? tb3 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, 8, w);
     IQ_LAUNCH_CHECK();
     kt_pre(st);
-    k_bnb_pass3<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w, e);
+    if (c % 16 == 0) {
+        static bool attr = false;
+        const int smem = 64 * kTab3P;
+        if (!attr) {
+            IQ_CUDA_CHECK(cudaFuncSetAttribute(k_bnb_p3w, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               smem));
+            attr = true;
+        }
+        const int bx = (c + 63) / 64;
+        int64_t by3 = (m + 63) / 64;
+        const int64_t cap3 = (152 * 8 + bx - 1) / bx;
+        if (by3 > cap3) by3 = cap3;
+        if (by3 > 65535) by3 = 65535;
+        k_bnb_p3w<<<dim3((unsigned)bx, (unsigned)by3), kThreads, smem, st>>>(e_a, a, xhat, m, c,
+                                                                             w, e);
+    } else {
+        k_bnb_pass3<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w, e);
+    }
     IQ_LAUNCH_CHECK();
     kt_post_bytes(st, IQ_KERNEL_BNB_PASS3, 5.0 * (double)m * c);
     if (dgamma)

@@ -171,6 +171,22 @@ def test_combine_small_values_and_negative_relu():
                 n, hw, c, False, True)
 
 
+def test_combine_ties_at_the_maximum():
+    """Every element at the tensor's largest magnitude (constant codes): the max pass must
+    take the exact form for all of them; then a three-operand int8 sum over 64 channels
+    and an odd pixel count (16 channels per thread, more than two operands per group)."""
+    n, hw, c = 2, 13 * 11, 64
+    run_combine([(np.full((n, hw, c), 77, np.int8), 0.013, 0, False, None, None),
+                 (np.full((n, hw, c), -5, np.int8), 0.2, 0, False, None, None)], n, hw, c,
+                False, False)
+    run_combine([(np.full((n, hw, c), 127, np.int8), 1e-6, 0, False, None, None)], n, hw, c,
+                False, True)
+    g = np.random.default_rng(22)
+    specs = [(g.integers(-127, 128, size=(n, hw, c)).astype(np.int8), s, 0, False, None, None)
+             for s in (3e-7, 1.1e-6, 2e-9)]
+    run_combine(specs, n, hw, c, False, False)
+
+
 def test_combine_edge_cases():
     # all zero, a single pixel, a single channel
     run_combine([(np.zeros((1, 5, 8), np.int8), 0.5, 0, False, None, None)], 1, 5, 8, False, False)
