@@ -8,6 +8,8 @@
 #include "iq_internal.cuh"
 #include "iq_conv_tc.cuh"
 
+#include <algorithm>
+
 #include <climits>
 
 namespace iq {
@@ -444,7 +446,7 @@ extern "C" iq_status iq_conv_dgrad_workspace_size(const iq_conv_desc* d, size_t*
     cur.take<char>(requant_ws_bytes());
     cur.take<double>(1);
     bn_stats_carve(cur, d->c);
-    cur.take<char>(conv_dgrad_tc_ws_bytes(d));
+    cur.take<char>(std::max(conv_dgrad_tc_ws_bytes(d), conv_dgrad_tc_stride2_ws_bytes(d)));
     *bytes = cur.off + 256;
     return IQ_OK;
 }
@@ -697,7 +699,8 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     void* rq = cur.take<char>(requant_ws_bytes());
     double* s_in = cur.take<double>(1);
     BnStats stats = bn_stats_carve(cur, d->c);
-    void* tcws = cur.take<char>(conv_dgrad_tc_ws_bytes(d));
+    const size_t tcb = std::max(conv_dgrad_tc_ws_bytes(d), conv_dgrad_tc_stride2_ws_bytes(d));
+    void* tcws = cur.take<char>(tcb);
     const int64_t total = (int64_t)d->n * d->h * d->w * d->c;
     unsigned long long* cell = (unsigned long long*)rq;
     k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, -7, s_in);
@@ -733,6 +736,22 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
                 return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx,
                                      IQ_I8, s_dx, rq, st, true);
             }
+        }
+    }
+    // stride 2: the four parity phases of the input as stride-1 problems on the tensor cores
+    if (!wide && d->stride_h == 2 && d->stride_w == 2) {
+        iq_status r = bn_stats_init(stats, d->c, st);
+        if (r != IQ_OK) return r;
+        bool done = false;
+        r = conv_dgrad_tc_stride2(d, e, w, acc, stats.s1, stats.hi, stats.lo, tcws, tcb, st,
+                                  &done, (const __half*)e_f16);
+        if (r != IQ_OK) return r;
+        if (done) {
+            k_max_from_stats<<<1, 1024, 0, st>>>(stats.hi, stats.lo, d->c, 0, s_in, cell,
+                                                 rq_params_slot(rq), s_dx);
+            IQ_LAUNCH_CHECK();
+            return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
+                                 s_dx, rq, st, true);
         }
     }
     int64_t wn = (int64_t)d->k * d->r * d->s * cp.Cg;

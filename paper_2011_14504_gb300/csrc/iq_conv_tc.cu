@@ -33,6 +33,8 @@
 // the device's sticky status word, drains what it issued and returns, and every later
 // launch exits at once until the host reads the status (iq_device_status).
 #include "iq_conv_tc.cuh"
+
+#include <algorithm>
 #include "iq_tc_ptx.cuh"
 
 #include <climits>
@@ -2645,6 +2647,183 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
         }
         if (!used) r = launch(map, p, 1, e, nullptr, out32, out64, s1, hi, lo, err, st);
         if (r != IQ_OK) return r;
+    }
+    *done = true;
+    return IQ_OK;
+}
+
+// ================================================================ stride-2 data gradient
+//
+// With stride 2 the input pixels split into four phases by the parity of their row and
+// column.  Input row h = 2i + a takes the taps r with r dil + a + pad even: p = (h + pad -
+// r dil) / 2 = i + o_r.  Those taps form an arithmetic progression (every second tap when dil
+// is odd; all or none when dil is even), so phase (a, b) is the stride-1 data gradient of a
+// sub-kernel -- the taps of the progression, dilation dil' = step dil / 2, padding
+// o_{first tap} -- over the same errors, with ceil((h - a) / 2) rows.  Each phase runs on the
+// stride-1 tensor-core path into a scratch tensor that one kernel interleaves into dx; a phase
+// that no tap reaches is zero.
+
+namespace {
+
+struct Phase1d {
+    int n;        // taps of the phase (0: the phase is zero)
+    int first;    // first tap
+    int step;     // tap step
+    int pad;      // padding of the phase's stride-1 problem
+    int dil;      // its dilation
+    int len;      // input rows (columns) of the phase
+};
+
+Phase1d phase_1d(int extent, int taps, int pad, int dil, int a) {
+    Phase1d f;
+    f.len = (extent - a + 1) / 2;
+    f.step = (dil & 1) ? 2 : 1;
+    f.first = (dil & 1) ? ((a + pad) & 1) : 0;
+    f.n = 0;
+    if (!(dil & 1) && ((a + pad) & 1)) return f;   // even dilation: every tap or none
+    for (int r = f.first; r < taps; r += f.step) f.n++;
+    f.dil = f.step * dil / 2;
+    f.pad = (a + pad - f.first * dil) / 2;          // a + pad - first dil is even
+    return f;
+}
+
+// wsub[k][t][u][c] = w[k][rf + t rs][sf + u ss][c]
+__global__ void k_gather_taps(const int8_t* __restrict__ w, int K, int R, int S, int C, int rf,
+                              int rs, int nr, int sf, int ss, int ns, int8_t* __restrict__ wsub) {
+    const int64_t n = (int64_t)K * nr * ns * C;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % C);
+        int64_t t = i / C;
+        const int u = (int)(t % ns);
+        t /= ns;
+        const int tr = (int)(t % nr);
+        const int k = (int)(t / nr);
+        wsub[i] = w[(((int64_t)k * R + rf + tr * rs) * S + sf + u * ss) * C + c];
+    }
+}
+
+// dx[n][2i + a][2j + b][c] = src[n][i][j][c] (src NULL: 0)
+__global__ void k_phase_scatter(const int32_t* __restrict__ src, int N, int Ha, int Wb, int C,
+                                int H, int W, int a, int b, int32_t* __restrict__ dx) {
+    const int64_t n4 = (int64_t)N * Ha * Wb * (C / 4);
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c4 = (int)(i % (C / 4));
+        int64_t t = i / (C / 4);
+        const int j = (int)(t % Wb);
+        t /= Wb;
+        const int ii = (int)(t % Ha);
+        const int nn = (int)(t / Ha);
+        const int4 v = src ? reinterpret_cast<const int4*>(src)[i] : make_int4(0, 0, 0, 0);
+        reinterpret_cast<int4*>(dx)[(((int64_t)nn * H + 2 * ii + a) * W + 2 * j + b) * (C / 4) + c4] = v;
+    }
+}
+
+}  // namespace
+
+static bool conv_dgrad_tc_stride2_plan(const iq_conv_desc* d, iq_conv_desc sub[4],
+                                       Phase1d* ph = nullptr, Phase1d* pw = nullptr) {
+    if (tc_env_disabled()) return false;
+    if (d->groups != 1 || d->stride_h != 2 || d->stride_w != 2 || d->c % 4) return false;
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / 2 + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / 2 + 1;
+    for (int a = 0; a < 2; a++)
+        for (int b = 0; b < 2; b++) {
+            const Phase1d fr = phase_1d(d->h, d->r, d->pad_h, d->dil_h, a);
+            const Phase1d fs = phase_1d(d->w, d->s, d->pad_w, d->dil_w, b);
+            if (ph) ph[2 * a + b] = fr;
+            if (pw) pw[2 * a + b] = fs;
+            iq_conv_desc& g = sub[2 * a + b];
+            g = *d;
+            g.stride_h = g.stride_w = 1;
+            if (fr.n == 0 || fs.n == 0 || fr.len < 1 || fs.len < 1) {
+                g.r = 0;                       // a zero phase
+                continue;
+            }
+            g.h = fr.len; g.w = fs.len;
+            g.r = fr.n; g.s = fs.n;
+            g.pad_h = fr.pad; g.pad_w = fs.pad;
+            g.dil_h = fr.dil; g.dil_w = fs.dil;
+            if (g.pad_h < 0 || g.pad_w < 0) return false;
+            // the phase's stride-1 problem must read exactly the P x Q errors
+            if (g.h + 2 * g.pad_h - g.dil_h * (g.r - 1) != P ||
+                g.w + 2 * g.pad_w - g.dil_w * (g.s - 1) != Q)
+                return false;
+            if (!conv_dgrad_tc_supported(&g) || conv_dgrad_tc_slices(&g) != 1) return false;
+        }
+    return true;
+}
+
+size_t conv_dgrad_tc_stride2_ws_bytes(const iq_conv_desc* d) {
+    iq_conv_desc sub[4];
+    if (!conv_dgrad_tc_stride2_plan(d, sub)) return 0;
+    size_t b = 0;
+    for (int i = 0; i < 4; i++)
+        if (sub[i].r) b = std::max(b, conv_dgrad_tc_ws_bytes(&sub[i]));
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / 2 + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / 2 + 1;
+    const size_t ef = ((size_t)d->n * P * Q * d->k * 2 + 255) / 256 * 256;
+    const size_t wsub = ((size_t)d->k * d->r * d->s * d->c + 255) / 256 * 256;
+    const size_t scr = ((size_t)d->n * ((d->h + 1) / 2) * ((d->w + 1) / 2) * d->c * 4 + 255) / 256 * 256;
+    return b + ef + wsub + scr + 1024;
+}
+
+iq_status conv_dgrad_tc_stride2(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
+                                int32_t* out32, unsigned long long* s1, int* hi, int* lo,
+                                void* ws, size_t ws_bytes, cudaStream_t st, bool* done,
+                                const __half* ef_given) {
+    *done = false;
+    iq_conv_desc sub[4];
+    Phase1d ph[4], pw[4];
+    if (!conv_dgrad_tc_stride2_plan(d, sub, ph, pw) || !out32 || !s1 || !hi || !lo ||
+        ((uintptr_t)e & 15) || !get_encode())
+        return IQ_OK;
+    if (ws_bytes < conv_dgrad_tc_stride2_ws_bytes(d)) return IQ_ERR_WORKSPACE;
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / 2 + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / 2 + 1;
+    const int64_t ne = (int64_t)d->n * P * Q * d->k;
+    if (ne % 16) return IQ_OK;
+    size_t b = 0;
+    for (int i = 0; i < 4; i++)
+        if (sub[i].r) b = std::max(b, conv_dgrad_tc_ws_bytes(&sub[i]));
+    b = (b + 255) / 256 * 256;
+    char* base = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
+    char* tcws = base;
+    __half* ef = reinterpret_cast<__half*>(base + b);
+    int8_t* wsub = reinterpret_cast<int8_t*>(base + b + ((size_t)ne * 2 + 255) / 256 * 256);
+    int32_t* scr = reinterpret_cast<int32_t*>(
+        (char*)wsub + ((size_t)d->k * d->r * d->s * d->c + 255) / 256 * 256);
+    if (ef_given) {
+        ef = const_cast<__half*>(ef_given);
+    } else {
+        iq_status r = codes_to_f16(e, ef, ne, st);
+        if (r != IQ_OK) return r;
+    }
+    for (int i = 0; i < 4; i++) {
+        const int a = i >> 1, bb = i & 1;
+        const int Ha = (d->h - a + 1) / 2, Wb = (d->w - bb + 1) / 2;
+        if (Ha < 1 || Wb < 1) continue;
+        const int64_t n4 = (int64_t)d->n * Ha * Wb * (d->c / 4);
+        if (!sub[i].r) {
+            k_phase_scatter<<<grid_for(n4), kThreads, 0, st>>>(nullptr, d->n, Ha, Wb, d->c, d->h,
+                                                               d->w, a, bb, out32);
+            IQ_LAUNCH_CHECK();
+            continue;
+        }
+        const int64_t nw = (int64_t)d->k * sub[i].r * sub[i].s * d->c;
+        k_gather_taps<<<grid_for(nw), kThreads, 0, st>>>(w, d->k, d->r, d->s, d->c, ph[i].first,
+                                                         ph[i].step, sub[i].r, pw[i].first,
+                                                         pw[i].step, sub[i].s, wsub);
+        IQ_LAUNCH_CHECK();
+        bool pdone = false;
+        iq_status r = conv_dgrad_tc(&sub[i], e, wsub, scr, nullptr, s1, hi, lo, tcws, st, &pdone,
+                                    ef);
+        if (r != IQ_OK) return r;
+        if (!pdone) return IQ_ERR_CUDA;   // the plan admitted every phase
+        k_phase_scatter<<<grid_for(n4), kThreads, 0, st>>>(scr, d->n, Ha, Wb, d->c, d->h, d->w, a,
+                                                           bb, out32);
+        IQ_LAUNCH_CHECK();
     }
     *done = true;
     return IQ_OK;

@@ -40,6 +40,17 @@ iq_status conv_dgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
                         long long* out64, unsigned long long* s1, int* hi, int* lo, void* ws,
                         cudaStream_t st, bool* done, const __half* ef = nullptr);
 
+// Stride-2 data gradient on the tensor-core path by phase decomposition (groups 1, the
+// int32 path): the four parity phases of the input run as stride-1 data gradients of
+// sub-kernels and are interleaved into out32; the per-channel statistics (s1, hi, lo: C
+// entries each, all written by the kernels) accumulate over the phases.  ef: the fp16 carrier
+// of e when the caller wrote it.  *done = false when the shape is not covered.
+size_t conv_dgrad_tc_stride2_ws_bytes(const iq_conv_desc* d);
+iq_status conv_dgrad_tc_stride2(const iq_conv_desc* d, const int8_t* e, const int8_t* w,
+                                int32_t* out32, unsigned long long* s1, int* hi, int* lo,
+                                void* ws, size_t ws_bytes, cudaStream_t st, bool* done,
+                                const __half* ef = nullptr);
+
 // Weight gradient: writes the exact int64 sums to G (KRSC).  When *amax_done, max |G| has
 // also been folded into *amax (an atomicMax cell the caller zeroed).
 size_t conv_wgrad_tc_ws_bytes(const iq_conv_desc* d);
