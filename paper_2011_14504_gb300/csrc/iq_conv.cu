@@ -320,6 +320,30 @@ __global__ void k_transpose_w(const int8_t* __restrict__ w, int8_t* __restrict__
 
 // ------------------------------------------------------------------ small scale kernels
 
+// Channel padding for the tensor-core kernels (output channels a multiple of 8 in the
+// forward, error channels a multiple of 8 in the data gradient):
+// dst[i][j] = j < cols ? src[i][j] : 0 for rows of cols_p >= cols bytes.
+__global__ void k_pad_cols_i8(const int8_t* __restrict__ src, int64_t rows, int cols, int cols_p,
+                              int8_t* __restrict__ dst) {
+    const int64_t n = rows * cols_p;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = i / cols_p;
+        const int j = (int)(i - r * cols_p);
+        dst[i] = j < cols ? src[r * cols + j] : (int8_t)0;
+    }
+}
+// dst[i][j] = src[i][j] for j < cols from rows of cols_p int32
+__global__ void k_compact_cols_i32(const int32_t* __restrict__ src, int64_t rows, int cols,
+                                   int cols_p, int32_t* __restrict__ dst) {
+    const int64_t n = rows * cols;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = i / cols;
+        dst[i] = src[r * cols_p + (i - r * cols)];
+    }
+}
+
 __global__ void k_scale_mul_pow2(const double* __restrict__ a, int e, double* __restrict__ out) {
     *out = ldexp(*a, e);
 }
@@ -396,18 +420,31 @@ struct FwdWs {
     void* rq;
     double* s_acc;
     void* tc;
+    int32_t* accp;     // output channels padded to a multiple of 8: the padded sums
+    int8_t* wp;        //   and the weights with zero rows appended
 };
+
+// output channels not a multiple of 8 (single group): the tensor-core forward runs on
+// weights padded to kpad(d) rows
+static int fwd_kpad(const iq_conv_desc* d) {
+    return (d->groups == 1 && d->k % 8 && d->c % 4 == 0) ? (d->k + 7) / 8 * 8 : 0;
+}
 
 static size_t fwd_ws_layout(const iq_conv_desc* d, int with_acc, void* base, size_t cap,
                             FwdWs* out) {
     ConvP cp = make_params(d);
     WsCursor cur(base, cap);
     FwdWs w;
+    const int kp = fwd_kpad(d);
     w.acc = with_acc ? cur.take<int32_t>((size_t)cp.npq * cp.K) : nullptr;
-    w.st = bn_stats_carve(cur, cp.K);
+    w.st = bn_stats_carve(cur, kp ? kp : cp.K);
     w.rq = cur.take<char>(requant_ws_bytes());
     w.s_acc = cur.take<double>(1);
-    w.tc = cur.take<char>(conv_fwd_tc_ws_bytes(d));
+    iq_conv_desc dp = *d;
+    if (kp) dp.k = kp;
+    w.tc = cur.take<char>(conv_fwd_tc_ws_bytes(&dp));
+    w.accp = kp ? cur.take<int32_t>((size_t)cp.npq * kp) : nullptr;
+    w.wp = kp ? cur.take<int8_t>((size_t)kp * d->r * d->s * d->c) : nullptr;
     if (out) *out = w;
     return cur.off + 256;
 }
@@ -438,6 +475,29 @@ static bool dgrad_wide(const iq_conv_desc* d) {
     return krs * 127 * 127 >= (int64_t(1) << 31);
 }
 
+// error channels not a multiple of 8 (single group, stride 1, int32 sums): the tensor-core
+// data gradient runs on errors and weights zero-padded to dgrad_kpad(d) channels
+static int dgrad_kpad(const iq_conv_desc* d) {
+    if (d->groups != 1 || d->stride_h != 1 || d->stride_w != 1 || d->k % 8 == 0 || d->c % 8)
+        return 0;
+    const int kp = (d->k + 7) / 8 * 8;
+    if ((int64_t)kp * d->r * d->s * 16129 >= (int64_t(1) << 31)) return 0;
+    iq_conv_desc dp = *d;
+    dp.k = kp;
+    return conv_dgrad_tc_supported(&dp) ? kp : 0;
+}
+
+static size_t dgrad_pad_ws(const iq_conv_desc* d) {
+    const int kp = dgrad_kpad(d);
+    if (!kp) return 0;
+    iq_conv_desc dp = *d;
+    dp.k = kp;
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    return conv_dgrad_tc_ws_bytes(&dp) + ((size_t)d->n * P * Q * kp + 255) / 256 * 256 +
+           ((size_t)kp * d->r * d->s * d->c + 255) / 256 * 256 + 512;
+}
+
 extern "C" iq_status iq_conv_dgrad_workspace_size(const iq_conv_desc* d, size_t* bytes) {
     if (!desc_ok(d) || !bytes) return IQ_ERR_INVALID_ARG;
     WsCursor cur(nullptr, 0);
@@ -446,7 +506,8 @@ extern "C" iq_status iq_conv_dgrad_workspace_size(const iq_conv_desc* d, size_t*
     cur.take<char>(requant_ws_bytes());
     cur.take<double>(1);
     bn_stats_carve(cur, d->c);
-    cur.take<char>(std::max(conv_dgrad_tc_ws_bytes(d), conv_dgrad_tc_stride2_ws_bytes(d)));
+    cur.take<char>(std::max({conv_dgrad_tc_ws_bytes(d), conv_dgrad_tc_stride2_ws_bytes(d),
+                             dgrad_pad_ws(d)}));
     *bytes = cur.off + 256;
     return IQ_OK;
 }
@@ -655,9 +716,31 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     // batch norm reads the sums and both extremes; SQ of ReLU(acc) only the maxima
     // (the batch-norm deviation pass computes the per-channel extremes itself)
     const unsigned want = use_bn ? (TC_STATS_SUM | TC_STATS_NOEXT) : (relu ? 0u : TC_STATS_LO);
-    r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done,
-                    (const __half*)x_f16, want);
-    if (r != IQ_OK) return r;
+    const int kp = use_bn ? 0 : fwd_kpad(d);
+    if (kp) {
+        // zero weight rows up to kp output channels, the padded sums compacted to k columns
+        // (the zero channels cannot raise the maximum the requantizer takes)
+        iq_conv_desc dp = *d;
+        dp.k = kp;
+        const int64_t rsc = (int64_t)d->r * d->s * d->c;
+        k_pad_cols_i8<<<grid_for((int64_t)kp * rsc), kThreads, 0, st>>>(w, 1, (int)(d->k * rsc),
+                                                                         (int)(kp * rsc), L.wp);
+        IQ_LAUNCH_CHECK();
+        r = bn_stats_init(L.st, kp, st);
+        if (r != IQ_OK) return r;
+        r = conv_fwd_tc(&dp, x, L.wp, L.accp, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done,
+                        (const __half*)x_f16, want);
+        if (r != IQ_OK) return r;
+        if (done) {
+            k_compact_cols_i32<<<grid_for(cp.npq * cp.K), kThreads, 0, st>>>(L.accp, cp.npq, cp.K,
+                                                                            kp, acc);
+            IQ_LAUNCH_CHECK();
+        }
+    } else {
+        r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done,
+                        (const __half*)x_f16, want);
+        if (r != IQ_OK) return r;
+    }
     if (!done) {
         dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
         kt_pre(st);
@@ -699,7 +782,8 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     void* rq = cur.take<char>(requant_ws_bytes());
     double* s_in = cur.take<double>(1);
     BnStats stats = bn_stats_carve(cur, d->c);
-    const size_t tcb = std::max(conv_dgrad_tc_ws_bytes(d), conv_dgrad_tc_stride2_ws_bytes(d));
+    const size_t tcb = std::max({conv_dgrad_tc_ws_bytes(d), conv_dgrad_tc_stride2_ws_bytes(d),
+                                 dgrad_pad_ws(d)});
     void* tcws = cur.take<char>(tcb);
     const int64_t total = (int64_t)d->n * d->h * d->w * d->c;
     unsigned long long* cell = (unsigned long long*)rq;
@@ -736,6 +820,35 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
                 return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx,
                                      IQ_I8, s_dx, rq, st, true);
             }
+        }
+    }
+    // error channels padded to a multiple of 8: zero error channels and zero weight rows
+    if (const int kp = !wide ? dgrad_kpad(d) : 0) {
+        iq_conv_desc dp = *d;
+        dp.k = kp;
+        const int64_t npq = (int64_t)d->n * cp.P * cp.Q;
+        const int64_t rsc = (int64_t)d->r * d->s * d->c;
+        char* b = (char*)tcws;
+        int8_t* ep = reinterpret_cast<int8_t*>(b);
+        int8_t* wp = reinterpret_cast<int8_t*>(b + ((size_t)npq * kp + 255) / 256 * 256);
+        void* tws = b + ((size_t)npq * kp + 255) / 256 * 256 + ((size_t)kp * rsc + 255) / 256 * 256;
+        k_pad_cols_i8<<<grid_for(npq * kp), kThreads, 0, st>>>(e, npq, d->k, kp, ep);
+        IQ_LAUNCH_CHECK();
+        k_pad_cols_i8<<<grid_for((int64_t)kp * rsc), kThreads, 0, st>>>(w, 1, (int)(d->k * rsc),
+                                                                         (int)(kp * rsc), wp);
+        IQ_LAUNCH_CHECK();
+        iq_status r = bn_stats_init(stats, d->c, st);
+        if (r != IQ_OK) return r;
+        bool done = false;
+        r = conv_dgrad_tc(&dp, ep, wp, acc, nullptr, stats.s1, stats.hi, stats.lo, tws, st, &done,
+                          nullptr);
+        if (r != IQ_OK) return r;
+        if (done) {
+            k_max_from_stats<<<1, 1024, 0, st>>>(stats.hi, stats.lo, d->c, 0, s_in, cell,
+                                                 rq_params_slot(rq), s_dx);
+            IQ_LAUNCH_CHECK();
+            return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
+                                 s_dx, rq, st, true);
         }
     }
     // stride 2: the four parity phases of the input as stride-1 problems on the tensor cores
