@@ -60,15 +60,26 @@ enum {
     IQ_MODE_RQ_GQ2 = 5   /* Eq. (GQ2): RQ(G/Scale(G), k), magnitude dropped             */
 };
 
-/* Convolution geometry.  Input NHWC [n][h][w][c]; filters KRSC [k][r][s][c/groups];
- * output [n][p][q][k] with p = (h + 2 pad_h - dil_h (r-1) - 1) / stride_h + 1 (q alike).
- * Output pixel (p,q), tap (r,s) reads input row p*stride_h + r*dil_h - pad_h and
- * column q*stride_w + s*dil_w - pad_w; outside the image the input is zero.
- * Group g maps input channels [g c/G, (g+1) c/G) to outputs [g k/G, (g+1) k/G). */
+/* Convolution geometry and code widths (Sec. 3.2, Eqs. (WQ1), (AQ1); the problem statement of
+ * Sec. 3 fixes no memory layout).  With layout IQ_LAYOUT_NHWC: input NHWC [n][h][w][c],
+ * filters KRSC [k][r][s][c/groups], output and errors [n][p][q][k].  With IQ_LAYOUT_NCHW:
+ * input [n][c][h][w], filters KCRS [k][c/groups][r][s], output and errors [n][k][p][q]
+ * (the gradient codes and sums of iq_conv_wgrad follow the filter layout); the library
+ * transposes through the workspace and computes in NHWC.  p = (h + 2 pad_h - dil_h (r-1)
+ * - 1) / stride_h + 1 (q alike).  Output pixel (p,q), tap (r,s) reads input row
+ * p*stride_h + r*dil_h - pad_h and column q*stride_w + s*dil_w - pad_w; outside the image the
+ * input is zero.  Group g maps input channels [g c/G, (g+1) c/G) to outputs [g k/G, (g+1) k/G).
+ *   k_w  bit width of the weight codes W_q = UQ(W_m, k_w) (Eq. (WQ1)), 2..8, 0 = 8: their
+ *        step 2^(1-k_w) is the weight factor of the accumulator scale
+ *   k_a  bit width of the output activation codes Q_A = SQ(., k_a) (Eq. (AQ1)), 2..8,
+ *        0 = 8 (with batch norm the bits argument's k_a, when given, must agree)
+ * A zero-initialised descriptor tail gives the paper's setting (NHWC, 8-bit codes). */
+enum { IQ_LAYOUT_NHWC = 0, IQ_LAYOUT_NCHW = 1 };
 typedef struct {
     int32_t n, h, w, c;
     int32_t k, r, s;
     int32_t stride_h, stride_w, pad_h, pad_w, dil_h, dil_w, groups;
+    int32_t layout, k_w, k_a;
 } iq_conv_desc;
 
 /* Bit widths of the quantized L1BN objects (Sec. 3.2.2 equation block, Eq. (AQ1)). */
@@ -215,7 +226,7 @@ iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_
  *   bn != NULL:  quantized L1BN (Eqs. (BN2),(BN4),(BN5) and the QBN block; the same
  *                computation as iq_bn_int_fwd) + ReLU + Q_A.
  *   x      int8 NHWC [n][h][w][c];  s_x: device double (scale of x)
- *   w      int8 KRSC, codes of W_q = UQ(W_m, 8) (scale 2^-7; s_acc = s_x 2^-7)
+ *   w      int8 KRSC, codes of W_q = UQ(W_m, k_w) (scale 2^(1-k_w); s_acc = s_x 2^(1-k_w))
  *   gamma, beta  device int32[k]: codes of gamma_q = 2 UQ(gamma/2, k_gamma) etc. (bn only)
  *   bits   bit widths (bn only; NULL = paper defaults)
  *   a      out int8 NHWC [n][p][q][k];  s_a: out device double
@@ -224,8 +235,9 @@ iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_
  *   bn_scales out device double[IQ_BN_SCALES] (bn only, may be NULL)
  *   acc_out   optional out int32 [n][p][q][k]: the raw accumulators
  *   x_f16     optional out fp16 [n][h][w][c] (16-byte aligned, n h w c % 16 == 0, else
- *             IQ_ERR_INVALID_ARG): the exact fp16 copy of the codes x that the tensor-core
- *             kernels read (every int8 code is exact in fp16).  When given it is written first
+ *             IQ_ERR_INVALID_ARG): the exact fp16 copy of the codes x (of their NHWC
+ *             transpose with IQ_LAYOUT_NCHW) that the tensor-core kernels read (every int8
+ *             code is exact in fp16).  When given it is written first
  *             and the kernels read it; keep it for iq_conv_wgrad of the same layer, which then
  *             skips its own conversion of x.  (The paper has no counterpart: it is the
  *             operand format of this implementation's tensor-core path.)
@@ -239,8 +251,8 @@ iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
 /* iq_conv_dgrad -- error of the layer input (Sec. 3.3.1, Eq. (EQ)):
  * dx = conv_transpose(e, w) in exact int32, then E_1 = SQ(dx, 8).
  *   e    int8 [n][p][q][k] error codes at the conv output; s_e device double
- *   w    int8 KRSC forward weights (scale 2^-7)
- *   dx   out int8 NHWC [n][h][w][c]; s_dx out device double = (s_e 2^-7 M) 2^-7
+ *   w    int8 KRSC forward weights (scale 2^(1-k_w))
+ *   dx   out int8 NHWC [n][h][w][c]; s_dx out device double = (s_e 2^(1-k_w) M) 2^-7
  *   acc_out optional out int32 [n][h][w][c]; must be NULL when (k/groups) r s 127^2 >= 2^31,
  *           where the sums are accumulated in int64 (IQ_ERR_UNSUPPORTED otherwise)
  *   e_f16   optional out fp16 [n][p][q][k], as x_f16 of iq_conv_fwd for the errors e: written

@@ -357,7 +357,7 @@ __global__ void k_scale_mul(const double* __restrict__ a, const double* __restri
 __global__ void k_max_from_stats(const int* __restrict__ hi, const int* __restrict__ lo, int C,
                                  int relu, const double* __restrict__ s_in,
                                  unsigned long long* __restrict__ cell, RqParams* __restrict__ prm,
-                                 double* __restrict__ s_out) {
+                                 double* __restrict__ s_out, int k = 8) {
     __shared__ unsigned long long red[32];
     uint64_t m = 0;
     for (int c = threadIdx.x; c < C; c += blockDim.x) {
@@ -377,7 +377,7 @@ __global__ void k_max_from_stats(const int* __restrict__ hi, const int* __restri
         r = warp_max_u64(r);
         if (threadIdx.x == 0) {
             *cell = r;
-            const RqParams p = rq_params_make(r, *s_in, 8, relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ);
+            const RqParams p = rq_params_make(r, *s_in, k, relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ);
             *prm = p;
             *s_out = p.s_out;
         }
@@ -394,9 +394,21 @@ static bool desc_ok(const iq_conv_desc* d) {
         d->dil_w <= 0 || d->groups <= 0)
         return false;
     if (d->c % d->groups || d->k % d->groups) return false;
+    if (d->layout != IQ_LAYOUT_NHWC && d->layout != IQ_LAYOUT_NCHW) return false;
+    if (d->k_w != 0 && (d->k_w < 2 || d->k_w > 8)) return false;
+    if (d->k_a != 0 && (d->k_a < 2 || d->k_a > 8)) return false;
     int p = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1);
     int q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1);
     return p >= 0 && q >= 0;
+}
+
+// the code widths of a descriptor (0: the paper's 8 bits)
+static int code_kw(const iq_conv_desc* d) { return d->k_w ? d->k_w : 8; }
+// Q_A width: the descriptor's, else the bits argument's (batch norm), else 8; -1 when both
+// are given and differ
+static int code_ka(const iq_conv_desc* d, const iq_bn_bits* bits) {
+    if (d->k_a && bits && bits->k_a != d->k_a) return -1;
+    return d->k_a ? d->k_a : (bits ? bits->k_a : 8);
 }
 
 static ConvP make_params(const iq_conv_desc* d) {
@@ -463,10 +475,13 @@ extern "C" iq_status iq_conv_out_size(const iq_conv_desc* d, int32_t* p, int32_t
     return IQ_OK;
 }
 
+// bytes of the NCHW staging buffers in front of the NHWC workspace (0 for NHWC)
+static size_t nchw_stage_bytes(const iq_conv_desc* d, int op);
+
 extern "C" iq_status iq_conv_fwd_workspace_size(const iq_conv_desc* d, int with_bn, size_t* bytes) {
     (void)with_bn;
     if (!desc_ok(d) || !bytes) return IQ_ERR_INVALID_ARG;
-    *bytes = fwd_ws_layout(d, 1, nullptr, 0, nullptr);
+    *bytes = fwd_ws_layout(d, 1, nullptr, 0, nullptr) + nchw_stage_bytes(d, 1);
     return IQ_OK;
 }
 
@@ -508,7 +523,7 @@ extern "C" iq_status iq_conv_dgrad_workspace_size(const iq_conv_desc* d, size_t*
     bn_stats_carve(cur, d->c);
     cur.take<char>(std::max({conv_dgrad_tc_ws_bytes(d), conv_dgrad_tc_stride2_ws_bytes(d),
                              dgrad_pad_ws(d)}));
-    *bytes = cur.off + 256;
+    *bytes = cur.off + 256 + nchw_stage_bytes(d, 2);
     return IQ_OK;
 }
 
@@ -519,7 +534,7 @@ extern "C" iq_status iq_conv_wgrad_workspace_size(const iq_conv_desc* d, size_t*
     cur.take<char>(requant_ws_bytes());
     cur.take<double>(1);
     cur.take<char>(conv_wgrad_tc_ws_bytes(d));
-    *bytes = cur.off + 256;
+    *bytes = cur.off + 256 + nchw_stage_bytes(d, 3);
     return IQ_OK;
 }
 
@@ -676,18 +691,21 @@ extern "C" iq_status iq_kernel_timing_end(iq_kernel_time* out, int32_t capacity,
     return r;
 }
 
-extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
-                                 const int8_t* w, const int32_t* gamma, const int32_t* beta,
-                                 const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
-                                 double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
-                                 int32_t* acc_out, void* x_f16, void* ws, size_t ws_bytes,
-                                 iq_stream stream) {
+static iq_status conv_fwd_nhwc(const iq_conv_desc* d, const int8_t* x, const double* s_x,
+                               const int8_t* w, const int32_t* gamma, const int32_t* beta,
+                               const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
+                               double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
+                               int32_t* acc_out, void* x_f16, void* ws, size_t ws_bytes,
+                               iq_stream stream) {
     if (!desc_ok(d) || !x || !s_x || !w || !a || !s_a) return IQ_ERR_INVALID_ARG;
     const int64_t nx = (int64_t)d->n * d->h * d->w * d->c;
     if (x_f16 && (nx % 16 || (((uintptr_t)x | (uintptr_t)x_f16) & 15))) return IQ_ERR_INVALID_ARG;
     if (crs_overflow(d)) return IQ_ERR_OVERFLOW_RISK;
     kt_set_op(1, conv_macs(d), conv_macs_dense(d));
     iq_bn_bits b = bn_bits_or_default(bits);
+    const int ka = code_ka(d, bits);
+    if (ka < 0) return IQ_ERR_INVALID_ARG;
+    b.k_a = ka;
     if (use_bn) {
         if (!gamma || !beta || !bn_bits_valid(b)) return IQ_ERR_INVALID_ARG;
         if (d->k % 4) return IQ_ERR_UNSUPPORTED;
@@ -706,7 +724,7 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
 
     iq_status r = bn_stats_init(L.st, cp.K, st);
     if (r != IQ_OK) return r;
-    k_scale_mul_pow2<<<1, 1, 0, st>>>(s_x, -7, L.s_acc);  // s_acc = s_x * 2^-7 (W_q step)
+    k_scale_mul_pow2<<<1, 1, 0, st>>>(s_x, 1 - code_kw(d), L.s_acc);  // s_acc = s_x 2^(1-k_w)
     IQ_LAUNCH_CHECK();
     bool done = false;
     if (x_f16) {
@@ -755,16 +773,16 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     // Q_A = SQ(act(acc), 8) with M from the per-channel extremes
     unsigned long long* cell = (unsigned long long*)L.rq;
     k_max_from_stats<<<1, 1024, 0, st>>>(L.st.hi, L.st.lo, cp.K, relu, L.s_acc, cell,
-                                         rq_params_slot(L.rq), s_a);
+                                         rq_params_slot(L.rq), s_a, ka);
     IQ_LAUNCH_CHECK();
-    return requant_apply(acc, IQ_I32, cp.npq * cp.K, L.s_acc, 8,
+    return requant_apply(acc, IQ_I32, cp.npq * cp.K, L.s_acc, ka,
                          relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ, 0, 0, 0, 0, a, IQ_I8, s_a, L.rq, st,
                          true);
 }
 
-extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
-                                   const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
-                                   void* e_f16, void* ws, size_t ws_bytes, iq_stream stream) {
+static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const double* s_e,
+                                 const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
+                                 void* e_f16, void* ws, size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d) || !e || !s_e || !w || !dx || !s_dx) return IQ_ERR_INVALID_ARG;
     const bool wide = dgrad_wide(d);
     if (wide && acc_out) return IQ_ERR_UNSUPPORTED;   // the sums need 64 bits: no int32 copy
@@ -787,7 +805,7 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     void* tcws = cur.take<char>(tcb);
     const int64_t total = (int64_t)d->n * d->h * d->w * d->c;
     unsigned long long* cell = (unsigned long long*)rq;
-    k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, -7, s_in);
+    k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, 1 - code_kw(d), s_in);   // the W_q step 2^(1-k_w)
     IQ_LAUNCH_CHECK();
     int32_t* acc = acc_out ? acc_out : reinterpret_cast<int32_t*>(accw);
     if (e_f16) {
@@ -893,11 +911,11 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
                          st);
 }
 
-extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
-                                   const int8_t* x, const double* s_x, int gq_mode, uint64_t seed,
-                                   uint64_t layer, uint64_t step, int8_t* g, double* s_g,
-                                   int64_t* g_acc_out, const void* e_f16, const void* x_f16,
-                                   void* ws, size_t ws_bytes, iq_stream stream) {
+static iq_status conv_wgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const double* s_e,
+                                 const int8_t* x, const double* s_x, int gq_mode, uint64_t seed,
+                                 uint64_t layer, uint64_t step, int8_t* g, double* s_g,
+                                 int64_t* g_acc_out, const void* e_f16, const void* x_f16,
+                                 void* ws, size_t ws_bytes, iq_stream stream) {
     if ((((uintptr_t)e_f16 | (uintptr_t)x_f16) & 15)) return IQ_ERR_INVALID_ARG;
     if (!desc_ok(d) || !e || !s_e || !x || !s_x || !g || !s_g) return IQ_ERR_INVALID_ARG;
     if (gq_mode != 1 && gq_mode != 2) return IQ_ERR_INVALID_ARG;
@@ -960,4 +978,205 @@ extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const
     kt_post(st, IQ_KERNEL_CONV_SIMT);
     return requant_int(G, IQ_I64, gn, s_in, 8, gq_mode == 1 ? IQ_MODE_RQ_GQ1 : IQ_MODE_RQ_GQ2,
                        seed, layer, step, 0, g, IQ_I8, s_g, rq, st);
+}
+
+// ==================================================================== NCHW layout
+// Sec. 3 states the problem without a memory layout; the kernels compute in NHWC (channels
+// innermost, the TMA boxes' contiguous dimension).  With IQ_LAYOUT_NCHW the entry points
+// transpose their activation / error inputs (NCHW -> NHWC) and filters (KCRS -> KRSC) into
+// the workspace, run the NHWC computation, and transpose the outputs back.
+
+namespace iq {
+namespace {
+
+// dst[b][c][r] = src[b][r][c] for b < gridDim.z: 32 x 32 tiles through shared memory
+template <typename T>
+__global__ void k_transpose_b(const T* __restrict__ src, T* __restrict__ dst, int64_t rows,
+                              int64_t cols) {
+    __shared__ T tile[32][33];
+    const int64_t off = (int64_t)blockIdx.z * rows * cols;
+    const int64_t r0 = (int64_t)blockIdx.y * 32, c0 = (int64_t)blockIdx.x * 32;
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int64_t r = r0 + i, c = c0 + threadIdx.x;
+        if (r < rows && c < cols) tile[i][threadIdx.x] = src[off + r * cols + c];
+    }
+    __syncthreads();
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int64_t c = c0 + i, r = r0 + threadIdx.x;
+        if (r < rows && c < cols) dst[off + c * rows + r] = tile[threadIdx.x][i];
+    }
+}
+
+iq_status transpose_b(const void* src, void* dst, int64_t batches, int64_t rows, int64_t cols,
+                      int esize, cudaStream_t st) {
+    if (batches < 1 || rows < 1 || cols < 1) return IQ_OK;
+    const int64_t gx = (cols + 31) / 32, gy = (rows + 31) / 32;
+    if (batches > 65535 || gy > 65535 || gx > 0x7fffffff) return IQ_ERR_UNSUPPORTED;
+    const dim3 grid((unsigned)gx, (unsigned)gy, (unsigned)batches), blk(32, 8);
+    switch (esize) {
+        case 1: k_transpose_b<int8_t><<<grid, blk, 0, st>>>((const int8_t*)src, (int8_t*)dst, rows, cols); break;
+        case 2: k_transpose_b<int16_t><<<grid, blk, 0, st>>>((const int16_t*)src, (int16_t*)dst, rows, cols); break;
+        case 4: k_transpose_b<int32_t><<<grid, blk, 0, st>>>((const int32_t*)src, (int32_t*)dst, rows, cols); break;
+        default: k_transpose_b<long long><<<grid, blk, 0, st>>>((const long long*)src, (long long*)dst, rows, cols); break;
+    }
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+// NCHW image tensor [n][c][hw] <-> NHWC [n][hw][c]
+iq_status to_nhwc(const void* src, void* dst, int64_t n, int64_t c, int64_t hw, int es,
+                  cudaStream_t st) {
+    return transpose_b(src, dst, n, c, hw, es, st);
+}
+iq_status to_nchw(const void* src, void* dst, int64_t n, int64_t c, int64_t hw, int es,
+                  cudaStream_t st) {
+    return transpose_b(src, dst, n, hw, c, es, st);
+}
+
+struct NchwWs {
+    size_t off_x, off_w, off_y, off_y16, off_acc, off_rest;
+};
+
+size_t al256(size_t v) { return (v + 255) / 256 * 256; }
+
+// the NCHW staging buffers of one call: input codes, filters, output codes (int8), int16
+// codes, sums (int64 bytes per element), then the NHWC computation's own workspace
+NchwWs nchw_layout(int64_t nin, int64_t nw, int64_t nout) {
+    NchwWs L;
+    L.off_x = 0;
+    L.off_w = L.off_x + al256((size_t)nin);
+    L.off_y = L.off_w + al256((size_t)nw);
+    L.off_y16 = L.off_y + al256((size_t)nout);
+    L.off_acc = L.off_y16 + al256((size_t)nout * 2);
+    L.off_rest = L.off_acc + al256((size_t)nout * 8);
+    return L;
+}
+
+void conv_sizes(const iq_conv_desc* d, int64_t* nin, int64_t* nw, int64_t* nout, int64_t* pq) {
+    const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+    const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+    *nin = (int64_t)d->n * d->h * d->w * d->c;
+    *nw = (int64_t)d->k * d->r * d->s * (d->c / d->groups);
+    *nout = (int64_t)d->n * P * Q * d->k;
+    *pq = (int64_t)P * Q;
+}
+
+}  // namespace
+}  // namespace iq
+
+extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
+                                 const int8_t* w, const int32_t* gamma, const int32_t* beta,
+                                 const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
+                                 double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
+                                 int32_t* acc_out, void* x_f16, void* ws, size_t ws_bytes,
+                                 iq_stream stream) {
+    if (!desc_ok(d)) return IQ_ERR_INVALID_ARG;
+    if (d->layout == IQ_LAYOUT_NHWC)
+        return conv_fwd_nhwc(d, x, s_x, w, gamma, beta, bits, use_bn, relu, a, s_a, xhat,
+                             bn_codes, bn_scales, acc_out, x_f16, ws, ws_bytes, stream);
+    if (!x || !s_x || !w || !a || !s_a) return IQ_ERR_INVALID_ARG;
+    int64_t nin, nw, nout, pq;
+    conv_sizes(d, &nin, &nw, &nout, &pq);
+    const NchwWs L = nchw_layout(nin, nw, nout);
+    if (!ws || ws_bytes < L.off_rest + 256) return IQ_ERR_WORKSPACE;
+    char* b = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
+    ws_bytes -= (size_t)(b - (char*)ws);
+    iq_conv_desc dn = *d;
+    dn.layout = IQ_LAYOUT_NHWC;
+    cudaStream_t st = (cudaStream_t)stream;
+    const int cg = d->c / d->groups;
+    iq_status r = to_nhwc(x, b + L.off_x, d->n, d->c, (int64_t)d->h * d->w, 1, st);
+    if (r == IQ_OK) r = transpose_b(w, b + L.off_w, d->k, cg, (int64_t)d->r * d->s, 1, st);
+    if (r != IQ_OK) return r;
+    int8_t* an = (int8_t*)(b + L.off_y);
+    int16_t* xn = xhat ? (int16_t*)(b + L.off_y16) : nullptr;
+    int32_t* accn = acc_out ? (int32_t*)(b + L.off_acc) : nullptr;
+    r = conv_fwd_nhwc(&dn, (const int8_t*)(b + L.off_x), s_x, (const int8_t*)(b + L.off_w), gamma,
+                      beta, bits, use_bn, relu, an, s_a, xn, bn_codes, bn_scales, accn, x_f16,
+                      b + L.off_rest, ws_bytes - L.off_rest, stream);
+    if (r != IQ_OK) return r;
+    r = to_nchw(an, a, d->n, d->k, pq, 1, st);
+    if (r == IQ_OK && xhat) r = to_nchw(xn, xhat, d->n, d->k, pq, 2, st);
+    if (r == IQ_OK && acc_out) r = to_nchw(accn, acc_out, d->n, d->k, pq, 4, st);
+    return r;
+}
+
+extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
+                                   const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
+                                   void* e_f16, void* ws, size_t ws_bytes, iq_stream stream) {
+    if (!desc_ok(d)) return IQ_ERR_INVALID_ARG;
+    if (d->layout == IQ_LAYOUT_NHWC)
+        return conv_dgrad_nhwc(d, e, s_e, w, dx, s_dx, acc_out, e_f16, ws, ws_bytes, stream);
+    if (!e || !s_e || !w || !dx || !s_dx) return IQ_ERR_INVALID_ARG;
+    int64_t nin, nw, nout, pq;
+    conv_sizes(d, &nin, &nw, &nout, &pq);
+    // staging: errors (the "input" slot holds nout codes), filters, dx codes and sums
+    const NchwWs L = nchw_layout(nout, nw, nin);
+    if (!ws || ws_bytes < L.off_rest + 256) return IQ_ERR_WORKSPACE;
+    char* b = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
+    ws_bytes -= (size_t)(b - (char*)ws);
+    iq_conv_desc dn = *d;
+    dn.layout = IQ_LAYOUT_NHWC;
+    cudaStream_t st = (cudaStream_t)stream;
+    const int cg = d->c / d->groups;
+    iq_status r = to_nhwc(e, b + L.off_x, d->n, d->k, pq, 1, st);
+    if (r == IQ_OK) r = transpose_b(w, b + L.off_w, d->k, cg, (int64_t)d->r * d->s, 1, st);
+    if (r != IQ_OK) return r;
+    int8_t* dxn = (int8_t*)(b + L.off_y);
+    int32_t* accn = acc_out ? (int32_t*)(b + L.off_acc) : nullptr;
+    r = conv_dgrad_nhwc(&dn, (const int8_t*)(b + L.off_x), s_e, (const int8_t*)(b + L.off_w), dxn,
+                        s_dx, accn, e_f16, b + L.off_rest, ws_bytes - L.off_rest, stream);
+    if (r != IQ_OK) return r;
+    const int64_t hw = (int64_t)d->h * d->w;
+    r = to_nchw(dxn, dx, d->n, d->c, hw, 1, st);
+    if (r == IQ_OK && acc_out) r = to_nchw(accn, acc_out, d->n, d->c, hw, 4, st);
+    return r;
+}
+
+extern "C" iq_status iq_conv_wgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
+                                   const int8_t* x, const double* s_x, int gq_mode, uint64_t seed,
+                                   uint64_t layer, uint64_t step, int8_t* g, double* s_g,
+                                   int64_t* g_acc_out, const void* e_f16, const void* x_f16,
+                                   void* ws, size_t ws_bytes, iq_stream stream) {
+    if (!desc_ok(d)) return IQ_ERR_INVALID_ARG;
+    if (d->layout == IQ_LAYOUT_NHWC)
+        return conv_wgrad_nhwc(d, e, s_e, x, s_x, gq_mode, seed, layer, step, g, s_g, g_acc_out,
+                               e_f16, x_f16, ws, ws_bytes, stream);
+    if (!e || !s_e || !x || !s_x || !g || !s_g) return IQ_ERR_INVALID_ARG;
+    int64_t nin, nw, nout, pq;
+    conv_sizes(d, &nin, &nw, &nout, &pq);
+    // staging: x in the input slot, e in the output-code slot (nout codes), gradient codes in
+    // the filter slot, int64 sums in the sum slot (nw <= the slot's elements is checked)
+    const int64_t nmax = nout > nw ? nout : nw;
+    const NchwWs L = nchw_layout(nin, nw, nmax);
+    if (!ws || ws_bytes < L.off_rest + 256) return IQ_ERR_WORKSPACE;
+    char* b = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
+    ws_bytes -= (size_t)(b - (char*)ws);
+    iq_conv_desc dn = *d;
+    dn.layout = IQ_LAYOUT_NHWC;
+    cudaStream_t st = (cudaStream_t)stream;
+    const int cg = d->c / d->groups;
+    iq_status r = to_nhwc(x, b + L.off_x, d->n, d->c, (int64_t)d->h * d->w, 1, st);
+    if (r == IQ_OK) r = to_nhwc(e, b + L.off_y, d->n, d->k, pq, 1, st);
+    if (r != IQ_OK) return r;
+    int8_t* gn = (int8_t*)(b + L.off_w);
+    int64_t* accn = g_acc_out ? (int64_t*)(b + L.off_acc) : nullptr;
+    r = conv_wgrad_nhwc(&dn, (const int8_t*)(b + L.off_y), s_e, (const int8_t*)(b + L.off_x),
+                        s_x, gq_mode, seed, layer, step, gn, s_g, accn, e_f16, x_f16,
+                        b + L.off_rest, ws_bytes - L.off_rest, stream);
+    if (r != IQ_OK) return r;
+    // KRSC -> KCRS per output channel
+    r = transpose_b(gn, g, d->k, (int64_t)d->r * d->s, cg, 1, st);
+    if (r == IQ_OK && g_acc_out)
+        r = transpose_b(accn, g_acc_out, d->k, (int64_t)d->r * d->s, cg, 8, st);
+    return r;
+}
+
+static size_t nchw_stage_bytes(const iq_conv_desc* d, int op) {
+    if (d->layout != IQ_LAYOUT_NCHW) return 0;
+    int64_t nin, nw, nout, pq;
+    iq::conv_sizes(d, &nin, &nw, &nout, &pq);
+    if (op == 1) return iq::nchw_layout(nin, nw, nout).off_rest + 256;
+    if (op == 2) return iq::nchw_layout(nout, nw, nin).off_rest + 256;
+    return iq::nchw_layout(nin, nw, nout > nw ? nout : nw).off_rest + 256;
 }

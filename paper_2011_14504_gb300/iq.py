@@ -56,7 +56,10 @@ class IqError(RuntimeError):
 class ConvDesc(C.Structure):
     _fields_ = [(n, C.c_int32) for n in
                 ("n", "h", "w", "c", "k", "r", "s", "stride_h", "stride_w", "pad_h", "pad_w",
-                 "dil_h", "dil_w", "groups")]
+                 "dil_h", "dil_w", "groups", "layout", "k_w", "k_a")]
+
+
+IQ_LAYOUT_NHWC, IQ_LAYOUT_NCHW = 0, 1
 
 
 class BnBits(C.Structure):
@@ -230,8 +233,12 @@ def _ws(nbytes: int, device) -> torch.Tensor:
     return torch.empty(max(int(nbytes), 1), dtype=torch.uint8, device=device)
 
 
-def conv_desc(n, h, w, c, k, r, s, stride=1, pad=0, dil=1, groups=1) -> ConvDesc:
-    return ConvDesc(n, h, w, c, k, r, s, stride, stride, pad, pad, dil, dil, groups)
+def conv_desc(n, h, w, c, k, r, s, stride=1, pad=0, dil=1, groups=1, layout=IQ_LAYOUT_NHWC,
+              k_w=0, k_a=0) -> ConvDesc:
+    """iq_conv_desc; layout IQ_LAYOUT_NCHW takes NCHW activations / errors and KCRS filters,
+    k_w / k_a the weight and activation code widths (0: 8 bits)."""
+    return ConvDesc(n, h, w, c, k, r, s, stride, stride, pad, pad, dil, dil, groups, layout, k_w,
+                    k_a)
 
 
 def bn_bits(k_mu=16, k_sigma=16, k_xhat=16, k_gamma=8, k_beta=8, k_a=8) -> BnBits:

@@ -53,6 +53,24 @@ def test_conv_out_size_and_workspace_queries(lib):
     assert iq.iq_conv_dgrad_workspace_size(d) >= 32 * 32 * 64 * 4
     assert iq.iq_conv_wgrad_workspace_size(d) >= 64 * 9 * 64 * 8
     assert iq.iq_bn_int_workspace_size(1024, 64) > 0
+    # NCHW calls stage their transposes in front of the NHWC workspace
+    dn = iq.conv_desc(1, 32, 32, 64, 64, 3, 3, 1, 1, layout=iq.IQ_LAYOUT_NCHW)
+    for f in (iq.iq_conv_fwd_workspace_size, iq.iq_conv_dgrad_workspace_size,
+              iq.iq_conv_wgrad_workspace_size):
+        assert f(dn) >= f(d) + 2 * 32 * 32 * 64
+
+
+def test_conv_desc_layout_and_widths_validated(lib):
+    """The descriptor's layout and code widths: NHWC / NCHW, k_w and k_a in 2..8 (0: 8 bits);
+    anything else is rejected by the host-side checks."""
+    ok = [dict(), dict(layout=iq.IQ_LAYOUT_NCHW), dict(k_w=4, k_a=4), dict(k_w=2, k_a=8)]
+    bad = [dict(layout=2), dict(layout=-1), dict(k_w=1), dict(k_w=9), dict(k_a=1), dict(k_a=16)]
+    for kw in ok:
+        assert iq.iq_conv_out_size(iq.conv_desc(1, 8, 8, 8, 8, 3, 3, 1, 1, **kw)) == (8, 8)
+    for kw in bad:
+        with pytest.raises(iq.IqError) as e:
+            iq.iq_conv_out_size(iq.conv_desc(1, 8, 8, 8, 8, 3, 3, 1, 1, **kw))
+        assert e.value.code == iq.IQ_ERR_INVALID_ARG
 
 
 def test_kernel_timing_host_side(lib):

@@ -88,7 +88,7 @@ def sq_exact_int(q, k, relu=False):
     return [clip(rhu_exact(Fr(v, M) * 2 ** (k - 1)), k) for v in q]
 
 
-@pytest.mark.parametrize("k", [8, 16])
+@pytest.mark.parametrize("k", [4, 8, 16])
 @pytest.mark.parametrize("relu", [False, True])
 def test_sq_int_matches_exact_rationals(k, relu):
     g = S.rng(11 + k + relu)
