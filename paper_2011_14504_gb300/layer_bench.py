@@ -1,8 +1,9 @@
 """Time one integer 3x3 convolution layer (stride 1, padding 1), or one integer L1BN,
-through the C ABI.
+through the C ABI; or run one step of a network once (a profiling target).
 
     python -m paper_2011_14504_gb300.layer_bench [N,H,C,K] [time|once]
     python -m paper_2011_14504_gb300.layer_bench bn M,C [time|once]
+    python -m paper_2011_14504_gb300.layer_bench step deeplab|fcn BATCH [train|infer]
 
 Runs iq_conv_fwd (with ReLU and the SQ8 requantisation of the output), iq_conv_dgrad and
 iq_conv_wgrad (GQ8 gradient) of an N x H x H x C -> K layer on random 8-bit codes.  "time"
@@ -69,10 +70,44 @@ def bn_main(argv):
     print("ok")
 
 
+def step_main(argv):
+    """Exactly one training step (or inference pass) of the full-width network on synthetic
+    inputs (batch BATCH, 513 x 513 or 512 x 512), no warm-up: under a profiler every launch
+    of the run belongs to that one step."""
+    import numpy as np
+    from . import synthetic as S
+    net_name, batch = argv[0], int(argv[1])
+    train = (argv[2] if len(argv) > 2 else "train") == "train"
+    g = S.rng(7)
+    if net_name == "deeplab":
+        from .deeplab import DeepLabV3R50
+        net = DeepLabV3R50(batch, 513, 513, classes=21, train=train)
+        img = torch.from_numpy(S.images_u8(g, batch, 513, 513)).cuda()
+        lab = torch.from_numpy(S.labels_uniform_ignore(g, batch, 513, 513, 21)).cuda()
+    else:
+        from .fcn import FcnVgg16
+        net = FcnVgg16(batch, 512, 512, classes=150, train=train)
+        img = torch.from_numpy(S.images_u8(g, batch, 512, 512)).cuda()
+        lab = torch.from_numpy(S.labels_voronoi(g, batch, 512, 512, 150)).cuda()
+    torch.cuda.synchronize()
+    l0 = iq.launch_count()
+    if train:
+        net.train_step(img, lab)
+    else:
+        net.forward(img)
+    torch.cuda.synchronize()
+    assert iq.iq_device_status() == 0
+    print(f"{net_name} batch {batch} {'train step' if train else 'inference'}: "
+          f"{iq.launch_count() - l0} library launches")
+    print("ok")
+
+
 def main(argv=None):
     argv = sys.argv[1:] if argv is None else argv
     if argv and argv[0] == "bn":
         return bn_main(argv[1:])
+    if argv and argv[0] == "step":
+        return step_main(argv[1:])
     n, h, c, k = [int(v) for v in (argv[0] if argv else "8,128,256,256").split(",")]
     mode = argv[1] if len(argv) > 1 else "time"
     dev = "cuda"
