@@ -108,12 +108,21 @@ unsigned long long iq_launch_count(void);
 /* iq_device_status -- the library's sticky device status (the paper has no counterpart).
  * Every wait inside the tensor-core convolution kernels is bounded (about one second); a
  * wait that gives up records a code (1: operand loads, 2: MMA issue, 3: epilogue, 4: a
- * TMA-fed producer), the kernel returns without completing its tiles, and every later
+ * TMA-fed producer, 5: iq_wait_selftest), the kernel returns without completing its tiles, and every later
  * launch of those kernels returns at once, so the outputs of that call and of all later
  * calls are not valid.  This call synchronizes `stream`, stores the code in *code (0 when
  * nothing gave up), clears it and returns IQ_ERR_TIMEOUT when it was set, else IQ_OK.
  * Call it after a sequence of calls (a training step) to learn whether they completed. */
 iq_status iq_device_status(int32_t* code, iq_stream stream);
+
+/* iq_wait_selftest -- a check of the bounded-wait path above (the paper has no counterpart).
+ * Enqueues on `stream` one kernel whose single thread makes the tensor-core kernels' bounded
+ * mbarrier wait, with a limit of limit_cycles SM cycles (0 .. 2^31), on a barrier that
+ * nothing arrives on.  The wait gives up, the kernel records code 5 in the sticky status and
+ * returns; nothing else is in flight.  The next iq_device_status returns IQ_ERR_TIMEOUT with
+ * code 5 and clears the status (until then the tensor-core convolution kernels return at
+ * once).  IQ_ERR_INVALID_ARG for a limit outside the range. */
+iq_status iq_wait_selftest(long long limit_cycles, iq_stream stream);
 
 /* Kernel timing -- a measurement aid (the paper has no counterpart).  Between
  * iq_kernel_timing_begin and iq_kernel_timing_end, every launch of a convolution kernel and

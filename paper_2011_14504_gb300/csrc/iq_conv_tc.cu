@@ -2019,8 +2019,6 @@ struct TmaTile {
 // every later launch of these kernels returns at once.
 __device__ int g_tc_status;
 
-std::mutex g_tc_status_mu;
-int* g_tc_status_ptr[256] = {};
 
 // int8 KRSC weights -> fp16 [K][kpad] (zero beyond R*S*C)
 // int8 KRSC weights -> fp16 [K][kpad] (zero beyond R*S*C): blocks (x, rows y, y + gridDim.y,
@@ -2088,17 +2086,12 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     return fn;
 }
 
-// device address of g_tc_status on the current device (looked up once per device)
+// device address of g_tc_status in the CUDA context current at the call (an address that
+// belongs to a context, not to a device ordinal: looked up on every call)
 int* tc_status_ptr() {
-    int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return nullptr;
-    std::lock_guard<std::mutex> lock(g_tc_status_mu);
-    if (!g_tc_status_ptr[dev]) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_tc_status) != cudaSuccess || !p) return nullptr;
-        g_tc_status_ptr[dev] = static_cast<int*>(p);
-    }
-    return g_tc_status_ptr[dev];
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_tc_status) != cudaSuccess || !p) return nullptr;
+    return static_cast<int*>(p);
 }
 
 bool tc_env_disabled() {
@@ -3114,6 +3107,34 @@ iq_status conv_wgrad_tc(const iq_conv_desc* d, const int8_t* e, const int8_t* x,
 }
 
 }  // namespace iq
+
+namespace iq {
+namespace {
+// One thread waits, with the bounded wait of the tensor-core kernels and a limit of `limit`
+// SM cycles, on an mbarrier that nothing arrives on; when the wait gives up it records code 5
+// in the sticky status, as a kernel whose wait expired does.  The thread issues no copies and
+// no MMAs, so nothing is in flight when it returns.
+__global__ void k_wait_selftest(int* err, long long limit) {
+    __shared__ uint64_t bar;
+    __shared__ int never;
+    if (threadIdx.x == 0) {
+        tc::mbar_init(&bar, 1);
+        never = 0;
+        tc::mbar_fence_init();
+        if (!tc::mbar_wait(&bar, 0, &never, limit)) atomicExch(err, 5);
+    }
+}
+}  // namespace
+}  // namespace iq
+
+extern "C" iq_status iq_wait_selftest(long long limit_cycles, iq_stream stream) {
+    if (limit_cycles < 0 || limit_cycles > (1LL << 31)) return IQ_ERR_INVALID_ARG;
+    int* p = iq::tc_status_ptr();
+    if (!p) return IQ_ERR_CUDA;
+    iq::k_wait_selftest<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(p, limit_cycles);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
 
 extern "C" iq_status iq_device_status(int32_t* code, iq_stream stream) {
     if (!code) return IQ_ERR_INVALID_ARG;

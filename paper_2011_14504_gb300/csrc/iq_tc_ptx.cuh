@@ -47,16 +47,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Bounded wait: spins until the phase with `parity` completed, the shared abort
-// word is set by another role, or 2^31 SM cycles (about one second) passed.
-// Returns false when it gave up; the caller then records the timeout and leaves.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+// word is set by another role, or `limit` SM cycles (by default 2^31, about one second)
+// passed.  Returns false when it gave up; the caller then records the timeout and leaves.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          long long limit = (1LL << 31)) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     for (uint32_t i = 1;; i++) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 255) == 0) {
             if (*abort) return false;
-            if (clock64() - t0 > (1LL << 31)) return false;
+            if (clock64() - t0 > limit) return false;
         }
     }
 }

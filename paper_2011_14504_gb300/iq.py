@@ -31,7 +31,7 @@ EXPORTS = [
     "iq_spatial_sum_workspace_size", "iq_spatial_sum", "iq_avgpool_bwd", "iq_channel_slice",
     "iq_bilinear_workspace_size", "iq_bilinear_up_fwd", "iq_bilinear_up_bwd", "iq_ce_grad",
     "iq_bn_update", "iq_device_status", "iq_rq_epoch_advance", "iq_rq_epoch_set",
-    "iq_kernel_timing_begin", "iq_kernel_timing_end",
+    "iq_kernel_timing_begin", "iq_kernel_timing_end", "iq_wait_selftest",
 ]
 IQ_KERNEL_CONV_PIXEL_MAJOR, IQ_KERNEL_CONV_CHANNEL_MAJOR, IQ_KERNEL_CONV_WGRAD = 1, 2, 3
 IQ_KERNEL_CONV_CPASYNC, IQ_KERNEL_CONV_GATHER, IQ_KERNEL_CONV_SIMT = 4, 5, 6
@@ -159,6 +159,7 @@ def load(path: str | None = None):
     L.iq_kernel_timing_end.argtypes = [C.POINTER(KernelTime), _I32, C.POINTER(_I32)]
     L.iq_rq_epoch_advance.argtypes = [_P]
     L.iq_rq_epoch_set.argtypes = [_U64, _P]
+    L.iq_wait_selftest.argtypes = [C.c_longlong, _P]
     for f in EXPORTS:
         if f not in ("iq_status_str", "iq_version", "iq_launch_count"):
             getattr(L, f).restype = _I
@@ -193,6 +194,12 @@ def iq_device_status(stream=None) -> int:
     code = _I32(0)
     _check("iq_device_status", load().iq_device_status(C.byref(code), _stream(stream)))
     return code.value
+
+
+def iq_wait_selftest(limit_cycles=1 << 20, stream=None):
+    """Enqueue the bounded-wait self-test kernel (its wait must give up: status code 5)."""
+    _check("iq_wait_selftest", load().iq_wait_selftest(C.c_longlong(limit_cycles),
+                                                       _stream(stream)))
 
 
 def iq_rq_epoch_advance(stream=None):

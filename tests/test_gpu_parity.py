@@ -647,3 +647,76 @@ def test_kernel_timing_brackets_the_conv_kernels():
     sq = bw[iq.IQ_KERNEL_SQ_CODES]
     assert sq["launches"] == 2 and sq["bytes"] == 5.0 * n * h * h * (k + c)
     assert iq.iq_kernel_timing_end() == []      # stopped: nothing recorded since
+
+
+# ----------------------------------------------------------------- routing of the conv kernels
+
+ROUTES = [
+    # (n, h, w, c, k, r, stride, pad, dil), operation, kernels its call launches
+    ((1, 7, 7, 256, 32, 7, 1, 3, 1), "fwd", {iq.IQ_KERNEL_CONV_CPASYNC}),
+    ((16, 1, 1, 2048, 256, 1, 1, 0, 1), "dgrad", {iq.IQ_KERNEL_CONV_CPASYNC}),
+    ((1, 13, 11, 16, 24, 3, 1, 1, 1), "fwd", {iq.IQ_KERNEL_CONV_GATHER}),
+    ((3, 9, 10, 64, 80, 1, 1, 0, 1), "dgrad", {iq.IQ_KERNEL_CONV_GATHER}),
+    ((1, 32, 40, 64, 128, 3, 1, 1, 1), "fwd", {iq.IQ_KERNEL_CONV_CHANNEL_MAJOR}),
+    ((2, 16, 16, 512, 256, 3, 1, 1, 1), "dgrad", {iq.IQ_KERNEL_CONV_PIXEL_MAJOR}),
+    ((2, 16, 16, 512, 256, 3, 1, 1, 1), "wgrad", {iq.IQ_KERNEL_CONV_WGRAD}),
+    ((2, 31, 29, 4, 64, 3, 1, 1, 1), "dgrad", {iq.IQ_KERNEL_CONV_SIMT}),
+]
+
+
+@pytest.mark.parametrize("ri", range(len(ROUTES)))
+def test_conv_kernel_routing(ri):
+    """Which kernel a call runs on, read from the library's kernel timing, and its result
+    against the oracle: every fallback of the tensor-core path (the cp.async-fed and the
+    register-gather kernels, the channel-major kernel) and the CUDA-core kernel is reached by
+    a shape of its own, so each one's parity is shown rather than assumed."""
+    (n, h, w, c, k, r, st, pd, dl), op, want = ROUTES[ri]
+    cv = O.Conv(n, h, w, c, k, r, r, st, pd, dl)
+    d = iq.conv_desc(n, h, w, c, k, r, r, st, pd, dl)
+    p, q = cv.pq
+    g = S.rng(1200 + ri)
+    x = S.int8_uniform(g, (n, h, w, c))
+    wq = O.requant_master(O.uq(S.he_weights(g, (k, r, r, c), c * r * r), 24)).astype(np.int8)
+    e = S.int8_uniform(g, (n, p, q, k))
+    iq.iq_kernel_timing_begin()
+    if op == "fwd":
+        acc = torch.empty((n, p, q, k), dtype=torch.int32, device=DEV)
+        a = torch.empty((n, p, q, k), dtype=torch.int8, device=DEV)
+        iq.iq_conv_fwd(d, dev(x), dscal(0.02), dev(wq), a, dscal(), relu=True, acc_out=acc)
+        got, ref = acc, O.conv_fwd(cv, x, wq)
+    elif op == "dgrad":
+        acc = torch.empty((n, h, w, c), dtype=torch.int32, device=DEV)
+        dx = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
+        iq.iq_conv_dgrad(d, dev(e), dscal(1e-5), dev(wq), dx, dscal(), acc_out=acc)
+        got, ref = acc, O.conv_dgrad(cv, e, wq)
+    else:
+        gacc = torch.empty(wq.shape, dtype=torch.int64, device=DEV)
+        gq = torch.empty(wq.shape, dtype=torch.int8, device=DEV)
+        iq.iq_conv_wgrad(d, dev(e), dscal(1e-5), dev(x), dscal(0.02), gq, dscal(), gq_mode=1,
+                         g_acc_out=gacc)
+        got, ref = gacc, O.conv_wgrad(cv, e, x)
+    torch.cuda.synchronize()
+    ran = {t["kernel"] for t in iq.iq_kernel_timing_end() if t["kernel"] in iq.CONV_KERNELS}
+    assert ran == want, (ROUTES[ri], ran)
+    assert np.array_equal(host(got), ref)
+
+
+def test_bounded_wait_gives_up_and_reports():
+    """The bounded mbarrier wait of the tensor-core kernels, on a barrier nothing arrives on
+    (iq_wait_selftest): it gives up after its limit, the sticky status reports code 5 once
+    (IQ_ERR_TIMEOUT) and is cleared, and the context stays usable: a tensor-core convolution
+    afterwards is exact."""
+    import ctypes as C
+    iq.iq_wait_selftest(1 << 20)
+    code = C.c_int32(0)
+    rc = iq.load().iq_device_status(C.byref(code), None)
+    assert rc == iq.IQ_ERR_TIMEOUT and code.value == 5
+    assert iq.iq_device_status() == 0
+    cv, d, x, w, _ = _conv_case(0, 77)
+    p, q = cv.pq
+    acc = torch.empty((cv.n, p, q, cv.k), dtype=torch.int32, device=DEV)
+    a = torch.empty((cv.n, p, q, cv.k), dtype=torch.int8, device=DEV)
+    iq.iq_conv_fwd(d, dev(x), dscal(0.01), dev(w), a, dscal(), relu=True, acc_out=acc)
+    assert np.array_equal(host(acc), O.conv_fwd(cv, x, w))
+    with pytest.raises(iq.IqError):
+        iq.iq_wait_selftest(-1)
