@@ -242,6 +242,10 @@ iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_
  *   xhat   out int16 [n][p][q][k], the X codes kept for backward (bn only, may be NULL)
  *   bn_codes  out device int32[2k]: mu_q codes then sigma_q codes (bn only, may be NULL)
  *   bn_scales out device double[IQ_BN_SCALES] (bn only, may be NULL)
+ *   frozen_out optional out device int64: the constants of this call's output map, for
+ *             iq_conv_fwd_frozen on later batches -- with bn, int64[4k + 2]: the fixed-point
+ *             F[k], B[k], G[k], H[k] of the acc -> X -> A maps and the shifts P_x, P_a; without
+ *             bn, int64[1]: M, the maximum of act(acc) that Q_A divided by
  *   acc_out   optional out int32 [n][p][q][k]: the raw accumulators
  *   x_f16     optional out fp16 [n][h][w][c] (16-byte aligned, n h w c % 16 == 0, else
  *             IQ_ERR_INVALID_ARG): the exact fp16 copy of the codes x (of their NHWC
@@ -254,8 +258,27 @@ iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_
 iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
                       const int8_t* w, const int32_t* gamma, const int32_t* beta,
                       const iq_bn_bits* bits, int use_bn, int relu, int8_t* a, double* s_a,
-                      int16_t* xhat, int32_t* bn_codes, double* bn_scales, int32_t* acc_out,
-                      void* x_f16, void* ws, size_t ws_bytes, iq_stream stream);
+                      int16_t* xhat, int32_t* bn_codes, double* bn_scales, int64_t* frozen_out,
+                      int32_t* acc_out, void* x_f16, void* ws, size_t ws_bytes,
+                      iq_stream stream);
+
+/* iq_conv_fwd_frozen -- the inference forward with frozen statistics.  The paper defines no
+ * running estimate for its L1BN (Sec. 3.2.2 normalises with the batch's own statistics, and
+ * Scale(x) of Eq. (ScaleQ) is the tensor's own maximum); this entry point is the stated
+ * deviation that makes a single-pass inference possible: the output map of an earlier
+ * iq_conv_fwd call on a calibration batch (its frozen_out) is applied to this batch.
+ *   with use_bn: X = clip(floor((F acc + B) / 2^P_x), +-(2^(k_xhat-1)-1)) with the product
+ *     in 128 bits, A = clip(floor((G X + H) / 2^P_a), 0, 2^(k_a-1)-1);
+ *   without: A = clip(floor((2^k_a act(acc) + M) / (2M))), act = ReLU when relu.
+ * The scales are the calibration call's (s_a, bn_scales), which the caller keeps; x must carry
+ * the calibration's input scale for the codes to mean the same values.  No statistics are
+ * taken and no scale is written.  Arguments as iq_conv_fwd; frozen int64[4k + 2] (use_bn)
+ * or int64[1]; bits: the calibration's (NULL: defaults); xhat optional (use_bn only).
+ * Workspace: iq_conv_fwd_workspace_size. */
+iq_status iq_conv_fwd_frozen(const iq_conv_desc* d, const int8_t* x, const int8_t* w,
+                             const int64_t* frozen, const iq_bn_bits* bits, int use_bn,
+                             int relu, int8_t* a, int16_t* xhat, void* x_f16, void* ws,
+                             size_t ws_bytes, iq_stream stream);
 
 /* iq_conv_dgrad -- error of the layer input (Sec. 3.3.1, Eq. (EQ)):
  * dx = conv_transpose(e, w) in exact int32, then E_1 = SQ(dx, 8).

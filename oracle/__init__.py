@@ -106,6 +106,8 @@ def _declare(L):
                             _P, C.POINTER(C.c_double), _P, _P]
     L.or_bn_bwd.restype = _I32
     L.or_relu_bwd.argtypes = [_I64, _P, _P, _P]
+    L.or_bn_apply_fixed.argtypes = [_I64, _I32, _P, _P, _P, _P, _P, _I32, _I32, _I32, _I32, _P,
+                                    _P]
     L.or_update.argtypes = [_I64, _P, _P, _P, _D, _I32, _I32, _I32, _I32]
     L.or_quantize_image_u8.argtypes = [_P, _I64, _I32, _I32, _P]
     L.or_quantize_image_u8.restype = _D
@@ -366,6 +368,20 @@ def bn_fwd(acc, s_acc: float, gamma_codes, beta_codes, k_mu=16, k_sigma=16, k_xh
     if rc != 0:
         raise ValueError("or_bn_fwd: empty input")
     return BnResult(X, A, cm, cs, F, B, G, H, o.s_xhat, o.s_a, o.m_xhat, o.m_y, o.p_x, o.p_a)
+
+
+def bn_apply_fixed(acc, F, B, G, H, p_x: int, p_a: int, k_xhat=16, k_a=8):
+    """The L1BN element maps with constants fixed by an earlier call (frozen statistics):
+    returns (X, A) for accumulators acc[m, C]."""
+    acc = _c(acc, np.int32)
+    C_ = acc.shape[-1]
+    m = acc.size // C_
+    F, B, G, H = (_c(v, np.int64) for v in (F, B, G, H))
+    X = np.empty(acc.shape, np.int16)
+    A = np.empty(acc.shape, np.int8)
+    lib().or_bn_apply_fixed(m, C_, _ptr(acc), _ptr(F), _ptr(B), _ptr(G), _ptr(H), p_x, p_a,
+                            k_xhat, k_a, _ptr(X), _ptr(A))
+    return X, A
 
 
 def bn_bwd(eA, s_e: float, A, X, s_x: float, gamma_codes, c_sigma, k_sigma=16, k_gamma=8,

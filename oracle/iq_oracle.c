@@ -663,6 +663,29 @@ int or_bn_fwd(int64_t m, int32_t C, const int32_t* acc, double s_acc,
     return 0;
 }
 
+/* The element maps of the L1BN forward with constants fixed by an earlier
+ * call (F, B, G, H per channel and the shifts px, pa that or_bn_fwd returns
+ * for a calibration batch): the inference mode with frozen statistics, a
+ * reading of the paper's L1BN at inference (it defines no running estimate).
+ * X = clip(floor((F acc + B) / 2^px)), A = clip(floor((G X + H) / 2^pa), 0,
+ * 2^(k_a-1)-1), the products in 128 bits (an accumulator beyond the
+ * calibration range cannot overflow them). */
+void or_bn_apply_fixed(int64_t m, int32_t C, const int32_t* acc, const int64_t* F,
+                       const int64_t* B, const int64_t* G, const int64_t* H, int px,
+                       int pa, int k_xhat, int k_a, int16_t* X, int8_t* A) {
+    const int64_t xq = qmax(k_xhat), aq = qmax(k_a);
+    for (int64_t i = 0; i < m; i++)
+        for (int c = 0; c < C; c++) {
+            i128 t = (i128)F[c] * acc[i * C + c] + B[c];
+            i128 xs = t >> px;
+            int64_t xc = xs < -xq ? -xq : (xs > xq ? xq : (int64_t)xs);
+            if (X) X[i * C + c] = (int16_t)xc;
+            i128 u = (i128)G[c] * xc + H[c];
+            i128 as = u >> pa;
+            A[i * C + c] = (int8_t)(as < 0 ? 0 : (as > aq ? aq : (int64_t)as));
+        }
+}
+
 /* ------------------------------------------------------------------ */
 /* Sec. 3.3: backward through ReLU and quantized L1BN                   */
 /* ------------------------------------------------------------------ */

@@ -467,6 +467,89 @@ __global__ void __launch_bounds__(kThreads) k_bn_requant(const int32_t* __restri
     if (r < m) row(r * C4 + g, a4[r * C4 + g]);
 }
 
+// ------------------------------------------------------------------ frozen statistics
+// The element maps of the forward pass with constants fixed by an earlier call (fixed =
+// F[C], B[C], G[C], H[C], P_x, P_a): X = clip(floor((F acc + B) / 2^P_x)) with the product in
+// 128 bits (an accumulator beyond the calibration range cannot overflow it), A = clip(floor((G
+// X + H) / 2^P_a), 0, aq) (|X| <= 2^15 keeps the second map within int64 by the choice of P_a).
+
+// floor((F v + B) / 2^px) clipped to [-q, q], t = F v + B exact in 128 bits, 1 <= px <= 62
+__device__ __forceinline__ int64_t map128_clip(long long F, int v, long long B, int px,
+                                               int64_t q) {
+    const long long lo = F * (long long)v;                       // low 64 bits
+    long long hi = __mul64hi(F, (long long)v);                   // signed high 64 bits
+    const unsigned long long l2 = (unsigned long long)lo + (unsigned long long)B;
+    hi += (long long)(l2 < (unsigned long long)lo) + (B < 0 ? -1LL : 0LL);
+    const unsigned long long rl = (l2 >> px) | ((unsigned long long)hi << (64 - px));
+    const long long rh = hi >> px;                               // the shifted value rh:rl
+    if (rh > 0) return q;
+    if (rh == 0) return rl > (unsigned long long)q ? q : (int64_t)rl;
+    if (rh < -1) return -q;
+    const long long vv = (long long)rl;                          // rh == -1
+    return (vv >= 0 || vv < -q) ? -q : vv;
+}
+
+__global__ void __launch_bounds__(kThreads) k_bn_apply_fixed(const int32_t* __restrict__ acc,
+                                                             int64_t m, int32_t C,
+                                                             const int64_t* __restrict__ fx,
+                                                             int kx, int ka,
+                                                             int16_t* __restrict__ X,
+                                                             int8_t* __restrict__ A) {
+    const int C4 = C >> 2;
+    const int64_t T = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)(t % C4);
+    const int64_t rstride = T / C4;
+    const int px = (int)fx[4 * (int64_t)C], pa = (int)fx[4 * (int64_t)C + 1];
+    const int64_t xq = qmax(kx), aq = qmax(ka);
+    long long F[4], B[4], G[4], H[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        F[j] = fx[4 * g + j]; B[j] = fx[C + 4 * g + j];
+        G[j] = fx[2 * C + 4 * g + j]; H[j] = fx[3 * C + 4 * g + j];
+    }
+    const int4* a4 = reinterpret_cast<const int4*>(acc);
+    auto row = [&](int64_t v, const int4 in) {
+        const int vs[4] = {in.x, in.y, in.z, in.w};
+        int xo[4];
+        uint32_t ao = 0;
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            const int64_t xc = map128_clip(F[j], vs[j], B[j], px, xq);
+            xo[j] = (int)xc;
+            const long long ta = G[j] * xc + H[j];
+            const int64_t ac = clamp64(ta >> pa, 0, aq);
+            ao |= ((uint32_t)ac & 0xffu) << (8 * j);
+        }
+        if (X) {
+            uint2 xv;
+            xv.x = ((uint32_t)(uint16_t)xo[0]) | ((uint32_t)(uint16_t)xo[1] << 16);
+            xv.y = ((uint32_t)(uint16_t)xo[2]) | ((uint32_t)(uint16_t)xo[3] << 16);
+            reinterpret_cast<uint2*>(X)[v] = xv;
+        }
+        reinterpret_cast<uint32_t*>(A)[v] = ao;
+    };
+    int64_t r = t / C4;
+    for (; r + rstride < m; r += 2 * rstride) {
+        const int64_t v0 = r * C4 + g, v1 = (r + rstride) * C4 + g;
+        const int4 in0 = a4[v0], in1 = a4[v1];
+        row(v0, in0);
+        row(v1, in1);
+    }
+    if (r < m) row(r * C4 + g, a4[r * C4 + g]);
+}
+
+iq_status bn_apply_fixed(const int32_t* acc, int64_t m, int32_t C, const int64_t* fixed, int kx,
+                         int ka, int16_t* X, int8_t* A, cudaStream_t st) {
+    if (m == 0) return IQ_OK;
+    ChanGrid g2 = chan_grid(m, C / 4, 152 * 16);
+    kt_pre(st);
+    k_bn_apply_fixed<<<g2.blocks, kThreads, 0, st>>>(acc, m, C, fixed, kx, ka, X, A);
+    IQ_LAUNCH_CHECK();
+    kt_post_bytes(st, IQ_KERNEL_BN_REQUANT, (double)m * C * (X ? 7.0 : 5.0));
+    return IQ_OK;
+}
+
 __global__ void k_bn_export(BnStats s, int32_t C, const int32_t* __restrict__ codes_ws,
                             double* __restrict__ s_a, int32_t* __restrict__ bn_codes,
                             double* __restrict__ bn_scales, int64_t* __restrict__ bn_fixed) {

@@ -695,8 +695,8 @@ static iq_status conv_fwd_nhwc(const iq_conv_desc* d, const int8_t* x, const dou
                                const int8_t* w, const int32_t* gamma, const int32_t* beta,
                                const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
                                double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
-                               int32_t* acc_out, void* x_f16, void* ws, size_t ws_bytes,
-                               iq_stream stream) {
+                               int64_t* frozen_out, int32_t* acc_out, void* x_f16, void* ws,
+                               size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d) || !x || !s_x || !w || !a || !s_a) return IQ_ERR_INVALID_ARG;
     const int64_t nx = (int64_t)d->n * d->h * d->w * d->c;
     if (x_f16 && (nx % 16 || (((uintptr_t)x | (uintptr_t)x_f16) & 15))) return IQ_ERR_INVALID_ARG;
@@ -769,15 +769,101 @@ static iq_status conv_fwd_nhwc(const iq_conv_desc* d, const int8_t* x, const dou
     }
     if (use_bn)
         return bn_fwd_after_stats(acc, cp.M, cp.K, L.s_acc, gamma, beta, b, L.st, xhat, a, s_a,
-                                  bn_codes, bn_scales, nullptr, st);
+                                  bn_codes, bn_scales, frozen_out, st);
     // Q_A = SQ(act(acc), 8) with M from the per-channel extremes
     unsigned long long* cell = (unsigned long long*)L.rq;
     k_max_from_stats<<<1, 1024, 0, st>>>(L.st.hi, L.st.lo, cp.K, relu, L.s_acc, cell,
                                          rq_params_slot(L.rq), s_a, ka);
     IQ_LAUNCH_CHECK();
+    if (frozen_out)      // M, the maximum of act(acc) Q_A divides by
+        IQ_CUDA_CHECK(cudaMemcpyAsync(frozen_out, cell, sizeof(int64_t), cudaMemcpyDeviceToDevice,
+                                      st));
     return requant_apply(acc, IQ_I32, cp.npq * cp.K, L.s_acc, ka,
                          relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ, 0, 0, 0, 0, a, IQ_I8, s_a, L.rq, st,
                          true);
+}
+
+// frozen Q_A parameters from the calibration maximum M = frozen[0]
+__global__ void k_frozen_sq_params(const int64_t* __restrict__ frozen, int k, int relu,
+                                   RqParams* __restrict__ prm) {
+    const int64_t M = frozen[0];
+    *prm = rq_params_make(M > 0 ? (uint64_t)M : 0, 1.0, k, relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ);
+}
+
+// The inference forward with frozen statistics: the conv into int32 accumulators (no
+// statistics), then the calibration call's output map in one pass.
+static iq_status conv_fwd_frozen_nhwc(const iq_conv_desc* d, const int8_t* x, const int8_t* w,
+                                      const int64_t* frozen, const iq_bn_bits* bits, int use_bn,
+                                      int relu, int8_t* a, int16_t* xhat, void* x_f16, void* ws,
+                                      size_t ws_bytes, iq_stream stream) {
+    if (!desc_ok(d) || !x || !w || !frozen || !a) return IQ_ERR_INVALID_ARG;
+    const int64_t nx = (int64_t)d->n * d->h * d->w * d->c;
+    if (x_f16 && (nx % 16 || (((uintptr_t)x | (uintptr_t)x_f16) & 15))) return IQ_ERR_INVALID_ARG;
+    if (crs_overflow(d)) return IQ_ERR_OVERFLOW_RISK;
+    iq_bn_bits b = bn_bits_or_default(bits);
+    const int ka = code_ka(d, bits);
+    if (ka < 0) return IQ_ERR_INVALID_ARG;
+    b.k_a = ka;
+    if (use_bn) {
+        if (!bn_bits_valid(b)) return IQ_ERR_INVALID_ARG;
+        if (d->k % 4) return IQ_ERR_UNSUPPORTED;
+        if (((uintptr_t)a | (uintptr_t)xhat) & 15) return IQ_ERR_INVALID_ARG;
+    } else if (xhat) {
+        return IQ_ERR_INVALID_ARG;
+    }
+    kt_set_op(1, conv_macs(d), conv_macs_dense(d));
+    cudaStream_t st = (cudaStream_t)stream;
+    FwdWs L;
+    size_t need = fwd_ws_layout(d, 1, nullptr, 0, nullptr);
+    if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
+    fwd_ws_layout(d, 1, ws, ws_bytes, &L);
+    int32_t* acc = L.acc;
+    ConvP cp = make_params(d);
+    cp.M = cp.npq;
+    cp.ncols = cp.Kg;
+    cp.kin = (int)roundup(cp.Cg, BK);
+    if (x_f16) {
+        iq_status r = codes_to_f16(x, (__half*)x_f16, nx, st);
+        if (r != IQ_OK) return r;
+    }
+    const int kp = fwd_kpad(d);
+    iq_status r = bn_stats_init(L.st, kp ? kp : cp.K, st);
+    if (r != IQ_OK) return r;
+    bool done = false;
+    if (kp) {
+        iq_conv_desc dp = *d;
+        dp.k = kp;
+        const int64_t rsc = (int64_t)d->r * d->s * d->c;
+        k_pad_cols_i8<<<grid_for((int64_t)kp * rsc), kThreads, 0, st>>>(w, 1, (int)(d->k * rsc),
+                                                                         (int)(kp * rsc), L.wp);
+        IQ_LAUNCH_CHECK();
+        r = conv_fwd_tc(&dp, x, L.wp, L.accp, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done,
+                        (const __half*)x_f16, TC_STATS_NOEXT);
+        if (r != IQ_OK) return r;
+        if (done) {
+            k_compact_cols_i32<<<grid_for(cp.npq * cp.K), kThreads, 0, st>>>(L.accp, cp.npq, cp.K,
+                                                                            kp, acc);
+            IQ_LAUNCH_CHECK();
+        }
+    } else {
+        r = conv_fwd_tc(d, x, w, acc, L.st.s1, L.st.hi, L.st.lo, L.tc, st, &done,
+                        (const __half*)x_f16, TC_STATS_NOEXT);
+        if (r != IQ_OK) return r;
+    }
+    if (!done) {
+        dim3 grid((unsigned)((cp.M + BM - 1) / BM), (unsigned)((cp.ncols + BN - 1) / BN), cp.G);
+        kt_pre(st);
+        k_conv_simt<OP_FWD, false><<<grid, 256, 0, st>>>(cp, x, w, acc, nullptr, L.st.s1, L.st.hi,
+                                                  L.st.lo, nullptr);
+        IQ_LAUNCH_CHECK();
+        kt_post(st, IQ_KERNEL_CONV_SIMT);
+    }
+    if (use_bn) return bn_apply_fixed(acc, cp.M, cp.K, frozen, b.k_xhat, b.k_a, xhat, a, st);
+    k_frozen_sq_params<<<1, 1, 0, st>>>(frozen, ka, relu, rq_params_slot(L.rq));
+    IQ_LAUNCH_CHECK();
+    return requant_apply(acc, IQ_I32, cp.npq * cp.K, L.s_acc, ka,
+                         relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ, 0, 0, 0, 0, a, IQ_I8, L.s_acc, L.rq,
+                         st, true);
 }
 
 static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const double* s_e,
@@ -1068,12 +1154,13 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
                                  const int8_t* w, const int32_t* gamma, const int32_t* beta,
                                  const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
                                  double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
-                                 int32_t* acc_out, void* x_f16, void* ws, size_t ws_bytes,
-                                 iq_stream stream) {
+                                 int64_t* frozen_out, int32_t* acc_out, void* x_f16, void* ws,
+                                 size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d)) return IQ_ERR_INVALID_ARG;
     if (d->layout == IQ_LAYOUT_NHWC)
         return conv_fwd_nhwc(d, x, s_x, w, gamma, beta, bits, use_bn, relu, a, s_a, xhat,
-                             bn_codes, bn_scales, acc_out, x_f16, ws, ws_bytes, stream);
+                             bn_codes, bn_scales, frozen_out, acc_out, x_f16, ws, ws_bytes,
+                             stream);
     if (!x || !s_x || !w || !a || !s_a) return IQ_ERR_INVALID_ARG;
     int64_t nin, nw, nout, pq;
     conv_sizes(d, &nin, &nw, &nout, &pq);
@@ -1092,8 +1179,8 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     int16_t* xn = xhat ? (int16_t*)(b + L.off_y16) : nullptr;
     int32_t* accn = acc_out ? (int32_t*)(b + L.off_acc) : nullptr;
     r = conv_fwd_nhwc(&dn, (const int8_t*)(b + L.off_x), s_x, (const int8_t*)(b + L.off_w), gamma,
-                      beta, bits, use_bn, relu, an, s_a, xn, bn_codes, bn_scales, accn, x_f16,
-                      b + L.off_rest, ws_bytes - L.off_rest, stream);
+                      beta, bits, use_bn, relu, an, s_a, xn, bn_codes, bn_scales, frozen_out,
+                      accn, x_f16, b + L.off_rest, ws_bytes - L.off_rest, stream);
     if (r != IQ_OK) return r;
     r = to_nchw(an, a, d->n, d->k, pq, 1, st);
     if (r == IQ_OK && xhat) r = to_nchw(xn, xhat, d->n, d->k, pq, 2, st);
@@ -1179,4 +1266,38 @@ static size_t nchw_stage_bytes(const iq_conv_desc* d, int op) {
     if (op == 1) return iq::nchw_layout(nin, nw, nout).off_rest + 256;
     if (op == 2) return iq::nchw_layout(nout, nw, nin).off_rest + 256;
     return iq::nchw_layout(nin, nw, nout > nw ? nout : nw).off_rest + 256;
+}
+
+extern "C" iq_status iq_conv_fwd_frozen(const iq_conv_desc* d, const int8_t* x, const int8_t* w,
+                                        const int64_t* frozen, const iq_bn_bits* bits,
+                                        int use_bn, int relu, int8_t* a, int16_t* xhat,
+                                        void* x_f16, void* ws, size_t ws_bytes,
+                                        iq_stream stream) {
+    if (!desc_ok(d)) return IQ_ERR_INVALID_ARG;
+    if (d->layout == IQ_LAYOUT_NHWC)
+        return conv_fwd_frozen_nhwc(d, x, w, frozen, bits, use_bn, relu, a, xhat, x_f16, ws,
+                                    ws_bytes, stream);
+    if (!x || !w || !a) return IQ_ERR_INVALID_ARG;
+    int64_t nin, nw, nout, pq;
+    iq::conv_sizes(d, &nin, &nw, &nout, &pq);
+    const iq::NchwWs L = iq::nchw_layout(nin, nw, nout);
+    if (!ws || ws_bytes < L.off_rest + 256) return IQ_ERR_WORKSPACE;
+    char* b = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
+    ws_bytes -= (size_t)(b - (char*)ws);
+    iq_conv_desc dn = *d;
+    dn.layout = IQ_LAYOUT_NHWC;
+    cudaStream_t st = (cudaStream_t)stream;
+    iq_status r = iq::to_nhwc(x, b + L.off_x, d->n, d->c, (int64_t)d->h * d->w, 1, st);
+    if (r == IQ_OK)
+        r = iq::transpose_b(w, b + L.off_w, d->k, d->c / d->groups, (int64_t)d->r * d->s, 1, st);
+    if (r != IQ_OK) return r;
+    int8_t* an = (int8_t*)(b + L.off_y);
+    int16_t* xn = xhat ? (int16_t*)(b + L.off_y16) : nullptr;
+    r = conv_fwd_frozen_nhwc(&dn, (const int8_t*)(b + L.off_x), (const int8_t*)(b + L.off_w),
+                             frozen, bits, use_bn, relu, an, xn, x_f16, b + L.off_rest,
+                             ws_bytes - L.off_rest, stream);
+    if (r != IQ_OK) return r;
+    r = iq::to_nchw(an, a, d->n, d->k, pq, 1, st);
+    if (r == IQ_OK && xhat) r = iq::to_nchw(xn, xhat, d->n, d->k, pq, 2, st);
+    return r;
 }

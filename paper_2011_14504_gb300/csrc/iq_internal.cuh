@@ -78,6 +78,10 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
                              int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
                              cudaStream_t st);
 
+// the forward's element maps with frozen constants (F, B, G, H, P_x, P_a from an earlier call)
+iq_status bn_apply_fixed(const int32_t* acc, int64_t m, int32_t C, const int64_t* fixed, int kx,
+                         int ka, int16_t* X, int8_t* A, cudaStream_t st);
+
 inline iq_bn_bits bn_bits_or_default(const iq_bn_bits* b) {
     if (b) return *b;
     iq_bn_bits d;

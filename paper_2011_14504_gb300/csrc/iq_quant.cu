@@ -135,11 +135,14 @@ __global__ void k_rq_finalize(const unsigned long long* __restrict__ cell,
 }
 
 // SQ: code = floor((2^k (q + M) + M) / (2M)) - 2^(k-1), the non-negative shift of
-// floor((2^k q + M) / (2M)); the numerator is < 2^(k+1) M + M < 2^57.
+// floor((2^k q + M) / (2M)); the numerator is < 2^(k+1) M + M < 2^57.  q is first clipped to
+// [-M, M], which changes no code (both ends already give +-(2^(k-1) - 1)) and keeps the
+// numerator non-negative when M is a frozen maximum that this tensor exceeds.
 __device__ __forceinline__ int64_t sq_code(int64_t v, const RqParams& p, int k, int relu,
                                            int64_t lim) {
     if (relu && v < 0) v = 0;
     if (!p.M) return 0;
+    v = clamp64(v, -(int64_t)p.M, (int64_t)p.M);
     uint64_t num = ((uint64_t)(v + (int64_t)p.M) << k) + p.M;
     return clamp64((int64_t)udiv(num, p.div) - (int64_t(1) << (k - 1)), -lim, lim);
 }
@@ -151,6 +154,8 @@ __device__ __forceinline__ int64_t sq_code(int64_t v, const RqParams& p, int k, 
 // sides below 2^41).  Clipping to +-127 is q in [1, 255]; the code byte is q ^ 0x80.
 __device__ __forceinline__ uint32_t sq8_byte(int v, uint32_t M, uint32_t R8, int relu) {
     if (relu && v < 0) v = 0;
+    // v clipped to [-M, M]: no code changes, u stays in [0, 2M] (M = 2^31 bounds every int32)
+    if (M < 0x80000000u) v = min(max(v, -(int)M), (int)M);
     const uint32_t u = (uint32_t)v + M;
     const uint32_t t = __umulhi(u, R8);
     const uint64_t rhs = (uint64_t)u << 8;
@@ -214,6 +219,7 @@ __global__ void k_sq_int(const T* __restrict__ q, int64_t n, int k, int relu,
         if (relu && v < 0) v = 0;
         int64_t c = 0;
         if (p.M) {
+            v = clamp64(v, -(int64_t)p.M, (int64_t)p.M);
             uint64_t num = ((uint64_t)(v + (int64_t)p.M) << k) + p.M;
             c = (int64_t)udiv(num, p.div) - (int64_t(1) << (k - 1));
             c = clamp64(c, -lim, lim);

@@ -31,7 +31,7 @@ EXPORTS = [
     "iq_spatial_sum_workspace_size", "iq_spatial_sum", "iq_avgpool_bwd", "iq_channel_slice",
     "iq_bilinear_workspace_size", "iq_bilinear_up_fwd", "iq_bilinear_up_bwd", "iq_ce_grad",
     "iq_bn_update", "iq_device_status", "iq_rq_epoch_advance", "iq_rq_epoch_set",
-    "iq_kernel_timing_begin", "iq_kernel_timing_end", "iq_wait_selftest",
+    "iq_kernel_timing_begin", "iq_kernel_timing_end", "iq_wait_selftest", "iq_conv_fwd_frozen",
 ]
 IQ_KERNEL_CONV_PIXEL_MAJOR, IQ_KERNEL_CONV_CHANNEL_MAJOR, IQ_KERNEL_CONV_WGRAD = 1, 2, 3
 IQ_KERNEL_CONV_CPASYNC, IQ_KERNEL_CONV_GATHER, IQ_KERNEL_CONV_SIMT = 4, 5, 6
@@ -118,7 +118,9 @@ def load(path: str | None = None):
                                 _SZ, _P]
     L.iq_weight_requant.argtypes = [_P, _P, _I64, _I, _I, _P]
     L.iq_conv_fwd.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, C.POINTER(BnBits), _I, _I,
-                              _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
+                              _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
+    L.iq_conv_fwd_frozen.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, C.POINTER(BnBits), _I, _I,
+                                     _P, _P, _P, _P, _SZ, _P]
     L.iq_conv_dgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
     L.iq_conv_wgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _I, _U64, _U64, _U64, _P, _P,
                                 _P, _P, _P, _P, _SZ, _P]
@@ -326,15 +328,27 @@ def iq_weight_requant(master, wq, k_u=24, k_w=8, stream=None):
 
 
 def iq_conv_fwd(d: ConvDesc, x, s_x, w, a, s_a, gamma=None, beta=None, bits=None, use_bn=False,
-                relu=True, xhat=None, bn_codes=None, bn_scales=None, acc_out=None, x_f16=None,
-                ws=None, stream=None):
+                relu=True, xhat=None, bn_codes=None, bn_scales=None, frozen_out=None, acc_out=None,
+                x_f16=None, ws=None, stream=None):
     if ws is None:
         ws = _ws(iq_conv_fwd_workspace_size(d, use_bn), x.device)
     _check("iq_conv_fwd",
            load().iq_conv_fwd(C.byref(d), _p(x), _p(s_x), _p(w), _p(gamma), _p(beta),
                               C.byref(bits) if bits is not None else None, int(use_bn),
                               int(relu), _p(a), _p(s_a), _p(xhat), _p(bn_codes), _p(bn_scales),
-                              _p(acc_out), _p(x_f16), _p(ws), ws.numel(), _stream(stream)))
+                              _p(frozen_out), _p(acc_out), _p(x_f16), _p(ws), ws.numel(),
+                              _stream(stream)))
+
+
+def iq_conv_fwd_frozen(d: ConvDesc, x, w, frozen, a, use_bn=False, relu=True, bits=None,
+                       xhat=None, x_f16=None, ws=None, stream=None):
+    if ws is None:
+        ws = _ws(iq_conv_fwd_workspace_size(d, use_bn), x.device)
+    _check("iq_conv_fwd_frozen",
+           load().iq_conv_fwd_frozen(C.byref(d), _p(x), _p(w), _p(frozen),
+                                     C.byref(bits) if bits is not None else None, int(use_bn),
+                                     int(relu), _p(a), _p(xhat), _p(x_f16), _p(ws), ws.numel(),
+                                     _stream(stream)))
 
 
 def iq_conv_dgrad(d: ConvDesc, e, s_e, w, dx, s_dx, acc_out=None, e_f16=None, ws=None,

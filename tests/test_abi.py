@@ -93,20 +93,20 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert e.value.code == iq.IQ_ERR_INVALID_ARG
     d = iq.conv_desc(1, 8, 8, 8, 8, 3, 3, 1, 1)
     rc = lib.iq_conv_fwd(C.byref(d), None, None, None, None, None, None, 0, 1, None, None, None,
-                         None, None, None, None, None, 0, None)
+                         None, None, None, None, None, None, 0, None)
     assert rc == iq.IQ_ERR_INVALID_ARG
     # a shape beyond the int32 accumulation bound: 1024*12*12*127^2 >= 2^31
     big = iq.conv_desc(1, 12, 12, 1024, 8, 12, 12)
     rc = lib.iq_conv_fwd(C.byref(big), 1, 1, 1, None, None, None, 0, 1, 1, 1, None, None, None,
-                         None, None, None, 0, None)
+                         None, None, None, None, 0, None)
     assert rc == iq.IQ_ERR_OVERFLOW_RISK
     # workspace too small
     rc = lib.iq_conv_fwd(C.byref(d), 1, 1, 1, None, None, None, 0, 1, 1, 1, None, None, None,
-                         None, None, None, 16, None)
+                         None, None, None, None, 16, None)
     assert rc == iq.IQ_ERR_WORKSPACE
     # an fp16 carrier that is not 16-byte aligned
     rc = lib.iq_conv_fwd(C.byref(d), 16, 1, 1, None, None, None, 0, 1, 1, 1, None, None, None,
-                         None, 24, None, 1 << 30, None)
+                         None, None, 24, None, 1 << 30, None)
     assert rc == iq.IQ_ERR_INVALID_ARG
     # bad bit width / dtype combination
     rc = lib.iq_quantize(1, 10, 16, iq.IQ_MODE_UQ, iq.IQ_I8, 1, 1, 1, 4096, None)
