@@ -145,9 +145,10 @@ enum {
     IQ_KERNEL_CONV_SIMT = 6,           /* CUDA-core kernel (k_conv_simt)                         */
     IQ_KERNEL_BN_DEV = 10,             /* L1BN deviation pass (k_bn_dev)                         */
     IQ_KERNEL_BN_REQUANT = 11,         /* L1BN acc -> X -> A pass (k_bn_requant)                 */
-    IQ_KERNEL_BNB_PASS1 = 12,          /* L1BN backward passes (k_bnb_pass1..3)                  */
-    IQ_KERNEL_BNB_PASS2 = 13,
-    IQ_KERNEL_BNB_PASS3 = 14,
+    IQ_KERNEL_BNB_PASS1 = 12,          /* L1BN backward: max |e_y gamma| pass (k_bnb_max_s), or
+                                          the one-pass histogram (k_bnb_hist) for other C      */
+    IQ_KERNEL_BNB_PASS2 = 13,          /* L1BN backward sums pass (k_bnb_sums_s)                 */
+    IQ_KERNEL_BNB_PASS3 = 14,          /* L1BN backward output pass (k_bnb_out_s, k_bnb_p3w)     */
     IQ_KERNEL_COMBINE_MAX = 15,        /* iq_combine, max |z| pass                               */
     IQ_KERNEL_COMBINE_CODES = 16,      /* iq_combine, codes pass                                 */
     IQ_KERNEL_SQ_CODES = 17,           /* SQ codes of int32 / int64 sums (k_sq_i32_i8x4, k_sq_int) */
@@ -356,7 +357,10 @@ iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_t c, const 
  *   e = SQ(dx, 8), the conv-output error fed to iq_conv_dgrad / iq_conv_wgrad.
  *   e_a, s_e   int8 [m][c] error codes of this layer's activation and their scale
  *   a, xhat    the forward outputs;  gamma int32[c];  bn_codes, bn_scales from the forward
- *   e          out int8 [m][c];  s_e_out out device double */
+ *   e          out int8 [m][c];  s_e_out out device double
+ * Workspace: iq_bn_int_workspace_size(m, c) (for c not a power of two in [16, 1024] nor a
+ * multiple of 1024 it grows with m: a per-code histogram of each row tile).  Returns
+ * IQ_ERR_UNSUPPORTED for m > 65535 * 65536 rows. */
 iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const int8_t* a,
                         const int16_t* xhat, int64_t m, int32_t c, const int32_t* gamma,
                         const int32_t* bn_codes, const double* bn_scales,

@@ -8,6 +8,7 @@
 // add into global integer accumulators (order-independent, hence deterministic).
 // Loads are 16 bytes (4 int32 accumulators, or 4 int8 / int16 codes).
 #include "iq_internal.cuh"
+#include "iq_stream.cuh"
 
 #include <climits>
 
@@ -467,6 +468,134 @@ __global__ void __launch_bounds__(kThreads) k_bn_requant(const int32_t* __restri
     if (r < m) row(r * C4 + g, a4[r * C4 + g]);
 }
 
+// ------------------------------------------------------------------ streamed forward passes
+// The deviation and requantization passes over row chunks staged in shared memory by bulk
+// copies (iq_stream.cuh); the arithmetic is that of k_bn_dev / k_bn_requant.
+
+// |v - f| for int32 v and f: below 2^32, exact in 32-bit unsigned arithmetic
+__device__ __forceinline__ uint32_t absdiff_u32(int v, int f) {
+    return v >= f ? (uint32_t)v - (uint32_t)f : (uint32_t)f - (uint32_t)v;
+}
+
+__global__ void __launch_bounds__(kStreamThreads, 1) k_bn_dev_s(RowStream rs, BnStats s,
+                                                                  int* __restrict__ err) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    if (__syncthreads_or(threadIdx.x == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    const int CB4 = rs.CB >> 2;
+    const int g = threadIdx.x % CB4, rl = threadIdx.x / CB4;
+    const int c0 = blockIdx.x * rs.CB + 4 * g;
+    int f[4];                        // floor(S1 / m): a mean of int32 values, so int32
+#pragma unroll
+    for (int j = 0; j < 4; j++) f[j] = (int)floordiv_i64((int64_t)s.s1[c0 + j], rs.m);
+    unsigned long long d[4] = {0, 0, 0, 0}, n[4] = {0, 0, 0, 0};
+    int hi[4] = {INT_MIN, INT_MIN, INT_MIN, INT_MIN}, lo[4] = {INT_MAX, INT_MAX, INT_MAX, INT_MAX};
+    const bool ok = stream_chunks(rs, smem, err, [&](const uint8_t* st, int rows, int64_t) {
+        const int4* v4 = reinterpret_cast<const int4*>(st);
+#pragma unroll
+        for (int u = 0; u < kStreamRPT; u++) {
+            const int r = rl + u * rs.RL;
+            if (r >= rows) break;
+            const int4 v = v4[r * CB4 + g];
+            const int vs[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                d[j] += absdiff_u32(vs[j], f[j]);
+                n[j] += vs[j] > f[j];
+                hi[j] = max(hi[j], vs[j]);
+                lo[j] = min(lo[j], vs[j]);
+            }
+        }
+    });
+    if (!ok) return;
+    // the row lanes of each channel, through shared memory (the stages are free now)
+    unsigned long long* sd = reinterpret_cast<unsigned long long*>(smem);    // [RL][CB]
+    unsigned long long* sn = sd + kStreamThreads * 4;
+    int* sh = reinterpret_cast<int*>(sn + kStreamThreads * 4);
+    int* sl = sh + kStreamThreads * 4;
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        const int i = rl * rs.CB + 4 * g + j;
+        sd[i] = d[j]; sn[i] = n[j]; sh[i] = hi[j]; sl[i] = lo[j];
+    }
+    __syncthreads();
+    for (int col = threadIdx.x; col < rs.CB; col += blockDim.x) {
+        unsigned long long td = 0, tn = 0;
+        int th = INT_MIN, tl = INT_MAX;
+        for (int i = 0; i < rs.RL; i++) {
+            const int k = i * rs.CB + col;
+            td += sd[k]; tn += sn[k]; th = max(th, sh[k]); tl = min(tl, sl[k]);
+        }
+        const int c = blockIdx.x * rs.CB + col;
+        atomicAdd(&s.dev[c], td);
+        atomicAdd(&s.ngt[c], tn);
+        if (th >= tl) {
+            atomicMax(&s.hi[c], th);
+            atomicMin(&s.lo[c], tl);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kStreamThreads, 1) k_bn_requant_s(RowStream rs, BnStats s,
+                                                                      int kx, int ka,
+                                                                      int16_t* __restrict__ X,
+                                                                      int8_t* __restrict__ A,
+                                                                      int* __restrict__ err) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    if (__syncthreads_or(threadIdx.x == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    const int CB4 = rs.CB >> 2;
+    const int g = threadIdx.x % CB4, rl = threadIdx.x / CB4;
+    const int c0 = blockIdx.x * rs.CB + 4 * g;
+    const int px = s.px[0], pa = s.px[1];
+    const int64_t xq = qmax(kx), aq = qmax(ka);
+    long long F[4], B[4], G[4], H[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        F[j] = s.F[c0 + j]; B[j] = s.B[c0 + j];
+        G[j] = s.G[c0 + j]; H[j] = s.H[c0 + j];
+    }
+    stream_chunks(rs, smem, err, [&](const uint8_t* st, int rows, int64_t r0) {
+        const int4* v4 = reinterpret_cast<const int4*>(st);
+#pragma unroll
+        for (int u = 0; u < kStreamRPT; u++) {
+            const int r = rl + u * rs.RL;
+            if (r >= rows) break;
+            const int4 v = v4[r * CB4 + g];
+            const int vs[4] = {v.x, v.y, v.z, v.w};
+            int xo[4];
+            uint32_t ao = 0;
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                const long long tx = F[j] * (long long)vs[j] + B[j];
+                const int64_t xc = clamp64(tx >> px, -xq, xq);
+                xo[j] = (int)xc;
+                const long long ta = G[j] * xc + H[j];
+                const int64_t ac = clamp64(ta >> pa, 0, aq);
+                ao |= ((uint32_t)ac & 0xffu) << (8 * j);
+            }
+            const int64_t e = (r0 + r) * rs.C + c0;      // element index of channel c0
+            if (X) {
+                uint2 xv;
+                xv.x = ((uint32_t)(uint16_t)xo[0]) | ((uint32_t)(uint16_t)xo[1] << 16);
+                xv.y = ((uint32_t)(uint16_t)xo[2]) | ((uint32_t)(uint16_t)xo[3] << 16);
+                *reinterpret_cast<uint2*>(X + e) = xv;
+            }
+            *reinterpret_cast<uint32_t*>(A + e) = ao;
+        }
+    });
+}
+
+// the streamed kernels' dynamic shared memory, set once per kernel
+template <class K>
+iq_status stream_attr(K kernel, bool& done) {
+    if (!done) {
+        IQ_CUDA_CHECK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)(kStreamStages * kStreamElems * 4 +
+                                                 2 * kStreamStages * sizeof(uint64_t))));
+        done = true;
+    }
+    return IQ_OK;
+}
+
 // ------------------------------------------------------------------ frozen statistics
 // The element maps of the forward pass with constants fixed by an earlier call (fixed =
 // F[C], B[C], G[C], H[C], P_x, P_a): X = clip(floor((F acc + B) / 2^P_x)) with the product in
@@ -574,9 +703,23 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
                              const BnStats& s, int16_t* xhat, int8_t* a, double* s_a,
                              int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
                              cudaStream_t st) {
-    RowGrid rg = row_grid(m, C / 4);
+    RowStream rs;
+    const void* srcs[1] = {acc};
+    const int esz[1] = {4};
+    const bool streamed = row_stream_plan(rs, m, C, srcs, esz, 1);
+    int* err = device_status_ptr();
+    if (!err) return IQ_ERR_CUDA;
     kt_pre(st);
-    k_bn_dev<<<rg.grid, kThreads, 0, st>>>(acc, m, C, rg.cg, s);
+    if (streamed) {
+        static bool attr = false;
+        iq_status r = stream_attr(k_bn_dev_s, attr);
+        if (r != IQ_OK) return r;
+        k_bn_dev_s<<<row_stream_grid(rs, device_sms()), kStreamThreads, row_stream_smem(rs), st>>>(
+            rs, s, err);
+    } else {
+        RowGrid rg = row_grid(m, C / 4);
+        k_bn_dev<<<rg.grid, kThreads, 0, st>>>(acc, m, C, rg.cg, s);
+    }
     IQ_LAUNCH_CHECK();
     kt_post_bytes(st, IQ_KERNEL_BN_DEV, 4.0 * (double)m * C);
     const int fb = (C + kFinThreads - 1) / kFinThreads;
@@ -590,9 +733,17 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
     IQ_LAUNCH_CHECK();
     k_bn_fin5<<<fb, kFinThreads, 0, st>>>(s, C, s_acc, gamma, beta, b);
     IQ_LAUNCH_CHECK();
-    ChanGrid g2 = chan_grid(m, C / 4, 152 * 16);
     kt_pre(st);
-    k_bn_requant<<<g2.blocks, kThreads, 0, st>>>(acc, m, C, s, b.k_xhat, b.k_a, xhat, a);
+    if (streamed) {
+        static bool attr = false;
+        iq_status r = stream_attr(k_bn_requant_s, attr);
+        if (r != IQ_OK) return r;
+        k_bn_requant_s<<<row_stream_grid(rs, device_sms()), kStreamThreads, row_stream_smem(rs),
+                         st>>>(rs, s, b.k_xhat, b.k_a, xhat, a, err);
+    } else {
+        ChanGrid g2 = chan_grid(m, C / 4, 152 * 16);
+        k_bn_requant<<<g2.blocks, kThreads, 0, st>>>(acc, m, C, s, b.k_xhat, b.k_a, xhat, a);
+    }
     IQ_LAUNCH_CHECK();
     kt_post_bytes(st, IQ_KERNEL_BN_REQUANT, (double)m * C * (xhat ? 7.0 : 5.0));
     k_bn_export<<<(C + 255) / 256, 256, 0, st>>>(s, C, s.codes, s_a, bn_codes, bn_scales,
@@ -602,21 +753,36 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
 }
 
 // ==================================================================== backward
-// pass 1: e_y = e_a [a > 0]; per channel sum e_y, sum e_y X; max |e_y gamma|
+// hist  : e_y = e_a [a > 0]; per channel the histogram of the nonzero e_y codes (count and
+//         sum of X per code), sum sign X, the extreme e_y of each sign class of X, and
+//         max |e_y gamma|
 // fin 1 : E_2 = SQ_{k_e2}(e_y gamma) constants
-// pass 2: per channel sum E_2, sum E_2 X, sum sign X; E_2 extremes per sign class
+// hfin  : per channel sum e_y, sum e_y X, sum E_2, sum E_2 X and the E_2 extremes per sign
+//         class, all exactly from the histogram (below)
 // fin 2 : d x_i = w_c (E_2 + kap_c sgn + lam_c); M = max |d x|; fixed-point SQ8 map
 // pass 3: e = clip(floor((fw E_2 + fk sgn + fl) / 2^P))
+//
+// E_2 = SQ(e_y gamma) divides by the tensor-wide maximum of |e_y gamma|, which is known only
+// after every element has been read; but per channel E_2 is a function of the 8-bit code e_y
+// alone.  So one pass over the elements gathers, per channel and code v, the count n_v and
+// the sum S_v of X over the elements with e_y = v, and every sum of Sec. 3.3.1's backward
+// statistics follows exactly: sum e_y = sum_v v n_v, sum e_y X = sum_v v S_v, sum E_2 =
+// sum_v E_2(v) n_v, sum E_2 X = sum_v E_2(v) S_v (E_2(0) = 0, so code 0 needs no bin).
+// E_2(v) = SQ(v gamma_c) is monotone in v, so the E_2 extremes of a sign class of X are E_2
+// at the class's extreme codes.
 
 // Division by 2M for E_2 = SQ(z, k_e2): the numerator 2^k (z + M) + M is below 2^32 for the
 // paper's widths (|z| <= 127 * 127, k_e2 <= 16), where a 32-bit invariant divisor (Granlund
 // & Montgomery, Sec. 4, at N = 32) replaces the 64-bit one.
-// Per channel, E_2 depends on e_y alone and the output code on (sign X, e_y) alone, so
-// both are tabulated once per call (k_bnb_tab2 / k_bnb_tab3, the same arithmetic as the
-// per-element form) and passes 2 and 3 look them up in shared memory.
-constexpr int kTab2 = 256;          // entries per channel: e_y + 128
+// Per channel the output code depends on (sign X, e_y) alone, so it is tabulated once per
+// call (k_bnb_tab3, the same arithmetic as the per-element form) and pass 3 looks it up in
+// shared memory.
 constexpr int kTab3 = 3 * 256;      // (sign X + 1) 256 + e_y + 128
-constexpr int kTabCG = 8;           // channel groups (32 channels) per block of passes 2 / 3
+constexpr int kTab3P = kTab3 + 4;   // a table row in shared memory, padded by one word
+constexpr int kTabCG = 8;           // channel groups (32 channels) per block of pass 3
+constexpr int kHistCh = 32;         // channels per block of the histogram pass
+constexpr int kHistRows = 65536;    // rows per block at most: |S_v| < 2^15 2^16 in int32
+constexpr int kHistSmem = 2 * kHistCh * 256 * (int)sizeof(int);
 
 struct E2Div {
     uint64_t M;
@@ -640,6 +806,7 @@ struct BnBwd {
     unsigned* zmax;           // [1]
     int* pe;                  // [1]
     E2Div* e2div;             // [1]
+    int2* hist;               // [gy][C][256]: per row tile of the histogram pass, (n_v, S_v)
     int16_t* t2;              // [C][256]: E_2 of e_y = -128 .. 127
     int8_t* t3;               // [C][3][256]: the output code of (sign X, e_y)
     double* scal;             // [2]: s_e2, s_out
@@ -649,7 +816,25 @@ struct BnBwd {
     unsigned long long* red;  // [4]: maxima of non-negative doubles (bit patterns)
 };
 
-static BnBwd bnb_carve(WsCursor& cur, int32_t C) {
+// row tiles of the histogram pass: about three blocks per SM, at most kHistRows rows each
+static int hist_tiles(int64_t m, int32_t C) {
+    const int64_t gx = (C + kHistCh - 1) / kHistCh;
+    int64_t gy = (152 * 3 + gx - 1) / gx;
+    const int64_t by_rows = (m + 31) / 32;
+    if (gy > by_rows) gy = by_rows;
+    const int64_t need = (m + kHistRows - 1) / kHistRows;
+    if (gy < need) gy = need;
+    if (gy < 1) gy = 1;
+    return (int)gy;
+}
+
+// the channel counts of the streamed / tiled backward passes: row_stream_plan's, and whole
+// 64-channel slabs
+static bool bnb_fast(int32_t C) {
+    return ((C >= 64 && C <= 1024 && (C & (C - 1)) == 0) || (C > 1024 && C % 1024 == 0));
+}
+
+static BnBwd bnb_carve(WsCursor& cur, int64_t m, int32_t C) {
     BnBwd w;
     w.sb = cur.take<unsigned long long>(C);
     w.sg = cur.take<unsigned long long>(C);
@@ -669,8 +854,10 @@ static BnBwd bnb_carve(WsCursor& cur, int32_t C) {
     w.lam = cur.take<double>(C);
     w.wc = cur.take<double>(C);
     w.red = cur.take<unsigned long long>(4);
-    w.t2 = cur.take<int16_t>((size_t)kTab2 * C);
     w.t3 = cur.take<int8_t>((size_t)kTab3 * C);
+    w.t2 = cur.take<int16_t>((size_t)256 * C);
+    // the histogram pass runs only where the row streamer does not
+    w.hist = cur.take<int2>(bnb_fast(C) && m < (int64_t(1) << 31) ? 0 : (size_t)hist_tiles(m, C) * C * 256);
     return w;
 }
 
@@ -694,70 +881,115 @@ __device__ __forceinline__ void load4_e_a_x(int64_t v, const int8_t* ea, const i
     x[2] = (int)(int16_t)(xv.y & 0xffffu); x[3] = (int)(int16_t)(xv.y >> 16);
 }
 
-// sum e_y and sum e_y X per channel (e_y = e_a [A > 0]), max |e_y gamma|
-__global__ void __launch_bounds__(kThreads) k_bnb_pass1(const int8_t* __restrict__ ea,
-                                                        const int8_t* __restrict__ a,
-                                                        const int16_t* __restrict__ X,
-                                                        const int32_t* __restrict__ gam,
-                                                        int64_t m, int32_t C, int CG, BnBwd w) {
-    __shared__ long long sh_b[kThreads * 4], sh_g[kThreads * 4];
+// The histogram pass.  A block is 8 channel groups (32 channels) x 32 row lanes; each
+// thread reads 4 channels of a row (the e_a and activation codes, the X codes).  The block
+// keeps (n_v, S_v) of its 32 channels in shared memory (shared-memory atomics, for nonzero
+// codes only) and writes them to its row tile's slab of the scratch histogram; the sign
+// sums and the per-class extreme codes (four channels packed in the bytes of a word,
+// byte-wise SIMD maxima / minima) are reduced over the warp and added atomically.
+__global__ void __launch_bounds__(kThreads, 3) k_bnb_hist(const int8_t* __restrict__ ea,
+                                                          const int8_t* __restrict__ a,
+                                                          const int16_t* __restrict__ X,
+                                                          const int32_t* __restrict__ gam,
+                                                          int64_t m, int32_t C, BnBwd w) {
+    extern __shared__ int hsm[];                 // [2][32][256]: n_v, then S_v
+    for (int i = threadIdx.x; i < 2 * kHistCh * 256; i += blockDim.x) hsm[i] = 0;
+    __syncthreads();
     const int C4 = C >> 2;
-    const int cg = threadIdx.x % CG, rl = threadIdx.x / CG, RL = blockDim.x / CG;
-    const int g = blockIdx.x * CG + cg;
+    const int lane = threadIdx.x & 31;
+    const int cg = threadIdx.x & 7, rl = threadIdx.x >> 3;
+    const int g = blockIdx.x * 8 + cg;
     const bool act = g < C4;
-    int gm[4] = {0, 0, 0, 0};
+    int ss[4] = {0, 0, 0, 0};
+    // extreme e_y per sign class of X (-, 0, +); empty: max 0x80 < min 0x7f
+    uint32_t mx[3] = {0x80808080u, 0x80808080u, 0x80808080u};
+    uint32_t mn[3] = {0x7f7f7f7fu, 0x7f7f7f7fu, 0x7f7f7f7fu};
     if (act) {
-#pragma unroll
-        for (int j = 0; j < 4; j++) gm[j] = gam[4 * g + j];
-    }
-    long long sb[4] = {0, 0, 0, 0}, sg[4] = {0, 0, 0, 0};
-    uint32_t zm = 0;
-    const int64_t step = (int64_t)gridDim.y * RL;
-    if (act) {
-        int64_t r = (int64_t)blockIdx.y * RL + rl;
-        // two rows per iteration: both rows' loads are in flight together
-        for (; r + step < m; r += 2 * step) {
-            int e0[4], a0[4], x0[4], e1[4], a1[4], x1[4];
-            load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
-            load4_e_a_x((r + step) * C4 + g, ea, a, X, e1, a1, x1);
+        int* hn = hsm + 4 * cg * 256 + 128;      // channel 4 cg, code 0
+        int* hs = hn + kHistCh * 256;
+        auto row = [&](const uint32_t ev, const uint32_t av, const uint2 xv) {
+            const uint32_t ey = ev & __vcmpgts4(av, 0u);
+            const int x[4] = {(int)(int16_t)(xv.x & 0xffffu), (int)xv.x >> 16,
+                              (int)(int16_t)(xv.y & 0xffffu), (int)xv.y >> 16};
+            uint32_t neg = 0u, pos = 0u;
 #pragma unroll
             for (int j = 0; j < 4; j++) {
-                const int ey0 = a0[j] > 0 ? e0[j] : 0, ey1 = a1[j] > 0 ? e1[j] : 0;
-                sb[j] += ey0 + ey1;
-                sg[j] += (long long)(ey0 * x0[j]) + (long long)(ey1 * x1[j]);   // |ey X| < 2^22
-                const int z0 = ey0 * gm[j], z1 = ey1 * gm[j];
-                zm = max(zm, max((uint32_t)abs(z0), (uint32_t)abs(z1)));
+                neg |= x[j] < 0 ? 0xffu << (8 * j) : 0u;
+                pos |= x[j] > 0 ? 0xffu << (8 * j) : 0u;
+                ss[j] += (x[j] > 0) - (x[j] < 0);
+                const int v = (int)(int8_t)(ey >> (8 * j));
+                if (v) {
+                    atomicAdd(hn + j * 256 + v, 1);
+                    atomicAdd(hs + j * 256 + v, x[j]);
+                }
             }
+            const uint32_t cls[3] = {neg, ~(neg | pos), pos};
+#pragma unroll
+            for (int q = 0; q < 3; q++) {
+                mx[q] = __vmaxs4(mx[q], (ey & cls[q]) | (0x80808080u & ~cls[q]));
+                mn[q] = __vmins4(mn[q], (ey & cls[q]) | (0x7f7f7f7fu & ~cls[q]));
+            }
+        };
+        const uint32_t* e4 = reinterpret_cast<const uint32_t*>(ea);
+        const uint32_t* a4 = reinterpret_cast<const uint32_t*>(a);
+        const uint2* x4 = reinterpret_cast<const uint2*>(X);
+        const int64_t step = (int64_t)gridDim.y * 32;
+        int64_t r = (int64_t)blockIdx.y * 32 + rl;
+        // two rows per iteration: both rows' loads in flight together
+        for (; r + step < m; r += 2 * step) {
+            const int64_t v0 = r * C4 + g, v1 = (r + step) * C4 + g;
+            const uint32_t e0 = __ldg(e4 + v0), a0 = __ldg(a4 + v0);
+            const uint2 x0 = __ldg(x4 + v0);
+            const uint32_t e1 = __ldg(e4 + v1), a1 = __ldg(a4 + v1);
+            const uint2 x1 = __ldg(x4 + v1);
+            row(e0, a0, x0);
+            row(e1, a1, x1);
         }
         if (r < m) {
-            int e0[4], a0[4], x0[4];
-            load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
+            const int64_t v0 = r * C4 + g;
+            row(__ldg(e4 + v0), __ldg(a4 + v0), __ldg(x4 + v0));
+        }
+    }
+    // the warp's four row lanes of each channel group: lanes cg, cg + 8, cg + 16, cg + 24
 #pragma unroll
-            for (int j = 0; j < 4; j++) {
-                const int ey0 = a0[j] > 0 ? e0[j] : 0;
-                sb[j] += ey0;
-                sg[j] += (long long)(ey0 * x0[j]);
-                zm = max(zm, (uint32_t)abs(ey0 * gm[j]));
+    for (int o = 8; o < 32; o <<= 1) {
+#pragma unroll
+        for (int j = 0; j < 4; j++) ss[j] += __shfl_xor_sync(0xffffffffu, ss[j], o);
+#pragma unroll
+        for (int q = 0; q < 3; q++) {
+            mx[q] = __vmaxs4(mx[q], __shfl_xor_sync(0xffffffffu, mx[q], o));
+            mn[q] = __vmins4(mn[q], __shfl_xor_sync(0xffffffffu, mn[q], o));
+        }
+    }
+    uint32_t zm = 0;
+    if (lane < 8 && act) {
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            const int c = 4 * g + j;
+            if (ss[j]) atomicAdd(&w.ss[c], (unsigned long long)(long long)ss[j]);
+            int amax = 0;
+#pragma unroll
+            for (int q = 0; q < 3; q++) {
+                const int hi = (int)(int8_t)(mx[q] >> (8 * j)), lo = (int)(int8_t)(mn[q] >> (8 * j));
+                if (lo > hi) continue;           // no element of this class
+                atomicMin(&w.emin[3 * c + q], lo);
+                atomicMax(&w.emax[3 * c + q], hi);
+                amax = max(amax, max(abs(lo), abs(hi)));
             }
+            zm = max(zm, (uint32_t)amax * (uint32_t)abs(gam[c]));
         }
     }
     zm = warp_max_u32(zm);
-    if ((threadIdx.x & 31) == 0 && zm) atomicMax(w.zmax, zm);
-#pragma unroll
-    for (int j = 0; j < 4; j++) {
-        sh_b[rl * CG * 4 + 4 * cg + j] = sb[j];
-        sh_g[rl * CG * 4 + 4 * cg + j] = sg[j];
-    }
+    if (lane == 0 && zm) atomicMax(w.zmax, zm);
     __syncthreads();
-    const int col = threadIdx.x;                 // one channel of the block's 4 CG
-    if (col < CG * 4) {
-        const int c = 4 * blockIdx.x * CG + col;
-        if (c < C) {
-            long long tb = 0, tg = 0;
-            for (int i = 0; i < RL; i++) { tb += sh_b[i * CG * 4 + col]; tg += sh_g[i * CG * 4 + col]; }
-            atomicAdd(&w.sb[c], (unsigned long long)tb);
-            atomicAdd(&w.sg[c], (unsigned long long)tg);
-        }
+    // the block's 32 channels x 256 codes into its row tile's slab, 16 bytes a store
+    const int64_t c0 = (int64_t)blockIdx.x * kHistCh;
+    const int nch = (int)min((int64_t)kHistCh, (int64_t)C - c0);
+    int4* dst = reinterpret_cast<int4*>(w.hist + ((int64_t)blockIdx.y * C + c0) * 256);
+    for (int i = threadIdx.x; i < nch * 128; i += blockDim.x) {
+        const int b0 = 2 * i;                     // bins b0, b0 + 1 of the block's channels
+        dst[i] = make_int4(hsm[b0], hsm[kHistCh * 256 + b0], hsm[b0 + 1],
+                           hsm[kHistCh * 256 + b0 + 1]);
     }
 }
 
@@ -793,14 +1025,56 @@ __device__ __forceinline__ int e2_code(int z, const E2Div& d, int k) {
     return (int)clamp64(c, -qmax(k), qmax(k));
 }
 
-// the E_2 table: t2[c][e_y + 128] = SQ_kE2(e_y gamma_c)
-__global__ void k_bnb_tab2(const int32_t* __restrict__ gam, int32_t C, int k_e2, BnBwd w) {
+// Per channel (one warp each, eight codes a lane): the four sums over the histogram's row
+// tiles and the E_2 extremes per sign class (replacing the extreme codes in emin / emax).
+__global__ void k_bnb_hfin(const int32_t* __restrict__ gam, int64_t m, int32_t C, int gy,
+                           int k_e2, BnBwd w) {
+    const int c = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    if (c >= C) return;                           // whole warps leave together
     const E2Div d = *w.e2div;
-    const int64_t n = (int64_t)C * kTab2;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int c = (int)(i >> 8), ey = (int)(i & 255) - 128;
-        w.t2[i] = (int16_t)e2_code(ey * gam[c], d, k_e2);
+    const int gc = gam[c];
+    long long n[8] = {0, 0, 0, 0, 0, 0, 0, 0}, sv[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    for (int t = 0; t < gy; t++) {
+        const int4* src = reinterpret_cast<const int4*>(w.hist + ((int64_t)t * C + c) * 256);
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+            const int4 v = src[lane * 4 + i];     // bins 8 lane + 2 i, + 1
+            n[2 * i] += v.x; sv[2 * i] += v.y; n[2 * i + 1] += v.z; sv[2 * i + 1] += v.w;
+        }
+    }
+    long long sb = 0, sg = 0, se = 0, sex = 0;
+#pragma unroll
+    for (int i = 0; i < 8; i++) {
+        if (!n[i]) continue;
+        const int v = 8 * lane + i - 128;
+        const int e2 = e2_code(v * gc, d, k_e2);
+        sb += (long long)v * n[i];
+        sg += (long long)v * sv[i];
+        se += (long long)e2 * n[i];
+        sex += (long long)e2 * sv[i];
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        sb += __shfl_xor_sync(0xffffffffu, sb, o);
+        sg += __shfl_xor_sync(0xffffffffu, sg, o);
+        se += __shfl_xor_sync(0xffffffffu, se, o);
+        sex += __shfl_xor_sync(0xffffffffu, sex, o);
+    }
+    if (lane < 3) {
+        const int q = lane;
+        const int lo = w.emin[3 * c + q], hi = w.emax[3 * c + q];
+        if (lo <= hi) {
+            const int e0 = e2_code(lo * gc, d, k_e2), e1 = e2_code(hi * gc, d, k_e2);
+            w.emin[3 * c + q] = min(e0, e1);
+            w.emax[3 * c + q] = max(e0, e1);
+        }
+    }
+    if (lane == 0) {
+        w.sb[c] = (unsigned long long)sb;
+        w.sg[c] = (unsigned long long)sg;
+        w.se[c] = (unsigned long long)se;
+        w.sex[c] = (unsigned long long)sex;
     }
 }
 
@@ -813,115 +1087,6 @@ __device__ __forceinline__ void load_tables(const void* __restrict__ src, int64_
     for (int i = threadIdx.x; i < n16; i += blockDim.x) d4[i] = s4[i];
 }
 
-// E_2 = SQ_kE2(e_y gamma) (from the table): per channel sum E_2, sum E_2 X, sum sign X, and
-// the extremes of E_2 per sign class of X (-1, 0, +1).  The extremes travel packed as (max,
-// -min) int16 pairs (|E_2| <= 2^15 - 1), one __vmaxs2 per class.
-__global__ void __launch_bounds__(kThreads, 3) k_bnb_pass2(const int8_t* __restrict__ ea,
-                                                        const int8_t* __restrict__ a,
-                                                        const int16_t* __restrict__ X,
-                                                        int64_t m, int32_t C, int CG, BnBwd w) {
-    __shared__ long long sh_e[kThreads * 4], sh_x[kThreads * 4];
-    __shared__ __align__(16) int16_t tab[4 * kTabCG * kTab2];
-    __shared__ int sh_s[kThreads * 4];
-    __shared__ uint32_t sh_p[3][kThreads * 4];
-    const int C4 = C >> 2;
-    const int cg = threadIdx.x % CG, rl = threadIdx.x / CG, RL = blockDim.x / CG;
-    const int g = blockIdx.x * CG + cg;
-    const bool act = g < C4;
-    constexpr uint32_t kEmpty = 0x80008000u;      // (-32768, -32768): no element yet
-    {
-        const int64_t c0 = 4 * (int64_t)blockIdx.x * CG;
-        const int nch = (int)min((int64_t)4 * CG, (int64_t)C - c0);
-        load_tables(w.t2, c0, nch, 2 * kTab2, reinterpret_cast<uint8_t*>(tab));
-    }
-    __syncthreads();
-    const int16_t* tb = tab + 4 * cg * kTab2;
-    long long se64[4] = {0, 0, 0, 0}, sx[4] = {0, 0, 0, 0};
-    int ss[4] = {0, 0, 0, 0};
-    uint32_t pk[4][3];
-#pragma unroll
-    for (int j = 0; j < 4; j++)
-#pragma unroll
-        for (int q = 0; q < 3; q++) pk[j][q] = kEmpty;
-    const int64_t step = (int64_t)gridDim.y * RL;
-    if (act) {
-        int64_t r = (int64_t)blockIdx.y * RL + rl;
-        while (r < m) {
-            // int32 partial sums of E_2 over at most 2^15 rows (|E_2| < 2^15)
-            int se[4] = {0, 0, 0, 0};
-            auto row = [&](const int (&e0)[4], const int (&a0)[4], const int (&x0)[4]) {
-#pragma unroll
-                for (int j = 0; j < 4; j++) {
-                    const int ey = a0[j] > 0 ? e0[j] : 0;
-                    const int e2 = tb[j * kTab2 + ey + 128];
-                    const int sgn = (x0[j] > 0) - (x0[j] < 0);
-                    se[j] += e2;
-                    sx[j] += (long long)(e2 * x0[j]);     // |E_2 X| < 2^30
-                    ss[j] += sgn;
-                    const uint32_t cand = ((uint32_t)e2 & 0xffffu) | ((uint32_t)(-e2) << 16);
-                    if (sgn < 0) pk[j][0] = __vmaxs2(pk[j][0], cand);
-                    else if (sgn == 0) pk[j][1] = __vmaxs2(pk[j][1], cand);
-                    else pk[j][2] = __vmaxs2(pk[j][2], cand);
-                }
-            };
-            // two rows per iteration, both rows' loads in flight together
-            int it = 0;
-            for (; it < 32767 && r + step < m; it += 2, r += 2 * step) {
-                int e0[4], a0[4], x0[4], e1[4], a1[4], x1[4];
-                load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
-                load4_e_a_x((r + step) * C4 + g, ea, a, X, e1, a1, x1);
-                row(e0, a0, x0);
-                row(e1, a1, x1);
-            }
-            if (it < 32768 && r < m) {
-                int e0[4], a0[4], x0[4];
-                load4_e_a_x(r * C4 + g, ea, a, X, e0, a0, x0);
-                row(e0, a0, x0);
-                r += step;
-            }
-#pragma unroll
-            for (int j = 0; j < 4; j++) se64[j] += se[j];
-        }
-    }
-#pragma unroll
-    for (int j = 0; j < 4; j++) {
-        const int i = rl * CG * 4 + 4 * cg + j;
-        sh_e[i] = se64[j];
-        sh_x[i] = sx[j];
-        sh_s[i] = ss[j];
-#pragma unroll
-        for (int q = 0; q < 3; q++) sh_p[q][i] = pk[j][q];
-    }
-    __syncthreads();
-    const int col = threadIdx.x;
-    if (col < CG * 4) {
-        const int c = 4 * blockIdx.x * CG + col;
-        if (c < C) {
-            long long te = 0, tx = 0;
-            long long ts = 0;
-            uint32_t tp[3] = {kEmpty, kEmpty, kEmpty};
-            for (int i = 0; i < RL; i++) {
-                const int k = i * CG * 4 + col;
-                te += sh_e[k];
-                tx += sh_x[k];
-                ts += sh_s[k];
-#pragma unroll
-                for (int q = 0; q < 3; q++) tp[q] = __vmaxs2(tp[q], sh_p[q][k]);
-            }
-            atomicAdd(&w.se[c], (unsigned long long)te);
-            atomicAdd(&w.sex[c], (unsigned long long)tx);
-            atomicAdd(&w.ss[c], (unsigned long long)ts);
-#pragma unroll
-            for (int q = 0; q < 3; q++) {
-                if (tp[q] == kEmpty) continue;
-                const int hi = (int)(int16_t)(tp[q] & 0xffffu);
-                const int lo = -(int)(int16_t)(tp[q] >> 16);
-                atomicMin(&w.emin[3 * c + q], lo);
-                atomicMax(&w.emax[3 * c + q], hi);
-            }
-        }
-    }
-}
 // Per channel (oracle order): gx = (SEX s_x)/m; kap = -gx; lam = gx (SS/m) - SE/m;
 // w = s_e2 / ((c_sigma + 1) sg_step); d x = w ((E_2 + kap sgn) + lam).  Three launches of
 // C/64 blocks: M = max |d x| at the extremes of each sign class (red[0]), then the bound of
@@ -1008,6 +1173,292 @@ __global__ void k_bnb_tab3(const int32_t* __restrict__ gam, int32_t C, int k_e2,
     }
 }
 
+// ------------------------------------------------------------------ tiled backward passes
+// For C a power of two >= 64 or a multiple of 1024 the backward runs as three passes over 2-D
+// tiles (the histogram pass above is the fallback for other C): A, max |e_y| per channel,
+// sum sign X and the extreme codes of each sign class of X; B, the per-channel sums of e_y,
+// e_y X, E_2 and E_2 X; and the output pass.  The integer ALU work of the statistics is split
+// between A and B so that each stays near the memory rate.  A block owns a slab of kTileC = 64
+// channels, whose per-channel tables (E_2 of the code, or the output code of (sign X, code))
+// sit in shared memory, and row chunks of kTileR rows of it, each chunk one TMA tile per array
+// (e_a, the activation codes, X; rows past m read as zeros and are not counted).
+constexpr int kTileC = 64;
+constexpr int kTileR = 128;
+constexpr int kTileStages = 4;
+constexpr int kTileStage = kTileR * kTileC * 4;          // int8 e_a, int8 a, int16 X
+constexpr int kTab2P = 258;                              // E_2 table row, padded (int16)
+constexpr int kTileSmem = 1024 + kTileStages * kTileStage + 2 * kTileStages * 8;
+
+// byte permute with sign replication (a selector nibble with its msb set copies the sign of
+// the selected byte): 0x9180 / 0xb3a2 widen bytes 0, 1 / 2, 3 to two signed 16-bit lanes
+__device__ __forceinline__ uint32_t prmt_sext(uint32_t a, uint32_t sel) {
+    uint32_t r;
+    asm("prmt.b32 %0, %1, 0, %2;" : "=r"(r) : "r"(a), "r"(sel));
+    return r;
+}
+
+__device__ __forceinline__ uint8_t* align1k(uint8_t* p) {
+    return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+// the E_2 table: t2[c][e_y + 128] = SQ_kE2(e_y gamma_c)
+__global__ void k_bnb_tab2(const int32_t* __restrict__ gam, int32_t C, int k_e2, BnBwd w) {
+    const E2Div d = *w.e2div;
+    const int64_t n = (int64_t)C * 256;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i >> 8), ey = (int)(i & 255) - 128;
+        w.t2[i] = (int16_t)e2_code(ey * gam[c], d, k_e2);
+    }
+}
+
+// thread 0: chunk k of the slab's three tiles into `st`
+__device__ __forceinline__ void tile_issue(const CUtensorMap* me, const CUtensorMap* ma,
+                                           const CUtensorMap* mxh, uint8_t* st, uint64_t* bar,
+                                           int64_t k) {
+    tc::mbar_arrive_expect_tx(bar, kTileStage);
+    const int x = blockIdx.x * kTileC, y = (int)(k * kTileR);
+    tc::tma_load_2d(st, me, bar, x, y);
+    tc::tma_load_2d(st + kTileR * kTileC, ma, bar, x, y);
+    tc::tma_load_2d(st + 2 * kTileR * kTileC, mxh, bar, x, y);
+}
+
+// Pass A over tiles: max |e_y| per channel (for max |e_y gamma|), sum sign X, and the extreme
+// code e_y of each sign class of X (-, 0, +), four channels packed in the bytes of a word.
+__global__ void __launch_bounds__(kStreamThreads, 1)
+    k_bnb_a_t(const __grid_constant__ CUtensorMap me, const __grid_constant__ CUtensorMap ma,
+              const __grid_constant__ CUtensorMap mxh, int64_t m, int32_t C,
+              const int32_t* __restrict__ gam, BnBwd w, int* __restrict__ err) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = align1k(smem_raw);
+    if (__syncthreads_or(threadIdx.x == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    const int c_base = blockIdx.x * kTileC;
+    const int g = threadIdx.x & 15, rl = threadIdx.x >> 4;       // 16 groups x 32 row lanes
+    long long ss[4] = {0, 0, 0, 0};
+    uint32_t amax = 0;                                            // per byte: max |e_y|
+    uint32_t mx[3] = {0x80808080u, 0x80808080u, 0x80808080u};    // empty: max 0x80 < min 0x7f
+    uint32_t mn[3] = {0x7f7f7f7fu, 0x7f7f7f7fu, 0x7f7f7f7fu};
+    const int64_t nchunk = (m + kTileR - 1) / kTileR;
+    const bool ok = pipe_chunks<kTileStages>(
+        nchunk, kTileR, m, kTileStage, smem, err,
+        [&](uint8_t* st, uint64_t* bar, int64_t k) { tile_issue(&me, &ma, &mxh, st, bar, k); },
+        [&](const uint8_t* st, int rows, int64_t) {
+            const uint32_t* e4 = reinterpret_cast<const uint32_t*>(st);
+            const uint32_t* a4 = reinterpret_cast<const uint32_t*>(st + kTileR * kTileC);
+            const uint2* x4 = reinterpret_cast<const uint2*>(st + 2 * kTileR * kTileC);
+            uint32_t npos = 0, nneg = 0;     // the chunk's sign counts (<= 4 a byte)
+#pragma unroll
+            for (int u = 0; u < kTileR / 32; u++) {
+                const int r = rl + 32 * u;
+                if (r >= rows) break;
+                const int i = r * 16 + g;
+                const uint32_t ey = e4[i] & __vcmpgts4(a4[i], 0u);
+                const uint2 xv = x4[i];
+                // byte j of pos / neg: 0xff where X of channel j is > 0 / < 0
+                const uint32_t pos = __byte_perm(__vcmpgts2(xv.x, 0u), __vcmpgts2(xv.y, 0u), 0x6420);
+                const uint32_t neg = __byte_perm(__vcmplts2(xv.x, 0u), __vcmplts2(xv.y, 0u), 0x6420);
+                npos += pos & 0x01010101u;
+                nneg += neg & 0x01010101u;
+                amax = __vmaxu4(amax, __vabs4(ey));
+                const uint32_t cls[3] = {neg, ~(neg | pos), pos};
+#pragma unroll
+                for (int q = 0; q < 3; q++) {
+                    mx[q] = __vmaxs4(mx[q], (ey & cls[q]) | (0x80808080u & ~cls[q]));
+                    mn[q] = __vmins4(mn[q], (ey & cls[q]) | (0x7f7f7f7fu & ~cls[q]));
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 4; j++)
+                ss[j] += (int)((npos >> (8 * j)) & 0xffu) - (int)((nneg >> (8 * j)) & 0xffu);
+        });
+    if (!ok) return;
+    long long* sq = reinterpret_cast<long long*>(smem);                // [32][64]
+    uint32_t* sp = reinterpret_cast<uint32_t*>(sq + 32 * kTileC);      // [7][512]
+#pragma unroll
+    for (int j = 0; j < 4; j++) sq[rl * kTileC + 4 * g + j] = ss[j];
+#pragma unroll
+    for (int q = 0; q < 3; q++) {
+        sp[(2 * q) * kStreamThreads + threadIdx.x] = mx[q];
+        sp[(2 * q + 1) * kStreamThreads + threadIdx.x] = mn[q];
+    }
+    sp[6 * kStreamThreads + threadIdx.x] = amax;
+    __syncthreads();
+    const int col = threadIdx.x;
+    uint32_t zm = 0;
+    if (col < kTileC) {
+        long long t = 0;
+        for (int i = 0; i < 32; i++) t += sq[i * kTileC + col];
+        const int c = c_base + col;
+        atomicAdd(&w.ss[c], (unsigned long long)t);
+        const int gg = col >> 2, j = col & 3;
+        uint32_t am = 0;
+        for (int i = 0; i < 32; i++) am = __vmaxu4(am, sp[6 * kStreamThreads + i * 16 + gg]);
+        zm = ((am >> (8 * j)) & 0xffu) * (uint32_t)abs(gam[c]);
+#pragma unroll
+        for (int q = 0; q < 3; q++) {
+            uint32_t hx = 0x80808080u, ln = 0x7f7f7f7fu;
+            for (int i = 0; i < 32; i++) {
+                hx = __vmaxs4(hx, sp[(2 * q) * kStreamThreads + i * 16 + gg]);
+                ln = __vmins4(ln, sp[(2 * q + 1) * kStreamThreads + i * 16 + gg]);
+            }
+            const int hi = (int)(int8_t)(hx >> (8 * j)), lo = (int)(int8_t)(ln >> (8 * j));
+            if (lo > hi) continue;                 // no element of this class
+            atomicMin(&w.emin[3 * c + q], lo);     // codes; k_bnb_ext maps them to E_2
+            atomicMax(&w.emax[3 * c + q], hi);
+        }
+    }
+    if (threadIdx.x < 64) {
+        zm = warp_max_u32(zm);
+        if ((threadIdx.x & 31) == 0 && zm) atomicMax(w.zmax, zm);
+    }
+}
+
+// E_2 is monotone in e_y: the E_2 extremes of a sign class are E_2 at its extreme codes
+__global__ void k_bnb_ext(int32_t C, BnBwd w) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;         // 3 c + q
+    if (i >= 3 * C) return;
+    const int lo = w.emin[i], hi = w.emax[i];
+    if (lo > hi) return;
+    const int16_t* t = w.t2 + (int64_t)(i / 3) * 256 + 128;
+    const int e0 = t[lo], e1 = t[hi];
+    w.emin[i] = min(e0, e1);
+    w.emax[i] = max(e0, e1);
+}
+
+// Pass B over tiles: per channel sum e_y, sum e_y X, sum E_2 and sum E_2 X, E_2 from the
+// slab's table in shared memory
+__global__ void __launch_bounds__(kStreamThreads, 1)
+    k_bnb_b_t(const __grid_constant__ CUtensorMap me, const __grid_constant__ CUtensorMap ma,
+              const __grid_constant__ CUtensorMap mxh, int64_t m, int32_t C, BnBwd w,
+              int* __restrict__ err) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = align1k(smem_raw);
+    int16_t* tab = reinterpret_cast<int16_t*>(smem + kTileStages * kTileStage + 2 * kTileStages * 8);
+    if (__syncthreads_or(threadIdx.x == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    const int c_base = blockIdx.x * kTileC;
+    for (int i = threadIdx.x; i < kTileC * 128; i += blockDim.x) {
+        const int ch = i >> 7, k2 = i & 127;            // two entries a word
+        reinterpret_cast<uint32_t*>(tab + ch * kTab2P)[k2] =
+            reinterpret_cast<const uint32_t*>(w.t2 + (int64_t)(c_base + ch) * 256)[k2];
+    }
+    __syncthreads();
+    const int g = threadIdx.x & 15, rl = threadIdx.x >> 4;
+    const int16_t* tb = tab + 4 * g * kTab2P + 128;
+    long long sb[4] = {0, 0, 0, 0}, sg[4] = {0, 0, 0, 0}, se[4] = {0, 0, 0, 0};
+    long long sx[4] = {0, 0, 0, 0};
+    const int64_t nchunk = (m + kTileR - 1) / kTileR;
+    const bool ok = pipe_chunks<kTileStages>(
+        nchunk, kTileR, m, kTileStage, smem, err,
+        [&](uint8_t* st, uint64_t* bar, int64_t k) { tile_issue(&me, &ma, &mxh, st, bar, k); },
+        [&](const uint8_t* st, int rows, int64_t) {
+            const uint32_t* e4 = reinterpret_cast<const uint32_t*>(st);
+            const uint32_t* a4 = reinterpret_cast<const uint32_t*>(st + kTileR * kTileC);
+            const uint2* x4 = reinterpret_cast<const uint2*>(st + 2 * kTileR * kTileC);
+            // the chunk's partial sums in 32 bits (kTileR / 32 rows a thread: |e_y X| < 2^22,
+            // |E_2| < 2^15; a pair of E_2 X products < 2^31)
+            int cb[4] = {0, 0, 0, 0}, cg[4] = {0, 0, 0, 0}, ce[4] = {0, 0, 0, 0};
+#pragma unroll
+            for (int u = 0; u < kTileR / 32; u += 2) {
+                int p2[4] = {0, 0, 0, 0};
+#pragma unroll
+                for (int h = 0; h < 2; h++) {
+                    const int r = rl + 32 * (u + h);
+                    if (r >= rows) break;
+                    const int i = r * 16 + g;
+                    const uint32_t ey = e4[i] & __vcmpgts4(a4[i], 0u);
+                    const uint2 xv = x4[i];
+                    const int x[4] = {(int)(int16_t)(xv.x & 0xffffu), (int)xv.x >> 16,
+                                      (int)(int16_t)(xv.y & 0xffffu), (int)xv.y >> 16};
+#pragma unroll
+                    for (int j = 0; j < 4; j++) {
+                        const int v = (int)(int8_t)(ey >> (8 * j));
+                        const int e2 = tb[j * kTab2P + v];   // E_2(0) = 0
+                        cb[j] += v;
+                        cg[j] += v * x[j];
+                        ce[j] += e2;
+                        p2[j] += e2 * x[j];
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < 4; j++) sx[j] += p2[j];
+            }
+#pragma unroll
+            for (int j = 0; j < 4; j++) { sb[j] += cb[j]; sg[j] += cg[j]; se[j] += ce[j]; }
+        });
+    if (!ok) return;
+    constexpr int NQ = 4;
+    long long* sq = reinterpret_cast<long long*>(smem);             // [NQ][32][64]
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        const int i = rl * kTileC + 4 * g + j;
+        sq[0 * 32 * kTileC + i] = sb[j];
+        sq[1 * 32 * kTileC + i] = sg[j];
+        sq[2 * 32 * kTileC + i] = se[j];
+        sq[3 * 32 * kTileC + i] = sx[j];
+    }
+    __syncthreads();
+    const int col = threadIdx.x;
+    if (col < kTileC) {
+        long long t[NQ] = {0, 0, 0, 0};
+        for (int i = 0; i < 32; i++)
+#pragma unroll
+            for (int q = 0; q < NQ; q++) t[q] += sq[q * 32 * kTileC + i * kTileC + col];
+        const int c = c_base + col;
+        atomicAdd(&w.sb[c], (unsigned long long)t[0]);
+        atomicAdd(&w.sg[c], (unsigned long long)t[1]);
+        atomicAdd(&w.se[c], (unsigned long long)t[2]);
+        atomicAdd(&w.sex[c], (unsigned long long)t[3]);
+    }
+}
+
+__global__ void __launch_bounds__(kStreamThreads, 1)
+    k_bnb_out_t(const __grid_constant__ CUtensorMap me, const __grid_constant__ CUtensorMap ma,
+                const __grid_constant__ CUtensorMap mxh, int64_t m, int32_t C, BnBwd w,
+                int8_t* __restrict__ out, int* __restrict__ err) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = align1k(smem_raw);
+    uint8_t* tab = smem + kTileStages * kTileStage + 2 * kTileStages * 8;   // [64][kTab3P]
+    if (__syncthreads_or(threadIdx.x == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    const int c_base = blockIdx.x * kTileC;
+    {
+        const uint32_t* src = reinterpret_cast<const uint32_t*>(w.t3 + (int64_t)c_base * kTab3);
+        for (int i = threadIdx.x; i < kTileC * (kTab3 / 4); i += blockDim.x) {
+            const int ch = i / (kTab3 / 4), k = i - ch * (kTab3 / 4);
+            reinterpret_cast<uint32_t*>(tab + ch * kTab3P)[k] = src[i];
+        }
+    }
+    __syncthreads();
+    const int g = threadIdx.x & 15, rl = threadIdx.x >> 4;
+    const int8_t* tb = reinterpret_cast<const int8_t*>(tab) + 4 * g * kTab3P + 256 + 128;
+    const int64_t nchunk = (m + kTileR - 1) / kTileR;
+    pipe_chunks<kTileStages>(
+        nchunk, kTileR, m, kTileStage, smem, err,
+        [&](uint8_t* st, uint64_t* bar, int64_t k) { tile_issue(&me, &ma, &mxh, st, bar, k); },
+        [&](const uint8_t* st, int rows, int64_t r0) {
+            const uint32_t* e4 = reinterpret_cast<const uint32_t*>(st);
+            const uint32_t* a4 = reinterpret_cast<const uint32_t*>(st + kTileR * kTileC);
+            const uint2* x4 = reinterpret_cast<const uint2*>(st + 2 * kTileR * kTileC);
+#pragma unroll
+            for (int u = 0; u < kTileR / 32; u++) {
+                const int r = rl + 32 * u;
+                if (r >= rows) break;
+                const int i = r * 16 + g;
+                const uint32_t ey = e4[i] & __vcmpgts4(a4[i], 0u);
+                const uint2 xv = x4[i];
+                const int x[4] = {(int)(int16_t)(xv.x & 0xffffu), (int)xv.x >> 16,
+                                  (int)(int16_t)(xv.y & 0xffffu), (int)xv.y >> 16};
+                uint32_t o = 0;
+#pragma unroll
+                for (int j = 0; j < 4; j++) {
+                    const int v = (int)(int8_t)(ey >> (8 * j));
+                    const int sg = (x[j] > 0) - (x[j] < 0);
+                    o |= ((uint32_t)(uint8_t)tb[j * kTab3P + sg * 256 + v]) << (8 * j);
+                }
+                *reinterpret_cast<uint32_t*>(out + (r0 + r) * C + c_base + 4 * g) = o;
+            }
+        });
+}
+
 // e = the output code of (sign X, e_y) per element, from the block's tables in shared memory
 __global__ void __launch_bounds__(kThreads) k_bnb_pass3(const int8_t* __restrict__ ea,
                                                         const int8_t* __restrict__ a,
@@ -1068,7 +1519,6 @@ __device__ __forceinline__ int code16(const uint32_t* o, int j) {
 // (64 channels) x 64 row lanes; the 64 channels' tables sit in shared memory in rows of
 // 772 bytes (the 768-byte rows padded by one word, so that the rows of neighbouring
 // channels start in different banks).
-constexpr int kTab3P = kTab3 + 4;
 
 __global__ void __launch_bounds__(kThreads, 4) k_bnb_p3w(const int8_t* __restrict__ ea,
                                                          const int8_t* __restrict__ a,
@@ -1132,9 +1582,9 @@ __global__ void __launch_bounds__(kThreads, 4) k_bnb_p3w(const int8_t* __restric
     }
 }
 
-size_t bn_bwd_ws_bytes(int32_t C) {
+size_t bn_bwd_ws_bytes(int64_t m, int32_t C) {
     WsCursor c(nullptr, 0);
-    bnb_carve(c, C);
+    bnb_carve(c, m, C);
     return c.off + 256;
 }
 
@@ -1146,7 +1596,7 @@ using namespace iq;
 
 extern "C" iq_status iq_bn_int_workspace_size(int64_t m, int32_t c, size_t* bytes) {
     if (!bytes || m < 0 || c <= 0) return IQ_ERR_INVALID_ARG;
-    size_t f = bn_fwd_ws_bytes(c), b = bn_bwd_ws_bytes(c);
+    size_t f = bn_fwd_ws_bytes(c), b = bn_bwd_ws_bytes(m, c);
     *bytes = f > b ? f : b;
     return IQ_OK;
 }
@@ -1191,59 +1641,128 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
     if (!bn_bits_valid(b) || k_e2 < 2 || k_e2 > 16) return IQ_ERR_INVALID_ARG;
     if (((uintptr_t)e_a | (uintptr_t)a | (uintptr_t)xhat | (uintptr_t)e) & 15)
         return IQ_ERR_INVALID_ARG;
-    size_t need = bn_bwd_ws_bytes(c);
+    if (m > (int64_t)65535 * kHistRows) return IQ_ERR_UNSUPPORTED;
+    size_t need = bn_bwd_ws_bytes(m, c);
     if (!ws || ws_bytes < need) return IQ_ERR_WORKSPACE;
     cudaStream_t st = (cudaStream_t)stream;
     WsCursor cur(ws, ws_bytes);
-    BnBwd w = bnb_carve(cur, c);
+    BnBwd w = bnb_carve(cur, m, c);
     k_bnb_init<<<(c + 255) / 256, 256, 0, st>>>(w, c);
     IQ_LAUNCH_CHECK();
-    RowGrid rg = row_grid(m, c / 4);
-    kt_pre(st);
-    k_bnb_pass1<<<rg.grid, kThreads, 0, st>>>(e_a, a, xhat, gamma, m, c, rg.cg, w);
-    IQ_LAUNCH_CHECK();
-    kt_post_bytes(st, IQ_KERNEL_BNB_PASS1, 4.0 * (double)m * c);
-    k_bnb_fin1<<<1, 1, 0, st>>>(w, s_e, b.k_gamma, k_e2);
-    IQ_LAUNCH_CHECK();
-    const int tb2 = (int)(((int64_t)c * kTab2 + kThreads - 1) / kThreads);
-    k_bnb_tab2<<<tb2 < 152 * 4 ? tb2 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, w);
-    IQ_LAUNCH_CHECK();
-    RowGrid rt = row_grid(m, c / 4, 152 * 8, kTabCG);
-    kt_pre(st);
-    k_bnb_pass2<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w);
-    IQ_LAUNCH_CHECK();
-    kt_post_bytes(st, IQ_KERNEL_BNB_PASS2, 4.0 * (double)m * c);
+    int* err = device_status_ptr();
+    if (!err) return IQ_ERR_CUDA;
+    const bool streamed = bnb_fast(c) && m < (int64_t(1) << 31);
     const int fb = (c + kFinThreads - 1) / kFinThreads;
-    k_bnb_fin2a<<<fb, kFinThreads, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma);
-    IQ_LAUNCH_CHECK();
-    k_bnb_fin2b<<<fb, kFinThreads, 0, st>>>(w, c, k_e2, 8);
-    IQ_LAUNCH_CHECK();
-    k_bnb_fin2c<<<fb, kFinThreads, 0, st>>>(w, c, 8, s_e_out);
-    IQ_LAUNCH_CHECK();
-    const int tb3 = (int)(((int64_t)c * kTab3 + kThreads - 1) / kThreads);
-    k_bnb_tab3<<<tb3 < 152 * 4 ? tb3 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, 8, w);
-    IQ_LAUNCH_CHECK();
-    kt_pre(st);
-    if (c % 16 == 0) {
-        static bool attr = false;
-        const int smem = 64 * kTab3P;
-        if (!attr) {
-            IQ_CUDA_CHECK(cudaFuncSetAttribute(k_bnb_p3w, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               smem));
-            attr = true;
+    if (streamed) {
+        CUtensorMap me, ma, mxh;
+        iq_status r = encode_rows_2d(e_a, 1, m, c, kTileC, kTileR, &me);
+        if (r == IQ_OK) r = encode_rows_2d(a, 1, m, c, kTileC, kTileR, &ma);
+        if (r == IQ_OK) r = encode_rows_2d(xhat, 2, m, c, kTileC, kTileR, &mxh);
+        if (r != IQ_OK) return r;
+        static bool attr_a = false, attr_b = false, attr_o = false;
+        const int smem_a = kTileSmem, smem_b = kTileSmem + kTileC * kTab2P * 2,
+                  smem_o = kTileSmem + kTileC * kTab3P;
+        if (!attr_a) {
+            IQ_CUDA_CHECK(cudaFuncSetAttribute(k_bnb_a_t,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, smem_a));
+            attr_a = true;
         }
-        const int bx = (c + 63) / 64;
-        int64_t by3 = (m + 63) / 64;
-        const int64_t cap3 = (152 * 8 + bx - 1) / bx;
-        if (by3 > cap3) by3 = cap3;
-        if (by3 > 65535) by3 = 65535;
-        k_bnb_p3w<<<dim3((unsigned)bx, (unsigned)by3), kThreads, smem, st>>>(e_a, a, xhat, m, c,
-                                                                             w, e);
+        if (!attr_b) {
+            IQ_CUDA_CHECK(cudaFuncSetAttribute(k_bnb_b_t,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, smem_b));
+            attr_b = true;
+        }
+        if (!attr_o) {
+            IQ_CUDA_CHECK(cudaFuncSetAttribute(k_bnb_out_t,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, smem_o));
+            attr_o = true;
+        }
+        const int sms = device_sms();
+        const int slabs = c / kTileC;
+        int64_t gy = sms / slabs;               // one block per SM: no second wave
+        if (gy < 1) gy = 1;
+        const int64_t nchunk = (m + kTileR - 1) / kTileR;
+        if (gy > nchunk) gy = nchunk;
+        if (gy > 65535) gy = 65535;
+        const dim3 tgrid((unsigned)slabs, (unsigned)gy);
+        kt_pre(st);
+        k_bnb_a_t<<<tgrid, kStreamThreads, smem_a, st>>>(me, ma, mxh, m, c, gamma, w, err);
+        IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_BNB_PASS1, 4.0 * (double)m * c);
+        k_bnb_fin1<<<1, 1, 0, st>>>(w, s_e, b.k_gamma, k_e2);
+        IQ_LAUNCH_CHECK();
+        const int tb2 = (int)(((int64_t)c * 256 + kThreads - 1) / kThreads);
+        k_bnb_tab2<<<tb2 < 152 * 4 ? tb2 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, w);
+        IQ_LAUNCH_CHECK();
+        k_bnb_ext<<<(3 * c + kThreads - 1) / kThreads, kThreads, 0, st>>>(c, w);
+        IQ_LAUNCH_CHECK();
+        kt_pre(st);
+        k_bnb_b_t<<<tgrid, kStreamThreads, smem_b, st>>>(me, ma, mxh, m, c, w, err);
+        IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_BNB_PASS2, 4.0 * (double)m * c);
+        k_bnb_fin2a<<<fb, kFinThreads, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma);
+        IQ_LAUNCH_CHECK();
+        k_bnb_fin2b<<<fb, kFinThreads, 0, st>>>(w, c, k_e2, 8);
+        IQ_LAUNCH_CHECK();
+        k_bnb_fin2c<<<fb, kFinThreads, 0, st>>>(w, c, 8, s_e_out);
+        IQ_LAUNCH_CHECK();
+        const int tb3 = (int)(((int64_t)c * kTab3 + kThreads - 1) / kThreads);
+        k_bnb_tab3<<<tb3 < 152 * 4 ? tb3 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, 8, w);
+        IQ_LAUNCH_CHECK();
+        kt_pre(st);
+        k_bnb_out_t<<<tgrid, kStreamThreads, smem_o, st>>>(me, ma, mxh, m, c, w, e, err);
+        IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_BNB_PASS3, 5.0 * (double)m * c);
     } else {
-        k_bnb_pass3<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w, e);
+        const int gy = hist_tiles(m, c);
+        static bool hist_attr = false;
+        if (!hist_attr) {
+            IQ_CUDA_CHECK(cudaFuncSetAttribute(k_bnb_hist, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               kHistSmem));
+            hist_attr = true;
+        }
+        kt_pre(st);
+        k_bnb_hist<<<dim3((unsigned)((c + kHistCh - 1) / kHistCh), (unsigned)gy), kThreads, kHistSmem,
+                     st>>>(e_a, a, xhat, gamma, m, c, w);
+        IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_BNB_PASS1, 4.0 * (double)m * c);
+        k_bnb_fin1<<<1, 1, 0, st>>>(w, s_e, b.k_gamma, k_e2);
+        IQ_LAUNCH_CHECK();
+        k_bnb_hfin<<<(unsigned)(((int64_t)c * 32 + kThreads - 1) / kThreads), kThreads, 0, st>>>(
+            gamma, m, c, gy, k_e2, w);
+        IQ_LAUNCH_CHECK();
+        k_bnb_fin2a<<<fb, kFinThreads, 0, st>>>(w, m, c, bn_codes + c, bn_scales, b.k_sigma);
+        IQ_LAUNCH_CHECK();
+        k_bnb_fin2b<<<fb, kFinThreads, 0, st>>>(w, c, k_e2, 8);
+        IQ_LAUNCH_CHECK();
+        k_bnb_fin2c<<<fb, kFinThreads, 0, st>>>(w, c, 8, s_e_out);
+        IQ_LAUNCH_CHECK();
+        const int tb3 = (int)(((int64_t)c * kTab3 + kThreads - 1) / kThreads);
+        k_bnb_tab3<<<tb3 < 152 * 4 ? tb3 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, 8, w);
+        IQ_LAUNCH_CHECK();
+        kt_pre(st);
+        if (c % 16 == 0) {
+            static bool attr = false;
+            const int smem = 64 * kTab3P;
+            if (!attr) {
+                IQ_CUDA_CHECK(cudaFuncSetAttribute(k_bnb_p3w, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   smem));
+                attr = true;
+            }
+            const int bx = (c + 63) / 64;
+            int64_t by3 = (m + 63) / 64;
+            const int64_t cap3 = (152 * 8 + bx - 1) / bx;
+            if (by3 > cap3) by3 = cap3;
+            if (by3 > 65535) by3 = 65535;
+            k_bnb_p3w<<<dim3((unsigned)bx, (unsigned)by3), kThreads, smem, st>>>(e_a, a, xhat, m, c,
+                                                                                 w, e);
+        } else {
+            RowGrid rt = row_grid(m, c / 4, 152 * 8, kTabCG);
+            k_bnb_pass3<<<rt.grid, kThreads, 0, st>>>(e_a, a, xhat, m, c, rt.cg, w, e);
+        }
+        IQ_LAUNCH_CHECK();
+        kt_post_bytes(st, IQ_KERNEL_BNB_PASS3, 5.0 * (double)m * c);
     }
-    IQ_LAUNCH_CHECK();
-    kt_post_bytes(st, IQ_KERNEL_BNB_PASS3, 5.0 * (double)m * c);
     if (dgamma)
         IQ_CUDA_CHECK(cudaMemcpyAsync(dgamma, w.sg, sizeof(int64_t) * c, cudaMemcpyDeviceToDevice, st));
     if (dbeta)

@@ -2393,6 +2393,29 @@ constexpr int MAX_KB_INT32 = 133120 / 64;   // 2080 k-blocks: 133120 * 127^2 < 2
 
 }  // namespace
 
+// the sticky device status word of the current context (iq_device_status reads it)
+int* device_status_ptr() { return tc_status_ptr(); }
+
+// streaming multiprocessors of the current device
+int device_sms() { return num_sms(); }
+
+// 2-D tensor map of a row-major [m][C] array of 1- or 2-byte elements: box {box_c channels,
+// box_r rows}, no swizzle, zero fill outside the array
+iq_status encode_rows_2d(const void* base, int esz, int64_t m, int C, int box_c, int box_r,
+                         CUtensorMap* map) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
+    if (!enc || (esz != 1 && esz != 2)) return IQ_ERR_UNSUPPORTED;
+    cuuint64_t gdim[2] = {(cuuint64_t)C, (cuuint64_t)m};
+    cuuint64_t gstride[1] = {(cuuint64_t)C * esz};
+    cuuint32_t box[2] = {(cuuint32_t)box_c, (cuuint32_t)box_r};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, esz == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16,
+                     2, const_cast<void*>(base), gdim, gstride, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? IQ_OK : IQ_ERR_CUDA;
+}
+
 // ================================================================ forward
 
 // fp16 weights, a reserved 256-byte slot, then the fp16 carriers of the input

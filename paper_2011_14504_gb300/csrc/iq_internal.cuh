@@ -3,7 +3,21 @@
 
 #include "iq_common.cuh"
 
+#include <cuda.h>
+
 namespace iq {
+
+// Device address of the sticky status word that iq_device_status reads and clears (a kernel
+// whose bounded wait gave up stores its IQ_ERR_* code there), or NULL.
+int* device_status_ptr();
+
+// streaming multiprocessors of the current device
+int device_sms();
+
+// 2-D tensor map of a row-major [m][C] array of 1- or 2-byte elements: box {box_c channels,
+// box_r rows}, no swizzle, zero fill outside the array
+iq_status encode_rows_2d(const void* base, int esz, int64_t m, int C, int box_c, int box_r,
+                         CUtensorMap* map);
 
 // Scratch needed by requant_int (bytes).
 size_t requant_ws_bytes();

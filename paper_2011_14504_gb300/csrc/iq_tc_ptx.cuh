@@ -195,6 +195,24 @@ __device__ __forceinline__ void tma_load_5d_e(void* dst, const CUtensorMap* map,
         : "memory");
 }
 
+// ---------------------------------------------------------------- 1-D bulk copies
+// arrive on the barrier and add `bytes` to its expected transaction count
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+// global -> shared copy of `bytes` contiguous bytes (both addresses 16-byte aligned, bytes a
+// multiple of 16), completion counted on the barrier's transaction bytes
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes,
+                                         uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
 // ---------------------------------------------------------------- bulk tensor stores
 // 4-D tiled store from shared memory (dense box, no swizzle); elements outside the tensor are
 // not written.  The caller fences the generic-proxy writes of the box first
