@@ -1591,7 +1591,8 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                                 gmn = min(gmn, sum[i]);
                             }
                         }
-                    } else {
+                    } else if ((p.st_mask & (TC_STATS_SUM | TC_STATS_LO)) ||
+                               !(p.st_mask & ST_NOEXT)) {
 #pragma unroll
                         for (int cb = 0; cb < CW; cb += LDW)
                             col_stats<LDW>(p, sum + cb, valid, q.n0 + quarter * CW + cb, lane, s1,
@@ -2451,6 +2452,113 @@ static const iq_conv_desc* flat_pointwise(const iq_conv_desc* d, iq_conv_desc* t
     return tmp;
 }
 
+// ---------------------------------------------------------------- channel sums from the input
+// With batch norm the forward needs S1[k] = the sum over every output pixel of acc[.][k].  In
+// the pixel-major kernel that is a reduction across the lanes of the epilogue, about half the
+// time of a 1x1 layer; for a 1x1 convolution without padding it follows exactly from the
+// input instead: S1[k] = sum_c W[k][c] S_A[c], S_A[c] the sum of x[n][h][w][c] over the input
+// pixels the output pixels read (h = p sh, w = q sw).  Taken where the output has at least
+// twice the elements of the input (the expanding 1x1 layers), where reading the int8 input
+// costs a small fraction of the epilogue reduction it replaces.
+
+bool input_sums_ok(const iq_conv_desc* d) {
+    return d->r == 1 && d->s == 1 && d->pad_h == 0 && d->pad_w == 0 && d->groups == 1 &&
+           d->c % 4 == 0 && (int64_t)d->k * ((d->h - 1) / d->stride_h + 1) *
+                                    ((d->w - 1) / d->stride_w + 1) >= 2LL * d->c * d->h * d->w;
+}
+
+// S_A[c] += the sum of x over the sampled pixels: thread t owns channels 4 (t % C4) and a row
+// lane of the pixels; the block's lanes combine in shared memory, then one atomic per channel
+__global__ void __launch_bounds__(kThreads) k_input_colsums(const int8_t* __restrict__ x, int N,
+                                                            int H, int W, int C, int P, int Q,
+                                                            int sh, int sw,
+                                                            long long* __restrict__ SA) {
+    __shared__ long long sh_s[kThreads * 4];
+    const int C4 = C >> 2;
+    const int lanes = blockDim.x / C4;                  // blockDim.x % C4 == 0 (host)
+    const int g = threadIdx.x % C4, rl = threadIdx.x / C4;
+    const int64_t npix = (int64_t)N * P * Q;
+    const int64_t step = (int64_t)gridDim.x * lanes;
+    int a[4] = {0, 0, 0, 0};
+    long long acc[4] = {0, 0, 0, 0};
+    int cnt = 0;
+    for (int64_t m = (int64_t)blockIdx.x * lanes + rl; m < npix; m += step) {
+        const int q = (int)(m % Q);
+        const int64_t np = m / Q;
+        const int pp = (int)(np % P), n = (int)(np / P);
+        const uint32_t v = __ldg(reinterpret_cast<const uint32_t*>(
+                                     x + (((int64_t)n * H + (int64_t)pp * sh) * W + (int64_t)q * sw) * C) + g);
+        a[0] += (int)(int8_t)v; a[1] += (int)(int8_t)(v >> 8);
+        a[2] += (int)(int8_t)(v >> 16); a[3] += (int)(int8_t)(v >> 24);
+        if (++cnt == 1 << 20) {                          // |partial| < 2^27
+#pragma unroll
+            for (int j = 0; j < 4; j++) { acc[j] += a[j]; a[j] = 0; }
+            cnt = 0;
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; j++) sh_s[rl * C + 4 * g + j] = acc[j] + a[j];
+    __syncthreads();
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        long long t = 0;
+        for (int i = 0; i < lanes; i++) t += sh_s[i * C + c];
+        if (t) atomicAdd(reinterpret_cast<unsigned long long*>(SA + c), (unsigned long long)t);
+    }
+}
+
+// S1[k] = sum_c S_A[c] W[k][c] (one warp per output channel)
+__global__ void k_input_gemv(const long long* __restrict__ SA, const int8_t* __restrict__ w, int K,
+                             int C, unsigned long long* __restrict__ s1) {
+    const int k = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    if (k >= K) return;                              // whole warps leave together
+    const int8_t* wk = w + (int64_t)k * C;
+    long long a = 0;
+    for (int j = lane; j < C; j += 32) a += SA[j] * (long long)wk[j];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+    if (lane == 0) s1[k] = (unsigned long long)a;
+}
+
+// scratch of the input-side sums (S_A)
+size_t input_sums_bytes(const iq_conv_desc* d) { return (size_t)d->c * 8 + 256; }
+
+iq_status input_sums(const iq_conv_desc* d, const int8_t* x, const int8_t* w, char* scratch,
+                     unsigned long long* s1, cudaStream_t st) {
+    const int P = (d->h - 1) / d->stride_h + 1, Q = (d->w - 1) / d->stride_w + 1;
+    long long* SA = reinterpret_cast<long long*>(scratch);
+    IQ_CUDA_CHECK(cudaMemsetAsync(SA, 0, (size_t)d->c * sizeof(long long), st));
+    const int C4 = d->c / 4;
+    // a block is kThreads / C4 pixel lanes of all channels (C4 <= kThreads, dividing it), or
+    // for wider rows the general mapping does not apply
+    if (C4 > kThreads || kThreads % C4) return IQ_ERR_UNSUPPORTED;
+    const int lanes = kThreads / C4;
+    int64_t blocks = ((int64_t)d->n * P * Q + lanes * 16 - 1) / (lanes * 16);
+    if (blocks > 152 * 8) blocks = 152 * 8;
+    if (blocks < 1) blocks = 1;
+    k_input_colsums<<<(unsigned)blocks, kThreads, 0, st>>>(x, d->n, d->h, d->w, d->c, P, Q,
+                                                           d->stride_h, d->stride_w, SA);
+    IQ_LAUNCH_CHECK();
+    k_input_gemv<<<(unsigned)(((int64_t)d->k * 32 + kThreads - 1) / kThreads), kThreads, 0, st>>>(
+        SA, w, d->k, d->c, s1);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+// bytes of the fp16 copy of the input (or of its im2col) in the forward's workspace
+size_t conv_fwd_xf_bytes(const iq_conv_desc* d) {
+    int64_t kdim = (int64_t)d->r * d->s * (d->c / d->groups);
+    int64_t kpad = (kdim + 63) / 64 * 64;
+    size_t xb = (size_t)d->n * d->h * d->w * d->c * 2;
+    if (d->c % 64 != 0 && kpad <= IM2COL_MAX_K) {
+        const int P = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1) / d->stride_h + 1;
+        const int Q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1) / d->stride_w + 1;
+        const size_t ib = (size_t)d->n * P * Q * kpad * 2;
+        if (ib > xb) xb = ib;
+    }
+    return xb;
+}
+
 size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d) {
     int64_t kdim = (int64_t)d->r * d->s * (d->c / d->groups);
     int64_t kpad = (kdim + 63) / 64 * 64;
@@ -2462,7 +2570,7 @@ size_t conv_fwd_tc_ws_bytes(const iq_conv_desc* d) {
         const size_t ib = (size_t)d->n * P * Q * kpad * 2;
         if (ib > xb) xb = ib;
     }
-    return acts16_offset(wb) + xb + 512;
+    return (acts16_offset(wb) + xb + 511) / 256 * 256 + input_sums_bytes(d);
 }
 
 bool conv_fwd_tc_supported(const iq_conv_desc* d) {
@@ -2475,6 +2583,7 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
                       bool* done, const __half* xf_given, unsigned st_mask) {
     *done = false;
     if (!conv_fwd_tc_supported(d) || ((uintptr_t)x & 15) != 0 || !get_encode()) return IQ_OK;
+    const iq_conv_desc* d0 = d;
     iq_conv_desc dflat;
     d = flat_pointwise(d, &dflat);
     TcP p;
@@ -2493,6 +2602,12 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     p.kb_per_split = p.nkb_total;
     p.npq = 0;
     if (p.nkb_total > MAX_KB_INT32) return IQ_OK;   // cannot happen under the CRS bound
+    // for an expanding 1x1 layer the pixel-major kernel leaves the channel sums to input_sums
+    // (the other kernels, and other layers, take them from their epilogues)
+    const bool in_sums = (st_mask & TC_STATS_SUM) != 0 && input_sums_ok(d0) &&
+                         d0->c / 4 <= kThreads && kThreads % (d0->c / 4) == 0;
+    TcP pt = p;
+    if (in_sums) pt.st_mask &= ~(int)TC_STATS_SUM;
     char* wsb = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
     __half* wf = reinterpret_cast<__half*>(wsb);
     int* err = tc_status_ptr();
@@ -2505,7 +2620,7 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
     iq_status r = encode_weights(wf, p.K, p.kpad, pick_bn(p.ncols), &map);
     if (r != IQ_OK) return r;
     __half* xf = reinterpret_cast<__half*>(wsb + acts16_offset((size_t)p.K * p.kpad * 2));
-    bool used = false;
+    bool used = false, via_t = false;
     if (!p.tap_mode && p.kpad <= IM2COL_MAX_K && p.C % 4 == 0 && p.cstride % 4 == 0 &&
         p.cofs % 4 == 0 && !tma16_disabled() && p.N <= 65535 && p.P <= 65535) {
         // few input channels: the fp16 im2col, then a 1x1 problem over kpad channels
@@ -2523,9 +2638,12 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
                 if (r != IQ_OK) return r;
             }
             if (!used) {
-                r = try_launch_t(map, q, nullptr, xf, false, acc, nullptr, s1, hi, lo, err, st,
+                TcP qt = q;
+                qt.st_mask = pt.st_mask;
+                r = try_launch_t(map, qt, nullptr, xf, false, acc, nullptr, s1, hi, lo, err, st,
                                  &used);
                 if (r != IQ_OK) return r;
+                via_t = used;
             }
         }
     }
@@ -2535,10 +2653,18 @@ iq_status conv_fwd_tc(const iq_conv_desc* d, const int8_t* x, const int8_t* w, i
         const bool convert = xf_given == nullptr;
         r = try_launch_c(wf, p.K, p, x, xc, convert, acc, s1, hi, lo, err, st, &used);
         if (r != IQ_OK) return r;
-        if (!used) r = try_launch_t(map, p, x, xc, convert, acc, nullptr, s1, hi, lo, err, st, &used);
+        if (!used) {
+            r = try_launch_t(map, pt, x, xc, convert, acc, nullptr, s1, hi, lo, err, st, &used);
+            via_t = used;
+        }
         if (r != IQ_OK) return r;
     }
     if (!used) r = launch(map, p, 1, x, nullptr, acc, nullptr, s1, hi, lo, err, st);
+    if (r == IQ_OK && via_t && in_sums) {
+        char* scratch = wsb + (acts16_offset((size_t)p.K * p.kpad * 2) +
+                               conv_fwd_xf_bytes(d0) + 511) / 256 * 256;
+        r = input_sums(d0, x, w, scratch, s1, st);
+    }
     if (r == IQ_OK) *done = true;
     return r;
 }
