@@ -89,6 +89,10 @@ struct TcP {
     int64_t npq;     // WGRAD: reduction length N*P*Q
     int slices;      // FWD on the all-TMA kernel: reduction slices (channel ranges of C
     int slice_rows;  // channels each) run as separate tiles; weight rows per slice
+    int skip_taps;   // rectangle kernels: a tile skips the taps whose input box lies wholly
+                     // outside the image (their A tiles would be all zero fill): the row taps
+    uint32_t band_r[64];   // that meet the image for tile row band pt (bit r), the column
+    uint32_t band_s[64];   // taps for column band qt (bit s)
 };
 
 // ---------------------------------------------------------------- FWD gather (K-major A)
@@ -1106,11 +1110,32 @@ struct RectPos {
     int tile, kb;
     int n, p0, q0, n0;
     int slice;            // reduction slice (tiles beyond mt nt)
+    int e, ne;            // k-block kb is the tile's e-th of ne
+    int r, s, c0;         // its tap and first channel
+    uint32_t rm, sm;      // the tile's taps (bits r of rm, s of sm) in k-block order
 };
 
-__device__ __forceinline__ void rpos_set(RectPos& q, int tile, const RectGrid& g, int BN) {
+// whether an output index o in [o_lo, o_hi] reads an input index o stride + off in [0, extent)
+// (stride 1 or 2, as the rectangle kernels take)
+__host__ __device__ __forceinline__ bool tap_meets(int extent, int o_lo, int o_hi, int stride,
+                                                   int off) {
+    const int sh = stride - 1;
+    const int lo = off >= 0 ? 0 : (-off + sh) >> sh;
+    const int top = extent - 1 - off;
+    if (top < 0) return false;
+    const int hi = top >> sh;
+    return (lo > o_lo ? lo : o_lo) <= (hi < o_hi ? hi : o_hi);
+}
+
+// Tile `tile` and its first k-block.  k-blocks run over taps (r, s) in row-major order, 64
+// channels at a time; with skip_taps a tile keeps only the rows r and columns s of taps that
+// read inside the image for some of its output pixels (all of them if that leaves none).
+__device__ __forceinline__ void rpos_set(RectPos& q, int tile, const TcP& p, const RectGrid& g,
+                                         int BN) {
     q.tile = tile;
     q.kb = 0;
+    q.e = 0;
+    q.ne = 0;
     if (tile >= g.total) return;
     const int mt = tile % g.mt;
     const int rest = tile / g.mt;
@@ -1121,11 +1146,53 @@ __device__ __forceinline__ void rpos_set(RectPos& q, int tile, const RectGrid& g
     q.n = mt / (g.QT * g.PT);
     q.p0 = pt * g.BH;
     q.q0 = qt * g.BW;
+    if (!p.skip_taps) {
+        q.rm = (1u << p.R) - 1u;
+        q.sm = (1u << p.S) - 1u;
+        q.r = q.s = q.c0 = 0;
+        q.ne = p.nkb_total;
+        return;
+    }
+    uint32_t rm = (1u << p.R) - 1u, sm = (1u << p.S) - 1u;
+    {
+        const uint32_t a = p.band_r[pt], b = p.band_s[qt];
+        if (a && b) { rm = a; sm = b; }
+    }
+    q.rm = rm;
+    q.sm = sm;
+    q.r = __ffs(rm) - 1;
+    q.s = __ffs(sm) - 1;
+    q.c0 = 0;
+    q.ne = __popc(rm) * __popc(sm) * (p.C / BK);
+    q.kb = (q.r * p.S + q.s) * (p.C / BK);
 }
 
 __device__ __forceinline__ void rpos_next(RectPos& q, const TcP& p, const RectGrid& g, int BN) {
     if (q.tile >= g.total) return;
-    if (++q.kb >= p.nkb_total) rpos_set(q, q.tile + gridDim.x, g, BN);
+    if (++q.e >= q.ne) {
+        rpos_set(q, q.tile + gridDim.x, p, g, BN);
+        return;
+    }
+    q.c0 += BK;
+    if (!p.skip_taps) {          // every tap: k-blocks in plain order
+        q.kb++;
+        if (q.c0 >= p.C) {
+            q.c0 = 0;
+            if (++q.s == p.S) { q.s = 0; q.r++; }
+        }
+        return;
+    }
+    if (q.c0 >= p.C) {
+        q.c0 = 0;
+        const uint32_t sn = q.sm & (0xfffffffeu << q.s);      // the tile's taps after s
+        if (sn) {
+            q.s = __ffs(sn) - 1;
+        } else {
+            q.s = __ffs(q.sm) - 1;
+            q.r = __ffs(q.rm & (0xfffffffeu << q.r)) - 1;
+        }
+    }
+    q.kb = (q.r * p.S + q.s) * (p.C / BK) + q.c0 / BK;
 }
 
 // per-channel statistics of LDW columns over the warp's 32 rows (OUT_STATS): the maximum,
@@ -1275,22 +1342,26 @@ __device__ __forceinline__ void wpos_next(WgPos& q, const TcP& p, const RectGrid
 template <bool WG>
 struct TPos;
 
+// idx(): the k-block's place in its tile, cnt(): the tile's k-blocks
+// (the MMA issuer and the epilogue only count a tile's k-blocks: next() does not track taps)
 template <>
 struct TPos<false> : RectPos {
-    int nkb;
     __device__ void set(int t, const TcP& p, const RectGrid& g, int BN) {
-        rpos_set(*this, t, g, BN);
-        nkb = p.nkb_total;
+        rpos_set(*this, t, p, g, BN);
     }
     __device__ void next(const TcP& p, const RectGrid& g, int BN) {
-        rpos_next(*this, p, g, BN);
+        if (tile < g.total && ++e >= ne) rpos_set(*this, tile + gridDim.x, p, g, BN);
     }
+    __device__ int idx() const { return e; }
+    __device__ int cnt() const { return ne; }
 };
 
 template <>
 struct TPos<true> : WgPos {
     __device__ void set(int t, const TcP& p, const RectGrid& g, int BN) { wpos_set(*this, t, p, g, BN); }
     __device__ void next(const TcP& p, const RectGrid& g, int BN) { wpos_next(*this, p, g, BN); }
+    __device__ int idx() const { return kb; }
+    __device__ int cnt() const { return nkb; }
 };
 
 // WG: the weight gradient.  A k-block is a BW x BH rectangle of 64 output pixels of one
@@ -1420,8 +1491,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             }
         } else {
             RectPos q;
-            rpos_set(q, blockIdx.x, g, BN);
-            int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
+            rpos_set(q, blockIdx.x, p, g, BN);
             while (q.tile < g.total) {
                 if (!tc::mbar_wait_warp(&bars->empty[s], ph ^ 1, abort_flag)) {
                     bars->abort = 1;
@@ -1431,9 +1501,9 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 uint8_t* st = smem + s * STAGE_BYTES;
                 tc::mbar_expect_tx_e(&bars->full[s], tx);
                 if (side_a)
-                    tc::tma_load_4d_e(st, &amap, &bars->full[s], p.cofs + q.slice * p.C + c0,
-                                      q.q0 * p.sw + ss * p.dw - p.pw,
-                                      q.p0 * p.sh + r * p.dh - p.ph, q.n);
+                    tc::tma_load_4d_e(st, &amap, &bars->full[s], p.cofs + q.slice * p.C + q.c0,
+                                      q.q0 * p.sw + q.s * p.dw - p.pw,
+                                      q.p0 * p.sh + q.r * p.dh - p.ph, q.n);
                 else
                     tc::tma_load_2d_e(st + A_BYTES, &wmap, &bars->full[s], q.kb * BK,
                                       q.slice * p.slice_rows + q.n0);
@@ -1441,17 +1511,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
                 issued = (int)kbc + 1;
                 kbc++;
                 if (++s == NST) { s = 0; ph ^= 1; }
-                const int tile = q.tile;
                 rpos_next(q, p, g, BN);
-                if (q.tile != tile) {
-                    r = ss = c0 = 0;
-                } else {
-                    c0 += BK;
-                    if (c0 >= p.C) {
-                        c0 = 0;
-                        if (++ss == p.S) { ss = 0; r++; }
-                    }
-                }
             }
         }
         if (*abort_flag) {
@@ -1471,8 +1531,8 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             TPos<WG> q;
             q.set(blockIdx.x, p, g, BN);
             while (ok && q.tile < g.total) {
-                const bool first = (q.kb % CHUNK_KB) == 0;
-                const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
+                const bool first = (q.idx() % CHUNK_KB) == 0;
+                const bool last = ((q.idx() % CHUNK_KB) == CHUNK_KB - 1) || q.idx() == q.cnt() - 1;
                 const uint32_t buf = cc & 1;
                 if (first && cc >= 2 &&
                     !tc::mbar_wait_warp(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
@@ -1531,7 +1591,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         const int wr0 = (warp & 3) << 5;      // first tile row (pixel) of the warp
         uint8_t* stg = smem + CfgT<BN>::OUT_OFF + (warp - 4) * 2048;
         while (ok && q.tile < g.total) {
-            const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
+            const int nch = (q.cnt() + CHUNK_KB - 1) / CHUNK_KB;
             // the sums start at minus the FOLD_BIAS of the tile's nch chunks
             const int sum0 = (int)(0u - (uint32_t)nch * FOLD_BIAS);
 #pragma unroll
@@ -1708,8 +1768,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         int s = 0;
         uint32_t ph = 0;
         RectPos q;
-        rpos_set(q, blockIdx.x, g, CM_CH);
-        int r = 0, ss = 0, c0 = 0;          // tap and channel of k-block q.kb
+        rpos_set(q, blockIdx.x, p, g, CM_CH);
         uint32_t kbc = 0;
         int issued = 0;
         while (q.tile < g.total) {
@@ -1722,25 +1781,15 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             tc::mbar_expect_tx_e(&bars->full[s], tx);
             if (side_a)     // A: weight rows n0 .. n0 + 127 (zero past the last channel)
                 tc::tma_load_2d_e(st, &wmap, &bars->full[s], q.kb * BK, q.n0);
-            else            // B: the 256 input pixels of tap (r, ss), channels c0 .. c0 + 63
-                tc::tma_load_4d_e(st + A_BYTES, &amap, &bars->full[s], p.cofs + c0,
-                                  q.q0 * p.sw + ss * p.dw - p.pw, q.p0 * p.sh + r * p.dh - p.ph,
-                                  q.n);
+            else            // B: the 256 input pixels of tap (r, s), channels c0 .. c0 + 63
+                tc::tma_load_4d_e(st + A_BYTES, &amap, &bars->full[s], p.cofs + q.c0,
+                                  q.q0 * p.sw + q.s * p.dw - p.pw,
+                                  q.p0 * p.sh + q.r * p.dh - p.ph, q.n);
             tc::mbar_arrive_e(&bars->full[s]);
             issued = (int)kbc + 1;
             kbc++;
             if (++s == NST) { s = 0; ph ^= 1; }
-            const int tile = q.tile;
             rpos_next(q, p, g, CM_CH);
-            if (q.tile != tile) {
-                r = ss = c0 = 0;
-            } else {
-                c0 += BK;
-                if (c0 >= p.C) {
-                    c0 = 0;
-                    if (++ss == p.S) { ss = 0; r++; }
-                }
-            }
         }
         if (*abort_flag) {
             for (int kb = (issued > NST ? issued - NST : 0); kb < issued; kb++)
@@ -1758,8 +1807,8 @@ __global__ void __launch_bounds__(THREADS_T, 1)
             TPos<false> q;
             q.set(blockIdx.x, p, g, CM_CH);
             while (ok && q.tile < g.total) {
-                const bool first = (q.kb % CHUNK_KB) == 0;
-                const bool last = ((q.kb % CHUNK_KB) == CHUNK_KB - 1) || q.kb == q.nkb - 1;
+                const bool first = (q.idx() % CHUNK_KB) == 0;
+                const bool last = ((q.idx() % CHUNK_KB) == CHUNK_KB - 1) || q.idx() == q.cnt() - 1;
                 const uint32_t buf = cc & 1;
                 if (first && cc >= 2 &&
                     !tc::mbar_wait_warp(&bars->acce[buf], ((cc >> 1) - 1) & 1, abort_flag)) {
@@ -1807,7 +1856,7 @@ __global__ void __launch_bounds__(THREADS_T, 1)
         q.set(blockIdx.x, p, g, CM_CH);
         int sum[CW];
         while (ok && q.tile < g.total) {
-            const int nch = (q.nkb + CHUNK_KB - 1) / CHUNK_KB;
+            const int nch = (q.cnt() + CHUNK_KB - 1) / CHUNK_KB;
             // the sums start at minus the FOLD_BIAS of the tile's nch chunks
             const int sum0 = (int)(0u - (uint32_t)nch * FOLD_BIAS);
 #pragma unroll
@@ -2268,7 +2317,7 @@ bool tma16_disabled() {
 // 2, aligned slices, a rectangle tiling with little waste)
 bool tma16_ok(const TcP& p, TmaTile* t) {
     if (tma16_disabled() || !p.tap_mode || p.sh > 2 || p.sw > 2 || (p.cstride % 8) ||
-        (p.cofs % 64))
+        (p.cofs % 64) || p.R > 16 || p.S > 16)
         return false;
     if (!pick_tma_tile(p.P, p.Q, t, 0.6)) return false;
     return t->BW * p.sw <= 256 && t->BH * p.sh <= 256;
@@ -2295,6 +2344,31 @@ iq_status launch_t(const CUtensorMap& wmap, const CUtensorMap& amap, const CUten
     return IQ_OK;
 }
 
+// whether a BH x BW tile of the P x Q output (tiles of the tiling t) can skip a tap: some
+// tile row band or column band misses the image for some tap
+// (fills the band masks of q; false when no tile can skip, or there are over 64 bands)
+bool taps_skippable(TcP& q, const TmaTile& t) {
+    if ((q.R <= 1 && q.S <= 1) || t.PT > 64 || t.QT > 64) return false;
+    bool any = false;
+    for (int pt = 0; pt < t.PT; pt++) {
+        const int p0 = pt * t.BH, pe = std::min(p0 + t.BH, q.P) - 1;
+        uint32_t m = 0;
+        for (int r = 0; r < q.R; r++)
+            if (tap_meets(q.H, p0, pe, q.sh, r * q.dh - q.ph)) m |= 1u << r;
+        q.band_r[pt] = m;
+        any |= m != (1u << q.R) - 1u;
+    }
+    for (int qt = 0; qt < t.QT; qt++) {
+        const int q0 = qt * t.BW, qe = std::min(q0 + t.BW, q.Q) - 1;
+        uint32_t m = 0;
+        for (int s = 0; s < q.S; s++)
+            if (tap_meets(q.W, q0, qe, q.sw, s * q.dw - q.pw)) m |= 1u << s;
+        q.band_s[qt] = m;
+        any |= m != (1u << q.S) - 1u;
+    }
+    return any;
+}
+
 // widen the input codes into xf and run the all-TMA kernel; *used = false when not taken
 iq_status try_launch_t(const CUtensorMap& wmap, const TcP& p, const int8_t* x, __half* xf,
                        bool convert, int32_t* out32, long long* out64, unsigned long long* s1,
@@ -2313,6 +2387,7 @@ iq_status try_launch_t(const CUtensorMap& wmap, const TcP& p, const int8_t* x, _
     iq_status r = encode_acts16(xf, p.N, p.H, p.W, p.cstride, t, p.sh, p.sw, &amap);
     if (r != IQ_OK) return r;
     TcP q = p;
+    q.skip_taps = taps_skippable(q, t);
     // int32 output with statistics: TMA stores of the warps' pixel boxes
     q.tma_out = p.out == OUT_STATS && out32 && p.slices <= 1 &&
                 encode_out32(out32, p.N, p.P, p.Q, p.ncols, t, &omap) == IQ_OK;
@@ -2331,7 +2406,7 @@ iq_status try_launch_t(const CUtensorMap& wmap, const TcP& p, const int8_t* x, _
 // little waste)
 bool cm_ok(const TcP& p, TmaTile* t) {
     if (p.ncols > CM_CH || tma16_disabled() || !p.tap_mode || p.sh > 2 || p.sw > 2 ||
-        (p.cstride % 8) || (p.cofs % 64))
+        (p.cstride % 8) || (p.cofs % 64) || p.R > 16 || p.S > 16)
         return false;
     if (!pick_tma_tile(p.P, p.Q, t, 0.6, CM_PIX)) return false;
     return t->BW * p.sw <= 256 && t->BH * p.sh <= 256;
@@ -2366,8 +2441,10 @@ iq_status try_launch_c(const __half* wf, int rows, const TcP& p, const int8_t* x
     int bw_log2 = 0;
     while ((1 << bw_log2) < t.BW) bw_log2++;
     const int grid = g.total < num_sms() ? g.total : num_sms();
+    TcP pc = p;
+    pc.skip_taps = taps_skippable(pc, t);
     kt_pre(st);
-    k_conv_tcc<<<grid, THREADS_T, CfgT<256>::SMEM, st>>>(wmap, amap, p, g, bw_log2, out32, s1,
+    k_conv_tcc<<<grid, THREADS_T, CfgT<256>::SMEM, st>>>(wmap, amap, pc, g, bw_log2, out32, s1,
                                                           hi, lo, err);
     IQ_LAUNCH_CHECK();
     kt_post(st, IQ_KERNEL_CONV_CHANNEL_MAJOR);
@@ -2387,6 +2464,7 @@ void fill_geom(TcP& p, const iq_conv_desc* d) {
     p.slice_rows = 0;
     p.st_mask = TC_STATS_SUM | TC_STATS_LO;
     p.tma_out = 0;
+    p.skip_taps = 0;
 }
 
 // k-blocks per split so that each split's int32 running sum cannot overflow
