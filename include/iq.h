@@ -154,11 +154,13 @@ enum {
     IQ_KERNEL_SQ_CODES = 17,           /* SQ codes of int32 / int64 sums (k_sq_i32_i8x4, k_sq_int) */
     IQ_KERNEL_CODES_TO_F16 = 18,       /* fp16 carrier copy of int8 codes (k_codes_to_f16)       */
     IQ_KERNEL_ABSMAX = 19,             /* max |q| pass of SQ / RQ (k_absmax_int)                 */
-    IQ_KERNEL_RQ_CODES = 20            /* RQ codes (k_rq_int)                                    */
+    IQ_KERNEL_RQ_CODES = 20,           /* RQ codes (k_rq_int)                                    */
+    IQ_KERNEL_GEMM_NIBBLE = 21         /* nibble-split fp8 GEMM (k_gemm_nibble)                  */
 };
 typedef struct iq_kernel_time {
     int32_t kernel;     /* IQ_KERNEL_* */
-    int32_t op;         /* 1 iq_conv_fwd, 2 iq_conv_dgrad, 3 iq_conv_wgrad; 0 bandwidth kernels */
+    int32_t op;         /* 1 iq_conv_fwd, 2 iq_conv_dgrad, 3 iq_conv_wgrad, 4 iq_gemm_s8_nibble;
+                           0 bandwidth kernels */
     int32_t launches;   /* bracketed launches */
     int32_t pad;
     double ms;          /* summed event time of those launches, milliseconds */
@@ -223,6 +225,38 @@ iq_status iq_requantize(const void* q, int in_dtype, int64_t n, const double* s_
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
                         void* codes, int out_dtype, double* s_out, void* ws, size_t ws_bytes,
                         iq_stream stream);
+
+/* iq_requantize_per_channel -- Eq. (ScaleQ) with a per-channel Scale: Eq. (ScaleFactor)'s
+ * maximum taken over each channel's elements instead of the whole tensor (the per-channel
+ * reading of Scale(x); the paper's networks use the per-tensor form, iq_requantize).
+ *   q        integer codes viewed as [outer][c][inner]: NHWC activations or errors with
+ *            outer = n h w, inner = 1; NCHW with outer = n, inner = h w; KRSC filters or
+ *            filter gradients by output channel with outer = 1, inner = r s c
+ *   in_dtype IQ_I32 or IQ_I64 (|q| < 2^40);  s_in device double, the scale of q
+ *   relu     nonzero: ReLU(q) is quantized
+ *   k        2..16;  out_dtype IQ_I8 (k <= 8), IQ_I16 or IQ_I32
+ *   codes    out, like q;  s_out out device double[c]
+ * With M_c = max |q| over channel c: code = clip(floor((2^k q + M_c) / (2 M_c))),
+ * s_out[c] = (s_in M_c) 2^(1-k); a channel with M_c = 0 gets zero codes and s_in 2^(1-k).
+ * Workspace: iq_requantize_per_channel_workspace_size(c). */
+iq_status iq_requantize_per_channel_workspace_size(int32_t c, size_t* bytes);
+iq_status iq_requantize_per_channel(const void* q, int in_dtype, int64_t outer, int32_t c,
+                                    int64_t inner, const double* s_in, int k, int relu,
+                                    void* codes, int out_dtype, double* s_out, void* ws,
+                                    size_t ws_bytes, iq_stream stream);
+
+/* iq_gemm_s8_nibble -- C = A B^T for int8 A [m][k], B [n][k] (k contiguous) into int32 C
+ * [m][n], exactly, on the fp8 tensor-core path: each code splits into its signed high nibble
+ * and its low nibble (v = 16 h + l, both exact in e4m3), and four tcgen05 kind::f8f6f4 MMAs
+ * per k-step accumulate 256 H_A H_B^T + 16 (H_A L_B^T + L_A H_B^T) + L_A L_B^T in three
+ * exact fp32 sums.  An ablation of the exact tensor-core routes to the int8 products of
+ * Sec. 3.2-3.3, beside the fp16 carriers of iq_conv_* (a 1x1 iq_conv_fwd is the same GEMM).
+ * m, n multiples of 128, k a multiple of 128 and at most 65536 (else IQ_ERR_UNSUPPORTED);
+ * pointers 16-byte aligned.  Workspace: iq_gemm_s8_nibble_workspace_size (the split
+ * operands, 2 (m + n) k bytes). */
+iq_status iq_gemm_s8_nibble_workspace_size(int32_t m, int32_t n, int32_t k, size_t* bytes);
+iq_status iq_gemm_s8_nibble(const int8_t* a, const int8_t* b, int32_t* c, int32_t m, int32_t n,
+                            int32_t k, void* ws, size_t ws_bytes, iq_stream stream);
 
 /* iq_weight_requant -- forward weights from master weights, Eqs. (WQ0),(WQ1):
  * master codes m on the k_u grid (value m 2^(1-k_u)), wq = clip(floor((m + 2^(k_u-k_w-1))

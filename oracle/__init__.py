@@ -95,6 +95,8 @@ def _declare(L):
     for f in ("or_conv_fwd", "or_conv_dgrad", "or_conv_wgrad"):
         getattr(L, f).argtypes = [C.POINTER(ConvDesc), _P, _P, _P]
         getattr(L, f + "_at").argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _I64, _P]
+    L.or_sq_per_channel.argtypes = [_P, _I64, _I64, _I64, _D, _I32, _I32, _P, _P]
+    L.or_sq_per_channel.restype = None
     L.or_sq_at.argtypes = [_P, _I64, _I64, _D, _I32, _I32, _P]
     L.or_sq_at.restype = _D
     L.or_rq_at.argtypes = [_P, _P, _I64, _I64, _D, _I32, _I32, _U64, _U64, _U64, _U64, _P]
@@ -172,6 +174,17 @@ def sq_int(q, s: float, k: int, relu: bool = False):
     out = np.empty(q.shape, np.int32)
     so = lib().or_sq_int64(_ptr(q), q.size, float(s), k, int(relu), _ptr(out))
     return out, so
+
+
+def sq_per_channel(q, outer: int, C: int, inner: int, s: float, k: int, relu: bool = False):
+    """Eq. (ScaleQ) with a per-channel Scale (Eq. (ScaleFactor) over each channel's elements)
+    on an integer-coded tensor viewed as [outer][C][inner]: (codes, scales[C])."""
+    q = _c(q, np.int64)
+    assert q.size == outer * C * inner
+    out = np.empty(q.shape, np.int32)
+    sc = np.empty(C, np.float64)
+    lib().or_sq_per_channel(_ptr(q), outer, C, inner, float(s), k, int(relu), _ptr(out), _ptr(sc))
+    return out, sc
 
 
 def sq_at(q, M: int, s: float, k: int, relu: bool = False):

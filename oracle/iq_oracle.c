@@ -158,6 +158,38 @@ double or_sq_int32(const int32_t* q, int64_t n, double s, int k, int relu,
     return r;
 }
 
+/* Eqs. (ScaleFactor),(ScaleQ) with Scale(x) taken per channel (the per-channel reading of
+ * Scale): element (o, c, i) of q sits at (o C + c) inner + i; M_c = max over o and i of |q|
+ * (of ReLU(q) when relu); code = clip(floor((2^k q + M_c) / (2 M_c))) = floor(2^(k-1) q / M_c
+ * + 1/2) clipped to +-(2^(k-1) - 1); scale_c = s M_c 2^(1-k) (s 2^(1-k) when M_c = 0, codes 0). */
+void or_sq_per_channel(const int64_t* q, int64_t outer, int64_t C, int64_t inner, double s,
+                       int k, int relu, int32_t* code, double* scale) {
+    for (int64_t c = 0; c < C; c++) {
+        int64_t M = 0;
+        for (int64_t o = 0; o < outer; o++)
+            for (int64_t i = 0; i < inner; i++) {
+                int64_t v = q[(o * C + c) * inner + i];
+                if (relu && v < 0) v = 0;
+                int64_t a = v < 0 ? -v : v;
+                if (a > M) M = a;
+            }
+        scale[c] = M ? ldexp(s * (double)M, 1 - k) : ldexp(s, 1 - k);
+        for (int64_t o = 0; o < outer; o++)
+            for (int64_t i = 0; i < inner; i++) {
+                const int64_t at = (o * C + c) * inner + i;
+                int64_t v = q[at];
+                if (relu && v < 0) v = 0;
+                if (!M) {
+                    code[at] = 0;
+                    continue;
+                }
+                i128 num = ((i128)v << k) + M;
+                code[at] = (int32_t)clamp64((int64_t)floordiv128(num, (i128)2 * M), -qmax(k),
+                                            qmax(k));
+            }
+    }
+}
+
 /* ------------------------------------------------------------------ */
 /* Sec. 3.1.3: stochastic rounding with a counter-based generator       */
 /* ------------------------------------------------------------------ */

@@ -17,7 +17,7 @@ LIB = os.path.join(BUILD, "libiq.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
 SOURCES = ["iq_quant.cu", "iq_bn.cu", "iq_conv.cu", "iq_conv_tc.cu", "iq_glue.cu", "iq_merge.cu",
-           "iq_head.cu"]
+           "iq_head.cu", "iq_gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", INCLUDE]

@@ -470,6 +470,118 @@ __global__ void k_relu_bwd(const int8_t* __restrict__ ea, const int8_t* __restri
     for (int64_t i = n16 * 16 + i0; i < n; i += stride) e[i] = a[i] > 0 ? ea[i] : 0;
 }
 
+// ------------------------------------------------------------------ per-channel Scale
+// Eqs. (ScaleFactor),(ScaleQ) with the maximum taken over each channel instead of the whole
+// tensor; q is viewed as [outer][C][inner] (channel-innermost NHWC: inner = 1).
+
+// inner == 1: thread (x, y) owns channel 256 x + threadIdx.x and rows y, y + gridDim.y, ...
+// (a warp reads 32 neighbouring channels of a row)
+template <typename T>
+__global__ void k_pc_max_c(const T* __restrict__ q, int64_t outer, int32_t C, int relu,
+                           unsigned long long* __restrict__ M) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= C) return;
+    uint64_t m = 0;
+    for (int64_t o = blockIdx.y; o < outer; o += gridDim.y) {
+        int64_t v = (int64_t)q[o * C + c];
+        if (relu && v < 0) v = 0;
+        const uint64_t a = (uint64_t)(v < 0 ? -v : v);
+        m = a > m ? a : m;
+    }
+    if (m) atomicMax(M + c, (unsigned long long)m);
+}
+
+// inner > 1: one warp per row (o, c) of `inner` contiguous elements
+template <typename T>
+__global__ void k_pc_max_rows(const T* __restrict__ q, int64_t rows, int32_t C, int64_t inner,
+                              int relu, unsigned long long* __restrict__ M) {
+    const int lane = threadIdx.x & 31;
+    const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t row = w0; row < rows; row += nw) {         // warp-uniform
+        uint64_t m = 0;
+        for (int64_t i = lane; i < inner; i += 32) {
+            int64_t v = (int64_t)q[row * inner + i];
+            if (relu && v < 0) v = 0;
+            const uint64_t a = (uint64_t)(v < 0 ? -v : v);
+            m = a > m ? a : m;
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+            const uint64_t t = __shfl_xor_sync(0xffffffffu, m, o);
+            m = t > m ? t : m;
+        }
+        if (lane == 0 && m) atomicMax(M + (row % C), (unsigned long long)m);
+    }
+}
+
+// per channel: the divisor by 2 M_c and the output scale s_in M_c 2^(1-k)
+__global__ void k_pc_params(const unsigned long long* __restrict__ M, int32_t C,
+                            const double* __restrict__ s_in, int k, UDiv* __restrict__ div,
+                            double* __restrict__ s_out) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= C) return;
+    const uint64_t m = M[c];
+    div[c] = make_udiv(m ? 2 * m : 1);
+    s_out[c] = m ? ldexp(__dmul_rn(*s_in, (double)m), 1 - k) : ldexp(*s_in, 1 - k);
+}
+
+// code = clip(floor((2^k (v + M_c) + M_c) / (2 M_c)) - 2^(k-1)), 0 when M_c = 0
+template <typename T>
+__global__ void k_pc_codes(const T* __restrict__ q, int64_t n, int32_t C, int64_t inner, int k,
+                           int relu, const unsigned long long* __restrict__ M,
+                           const UDiv* __restrict__ div, void* __restrict__ out, int dtype) {
+    const int64_t lim = qmax(k);
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)((i / inner) % C);
+        const uint64_t m = M[c];
+        int64_t v = (int64_t)q[i];
+        if (relu && v < 0) v = 0;
+        int64_t code = 0;
+        if (m) {
+            const uint64_t num = ((uint64_t)(v + (int64_t)m) << k) + m;
+            code = clamp64((int64_t)udiv(num, div[c]) - (int64_t(1) << (k - 1)), -lim, lim);
+        }
+        store_code(out, dtype, i, code);
+    }
+}
+
+size_t pc_ws_bytes(int32_t C) {
+    return 256 + ((size_t)C * 8 + 255) / 256 * 256 + (size_t)C * sizeof(UDiv) + 256;
+}
+
+template <typename T>
+iq_status pc_run(const T* q, int64_t outer, int32_t C, int64_t inner, const double* s_in, int k,
+                 int relu, void* out, int dtype, double* s_out, void* ws, cudaStream_t st) {
+    char* b = (char*)(((uintptr_t)ws + 255) & ~uintptr_t(255));
+    unsigned long long* M = (unsigned long long*)b;
+    UDiv* div = (UDiv*)(b + ((size_t)C * 8 + 255) / 256 * 256);
+    IQ_CUDA_CHECK(cudaMemsetAsync(M, 0, (size_t)C * 8, st));
+    const int64_t n = outer * C * inner;
+    if (n > 0) {
+        if (inner == 1) {
+            const unsigned gx = (unsigned)((C + kThreads - 1) / kThreads);
+            int64_t gy = (152 * 8 + gx - 1) / gx;
+            if (gy > outer) gy = outer;
+            if (gy > 65535) gy = 65535;
+            k_pc_max_c<T><<<dim3(gx, (unsigned)gy), kThreads, 0, st>>>(q, outer, C, relu, M);
+        } else {
+            k_pc_max_rows<T><<<grid_for(outer * C * 32), kThreads, 0, st>>>(q, outer * C, C,
+                                                                            inner, relu, M);
+        }
+        IQ_LAUNCH_CHECK();
+    }
+    k_pc_params<<<(C + kThreads - 1) / kThreads, kThreads, 0, st>>>(M, C, s_in, k, div, s_out);
+    IQ_LAUNCH_CHECK();
+    if (n > 0) {
+        k_pc_codes<T><<<grid_for(n), kThreads, 0, st>>>(q, n, C, inner, k, relu, M, div, out,
+                                                        dtype);
+        IQ_LAUNCH_CHECK();
+    }
+    return IQ_OK;
+}
+
 }  // namespace iq
 
 using namespace iq;
@@ -589,6 +701,30 @@ extern "C" iq_status iq_requantize(const void* q, int in_dtype, int64_t n, const
     if (!ws || ws_bytes < requant_ws_bytes()) return IQ_ERR_WORKSPACE;
     return requant_int(q, in_dtype, n, s_in, k, mode, seed, layer, step, tag, codes, out_dtype,
                        s_out, ws, (cudaStream_t)stream);
+}
+
+extern "C" iq_status iq_requantize_per_channel_workspace_size(int32_t c, size_t* bytes) {
+    if (!bytes || c <= 0) return IQ_ERR_INVALID_ARG;
+    *bytes = pc_ws_bytes(c);
+    return IQ_OK;
+}
+
+extern "C" iq_status iq_requantize_per_channel(const void* q, int in_dtype, int64_t outer,
+                                               int32_t c, int64_t inner, const double* s_in,
+                                               int k, int relu, void* codes, int out_dtype,
+                                               double* s_out, void* ws, size_t ws_bytes,
+                                               iq_stream stream) {
+    if (outer < 0 || inner < 1 || c <= 0 || !s_in || !s_out) return IQ_ERR_INVALID_ARG;
+    if (outer > 0 && (!q || !codes)) return IQ_ERR_INVALID_ARG;
+    if (in_dtype != IQ_I32 && in_dtype != IQ_I64) return IQ_ERR_INVALID_ARG;
+    if (k < 2 || k > 16 || !dtype_holds(out_dtype, k)) return IQ_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < pc_ws_bytes(c)) return IQ_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    if (in_dtype == IQ_I32)
+        return pc_run((const int32_t*)q, outer, c, inner, s_in, k, relu, codes, out_dtype, s_out,
+                      ws, st);
+    return pc_run((const int64_t*)q, outer, c, inner, s_in, k, relu, codes, out_dtype, s_out, ws,
+                  st);
 }
 
 extern "C" iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_u,

@@ -24,6 +24,8 @@ EXPORTS = [
     "iq_status_str", "iq_version", "iq_launch_count", "iq_conv_out_size", "iq_quantize_workspace_size",
     "iq_conv_fwd_workspace_size", "iq_conv_dgrad_workspace_size", "iq_conv_wgrad_workspace_size",
     "iq_bn_int_workspace_size", "iq_quantize", "iq_quantize_image_u8", "iq_requantize",
+    "iq_requantize_per_channel_workspace_size", "iq_requantize_per_channel",
+    "iq_gemm_s8_nibble_workspace_size", "iq_gemm_s8_nibble",
     "iq_weight_requant", "iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad", "iq_bn_int_fwd",
     "iq_bn_int_bwd", "iq_relu_bwd", "iq_update", "iq_maxpool_fwd", "iq_maxpool_bwd",
     "iq_upsample_workspace_size", "iq_upsample_fwd", "iq_upsample_bwd", "iq_upsample_wgrad",
@@ -114,6 +116,11 @@ def load(path: str | None = None):
     L.iq_bn_int_workspace_size.argtypes = [_I64, _I32, C.POINTER(_SZ)]
     L.iq_quantize.argtypes = [_P, _I64, _I, _I, _I, _P, _P, _P, _SZ, _P]
     L.iq_quantize_image_u8.argtypes = [_P, _I32, _I32, _I32, _I32, _I, _I32, _P, _P, _P, _SZ, _P]
+    L.iq_gemm_s8_nibble_workspace_size.argtypes = [_I32, _I32, _I32, C.POINTER(_SZ)]
+    L.iq_gemm_s8_nibble.argtypes = [_P, _P, _P, _I32, _I32, _I32, _P, _SZ, _P]
+    L.iq_requantize_per_channel_workspace_size.argtypes = [_I32, C.POINTER(_SZ)]
+    L.iq_requantize_per_channel.argtypes = [_P, _I, _I64, _I32, _I64, _P, _I, _I, _P, _I, _P, _P,
+                                            _SZ, _P]
     L.iq_requantize.argtypes = [_P, _I, _I64, _P, _I, _I, _U64, _U64, _U64, _U64, _P, _I, _P, _P,
                                 _SZ, _P]
     L.iq_weight_requant.argtypes = [_P, _P, _I64, _I, _I, _P]
@@ -320,6 +327,40 @@ def iq_requantize(q, s_in, k, mode, codes, s_out, seed=0, layer=0, step=0, tag=0
            load().iq_requantize(_p(q), in_dtype, q.numel(), _p(s_in), k, mode, seed, layer, step,
                                 tag, _p(codes), out_dtype, _p(s_out), _p(ws), ws.numel(),
                                 _stream(stream)))
+
+
+def iq_requantize_per_channel_workspace_size(c: int) -> int:
+    n = _SZ(0)
+    _check("iq_requantize_per_channel_workspace_size",
+           load().iq_requantize_per_channel_workspace_size(c, C.byref(n)))
+    return n.value
+
+
+def iq_requantize_per_channel(q, outer, c, inner, s_in, k, codes, s_out, relu=False, ws=None,
+                              stream=None):
+    """Eq. (ScaleQ) with a per-channel Scale on q viewed as [outer][c][inner]; s_out[c]."""
+    in_dtype = {torch.int32: IQ_I32, torch.int64: IQ_I64}[q.dtype]
+    out_dtype = {torch.int8: IQ_I8, torch.int16: IQ_I16, torch.int32: IQ_I32}[codes.dtype]
+    if ws is None:
+        ws = _ws(iq_requantize_per_channel_workspace_size(c), q.device)
+    _check("iq_requantize_per_channel",
+           load().iq_requantize_per_channel(_p(q), in_dtype, outer, c, inner, _p(s_in), k,
+                                            int(relu), _p(codes), out_dtype, _p(s_out), _p(ws),
+                                            ws.numel(), _stream(stream)))
+
+
+def iq_gemm_s8_nibble(a, b, c, ws=None, stream=None):
+    """c[m][n] = a[m][k] b[n][k]^T (int8 -> int32, exact) on the fp8 nibble-split route."""
+    m, k = a.shape
+    n = b.shape[0]
+    if ws is None:
+        nb = _SZ(0)
+        _check("iq_gemm_s8_nibble_workspace_size",
+               load().iq_gemm_s8_nibble_workspace_size(m, n, k, C.byref(nb)))
+        ws = _ws(nb.value, a.device)
+    _check("iq_gemm_s8_nibble",
+           load().iq_gemm_s8_nibble(_p(a), _p(b), _p(c), m, n, k, _p(ws), ws.numel(),
+                                    _stream(stream)))
 
 
 def iq_weight_requant(master, wq, k_u=24, k_w=8, stream=None):

@@ -4,6 +4,7 @@ through the C ABI; or run one step of a network once (a profiling target).
     python -m paper_2011_14504_gb300.layer_bench [N,H,C,K] [time|once]
     python -m paper_2011_14504_gb300.layer_bench bn M,C [time|once]
     python -m paper_2011_14504_gb300.layer_bench step deeplab|fcn BATCH [train|infer]
+    python -m paper_2011_14504_gb300.layer_bench gemm M,N,K [time|once]
 
 Runs iq_conv_fwd (with ReLU and the SQ8 requantisation of the output), iq_conv_dgrad and
 iq_conv_wgrad (GQ8 gradient) of an N x H x H x C -> K layer on random 8-bit codes.  "time"
@@ -102,12 +103,50 @@ def step_main(argv):
     print("ok")
 
 
+def gemm_main(argv):
+    """The exact int8 GEMM C = A B^T two ways: the fp8 nibble-split route (iq_gemm_s8_nibble,
+    four kind::f8f6f4 MMAs per k-step) and the fp16-carrier route of a 1x1 iq_conv_fwd."""
+    m, n, k = [int(v) for v in (argv[0] if argv else "8192,8192,4096").split(",")]
+    mode = argv[1] if len(argv) > 1 else "time"
+    dev = "cuda"
+    g = torch.Generator(device=dev)
+    g.manual_seed(3)
+    a = torch.randint(-128, 128, (m, k), generator=g, device=dev, dtype=torch.int8)
+    b = torch.randint(-128, 128, (n, k), generator=g, device=dev, dtype=torch.int8)
+    c = torch.empty((m, n), dtype=torch.int32, device=dev)
+    d = iq.conv_desc(1, 1, m, k, n, 1, 1)
+    acc = torch.empty((1, 1, m, n), dtype=torch.int32, device=dev)
+    codes = torch.empty((1, 1, m, n), dtype=torch.int8, device=dev)
+    one = torch.ones(1, dtype=torch.float64, device=dev)
+    s_out = torch.empty(1, dtype=torch.float64, device=dev)
+    ws = torch.empty(iq.iq_conv_fwd_workspace_size(d, False), dtype=torch.uint8, device=dev)
+    routes = [("fp8 nibble split (kind::f8f6f4)", lambda: iq.iq_gemm_s8_nibble(a, b, c)),
+              ("fp16 carriers (kind::f16, 1x1 conv)",
+               lambda: iq.iq_conv_fwd(d, a, one, b, codes, s_out, relu=False, acc_out=acc, ws=ws))]
+    for name, f in routes:
+        ms = _time(f, mode)
+        if ms is not None:
+            print(f"{name}: {ms:.3f} ms  {2.0 * m * n * k / ms / 1e9:.0f} TOPS (whole call)")
+    if mode == "time":
+        iq.iq_kernel_timing_begin()
+        for _, f in routes:
+            f()
+        for r in iq.iq_kernel_timing_end():
+            if r["op"] in (1, 4):
+                print(f"kernel {r['kernel']}: {r['ms']:.3f} ms  "
+                      f"{2.0 * r['macs'] / r['ms'] / 1e9:.0f} TOPS")
+    torch.cuda.synchronize()
+    print("ok")
+
+
 def main(argv=None):
     argv = sys.argv[1:] if argv is None else argv
     if argv and argv[0] == "bn":
         return bn_main(argv[1:])
     if argv and argv[0] == "step":
         return step_main(argv[1:])
+    if argv and argv[0] == "gemm":
+        return gemm_main(argv[1:])
     n, h, c, k = [int(v) for v in (argv[0] if argv else "8,128,256,256").split(",")]
     mode = argv[1] if len(argv) > 1 else "time"
     dev = "cuda"
