@@ -245,6 +245,14 @@ iq_status iq_requantize_per_channel(const void* q, int in_dtype, int64_t outer, 
                                     void* codes, int out_dtype, double* s_out, void* ws,
                                     size_t ws_bytes, iq_stream stream);
 
+/* iq_weight_decay -- L2 weight decay of the master weights.  Sec. 5.1 gives the decay
+ * coefficient (5e-4 for FCN, 1e-5 for DeepLab) but not its quantized form; it is read here as
+ * a decoupled shrink applied after iq_update, with the decay step lambda lr = 2^-shift:
+ * master <- master - floor(master / 2^shift + 1/2) on the k_u grid, then wq = UQ(W_m, k_w)
+ * (Eq. (WQ1)).  shift 1..40; k_u, k_w as in iq_update. */
+iq_status iq_weight_decay(int32_t* master, int8_t* wq, int64_t n, int shift, int k_u, int k_w,
+                          iq_stream stream);
+
 /* iq_gemm_s8_nibble -- C = A B^T for int8 A [m][k], B [n][k] (k contiguous) into int32 C
  * [m][n], exactly, on the fp8 tensor-core path: each code splits into its signed high nibble
  * and its low nibble (v = 16 h + l, both exact in e4m3), and four tcgen05 kind::f8f6f4 MMAs

@@ -95,6 +95,8 @@ def _declare(L):
     for f in ("or_conv_fwd", "or_conv_dgrad", "or_conv_wgrad"):
         getattr(L, f).argtypes = [C.POINTER(ConvDesc), _P, _P, _P]
         getattr(L, f + "_at").argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _I64, _P]
+    L.or_weight_decay.argtypes = [_I64, _P, _P, _I32, _I32, _I32]
+    L.or_weight_decay.restype = None
     L.or_sq_per_channel.argtypes = [_P, _I64, _I64, _I64, _D, _I32, _I32, _P, _P]
     L.or_sq_per_channel.restype = None
     L.or_sq_at.argtypes = [_P, _I64, _I64, _D, _I32, _I32, _P]
@@ -433,6 +435,15 @@ def update(master, gcodes, s_g: float, lr_log2: int, k_u=24, k_w=8, x2=False):
     g = _c(gcodes, np.int32)
     wq = np.empty(m.shape, np.int32)
     lib().or_update(m.size, _ptr(m), _ptr(wq), _ptr(g), float(s_g), lr_log2, k_u, k_w, int(x2))
+    return m, wq
+
+
+def weight_decay(master, shift: int, k_u=24, k_w=8):
+    """Decoupled L2 weight decay of k_U-grid master codes (decay step 2^-shift); returns
+    (new master, new W_q)."""
+    m = np.array(master, dtype=np.int32, copy=True)
+    wq = np.empty(m.shape, np.int32)
+    lib().or_weight_decay(m.size, _ptr(m), _ptr(wq), shift, k_u, k_w)
     return m, wq
 
 

@@ -860,6 +860,20 @@ void or_update(int64_t n, int32_t* master, int32_t* wq, const int32_t* gc,
     or_requant_master(master, n, k_u, k_w, wq);
 }
 
+/* L2 weight decay (Sec. 5.1 states its coefficient, not its quantized form), read as a
+ * decoupled shrink of the k_u-grid master codes after each update: with the decay step
+ * lambda lr = 2^-shift, m <- m - floor(m / 2^shift + 1/2) (round half up, on the master
+ * grid), then W_q = UQ(W_m, k_w) regenerated (Eq. (WQ1)).  shift >= 1. */
+void or_weight_decay(int64_t n, int32_t* master, int32_t* wq, int shift, int k_u, int k_w) {
+    for (int64_t i = 0; i < n; i++) {
+        const int64_t m = master[i];
+        const int64_t d = (int64_t)floordiv128((i128)m + ((i128)1 << (shift - 1)),
+                                               (i128)1 << shift);
+        master[i] = (int32_t)(m - d);
+    }
+    or_requant_master(master, n, k_u, k_w, wq);
+}
+
 /* Correctly rounded conversion of a 128-bit unsigned integer to fp64 (the
  * conversion the sigma_B step applies to T); exposed for its test. */
 double or_u128_to_double(uint64_t hi, uint64_t lo) {

@@ -547,6 +547,20 @@ __global__ void k_pc_codes(const T* __restrict__ q, int64_t n, int32_t C, int64_
     }
 }
 
+// decoupled L2 weight decay: m <- m - floor(m / 2^shift + 1/2), then W_q = UQ(W_m, k_w)
+__global__ void k_weight_decay(int32_t* __restrict__ master, int8_t* __restrict__ wq, int64_t n,
+                               int shift, int k_u, int k_w) {
+    const int64_t lw = qmax(k_w);
+    const int dsh = k_u - k_w;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t m = master[i];
+        const int64_t nm = m - ((m + (int64_t(1) << (shift - 1))) >> shift);
+        master[i] = (int32_t)nm;
+        wq[i] = (int8_t)clamp64((nm + (int64_t(1) << (dsh - 1))) >> dsh, -lw, lw);
+    }
+}
+
 size_t pc_ws_bytes(int32_t C) {
     return 256 + ((size_t)C * 8 + 255) / 256 * 256 + (size_t)C * sizeof(UDiv) + 256;
 }
@@ -725,6 +739,18 @@ extern "C" iq_status iq_requantize_per_channel(const void* q, int in_dtype, int6
                       ws, st);
     return pc_run((const int64_t*)q, outer, c, inner, s_in, k, relu, codes, out_dtype, s_out, ws,
                   st);
+}
+
+extern "C" iq_status iq_weight_decay(int32_t* master, int8_t* wq, int64_t n, int shift,
+                                     int k_u, int k_w, iq_stream stream) {
+    if (!master || !wq || n < 0 || shift < 1 || shift > 40 || k_w < 2 || k_w > 8 ||
+        k_u <= k_w || k_u > 31)
+        return IQ_ERR_INVALID_ARG;
+    if (n == 0) return IQ_OK;
+    k_weight_decay<<<grid_for(n), kThreads, 0, (cudaStream_t)stream>>>(master, wq, n, shift, k_u,
+                                                                       k_w);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
 }
 
 extern "C" iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_u,

@@ -25,7 +25,7 @@ EXPORTS = [
     "iq_conv_fwd_workspace_size", "iq_conv_dgrad_workspace_size", "iq_conv_wgrad_workspace_size",
     "iq_bn_int_workspace_size", "iq_quantize", "iq_quantize_image_u8", "iq_requantize",
     "iq_requantize_per_channel_workspace_size", "iq_requantize_per_channel",
-    "iq_gemm_s8_nibble_workspace_size", "iq_gemm_s8_nibble",
+    "iq_gemm_s8_nibble_workspace_size", "iq_gemm_s8_nibble", "iq_weight_decay",
     "iq_weight_requant", "iq_conv_fwd", "iq_conv_dgrad", "iq_conv_wgrad", "iq_bn_int_fwd",
     "iq_bn_int_bwd", "iq_relu_bwd", "iq_update", "iq_maxpool_fwd", "iq_maxpool_bwd",
     "iq_upsample_workspace_size", "iq_upsample_fwd", "iq_upsample_bwd", "iq_upsample_wgrad",
@@ -116,6 +116,7 @@ def load(path: str | None = None):
     L.iq_bn_int_workspace_size.argtypes = [_I64, _I32, C.POINTER(_SZ)]
     L.iq_quantize.argtypes = [_P, _I64, _I, _I, _I, _P, _P, _P, _SZ, _P]
     L.iq_quantize_image_u8.argtypes = [_P, _I32, _I32, _I32, _I32, _I, _I32, _P, _P, _P, _SZ, _P]
+    L.iq_weight_decay.argtypes = [_P, _P, _I64, _I, _I, _I, _P]
     L.iq_gemm_s8_nibble_workspace_size.argtypes = [_I32, _I32, _I32, C.POINTER(_SZ)]
     L.iq_gemm_s8_nibble.argtypes = [_P, _P, _P, _I32, _I32, _I32, _P, _SZ, _P]
     L.iq_requantize_per_channel_workspace_size.argtypes = [_I32, C.POINTER(_SZ)]
@@ -347,6 +348,12 @@ def iq_requantize_per_channel(q, outer, c, inner, s_in, k, codes, s_out, relu=Fa
            load().iq_requantize_per_channel(_p(q), in_dtype, outer, c, inner, _p(s_in), k,
                                             int(relu), _p(codes), out_dtype, _p(s_out), _p(ws),
                                             ws.numel(), _stream(stream)))
+
+
+def iq_weight_decay(master, wq, shift, k_u=24, k_w=8, stream=None):
+    """Decoupled L2 decay of the k_u-grid masters (decay step 2^-shift), W_q regenerated."""
+    _check("iq_weight_decay", load().iq_weight_decay(_p(master), _p(wq), master.numel(), shift,
+                                                     k_u, k_w, _stream(stream)))
 
 
 def iq_gemm_s8_nibble(a, b, c, ws=None, stream=None):

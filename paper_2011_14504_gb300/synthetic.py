@@ -78,6 +78,17 @@ def fcn_vgg16_weights(seed: int, classes: int = 150, width: float = 1.0):
     return ws, bilinear_filters(classes, 64)
 
 
+def fcn8s_skip_weights(seed: int, classes: int = 150, width: float = 1.0):
+    """fp32 initial weights of the FCN8s decoder: He-initialised 1x1 score filters on pool4
+    and pool3 (KRSC), bilinear x2 (kernel 4) and x8 (kernel 16) per-class filters."""
+    g = rng(seed + 7919)
+    convs = [c for c in fcn_vgg16_channels(classes, width) if c[0] != "pool"]
+    c4, c3 = convs[9][2], convs[6][2]          # conv4_3 and conv3_3 outputs (pool4, pool3)
+    w4 = he_weights(g, (classes, 1, 1, c4), c4)
+    w3 = he_weights(g, (classes, 1, 1, c3), c3)
+    return w4, w3, bilinear_filters(classes, 4), bilinear_filters(classes, 16)
+
+
 def bn_gamma_beta_codes(g: np.random.Generator, channels: int):
     """BN gamma in [0.5, 1.5] and beta in [-0.5, 0.5] drawn as integer codes of the
     8-bit x2-scaled grid (value = code * 2^-6)."""

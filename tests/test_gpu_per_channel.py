@@ -57,3 +57,18 @@ def test_per_channel_sq_argument_checks():
     torch.cuda.synchronize()
     assert not codes.cpu().numpy().any()
     assert np.all(s_out.cpu().numpy() == 2.0 ** -7)
+
+
+@pytest.mark.parametrize("shift", [1, 11, 17, 30])
+def test_weight_decay_matches_oracle(shift):
+    """The decoupled L2 weight decay of the masters (decay step 2^-shift) and the regenerated
+    forward codes, against the oracle."""
+    g = np.random.default_rng(shift)
+    m = g.integers(-(1 << 23) + 1, 1 << 23, size=100003).astype(np.int32)
+    dm = torch.from_numpy(m).to(DEV)
+    wq = torch.empty(m.shape, dtype=torch.int8, device=DEV)
+    iq.iq_weight_decay(dm, wq, shift)
+    m2, w2 = O.weight_decay(m, shift)
+    torch.cuda.synchronize()
+    assert np.array_equal(dm.cpu().numpy(), m2)
+    assert np.array_equal(wq.cpu().numpy().astype(np.int32), w2)

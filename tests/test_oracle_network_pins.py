@@ -104,6 +104,66 @@ def test_fcn_step_is_equivariant_to_the_batch_order():
         assert np.array_equal(ob["ex"][li][0], ex[swap]) and ob["ex"][li][1] == s, li
 
 
+# ---------------------------------------------------------------- FCN8s decoder
+# The x2 (kernel 4, stride 2, padding 1) and x8 (kernel 16, stride 8, padding 4) transposed
+# convolutions map input column j to output columns 2j - 1 + t / 8j - 4 + t, so under a flip
+# tap t becomes 3 - t / 15 - t: with mirror-symmetric filters they commute with the flip, as
+# do the 1x1 score convolutions on the pools and the real-valued sums.
+
+def _net8(wts, up, skips):
+    return OracleFcn(S.fcn_vgg16_channels(CLASSES, WIDTH), wts, up, CLASSES, seed=SEED,
+                     lr_log2=6, skips=skips)
+
+
+def _mirrored_skips():
+    w4, w3, up2, up8 = S.fcn8s_skip_weights(SEED, CLASSES, WIDTH)
+    return w4, w3, 0.5 * (up2 + up2[..., ::-1]), 0.5 * (up8 + up8[..., ::-1])
+
+
+def test_fcn8s_step_commutes_with_a_horizontal_flip():
+    wts, up = _mirrored_weights()
+    sk = _mirrored_skips()
+    img, lab = _inputs()
+    a, b = _net8(wts, up, sk), _net8(wts, up, sk)
+    ta = a.forward(img)
+    tb = b.forward(np.ascontiguousarray(_fw(img)))
+    for key in ("up2a", "sp4", "up2b", "sp3", "up"):
+        assert np.array_equal(tb[key][4], _fw(ta[key][4])), key     # int32 sums
+        assert np.array_equal(tb[key][5], _fw(ta[key][5])) and tb[key][6] == ta[key][6], key
+    for key in ("fuse4", "fuse3"):
+        assert np.array_equal(tb[key][0], _fw(ta[key][0])) and tb[key][1] == ta[key][1], key
+    oa = a.backward_update(ta, lab)
+    ob = b.backward_update(tb, np.ascontiguousarray(_fw(lab)))
+    assert np.array_equal(ob["E"][0], _fw(oa["E"][0]))
+    for key in ("e_fuse3", "e_fuse4", "e_sp3", "e_sp4", "e_score"):
+        assert np.array_equal(ob[key][0], _fw(oa[key][0])) and ob[key][1] == oa[key][1], key
+    for key in ("up8_g", "up2b_g", "up2a_g"):
+        assert np.array_equal(ob[key][0], oa[key][0][..., ::-1]), key    # kernels mirrored
+    for key in ("sp3_g", "sp4_g"):
+        assert np.array_equal(ob[key][0], oa[key][0]), key                # 1x1: sums
+    # (the joined errors at the pools' outputs lie below pool5's argmax ties: not compared)
+
+
+def test_fcn8s_step_is_equivariant_to_the_batch_order():
+    wts, up = S.fcn_vgg16_weights(SEED, CLASSES, WIDTH)
+    sk = S.fcn8s_skip_weights(SEED, CLASSES, WIDTH)
+    img, lab = _inputs(n=3)
+    swap = [1, 2, 0]
+    a, b = _net8(wts, up, sk), _net8(wts, up, sk)
+    ta = a.forward(img)
+    tb = b.forward(np.ascontiguousarray(img[swap]))
+    for key in ("up2a", "sp4", "up2b", "sp3", "up"):
+        assert np.array_equal(tb[key][5], ta[key][5][swap]) and tb[key][6] == ta[key][6], key
+    oa = a.backward_update(ta, lab)
+    ob = b.backward_update(tb, np.ascontiguousarray(lab[swap]))
+    for key in ("up8_g", "up2b_g", "up2a_g", "sp3_g", "sp4_g"):
+        assert np.array_equal(ob[key][0], oa[key][0]), key
+    for li, (G, _, _) in oa["grads"].items():
+        assert np.array_equal(ob["grads"][li][0], G), li
+    for k, (e, s) in oa["e_pool"].items():
+        assert np.array_equal(ob["e_pool"][k][0], e[swap]) and ob["e_pool"][k][1] == s, k
+
+
 # ---------------------------------------------------------------- DeepLabv3-ResNet50
 
 def _deeplab(mirror, blocks=(1, 1, 2, 1), width=0.0625):

@@ -70,3 +70,33 @@ def test_monotone_and_top_code(k):
         i = np.argmax(np.abs(v))
         assert abs(int(cc[i])) == top
         assert np.abs(cc).max() <= top
+
+
+# ---------------------------------------------------------------- weight decay
+# The decoupled decay step m - rhu(m / 2^shift) is pinned to: the closed form on exact
+# multiples m = t 2^shift (m -> t (2^shift - 1)); no growth and no change of sign for any m;
+# the rounding tie m / 2^shift = j + 1/2 going to j + 1 (half up, also for negative m); and
+# W_q as the plain UQ of the new masters (Eq. (WQ1), pinned elsewhere).
+
+@pytest.mark.parametrize("shift", [1, 5, 17])
+def test_weight_decay_closed_form_and_monotone(shift):
+    g = np.random.default_rng(shift)
+    t = g.integers(-(1 << (23 - min(shift, 22))), 1 << (23 - min(shift, 22)), size=500)
+    m = (t << shift).astype(np.int64)
+    m = m[np.abs(m) < (1 << 23)].astype(np.int32)
+    m2, _ = O.weight_decay(m, shift)
+    assert np.array_equal(m2.astype(np.int64), (m.astype(np.int64) >> shift) * ((1 << shift) - 1))
+    r = g.integers(-(1 << 23) + 1, 1 << 23, size=5000).astype(np.int32)
+    r2, wq = O.weight_decay(r, shift)
+    assert np.all(np.abs(r2.astype(np.int64)) <= np.abs(r.astype(np.int64)))
+    assert np.all((np.sign(r2) == np.sign(r)) | (r2 == 0))
+    assert np.array_equal(wq, O.requant_master(r2, 24, 8))
+
+
+def test_weight_decay_ties_round_half_up():
+    shift = 4
+    m = np.array([8, 24, -8, -24, 7, -7, 9, -9], dtype=np.int32)      # m / 16 = +-0.5, +-1.5
+    m2, _ = O.weight_decay(m, shift)
+    # rhu(0.5) = 1, rhu(1.5) = 2, rhu(-0.5) = 0, rhu(-1.5) = -1; +-7/16 round to 0, 9/16 to 1,
+    # -9/16 to -1
+    assert m2.tolist() == [7, 22, -8, -23, 7, -7, 8, -8]
