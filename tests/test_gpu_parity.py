@@ -126,6 +126,28 @@ def test_requantize_sq_int32_vector_path(relu, M):
     assert host(so)[0] == ws
 
 
+@pytest.mark.parametrize("relu,M", [(True, 2 ** 31), (False, 1000), (False, 100), (True, 3 * 2 ** 20)])
+def test_requantize_sq_int32_large(relu, M):
+    # a tensor of 573 k elements (the grid-stride loops wrap several times): both extremes,
+    # ties spread over the whole tensor, and every branch
+    g = S.rng(M % 997 + 3 * relu)
+    n = 5 * 16384 * 7 + 12
+    q = g.integers(-M, min(M, 2 ** 31 - 1) + 1, size=n).astype(np.int64)
+    q[g.integers(n, size=64)] = -M
+    q[g.integers(n, size=1)] = M - 1 if M == 2 ** 31 else M
+    if M % 256 == 0:
+        ties = np.array([(2 * k + 1) * M // 256 - M for k in range(256)], np.int64)
+        q[g.integers(n, size=ties.size)] = ties
+    q = q.astype(np.int32)
+    out = torch.empty(n, dtype=torch.int8, device=DEV)
+    so = dscal()
+    iq.iq_requantize(dev(q), dscal(2.0 ** -20), 8, iq.IQ_MODE_SQ_RELU if relu else iq.IQ_MODE_SQ,
+                     out, so)
+    want, ws = O.sq_int(q, 2.0 ** -20, 8, relu)
+    assert np.array_equal(host(out).astype(np.int32), want)
+    assert host(so)[0] == ws
+
+
 def test_rq_epoch_changes_only_the_draws():
     # the epoch is the fourth Philox counter word: 0 reproduces the oracle; another value gives
     # other draws of the same stochastic rounding (every code within one of the exact value)
