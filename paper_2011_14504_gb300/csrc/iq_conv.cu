@@ -863,7 +863,7 @@ static iq_status conv_fwd_frozen_nhwc(const iq_conv_desc* d, const int8_t* x, co
     IQ_LAUNCH_CHECK();
     return requant_apply(acc, IQ_I32, cp.npq * cp.K, L.s_acc, ka,
                          relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ, 0, 0, 0, 0, a, IQ_I8, L.s_acc, L.rq,
-                         st, true);
+                         st, true, true);
 }
 
 static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const double* s_e,

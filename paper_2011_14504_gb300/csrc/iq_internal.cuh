@@ -55,11 +55,13 @@ __device__ inline RqParams rq_params_make(uint64_t M, double s, int k, int mode)
 inline RqParams* rq_params_slot(void* ws) { return (RqParams*)((char*)ws + 256); }
 
 // The same with max |q| already in the first 8 bytes of ws (an unsigned long long); with
-// params_ready the parameters (rq_params_slot) and *s_out have been written as well.
+// params_ready the parameters (rq_params_slot) and *s_out have been written as well.  clip:
+// the SQ modes' M is not the tensor's own maximum (frozen statistics), so q is clipped to
+// [-M, M] first.
 iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
                         void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st,
-                        bool params_ready = false);
+                        bool params_ready = false, bool clip = false);
 
 // Per-channel statistics buffers of a BN layer, in the workspace.
 struct BnStats {

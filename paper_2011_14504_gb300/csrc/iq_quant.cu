@@ -138,11 +138,12 @@ __global__ void k_rq_finalize(const unsigned long long* __restrict__ cell,
 // floor((2^k q + M) / (2M)); the numerator is < 2^(k+1) M + M < 2^57.  q is first clipped to
 // [-M, M], which changes no code (both ends already give +-(2^(k-1) - 1)) and keeps the
 // numerator non-negative when M is a frozen maximum that this tensor exceeds.
+template <bool CLIP>
 __device__ __forceinline__ int64_t sq_code(int64_t v, const RqParams& p, int k, int relu,
                                            int64_t lim) {
     if (relu && v < 0) v = 0;
     if (!p.M) return 0;
-    v = clamp64(v, -(int64_t)p.M, (int64_t)p.M);
+    if (CLIP) v = clamp64(v, -(int64_t)p.M, (int64_t)p.M);   // M not this tensor's maximum
     uint64_t num = ((uint64_t)(v + (int64_t)p.M) << k) + p.M;
     return clamp64((int64_t)udiv(num, p.div) - (int64_t(1) << (k - 1)), -lim, lim);
 }
@@ -152,10 +153,12 @@ __device__ __forceinline__ int64_t sq_code(int64_t v, const RqParams& p, int k, 
 // t = floor(u R8 / 2^32), R8 = floor(2^39 / M), lies in [floor(128 u / M) - 1,
 // floor(128 u / M)], so q = t + [(2t + 1) M <= 256 u] + [(2t + 3) M <= 256 u] exactly (both
 // sides below 2^41).  Clipping to +-127 is q in [1, 255]; the code byte is q ^ 0x80.
+template <bool CLIP>
 __device__ __forceinline__ uint32_t sq8_byte(int v, uint32_t M, uint32_t R8, int relu) {
     if (relu && v < 0) v = 0;
-    // v clipped to [-M, M]: no code changes, u stays in [0, 2M] (M = 2^31 bounds every int32)
-    if (M < 0x80000000u) v = min(max(v, -(int)M), (int)M);
+    // with an M that is not this tensor's maximum (frozen statistics) v is clipped to [-M, M]
+    // first: u stays in [0, 2M] (M = 2^31 bounds every int32)
+    if (CLIP && M < 0x80000000u) v = min(max(v, -(int)M), (int)M);
     const uint32_t u = (uint32_t)v + M;
     const uint32_t t = __umulhi(u, R8);
     const uint64_t rhs = (uint64_t)u << 8;
@@ -165,12 +168,14 @@ __device__ __forceinline__ uint32_t sq8_byte(int v, uint32_t M, uint32_t R8, int
     return q ^ 0x80u;
 }
 
+template <bool CLIP>
 __device__ __forceinline__ uint32_t sq8_word(const int4& v, uint32_t M, uint32_t R8, int relu) {
-    return sq8_byte(v.x, M, R8, relu) | (sq8_byte(v.y, M, R8, relu) << 8) |
-           (sq8_byte(v.z, M, R8, relu) << 16) | (sq8_byte(v.w, M, R8, relu) << 24);
+    return sq8_byte<CLIP>(v.x, M, R8, relu) | (sq8_byte<CLIP>(v.y, M, R8, relu) << 8) |
+           (sq8_byte<CLIP>(v.z, M, R8, relu) << 16) | (sq8_byte<CLIP>(v.w, M, R8, relu) << 24);
 }
 
 // int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores)
+template <bool CLIP>
 __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int relu,
                               const RqParams* __restrict__ prm, uint32_t* __restrict__ out) {
     const RqParams p = *prm;
@@ -187,7 +192,7 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
                 v[j] = i + j * stride < n4 ? __ldg(q + i + j * stride) : make_int4(0, 0, 0, 0);
 #pragma unroll
             for (int j = 0; j < 4; j++)
-                if (i + j * stride < n4) out[i + j * stride] = sq8_word(v[j], M, p.R8, relu);
+                if (i + j * stride < n4) out[i + j * stride] = sq8_word<CLIP>(v[j], M, p.R8, relu);
         }
         return;
     }
@@ -196,19 +201,19 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
         const int64_t i2 = i + stride;
         const int4 v = __ldg(q + i);
         const int4 v2 = i2 < n4 ? __ldg(q + i2) : make_int4(0, 0, 0, 0);
-        out[i] = ((uint32_t)sq_code(v.x, p, k, relu, lim) & 0xffu) |
-                 (((uint32_t)sq_code(v.y, p, k, relu, lim) & 0xffu) << 8) |
-                 (((uint32_t)sq_code(v.z, p, k, relu, lim) & 0xffu) << 16) |
-                 (((uint32_t)sq_code(v.w, p, k, relu, lim) & 0xffu) << 24);
+        out[i] = ((uint32_t)sq_code<CLIP>(v.x, p, k, relu, lim) & 0xffu) |
+                 (((uint32_t)sq_code<CLIP>(v.y, p, k, relu, lim) & 0xffu) << 8) |
+                 (((uint32_t)sq_code<CLIP>(v.z, p, k, relu, lim) & 0xffu) << 16) |
+                 (((uint32_t)sq_code<CLIP>(v.w, p, k, relu, lim) & 0xffu) << 24);
         if (i2 < n4)
-            out[i2] = ((uint32_t)sq_code(v2.x, p, k, relu, lim) & 0xffu) |
-                      (((uint32_t)sq_code(v2.y, p, k, relu, lim) & 0xffu) << 8) |
-                      (((uint32_t)sq_code(v2.z, p, k, relu, lim) & 0xffu) << 16) |
-                      (((uint32_t)sq_code(v2.w, p, k, relu, lim) & 0xffu) << 24);
+            out[i2] = ((uint32_t)sq_code<CLIP>(v2.x, p, k, relu, lim) & 0xffu) |
+                      (((uint32_t)sq_code<CLIP>(v2.y, p, k, relu, lim) & 0xffu) << 8) |
+                      (((uint32_t)sq_code<CLIP>(v2.z, p, k, relu, lim) & 0xffu) << 16) |
+                      (((uint32_t)sq_code<CLIP>(v2.w, p, k, relu, lim) & 0xffu) << 24);
     }
 }
 
-template <typename T>
+template <typename T, bool CLIP>
 __global__ void k_sq_int(const T* __restrict__ q, int64_t n, int k, int relu,
                          const RqParams* __restrict__ prm, void* __restrict__ out, int dtype) {
     const RqParams p = *prm;
@@ -219,7 +224,7 @@ __global__ void k_sq_int(const T* __restrict__ q, int64_t n, int k, int relu,
         if (relu && v < 0) v = 0;
         int64_t c = 0;
         if (p.M) {
-            v = clamp64(v, -(int64_t)p.M, (int64_t)p.M);
+            if (CLIP) v = clamp64(v, -(int64_t)p.M, (int64_t)p.M);
             uint64_t num = ((uint64_t)(v + (int64_t)p.M) << k) + p.M;
             c = (int64_t)udiv(num, p.div) - (int64_t(1) << (k - 1));
             c = clamp64(c, -lim, lim);
@@ -286,7 +291,7 @@ __global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
 iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
                         void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st,
-                        bool params_ready) {
+                        bool params_ready, bool clip) {
     unsigned long long* cell = (unsigned long long*)ws;
     RqParams* prm = rq_params_slot(ws);
     bool relu = mode == IQ_MODE_SQ_RELU;
@@ -300,16 +305,23 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
     const double osz = out_dtype == IQ_I8 ? 1.0 : (out_dtype == IQ_I16 ? 2.0 : 4.0);
     kt_pre(st);
     if (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) {
-        if (in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
-            (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0)
-            k_sq_i32_i8x4<<<grid_for(n / 4), kThreads, 0, st>>>((const int4*)q, n / 4, k, relu,
-                                                                prm, (uint32_t*)out);
+        const bool x4 = in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
+                        (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0;
+        if (x4 && clip)
+            k_sq_i32_i8x4<true><<<grid_for(n / 4), kThreads, 0, st>>>((const int4*)q, n / 4, k,
+                                                                      relu, prm, (uint32_t*)out);
+        else if (x4)
+            k_sq_i32_i8x4<false><<<grid_for(n / 4), kThreads, 0, st>>>((const int4*)q, n / 4, k,
+                                                                       relu, prm, (uint32_t*)out);
+        else if (in_dtype == IQ_I32 && clip)
+            k_sq_int<int32_t, true><<<g, kThreads, 0, st>>>((const int32_t*)q, n, k, relu, prm,
+                                                            out, out_dtype);
         else if (in_dtype == IQ_I32)
-            k_sq_int<int32_t><<<g, kThreads, 0, st>>>((const int32_t*)q, n, k, relu, prm, out,
-                                                      out_dtype);
+            k_sq_int<int32_t, false><<<g, kThreads, 0, st>>>((const int32_t*)q, n, k, relu, prm,
+                                                             out, out_dtype);
         else
-            k_sq_int<int64_t><<<g, kThreads, 0, st>>>((const int64_t*)q, n, k, relu, prm, out,
-                                                      out_dtype);
+            k_sq_int<int64_t, false><<<g, kThreads, 0, st>>>((const int64_t*)q, n, k, relu, prm,
+                                                             out, out_dtype);
     } else {
         int gb = grid_for((n + 7) / 8);
         const unsigned long long* ep = rq_epoch_ptr();
