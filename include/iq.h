@@ -73,13 +73,20 @@ enum {
  *        step 2^(1-k_w) is the weight factor of the accumulator scale
  *   k_a  bit width of the output activation codes Q_A = SQ(., k_a) (Eq. (AQ1)), 2..8,
  *        0 = 8 (with batch norm the bits argument's k_a, when given, must agree)
+ *   flags  0, or IQ_CONV_X_F16_READY: the x_f16 buffer given to iq_conv_fwd /
+ *        iq_conv_fwd_frozen already holds the fp16 copy of this call's input codes (an
+ *        earlier call on the same input wrote it), so the call reads it and does not write
+ *        it; the caller keeps the two in step (a carrier of other codes gives wrong sums).
+ *        A storage option with no counterpart in the paper.
  * A zero-initialised descriptor tail gives the paper's setting (NHWC, 8-bit codes). */
 enum { IQ_LAYOUT_NHWC = 0, IQ_LAYOUT_NCHW = 1 };
+enum { IQ_CONV_X_F16_READY = 1 };
 typedef struct {
     int32_t n, h, w, c;
     int32_t k, r, s;
     int32_t stride_h, stride_w, pad_h, pad_w, dil_h, dil_w, groups;
     int32_t layout, k_w, k_a;
+    int32_t flags;
 } iq_conv_desc;
 
 /* Bit widths of the quantized L1BN objects (Sec. 3.2.2 equation block, Eq. (AQ1)). */
@@ -293,9 +300,10 @@ iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_
  *   x_f16     optional out fp16 [n][h][w][c] (16-byte aligned, n h w c % 16 == 0, else
  *             IQ_ERR_INVALID_ARG): the exact fp16 copy of the codes x (of their NHWC
  *             transpose with IQ_LAYOUT_NCHW) that the tensor-core kernels read (every int8
- *             code is exact in fp16).  When given it is written first
- *             and the kernels read it; keep it for iq_conv_wgrad of the same layer, which then
- *             skips its own conversion of x.  (The paper has no counterpart: it is the
+ *             code is exact in fp16).  When given it is written first (not with
+ *             IQ_CONV_X_F16_READY in d->flags: then it is read as it is) and the kernels read
+ *             it; keep it for iq_conv_wgrad of the same layer, which then skips its own
+ *             conversion of x.  (The paper has no counterpart: it is the
  *             operand format of this implementation's tensor-core path.)
  * Returns IQ_ERR_OVERFLOW_RISK when (c/groups) r s 127^2 >= 2^31. */
 iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,

@@ -23,6 +23,22 @@ __device__ __forceinline__ int64_t clamp64(int64_t v, int64_t lo, int64_t hi) {
     return v < lo ? lo : (v > hi ? hi : v);
 }
 
+// int64 -> fp32 through the two 32-bit halves of |v| (64-bit conversions run on the narrow
+// FP64 pipe of this part): |v| = hi 2^32 + lo with hi < 2^24 (|v| < 2^56) is exact in
+// hi 2^32, so fma(hi, 2^32, fl(lo)) is fl(lo) when hi = 0 and otherwise within
+// 2^8 + u |v| <= 2u |v| of |v| (u = 2^-24): a relative error of at most 2u.
+__device__ __forceinline__ float f32_of_i64(long long v) {
+    const unsigned long long a = (unsigned long long)(v < 0 ? -v : v);
+    const float f = fmaf((float)(uint32_t)(a >> 32), 0x1p32f, __uint2float_rn((uint32_t)a));
+    return v < 0 ? -f : f;
+}
+// an fp32 upper bound of |v|
+__device__ __forceinline__ float f32_abs_up(long long v) {
+    const unsigned long long a = (unsigned long long)(v < 0 ? -v : v);
+    return __fmaf_ru(__uint2float_ru((uint32_t)(a >> 32)), 0x1p32f,
+                     __uint2float_ru((uint32_t)a));
+}
+
 // floor(y + 1/2) (the rounding of Eq. (UQ)) on an fp64 value: y - floor(y) is
 // exact, so comparing it with 1/2 never rounds.
 __device__ __forceinline__ double rhu(double y) {

@@ -397,6 +397,7 @@ static bool desc_ok(const iq_conv_desc* d) {
     if (d->layout != IQ_LAYOUT_NHWC && d->layout != IQ_LAYOUT_NCHW) return false;
     if (d->k_w != 0 && (d->k_w < 2 || d->k_w > 8)) return false;
     if (d->k_a != 0 && (d->k_a < 2 || d->k_a > 8)) return false;
+    if (d->flags & ~IQ_CONV_X_F16_READY) return false;
     int p = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1);
     int q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1);
     return p >= 0 && q >= 0;
@@ -727,7 +728,7 @@ static iq_status conv_fwd_nhwc(const iq_conv_desc* d, const int8_t* x, const dou
     k_scale_mul_pow2<<<1, 1, 0, st>>>(s_x, 1 - code_kw(d), L.s_acc);  // s_acc = s_x 2^(1-k_w)
     IQ_LAUNCH_CHECK();
     bool done = false;
-    if (x_f16) {
+    if (x_f16 && !(d->flags & IQ_CONV_X_F16_READY)) {
         r = codes_to_f16(x, (__half*)x_f16, nx, st);
         if (r != IQ_OK) return r;
     }
@@ -822,7 +823,7 @@ static iq_status conv_fwd_frozen_nhwc(const iq_conv_desc* d, const int8_t* x, co
     cp.M = cp.npq;
     cp.ncols = cp.Kg;
     cp.kin = (int)roundup(cp.Cg, BK);
-    if (x_f16) {
+    if (x_f16 && !(d->flags & IQ_CONV_X_F16_READY)) {
         iq_status r = codes_to_f16(x, (__half*)x_f16, nx, st);
         if (r != IQ_OK) return r;
     }

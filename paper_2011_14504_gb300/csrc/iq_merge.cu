@@ -8,6 +8,7 @@
 #include <climits>
 
 #include "iq_internal.cuh"
+#include "iq_stream.cuh"
 
 namespace iq {
 
@@ -520,21 +521,6 @@ __device__ __forceinline__ void cover4_of(const Terms& T, int concat, int co0, C
     }
 }
 
-// int64 -> fp32 through the two 32-bit halves of |v| (64-bit conversions run on the narrow
-// FP64 pipe of this part): |v| = hi 2^32 + lo with hi < 2^24 (|v| < 2^56) is exact in
-// hi 2^32, so fma(hi, 2^32, fl(lo)) is fl(lo) when hi = 0 and otherwise within
-// 2^8 + u |v| <= 2u |v| of |v| (u = 2^-24): a relative error of at most 2u.
-__device__ __forceinline__ float f32_of_i64(long long v) {
-    const unsigned long long a = (unsigned long long)(v < 0 ? -v : v);
-    const float f = fmaf((float)(uint32_t)(a >> 32), 0x1p32f, __uint2float_rn((uint32_t)a));
-    return v < 0 ? -f : f;
-}
-// an fp32 upper bound of |v|
-__device__ __forceinline__ float f32_abs_up(long long v) {
-    const unsigned long long a = (unsigned long long)(v < 0 ? -v : v);
-    return __fmaf_ru(__uint2float_ru((uint32_t)(a >> 32)), 0x1p32f,
-                     __uint2float_ru((uint32_t)a));
-}
 
 // CPT codes of one operand as loaded: 16 bytes (CPT = 8 int16 or 16 int8 codes) or
 // 8 bytes (CPT = 8 int8 codes)
@@ -759,6 +745,243 @@ __global__ void k_comb_params(CombHdr* hdr, double* s_out) {
     *s_out = M ? ldexp((double)M, -hdr->P - 7) : ldexp(1.0, -hdr->P - 7);
 }
 
+// ---------------------------------------------------------------- streamed two-operand joins
+//
+// The two passes of a sum of two operands that both cover every channel of every pixel (the
+// residual adds and the sums of two errors), with the operands' rows landed in shared memory
+// by bulk copies (iq_stream.cuh): the copy engine keeps about 130 KB per SM in flight, where
+// the register-fed k_comb4f keeps 32 KB.  The arithmetic is k_comb4f's, with 4 channels per
+// thread (the stream's channel group), and two changes that decide nothing differently:
+//  - codes reach fp32 without the conversion unit: a code v of an int16 word biased to
+//    u = v + 2^15 (an xor) and placed in the low mantissa bits of 2^23 by a byte permute is
+//    the float 2^23 + u, and subtracting 2^23 + 2^15 leaves v exactly (int8: 2^23 + 2^7);
+//  - the codes pass clamps y to [-126.5, 127.5] (the clamp of the code to [-127, 127]
+//    commutes with the floor there) and takes floor(y) = c from the bits of y + 1.5 2^23
+//    rounded downward (its low byte is the code), f = y - c exactly; the code is c when
+//    D <= f < 1 - D (D < 1/2): the exact value, within D of y, then has the same floor (a
+//    clamped y has f = 1/2 and an exact value beyond the clamp bound); otherwise the element
+//    takes the exact division.
+// The max pass shares its running maximum across the warp with one max-reduction over the
+// fp32 bit patterns (non-negative floats order as their bits) per row.
+
+__device__ __forceinline__ float f32_of_i16_lo(uint32_t wx) {
+    return __int_as_float((int)__byte_perm(wx, 0x4B000000u, 0x7410)) - 8421376.0f;
+}
+__device__ __forceinline__ float f32_of_i16_hi(uint32_t wx) {
+    return __int_as_float((int)__byte_perm(wx, 0x4B000000u, 0x7432)) - 8421376.0f;
+}
+template <int J>
+__device__ __forceinline__ float f32_of_i8(uint32_t wx) {
+    return __int_as_float((int)__byte_perm(wx, 0x4B000000u, 0x7440 + J)) - 8388736.0f;
+}
+
+// the 4 codes of one operand at a row of a stage, as fp32 and as raw words
+template <bool W16>
+__device__ __forceinline__ void stage_codes4(const uint8_t* p, float (&f)[4], uint2& raw) {
+    if (W16) {
+        raw = *reinterpret_cast<const uint2*>(p);
+        const uint32_t a = raw.x ^ 0x80008000u, b = raw.y ^ 0x80008000u;
+        f[0] = f32_of_i16_lo(a); f[1] = f32_of_i16_hi(a);
+        f[2] = f32_of_i16_lo(b); f[3] = f32_of_i16_hi(b);
+    } else {
+        raw.x = *reinterpret_cast<const uint32_t*>(p);
+        raw.y = 0u;
+        const uint32_t a = raw.x ^ 0x80808080u;
+        f[0] = f32_of_i8<0>(a); f[1] = f32_of_i8<1>(a);
+        f[2] = f32_of_i8<2>(a); f[3] = f32_of_i8<3>(a);
+    }
+}
+template <bool W16>
+__device__ __forceinline__ int32_t raw_code4(const uint2& r, int j) {
+    if (W16) {
+        const uint32_t w = j < 2 ? r.x : r.y;
+        return (j & 1) ? (int32_t)w >> 16 : (int32_t)(int16_t)(w & 0xffffu);
+    }
+    return (int32_t)(int8_t)((r.x >> (8 * j)) & 0xffu);
+}
+
+template <int PASS, bool A16, bool B16, bool PLAIN>
+__global__ void __launch_bounds__(kStreamThreads, 1)
+    k_comb_s(RowStream rs, Terms T, int relu, const long long* __restrict__ F,
+             const long long* __restrict__ B, CombHdr* hdr, int8_t* __restrict__ out,
+             int* __restrict__ err) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    if (__syncthreads_or(threadIdx.x == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
+    constexpr int FW = PLAIN ? 1 : 4;
+    const int CB4 = rs.CB >> 2;
+    const int g = threadIdx.x % CB4, rl = threadIdx.x / CB4;
+    const int c0 = blockIdx.x * rs.CB + 4 * g;
+    int fo[2];
+    float ff[2][FW], bf[FW];
+    long long fi[2];
+    float S = 0.f;
+    {
+        long long bs[FW];
+        float sv[FW];
+#pragma unroll
+        for (int j = 0; j < FW; j++) { bs[j] = 0; sv[j] = 0.f; }
+#pragma unroll
+        for (int k = 0; k < 2; k++) {
+            const TermDev& tt = T.t[k];
+            fo[k] = tt.base + c0;
+            const float vmax = (k == 0 ? A16 : B16) ? 32767.f : 127.f;
+#pragma unroll
+            for (int j = 0; j < FW; j++) {
+                const long long f = F[fo[k] + j];
+                ff[k][j] = f32_of_i64(f);
+                if (PLAIN) fi[k] = f;
+                if (!PLAIN) bs[j] += B[fo[k] + j];
+                sv[j] = __fmaf_ru(f32_abs_up(f), vmax, sv[j]);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < FW; j++) {
+            bf[j] = f32_of_i64(bs[j]);
+            S = fmaxf(S, __fadd_ru(sv[j], f32_abs_up(bs[j])));
+        }
+    }
+    const float E = __fmul_ru(__fmul_ru(5.f, 0x1p-24f), S);    // (nc + 3) u S, nc = 2
+    float E3 = __fmul_ru(3.f, E);
+    if (PASS == 0) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) E3 = fmaxf(E3, __shfl_xor_sync(0xffffffffu, E3, o));
+    }
+    uint64_t M = 0;
+    float kq = 0.f, D = 0.f, omd = 0.f;
+    bool fast = false;
+    if (PASS == 1) {
+        M = hdr->M;
+        kq = hdr->kq;
+        D = __fmaf_ru(E, hdr->c130, 0x1p-14f);
+        omd = __fsub_rd(1.f, D);
+        fast = D < 0.5f;
+    }
+    auto exact = [&](const uint2& ra, const uint2& rb, int j) -> int64_t {
+        int64_t z;
+        if (PLAIN) {
+            z = fi[0] * raw_code4<A16>(ra, j) + fi[1] * raw_code4<B16>(rb, j);
+        } else {
+            z = F[fo[0] + j] * raw_code4<A16>(ra, j) + B[fo[0] + j] +
+                F[fo[1] + j] * raw_code4<B16>(rb, j) + B[fo[1] + j];
+        }
+        return (relu && z < 0) ? 0 : z;
+    };
+    const int eszA = A16 ? 2 : 1, eszB = B16 ? 2 : 1;
+    uint32_t fmx = 0u;         // bits of the warp's largest |zf| so far
+    uint64_t mx = 0;
+    auto row = [&](const uint8_t* st, int r, int64_t r0) {
+            const int e = r * rs.CB + 4 * g;
+            float fa[4], fb[4];
+            uint2 ra, rb;
+            stage_codes4<A16>(st + rs.off[0] + e * eszA, fa, ra);
+            stage_codes4<B16>(st + rs.off[1] + e * eszB, fb, rb);
+            float zf[4];
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                const float b0 = PLAIN ? 0.f : bf[PLAIN ? 0 : j];
+                zf[j] = fmaf(ff[1][PLAIN ? 0 : j], fb[j], fmaf(ff[0][PLAIN ? 0 : j], fa[j], b0));
+            }
+            if (PASS == 0) {
+                float a[4], am = 0.f;
+#pragma unroll
+                for (int j = 0; j < 4; j++) {
+                    a[j] = fabsf(relu ? fmaxf(zf[j], 0.f) : zf[j]);
+                    am = fmaxf(am, a[j]);
+                }
+                fmx = max(fmx, __reduce_max_sync(0xffffffffu, __float_as_uint(am)));
+                const float thr = __uint_as_float(fmx) - E3;
+                if (am >= thr) {
+#pragma unroll
+                    for (int j = 0; j < 4; j++)
+                        if (a[j] >= thr) {
+                            const int64_t z = exact(ra, rb, j);
+                            const uint64_t az = (uint64_t)(z < 0 ? -z : z);
+                            mx = az > mx ? az : mx;
+                        }
+                }
+            } else {
+                uint32_t w = 0u;
+                if (M) {
+                    uint32_t tb[4];
+                    bool ok[4];
+#pragma unroll
+                    for (int j = 0; j < 4; j++) {
+                        const float y = fminf(fmaxf(fmaf(relu ? fmaxf(zf[j], 0.f) : zf[j], kq,
+                                                         0.5f), -126.5f), 127.5f);
+                        const float t = __fadd_rd(y, 12582912.0f);
+                        const float f = y - (t - 12582912.0f);
+                        tb[j] = __float_as_uint(t);
+                        ok[j] = f >= D && f < omd;
+                    }
+                    // one branch per row for the rare elements fp32 does not decide
+                    if (!(fast && ok[0] && ok[1] && ok[2] && ok[3])) {
+                        const UDiv d2m = hdr->div;
+#pragma unroll
+                        for (int j = 0; j < 4; j++)
+                            if (!(fast && ok[j])) {
+                                const uint64_t num =
+                                    ((uint64_t)(exact(ra, rb, j) + (int64_t)M) << 8) + M;
+                                tb[j] = (uint32_t)(int)clamp64((int64_t)udiv(num, d2m) - 128,
+                                                               -127, 127);
+                            }
+                    }
+                    w = __byte_perm(__byte_perm(tb[0], tb[1], 0x0040),
+                                    __byte_perm(tb[2], tb[3], 0x0040), 0x5410);
+                }
+                *reinterpret_cast<uint32_t*>(out + (r0 + r) * rs.C + c0) = w;
+            }
+    };
+    const bool ok = stream_chunks(rs, smem, err, [&](const uint8_t* st, int rows, int64_t r0) {
+        // rl is the same on every lane of a warp (CB >= 128), so the row loop is warp-uniform;
+        // a whole chunk runs fully unrolled (the rows' loads and arithmetic interleave)
+        if (rows == rs.R) {
+#pragma unroll
+            for (int u = 0; u < kStreamRPT; u++) row(st, rl + u * rs.RL, r0);
+        } else {
+            for (int u = 0; u < kStreamRPT; u++) {
+                const int r = rl + u * rs.RL;
+                if (r >= rows) break;
+                row(st, r, r0);
+            }
+        }
+    });
+    if (!ok) return;
+    if (PASS == 0) {
+        mx = warp_max_u64(mx);
+        if ((threadIdx.x & 31) == 0 && mx) atomicMax(&hdr->maxz, (unsigned long long)mx);
+    }
+}
+
+// the dynamic shared memory of one instantiation, set once
+template <int PASS, bool A16, bool B16, bool PLAIN>
+iq_status comb_s_launch(const RowStream& rs, const Terms& T, int relu, const long long* F,
+                        const long long* B, CombHdr* hdr, int8_t* out, int* err,
+                        cudaStream_t st) {
+    static bool attr = false;
+    auto kern = k_comb_s<PASS, A16, B16, PLAIN>;
+    if (!attr) {
+        IQ_CUDA_CHECK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)row_stream_smem(rs)));
+        attr = true;
+    }
+    kern<<<row_stream_grid(rs, device_sms()), kStreamThreads, row_stream_smem(rs), st>>>(
+        rs, T, relu, F, B, hdr, out, err);
+    IQ_LAUNCH_CHECK();
+    return IQ_OK;
+}
+
+template <int PASS>
+iq_status comb_s_pass(const RowStream& rs, const Terms& T, bool plain, int relu,
+                      const long long* F, const long long* B, CombHdr* hdr, int8_t* out,
+                      int* err, cudaStream_t st) {
+    const bool a16 = T.t[0].is16 != 0, b16 = T.t[1].is16 != 0;
+    if (plain) return comb_s_launch<PASS, false, false, true>(rs, T, relu, F, B, hdr, out, err, st);
+    if (a16 && b16) return comb_s_launch<PASS, true, true, false>(rs, T, relu, F, B, hdr, out, err, st);
+    if (a16) return comb_s_launch<PASS, true, false, false>(rs, T, relu, F, B, hdr, out, err, st);
+    if (b16) return comb_s_launch<PASS, false, true, false>(rs, T, relu, F, B, hdr, out, err, st);
+    return comb_s_launch<PASS, false, false, false>(rs, T, relu, F, B, hdr, out, err, st);
+}
+
 // ---------------------------------------------------------------- spatial sums
 
 // sums[i][j] += sum over a slice of image i's pixels of x[i][p][c_off + j]
@@ -933,6 +1156,30 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
     for (int i = 0; i < n_terms; i++) {
         plain = plain && !T.t[i].gamma && !T.t[i].beta && !T.t[i].is16;
         any16 = any16 || T.t[i].is16;
+    }
+    // two operands that cover every channel of every pixel (residual adds, sums of two
+    // errors): the streamed passes, when the stream takes the shape with at least 128
+    // channels per slab (a warp's lanes then share their rows)
+    if (n_terms == 2 && !concat && !any_bcast && ((uintptr_t)out & 3) == 0) {
+        RowStream rs;
+        const void* srcs[2] = {T.t[0].codes, T.t[1].codes};
+        const int esz[2] = {T.t[0].is16 ? 2 : 1, T.t[1].is16 ? 2 : 1};
+        if (row_stream_plan(rs, n * hw, c_out, srcs, esz, 2) && rs.CB >= 128) {
+            int* err = device_status_ptr();
+            if (!err) return IQ_ERR_CUDA;
+            const int rl = relu != 0;
+            kt_pre(st);
+            iq_status r = comb_s_pass<0>(rs, T, plain, rl, F, B, hdr, out, err, st);
+            if (r != IQ_OK) return r;
+            kt_post_bytes(st, IQ_KERNEL_COMBINE_MAX, in_b);
+            k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
+            IQ_LAUNCH_CHECK();
+            kt_pre(st);
+            r = comb_s_pass<1>(rs, T, plain, rl, F, B, hdr, out, err, st);
+            if (r != IQ_OK) return r;
+            kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b);
+            return IQ_OK;
+        }
     }
     const int cpt = plain ? 16 : 8;
     bool wide = c_out % cpt == 0 && ((uintptr_t)out & (cpt - 1)) == 0;

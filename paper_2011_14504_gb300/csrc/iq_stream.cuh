@@ -2,8 +2,8 @@
 // bandwidth-bound per-channel passes (integer L1BN forward and backward).
 //
 // A block of kStreamThreads threads (one per SM) owns a slab of CB channels (all C
-// channels when C <= 1024, else 1024 of them) and a strided sequence of row chunks of that
-// slab.  Thread 0 keeps kStreamStages chunks in flight with 1-D bulk copies
+// channels when C is a power of two up to 4 kStreamThreads = 2048, else 1024 of them) and a
+// strided sequence of row chunks of that slab.  Thread 0 keeps kStreamStages chunks in flight with 1-D bulk copies
 // (cp.async.bulk, one per array per chunk when the slab is the whole row, else one per row)
 // whose bytes complete an mbarrier; the warps read a landed chunk from shared memory and
 // release its stage on a second mbarrier (one arrival per warp), after which thread 0
@@ -41,11 +41,12 @@ struct RowStream {
 
 // Host: plan the streaming of up to three [m][C] arrays (src[i] with esz[i]-byte elements,
 // 16-byte aligned).  False when the shape does not fit: C must be a power of two in
-// [16, 1024] or a multiple of 1024.
+// [16, 2048] or a multiple of 1024.  A slab of whole rows lands with one copy per array
+// per chunk, a narrower one with one copy per row.
 inline bool row_stream_plan(RowStream& s, int64_t m, int32_t C, const void* const* src,
                             const int* esz, int narr) {
     if (m <= 0 || narr < 1 || narr > kStreamMaxArr) return false;
-    if (C >= 16 && C <= 1024 && (C & (C - 1)) == 0) s.CB = C;
+    if (C >= 16 && C <= 4 * kStreamThreads && (C & (C - 1)) == 0) s.CB = C;
     else if (C > 1024 && C % 1024 == 0) s.CB = 1024;
     else return false;
     s.m = m;

@@ -205,20 +205,23 @@ class DeepLabV3R50:
             self.s_e_c4 = self.scal()
             self.e_stem = torch.empty(self.stem.out_shape, dtype=torch.int8, device=dev)
             self.s_e_stem = self.scal()
+        # fp16 copies of the codes the tensor-core kernels read: one per distinct conv input,
+        # written by the forward of the first layer (in forward order) that reads it and read
+        # as it is by the others (IQ_CONV_X_F16_READY: the ASPP branches, a block's first conv
+        # and its projection shortcut) and by the weight gradients; and one error buffer
+        # (written by a layer's data gradient, reused by its weight gradient)
+        x16, e16 = {}, 0
+        for L in self.layers.values():
+            if L.spec.cin % 64 == 0 and L.x.numel() % 16 == 0:
+                key = L.x.data_ptr()
+                if key not in x16:
+                    x16[key] = torch.empty(L.x.numel(), dtype=torch.float16, device=dev)
+                else:
+                    L.desc.flags = iq.IQ_CONV_X_F16_READY
+                L.x16 = x16[key]
+            if L.spec.cout % 64 == 0:
+                e16 = max(e16, L.a.numel())
         if train:
-            # fp16 copies of the codes the tensor-core kernels read: one per distinct conv
-            # input (written by the forward of each layer reading it, reused by their weight
-            # gradients) and one error buffer (written by a layer's data gradient, reused by its
-            # weight gradient)
-            x16, e16 = {}, 0
-            for L in self.layers.values():
-                if L.spec.cin % 64 == 0 and L.x.numel() % 16 == 0:
-                    key = L.x.data_ptr()
-                    if key not in x16:
-                        x16[key] = torch.empty(L.x.numel(), dtype=torch.float16, device=dev)
-                    L.x16 = x16[key]
-                if L.spec.cout % 64 == 0:
-                    e16 = max(e16, L.a.numel())
             self.e16 = torch.empty(max(e16, 16), dtype=torch.float16, device=dev)
         self.ws = torch.empty(self._ws_bytes(), dtype=torch.uint8, device=dev)
 

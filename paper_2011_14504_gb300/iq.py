@@ -58,10 +58,11 @@ class IqError(RuntimeError):
 class ConvDesc(C.Structure):
     _fields_ = [(n, C.c_int32) for n in
                 ("n", "h", "w", "c", "k", "r", "s", "stride_h", "stride_w", "pad_h", "pad_w",
-                 "dil_h", "dil_w", "groups", "layout", "k_w", "k_a")]
+                 "dil_h", "dil_w", "groups", "layout", "k_w", "k_a", "flags")]
 
 
 IQ_LAYOUT_NHWC, IQ_LAYOUT_NCHW = 0, 1
+IQ_CONV_X_F16_READY = 1
 
 
 class BnBits(C.Structure):
@@ -251,11 +252,12 @@ def _ws(nbytes: int, device) -> torch.Tensor:
 
 
 def conv_desc(n, h, w, c, k, r, s, stride=1, pad=0, dil=1, groups=1, layout=IQ_LAYOUT_NHWC,
-              k_w=0, k_a=0) -> ConvDesc:
+              k_w=0, k_a=0, flags=0) -> ConvDesc:
     """iq_conv_desc; layout IQ_LAYOUT_NCHW takes NCHW activations / errors and KCRS filters,
-    k_w / k_a the weight and activation code widths (0: 8 bits)."""
+    k_w / k_a the weight and activation code widths (0: 8 bits); flags
+    IQ_CONV_X_F16_READY: the x_f16 buffer of the forward already holds the input's fp16 copy."""
     return ConvDesc(n, h, w, c, k, r, s, stride, stride, pad, pad, dil, dil, groups, layout, k_w,
-                    k_a)
+                    k_a, flags)
 
 
 def bn_bits(k_mu=16, k_sigma=16, k_xhat=16, k_gamma=8, k_beta=8, k_a=8) -> BnBits:

@@ -61,10 +61,12 @@ def test_conv_out_size_and_workspace_queries(lib):
 
 
 def test_conv_desc_layout_and_widths_validated(lib):
-    """The descriptor's layout and code widths: NHWC / NCHW, k_w and k_a in 2..8 (0: 8 bits);
-    anything else is rejected by the host-side checks."""
-    ok = [dict(), dict(layout=iq.IQ_LAYOUT_NCHW), dict(k_w=4, k_a=4), dict(k_w=2, k_a=8)]
-    bad = [dict(layout=2), dict(layout=-1), dict(k_w=1), dict(k_w=9), dict(k_a=1), dict(k_a=16)]
+    """The descriptor's layout and code widths: NHWC / NCHW, k_w and k_a in 2..8 (0: 8 bits),
+    flags 0 or IQ_CONV_X_F16_READY; anything else is rejected by the host-side checks."""
+    ok = [dict(), dict(layout=iq.IQ_LAYOUT_NCHW), dict(k_w=4, k_a=4), dict(k_w=2, k_a=8),
+          dict(flags=iq.IQ_CONV_X_F16_READY)]
+    bad = [dict(layout=2), dict(layout=-1), dict(k_w=1), dict(k_w=9), dict(k_a=1), dict(k_a=16),
+           dict(flags=2), dict(flags=-1)]
     for kw in ok:
         assert iq.iq_conv_out_size(iq.conv_desc(1, 8, 8, 8, 8, 3, 3, 1, 1, **kw)) == (8, 8)
     for kw in bad:

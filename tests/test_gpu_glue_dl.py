@@ -136,6 +136,50 @@ def test_combine_four_channel_groups(n, hw, c):
                 n, hw, c, False, False)
 
 
+@pytest.mark.parametrize("n,hw,c,kinds,relu", [
+    (3, 37 * 41, 512, ("x16", "x16"), True),      # downsample join, ragged last chunk
+    (2, 29 * 31, 128, ("i8", "x16"), True),       # identity first, 16 row lanes
+    (2, 23 * 19, 2048, ("e8", "e8"), False),      # sum of two errors over two slabs
+    (1, 11 * 13, 3072, ("x16", "i8"), False),     # three slabs of 1024 channels
+    (4, 65 * 65, 1024, ("e8", "e8"), False),      # a full-size stage-3 error sum
+])
+def test_combine_streamed_two_operands(n, hw, c, kinds, relu):
+    """Two operands covering every channel with at least 128 channels (the streamed passes):
+    int16 codes with the BN affine, int8 codes of a shortcut, and plain int8 errors."""
+    g = np.random.default_rng(31 + c + hw)
+    specs = []
+    for k, kind in enumerate(kinds):
+        if kind == "x16":
+            X = g.integers(-32767, 32768, size=(n, hw, c)).astype(np.int16)
+            gam = g.integers(-127, 128, size=c).astype(np.int32)
+            bet = g.integers(-127, 128, size=c).astype(np.int32)
+            specs.append((X, 2.0 ** -15 * (1.7 + k), 0, False, gam, bet))
+        else:
+            lo = 0 if kind == "i8" else -127
+            v = g.integers(lo, 128, size=(n, hw, c)).astype(np.int8)
+            specs.append((v, 0.021 if k else 3e-5, 0, False, None, None))
+    run_combine(specs, n, hw, c, False, relu)
+
+
+def test_combine_streamed_exact_paths():
+    """The streamed passes where fp32 cannot decide: codes of magnitude <= 3 far below the
+    fixed-point bound (every element exact), constant codes (every element at the maximum),
+    and a ReLU sum that is negative everywhere (every code 0)."""
+    g = np.random.default_rng(41)
+    n, hw, c = 2, 17 * 19, 256
+    X = g.integers(-3, 4, size=(n, hw, c)).astype(np.int16)
+    sc = g.integers(-127, 128, size=(n, hw, c)).astype(np.int8)
+    gam = g.integers(-127, 128, size=c).astype(np.int32)
+    run_combine([(X, 2.0 ** -15, 0, False, gam, np.zeros(c, np.int32)),
+                 (sc, 2.0 ** -30, 0, False, None, None)], n, hw, c, False, False)
+    run_combine([(np.full((n, hw, c), 77, np.int8), 0.013, 0, False, None, None),
+                 (np.full((n, hw, c), -5, np.int8), 0.2, 0, False, None, None)], n, hw, c,
+                False, False)
+    neg = -np.abs(g.integers(1, 128, size=(n, hw, c))).astype(np.int8)
+    run_combine([(neg, 0.01, 0, False, None, None), (neg, 0.02, 0, False, None, None)],
+                n, hw, c, False, True)
+
+
 def test_combine_unaligned_operands():
     """Operands whose codes start 8 bytes past a 16-byte boundary (4-byte loads of int8
     codes, 8-byte loads of int16 codes stay aligned): a two-operand residual join and a

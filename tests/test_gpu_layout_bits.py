@@ -168,3 +168,43 @@ def test_four_bit_layer_matches_oracle(ci):
     m2, w2 = O.update(master, gw, gs, 6, k_u=24, k_w=kw)
     assert np.array_equal(host(dm), m2)
     assert np.array_equal(host(dwq).astype(np.int32), w2)
+
+
+def test_shared_input_carrier_ready_flag():
+    """Two layers on one input (a block's first conv and its projection shortcut, the ASPP
+    branches): the first forward writes the input's fp16 copy, the second reads it as it is
+    (IQ_CONV_X_F16_READY); every forward and the weight gradients that read the same copy
+    match the oracle."""
+    n, h, w, c = 2, 33, 31, 128
+    g = S.rng(911)
+    x = S.int8_uniform(g, (n, h, w, c))
+    x16 = torch.empty(x.size, dtype=torch.float16, device=DEV)
+    xd = dev(x)
+    s_x = 0.017
+    for i, (k, r, pd, dl, bn, flags) in enumerate([(256, 1, 0, 1, True, 0),
+                                                   (128, 3, 2, 2, True, iq.IQ_CONV_X_F16_READY),
+                                                   (64, 3, 1, 1, False, iq.IQ_CONV_X_F16_READY)]):
+        cv = O.Conv(n, h, w, c, k, r, r, 1, pd, dl)
+        d = iq.conv_desc(n, h, w, c, k, r, r, 1, pd, dl, flags=flags)
+        p, q = cv.pq
+        wq = O.requant_master(O.uq(S.he_weights(g, (k, r, r, c), c * r * r), 24)).astype(np.int8)
+        acc = O.conv_fwd(cv, x, wq)
+        a = torch.empty((n, p, q, k), dtype=torch.int8, device=DEV)
+        accd = torch.empty((n, p, q, k), dtype=torch.int32, device=DEV)
+        s_a = sc()
+        if bn:
+            gam, bet = S.bn_gamma_beta_codes(g, k)
+            iq.iq_conv_fwd(d, xd, sc(s_x), dev(wq), a, s_a, dev(gam), dev(bet), use_bn=True,
+                           relu=True, acc_out=accd, x_f16=x16)
+            r_ = O.bn_fwd(acc.reshape(-1, k), s_x * 2.0 ** -7, gam, bet)
+            assert np.array_equal(host(a).reshape(-1, k), r_.A)
+        else:
+            iq.iq_conv_fwd(d, xd, sc(s_x), dev(wq), a, s_a, relu=True, acc_out=accd, x_f16=x16)
+        assert np.array_equal(host(accd), acc), i
+        # the weight gradient of this layer reads the same copy
+        e = S.int8_uniform(g, (n, p, q, k))
+        gacc = torch.empty((k, r, r, c), dtype=torch.int64, device=DEV)
+        gq = torch.empty((k, r, r, c), dtype=torch.int8, device=DEV)
+        iq.iq_conv_wgrad(d, dev(e), sc(1e-6), xd, sc(s_x), gq, sc(), gq_mode=1, seed=1, layer=i,
+                         step=0, g_acc_out=gacc, x_f16=x16)
+        assert np.array_equal(host(gacc), O.conv_wgrad(cv, e, x)), i
