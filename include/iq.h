@@ -73,14 +73,16 @@ enum {
  *        step 2^(1-k_w) is the weight factor of the accumulator scale
  *   k_a  bit width of the output activation codes Q_A = SQ(., k_a) (Eq. (AQ1)), 2..8,
  *        0 = 8 (with batch norm the bits argument's k_a, when given, must agree)
- *   flags  0, or IQ_CONV_X_F16_READY: the x_f16 buffer given to iq_conv_fwd /
- *        iq_conv_fwd_frozen already holds the fp16 copy of this call's input codes (an
- *        earlier call on the same input wrote it), so the call reads it and does not write
- *        it; the caller keeps the two in step (a carrier of other codes gives wrong sums).
- *        A storage option with no counterpart in the paper.
+ *   flags  0 or a combination of IQ_CONV_X_F16_READY: the x_f16 buffer given to
+ *        iq_conv_fwd / iq_conv_fwd_frozen already holds the fp16 copy of this call's input
+ *        codes (an earlier call on the same input, or the call that produced the input with
+ *        an fp16 output copy, wrote it), so the call reads it and does not write it; and
+ *        IQ_CONV_E_F16_READY: the same for the e_f16 buffer of iq_conv_dgrad and the errors
+ *        e.  The caller keeps a copy and its codes in step (a copy of other codes gives
+ *        wrong sums).  A storage option with no counterpart in the paper.
  * A zero-initialised descriptor tail gives the paper's setting (NHWC, 8-bit codes). */
 enum { IQ_LAYOUT_NHWC = 0, IQ_LAYOUT_NCHW = 1 };
-enum { IQ_CONV_X_F16_READY = 1 };
+enum { IQ_CONV_X_F16_READY = 1, IQ_CONV_E_F16_READY = 2 };
 typedef struct {
     int32_t n, h, w, c;
     int32_t k, r, s;
@@ -305,12 +307,16 @@ iq_status iq_weight_requant(const int32_t* master, int8_t* wq, int64_t n, int k_
  *             it; keep it for iq_conv_wgrad of the same layer, which then skips its own
  *             conversion of x.  (The paper has no counterpart: it is the
  *             operand format of this implementation's tensor-core path.)
+ *   a_f16     optional out fp16 [n][p][q][k] (16-byte aligned, n p q k % 16 == 0, else
+ *             IQ_ERR_INVALID_ARG): the exact fp16 copy of the output codes a (of their NHWC
+ *             transpose with IQ_LAYOUT_NCHW), written by the pass that writes a; the x_f16 of
+ *             the next layer that reads a, under IQ_CONV_X_F16_READY
  * Returns IQ_ERR_OVERFLOW_RISK when (c/groups) r s 127^2 >= 2^31. */
 iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const double* s_x,
                       const int8_t* w, const int32_t* gamma, const int32_t* beta,
                       const iq_bn_bits* bits, int use_bn, int relu, int8_t* a, double* s_a,
                       int16_t* xhat, int32_t* bn_codes, double* bn_scales, int64_t* frozen_out,
-                      int32_t* acc_out, void* x_f16, void* ws, size_t ws_bytes,
+                      int32_t* acc_out, void* x_f16, void* a_f16, void* ws, size_t ws_bytes,
                       iq_stream stream);
 
 /* iq_conv_fwd_frozen -- the inference forward with frozen statistics.  The paper defines no
@@ -339,7 +345,8 @@ iq_status iq_conv_fwd_frozen(const iq_conv_desc* d, const int8_t* x, const int8_
  *   acc_out optional out int32 [n][h][w][c]; must be NULL when (k/groups) r s 127^2 >= 2^31,
  *           where the sums are accumulated in int64 (IQ_ERR_UNSUPPORTED otherwise)
  *   e_f16   optional out fp16 [n][p][q][k], as x_f16 of iq_conv_fwd for the errors e: written
- *           first and read by the kernels; pass it to iq_conv_wgrad of the same layer */
+ *           first (not with IQ_CONV_E_F16_READY in d->flags: then it is read as it is) and
+ *           read by the kernels; pass it to iq_conv_wgrad of the same layer */
 iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
                         const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
                         void* e_f16, void* ws, size_t ws_bytes, iq_stream stream);
@@ -408,6 +415,9 @@ iq_status iq_bn_int_fwd_noalloc(const int32_t* acc, int64_t m, int32_t c, const 
  *   e_a, s_e   int8 [m][c] error codes of this layer's activation and their scale
  *   a, xhat    the forward outputs;  gamma int32[c];  bn_codes, bn_scales from the forward
  *   e          out int8 [m][c];  s_e_out out device double
+ *   e_f16      optional out fp16 [m][c] (16-byte aligned, m c % 16 == 0, else
+ *              IQ_ERR_INVALID_ARG): the exact fp16 copy of e, written with it, for
+ *              iq_conv_dgrad under IQ_CONV_E_F16_READY (no counterpart in the paper)
  * Workspace: iq_bn_int_workspace_size(m, c) (for c not a power of two in [16, 1024] nor a
  * multiple of 1024 it grows with m: a per-code histogram of each row tile).  Returns
  * IQ_ERR_UNSUPPORTED for m > 65535 * 65536 rows. */
@@ -415,11 +425,13 @@ iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const int8_t* a,
                         const int16_t* xhat, int64_t m, int32_t c, const int32_t* gamma,
                         const int32_t* bn_codes, const double* bn_scales,
                         const iq_bn_bits* bits, int k_e2, int8_t* e, double* s_e_out,
-                        int64_t* dgamma, int64_t* dbeta, void* ws, size_t ws_bytes,
-                        iq_stream stream);
+                        int64_t* dgamma, int64_t* dbeta, void* e_f16, void* ws,
+                        size_t ws_bytes, iq_stream stream);
 
-/* iq_relu_bwd -- layers without BN: e = e_a where a > 0, else 0 (same scale). */
-iq_status iq_relu_bwd(const int8_t* e_a, const int8_t* a, int64_t n, int8_t* e,
+/* iq_relu_bwd -- layers without BN: e = e_a where a > 0, else 0 (same scale).  e_f16:
+ * optional out fp16 [n], the exact fp16 copy of e (e_a, a, e and e_f16 16-byte aligned and
+ * n % 16 == 0, else IQ_ERR_INVALID_ARG), as e_f16 of iq_bn_int_bwd. */
+iq_status iq_relu_bwd(const int8_t* e_a, const int8_t* a, int64_t n, int8_t* e, void* e_f16,
                       iq_stream stream);
 
 /* iq_update -- Eq. (UQ2): Delta W = UQ(G_q lr, k_u) with lr = 2^-lr_log2, plain SGD
@@ -435,9 +447,12 @@ iq_status iq_update(int32_t* master, int8_t* wq, const int8_t* g, const double* 
 
 /* iq_maxpool_fwd -- k x k max pooling, stride s, padding p (padding never wins), on int8
  * codes (positive scale: the scale passes through unchanged).  arg (uint8, output shape)
- * records the tap index r*k + t of the first maximum in scan order for the backward. */
+ * records the tap index r*k + t of the first maximum in scan order for the backward.  y_f16:
+ * optional out fp16 copy of y (16-byte aligned, its size % 16 == 0, else
+ * IQ_ERR_INVALID_ARG), the x_f16 of the conv that reads y under IQ_CONV_X_F16_READY. */
 iq_status iq_maxpool_fwd(const int8_t* x, int32_t n, int32_t h, int32_t w, int32_t c, int32_t k,
-                         int32_t s, int32_t p, int8_t* y, uint8_t* arg, iq_stream stream);
+                         int32_t s, int32_t p, int8_t* y, uint8_t* arg, void* y_f16,
+                         iq_stream stream);
 
 /* iq_maxpool_bwd -- routes each output error to its window's first maximum.  Without
  * overlap (k <= s) the codes pass through and s_ex = s_e; with overlap the int32 sums are
@@ -524,10 +539,13 @@ iq_status iq_combine_workspace_size(const iq_term* terms, int32_t n_terms, size_
  * (|a| vmax + |b|)) (vmax 127 or 32767), at most 62; then code = floor((256 z + M)/(2M))
  * clipped to +-127 with M = max |z|, and s_out = M 2^(-P-7) (M = 0: zero codes,
  * s_out = 2^(-P-7)).  n images of hw pixels; terms is a host array of 1..IQ_MAX_TERMS
- * descriptors (device pointers inside); out int8 [n][hw][c_out]; s_out device double. */
+ * descriptors (device pointers inside); out int8 [n][hw][c_out]; s_out device double.
+ * out_f16: optional out fp16 copy of out (16-byte aligned, n hw c_out % 16 == 0, else
+ * IQ_ERR_INVALID_ARG), the x_f16 of a conv that reads out under IQ_CONV_X_F16_READY (no
+ * counterpart in the paper). */
 iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t concat, int64_t n,
                      int64_t hw, int32_t c_out, int32_t relu, int8_t* out, double* s_out,
-                     void* ws, size_t ws_bytes, iq_stream stream);
+                     void* out_f16, void* ws, size_t ws_bytes, iq_stream stream);
 
 /* Workspace of iq_spatial_sum. */
 iq_status iq_spatial_sum_workspace_size(int64_t n, int32_t c, size_t* bytes);

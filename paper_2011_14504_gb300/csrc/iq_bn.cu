@@ -421,7 +421,8 @@ __global__ void __launch_bounds__(kThreads) k_bn_requant(const int32_t* __restri
                                                          int64_t m, int32_t C, BnStats s,
                                                          int kx, int ka,
                                                          int16_t* __restrict__ X,
-                                                         int8_t* __restrict__ A) {
+                                                         int8_t* __restrict__ A,
+                                                         uint2* __restrict__ A16) {
     const int C4 = C >> 2;
     const int64_t T = (int64_t)gridDim.x * blockDim.x;
     const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -456,6 +457,11 @@ __global__ void __launch_bounds__(kThreads) k_bn_requant(const int32_t* __restri
             reinterpret_cast<uint2*>(X)[v] = xv;
         }
         reinterpret_cast<uint32_t*>(A)[v] = ao;
+        if (A16) {                    // the fp16 copy of the 4 A codes
+            uint2 hv;
+            tc::i8x4_to_f16x4(ao, hv.x, hv.y);
+            A16[v] = hv;
+        }
     };
     int64_t r = t / C4;
     // two rows per iteration: both loads in flight together
@@ -539,6 +545,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) k_bn_requant_s(RowStream rs
                                                                       int kx, int ka,
                                                                       int16_t* __restrict__ X,
                                                                       int8_t* __restrict__ A,
+                                                                      uint2* __restrict__ A16,
                                                                       int* __restrict__ err) {
     extern __shared__ __align__(128) uint8_t smem[];
     if (__syncthreads_or(threadIdx.x == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
@@ -580,6 +587,11 @@ __global__ void __launch_bounds__(kStreamThreads, 1) k_bn_requant_s(RowStream rs
                 *reinterpret_cast<uint2*>(X + e) = xv;
             }
             *reinterpret_cast<uint32_t*>(A + e) = ao;
+            if (A16) {                // the fp16 copy of the 4 A codes
+                uint2 hv;
+                tc::i8x4_to_f16x4(ao, hv.x, hv.y);
+                A16[e >> 2] = hv;
+            }
         }
     });
 }
@@ -702,7 +714,8 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
                              const int32_t* gamma, const int32_t* beta, const iq_bn_bits& b,
                              const BnStats& s, int16_t* xhat, int8_t* a, double* s_a,
                              int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
-                             cudaStream_t st) {
+                             cudaStream_t st, __half* a16) {
+    if (a16 && !f16_copy_ok(a, a16, m * C)) return IQ_ERR_INVALID_ARG;
     RowStream rs;
     const void* srcs[1] = {acc};
     const int esz[1] = {4};
@@ -739,13 +752,15 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
         iq_status r = stream_attr(k_bn_requant_s, attr);
         if (r != IQ_OK) return r;
         k_bn_requant_s<<<row_stream_grid(rs, device_sms()), kStreamThreads, row_stream_smem(rs),
-                         st>>>(rs, s, b.k_xhat, b.k_a, xhat, a, err);
+                         st>>>(rs, s, b.k_xhat, b.k_a, xhat, a, (uint2*)a16, err);
     } else {
         ChanGrid g2 = chan_grid(m, C / 4, 152 * 16);
-        k_bn_requant<<<g2.blocks, kThreads, 0, st>>>(acc, m, C, s, b.k_xhat, b.k_a, xhat, a);
+        k_bn_requant<<<g2.blocks, kThreads, 0, st>>>(acc, m, C, s, b.k_xhat, b.k_a, xhat, a,
+                                                     (uint2*)a16);
     }
     IQ_LAUNCH_CHECK();
-    kt_post_bytes(st, IQ_KERNEL_BN_REQUANT, (double)m * C * (xhat ? 7.0 : 5.0));
+    kt_post_bytes(st, IQ_KERNEL_BN_REQUANT,
+                  (double)m * C * ((xhat ? 7.0 : 5.0) + (a16 ? 2.0 : 0.0)));
     k_bn_export<<<(C + 255) / 256, 256, 0, st>>>(s, C, s.codes, s_a, bn_codes, bn_scales,
                                                  bn_fixed);
     IQ_LAUNCH_CHECK();
@@ -1414,7 +1429,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
 __global__ void __launch_bounds__(kStreamThreads, 1)
     k_bnb_out_t(const __grid_constant__ CUtensorMap me, const __grid_constant__ CUtensorMap ma,
                 const __grid_constant__ CUtensorMap mxh, int64_t m, int32_t C, BnBwd w,
-                int8_t* __restrict__ out, int* __restrict__ err) {
+                int8_t* __restrict__ out, uint2* __restrict__ out16, int* __restrict__ err) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1k(smem_raw);
     uint8_t* tab = smem + kTileStages * kTileStage + 2 * kTileStages * 8;   // [64][kTab3P]
@@ -1454,7 +1469,13 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
                     const int sg = (x[j] > 0) - (x[j] < 0);
                     o |= ((uint32_t)(uint8_t)tb[j * kTab3P + sg * 256 + v]) << (8 * j);
                 }
-                *reinterpret_cast<uint32_t*>(out + (r0 + r) * C + c_base + 4 * g) = o;
+                const int64_t oi = (r0 + r) * C + c_base + 4 * g;
+                *reinterpret_cast<uint32_t*>(out + oi) = o;
+                if (out16) {          // the fp16 copy of the 4 error codes
+                    uint2 hv;
+                    tc::i8x4_to_f16x4(o, hv.x, hv.y);
+                    out16[oi >> 2] = hv;
+                }
             }
         });
 }
@@ -1633,9 +1654,10 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
                                    const int32_t* gamma, const int32_t* bn_codes,
                                    const double* bn_scales, const iq_bn_bits* bits, int k_e2,
                                    int8_t* e, double* s_e_out, int64_t* dgamma, int64_t* dbeta,
-                                   void* ws, size_t ws_bytes, iq_stream stream) {
+                                   void* e_f16, void* ws, size_t ws_bytes, iq_stream stream) {
     if (!e_a || !s_e || !a || !xhat || !gamma || !bn_codes || !bn_scales || !e || !s_e_out)
         return IQ_ERR_INVALID_ARG;
+    if (e_f16 && !f16_copy_ok(e, e_f16, m * (int64_t)c)) return IQ_ERR_INVALID_ARG;
     if (!bn_shape_ok(m, c)) return (m > 0 && c > 0) ? IQ_ERR_UNSUPPORTED : IQ_ERR_INVALID_ARG;
     iq_bn_bits b = bn_bits_or_default(bits);
     if (!bn_bits_valid(b) || k_e2 < 2 || k_e2 > 16) return IQ_ERR_INVALID_ARG;
@@ -1710,9 +1732,10 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
         k_bnb_tab3<<<tb3 < 152 * 4 ? tb3 : 152 * 4, kThreads, 0, st>>>(gamma, c, k_e2, 8, w);
         IQ_LAUNCH_CHECK();
         kt_pre(st);
-        k_bnb_out_t<<<tgrid, kStreamThreads, smem_o, st>>>(me, ma, mxh, m, c, w, e, err);
+        k_bnb_out_t<<<tgrid, kStreamThreads, smem_o, st>>>(me, ma, mxh, m, c, w, e,
+                                                           (uint2*)e_f16, err);
         IQ_LAUNCH_CHECK();
-        kt_post_bytes(st, IQ_KERNEL_BNB_PASS3, 5.0 * (double)m * c);
+        kt_post_bytes(st, IQ_KERNEL_BNB_PASS3, (e_f16 ? 7.0 : 5.0) * (double)m * c);
     } else {
         const int gy = hist_tiles(m, c);
         static bool hist_attr = false;
@@ -1762,6 +1785,10 @@ extern "C" iq_status iq_bn_int_bwd(const int8_t* e_a, const double* s_e, const i
         }
         IQ_LAUNCH_CHECK();
         kt_post_bytes(st, IQ_KERNEL_BNB_PASS3, 5.0 * (double)m * c);
+        if (e_f16) {
+            iq_status r = codes_to_f16(e, (__half*)e_f16, m * (int64_t)c, st);
+            if (r != IQ_OK) return r;
+        }
     }
     if (dgamma)
         IQ_CUDA_CHECK(cudaMemcpyAsync(dgamma, w.sg, sizeof(int64_t) * c, cudaMemcpyDeviceToDevice, st));

@@ -397,7 +397,7 @@ static bool desc_ok(const iq_conv_desc* d) {
     if (d->layout != IQ_LAYOUT_NHWC && d->layout != IQ_LAYOUT_NCHW) return false;
     if (d->k_w != 0 && (d->k_w < 2 || d->k_w > 8)) return false;
     if (d->k_a != 0 && (d->k_a < 2 || d->k_a > 8)) return false;
-    if (d->flags & ~IQ_CONV_X_F16_READY) return false;
+    if (d->flags & ~(IQ_CONV_X_F16_READY | IQ_CONV_E_F16_READY)) return false;
     int p = (d->h + 2 * d->pad_h - d->dil_h * (d->r - 1) - 1);
     int q = (d->w + 2 * d->pad_w - d->dil_w * (d->s - 1) - 1);
     return p >= 0 && q >= 0;
@@ -696,11 +696,16 @@ static iq_status conv_fwd_nhwc(const iq_conv_desc* d, const int8_t* x, const dou
                                const int8_t* w, const int32_t* gamma, const int32_t* beta,
                                const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
                                double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
-                               int64_t* frozen_out, int32_t* acc_out, void* x_f16, void* ws,
-                               size_t ws_bytes, iq_stream stream) {
+                               int64_t* frozen_out, int32_t* acc_out, void* x_f16, void* a_f16,
+                               void* ws, size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d) || !x || !s_x || !w || !a || !s_a) return IQ_ERR_INVALID_ARG;
     const int64_t nx = (int64_t)d->n * d->h * d->w * d->c;
     if (x_f16 && (nx % 16 || (((uintptr_t)x | (uintptr_t)x_f16) & 15))) return IQ_ERR_INVALID_ARG;
+    if (a_f16) {
+        int32_t pp = 0, qq = 0;
+        iq_conv_out_size(d, &pp, &qq);
+        if (!f16_copy_ok(a, a_f16, (int64_t)d->n * pp * qq * d->k)) return IQ_ERR_INVALID_ARG;
+    }
     if (crs_overflow(d)) return IQ_ERR_OVERFLOW_RISK;
     kt_set_op(1, conv_macs(d), conv_macs_dense(d));
     iq_bn_bits b = bn_bits_or_default(bits);
@@ -770,7 +775,7 @@ static iq_status conv_fwd_nhwc(const iq_conv_desc* d, const int8_t* x, const dou
     }
     if (use_bn)
         return bn_fwd_after_stats(acc, cp.M, cp.K, L.s_acc, gamma, beta, b, L.st, xhat, a, s_a,
-                                  bn_codes, bn_scales, frozen_out, st);
+                                  bn_codes, bn_scales, frozen_out, st, (__half*)a_f16);
     // Q_A = SQ(act(acc), 8) with M from the per-channel extremes
     unsigned long long* cell = (unsigned long long*)L.rq;
     k_max_from_stats<<<1, 1024, 0, st>>>(L.st.hi, L.st.lo, cp.K, relu, L.s_acc, cell,
@@ -781,7 +786,7 @@ static iq_status conv_fwd_nhwc(const iq_conv_desc* d, const int8_t* x, const dou
                                       st));
     return requant_apply(acc, IQ_I32, cp.npq * cp.K, L.s_acc, ka,
                          relu ? IQ_MODE_SQ_RELU : IQ_MODE_SQ, 0, 0, 0, 0, a, IQ_I8, s_a, L.rq, st,
-                         true);
+                         true, false, (__half*)a_f16);
 }
 
 // frozen Q_A parameters from the calibration maximum M = frozen[0]
@@ -895,7 +900,7 @@ static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const d
     k_scale_mul_pow2<<<1, 1, 0, st>>>(s_e, 1 - code_kw(d), s_in);   // the W_q step 2^(1-k_w)
     IQ_LAUNCH_CHECK();
     int32_t* acc = acc_out ? acc_out : reinterpret_cast<int32_t*>(accw);
-    if (e_f16) {
+    if (e_f16 && !(d->flags & IQ_CONV_E_F16_READY)) {
         const int64_t ne = (int64_t)d->n * cp.P * cp.Q * d->k;
         iq_status r0 = codes_to_f16(e, (__half*)e_f16, ne, st);
         if (r0 != IQ_OK) return r0;
@@ -1155,13 +1160,13 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
                                  const int8_t* w, const int32_t* gamma, const int32_t* beta,
                                  const iq_bn_bits* bits, int use_bn, int relu, int8_t* a,
                                  double* s_a, int16_t* xhat, int32_t* bn_codes, double* bn_scales,
-                                 int64_t* frozen_out, int32_t* acc_out, void* x_f16, void* ws,
-                                 size_t ws_bytes, iq_stream stream) {
+                                 int64_t* frozen_out, int32_t* acc_out, void* x_f16,
+                                 void* a_f16, void* ws, size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d)) return IQ_ERR_INVALID_ARG;
     if (d->layout == IQ_LAYOUT_NHWC)
         return conv_fwd_nhwc(d, x, s_x, w, gamma, beta, bits, use_bn, relu, a, s_a, xhat,
-                             bn_codes, bn_scales, frozen_out, acc_out, x_f16, ws, ws_bytes,
-                             stream);
+                             bn_codes, bn_scales, frozen_out, acc_out, x_f16, a_f16, ws,
+                             ws_bytes, stream);
     if (!x || !s_x || !w || !a || !s_a) return IQ_ERR_INVALID_ARG;
     int64_t nin, nw, nout, pq;
     conv_sizes(d, &nin, &nw, &nout, &pq);
@@ -1181,7 +1186,7 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
     int32_t* accn = acc_out ? (int32_t*)(b + L.off_acc) : nullptr;
     r = conv_fwd_nhwc(&dn, (const int8_t*)(b + L.off_x), s_x, (const int8_t*)(b + L.off_w), gamma,
                       beta, bits, use_bn, relu, an, s_a, xn, bn_codes, bn_scales, frozen_out,
-                      accn, x_f16, b + L.off_rest, ws_bytes - L.off_rest, stream);
+                      accn, x_f16, a_f16, b + L.off_rest, ws_bytes - L.off_rest, stream);
     if (r != IQ_OK) return r;
     r = to_nchw(an, a, d->n, d->k, pq, 1, st);
     if (r == IQ_OK && xhat) r = to_nchw(xn, xhat, d->n, d->k, pq, 2, st);

@@ -4,6 +4,7 @@
 // the quantized gradient of the MSE loss on quantized logits (Sec. 5).
 // All of these are bandwidth-bound element-wise or windowed kernels on NHWC codes.
 #include "iq_internal.cuh"
+#include "iq_tc_ptx.cuh"
 
 #include <climits>
 
@@ -42,7 +43,7 @@ __global__ void k_maxpool_fwd(const int8_t* __restrict__ x, int n, int h, int w,
 // row's Q x c/4 channel groups); 4-byte loads and stores, no 64-bit divisions
 __global__ void k_maxpool_fwd4(const int8_t* __restrict__ x, int h, int w, int c, int k, int s,
                                int p, int P, int Q, int8_t* __restrict__ y,
-                               uint8_t* __restrict__ arg) {
+                               uint8_t* __restrict__ arg, uint2* __restrict__ y16) {
     const int c4 = c >> 2;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= Q * c4) return;
@@ -73,6 +74,11 @@ __global__ void k_maxpool_fwd4(const int8_t* __restrict__ x, int h, int w, int c
     const int64_t o = (((int64_t)b * P + i) * Q + j) * c + 4 * cg;
     *reinterpret_cast<uint32_t*>(y + o) = yo;
     *reinterpret_cast<uint32_t*>(arg + o) = ao;
+    if (y16) {                        // the fp16 copy of the 4 output codes
+        uint2 hv;
+        tc::i8x4_to_f16x4(yo, hv.x, hv.y);
+        y16[o >> 2] = hv;
+    }
 }
 
 // gather form of the backward: input position (hh, ww) sums the errors of the
@@ -715,23 +721,25 @@ using namespace iq;
 
 extern "C" iq_status iq_maxpool_fwd(const int8_t* x, int32_t n, int32_t h, int32_t w, int32_t c,
                                     int32_t k, int32_t s, int32_t p, int8_t* y, uint8_t* arg,
-                                    iq_stream stream) {
+                                    void* y_f16, iq_stream stream) {
     if (!x || !y || !arg || n <= 0 || h <= 0 || w <= 0 || c <= 0 || k <= 0 || s <= 0 || p < 0 ||
         k > 15 || 2 * p >= k + 1 || h + 2 * p < k || w + 2 * p < k)
         return IQ_ERR_INVALID_ARG;
     int P = (h + 2 * p - k) / s + 1, Q = (w + 2 * p - k) / s + 1;
     int64_t total = (int64_t)n * P * Q * c;
+    if (y_f16 && !f16_copy_ok(y, y_f16, total)) return IQ_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
     if (c % 4 == 0 && (((uintptr_t)x | (uintptr_t)y | (uintptr_t)arg) & 3) == 0 && n <= 65535 &&
         P <= 65535) {
         dim3 grid((unsigned)((Q * (c / 4) + kThreads - 1) / kThreads), (unsigned)P, (unsigned)n);
-        k_maxpool_fwd4<<<grid, kThreads, 0, (cudaStream_t)stream>>>(x, h, w, c, k, s, p, P, Q, y,
-                                                                   arg);
+        k_maxpool_fwd4<<<grid, kThreads, 0, st>>>(x, h, w, c, k, s, p, P, Q, y, arg,
+                                                   (uint2*)y_f16);
         IQ_LAUNCH_CHECK();
         return IQ_OK;
     }
-    k_maxpool_fwd<<<grid_for(total), kThreads, 0, (cudaStream_t)stream>>>(x, n, h, w, c, k, s, p,
-                                                                          P, Q, y, arg);
+    k_maxpool_fwd<<<grid_for(total), kThreads, 0, st>>>(x, n, h, w, c, k, s, p, P, Q, y, arg);
     IQ_LAUNCH_CHECK();
+    if (y_f16) return codes_to_f16(y, (__half*)y_f16, total, st);
     return IQ_OK;
 }
 

@@ -2,6 +2,7 @@
 #pragma once
 
 #include "iq_common.cuh"
+#include <cuda_fp16.h>
 
 #include <cuda.h>
 
@@ -58,10 +59,19 @@ inline RqParams* rq_params_slot(void* ws) { return (RqParams*)((char*)ws + 256);
 // params_ready the parameters (rq_params_slot) and *s_out have been written as well.  clip:
 // the SQ modes' M is not the tensor's own maximum (frozen statistics), so q is clipped to
 // [-M, M] first.
+// out16 (optional, int8 SQ codes only): the fp16 copy of the output codes is written too
+// (n % 16 == 0, out and out16 16-byte aligned).
 iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
                         void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st,
-                        bool params_ready = false, bool clip = false);
+                        bool params_ready = false, bool clip = false, __half* out16 = nullptr);
+
+// int8 codes -> their exact fp16 copies (n % 16 == 0, both 16-byte aligned)
+iq_status codes_to_f16(const int8_t* x, __half* xf, int64_t n, cudaStream_t st);
+// an fp16 output copy is valid for n codes at these addresses
+inline bool f16_copy_ok(const void* codes, const void* xf, int64_t n) {
+    return n % 16 == 0 && (((uintptr_t)codes | (uintptr_t)xf) & 15) == 0;
+}
 
 // Per-channel statistics buffers of a BN layer, in the workspace.
 struct BnStats {
@@ -92,7 +102,7 @@ iq_status bn_fwd_after_stats(const int32_t* acc, int64_t m, int32_t C, const dou
                              const int32_t* gamma, const int32_t* beta, const iq_bn_bits& b,
                              const BnStats& s, int16_t* xhat, int8_t* a, double* s_a,
                              int32_t* bn_codes, double* bn_scales, int64_t* bn_fixed,
-                             cudaStream_t st);
+                             cudaStream_t st, __half* a16 = nullptr);
 
 // the forward's element maps with frozen constants (F, B, G, H, P_x, P_a from an earlier call)
 iq_status bn_apply_fixed(const int32_t* acc, int64_t m, int32_t C, const int64_t* fixed, int kx,

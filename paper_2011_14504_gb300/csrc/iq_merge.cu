@@ -804,7 +804,7 @@ template <int PASS, bool A16, bool B16, bool PLAIN>
 __global__ void __launch_bounds__(kStreamThreads, 1)
     k_comb_s(RowStream rs, Terms T, int relu, const long long* __restrict__ F,
              const long long* __restrict__ B, CombHdr* hdr, int8_t* __restrict__ out,
-             int* __restrict__ err) {
+             uint2* __restrict__ out16, int* __restrict__ err) {
     extern __shared__ __align__(128) uint8_t smem[];
     if (__syncthreads_or(threadIdx.x == 0 ? *reinterpret_cast<volatile int*>(err) : 0)) return;
     constexpr int FW = PLAIN ? 1 : 4;
@@ -928,7 +928,13 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
                     w = __byte_perm(__byte_perm(tb[0], tb[1], 0x0040),
                                     __byte_perm(tb[2], tb[3], 0x0040), 0x5410);
                 }
-                *reinterpret_cast<uint32_t*>(out + (r0 + r) * rs.C + c0) = w;
+                const int64_t oi = (r0 + r) * rs.C + c0;
+                *reinterpret_cast<uint32_t*>(out + oi) = w;
+                if (out16) {          // the fp16 copy of the 4 codes
+                    uint2 hv;
+                    tc::i8x4_to_f16x4(w, hv.x, hv.y);
+                    out16[oi >> 2] = hv;
+                }
             }
     };
     const bool ok = stream_chunks(rs, smem, err, [&](const uint8_t* st, int rows, int64_t r0) {
@@ -955,7 +961,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
 // the dynamic shared memory of one instantiation, set once
 template <int PASS, bool A16, bool B16, bool PLAIN>
 iq_status comb_s_launch(const RowStream& rs, const Terms& T, int relu, const long long* F,
-                        const long long* B, CombHdr* hdr, int8_t* out, int* err,
+                        const long long* B, CombHdr* hdr, int8_t* out, uint2* out16, int* err,
                         cudaStream_t st) {
     static bool attr = false;
     auto kern = k_comb_s<PASS, A16, B16, PLAIN>;
@@ -965,7 +971,7 @@ iq_status comb_s_launch(const RowStream& rs, const Terms& T, int relu, const lon
         attr = true;
     }
     kern<<<row_stream_grid(rs, device_sms()), kStreamThreads, row_stream_smem(rs), st>>>(
-        rs, T, relu, F, B, hdr, out, err);
+        rs, T, relu, F, B, hdr, out, out16, err);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }
@@ -973,13 +979,17 @@ iq_status comb_s_launch(const RowStream& rs, const Terms& T, int relu, const lon
 template <int PASS>
 iq_status comb_s_pass(const RowStream& rs, const Terms& T, bool plain, int relu,
                       const long long* F, const long long* B, CombHdr* hdr, int8_t* out,
-                      int* err, cudaStream_t st) {
+                      uint2* o16, int* err, cudaStream_t st) {
     const bool a16 = T.t[0].is16 != 0, b16 = T.t[1].is16 != 0;
-    if (plain) return comb_s_launch<PASS, false, false, true>(rs, T, relu, F, B, hdr, out, err, st);
-    if (a16 && b16) return comb_s_launch<PASS, true, true, false>(rs, T, relu, F, B, hdr, out, err, st);
-    if (a16) return comb_s_launch<PASS, true, false, false>(rs, T, relu, F, B, hdr, out, err, st);
-    if (b16) return comb_s_launch<PASS, false, true, false>(rs, T, relu, F, B, hdr, out, err, st);
-    return comb_s_launch<PASS, false, false, false>(rs, T, relu, F, B, hdr, out, err, st);
+    if (plain)
+        return comb_s_launch<PASS, false, false, true>(rs, T, relu, F, B, hdr, out, o16, err, st);
+    if (a16 && b16)
+        return comb_s_launch<PASS, true, true, false>(rs, T, relu, F, B, hdr, out, o16, err, st);
+    if (a16)
+        return comb_s_launch<PASS, true, false, false>(rs, T, relu, F, B, hdr, out, o16, err, st);
+    if (b16)
+        return comb_s_launch<PASS, false, true, false>(rs, T, relu, F, B, hdr, out, o16, err, st);
+    return comb_s_launch<PASS, false, false, false>(rs, T, relu, F, B, hdr, out, o16, err, st);
 }
 
 // ---------------------------------------------------------------- spatial sums
@@ -1092,12 +1102,32 @@ extern "C" iq_status iq_combine_workspace_size(const iq_term* terms, int32_t n_t
     return IQ_OK;
 }
 
+static iq_status combine_codes(const iq_term* terms, int32_t n_terms, int32_t concat, int64_t n,
+                               int64_t hw, int32_t c_out, int32_t relu, int8_t* out,
+                               double* s_out, uint2* out16, bool& wrote16, void* ws,
+                               size_t ws_bytes, iq_stream stream);
+
 extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t concat, int64_t n,
                                 int64_t hw, int32_t c_out, int32_t relu, int8_t* out,
-                                double* s_out, void* ws, size_t ws_bytes, iq_stream stream) {
+                                double* s_out, void* out_f16, void* ws, size_t ws_bytes,
+                                iq_stream stream) {
     if (!terms_ok(terms, n_terms) || !out || !s_out || n < 1 || hw < 1 || c_out < 1)
         return IQ_ERR_INVALID_ARG;
     if (n * hw > (int64_t(1) << 40)) return IQ_ERR_INVALID_ARG;
+    if (out_f16 && !f16_copy_ok(out, out_f16, n * hw * (int64_t)c_out)) return IQ_ERR_INVALID_ARG;
+    bool wrote16 = false;
+    iq_status r = combine_codes(terms, n_terms, concat, n, hw, c_out, relu, out, s_out,
+                                (uint2*)out_f16, wrote16, ws, ws_bytes, stream);
+    if (r != IQ_OK || !out_f16 || wrote16) return r;
+    // the kernels without the fused copy: one conversion pass
+    return codes_to_f16(out, (__half*)out_f16, n * hw * (int64_t)c_out, (cudaStream_t)stream);
+}
+
+// the joins; out16 is written by the streamed codes pass (wrote16), else left to the caller
+static iq_status combine_codes(const iq_term* terms, int32_t n_terms, int32_t concat, int64_t n,
+                               int64_t hw, int32_t c_out, int32_t relu, int8_t* out,
+                               double* s_out, uint2* out16, bool& wrote16, void* ws,
+                               size_t ws_bytes, iq_stream stream) {
     Terms T;
     T.n = n_terms;
     int32_t base = 0;
@@ -1169,15 +1199,16 @@ extern "C" iq_status iq_combine(const iq_term* terms, int32_t n_terms, int32_t c
             if (!err) return IQ_ERR_CUDA;
             const int rl = relu != 0;
             kt_pre(st);
-            iq_status r = comb_s_pass<0>(rs, T, plain, rl, F, B, hdr, out, err, st);
+            iq_status r = comb_s_pass<0>(rs, T, plain, rl, F, B, hdr, out, nullptr, err, st);
             if (r != IQ_OK) return r;
             kt_post_bytes(st, IQ_KERNEL_COMBINE_MAX, in_b);
             k_comb_params<<<1, 1, 0, st>>>(hdr, s_out);
             IQ_LAUNCH_CHECK();
             kt_pre(st);
-            r = comb_s_pass<1>(rs, T, plain, rl, F, B, hdr, out, err, st);
+            r = comb_s_pass<1>(rs, T, plain, rl, F, B, hdr, out, out16, err, st);
             if (r != IQ_OK) return r;
-            kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b);
+            kt_post_bytes(st, IQ_KERNEL_COMBINE_CODES, in_b + out_b * (out16 ? 3.0 : 1.0));
+            wrote16 = out16 != nullptr;
             return IQ_OK;
         }
     }

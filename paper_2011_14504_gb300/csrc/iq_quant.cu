@@ -4,6 +4,7 @@
 // grid-stride loops over a grid of a few blocks per SM, warp-shuffle + one
 // atomic per warp for the tensor-wide max |x| that Scale(x) needs.
 #include "iq_internal.cuh"
+#include "iq_tc_ptx.cuh"
 
 #include <atomic>
 #include <mutex>
@@ -174,10 +175,21 @@ __device__ __forceinline__ uint32_t sq8_word(const int4& v, uint32_t M, uint32_t
            (sq8_byte<CLIP>(v.z, M, R8, relu) << 16) | (sq8_byte<CLIP>(v.w, M, R8, relu) << 24);
 }
 
-// int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores)
+// the fp16 copy of 4 codes (one 8-byte store) when the caller asked for it
+__device__ __forceinline__ void put_f16x4(uint2* __restrict__ out16, int64_t i, uint32_t w) {
+    if (out16) {
+        uint2 h;
+        tc::i8x4_to_f16x4(w, h.x, h.y);
+        out16[i] = h;
+    }
+}
+
+// int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores), and
+// optionally their fp16 copies
 template <bool CLIP>
 __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int relu,
-                              const RqParams* __restrict__ prm, uint32_t* __restrict__ out) {
+                              const RqParams* __restrict__ prm, uint32_t* __restrict__ out,
+                              uint2* __restrict__ out16) {
     const RqParams p = *prm;
     const int64_t lim = qmax(k);
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -192,7 +204,11 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
                 v[j] = i + j * stride < n4 ? __ldg(q + i + j * stride) : make_int4(0, 0, 0, 0);
 #pragma unroll
             for (int j = 0; j < 4; j++)
-                if (i + j * stride < n4) out[i + j * stride] = sq8_word<CLIP>(v[j], M, p.R8, relu);
+                if (i + j * stride < n4) {
+                    const uint32_t w = sq8_word<CLIP>(v[j], M, p.R8, relu);
+                    out[i + j * stride] = w;
+                    put_f16x4(out16, i + j * stride, w);
+                }
         }
         return;
     }
@@ -201,15 +217,20 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
         const int64_t i2 = i + stride;
         const int4 v = __ldg(q + i);
         const int4 v2 = i2 < n4 ? __ldg(q + i2) : make_int4(0, 0, 0, 0);
-        out[i] = ((uint32_t)sq_code<CLIP>(v.x, p, k, relu, lim) & 0xffu) |
-                 (((uint32_t)sq_code<CLIP>(v.y, p, k, relu, lim) & 0xffu) << 8) |
-                 (((uint32_t)sq_code<CLIP>(v.z, p, k, relu, lim) & 0xffu) << 16) |
-                 (((uint32_t)sq_code<CLIP>(v.w, p, k, relu, lim) & 0xffu) << 24);
-        if (i2 < n4)
-            out[i2] = ((uint32_t)sq_code<CLIP>(v2.x, p, k, relu, lim) & 0xffu) |
-                      (((uint32_t)sq_code<CLIP>(v2.y, p, k, relu, lim) & 0xffu) << 8) |
-                      (((uint32_t)sq_code<CLIP>(v2.z, p, k, relu, lim) & 0xffu) << 16) |
-                      (((uint32_t)sq_code<CLIP>(v2.w, p, k, relu, lim) & 0xffu) << 24);
+        const uint32_t w = ((uint32_t)sq_code<CLIP>(v.x, p, k, relu, lim) & 0xffu) |
+                           (((uint32_t)sq_code<CLIP>(v.y, p, k, relu, lim) & 0xffu) << 8) |
+                           (((uint32_t)sq_code<CLIP>(v.z, p, k, relu, lim) & 0xffu) << 16) |
+                           (((uint32_t)sq_code<CLIP>(v.w, p, k, relu, lim) & 0xffu) << 24);
+        out[i] = w;
+        put_f16x4(out16, i, w);
+        if (i2 < n4) {
+            const uint32_t w2 = ((uint32_t)sq_code<CLIP>(v2.x, p, k, relu, lim) & 0xffu) |
+                                (((uint32_t)sq_code<CLIP>(v2.y, p, k, relu, lim) & 0xffu) << 8) |
+                                (((uint32_t)sq_code<CLIP>(v2.z, p, k, relu, lim) & 0xffu) << 16) |
+                                (((uint32_t)sq_code<CLIP>(v2.w, p, k, relu, lim) & 0xffu) << 24);
+            out[i2] = w2;
+            put_f16x4(out16, i2, w2);
+        }
     }
 }
 
@@ -291,7 +312,10 @@ __global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
 iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
                         void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st,
-                        bool params_ready, bool clip) {
+                        bool params_ready, bool clip, __half* out16) {
+    if (out16 && (out_dtype != IQ_I8 || !f16_copy_ok(out, out16, n) ||
+                  (mode != IQ_MODE_SQ && mode != IQ_MODE_SQ_RELU)))
+        return IQ_ERR_INVALID_ARG;
     unsigned long long* cell = (unsigned long long*)ws;
     RqParams* prm = rq_params_slot(ws);
     bool relu = mode == IQ_MODE_SQ_RELU;
@@ -308,11 +332,11 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
         const bool x4 = in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
                         (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0;
         if (x4 && clip)
-            k_sq_i32_i8x4<true><<<grid_for(n / 4), kThreads, 0, st>>>((const int4*)q, n / 4, k,
-                                                                      relu, prm, (uint32_t*)out);
+            k_sq_i32_i8x4<true><<<grid_for(n / 4), kThreads, 0, st>>>(
+                (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16);
         else if (x4)
-            k_sq_i32_i8x4<false><<<grid_for(n / 4), kThreads, 0, st>>>((const int4*)q, n / 4, k,
-                                                                       relu, prm, (uint32_t*)out);
+            k_sq_i32_i8x4<false><<<grid_for(n / 4), kThreads, 0, st>>>(
+                (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16);
         else if (in_dtype == IQ_I32 && clip)
             k_sq_int<int32_t, true><<<g, kThreads, 0, st>>>((const int32_t*)q, n, k, relu, prm,
                                                             out, out_dtype);
@@ -334,9 +358,13 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
                                                        step, tag, ep, out, out_dtype);
     }
     IQ_LAUNCH_CHECK();
+    const bool fused16 = out16 && in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
+                         (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0;
     kt_post_bytes(st, (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) ? IQ_KERNEL_SQ_CODES
                                                                        : IQ_KERNEL_RQ_CODES,
-                  (double)n * (isz + osz));
+                  (double)n * (isz + osz + (fused16 ? 2.0 : 0.0)));
+    // the kernels without the fused copy: one conversion pass
+    if (out16 && !fused16) return codes_to_f16((const int8_t*)out, out16, n, st);
     return IQ_OK;
 }
 
@@ -457,7 +485,7 @@ __global__ void k_update(int32_t* __restrict__ master, int8_t* __restrict__ wq,
 }
 
 __global__ void k_relu_bwd(const int8_t* __restrict__ ea, const int8_t* __restrict__ a,
-                           int64_t n, int8_t* __restrict__ e) {
+                           int64_t n, int8_t* __restrict__ e, uint2* __restrict__ e16) {
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
     int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     bool vec = (((uintptr_t)ea | (uintptr_t)a | (uintptr_t)e) & 15) == 0;
@@ -476,6 +504,7 @@ __global__ void k_relu_bwd(const int8_t* __restrict__ ea, const int8_t* __restri
                 r |= (mv > 0 ? xv : 0u) << (8 * b);
             }
             xs[j] = (int)r;
+            put_f16x4(e16, 4 * v + j, r);
         }
         reinterpret_cast<int4*>(e)[v] = make_int4(xs[0], xs[1], xs[2], xs[3]);
     }
@@ -791,10 +820,14 @@ extern "C" iq_status iq_update(int32_t* master, int8_t* wq, const int8_t* g, con
 }
 
 extern "C" iq_status iq_relu_bwd(const int8_t* e_a, const int8_t* a, int64_t n, int8_t* e,
-                                 iq_stream stream) {
+                                 void* e_f16, iq_stream stream) {
     if (!e_a || !a || !e || n < 0) return IQ_ERR_INVALID_ARG;
+    // the fp16 copy rides on the 16-code vector loop: every operand 16-byte aligned
+    if (e_f16 && (!f16_copy_ok(e, e_f16, n) || (((uintptr_t)e_a | (uintptr_t)a) & 15)))
+        return IQ_ERR_INVALID_ARG;
     if (n == 0) return IQ_OK;
-    k_relu_bwd<<<grid_for(n / 16 + 1), kThreads, 0, (cudaStream_t)stream>>>(e_a, a, n, e);
+    k_relu_bwd<<<grid_for(n / 16 + 1), kThreads, 0, (cudaStream_t)stream>>>(e_a, a, n, e,
+                                                                           (uint2*)e_f16);
     IQ_LAUNCH_CHECK();
     return IQ_OK;
 }

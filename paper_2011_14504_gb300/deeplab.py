@@ -42,6 +42,7 @@ class Layer:
         p, q = iq.iq_conv_out_size(self.desc)
         self.out_shape = (n, p, q, spec.cout)
         self.x16 = None
+        self.a16 = None        # the next layer's x16 when that layer reads a: written here
         self.master = net.master(w_fp32)
         self.wq = torch.empty((spec.cout, spec.r, spec.r, spec.cin), dtype=torch.int8, device=dev)
         iq.iq_weight_requant(self.master, self.wq)
@@ -95,23 +96,26 @@ class Layer:
         if self.spec.bn:
             iq.iq_conv_fwd(self.desc, self.x, self.s_x, self.wq, self.a, self.s_a, self.gamma,
                            self.beta, use_bn=True, relu=True, xhat=self.X, bn_codes=self.bn_codes,
-                           bn_scales=self.bn_scales, x_f16=self.x16, ws=ws, stream=stream)
+                           bn_scales=self.bn_scales, x_f16=self.x16, a_f16=self.a16, ws=ws,
+                           stream=stream)
         else:
             iq.iq_conv_fwd(self.desc, self.x, self.s_x, self.wq, self.a, self.s_a, relu=False,
-                           x_f16=self.x16, ws=ws, stream=stream)
+                           x_f16=self.x16, a_f16=self.a16, ws=ws, stream=stream)
 
     def backward(self, net, e_a, s_ea, mask=None, need_dx=True, stream=None):
         """From the error of the output codes (before the ReLU mask) to the error of the
         input, with the weight and gamma / beta updates of this layer."""
         ws, step, seed, lr = net.ws, net.step_count, net.seed, net.lr_log2
+        e16 = net.e16 if need_dx and self.spec.cout % 64 == 0 else None
         if self.spec.bn:
+            # the errors and their fp16 copy for this layer's data and weight gradients
+            # (the descriptor carries IQ_CONV_E_F16_READY)
             iq.iq_bn_int_bwd(e_a, s_ea, self.a if mask is None else mask, self.X, self.gamma,
                              self.bn_codes, self.bn_scales, self.e, self.s_e, self.dgamma,
-                             self.dbeta, k_e2=K_E2, ws=ws, stream=stream)
+                             self.dbeta, k_e2=K_E2, e_f16=e16, ws=ws, stream=stream)
             e, s_e = self.e, self.s_e
         else:
             e, s_e = e_a, s_ea
-        e16 = net.e16 if need_dx and self.spec.cout % 64 == 0 else None
         if need_dx:
             iq.iq_conv_dgrad(self.desc, e, s_e, self.wq, self.ex, self.s_ex, e_f16=e16, ws=ws,
                              stream=stream)
@@ -206,21 +210,40 @@ class DeepLabV3R50:
             self.e_stem = torch.empty(self.stem.out_shape, dtype=torch.int8, device=dev)
             self.s_e_stem = self.scal()
         # fp16 copies of the codes the tensor-core kernels read: one per distinct conv input,
-        # written by the forward of the first layer (in forward order) that reads it and read
-        # as it is by the others (IQ_CONV_X_F16_READY: the ASPP branches, a block's first conv
-        # and its projection shortcut) and by the weight gradients; and one error buffer
-        # (written by a layer's data gradient, reused by its weight gradient)
+        # written by the layer whose output codes it is (a layer's requantization writes its
+        # successor's copy: conv1 -> conv2 -> conv3 of a block, project -> head -> cls), by
+        # the stem's max pool, by the join that produces it (block outputs, the ASPP
+        # concatenation), or else by the forward of the first layer (in forward order) that
+        # reads it; read as it is by the others (IQ_CONV_X_F16_READY: the ASPP
+        # branches, a block's first conv and its projection shortcut) and by the weight
+        # gradients.  One error buffer: written with the errors by a BN layer's backward,
+        # read by its data and weight gradients (IQ_CONV_E_F16_READY)
         x16, e16 = {}, 0
+        producer = {L.a.data_ptr(): L for L in self.layers.values()}
+        joins = {blk["out"].data_ptr() for blk in self.blocks} | {self.cat.data_ptr()}
+        self.pool16, self.join16 = None, {}
         for L in self.layers.values():
             if L.spec.cin % 64 == 0 and L.x.numel() % 16 == 0:
                 key = L.x.data_ptr()
                 if key not in x16:
                     x16[key] = torch.empty(L.x.numel(), dtype=torch.float16, device=dev)
+                    P = producer.get(key)
+                    if P is not None:
+                        P.a16 = x16[key]
+                        L.desc.flags |= iq.IQ_CONV_X_F16_READY
+                    elif key == self.pool.data_ptr():
+                        self.pool16 = x16[key]
+                        L.desc.flags |= iq.IQ_CONV_X_F16_READY
+                    elif key in joins:
+                        self.join16[key] = x16[key]
+                        L.desc.flags |= iq.IQ_CONV_X_F16_READY
                 else:
-                    L.desc.flags = iq.IQ_CONV_X_F16_READY
+                    L.desc.flags |= iq.IQ_CONV_X_F16_READY
                 L.x16 = x16[key]
             if L.spec.cout % 64 == 0:
                 e16 = max(e16, L.a.numel())
+                if L.spec.bn:
+                    L.desc.flags |= iq.IQ_CONV_E_F16_READY
         if train:
             self.e16 = torch.empty(max(e16, 16), dtype=torch.float16, device=dev)
         self.ws = torch.empty(self._ws_bytes(), dtype=torch.uint8, device=dev)
@@ -298,7 +321,8 @@ class DeepLabV3R50:
         n = self.n
         iq.iq_quantize_image_u8(img_u8, False, 4, self.img, self.s_img, ws=ws, stream=stream)
         self.stem.forward(ws, stream)
-        iq.iq_maxpool_fwd(self.stem.a, 3, 2, 1, self.pool, self.pool_arg, stream=stream)
+        iq.iq_maxpool_fwd(self.stem.a, 3, 2, 1, self.pool, self.pool_arg, y_f16=self.pool16,
+                          stream=stream)
         for blk in self.blocks:
             for key in ("l1", "l2", "l3", "down"):
                 if blk[key] is not None:
@@ -306,13 +330,14 @@ class DeepLabV3R50:
             out = blk["out"]
             _, hh, ww, c = out.shape
             iq.iq_combine(self._res_terms(blk), n, hh * ww, c, out, blk["s_out"], relu=True,
-                          ws=ws, stream=stream)
+                          out_f16=self.join16.get(out.data_ptr()), ws=ws, stream=stream)
         for L in self.aspp:
             L.forward(ws, stream)
         iq.iq_spatial_sum(self.c4, self.s_c4, self.pooled.view(n, -1), self.s_pooled, mean=True,
                           ws=ws, stream=stream)
         self.pconv.forward(ws, stream)
         iq.iq_combine(self._cat_terms(), n, self.hw4, self.cat.shape[-1], self.cat, self.s_cat,
+                      out_f16=self.join16.get(self.cat.data_ptr()),
                       concat=True, ws=ws, stream=stream)
         for L in (self.project, self.head, self.cls):
             L.forward(ws, stream)

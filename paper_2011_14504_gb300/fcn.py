@@ -56,7 +56,8 @@ class Conv:
     e: torch.Tensor = None        # error after the ReLU mask
     ex: torch.Tensor = None       # error of the input (dgrad output)
     s_ex: torch.Tensor = None
-    x16: torch.Tensor = None      # fp16 copy of x written by the forward, read by the wgrad
+    x16: torch.Tensor = None      # fp16 copy of x, read by the forward and the wgrad
+    a16: torch.Tensor = None      # the next conv's x16 when that conv reads a: written here
     macs: int = 0                 # in-bounds multiply-accumulates of one pass
     macs_dense: int = 0           # every tap, the zero padding included
 
@@ -66,6 +67,7 @@ class Pool:
     x: torch.Tensor
     y: torch.Tensor
     arg: torch.Tensor
+    y16: torch.Tensor = None      # the next conv's x16 when it reads y: written by the pool
     ey: torch.Tensor = None       # error of the pooled output
     s_ey: torch.Tensor = None
     ex: torch.Tensor = None       # error of the pool input
@@ -138,6 +140,7 @@ class FcnVgg16:
         self.skip_convs = []
         if skips:
             self._build_fcn8s(lid, seed, width)
+            self._alloc_carriers()
             self._alloc_backward()
             self.ws = torch.empty(self._ws_bytes(), dtype=torch.uint8, device=dev)
             return
@@ -159,6 +162,7 @@ class FcnVgg16:
         self.up_macs, self.up_macs_dense = transposed_macs(n, self.score_hw[0],
                                                            self.score_hw[1], classes, UP_R,
                                                            UP_STRIDE, UP_PAD)
+        self._alloc_carriers()
         self._alloc_backward()
         self.ws = torch.empty(self._ws_bytes(), dtype=torch.uint8, device=dev)
 
@@ -271,16 +275,34 @@ class FcnVgg16:
             if isinstance(P, Pool):
                 P.ex = torch.empty_like(P.x)
                 P.s_ex = torch.zeros(1, dtype=torch.float64, device=dev)
-        # fp16 copies of the codes that the tensor-core kernels read: each conv input (written by
-        # the forward, reused by the weight gradient) and one error buffer (written by the data
-        # gradient, reused by the weight gradient of the same layer)
+        # one fp16 error buffer: written with the errors by the ReLU backward of a layer,
+        # read by its data and weight gradients (IQ_CONV_E_F16_READY)
         e16 = 0
         for L in self.convs:
-            if L.cin % 64 == 0 and L.x.numel() % 16 == 0:
-                L.x16 = torch.empty(L.x.numel(), dtype=torch.float16, device=dev)
-            if L.layer_id > 0 and L.cout % 64 == 0:
+            if L.cout % 64 == 0:
                 e16 = max(e16, L.a.numel())
+                if L.relu:
+                    L.desc.flags |= iq.IQ_CONV_E_F16_READY
         self.e16 = torch.empty(max(e16, 16), dtype=torch.float16, device=dev)
+
+    def _alloc_carriers(self):
+        """fp16 copies of the codes that the tensor-core kernels read: one per conv input,
+        written by the item that produces the input (the previous conv's requantization or
+        the pool) and read as it is by the conv's forward (IQ_CONV_X_F16_READY) and weight
+        gradient."""
+        prev = None
+        for item in self.layers:
+            if isinstance(item, Conv):
+                L = item
+                if L.cin % 64 == 0 and L.x.numel() % 16 == 0:
+                    L.x16 = torch.empty(L.x.numel(), dtype=torch.float16, device=self.dev)
+                    if isinstance(prev, Conv) and prev.a is L.x:
+                        prev.a16 = L.x16
+                        L.desc.flags |= iq.IQ_CONV_X_F16_READY
+                    elif isinstance(prev, Pool) and prev.y is L.x:
+                        prev.y16 = L.x16
+                        L.desc.flags |= iq.IQ_CONV_X_F16_READY
+            prev = item
 
     def _ws_bytes(self) -> int:
         b = iq.iq_quantize_workspace_size(self.img_codes.numel())
@@ -336,11 +358,12 @@ class FcnVgg16:
         iq.iq_quantize_image_u8(img_u8, False, 4, self.img_codes, self.s_img, ws=ws, stream=stream)
         for item in self.layers:
             if isinstance(item, Pool):
-                iq.iq_maxpool_fwd(item.x, 2, 2, 0, item.y, item.arg, stream=stream)
+                iq.iq_maxpool_fwd(item.x, 2, 2, 0, item.y, item.arg, y_f16=item.y16,
+                                  stream=stream)
                 continue
             L = item
             iq.iq_conv_fwd(L.desc, L.x, L.s_x, L.wq, L.a, L.s_a, relu=L.relu, x_f16=L.x16,
-                           ws=ws, stream=stream)
+                           a_f16=L.a16, ws=ws, stream=stream)
         if self.skips:
             self._forward_fcn8s(stream)
             return
@@ -399,12 +422,13 @@ class FcnVgg16:
                 err, s_err = item.ex, item.s_ex
                 continue
             L = item
+            e16 = self.e16 if L.cout % 64 == 0 else None
             if L.relu:
-                iq.iq_relu_bwd(err, L.a, L.e, stream=stream)
+                # the errors and, for the data and weight gradients, their fp16 copy
+                iq.iq_relu_bwd(err, L.a, L.e, e_f16=e16, stream=stream)
                 e = L.e
             else:
                 e = err
-            e16 = self.e16 if L.layer_id > 0 and L.cout % 64 == 0 else None
             if L.layer_id > 0:
                 iq.iq_conv_dgrad(L.desc, e, s_err, L.wq, L.ex, L.s_ex, e_f16=e16, ws=ws,
                                  stream=stream)

@@ -62,7 +62,7 @@ class ConvDesc(C.Structure):
 
 
 IQ_LAYOUT_NHWC, IQ_LAYOUT_NCHW = 0, 1
-IQ_CONV_X_F16_READY = 1
+IQ_CONV_X_F16_READY, IQ_CONV_E_F16_READY = 1, 2
 
 
 class BnBits(C.Structure):
@@ -127,7 +127,7 @@ def load(path: str | None = None):
                                 _SZ, _P]
     L.iq_weight_requant.argtypes = [_P, _P, _I64, _I, _I, _P]
     L.iq_conv_fwd.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, C.POINTER(BnBits), _I, _I,
-                              _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
+                              _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
     L.iq_conv_fwd_frozen.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, C.POINTER(BnBits), _I, _I,
                                      _P, _P, _P, _P, _SZ, _P]
     L.iq_conv_dgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
@@ -136,10 +136,10 @@ def load(path: str | None = None):
     L.iq_bn_int_fwd.argtypes = [_P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _P, _P, _P, _P, _P,
                                 _P, _P, _SZ, _P]
     L.iq_bn_int_bwd.argtypes = [_P, _P, _P, _P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _I, _P,
-                                _P, _P, _P, _P, _SZ, _P]
-    L.iq_relu_bwd.argtypes = [_P, _P, _I64, _P, _P]
+                                _P, _P, _P, _P, _P, _SZ, _P]
+    L.iq_relu_bwd.argtypes = [_P, _P, _I64, _P, _P, _P]
     L.iq_update.argtypes = [_P, _P, _P, _P, _I64, _I, _I, _I, _I, _P]
-    L.iq_maxpool_fwd.argtypes = [_P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P]
+    L.iq_maxpool_fwd.argtypes = [_P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P, _P]
     L.iq_maxpool_bwd.argtypes = [_P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P,
                                  _SZ, _P]
     L.iq_upsample_workspace_size.argtypes = [_I32, _I32, _I32, _I32, _I32, C.POINTER(_SZ)]
@@ -153,8 +153,8 @@ def load(path: str | None = None):
     L.iq_bn_int_fwd_noalloc.argtypes = [_P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _P, _P,
                                         _P, _P, _P, _P, _P]
     L.iq_combine_workspace_size.argtypes = [C.POINTER(Term), _I32, C.POINTER(_SZ)]
-    L.iq_combine.argtypes = [C.POINTER(Term), _I32, _I32, _I64, _I64, _I32, _I32, _P, _P, _P, _SZ,
-                             _P]
+    L.iq_combine.argtypes = [C.POINTER(Term), _I32, _I32, _I64, _I64, _I32, _I32, _P, _P, _P, _P,
+                             _SZ, _P]
     L.iq_spatial_sum_workspace_size.argtypes = [_I64, _I32, C.POINTER(_SZ)]
     L.iq_spatial_sum.argtypes = [_P, _P, _I64, _I64, _I32, _I32, _I32, _I32, _P, _P, _P, _SZ, _P]
     L.iq_avgpool_bwd.argtypes = [_P, _P, _I64, _I64, _I32, _P, _P, _P]
@@ -379,15 +379,15 @@ def iq_weight_requant(master, wq, k_u=24, k_w=8, stream=None):
 
 def iq_conv_fwd(d: ConvDesc, x, s_x, w, a, s_a, gamma=None, beta=None, bits=None, use_bn=False,
                 relu=True, xhat=None, bn_codes=None, bn_scales=None, frozen_out=None, acc_out=None,
-                x_f16=None, ws=None, stream=None):
+                x_f16=None, a_f16=None, ws=None, stream=None):
     if ws is None:
         ws = _ws(iq_conv_fwd_workspace_size(d, use_bn), x.device)
     _check("iq_conv_fwd",
            load().iq_conv_fwd(C.byref(d), _p(x), _p(s_x), _p(w), _p(gamma), _p(beta),
                               C.byref(bits) if bits is not None else None, int(use_bn),
                               int(relu), _p(a), _p(s_a), _p(xhat), _p(bn_codes), _p(bn_scales),
-                              _p(frozen_out), _p(acc_out), _p(x_f16), _p(ws), ws.numel(),
-                              _stream(stream)))
+                              _p(frozen_out), _p(acc_out), _p(x_f16), _p(a_f16), _p(ws),
+                              ws.numel(), _stream(stream)))
 
 
 def iq_conv_fwd_frozen(d: ConvDesc, x, w, frozen, a, use_bn=False, relu=True, bits=None,
@@ -434,7 +434,7 @@ def iq_bn_int_fwd(acc, s_acc, gamma, beta, a, s_a, xhat=None, bn_codes=None, bn_
 
 
 def iq_bn_int_bwd(e_a, s_e, a, xhat, gamma, bn_codes, bn_scales, e, s_e_out, dgamma=None,
-                  dbeta=None, k_e2=16, bits=None, ws=None, stream=None):
+                  dbeta=None, k_e2=16, bits=None, e_f16=None, ws=None, stream=None):
     c = e_a.shape[-1]
     m = e_a.numel() // c
     if ws is None:
@@ -442,12 +442,13 @@ def iq_bn_int_bwd(e_a, s_e, a, xhat, gamma, bn_codes, bn_scales, e, s_e_out, dga
     _check("iq_bn_int_bwd",
            load().iq_bn_int_bwd(_p(e_a), _p(s_e), _p(a), _p(xhat), m, c, _p(gamma), _p(bn_codes),
                                 _p(bn_scales), C.byref(bits) if bits is not None else None, k_e2,
-                                _p(e), _p(s_e_out), _p(dgamma), _p(dbeta), _p(ws), ws.numel(),
-                                _stream(stream)))
+                                _p(e), _p(s_e_out), _p(dgamma), _p(dbeta), _p(e_f16), _p(ws),
+                                ws.numel(), _stream(stream)))
 
 
-def iq_relu_bwd(e_a, a, e, stream=None):
-    _check("iq_relu_bwd", load().iq_relu_bwd(_p(e_a), _p(a), e_a.numel(), _p(e), _stream(stream)))
+def iq_relu_bwd(e_a, a, e, e_f16=None, stream=None):
+    _check("iq_relu_bwd", load().iq_relu_bwd(_p(e_a), _p(a), e_a.numel(), _p(e), _p(e_f16),
+                                             _stream(stream)))
 
 
 def iq_update(master, wq, g, s_g, lr_log2, k_u=24, k_w=8, x2=False, stream=None):
@@ -457,10 +458,10 @@ def iq_update(master, wq, g, s_g, lr_log2, k_u=24, k_w=8, x2=False, stream=None)
 
 # ---------------------------------------------------------------- network glue
 
-def iq_maxpool_fwd(x, k, s, p, y, arg, stream=None):
+def iq_maxpool_fwd(x, k, s, p, y, arg, y_f16=None, stream=None):
     n, h, w, c = x.shape
     _check("iq_maxpool_fwd", load().iq_maxpool_fwd(_p(x), n, h, w, c, k, s, p, _p(y), _p(arg),
-                                                   _stream(stream)))
+                                                   _p(y_f16), _stream(stream)))
 
 
 def iq_maxpool_bwd(e, s_e, arg, in_shape, k, s, p, ex, s_ex, ws=None, stream=None):
@@ -543,12 +544,13 @@ def iq_combine_workspace_size(terms) -> int:
     return b.value
 
 
-def iq_combine(terms, n, hw, c_out, out, s_out, concat=False, relu=False, ws=None, stream=None):
+def iq_combine(terms, n, hw, c_out, out, s_out, concat=False, relu=False, out_f16=None, ws=None,
+               stream=None):
     arr = (Term * len(terms))(*terms)
     if ws is None:
         ws = _ws(iq_combine_workspace_size(terms), out.device)
     _check("iq_combine", load().iq_combine(arr, len(terms), int(concat), n, hw, c_out, int(relu),
-                                           _p(out), _p(s_out), _p(ws), ws.numel(),
+                                           _p(out), _p(s_out), _p(out_f16), _p(ws), ws.numel(),
                                            _stream(stream)))
 
 

@@ -62,11 +62,13 @@ def test_conv_out_size_and_workspace_queries(lib):
 
 def test_conv_desc_layout_and_widths_validated(lib):
     """The descriptor's layout and code widths: NHWC / NCHW, k_w and k_a in 2..8 (0: 8 bits),
-    flags 0 or IQ_CONV_X_F16_READY; anything else is rejected by the host-side checks."""
+    flags from IQ_CONV_X_F16_READY | IQ_CONV_E_F16_READY; anything else is rejected by the
+    host-side checks."""
     ok = [dict(), dict(layout=iq.IQ_LAYOUT_NCHW), dict(k_w=4, k_a=4), dict(k_w=2, k_a=8),
-          dict(flags=iq.IQ_CONV_X_F16_READY)]
+          dict(flags=iq.IQ_CONV_X_F16_READY), dict(flags=iq.IQ_CONV_E_F16_READY),
+          dict(flags=iq.IQ_CONV_X_F16_READY | iq.IQ_CONV_E_F16_READY)]
     bad = [dict(layout=2), dict(layout=-1), dict(k_w=1), dict(k_w=9), dict(k_a=1), dict(k_a=16),
-           dict(flags=2), dict(flags=-1)]
+           dict(flags=4), dict(flags=-1)]
     for kw in ok:
         assert iq.iq_conv_out_size(iq.conv_desc(1, 8, 8, 8, 8, 3, 3, 1, 1, **kw)) == (8, 8)
     for kw in bad:
@@ -95,21 +97,29 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert e.value.code == iq.IQ_ERR_INVALID_ARG
     d = iq.conv_desc(1, 8, 8, 8, 8, 3, 3, 1, 1)
     rc = lib.iq_conv_fwd(C.byref(d), None, None, None, None, None, None, 0, 1, None, None, None,
-                         None, None, None, None, None, None, 0, None)
+                         None, None, None, None, None, None, None, 0, None)
     assert rc == iq.IQ_ERR_INVALID_ARG
     # a shape beyond the int32 accumulation bound: 1024*12*12*127^2 >= 2^31
     big = iq.conv_desc(1, 12, 12, 1024, 8, 12, 12)
     rc = lib.iq_conv_fwd(C.byref(big), 1, 1, 1, None, None, None, 0, 1, 1, 1, None, None, None,
-                         None, None, None, None, 0, None)
+                         None, None, None, None, None, 0, None)
     assert rc == iq.IQ_ERR_OVERFLOW_RISK
     # workspace too small
     rc = lib.iq_conv_fwd(C.byref(d), 1, 1, 1, None, None, None, 0, 1, 1, 1, None, None, None,
-                         None, None, None, None, 16, None)
+                         None, None, None, None, None, 16, None)
     assert rc == iq.IQ_ERR_WORKSPACE
     # an fp16 carrier that is not 16-byte aligned
     rc = lib.iq_conv_fwd(C.byref(d), 16, 1, 1, None, None, None, 0, 1, 1, 1, None, None, None,
-                         None, None, 24, None, 1 << 30, None)
+                         None, None, 24, None, None, 1 << 30, None)
     assert rc == iq.IQ_ERR_INVALID_ARG
+    # an fp16 output copy that is not 16-byte aligned
+    rc = lib.iq_conv_fwd(C.byref(d), 16, 1, 16, None, None, None, 0, 1, 16, 1, None, None, None,
+                         None, None, None, 24, None, 1 << 30, None)
+    assert rc == iq.IQ_ERR_INVALID_ARG
+    # the same for the other producers of fp16 copies, rejected before any launch
+    assert lib.iq_relu_bwd(16, 16, 32, 16, 24, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_relu_bwd(16, 16, 40, 16, 32, None) == iq.IQ_ERR_INVALID_ARG   # n % 16
+    assert lib.iq_maxpool_fwd(16, 1, 8, 8, 16, 2, 2, 0, 16, 16, 24, None) == iq.IQ_ERR_INVALID_ARG
     # bad bit width / dtype combination
     rc = lib.iq_quantize(1, 10, 16, iq.IQ_MODE_UQ, iq.IQ_I8, 1, 1, 1, 4096, None)
     assert rc == iq.IQ_ERR_INVALID_ARG
@@ -127,21 +137,23 @@ def test_glue_arguments_rejected_before_launch(lib):
     T = iq.Term
     ok = T(16, iq.IQ_I8, 8, 0, 0, 16, None, None, 8, 8)
     arr = (T * 9)(*([ok] * 9))
-    assert lib.iq_combine(arr, 0, 0, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
-    assert lib.iq_combine(arr, 9, 0, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_combine(arr, 0, 0, 1, 4, 8, 0, 16, 16, None, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_combine(arr, 9, 0, 1, 4, 8, 0, 16, 16, None, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
     # a sum whose operand does not cover every output channel
-    assert lib.iq_combine(arr, 2, 0, 1, 4, 16, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_combine(arr, 2, 0, 1, 4, 16, 0, 16, 16, None, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
     # a concatenation operand past the last channel
     off = (T * 1)(T(16, iq.IQ_I8, 8, 4, 0, 16, None, None, 8, 8))
-    assert lib.iq_combine(off, 1, 1, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_combine(off, 1, 1, 1, 4, 8, 0, 16, 16, None, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
     # gamma without beta, bad dtype
     half = (T * 1)(T(16, iq.IQ_I8, 8, 0, 0, 16, 16, None, 8, 8))
-    assert lib.iq_combine(half, 1, 0, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_combine(half, 1, 0, 1, 4, 8, 0, 16, 16, None, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
     wide = (T * 1)(T(16, iq.IQ_I32, 8, 0, 0, 16, None, None, 8, 8))
-    assert lib.iq_combine(wide, 1, 0, 1, 4, 8, 0, 16, 16, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
+    assert lib.iq_combine(wide, 1, 0, 1, 4, 8, 0, 16, 16, None, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
     need = C.c_size_t()
     assert lib.iq_combine_workspace_size(arr, 2, C.byref(need)) == 0 and need.value >= 256 + 2 * 128
-    assert lib.iq_combine(arr, 2, 0, 1, 4, 8, 0, 16, 16, 16, 64, None) == iq.IQ_ERR_WORKSPACE
+    assert lib.iq_combine(arr, 2, 0, 1, 4, 8, 0, 16, 16, None, 16, 64, None) == iq.IQ_ERR_WORKSPACE
+    # an fp16 output copy off a 16-byte boundary
+    assert lib.iq_combine(arr, 2, 0, 1, 4, 8, 0, 16, 16, 24, 16, 1 << 20, None) == iq.IQ_ERR_INVALID_ARG
     assert lib.iq_spatial_sum(16, 16, 2, 9, 8, 4, 8, 1, 16, 16, 16, 4096, None) == iq.IQ_ERR_INVALID_ARG
     assert lib.iq_spatial_sum(16, 16, 2, 9, 8, 0, 8, 1, 16, 16, 16, 8, None) == iq.IQ_ERR_WORKSPACE
     assert lib.iq_avgpool_bwd(None, 16, 2, 9, 8, None, 16, None) == iq.IQ_ERR_INVALID_ARG

@@ -55,10 +55,15 @@ def run_combine(specs, n, hw, c_out, concat, relu, misalign=False):
         oterms.append(O.CombineTerm(codes, s, off, bc, gam, bet))
     out = torch.empty(n * hw * c_out, dtype=torch.int8, device=DEV)
     so = scal()
-    iq.iq_combine(terms, n, hw, c_out, out, so, concat=concat, relu=relu)
+    # the fp16 copy of the output codes wherever its size allows one
+    out16 = (torch.empty(out.numel(), dtype=torch.float16, device=DEV)
+             if out.numel() % 16 == 0 else None)
+    iq.iq_combine(terms, n, hw, c_out, out, so, concat=concat, relu=relu, out_f16=out16)
     ref, sref = O.combine(oterms, n, hw, c_out, concat=concat, relu=relu)
     assert np.array_equal(host(out), ref)
     assert host(so)[0] == sref
+    if out16 is not None:
+        assert np.array_equal(host(out16).astype(np.float32), ref.astype(np.float32))
 
 
 def test_combine_residual_bn_affine_plus_shortcut():

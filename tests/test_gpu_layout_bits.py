@@ -208,3 +208,97 @@ def test_shared_input_carrier_ready_flag():
         iq.iq_conv_wgrad(d, dev(e), sc(1e-6), xd, sc(s_x), gq, sc(), gq_mode=1, seed=1, layer=i,
                          step=0, g_acc_out=gacc, x_f16=x16)
         assert np.array_equal(host(gacc), O.conv_wgrad(cv, e, x)), i
+
+
+def _f16_codes(t16):
+    """The int8 codes an fp16 copy holds (every int8 code is exact in fp16)."""
+    torch.cuda.synchronize()
+    v = t16.float().cpu().numpy()
+    assert np.array_equal(v, np.round(v)) and np.abs(v).max() <= 127
+    return v.astype(np.int8)
+
+
+@pytest.mark.parametrize("bn,k_a", [(True, 0), (False, 0), (False, 4)])
+def test_output_carrier_of_the_forward(bn, k_a):
+    """a_f16: the requantization pass (the L1BN one, or the SQ one at 8 and at 4 bits) writes
+    the fp16 copy of the output codes; a second layer reads it under IQ_CONV_X_F16_READY and
+    matches the oracle."""
+    n, h, w, c, k = 2, 19, 23, 64, 128
+    g = S.rng(930 + 2 * bn + k_a)
+    x = S.int8_uniform(g, (n, h, w, c))
+    cv = O.Conv(n, h, w, c, k, 3, 3, 1, 1, 1)
+    d = iq.conv_desc(n, h, w, c, k, 3, 3, 1, 1, k_a=k_a)
+    wq = O.requant_master(O.uq(S.he_weights(g, (k, 3, 3, c), c * 9), 24)).astype(np.int8)
+    a = torch.empty((n, h, w, k), dtype=torch.int8, device=DEV)
+    a16 = torch.empty(a.numel(), dtype=torch.float16, device=DEV)
+    s_a = sc()
+    acc = O.conv_fwd(cv, x, wq)
+    if bn:
+        gam, bet = S.bn_gamma_beta_codes(g, k)
+        iq.iq_conv_fwd(d, dev(x), sc(0.02), dev(wq), a, s_a, dev(gam), dev(bet), use_bn=True,
+                       relu=True, a_f16=a16)
+        want = O.bn_fwd(acc.reshape(-1, k), 0.02 * 2.0 ** -7, gam, bet).A.reshape(n, h, w, k)
+    else:
+        iq.iq_conv_fwd(d, dev(x), sc(0.02), dev(wq), a, s_a, relu=True, a_f16=a16)
+        want, _ = O.sq_int(acc, 0.02 * 2.0 ** -7, 4 if k_a else 8, True)
+    assert np.array_equal(host(a).astype(np.int32), want.astype(np.int32))
+    assert np.array_equal(_f16_codes(a16).reshape(n, h, w, k), host(a))
+    # the next layer reads the copy as it is
+    k2 = 64
+    cv2 = O.Conv(n, h, w, k, k2, 1, 1, 1, 0, 1)
+    d2 = iq.conv_desc(n, h, w, k, k2, 1, 1, 1, 0, flags=iq.IQ_CONV_X_F16_READY)
+    w2 = O.requant_master(O.uq(S.he_weights(g, (k2, 1, 1, k), k), 24)).astype(np.int8)
+    acc2 = torch.empty((n, h, w, k2), dtype=torch.int32, device=DEV)
+    iq.iq_conv_fwd(d2, a, s_a, dev(w2), torch.empty((n, h, w, k2), dtype=torch.int8, device=DEV),
+                   sc(), relu=True, acc_out=acc2, x_f16=a16)
+    assert np.array_equal(host(acc2), O.conv_fwd(cv2, host(a), w2))
+
+
+def test_carriers_of_pool_relu_and_bn_backward():
+    """y_f16 of the max pool, e_f16 of the ReLU backward and of the L1BN backward (the
+    streamed tiles at 256 channels, the histogram path at 48) hold the fp16 copies of the
+    codes they write; a data gradient reads the error copy under IQ_CONV_E_F16_READY."""
+    g = S.rng(951)
+    n, h, w, c = 2, 20, 22, 64
+    x = S.int8_uniform(g, (n, h, w, c))
+    y = torch.empty((n, h // 2, w // 2, c), dtype=torch.int8, device=DEV)
+    arg = torch.empty_like(y, dtype=torch.uint8)
+    y16 = torch.empty(y.numel(), dtype=torch.float16, device=DEV)
+    iq.iq_maxpool_fwd(dev(x), 2, 2, 0, y, arg, y_f16=y16)
+    yo, _ = O.maxpool_fwd(x, 2, 2, 0)
+    assert np.array_equal(host(y), yo)
+    assert np.array_equal(_f16_codes(y16).reshape(y.shape), yo)
+    ea = S.int8_uniform(g, (n, h, w, c))
+    e = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
+    e16 = torch.empty(e.numel(), dtype=torch.float16, device=DEV)
+    iq.iq_relu_bwd(dev(ea), dev(x), e, e_f16=e16)
+    assert np.array_equal(host(e), O.relu_bwd(ea, x))
+    assert np.array_equal(_f16_codes(e16).reshape(e.shape), host(e))
+    for C in (256, 48):
+        m = 777
+        acc = (g.standard_normal((m, C)) * 3000).astype(np.int32)
+        gam, bet = S.bn_gamma_beta_codes(g, C)
+        r = O.bn_fwd(acc, 2.0 ** -14, gam, bet)
+        eA = S.int8_uniform(g, (m, C))
+        want = O.bn_bwd(eA, 3e-6, r.A, r.X, r.s_xhat, gam, r.c_sigma)[0]
+        codes = dev(np.concatenate([r.c_mu, r.c_sigma]))
+        scal = torch.zeros(iq.IQ_BN_SCALES, dtype=torch.float64, device=DEV)
+        scal[iq.IQ_BN_S_XHAT] = r.s_xhat
+        eo = torch.empty((m, C), dtype=torch.int8, device=DEV)
+        eo16 = torch.empty(eo.numel(), dtype=torch.float16, device=DEV)
+        iq.iq_bn_int_bwd(dev(eA), sc(3e-6), dev(r.A), dev(r.X), dev(gam), codes, scal, eo, sc(),
+                         e_f16=eo16)
+        assert np.array_equal(host(eo), want), C
+        assert np.array_equal(_f16_codes(eo16).reshape(m, C), want), C
+    # a data gradient over an error copy written beforehand
+    k = 64
+    cv = O.Conv(n, h, w, c, k, 3, 3, 1, 1, 1)
+    wq = O.requant_master(O.uq(S.he_weights(g, (k, 3, 3, c), c * 9), 24)).astype(np.int8)
+    ee = S.int8_uniform(g, (n, h, w, k))
+    ee16 = torch.empty(ee.size, dtype=torch.float16, device=DEV)
+    iq.iq_relu_bwd(dev(ee), dev(np.full_like(ee, 1)), torch.empty_like(dev(ee)), e_f16=ee16)
+    d = iq.conv_desc(n, h, w, c, k, 3, 3, 1, 1, flags=iq.IQ_CONV_E_F16_READY)
+    dacc = torch.empty((n, h, w, c), dtype=torch.int32, device=DEV)
+    dx = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
+    iq.iq_conv_dgrad(d, dev(ee), sc(1e-5), dev(wq), dx, sc(), acc_out=dacc, e_f16=ee16)
+    assert np.array_equal(host(dacc), O.conv_dgrad(cv, ee, wq))
