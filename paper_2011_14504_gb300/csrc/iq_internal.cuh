@@ -38,6 +38,7 @@ struct RqParams {
     UDiv div;      // by 2M (SQ) or by M (RQ)
     double s_out;
     uint32_t R8;   // SQ with k = 8 and 128 < M <= 2^31: floor(2^39 / M), else 0
+    float kq;      // with R8: fl(128 / M)
 };
 
 __device__ inline RqParams rq_params_make(uint64_t M, double s, int k, int mode) {
@@ -47,6 +48,7 @@ __device__ inline RqParams rq_params_make(uint64_t M, double s, int k, int mode)
     p.div = make_udiv(M == 0 ? 1 : (rq ? M : 2 * M));
     p.R8 = (!rq && k == 8 && M > 128 && M <= (uint64_t(1) << 31))
                ? (uint32_t)((uint64_t(1) << 39) / M) : 0u;
+    p.kq = p.R8 ? __double2float_rn(__ddiv_rn(128.0, (double)M)) : 0.0f;
     if (mode == IQ_MODE_RQ_GQ2) p.s_out = ldexp(1.0, 1 - k);
     else p.s_out = M ? ldexp(__dmul_rn(s, (double)M), 1 - k) : ldexp(s, 1 - k);
     return p;

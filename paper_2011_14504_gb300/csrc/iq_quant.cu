@@ -169,10 +169,47 @@ __device__ __forceinline__ uint32_t sq8_byte(int v, uint32_t M, uint32_t R8, int
     return q ^ 0x80u;
 }
 
+// 4 codes of sq8_byte, each decided in fp32 where that provably gives q = floor(128 u / M + 1/2)
+// (u = v + M in [0, 2M]; the integer pipe, which sq8_byte's 64-bit comparisons saturate, is
+// left mostly idle): u = 2^16 uh + ul with both halves exact in fp32 (the low mantissa bits
+// of 2^23, by a mask or a byte permute), y = fl(uh 2^16 kq + fl(ul kq + 1/2)) with
+// kq = fl(128 / M).  Against Y* = 128 u / M + 1/2 (u K <= 256, K = 128 / M): the kq rounding
+// adds at most 256 2^-24 and each of the two fma roundings at most 257 2^-24, so
+// |y - Y*| < 2^-14.  y clamped to [3/2, 255 + 1/2] (the clamp of q to [1, 255] commutes with
+// the floor there), q = floor(y) and f = y - q exactly through y + 1.5 2^23 rounded
+// downward (its low byte is q); q is taken when 2^-13 <= f < 1 - 2^-13, so Y* has the same
+// floor.  Otherwise (about one element in four thousand) sq8_byte decides, under one branch
+// per word.  The code byte is q ^ 0x80.
 template <bool CLIP>
-__device__ __forceinline__ uint32_t sq8_word(const int4& v, uint32_t M, uint32_t R8, int relu) {
-    return sq8_byte<CLIP>(v.x, M, R8, relu) | (sq8_byte<CLIP>(v.y, M, R8, relu) << 8) |
-           (sq8_byte<CLIP>(v.z, M, R8, relu) << 16) | (sq8_byte<CLIP>(v.w, M, R8, relu) << 24);
+__device__ __forceinline__ uint32_t sq8_word_f(const int4& v, uint32_t M, uint32_t R8, float kq,
+                                               int relu) {
+    constexpr float MAG = 12582912.0f;                  // 1.5 2^23
+    const int vs[4] = {v.x, v.y, v.z, v.w};
+    uint32_t tb[4];
+    bool ok[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        int vv = vs[j];
+        if (relu && vv < 0) vv = 0;
+        if (CLIP && M < 0x80000000u) vv = min(max(vv, -(int)M), (int)M);
+        const uint32_t u = (uint32_t)vv + M;
+        const float fl = __int_as_float((int)(0x4B000000u | (u & 0xffffu))) - 8388608.0f;
+        const float fh = __int_as_float((int)__byte_perm(u, 0x4B000000u, 0x7432)) - 8388608.0f;
+        const float y = fminf(fmaxf(fmaf(fh * 65536.0f, kq, fmaf(fl, kq, 0.5f)), 1.5f), 255.5f);
+        const float t = __fadd_rd(y, MAG);
+        const float f = y - (t - MAG);
+        tb[j] = __float_as_uint(t);
+        ok[j] = f >= 0x1p-13f && f < 1.0f - 0x1p-13f;
+    }
+    uint32_t w = __byte_perm(__byte_perm(tb[0], tb[1], 0x0040), __byte_perm(tb[2], tb[3], 0x0040),
+                             0x5410) ^ 0x80808080u;
+    if (!(ok[0] && ok[1] && ok[2] && ok[3])) {
+#pragma unroll
+        for (int j = 0; j < 4; j++)
+            if (!ok[j])
+                w = (w & ~(0xffu << (8 * j))) | (sq8_byte<CLIP>(vs[j], M, R8, relu) << (8 * j));
+    }
+    return w;
 }
 
 // the fp16 copy of 4 codes (one 8-byte store) when the caller asked for it
@@ -196,6 +233,7 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
     if (p.R8) {
         // four 16-byte loads in flight per thread
         const uint32_t M = (uint32_t)p.M;
+        const float kq = p.kq;
         for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
              i += 4 * stride) {
             int4 v[4];
@@ -205,7 +243,7 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
 #pragma unroll
             for (int j = 0; j < 4; j++)
                 if (i + j * stride < n4) {
-                    const uint32_t w = sq8_word<CLIP>(v[j], M, p.R8, relu);
+                    const uint32_t w = sq8_word_f<CLIP>(v[j], M, p.R8, kq, relu);
                     out[i + j * stride] = w;
                     put_f16x4(out16, i + j * stride, w);
                 }

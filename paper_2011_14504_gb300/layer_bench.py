@@ -5,6 +5,7 @@ through the C ABI; or run one step of a network once (a profiling target).
     python -m paper_2011_14504_gb300.layer_bench bn M,C [time|once]
     python -m paper_2011_14504_gb300.layer_bench step deeplab|fcn BATCH [train|infer]
     python -m paper_2011_14504_gb300.layer_bench gemm M,N,K [time|once]
+    python -m paper_2011_14504_gb300.layer_bench join C16,C8 [time|once]
 
 Runs iq_conv_fwd (with ReLU and the SQ8 requantisation of the output), iq_conv_dgrad and
 iq_conv_wgrad (GQ8 gradient) of an N x H x H x C -> K layer on random 8-bit codes.  "time"
@@ -12,7 +13,8 @@ iq_conv_wgrad (GQ8 gradient) of an N x H x H x C -> K layer on random 8-bit code
 the int8 multiply-accumulate rate it implies (2 ops per MAC); "once" makes one call of each,
 which is the form used under a profiler.  The bn form runs iq_bn_int_fwd on M x C random
 int32 accumulators (L1BN, ReLU, Q_A) and iq_bn_int_bwd on random 8-bit errors, and prints
-each call's duration and its DRAM bytes per element over that time.
+each call's duration and its DRAM bytes per element over that time.  The join form times
+iq_combine on a residual join of two int16 operands and a sum of two int8 errors.
 """
 import sys
 
@@ -68,6 +70,54 @@ def bn_main(argv):
         if ms is not None:
             print(f"{name}: {ms:.3f} ms  {nb * m * c / ms / 1e6:.0f} GB/s at {nb} B/element")
     torch.cuda.synchronize()
+    print("ok")
+
+
+def join_main(argv):
+    """One residual join of two int16 X-code operands with the BN affine and ReLU (the
+    downsampling blocks' form) and one sum of two int8 errors, both 65 x 65 x C at batch 16
+    (the stage-3 and stage-4 shapes of the DeepLab step), through iq_combine with the fp16
+    output copy."""
+    c16, c8 = [int(v) for v in (argv[0] if argv else "1024,2048").split(",")]
+    mode = argv[1] if len(argv) > 1 else "time"
+    dev = "cuda"
+    g = torch.Generator(device=dev)
+    g.manual_seed(3)
+    n, hw = 16, 65 * 65
+
+    def sc(v):
+        return torch.tensor([v], dtype=torch.float64, device=dev)
+
+    keep = []
+    cases = []
+    X = [torch.randint(-32767, 32768, (n, hw, c16), generator=g, device=dev, dtype=torch.int16)
+         for _ in range(2)]
+    gb = [torch.randint(-127, 128, (c16,), generator=g, device=dev, dtype=torch.int32)
+          for _ in range(4)]
+    s16 = [sc(2.5e-5), sc(3.1e-5)]
+    keep += X + gb + s16
+    cases.append(("residual join, int16 + int16", c16, True, 9,
+                  [iq.term(X[0], s16[0], gamma=gb[0], beta=gb[1]),
+                   iq.term(X[1], s16[1], gamma=gb[2], beta=gb[3])]))
+    E = [torch.randint(-127, 128, (n, hw, c8), generator=g, device=dev, dtype=torch.int8)
+         for _ in range(2)]
+    s8 = [sc(1.1e-6), sc(0.9e-6)]
+    keep += E + s8
+    cases.append(("error sum, int8 + int8", c8, False, 5, [iq.term(E[0], s8[0]),
+                                                           iq.term(E[1], s8[1])]))
+    for name, c, relu, nb, terms in cases:
+        out = torch.empty((n, hw, c), dtype=torch.int8, device=dev)
+        out16 = torch.empty(out.numel(), dtype=torch.float16, device=dev)
+        so = sc(0.0)
+        ws = torch.empty(iq.iq_combine_workspace_size(terms), dtype=torch.uint8, device=dev)
+        f = lambda: iq.iq_combine(terms, n, hw, c, out, so, relu=relu, out_f16=out16, ws=ws)
+        ms = _time(f, mode)
+        if ms is not None:
+            # both passes read the operands, the codes pass writes the codes and their copy
+            print(f"{name} (c = {c}): {ms:.3f} ms  {(nb + 2) * n * hw * c / ms / 1e6:.0f} GB/s "
+                  f"at {nb + 2} B/element")
+    torch.cuda.synchronize()
+    assert iq.iq_device_status() == 0
     print("ok")
 
 
@@ -147,6 +197,8 @@ def main(argv=None):
         return step_main(argv[1:])
     if argv and argv[0] == "gemm":
         return gemm_main(argv[1:])
+    if argv and argv[0] == "join":
+        return join_main(argv[1:])
     n, h, c, k = [int(v) for v in (argv[0] if argv else "8,128,256,256").split(",")]
     mode = argv[1] if len(argv) > 1 else "time"
     dev = "cuda"

@@ -148,6 +148,33 @@ def test_requantize_sq_int32_large(relu, M):
     assert host(so)[0] == ws
 
 
+@pytest.mark.parametrize("relu", [False, True])
+@pytest.mark.parametrize("M", [2 ** 31, 2 ** 31 - 1, 2 ** 30 + 3, 3 * 2 ** 20 + 7, 1000])
+def test_requantize_sq_int32_code_boundaries(relu, M):
+    """Values one unit below, at and above every code boundary of SQ8 (the smallest u = v + M
+    with floor(128 u / M + 1/2) >= k, for every k): the 4-wide kernel's fp32 evaluation cannot
+    tell these apart at large M, so its exact fallback decides them."""
+    ks = np.arange(1, 256, dtype=np.int64)
+    u_k = ((2 * ks - 1) * M + 255) // 256          # ceil((2k - 1) M / 256)
+    u = np.concatenate([u_k - 1, u_k, u_k + 1, [0, 2 * M]])
+    u = np.clip(u, 0, 2 * M)
+    v = u - M
+    v = v[(v >= -(2 ** 31)) & (v <= 2 ** 31 - 1)]
+    g = S.rng(M % 1009 + relu)
+    v = np.concatenate([v, [-M if M <= 2 ** 31 else -(2 ** 31)]])
+    v = v[g.permutation(v.size)]
+    v = v[: v.size // 4 * 4].astype(np.int32)
+    if np.abs(v.astype(np.int64)).max() != M:           # the tensor's maximum must be M
+        v[0] = np.int32(-M if M <= 2 ** 31 else 0)
+    out = torch.empty(v.size, dtype=torch.int8, device=DEV)
+    so = dscal()
+    iq.iq_requantize(dev(v), dscal(2.0 ** -20), 8, iq.IQ_MODE_SQ_RELU if relu else iq.IQ_MODE_SQ,
+                     out, so)
+    want, ws = O.sq_int(v, 2.0 ** -20, 8, relu)
+    assert np.array_equal(host(out).astype(np.int32), want)
+    assert host(so)[0] == ws
+
+
 def test_rq_epoch_changes_only_the_draws():
     # the epoch is the fourth Philox counter word: 0 reproduces the oracle; another value gives
     # other draws of the same stochastic rounding (every code within one of the exact value)
