@@ -1238,8 +1238,19 @@ __device__ __forceinline__ void tile_issue(const CUtensorMap* me, const CUtensor
     tc::tma_load_2d(st + 2 * kTileR * kTileC, mxh, bar, x, y);
 }
 
-// Pass A over tiles: max |e_y| per channel (for max |e_y gamma|), sum sign X, and the extreme
-// code e_y of each sign class of X (-, 0, +), four channels packed in the bytes of a word.
+// PTX prmt with its sign-replicating selectors (a selector nibble with bit 3 set fills the
+// byte with the sign of the byte it selects); __byte_perm uses only the low 3 bits
+__device__ __forceinline__ uint32_t prmt_sx(uint32_t a, uint32_t b, uint32_t sel) {
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+    return d;
+}
+
+// Pass A over tiles: sum sign X per channel, and the extreme code e_y of each sign class of X
+// (-, 0, +), two channels per word in int16 lanes (packed 16-bit min / max; the codes are
+// widened by sign-replicating byte permutes, the class masks taken from the sign bytes of X
+// and min(X, 1) per lane); max |e_y| per channel (for max |e_y gamma|) follows from the
+// class extremes.
 __global__ void __launch_bounds__(kStreamThreads, 1)
     k_bnb_a_t(const __grid_constant__ CUtensorMap me, const __grid_constant__ CUtensorMap ma,
               const __grid_constant__ CUtensorMap mxh, int64_t m, int32_t C,
@@ -1250,9 +1261,15 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     const int c_base = blockIdx.x * kTileC;
     const int g = threadIdx.x & 15, rl = threadIdx.x >> 4;       // 16 groups x 32 row lanes
     long long ss[4] = {0, 0, 0, 0};
-    uint32_t amax = 0;                                            // per byte: max |e_y|
-    uint32_t mx[3] = {0x80808080u, 0x80808080u, 0x80808080u};    // empty: max 0x80 < min 0x7f
-    uint32_t mn[3] = {0x7f7f7f7fu, 0x7f7f7f7fu, 0x7f7f7f7fu};
+    // per sign class q (X < 0, X = 0, X > 0) the extremes of e_y, two channels per word as
+    // packed int16 (native 16-bit min / max): [q][0, 1] max of channels (0,1), (2,3); [q][2, 3]
+    // the minima.  Empty: max 0x8000 (below every code), min 0x7fff.
+    uint32_t ext[3][4];
+#pragma unroll
+    for (int q = 0; q < 3; q++) {
+        ext[q][0] = ext[q][1] = 0x80008000u;
+        ext[q][2] = ext[q][3] = 0x7fff7fffu;
+    }
     const int64_t nchunk = (m + kTileR - 1) / kTileR;
     const bool ok = pipe_chunks<kTileStages>(
         nchunk, kTileR, m, kTileStage, smem, err,
@@ -1261,42 +1278,58 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
             const uint32_t* e4 = reinterpret_cast<const uint32_t*>(st);
             const uint32_t* a4 = reinterpret_cast<const uint32_t*>(st + kTileR * kTileC);
             const uint2* x4 = reinterpret_cast<const uint2*>(st + 2 * kTileR * kTileC);
-            uint32_t npos = 0, nneg = 0;     // the chunk's sign counts (<= 4 a byte)
+            // the chunk's counts per channel, two int16 lanes a word: X < 0 and X != 0
+            uint32_t nneg[2] = {0u, 0u}, nnz[2] = {0u, 0u};
 #pragma unroll
             for (int u = 0; u < kTileR / 32; u++) {
                 const int r = rl + 32 * u;
                 if (r >= rows) break;
                 const int i = r * 16 + g;
-                const uint32_t ey = e4[i] & __vcmpgts4(a4[i], 0u);
+                const uint32_t a = a4[i];
+                // byte j of am: 0xff where A_j > 0 (nonzero with a clear sign bit)
+                const uint32_t nzb = ((a & 0x7f7f7f7fu) + 0x7f7f7f7fu) | a;
+                const uint32_t am = prmt_sx(nzb, 0u, 0xBA98) & ~prmt_sx(a, 0u, 0xBA98);
+                const uint32_t ey = e4[i] & am;
+                // e_y of channels (0,1) and (2,3) sign-extended to int16 lanes
+                const uint32_t ey16[2] = {prmt_sx(ey, 0u, 0x9180), prmt_sx(ey, 0u, 0xB3A2)};
                 const uint2 xv = x4[i];
-                // byte j of pos / neg: 0xff where X of channel j is > 0 / < 0
-                const uint32_t pos = __byte_perm(__vcmpgts2(xv.x, 0u), __vcmpgts2(xv.y, 0u), 0x6420);
-                const uint32_t neg = __byte_perm(__vcmplts2(xv.x, 0u), __vcmplts2(xv.y, 0u), 0x6420);
-                npos += pos & 0x01010101u;
-                nneg += neg & 0x01010101u;
-                amax = __vmaxu4(amax, __vabs4(ey));
-                const uint32_t cls[3] = {neg, ~(neg | pos), pos};
+                const uint32_t xw[2] = {xv.x, xv.y};
 #pragma unroll
-                for (int q = 0; q < 3; q++) {
-                    mx[q] = __vmaxs4(mx[q], (ey & cls[q]) | (0x80808080u & ~cls[q]));
-                    mn[q] = __vmins4(mn[q], (ey & cls[q]) | (0x7f7f7f7fu & ~cls[q]));
+                for (int h = 0; h < 2; h++) {
+                    // per int16 lane: 0xffff where X < 0 (its sign), 1 / 0xffff where X != 0
+                    const uint32_t neg = prmt_sx(xw[h], 0u, 0xBB99);
+                    uint32_t nz1;
+                    asm("min.u16x2 %0, %1, %2;" : "=r"(nz1) : "r"(xw[h]), "r"(0x00010001u));
+                    const uint32_t nz = nz1 * 0xffffu;
+                    nneg[h] += neg & 0x00010001u;
+                    nnz[h] += nz1;
+                    const uint32_t cls[3] = {neg, ~nz, nz & ~neg};
+#pragma unroll
+                    for (int q = 0; q < 3; q++) {
+                        const uint32_t vx = (ey16[h] & cls[q]) | (0x80008000u & ~cls[q]);
+                        const uint32_t vn = (ey16[h] & cls[q]) | (0x7fff7fffu & ~cls[q]);
+                        asm("max.s16x2 %0, %0, %1;" : "+r"(ext[q][h]) : "r"(vx));
+                        asm("min.s16x2 %0, %0, %1;" : "+r"(ext[q][2 + h]) : "r"(vn));
+                    }
                 }
             }
+            // sum sign X = #(X > 0) - #(X < 0) = #(X != 0) - 2 #(X < 0)
 #pragma unroll
-            for (int j = 0; j < 4; j++)
-                ss[j] += (int)((npos >> (8 * j)) & 0xffu) - (int)((nneg >> (8 * j)) & 0xffu);
+            for (int j = 0; j < 4; j++) {
+                const int sh = 16 * (j & 1);
+                ss[j] += (int)((nnz[j >> 1] >> sh) & 0xffffu) -
+                         2 * (int)((nneg[j >> 1] >> sh) & 0xffffu);
+            }
         });
     if (!ok) return;
     long long* sq = reinterpret_cast<long long*>(smem);                // [32][64]
-    uint32_t* sp = reinterpret_cast<uint32_t*>(sq + 32 * kTileC);      // [7][512]
+    uint32_t* sp = reinterpret_cast<uint32_t*>(sq + 32 * kTileC);      // [12][512]
 #pragma unroll
     for (int j = 0; j < 4; j++) sq[rl * kTileC + 4 * g + j] = ss[j];
 #pragma unroll
-    for (int q = 0; q < 3; q++) {
-        sp[(2 * q) * kStreamThreads + threadIdx.x] = mx[q];
-        sp[(2 * q + 1) * kStreamThreads + threadIdx.x] = mn[q];
-    }
-    sp[6 * kStreamThreads + threadIdx.x] = amax;
+    for (int q = 0; q < 3; q++)
+#pragma unroll
+        for (int w = 0; w < 4; w++) sp[(4 * q + w) * kStreamThreads + threadIdx.x] = ext[q][w];
     __syncthreads();
     const int col = threadIdx.x;
     uint32_t zm = 0;
@@ -1305,22 +1338,22 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
         for (int i = 0; i < 32; i++) t += sq[i * kTileC + col];
         const int c = c_base + col;
         atomicAdd(&w.ss[c], (unsigned long long)t);
-        const int gg = col >> 2, j = col & 3;
-        uint32_t am = 0;
-        for (int i = 0; i < 32; i++) am = __vmaxu4(am, sp[6 * kStreamThreads + i * 16 + gg]);
-        zm = ((am >> (8 * j)) & 0xffu) * (uint32_t)abs(gam[c]);
+        const int gg = col >> 2, j = col & 3, wd = j >> 1, sh = 16 * (j & 1);
+        int amax = 0;                              // max |e_y| over every class
 #pragma unroll
         for (int q = 0; q < 3; q++) {
-            uint32_t hx = 0x80808080u, ln = 0x7f7f7f7fu;
+            int hi = -32768, lo = 32767;
             for (int i = 0; i < 32; i++) {
-                hx = __vmaxs4(hx, sp[(2 * q) * kStreamThreads + i * 16 + gg]);
-                ln = __vmins4(ln, sp[(2 * q + 1) * kStreamThreads + i * 16 + gg]);
+                const int k = i * 16 + gg;
+                hi = max(hi, (int)(int16_t)(sp[(4 * q + wd) * kStreamThreads + k] >> sh));
+                lo = min(lo, (int)(int16_t)(sp[(4 * q + 2 + wd) * kStreamThreads + k] >> sh));
             }
-            const int hi = (int)(int8_t)(hx >> (8 * j)), lo = (int)(int8_t)(ln >> (8 * j));
             if (lo > hi) continue;                 // no element of this class
+            amax = max(amax, max(abs(hi), abs(lo)));
             atomicMin(&w.emin[3 * c + q], lo);     // codes; k_bnb_ext maps them to E_2
             atomicMax(&w.emax[3 * c + q], hi);
         }
+        zm = (uint32_t)amax * (uint32_t)abs(gam[c]);
     }
     if (threadIdx.x < 64) {
         zm = warp_max_u32(zm);
