@@ -526,6 +526,34 @@ __global__ void k_relu_bwd(const int8_t* __restrict__ ea, const int8_t* __restri
                            int64_t n, int8_t* __restrict__ e, uint2* __restrict__ e16) {
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
     int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e16) {
+        // with the fp16 copy (n % 16 == 0, all aligned): 8 codes a thread, so that a warp's
+        // 16-byte stores of the copy are contiguous
+        const int64_t n8 = n / 8;
+        for (int64_t v = i0; v < n8; v += stride) {
+            const uint2 x = reinterpret_cast<const uint2*>(ea)[v];
+            const uint2 m = reinterpret_cast<const uint2*>(a)[v];
+            const uint32_t xs[2] = {x.x, x.y}, ms[2] = {m.x, m.y};
+            uint32_t r[2];
+#pragma unroll
+            for (int j = 0; j < 2; j++) {
+                uint32_t t = 0;
+#pragma unroll
+                for (int b = 0; b < 4; b++) {
+                    const int8_t mv = (int8_t)(ms[j] >> (8 * b));
+                    const uint32_t xv = (xs[j] >> (8 * b)) & 0xffu;
+                    t |= (mv > 0 ? xv : 0u) << (8 * b);
+                }
+                r[j] = t;
+            }
+            reinterpret_cast<uint2*>(e)[v] = make_uint2(r[0], r[1]);
+            uint4 h;
+            tc::i8x4_to_f16x4(r[0], h.x, h.y);
+            tc::i8x4_to_f16x4(r[1], h.z, h.w);
+            reinterpret_cast<uint4*>(e16)[v] = h;
+        }
+        return;
+    }
     bool vec = (((uintptr_t)ea | (uintptr_t)a | (uintptr_t)e) & 15) == 0;
     int64_t n16 = vec ? n / 16 : 0;
     for (int64_t v = i0; v < n16; v += stride) {
@@ -542,7 +570,6 @@ __global__ void k_relu_bwd(const int8_t* __restrict__ ea, const int8_t* __restri
                 r |= (mv > 0 ? xv : 0u) << (8 * b);
             }
             xs[j] = (int)r;
-            put_f16x4(e16, 4 * v + j, r);
         }
         reinterpret_cast<int4*>(e)[v] = make_int4(xs[0], xs[1], xs[2], xs[3]);
     }
