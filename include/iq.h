@@ -346,10 +346,19 @@ iq_status iq_conv_fwd_frozen(const iq_conv_desc* d, const int8_t* x, const int8_
  *           where the sums are accumulated in int64 (IQ_ERR_UNSUPPORTED otherwise)
  *   e_f16   optional out fp16 [n][p][q][k], as x_f16 of iq_conv_fwd for the errors e: written
  *           first (not with IQ_CONV_E_F16_READY in d->flags: then it is read as it is) and
- *           read by the kernels; pass it to iq_conv_wgrad of the same layer */
+ *           read by the kernels; pass it to iq_conv_wgrad of the same layer
+ *   dx_mask optional int8 [n][h][w][c]: the dx codes are zeroed where dx_mask <= 0 after Q_E
+ *           (s_dx stays the unmasked tensor's): the ReLU backward of the layer whose
+ *           activation codes dx_mask holds, usually this layer's own input x (what
+ *           iq_relu_bwd would do next, Eq. (EQ) then the mask of Sec. 3.3.1)
+ *   dx_f16  optional out fp16 [n][h][w][c]: the exact fp16 copy of the (masked) dx codes, for
+ *           the layer below under IQ_CONV_E_F16_READY (16-byte aligned with dx and dx_mask,
+ *           n h w c % 16 == 0, else IQ_ERR_INVALID_ARG).  dx_mask and dx_f16: NHWC only
+ *           (IQ_ERR_UNSUPPORTED with IQ_LAYOUT_NCHW); no counterpart in the paper */
 iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
                         const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
-                        void* e_f16, void* ws, size_t ws_bytes, iq_stream stream);
+                        void* e_f16, const int8_t* dx_mask, void* dx_f16, void* ws,
+                        size_t ws_bytes, iq_stream stream);
 
 /* iq_conv_wgrad -- weight gradient and its quantization (Sec. 3.3.2):
  * G[k][r][s][c] = sum_{n,p,q} e[n,p,q,k] x[n, h(p,r), w(q,s), c] in exact int64, then

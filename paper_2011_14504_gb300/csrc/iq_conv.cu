@@ -874,8 +874,13 @@ static iq_status conv_fwd_frozen_nhwc(const iq_conv_desc* d, const int8_t* x, co
 
 static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const double* s_e,
                                  const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
-                                 void* e_f16, void* ws, size_t ws_bytes, iq_stream stream) {
+                                 void* e_f16, const int8_t* dx_mask, void* dx_f16, void* ws,
+                                 size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d) || !e || !s_e || !w || !dx || !s_dx) return IQ_ERR_INVALID_ARG;
+    const int64_t ndx = (int64_t)d->n * d->h * d->w * d->c;
+    if (dx_f16 && (!f16_copy_ok(dx, dx_f16, ndx) || ((uintptr_t)dx_mask & 15)))
+        return IQ_ERR_INVALID_ARG;
+    __half* dx16 = (__half*)dx_f16;
     const bool wide = dgrad_wide(d);
     if (wide && acc_out) return IQ_ERR_UNSUPPORTED;   // the sums need 64 bits: no int32 copy
     if ((int64_t)(d->k / d->groups) * d->r * d->s >= (int64_t(1) << 31) / 4)
@@ -914,9 +919,12 @@ static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const d
             r = conv_dgrad_tc(d, e, w, nullptr, (long long*)accw, nullptr, nullptr, nullptr, tcws,
                               st, &done, (const __half*)e_f16);
             if (r != IQ_OK) return r;
-            if (done)
-                return requant_int(accw, IQ_I64, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
-                                   s_dx, rq, st);
+            if (done) {
+                r = requant_int(accw, IQ_I64, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
+                                s_dx, rq, st);
+                if (r != IQ_OK || (!dx_mask && !dx16)) return r;
+                return codes_mask_copy(dx, dx_mask, total, dx16, st);
+            }
         } else {
             r = bn_stats_init(stats, d->c, st);
             if (r != IQ_OK) return r;
@@ -928,7 +936,7 @@ static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const d
                                                      rq_params_slot(rq), s_dx);
                 IQ_LAUNCH_CHECK();
                 return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx,
-                                     IQ_I8, s_dx, rq, st, true);
+                                     IQ_I8, s_dx, rq, st, true, false, dx16, dx_mask);
             }
         }
     }
@@ -958,7 +966,7 @@ static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const d
                                                  rq_params_slot(rq), s_dx);
             IQ_LAUNCH_CHECK();
             return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
-                                 s_dx, rq, st, true);
+                                 s_dx, rq, st, true, false, dx16, dx_mask);
         }
     }
     // stride 2: the four parity phases of the input as stride-1 problems on the tensor cores
@@ -974,7 +982,7 @@ static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const d
                                                  rq_params_slot(rq), s_dx);
             IQ_LAUNCH_CHECK();
             return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
-                                 s_dx, rq, st, true);
+                                 s_dx, rq, st, true, false, dx16, dx_mask);
         }
     }
     int64_t wn = (int64_t)d->k * d->r * d->s * cp.Cg;
@@ -992,7 +1000,7 @@ static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const d
         IQ_LAUNCH_CHECK();
         kt_post(st, IQ_KERNEL_CONV_SIMT);
         return requant_apply(accw, IQ_I64, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8,
-                             s_dx, rq, st);
+                             s_dx, rq, st, false, false, dx16, dx_mask);
     }
     kt_pre(st);
     k_conv_simt<OP_DGRAD, false><<<grid, 256, 0, st>>>(cp, e, wt, acc, nullptr, nullptr, nullptr,
@@ -1000,7 +1008,7 @@ static iq_status conv_dgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const d
     IQ_LAUNCH_CHECK();
     kt_post(st, IQ_KERNEL_CONV_SIMT);
     return requant_apply(acc, IQ_I32, total, s_in, 8, IQ_MODE_SQ, 0, 0, 0, 0, dx, IQ_I8, s_dx, rq,
-                         st);
+                         st, false, false, dx16, dx_mask);
 }
 
 static iq_status conv_wgrad_nhwc(const iq_conv_desc* d, const int8_t* e, const double* s_e,
@@ -1196,10 +1204,13 @@ extern "C" iq_status iq_conv_fwd(const iq_conv_desc* d, const int8_t* x, const d
 
 extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const double* s_e,
                                    const int8_t* w, int8_t* dx, double* s_dx, int32_t* acc_out,
-                                   void* e_f16, void* ws, size_t ws_bytes, iq_stream stream) {
+                                   void* e_f16, const int8_t* dx_mask, void* dx_f16, void* ws,
+                                   size_t ws_bytes, iq_stream stream) {
     if (!desc_ok(d)) return IQ_ERR_INVALID_ARG;
     if (d->layout == IQ_LAYOUT_NHWC)
-        return conv_dgrad_nhwc(d, e, s_e, w, dx, s_dx, acc_out, e_f16, ws, ws_bytes, stream);
+        return conv_dgrad_nhwc(d, e, s_e, w, dx, s_dx, acc_out, e_f16, dx_mask, dx_f16, ws,
+                               ws_bytes, stream);
+    if (dx_mask || dx_f16) return IQ_ERR_UNSUPPORTED;      // NHWC only
     if (!e || !s_e || !w || !dx || !s_dx) return IQ_ERR_INVALID_ARG;
     int64_t nin, nw, nout, pq;
     conv_sizes(d, &nin, &nw, &nout, &pq);
@@ -1218,7 +1229,8 @@ extern "C" iq_status iq_conv_dgrad(const iq_conv_desc* d, const int8_t* e, const
     int8_t* dxn = (int8_t*)(b + L.off_y);
     int32_t* accn = acc_out ? (int32_t*)(b + L.off_acc) : nullptr;
     r = conv_dgrad_nhwc(&dn, (const int8_t*)(b + L.off_x), s_e, (const int8_t*)(b + L.off_w), dxn,
-                        s_dx, accn, e_f16, b + L.off_rest, ws_bytes - L.off_rest, stream);
+                        s_dx, accn, e_f16, nullptr, nullptr, b + L.off_rest,
+                        ws_bytes - L.off_rest, stream);
     if (r != IQ_OK) return r;
     const int64_t hw = (int64_t)d->h * d->w;
     r = to_nchw(dxn, dx, d->n, d->c, hw, 1, st);

@@ -62,11 +62,19 @@ inline RqParams* rq_params_slot(void* ws) { return (RqParams*)((char*)ws + 256);
 // the SQ modes' M is not the tensor's own maximum (frozen statistics), so q is clipped to
 // [-M, M] first.
 // out16 (optional, int8 SQ codes only): the fp16 copy of the output codes is written too
-// (n % 16 == 0, out and out16 16-byte aligned).
+// (n % 16 == 0, out and out16 16-byte aligned).  mask (optional, int8 SQ codes only): a code
+// is kept where mask > 0 and zeroed elsewhere (the ReLU backward of the layer whose
+// activation codes mask holds; the scale is the unmasked tensor's), 16-byte aligned with out16.
 iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
                         void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st,
-                        bool params_ready = false, bool clip = false, __half* out16 = nullptr);
+                        bool params_ready = false, bool clip = false, __half* out16 = nullptr,
+                        const int8_t* mask = nullptr);
+
+// finished int8 codes x: zeroed in place where mask <= 0 (mask optional), and their fp16
+// copy written (x16 optional: n % 16 == 0, x, mask, x16 16-byte aligned)
+iq_status codes_mask_copy(int8_t* x, const int8_t* mask, int64_t n, __half* x16,
+                          cudaStream_t st);
 
 // int8 codes -> their exact fp16 copies (n % 16 == 0, both 16-byte aligned)
 iq_status codes_to_f16(const int8_t* x, __half* xf, int64_t n, cudaStream_t st);

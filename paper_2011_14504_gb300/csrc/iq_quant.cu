@@ -212,6 +212,16 @@ __device__ __forceinline__ uint32_t sq8_word_f(const int4& v, uint32_t M, uint32
     return w;
 }
 
+// bytes 0xff where the 4 int8 codes of a are > 0 (nonzero with a clear sign bit), through
+// prmt's sign-replicating selectors
+__device__ __forceinline__ uint32_t pos_bytes(uint32_t a) {
+    const uint32_t nz = ((a & 0x7f7f7f7fu) + 0x7f7f7f7fu) | a;
+    uint32_t pn, sg;
+    asm("prmt.b32 %0, %1, 0, 0xBA98;" : "=r"(pn) : "r"(nz));
+    asm("prmt.b32 %0, %1, 0, 0xBA98;" : "=r"(sg) : "r"(a));
+    return pn & ~sg;
+}
+
 // the fp16 copy of 4 codes (one 8-byte store) when the caller asked for it
 __device__ __forceinline__ void put_f16x4(uint2* __restrict__ out16, int64_t i, uint32_t w) {
     if (out16) {
@@ -221,12 +231,12 @@ __device__ __forceinline__ void put_f16x4(uint2* __restrict__ out16, int64_t i, 
     }
 }
 
-// int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores), and
-// optionally their fp16 copies
+// int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores), optionally
+// zeroed where mask4's codes are not positive, and optionally their fp16 copies
 template <bool CLIP>
 __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int relu,
                               const RqParams* __restrict__ prm, uint32_t* __restrict__ out,
-                              uint2* __restrict__ out16) {
+                              uint2* __restrict__ out16, const uint32_t* __restrict__ mask4) {
     const RqParams p = *prm;
     const int64_t lim = qmax(k);
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -237,13 +247,19 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
         for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
              i += 4 * stride) {
             int4 v[4];
+            uint32_t mk[4];
+            // the mask words are loaded beside the sums, so that both are in flight at once
 #pragma unroll
-            for (int j = 0; j < 4; j++)
-                v[j] = i + j * stride < n4 ? __ldg(q + i + j * stride) : make_int4(0, 0, 0, 0);
+            for (int j = 0; j < 4; j++) {
+                const bool in = i + j * stride < n4;
+                v[j] = in ? __ldg(q + i + j * stride) : make_int4(0, 0, 0, 0);
+                mk[j] = in && mask4 ? __ldg(mask4 + i + j * stride) : 0x01010101u;
+            }
 #pragma unroll
             for (int j = 0; j < 4; j++)
                 if (i + j * stride < n4) {
-                    const uint32_t w = sq8_word_f<CLIP>(v[j], M, p.R8, kq, relu);
+                    uint32_t w = sq8_word_f<CLIP>(v[j], M, p.R8, kq, relu);
+                    if (mask4) w &= pos_bytes(mk[j]);
                     out[i + j * stride] = w;
                     put_f16x4(out16, i + j * stride, w);
                 }
@@ -255,17 +271,21 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
         const int64_t i2 = i + stride;
         const int4 v = __ldg(q + i);
         const int4 v2 = i2 < n4 ? __ldg(q + i2) : make_int4(0, 0, 0, 0);
-        const uint32_t w = ((uint32_t)sq_code<CLIP>(v.x, p, k, relu, lim) & 0xffu) |
-                           (((uint32_t)sq_code<CLIP>(v.y, p, k, relu, lim) & 0xffu) << 8) |
-                           (((uint32_t)sq_code<CLIP>(v.z, p, k, relu, lim) & 0xffu) << 16) |
-                           (((uint32_t)sq_code<CLIP>(v.w, p, k, relu, lim) & 0xffu) << 24);
+        const uint32_t mk = mask4 ? __ldg(mask4 + i) : 0x01010101u;
+        const uint32_t mk2 = mask4 && i2 < n4 ? __ldg(mask4 + i2) : 0x01010101u;
+        uint32_t w = ((uint32_t)sq_code<CLIP>(v.x, p, k, relu, lim) & 0xffu) |
+                     (((uint32_t)sq_code<CLIP>(v.y, p, k, relu, lim) & 0xffu) << 8) |
+                     (((uint32_t)sq_code<CLIP>(v.z, p, k, relu, lim) & 0xffu) << 16) |
+                     (((uint32_t)sq_code<CLIP>(v.w, p, k, relu, lim) & 0xffu) << 24);
+        if (mask4) w &= pos_bytes(mk);
         out[i] = w;
         put_f16x4(out16, i, w);
         if (i2 < n4) {
-            const uint32_t w2 = ((uint32_t)sq_code<CLIP>(v2.x, p, k, relu, lim) & 0xffu) |
-                                (((uint32_t)sq_code<CLIP>(v2.y, p, k, relu, lim) & 0xffu) << 8) |
-                                (((uint32_t)sq_code<CLIP>(v2.z, p, k, relu, lim) & 0xffu) << 16) |
-                                (((uint32_t)sq_code<CLIP>(v2.w, p, k, relu, lim) & 0xffu) << 24);
+            uint32_t w2 = ((uint32_t)sq_code<CLIP>(v2.x, p, k, relu, lim) & 0xffu) |
+                          (((uint32_t)sq_code<CLIP>(v2.y, p, k, relu, lim) & 0xffu) << 8) |
+                          (((uint32_t)sq_code<CLIP>(v2.z, p, k, relu, lim) & 0xffu) << 16) |
+                          (((uint32_t)sq_code<CLIP>(v2.w, p, k, relu, lim) & 0xffu) << 24);
+            if (mask4) w2 &= pos_bytes(mk2);
             out[i2] = w2;
             put_f16x4(out16, i2, w2);
         }
@@ -347,12 +367,37 @@ __global__ void k_rq_int(const T* __restrict__ q, int64_t n, int k,
     }
 }
 
+// x[i] = 0 where mask[i] <= 0, in place, and optionally the fp16 copy of the result (x16:
+// n % 16 == 0, x, mask and x16 16-byte aligned, 8 codes a thread; else one code a thread)
+__global__ void k_mask_inplace(int8_t* x, const int8_t* __restrict__ mask, int64_t n,
+                               uint4* __restrict__ x16) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (x16) {
+        for (int64_t v = i0; v < n / 8; v += stride) {
+            uint2 c = reinterpret_cast<const uint2*>(x)[v];
+            const uint2 m = reinterpret_cast<const uint2*>(mask)[v];
+            c.x &= pos_bytes(m.x);
+            c.y &= pos_bytes(m.y);
+            reinterpret_cast<uint2*>(x)[v] = c;
+            uint4 h;
+            tc::i8x4_to_f16x4(c.x, h.x, h.y);
+            tc::i8x4_to_f16x4(c.y, h.z, h.w);
+            x16[v] = h;
+        }
+        return;
+    }
+    for (int64_t i = i0; i < n; i += stride)
+        if (mask[i] <= 0) x[i] = 0;
+}
+
 iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_in, int k,
                         int mode, uint64_t seed, uint64_t layer, uint64_t step, uint64_t tag,
                         void* out, int out_dtype, double* s_out, void* ws, cudaStream_t st,
-                        bool params_ready, bool clip, __half* out16) {
-    if (out16 && (out_dtype != IQ_I8 || !f16_copy_ok(out, out16, n) ||
-                  (mode != IQ_MODE_SQ && mode != IQ_MODE_SQ_RELU)))
+                        bool params_ready, bool clip, __half* out16, const int8_t* mask) {
+    if ((out16 || mask) && (out_dtype != IQ_I8 || (mode != IQ_MODE_SQ && mode != IQ_MODE_SQ_RELU)))
+        return IQ_ERR_INVALID_ARG;
+    if (out16 && (!f16_copy_ok(out, out16, n) || ((uintptr_t)mask & 15)))
         return IQ_ERR_INVALID_ARG;
     unsigned long long* cell = (unsigned long long*)ws;
     RqParams* prm = rq_params_slot(ws);
@@ -369,12 +414,16 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
     if (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) {
         const bool x4 = in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
                         (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0;
-        if (x4 && clip)
+        // the mask rides on the 4-wide kernel when its codes are 4-byte aligned
+        const bool m4 = !mask || ((uintptr_t)mask & 3) == 0;
+        if (x4 && m4 && clip)
             k_sq_i32_i8x4<true><<<grid_for(n / 4), kThreads, 0, st>>>(
-                (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16);
-        else if (x4)
+                (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16,
+                (const uint32_t*)mask);
+        else if (x4 && m4)
             k_sq_i32_i8x4<false><<<grid_for(n / 4), kThreads, 0, st>>>(
-                (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16);
+                (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16,
+                (const uint32_t*)mask);
         else if (in_dtype == IQ_I32 && clip)
             k_sq_int<int32_t, true><<<g, kThreads, 0, st>>>((const int32_t*)q, n, k, relu, prm,
                                                             out, out_dtype);
@@ -396,13 +445,26 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
                                                        step, tag, ep, out, out_dtype);
     }
     IQ_LAUNCH_CHECK();
-    const bool fused16 = out16 && in_dtype == IQ_I32 && out_dtype == IQ_I8 && n % 4 == 0 &&
-                         (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0;
+    const bool fused = (out16 || mask) && in_dtype == IQ_I32 && out_dtype == IQ_I8 &&
+                       n % 4 == 0 && (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0 &&
+                       (!mask || ((uintptr_t)mask & 3) == 0);
     kt_post_bytes(st, (mode == IQ_MODE_SQ || mode == IQ_MODE_SQ_RELU) ? IQ_KERNEL_SQ_CODES
                                                                        : IQ_KERNEL_RQ_CODES,
-                  (double)n * (isz + osz + (fused16 ? 2.0 : 0.0)));
-    // the kernels without the fused copy: one conversion pass
-    if (out16 && !fused16) return codes_to_f16((const int8_t*)out, out16, n, st);
+                  (double)n * (isz + osz + (fused && out16 ? 2.0 : 0.0) +
+                               (fused && mask ? 1.0 : 0.0)));
+    if ((out16 || mask) && !fused) {
+        // the kernels without the fused mask / copy: one pass over the codes, in place
+        return codes_mask_copy((int8_t*)out, mask, n, out16, st);
+    }
+    return IQ_OK;
+}
+
+iq_status codes_mask_copy(int8_t* x, const int8_t* mask, int64_t n, __half* x16,
+                          cudaStream_t st) {
+    if (n == 0 || (!mask && !x16)) return IQ_OK;
+    if (!mask) return codes_to_f16(x, x16, n, st);
+    k_mask_inplace<<<grid_for(x16 ? n / 8 : n), kThreads, 0, st>>>(x, mask, n, (uint4*)x16);
+    IQ_LAUNCH_CHECK();
     return IQ_OK;
 }
 

@@ -58,6 +58,7 @@ class Conv:
     s_ex: torch.Tensor = None
     x16: torch.Tensor = None      # fp16 copy of x, read by the forward and the wgrad
     a16: torch.Tensor = None      # the next conv's x16 when that conv reads a: written here
+    ex_masked: bool = False       # ex carries the ReLU mask of the conv below (x > 0)
     macs: int = 0                 # in-bounds multiply-accumulates of one pass
     macs_dense: int = 0           # every tap, the zero padding included
 
@@ -275,15 +276,18 @@ class FcnVgg16:
             if isinstance(P, Pool):
                 P.ex = torch.empty_like(P.x)
                 P.s_ex = torch.zeros(1, dtype=torch.float64, device=dev)
-        # one fp16 error buffer: written with the errors by the ReLU backward of a layer,
-        # read by its data and weight gradients (IQ_CONV_E_F16_READY)
+        # fp16 error buffers: written with the errors by the ReLU backward of a layer or by
+        # the data gradient of the conv above it, read by its data and weight gradients
+        # (IQ_CONV_E_F16_READY)
         e16 = 0
         for L in self.convs:
             if L.cout % 64 == 0:
                 e16 = max(e16, L.a.numel())
                 if L.relu:
                     L.desc.flags |= iq.IQ_CONV_E_F16_READY
-        self.e16 = torch.empty(max(e16, 16), dtype=torch.float16, device=dev)
+        # two of them: a data gradient writes the next layer's copy (with the ReLU mask
+        # fused, below) while this layer's weight gradient still reads its own
+        self.e16 = [torch.empty(max(e16, 16), dtype=torch.float16, device=dev) for _ in range(2)]
 
     def _alloc_carriers(self):
         """fp16 copies of the codes that the tensor-core kernels read: one per conv input,
@@ -410,7 +414,9 @@ class FcnVgg16:
         # error arriving at the output of the current item, walking backwards
         err, s_err = self.e_score, self.s_e_score
         npool = len(self.pools)
-        for item in reversed(self.layers):
+        items = list(reversed(self.layers))
+        masked, buf = False, 0        # err already carries the ReLU mask, in e16[buf]
+        for idx, item in enumerate(items):
             if isinstance(item, Pool):
                 npool -= 1
                 if npool in extra:        # the skip's error joins the main path's
@@ -422,15 +428,25 @@ class FcnVgg16:
                 err, s_err = item.ex, item.s_ex
                 continue
             L = item
-            e16 = self.e16 if L.cout % 64 == 0 else None
-            if L.relu:
+            e16 = self.e16[buf] if L.cout % 64 == 0 else None
+            if masked:
+                e = err                   # the conv above applied this layer's ReLU mask
+            elif L.relu:
                 # the errors and, for the data and weight gradients, their fp16 copy
                 iq.iq_relu_bwd(err, L.a, L.e, e_f16=e16, stream=stream)
                 e = L.e
             else:
                 e = err
+            # the conv below, when it feeds this one directly: its ReLU backward rides on
+            # this data gradient (dx masked by the input codes, which are its output), with
+            # the fp16 copy for its own gradients
+            below = items[idx + 1] if idx + 1 < len(items) else None
+            fuse = (L.layer_id > 0 and isinstance(below, Conv) and below.relu and
+                    below.a is L.x and below.cout % 64 == 0)
             if L.layer_id > 0:
-                iq.iq_conv_dgrad(L.desc, e, s_err, L.wq, L.ex, L.s_ex, e_f16=e16, ws=ws,
+                iq.iq_conv_dgrad(L.desc, e, s_err, L.wq, L.ex, L.s_ex, e_f16=e16,
+                                 dx_mask=L.x if fuse else None,
+                                 dx_f16=self.e16[1 - buf] if fuse else None, ws=ws,
                                  stream=stream)
             iq.iq_conv_wgrad(L.desc, e, s_err, L.x, L.s_x, L.g, L.s_g, gq_mode=2, seed=seed,
                              layer=L.layer_id, step=step, e_f16=e16, x_f16=L.x16, ws=ws,
@@ -438,6 +454,10 @@ class FcnVgg16:
             self._update(L.master, L.wq, L.g, L.s_g, stream)
             if L.layer_id > 0:
                 err, s_err = L.ex, L.s_ex
+            L.ex_masked = fuse
+            masked = fuse
+            if fuse:
+                buf = 1 - buf
         self.step_count += 1
 
     def _update(self, master, wq, g, s_g, stream):

@@ -130,7 +130,8 @@ def load(path: str | None = None):
                               _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
     L.iq_conv_fwd_frozen.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, C.POINTER(BnBits), _I, _I,
                                      _P, _P, _P, _P, _SZ, _P]
-    L.iq_conv_dgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]
+    L.iq_conv_dgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ,
+                                _P]
     L.iq_conv_wgrad.argtypes = [C.POINTER(ConvDesc), _P, _P, _P, _P, _I, _U64, _U64, _U64, _P, _P,
                                 _P, _P, _P, _P, _SZ, _P]
     L.iq_bn_int_fwd.argtypes = [_P, _I64, _I32, _P, _P, _P, C.POINTER(BnBits), _P, _P, _P, _P, _P,
@@ -401,13 +402,14 @@ def iq_conv_fwd_frozen(d: ConvDesc, x, w, frozen, a, use_bn=False, relu=True, bi
                                      _stream(stream)))
 
 
-def iq_conv_dgrad(d: ConvDesc, e, s_e, w, dx, s_dx, acc_out=None, e_f16=None, ws=None,
-                  stream=None):
+def iq_conv_dgrad(d: ConvDesc, e, s_e, w, dx, s_dx, acc_out=None, e_f16=None, dx_mask=None,
+                  dx_f16=None, ws=None, stream=None):
     if ws is None:
         ws = _ws(iq_conv_dgrad_workspace_size(d), e.device)
     _check("iq_conv_dgrad",
            load().iq_conv_dgrad(C.byref(d), _p(e), _p(s_e), _p(w), _p(dx), _p(s_dx), _p(acc_out),
-                                _p(e_f16), _p(ws), ws.numel(), _stream(stream)))
+                                _p(e_f16), _p(dx_mask), _p(dx_f16), _p(ws), ws.numel(),
+                                _stream(stream)))
 
 
 def iq_conv_wgrad(d: ConvDesc, e, s_e, x, s_x, g, s_g, gq_mode=1, seed=0, layer=0, step=0,

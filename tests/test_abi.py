@@ -120,6 +120,12 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert lib.iq_relu_bwd(16, 16, 32, 16, 24, None) == iq.IQ_ERR_INVALID_ARG
     assert lib.iq_relu_bwd(16, 16, 40, 16, 32, None) == iq.IQ_ERR_INVALID_ARG   # n % 16
     assert lib.iq_maxpool_fwd(16, 1, 8, 8, 16, 2, 2, 0, 16, 16, 24, None) == iq.IQ_ERR_INVALID_ARG
+    # the data gradient's ReLU mask and fp16 copy: NHWC only, the copy 16-byte aligned
+    dn = iq.conv_desc(1, 8, 8, 16, 16, 3, 3, 1, 1, layout=iq.IQ_LAYOUT_NCHW)
+    assert lib.iq_conv_dgrad(C.byref(dn), 16, 16, 16, 16, 16, None, None, 16, None, 16, 1 << 20,
+                             None) == iq.IQ_ERR_UNSUPPORTED
+    assert lib.iq_conv_dgrad(C.byref(d), 16, 16, 16, 16, 16, None, None, 16, 24, 16, 1 << 30,
+                             None) == iq.IQ_ERR_INVALID_ARG
     # bad bit width / dtype combination
     rc = lib.iq_quantize(1, 10, 16, iq.IQ_MODE_UQ, iq.IQ_I8, 1, 1, 1, 4096, None)
     assert rc == iq.IQ_ERR_INVALID_ARG

@@ -53,7 +53,11 @@ def test_fcn_train_steps_match_oracle(classes, width, n, h):
             assert np.array_equal(host(L.g), gq.astype(np.int8)), (step, L.name)
             assert host(L.s_g)[0] == s_g
             if L.layer_id > 0:
-                assert np.array_equal(host(L.ex), out["ex"][L.layer_id][0]), (step, L.name)
+                want = out["ex"][L.layer_id][0]
+                if L.ex_masked:      # the ReLU backward of the conv below, fused (mask: x > 0;
+                    # x is the conv below's output, checked against the oracle above)
+                    want = O.relu_bwd(want, host(L.x))
+                assert np.array_equal(host(L.ex), want), (step, L.name)
             assert np.array_equal(host(L.master), ora.masters[L.layer_id]), (step, L.name)
         assert np.array_equal(host(net.up_master), ora.up_master)
 
@@ -110,7 +114,11 @@ def test_fcn8s_train_steps_match_oracle(classes, width, n, h, wd):
             G, gq, s_g = out["grads"][L.layer_id]
             assert np.array_equal(host(L.g), gq.astype(np.int8)), (step, L.name)
             if L.layer_id > 0:
-                assert np.array_equal(host(L.ex), out["ex"][L.layer_id][0]), (step, L.name)
+                want = out["ex"][L.layer_id][0]
+                if L.ex_masked:      # the ReLU backward of the conv below, fused (mask: x > 0;
+                    # x is the conv below's output, checked against the oracle above)
+                    want = O.relu_bwd(want, host(L.x))
+                assert np.array_equal(host(L.ex), want), (step, L.name)
             assert np.array_equal(host(L.master), ora.masters[L.layer_id]), (step, L.name)
         for U, m in ((net.up8, ora.up8_master), (net.up2b, ora.up2b_master),
                      (net.up2a, ora.up2a_master), (net.sp4, ora.sp4_master),

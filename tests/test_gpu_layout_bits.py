@@ -302,3 +302,39 @@ def test_carriers_of_pool_relu_and_bn_backward():
     dx = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
     iq.iq_conv_dgrad(d, dev(ee), sc(1e-5), dev(wq), dx, sc(), acc_out=dacc, e_f16=ee16)
     assert np.array_equal(host(dacc), O.conv_dgrad(cv, ee, wq))
+
+
+@pytest.mark.parametrize("case", ["tensor", "stride2", "int64"])
+def test_dgrad_with_relu_mask_and_copy(case):
+    """dx_mask / dx_f16: the data gradient's Q_E codes zeroed where the mask codes are not
+    positive (the ReLU backward of the layer below, which iq_relu_bwd would apply next) and
+    their fp16 copy, on the 4-wide SQ8 pass (tensor-core data gradient, stride-2 phases) and
+    after the int64-sum form; the scale is the unmasked tensor's."""
+    g = S.rng({"tensor": 971, "stride2": 972, "int64": 973}[case])
+    if case == "tensor":
+        n, h, w, c, k, r, st, pd = 2, 21, 19, 64, 128, 3, 1, 1
+    elif case == "stride2":
+        n, h, w, c, k, r, st, pd = 2, 18, 20, 64, 128, 3, 2, 1
+    else:
+        n, h, w, c, k, r, st, pd = 1, 8, 8, 64, 2720, 7, 1, 3    # (k r s) 127^2 >= 2^31
+    cv = O.Conv(n, h, w, c, k, r, r, st, pd, 1)
+    d = iq.conv_desc(n, h, w, c, k, r, r, st, pd)
+    p, q = cv.pq
+    if case == "int64":
+        e = np.full((n, p, q, k), 127, np.int8)
+        wq = np.full((k, r, r, c), 127, np.int8)
+        wq[:, :, :, 3] = -127
+    else:
+        e = S.int8_uniform(g, (n, p, q, k))
+        wq = O.requant_master(O.uq(S.he_weights(g, (k, r, r, c), c * r * r), 24)).astype(np.int8)
+    mask = S.int8_uniform(g, (n, h, w, c))            # codes of either sign, zeros among them
+    dx = torch.empty((n, h, w, c), dtype=torch.int8, device=DEV)
+    dx16 = torch.full((dx.numel(),), float("nan"), dtype=torch.float16, device=DEV)
+    s_dx = sc()
+    iq.iq_conv_dgrad(d, dev(e), sc(1e-4), dev(wq), dx, s_dx, dx_mask=dev(mask), dx_f16=dx16)
+    acc = O.conv_dgrad(cv, e, wq)
+    codes, s_want = O.sq_int(acc, 1e-4 * 2.0 ** -7, 8)
+    want = O.relu_bwd(codes.astype(np.int8), mask)
+    assert np.array_equal(host(dx), want)
+    assert s_dx.item() == s_want
+    assert np.array_equal(_f16_codes(dx16).reshape(dx.shape), want)
