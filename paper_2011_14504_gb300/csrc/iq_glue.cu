@@ -156,6 +156,60 @@ __global__ void k_maxpool_bwd_tiled(const int8_t* __restrict__ e, const uint8_t*
     }
 }
 
+// Overlapping windows: one thread per 4 channels of an input pixel, for kPoolRows rows (grid:
+// pixel-channel groups of a row, row groups, images; 32-bit index arithmetic).  Each input
+// sums the errors of the windows whose first maximum it is; the block's largest |sum| goes to
+// *amax with one atomic (a single address takes every block's atomic).
+constexpr int kPoolRows = 4;
+
+__global__ void __launch_bounds__(kThreads) k_maxpool_bwd4(
+    const uint32_t* __restrict__ e4, const uint32_t* __restrict__ arg4, int h, int w, int c4,
+    int k, int s, int p, int P, int Q, int4* __restrict__ sums4,
+    unsigned long long* __restrict__ amax) {
+    __shared__ unsigned long long wmax[kThreads / 32];
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    const int b = blockIdx.z;
+    uint64_t mx = 0;
+    if (idx < w * c4) {
+        const int ww = idx / c4, cg = idx - ww * c4;
+        // windows j with j s - p <= ww <= j s - p + k - 1 (likewise i for hh)
+        const int j_lo = ww + p - k + 1 > 0 ? (ww + p - k + s) / s : 0;
+        const int j_hi = min((ww + p) / s, Q - 1);
+        const int h_end = min(h, (int)(blockIdx.y + 1) * kPoolRows);
+        for (int hh = blockIdx.y * kPoolRows; hh < h_end; hh++) {
+            int sum[4] = {0, 0, 0, 0};
+            const int i_lo = hh + p - k + 1 > 0 ? (hh + p - k + s) / s : 0;
+            const int i_hi = min((hh + p) / s, P - 1);
+            for (int i = i_lo; i <= i_hi; i++) {
+                const int r = hh - (i * s - p);
+                for (int j = j_lo; j <= j_hi; j++) {
+                    const uint32_t tap = (uint32_t)(r * k + ww - (j * s - p));
+                    const int64_t oo = (((int64_t)b * P + i) * Q + j) * c4 + cg;
+                    const uint32_t av = __ldg(arg4 + oo), ev = __ldg(e4 + oo);
+#pragma unroll
+                    for (int l = 0; l < 4; l++)
+                        if (((av >> (8 * l)) & 0xffu) == tap)
+                            sum[l] += (int)(int8_t)(ev >> (8 * l));
+                }
+            }
+            sums4[(((int64_t)b * h + hh) * w + ww) * c4 + cg] =
+                make_int4(sum[0], sum[1], sum[2], sum[3]);
+#pragma unroll
+            for (int l = 0; l < 4; l++) {
+                const uint64_t a = (uint64_t)(sum[l] < 0 ? -sum[l] : sum[l]);
+                mx = a > mx ? a : mx;
+            }
+        }
+    }
+    mx = warp_max_u64(mx);
+    if ((threadIdx.x & 31) == 0) wmax[threadIdx.x >> 5] = mx;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int i = 1; i < kThreads / 32; i++) mx = wmax[i] > mx ? wmax[i] : mx;
+        if (mx) atomicMax(amax, (unsigned long long)mx);
+    }
+}
+
 __global__ void k_copy_scale(const double* __restrict__ a, double* __restrict__ b) { *b = *a; }
 __global__ void k_scale_pow2(const double* __restrict__ a, int e, double* __restrict__ out) {
     *out = ldexp(*a, e);
@@ -776,8 +830,18 @@ extern "C" iq_status iq_maxpool_bwd(const int8_t* e, const double* s_e, const ui
     void* rq = cur.take<char>(requant_ws_bytes());
     unsigned long long* cell = (unsigned long long*)rq;
     IQ_CUDA_CHECK(cudaMemsetAsync(cell, 0, 8, st));
-    k_maxpool_bwd<<<grid_for(total), kThreads, 0, st>>>(e, arg, n, h, w, c, k, s, p, P, Q, sums,
-                                                        nullptr, cell);
+    // 4 channels a thread over kPoolRows rows, a block row of (pixel, channel group)s
+    const bool vec4 = c % 4 == 0 && n <= 65535 && (h + kPoolRows - 1) / kPoolRows <= 65535 &&
+                      (int64_t)w * (c / 4) < (1 << 30) &&
+                      ((((uintptr_t)e) | (uintptr_t)arg) & 3) == 0;
+    if (vec4)
+        k_maxpool_bwd4<<<dim3((unsigned)((w * (c / 4) + kThreads - 1) / kThreads),
+                              (unsigned)((h + kPoolRows - 1) / kPoolRows), (unsigned)n),
+                         kThreads, 0, st>>>((const uint32_t*)e, (const uint32_t*)arg, h, w, c / 4,
+                                            k, s, p, P, Q, (int4*)sums, cell);
+    else
+        k_maxpool_bwd<<<grid_for(total), kThreads, 0, st>>>(e, arg, n, h, w, c, k, s, p, P, Q,
+                                                            sums, nullptr, cell);
     IQ_LAUNCH_CHECK();
     // overlapping windows add errors: Q_E = SQ(., 8) of the sums, same element scale s_e
     return requant_apply(sums, IQ_I32, total, s_e, 8, IQ_MODE_SQ, 0, 0, 0, 0, ex, IQ_I8, s_ex, rq,

@@ -5,6 +5,7 @@
 // The paper (Sec. 5) runs DeepLabv3 fully quantized but does not say how its joins are
 // quantized; here each join evaluates the real-valued operation on the codes and then
 // applies Q_A / Q_E = SQ(., 8) (Eq. (ScaleQ) with Scale = max|.| of the whole tensor).
+#include <algorithm>
 #include <climits>
 
 #include "iq_internal.cuh"
@@ -36,7 +37,9 @@ struct CombHdr {
     UDiv div;
     float kq;      // fl(128 / M) (0 when M = 0)
     float c130;    // 130 / M rounded up
+    unsigned long long bound[IQ_MAX_TERMS];   // per operand max_ch(|a| vmax + |b|), as bits
 };
+static_assert(sizeof(CombHdr) <= 256, "the join header fits its 256 bytes");
 
 __device__ __forceinline__ double term_a(const TermDev& t, double s, int ch) {
     if (!t.gamma) return s;
@@ -46,47 +49,44 @@ __device__ __forceinline__ double term_b(const TermDev& t, int ch) {
     return t.beta ? __dmul_rn((double)t.beta[ch], ldexp(1.0, 2 - t.k_beta)) : 0.0;
 }
 
-// One block: per operand the bound max_ch(|a| vmax + |b|), the shift P from their sum (in
-// operand order), then the tables F = rhu(a 2^P), B = rhu(b 2^P).
-__global__ void k_comb_tables(Terms T, CombHdr* hdr, long long* F, long long* B) {
-    __shared__ unsigned long long lt[IQ_MAX_TERMS];
-    __shared__ int sP;
-    if (threadIdx.x < IQ_MAX_TERMS) lt[threadIdx.x] = 0ull;
-    __syncthreads();
-    for (int i = 0; i < T.n; i++) {
-        const TermDev& t = T.t[i];
-        const double s = *t.scale;
+// The tables, over ceil(c / 64) x operands blocks of 64 threads (the fp64 pipe of one SM is
+// narrow).  Stage 1: per operand the bound max_ch(|a| vmax + |b|), kept as the bit pattern
+// of a non-negative double (such doubles order as their bits; the cells are zeroed first).
+constexpr int kTabThreads = 64;
+
+__global__ void __launch_bounds__(kTabThreads) k_comb_bound(Terms T, CombHdr* hdr) {
+    const TermDev& t = T.t[blockIdx.y];
+    const int ch = blockIdx.x * blockDim.x + threadIdx.x;
+    double v = 0.0;
+    if (ch < t.c) {
         const double vmax = t.is16 ? 32767.0 : 127.0;
-        double l = 0.0;
-        for (int ch = threadIdx.x; ch < t.c; ch += blockDim.x) {
-            double v = __dadd_rn(__dmul_rn(fabs(term_a(t, s, ch)), vmax), fabs(term_b(t, ch)));
-            l = v > l ? v : l;
-        }
-        // non-negative doubles order as their bit patterns
-        atomicMax(&lt[i], (unsigned long long)__double_as_longlong(l));
+        v = __dadd_rn(__dmul_rn(fabs(term_a(t, *t.scale, ch)), vmax), fabs(term_b(t, ch)));
     }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        double bound = 0.0;
-        for (int i = 0; i < T.n; i++) bound = __dadd_rn(bound, __longlong_as_double((long long)lt[i]));
-        int e;
-        frexp(__dadd_rn(bound, 1.0), &e);
-        int P = 50 - e;
-        if (P > 62) P = 62;
-        sP = P;
+    const uint64_t m = warp_max_u64((uint64_t)__double_as_longlong(v));
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(&hdr->bound[blockIdx.y], (unsigned long long)m);
+}
+
+// Stage 2: the shift P from the bounds' sum (in operand order), then F = rhu(a 2^P) and
+// B = rhu(b 2^P); block (0, 0) publishes P and clears the max cell of the join's first pass.
+__global__ void __launch_bounds__(kTabThreads) k_comb_tab(Terms T, CombHdr* hdr, long long* F,
+                                                          long long* B) {
+    double bound = 0.0;
+    for (int i = 0; i < T.n; i++)
+        bound = __dadd_rn(bound, __longlong_as_double((long long)hdr->bound[i]));
+    int e;
+    frexp(__dadd_rn(bound, 1.0), &e);
+    int P = 50 - e;
+    if (P > 62) P = 62;
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) {
         hdr->P = P;
         hdr->maxz = 0ull;
     }
-    __syncthreads();
-    const int P = sP;
-    for (int i = 0; i < T.n; i++) {
-        const TermDev& t = T.t[i];
-        const double s = *t.scale;
-        for (int ch = threadIdx.x; ch < t.c; ch += blockDim.x) {
-            F[t.base + ch] = (long long)rhu(ldexp(term_a(t, s, ch), P));
-            B[t.base + ch] = (long long)rhu(ldexp(term_b(t, ch), P));
-        }
-    }
+    const TermDev& t = T.t[blockIdx.y];
+    const int ch = blockIdx.x * blockDim.x + threadIdx.x;
+    if (ch >= t.c) return;
+    const double s = *t.scale;
+    F[t.base + ch] = (long long)rhu(ldexp(term_a(t, s, ch), P));
+    B[t.base + ch] = (long long)rhu(ldexp(term_b(t, ch), P));
 }
 
 __device__ __forceinline__ int64_t load_code(const TermDev& t, int64_t idx) {
@@ -1158,7 +1158,14 @@ static iq_status combine_codes(const iq_term* terms, int32_t n_terms, int32_t co
     const size_t tab = (((size_t)base * 8) + 255) & ~size_t(255);
     long long* F = (long long*)((char*)ws + 256);
     long long* B = (long long*)((char*)ws + 256 + tab);
-    k_comb_tables<<<1, 1024, 0, st>>>(T, hdr, F, B);
+    int max_c = 0;
+    for (int i = 0; i < n_terms; i++) max_c = std::max(max_c, (int)T.t[i].c);
+    if (max_c < 1) return IQ_ERR_INVALID_ARG;
+    const dim3 tg((unsigned)((max_c + kTabThreads - 1) / kTabThreads), (unsigned)n_terms);
+    IQ_CUDA_CHECK(cudaMemsetAsync(hdr->bound, 0, sizeof(hdr->bound), st));
+    k_comb_bound<<<tg, kTabThreads, 0, st>>>(T, hdr);
+    IQ_LAUNCH_CHECK();
+    k_comb_tab<<<tg, kTabThreads, 0, st>>>(T, hdr, F, B);
     IQ_LAUNCH_CHECK();
     const int64_t total = n * hw * (int64_t)c_out;
     bool vec = c_out % 8 == 0 && ((uintptr_t)out & 7) == 0;

@@ -540,7 +540,9 @@ def test_conv_fwd_adversarial_full_scale(sign, h, k):
 
 # ----------------------------------------------------------------- network glue
 
-@pytest.mark.parametrize("k,s,p,c", [(2, 2, 0, 24), (3, 2, 1, 24), (3, 2, 1, 6)])
+@pytest.mark.parametrize("k,s,p,c", [(2, 2, 0, 24), (3, 2, 1, 24), (3, 2, 1, 6), (2, 2, 0, 64),
+                                     (3, 2, 1, 64), (3, 1, 1, 8), (2, 3, 0, 8), (3, 3, 1, 16),
+                                     (2, 2, 0, 6)])
 def test_maxpool(k, s, p, c):
     g = S.rng(k * 10 + s)
     x = S.int8_uniform(g, (2, 37, 30, c), -9, 9)
