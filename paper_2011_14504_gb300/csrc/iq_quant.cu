@@ -231,9 +231,10 @@ __device__ __forceinline__ void put_f16x4(uint2* __restrict__ out16, int64_t i, 
     }
 }
 
-// int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores), optionally
-// zeroed where mask4's codes are not positive, and optionally their fp16 copies
-template <bool CLIP>
+// int32 accumulators -> int8 codes, 4 per thread (16-byte loads, 4-byte stores), and
+// optionally their fp16 copies.  MASK: the codes are zeroed where mask4's codes are not
+// positive (a compile-time switch, so that the unmasked form carries no mask loads)
+template <bool CLIP, bool MASK>
 __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int relu,
                               const RqParams* __restrict__ prm, uint32_t* __restrict__ out,
                               uint2* __restrict__ out16, const uint32_t* __restrict__ mask4) {
@@ -253,13 +254,13 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
             for (int j = 0; j < 4; j++) {
                 const bool in = i + j * stride < n4;
                 v[j] = in ? __ldg(q + i + j * stride) : make_int4(0, 0, 0, 0);
-                mk[j] = in && mask4 ? __ldg(mask4 + i + j * stride) : 0x01010101u;
+                if (MASK) mk[j] = in ? __ldg(mask4 + i + j * stride) : 0u;
             }
 #pragma unroll
             for (int j = 0; j < 4; j++)
                 if (i + j * stride < n4) {
                     uint32_t w = sq8_word_f<CLIP>(v[j], M, p.R8, kq, relu);
-                    if (mask4) w &= pos_bytes(mk[j]);
+                    if (MASK) w &= pos_bytes(mk[j]);
                     out[i + j * stride] = w;
                     put_f16x4(out16, i + j * stride, w);
                 }
@@ -271,13 +272,13 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
         const int64_t i2 = i + stride;
         const int4 v = __ldg(q + i);
         const int4 v2 = i2 < n4 ? __ldg(q + i2) : make_int4(0, 0, 0, 0);
-        const uint32_t mk = mask4 ? __ldg(mask4 + i) : 0x01010101u;
-        const uint32_t mk2 = mask4 && i2 < n4 ? __ldg(mask4 + i2) : 0x01010101u;
+        const uint32_t mk = MASK ? __ldg(mask4 + i) : 0u;
+        const uint32_t mk2 = MASK && i2 < n4 ? __ldg(mask4 + i2) : 0u;
         uint32_t w = ((uint32_t)sq_code<CLIP>(v.x, p, k, relu, lim) & 0xffu) |
                      (((uint32_t)sq_code<CLIP>(v.y, p, k, relu, lim) & 0xffu) << 8) |
                      (((uint32_t)sq_code<CLIP>(v.z, p, k, relu, lim) & 0xffu) << 16) |
                      (((uint32_t)sq_code<CLIP>(v.w, p, k, relu, lim) & 0xffu) << 24);
-        if (mask4) w &= pos_bytes(mk);
+        if (MASK) w &= pos_bytes(mk);
         out[i] = w;
         put_f16x4(out16, i, w);
         if (i2 < n4) {
@@ -285,11 +286,20 @@ __global__ void k_sq_i32_i8x4(const int4* __restrict__ q, int64_t n4, int k, int
                           (((uint32_t)sq_code<CLIP>(v2.y, p, k, relu, lim) & 0xffu) << 8) |
                           (((uint32_t)sq_code<CLIP>(v2.z, p, k, relu, lim) & 0xffu) << 16) |
                           (((uint32_t)sq_code<CLIP>(v2.w, p, k, relu, lim) & 0xffu) << 24);
-            if (mask4) w2 &= pos_bytes(mk2);
+            if (MASK) w2 &= pos_bytes(mk2);
             out[i2] = w2;
             put_f16x4(out16, i2, w2);
         }
     }
+}
+
+// the 4-code kernel over n codes (n % 4 == 0, aligned operands)
+template <bool CLIP, bool MASK>
+void sq_x4_launch(const void* q, int64_t n, int k, int relu, const RqParams* prm, void* out,
+                  __half* out16, const int8_t* mask, cudaStream_t st) {
+    k_sq_i32_i8x4<CLIP, MASK><<<grid_for(n / 4), kThreads, 0, st>>>(
+        (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16,
+        (const uint32_t*)mask);
 }
 
 template <typename T, bool CLIP>
@@ -416,15 +426,13 @@ iq_status requant_apply(const void* q, int in_dtype, int64_t n, const double* s_
                         (((uintptr_t)q & 15) | ((uintptr_t)out & 3)) == 0;
         // the mask rides on the 4-wide kernel when its codes are 4-byte aligned
         const bool m4 = !mask || ((uintptr_t)mask & 3) == 0;
-        if (x4 && m4 && clip)
-            k_sq_i32_i8x4<true><<<grid_for(n / 4), kThreads, 0, st>>>(
-                (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16,
-                (const uint32_t*)mask);
-        else if (x4 && m4)
-            k_sq_i32_i8x4<false><<<grid_for(n / 4), kThreads, 0, st>>>(
-                (const int4*)q, n / 4, k, relu, prm, (uint32_t*)out, (uint2*)out16,
-                (const uint32_t*)mask);
-        else if (in_dtype == IQ_I32 && clip)
+        if (x4 && m4) {
+            using Launch = void (*)(const void*, int64_t, int, int, const RqParams*, void*,
+                                    __half*, const int8_t*, cudaStream_t);
+            const Launch f = clip ? (mask ? sq_x4_launch<true, true> : sq_x4_launch<true, false>)
+                                  : (mask ? sq_x4_launch<false, true> : sq_x4_launch<false, false>);
+            f(q, n, k, relu, prm, out, out16, mask, st);
+        } else if (in_dtype == IQ_I32 && clip)
             k_sq_int<int32_t, true><<<g, kThreads, 0, st>>>((const int32_t*)q, n, k, relu, prm,
                                                             out, out_dtype);
         else if (in_dtype == IQ_I32)
