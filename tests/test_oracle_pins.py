@@ -549,6 +549,26 @@ def test_maxpool_matches_torch_and_routes_first_max():
             assert a[b, i, j, c] == r * k + q
 
 
+@pytest.mark.parametrize("k,s,p", [(2, 2, 0), (3, 2, 1), (3, 1, 1), (2, 3, 0), (3, 3, 1)])
+def test_maxpool_backward_matches_autograd_without_ties(k, s, p):
+    """Distinct values in every channel plane, so each window has one maximum: the routed
+    errors (summed where windows overlap) are torch's max_pool2d gradient."""
+    g = S.rng(72 + 10 * k + s)
+    n, h, w, c = 2, 7, 6, 3
+    x = np.empty((n, h, w, c), np.int8)
+    for b in range(n):
+        for ch in range(c):
+            x[b, :, :, ch] = g.permutation(np.arange(-127, 128))[:h * w].reshape(h, w)
+    y, a = O.maxpool_fwd(x, k, s, p)
+    t = torch.from_numpy(x.astype(np.float64)).permute(0, 3, 1, 2).requires_grad_(True)
+    ty = torch.nn.functional.max_pool2d(t, k, s, p)
+    assert np.array_equal(y, ty.detach().permute(0, 2, 3, 1).numpy().astype(np.int8))
+    e = S.int8_uniform(g, y.shape)
+    ty.backward(torch.from_numpy(e.astype(np.float64)).permute(0, 3, 1, 2))
+    want = t.grad.permute(0, 2, 3, 1).numpy()
+    assert np.array_equal(O.maxpool_bwd(e, a, x.shape, k, s, p), want.astype(np.int32))
+
+
 def test_mse_grad_exact_rationals():
     g = S.rng(71)
     z = S.int8_uniform(g, (2, 7, 5, 6))
